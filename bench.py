@@ -1,0 +1,349 @@
+#!/usr/bin/env python3
+"""Throughput of local SGD over K simulated workers on one GB300 (samples/s).
+
+Workload: MLP 3072-1024-1024-10 (ReLU, He-normal init), bf16 GEMM operands with fp32 accumulation
+and fp32 master weights, K = 16 workers, B_loc = 128, H = 16, Nesterov momentum 0.9 kept local,
+weight decay 5e-4, lr 0.1 scaled by K with 5-epoch linear warm-up, on N = 50,000 synthetic
+CIFAR-shaped Gaussian-mixture points (32x32x3, 10 classes).  One timed step = one local step of all
+K replicas (sampling, gather + cast, forward, loss, backward, fused update) plus, every H-th step,
+the K-way average.  `value` is device-timed with inputs resident in HBM; `e2e` drives the same
+steps through lsgd_local_step_batch with each step's mini-batch copied from pinned host memory and
+its losses read back.
+
+--impl reference times the oracle (single-threaded C++, fp64) on the host cores instead.
+Under torchrun (N > 1) every rank runs an independent replica of the workload (no collective on the
+data path); the time is the maximum over ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+WORKLOAD = dict(name="mlp_3072-1024-1024-10_K16_B128_H16_bf16", widths=(3072, 1024, 1024, 10),
+                K=16, B=128, H=16, N=50000, C=10, base_lr=0.1, scale_by_K=True, warmup_epochs=5.0,
+                momentum=0.9, nesterov=True, weight_decay=5e-4, seed=0, data_seed=1234)
+
+# Bytes the algorithm moves per parameter and replica (fp32 w, u, g; bf16 shadow):
+#   update  = read g, w, u + write w, u (4 B each) + write bf16 shadow (2 B) = 22
+#   average = read w + write w (4 B each) + write bf16 shadow (2 B) = 10
+UPDATE_BYTES_PER_PARAM = 22
+AVERAGE_BYTES_PER_PARAM = 10
+# DRAM bytes per launch of the update kernel from the ncu capture summarised in
+# profiles/sgd_update_kernel_mlp3072_K16.md (None until captured for the current kernel).
+UPDATE_TRAFFIC_PER_LAUNCH = None
+
+FALLBACK_HBM_GBS = 6800.0
+FALLBACK_BF16_TFLOPS = 1900.0
+
+
+def _peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), float(p["bf16_tflops_sustained"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, FALLBACK_BF16_TFLOPS, "fallback"
+
+
+def _dist():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons while a timed region runs."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index: int):
+        self.dev = device_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "100", "-i", str(self.dev)],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if not self.proc:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        rows = []
+        for line in open(self.path):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                rows.append((float(parts[1]), float(parts[2]), parts[5:9]))
+            except ValueError:
+                continue
+        os.unlink(self.path)
+        if not rows:
+            return None
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for _, _, r in rows for i, v in enumerate(r) if v.lower() == "active"})
+        return {"sm_mhz": statistics.median(r[0] for r in rows), "sm_max_mhz": max(r[1] for r in rows),
+                "reasons": reasons, "samples": len(rows)}
+
+
+def _make_cfg(P, total_steps):
+    w = WORKLOAD
+    return P.make_config(K=w["K"], B_loc=w["B"], H=w["H"], total_steps=total_steps, N=w["N"],
+                         widths=w["widths"], base_lr=w["base_lr"], scale_by_K=w["scale_by_K"],
+                         warmup_epochs=w["warmup_epochs"], momentum=w["momentum"],
+                         nesterov=w["nesterov"], weight_decay=w["weight_decay"], seed=w["seed"],
+                         precision=P.BF16)
+
+
+def _oracle_cfg(oracle, total_steps):
+    w = WORKLOAD
+    return oracle.make_cfg(widths=w["widths"], bf16=True, K=w["K"], B=w["B"], H=w["H"],
+                           T=total_steps, N=w["N"], base_lr=w["base_lr"],
+                           scale_by_K=w["scale_by_K"], warmup_epochs=w["warmup_epochs"],
+                           momentum=w["momentum"], nesterov=w["nesterov"],
+                           weight_decay=w["weight_decay"], seed=w["seed"])
+
+
+def oracle_sample(X, y, replica_steps: int, rows: int, budget_s: float):
+    """Time the oracle on `replica_steps` local steps of single replicas (first `rows` rows of each
+    worker's mini-batch, then the update of all parameters).  Returns (seconds, samples, steps)."""
+    import numpy as np
+
+    import oracle
+
+    o = _oracle_cfg(oracle, 1 << 20)
+    w = oracle.init_params(o)
+    u = np.zeros_like(w)
+    t0 = time.perf_counter()
+    done = 0
+    for i in range(replica_steps):
+        idx = oracle.sample_indices(o, i % o.K, i // o.K)[:rows]
+        _, g = oracle.loss_grad(o, w, X, y=y, idx=idx)
+        w, u = oracle.sgd_update(o, oracle.lr(o, i // o.K), w, u, g)
+        done += 1
+        if time.perf_counter() - t0 > budget_s:
+            break
+    return time.perf_counter() - t0, done * rows, done
+
+
+def run_reference(args, world, rank):
+    if rank != 0:
+        return
+    import synthdata
+
+    w = WORKLOAD
+    X, y = synthdata.gaussian_mixture_cached(w["N"], w["widths"][0], w["C"], w["data_seed"])
+    rows = 32
+    for _ in range(args.warmup):
+        oracle_sample(X, y, 1, rows, 1e9)
+    t, samples, steps = oracle_sample(X, y, args.steps, rows, 1e9)
+    v = samples / t
+    sample = (f"{steps} single-replica local steps, each on {rows} of the worker's {w['B']} "
+              f"mini-batch rows plus the update of all parameters")
+    line = {
+        "impl": "reference", "metric": "samples/s over K simulated workers (1 GB300)",
+        "value": v, "unit": "samples/s", "n_gpus": args.gpus, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": 1000.0 * t / steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": w["name"], "global_batch": w["K"] * w["B"], "parallelism": "replicas"},
+        "cpu_baseline": {"value": v, "unit": "samples/s", "cores": 1, "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": v, "unit": "samples/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=48)
+    ap.add_argument("--warmup", type=int, default=16)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    world, rank, local = _dist()
+
+    if args.impl == "reference":
+        run_reference(args, world, rank)
+        return
+
+    import numpy as np
+    import torch
+
+    import synthdata
+
+    if world > 1:
+        import torch.distributed as dist
+
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    else:
+        torch.cuda.set_device(0)
+    from paper_1808_07217_gb300 import _build
+
+    _build.build()
+    import paper_1808_07217_gb300 as P
+
+    w = WORKLOAD
+    K, B, H = w["K"], w["B"], w["H"]
+    X, y = synthdata.gaussian_mixture_cached(w["N"], w["widths"][0], w["C"], w["data_seed"])
+    W_, S_ = max(3, args.warmup), args.steps
+    e2e_warm = 2
+    total = W_ + S_ + e2e_warm + S_
+    stream = torch.cuda.current_stream()
+    ctx = P.lsgd_create(_make_cfg(P, total), stream=stream.cuda_stream)
+    P.lsgd_set_dataset(ctx, X, y)
+    d = P.lsgd_num_params(ctx)
+
+    # ---- device-resident timing ----
+    P.lsgd_run(ctx, W_)
+    torch.cuda.synchronize()
+    clocks = ClockSampler(local)
+    clocks.start()
+    time.sleep(0.3)
+    n0 = P.lsgd_kernel_launches(ctx)
+    syncs0 = P.lsgd_sync_count(ctx)
+    P.lsgd_profile_enable(ctx, True)
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    P.lsgd_run(ctx, S_)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    t_ms = e0.elapsed_time(e1)
+    launches = P.lsgd_kernel_launches(ctx) - n0
+    n_syncs = P.lsgd_sync_count(ctx) - syncs0
+    prof = P.lsgd_profile_read(ctx)
+    P.lsgd_profile_enable(ctx, False)
+    clk = clocks.stop()
+    if world > 1:
+        tt = torch.tensor([t_ms], device="cuda")
+        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
+        t_ms = float(tt.item())
+    samples_per_rank = S_ * K * B
+    value = world * samples_per_rank / (t_ms / 1000.0)
+
+    # ---- end to end through the C ABI with host buffers ----
+    rng = np.random.default_rng(0)
+    n_stage = 4
+    xs, ys = [], []
+    for i in range(n_stage):
+        idx = P.lsgd_debug_indices(ctx, W_ + S_ + i, K, B).reshape(-1)
+        xs.append(torch.from_numpy(X[idx].reshape(K, B, -1)).pin_memory())
+        ys.append(torch.from_numpy(y[idx].reshape(K, B).copy()).pin_memory())
+    del rng
+    loss_host = np.empty((1, K), dtype=np.float32)
+
+    def e2e_step(i):
+        s = P.lsgd_step_count(ctx)
+        P.lsgd_local_step_batch(ctx, xs[i % n_stage], ys[i % n_stage])
+        if (s + 1) % H == 0 or s == total - 1:
+            P.lsgd_sync_average(ctx)
+        P.lib().lsgd_losses(ctx.handle, P._ptr(loss_host), 1)  # device -> host read, synchronises
+
+    for i in range(e2e_warm):
+        e2e_step(i)
+    torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    t0 = time.perf_counter()
+    for i in range(S_):
+        e2e_step(i)
+    torch.cuda.synchronize()
+    t_e2e = time.perf_counter() - t0
+    if world > 1:
+        tt = torch.tensor([t_e2e], device="cuda")
+        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
+        t_e2e = float(tt.item())
+    e2e_value = world * samples_per_rank / t_e2e
+    h2d = K * B * w["widths"][0] * 4 + K * B * 4
+    d2h = K * 4
+
+    # ---- roofline of the dominant kernel (the fused update) ----
+    hbm, bf16_peak, peak_src = _peaks()
+    upd_n, upd_ms = prof["update"]
+    avg_n, avg_ms = prof["average"]
+    upd_bytes = UPDATE_BYTES_PER_PARAM * K * d
+    upd_gbs = upd_bytes / (upd_ms / upd_n / 1000.0) / 1e9
+    avg_gbs = (AVERAGE_BYTES_PER_PARAM * K * d / (avg_ms / avg_n / 1000.0) / 1e9) if avg_n else None
+    widths = w["widths"]
+    gemm_flops = 0
+    for l in range(len(widths) - 1):
+        mac = B * widths[l] * widths[l + 1]
+        gemm_flops += 2 * mac * (3 if l > 0 else 2)
+    gemm_flops *= K
+    gemm_ms = (prof["forward"][1] + prof["backward"][1]) / max(prof["forward"][0], 1)
+    gemm_tflops = gemm_flops / (gemm_ms / 1000.0) / 1e12
+    phase_ms = {k: v[1] for k, v in prof.items()}
+    tot_phase = sum(phase_ms.values())
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        t_cpu, samples_cpu, steps_cpu = oracle_sample(X, y, 64, B, 15.0)
+        cpu = {"value": samples_cpu / t_cpu, "unit": "samples/s", "cores": 1, "kind": "oracle",
+               "sample": f"{steps_cpu} single-replica local steps of the workload (B = {B} rows "
+                         f"each, forward, backward and update) timed on one host core"}
+
+    line = {
+        "metric": "samples/s over K simulated workers (1 GB300)",
+        "value": value, "unit": "samples/s", "n_gpus": world, "steps": S_, "warmup": W_,
+        "ms_per_step": t_ms / S_, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": w["name"], "global_batch": K * B, "K": K, "B_loc": B, "H": H,
+                   "params_per_replica": d, "parallelism": "replicas" if world > 1 else "single",
+                   "l2": "per-step working set (w, u, g, shadow: 1.0 GB) exceeds the 129 MB L2",
+                   "syncs_in_timed_region": n_syncs},
+        "e2e": {"value": e2e_value, "unit": "samples/s", "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h},
+        "gpu_launches": launches,
+        "roofline": {"kernel": "sgd_update_kernel", "bound": "hbm", "achieved": upd_gbs,
+                     "peak": hbm, "unit": "GB/s", "frac": upd_gbs / hbm,
+                     "peak_source": f"{peak_src} hbm_gbs", "traffic": UPDATE_TRAFFIC_PER_LAUNCH,
+                     "algorithmic_bytes_per_launch": upd_bytes},
+        "sync_average": {"gbs": avg_gbs, "frac_of_hbm": (avg_gbs / hbm) if avg_gbs else None,
+                         "ms_per_sync": (avg_ms / avg_n) if avg_n else None},
+        "step_split": {"local_frac": 1.0 - phase_ms["average"] / tot_phase,
+                       "sync_frac": phase_ms["average"] / tot_phase,
+                       "phase_ms_per_step": {k: v / S_ for k, v in phase_ms.items()}},
+        "gemm": {"tflops": gemm_tflops, "frac_of_bf16_peak": gemm_tflops / bf16_peak,
+                 "peak_source": f"{peak_src} bf16_tflops_sustained"},
+        "clocks": clk,
+        "cpu_baseline": cpu,
+    }
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    P.lsgd_destroy(ctx)
+    if world > 1:
+        torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

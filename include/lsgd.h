@@ -1,0 +1,226 @@
+/* lsgd.h -- C ABI of the GB300 local / post-local SGD hot path.
+ *
+ * Method: "Don't Use Large Mini-Batches, Use Local SGD" (Lin, Stich, Patel, Jaggi).  K workers
+ * are simulated on one GPU as K model replicas held in one replica-major buffer.  One local step
+ * (Eq. 2, left part; the inner loop of Algorithm 1) samples each worker's mini-batch from its own
+ * shard, runs forward/backward per replica and applies a local momentum-SGD update; a round ends
+ * with the K-way model average (Eq. 2, right part).  Post-local SGD (Sec. 3, Algorithm 2) averages
+ * after every step before the switch step t' and every H steps after it.
+ *
+ * Conventions (every entry point):
+ *  - Returns an lsgd_status; on error, out-parameters are left untouched and lsgd_last_error()
+ *    describes the failure.  A failed call leaves the context usable unless it returns LSGD_ECUDA.
+ *  - The library owns every device buffer it allocates (through the caller's allocator if one is
+ *    given); the caller owns every buffer it passes in, and the library copies what it keeps.
+ *  - Step calls are asynchronous on the stream given at creation; calls that return host data
+ *    synchronise that stream first.  A context is not thread-safe: one host thread at a time.
+ *  - Parameter vectors use the canonical packed order: for each dense layer l = 1..L, W_l row-major
+ *    [out_l][in_l] then b_l [out_l]; for ResNet-20, per convolution (stem first) its weight
+ *    [Cout][3][3][Cin], BN gamma [Cout], BN beta [Cout], then the classifier W [classes][4 base]
+ *    and b [classes].  Internally each tensor is padded to 256-byte alignment.
+ *  - Dataset rows are fp32, HWC for images; labels are int32 class ids, targets fp32.
+ */
+#ifndef LSGD_H
+#define LSGD_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define LSGD_MAX_LAYERS 8
+#define LSGD_MAX_MILESTONES 4
+
+typedef enum {
+  LSGD_OK = 0,
+  LSGD_EINVAL = 1,       /* bad argument or configuration */
+  LSGD_ENOMEM = 2,       /* allocation failed (the context stays valid) */
+  LSGD_ECUDA = 3,        /* a CUDA call failed; the context should be destroyed */
+  LSGD_ESTATE = 4,       /* call out of order (e.g. a step before lsgd_set_dataset) */
+  LSGD_ENONFINITE = 5,   /* lsgd_check_finite found a NaN or Inf */
+  LSGD_ETIMEOUT = 6,     /* a bounded device-side wait ran out */
+  LSGD_EUNSUPPORTED = 7, /* valid but not supported by this build (e.g. shape limits) */
+  LSGD_EIO = 8           /* checkpoint file error */
+} lsgd_status;
+
+typedef enum {
+  LSGD_MLP = 0,      /* dense ReLU network with softmax cross-entropy; 1 layer = softmax regression */
+  LSGD_LSQ = 1,      /* least squares f_i(w) = 1/2 (a_i^T w - t_i)^2, one layer, no bias */
+  LSGD_RESNET20 = 2  /* CIFAR ResNet-20 (He et al. 2016) with option-A shortcuts */
+} lsgd_model_kind;
+
+typedef enum { LSGD_FP32 = 0, LSGD_BF16 = 1 } lsgd_precision;
+typedef enum { LSGD_INIT_ZERO = 0, LSGD_INIT_HE = 1 } lsgd_init_kind;
+
+typedef struct {
+  lsgd_model_kind kind;
+  int n_layers;                         /* dense layers (MLP, LSQ) */
+  int widths[LSGD_MAX_LAYERS + 1];      /* widths[0] = input dim ... widths[n_layers] = outputs */
+  int init;                             /* lsgd_init_kind: He-normal (fan-in) or zeros */
+  int in_h, in_w, in_c;                 /* ResNet: image geometry (32, 32, 3) */
+  int n_classes, base_ch, res_blocks;   /* ResNet: 10, 16, 3 */
+} lsgd_model;
+
+/* gamma(s), Sec. A.3 / A.4: eta_hat = K eta if scale_by_K; linear warm-up from eta adding
+ * (eta_hat - eta) / (warmup_epochs N / (K B)) per step, capped at eta_hat; then gamma is
+ * multiplied by `decay` at every step s >= floor(milestone_frac[i] * T). */
+typedef struct {
+  double base_lr;
+  int scale_by_K;
+  double warmup_epochs;
+  int n_milestones;
+  double milestone_frac[LSGD_MAX_MILESTONES];
+  double decay;
+} lsgd_lr_schedule;
+
+/* Optional device allocator (NULL: cudaMallocAsync / cudaFreeAsync on the context's stream).
+ * alloc returns a device pointer aligned to at least 256 bytes, or NULL on failure. */
+typedef struct {
+  void* (*alloc)(void* user, size_t bytes, void* stream);
+  void (*free)(void* user, void* ptr, void* stream);
+  void* user;
+} lsgd_allocator;
+
+typedef struct {
+  int K;                 /* workers (replicas), >= 1 */
+  int B_loc;             /* local mini-batch size, >= 1 */
+  int H;                 /* local steps per averaging round after the switch, >= 1 */
+  int64_t t_switch;      /* post-local switch step t' (H = 1 for steps s < t'); < 0: plain local SGD */
+  int64_t total_steps;   /* T; 0 derives T = ceil(epochs N / (K B)) */
+  double epochs;
+  int64_t N;             /* dataset rows that lsgd_set_dataset will provide; >= K */
+  lsgd_model model;
+  lsgd_lr_schedule lr;
+  double momentum;       /* m; 0 = plain SGD */
+  int nesterov;
+  double weight_decay;   /* lambda; never applied to BatchNorm gamma / beta */
+  uint64_t seed;         /* keys Philox4x32-10 for sampling and initialisation */
+  int precision;         /* lsgd_precision: FP32 = fp32 everywhere; BF16 = bf16 GEMM operands,
+                            fp32 accumulation, fp32 master weights and optimizer state */
+} lsgd_config;
+
+typedef struct lsgd_ctx lsgd_ctx;
+
+/* Create a context: validates cfg, allocates the replica-major buffers (w, u, g fp32 and the bf16
+ * shadow of w in BF16 mode, all [K][d_pad]), initialises w_(0) from cfg.seed and copies it to
+ * every replica ("synchronize to have the same initial models", Algorithm 1).  `cuda_stream` is a
+ * cudaStream_t (NULL = legacy default stream).  LSGD_EINVAL for K, B_loc, H < 1, N < K, bad model
+ * widths; LSGD_EUNSUPPORTED for BF16 dense layers whose input width is not a multiple of 8. */
+lsgd_status lsgd_create(const lsgd_config* cfg, const lsgd_allocator* alloc, void* cuda_stream,
+                        lsgd_ctx** out);
+void lsgd_destroy(lsgd_ctx* ctx);
+
+/* Copy the training set (host pointers, N rows of widths[0] fp32 and N int32 labels in
+ * [0, classes)) to the device.  Worker k owns rows [k floor(N/K), (k+1) floor(N/K)) (the data is
+ * "partitioned among the GPUs", Sec. A.4).  N must equal cfg.N.  LSQ uses lsgd_set_targets. */
+lsgd_status lsgd_set_dataset(lsgd_ctx* ctx, const float* X, const int32_t* labels, int64_t N);
+lsgd_status lsgd_set_targets(lsgd_ctx* ctx, const float* X, const float* targets, int64_t N);
+
+/* One local step s on all K replicas (Eq. 2 left / Algorithm 1 inner loop): sample
+ * I^k_s = k floor(N/K) + mulhi(Philox(ctr = (j/4, s, k, 0), key = seed)[j mod 4], floor(N/K)),
+ * gather and cast the rows, forward, loss, backward, then the fused update
+ * g' = g + lambda w; u = m u + g'; w -= gamma(s) (g' + m u | u | g').  Does not average. */
+lsgd_status lsgd_local_step(lsgd_ctx* ctx);
+
+/* Same step, but on a caller-supplied mini-batch x [K][B_loc][widths[0]] fp32 and labels
+ * [K][B_loc] (or targets for LSQ), replica-major, instead of sampling the resident dataset.
+ * `on_device` = 0: host pointers (pinned memory is copied asynchronously, pageable memory
+ * synchronously); either way the caller keeps the buffers unchanged until the stream has reached
+ * the step (e.g. until lsgd_losses for that step returns). */
+lsgd_status lsgd_local_step_batch(lsgd_ctx* ctx, const float* x, const void* labels_or_targets,
+                                  int on_device);
+
+/* The K-way average w^k := (1/K) sum_k w^k for every k (Eq. 2 right; the all-reduce and model
+ * update that close each round of Algorithm 1); momentum buffers stay local (Sec. A.4).
+ * Refreshes the bf16 shadow. */
+lsgd_status lsgd_sync_average(lsgd_ctx* ctx);
+
+/* n_steps local steps from the current step counter, averaging after every step s that ends a
+ * round: s < t' (post-local first phase), (s + 1 - max(t', 0)) mod H == 0, or s == T - 1. */
+lsgd_status lsgd_run(lsgd_ctx* ctx, int64_t n_steps);
+
+/* Replica k's fp32 parameters (k = -1: the element-wise mean over replicas, computed in fp64 on
+ * the host) in canonical order, n = lsgd_num_params() elements, to host or device memory. */
+lsgd_status lsgd_params(lsgd_ctx* ctx, int k, float* dst, int dst_is_device, size_t n);
+lsgd_status lsgd_momentum(lsgd_ctx* ctx, int k, float* dst, int dst_is_device, size_t n);
+/* Overwrite replica k's parameters / momentum (k = -1: every replica) from host memory. */
+lsgd_status lsgd_set_params(lsgd_ctx* ctx, int k, const float* src, size_t n);
+lsgd_status lsgd_set_momentum(lsgd_ctx* ctx, int k, const float* src, size_t n);
+
+/* Per-replica mean mini-batch loss of the last `n_steps` steps, [n_steps][K] fp32, oldest first.
+ * The history holds the last T steps. */
+lsgd_status lsgd_losses(lsgd_ctx* ctx, float* dst, int64_t n_steps);
+
+/* The mini-batch indices I^k_s of step s for every worker, [K][B_loc] int32 (host). */
+lsgd_status lsgd_debug_indices(lsgd_ctx* ctx, int64_t step, int32_t* dst);
+
+/* Mean loss of replica k (k = -1: replica 0 right after a sync) over the first n dataset rows,
+ * computed with the same forward kernels (no update). */
+lsgd_status lsgd_eval_loss(lsgd_ctx* ctx, int k, int64_t n, double* loss);
+
+/* LSGD_ENONFINITE if any replica parameter is NaN or Inf. */
+lsgd_status lsgd_check_finite(lsgd_ctx* ctx);
+
+/* Checkpoint / resume of w, u (all replicas), the step and sync counters.  Philox is counter based
+ * so no generator state is stored.  lsgd_load requires a context created with the same config. */
+lsgd_status lsgd_save(lsgd_ctx* ctx, const char* path);
+lsgd_status lsgd_load(lsgd_ctx* ctx, const char* path);
+
+int64_t lsgd_num_params(const lsgd_ctx* ctx);   /* d, canonical (unpadded) */
+int64_t lsgd_step_count(const lsgd_ctx* ctx);   /* local steps taken so far (next step's s) */
+int64_t lsgd_sync_count(const lsgd_ctx* ctx);   /* averages performed so far */
+int64_t lsgd_total_steps(const lsgd_ctx* ctx);  /* T */
+double lsgd_lr_at(const lsgd_ctx* ctx, int64_t step); /* gamma(s) as used by the update */
+/* Kernel launches issued by this context since creation (for launch accounting). */
+int64_t lsgd_kernel_launches(const lsgd_ctx* ctx);
+/* Message for the last failed call on this context (or creation failure if ctx is NULL);
+ * valid until the next call on the same context. */
+const char* lsgd_last_error(const lsgd_ctx* ctx);
+
+/* ---- Tracing: CUDA-event timing of each phase of the step on the context's stream ---- */
+typedef enum {
+  LSGD_PH_INPUT = 0,    /* index sampling + row gather / cast (or the caller batch's copy) */
+  LSGD_PH_FORWARD = 1,  /* forward GEMMs / convolutions */
+  LSGD_PH_LOSS = 2,     /* softmax cross-entropy (or least-squares) loss and its gradient */
+  LSGD_PH_BACKWARD = 3, /* weight / data gradient products and bias sums */
+  LSGD_PH_UPDATE = 4,   /* the fused local update kernel */
+  LSGD_PH_AVERAGE = 5,  /* the K-way average kernel */
+  LSGD_NUM_PHASES = 6
+} lsgd_phase;
+
+typedef struct {
+  int64_t count[LSGD_NUM_PHASES]; /* timed intervals per phase */
+  double ms[LSGD_NUM_PHASES];     /* summed device time per phase (CUDA events) */
+} lsgd_profile;
+
+/* Start (enable = 1) or stop recording; enabling clears the accumulated times.  While enabled,
+ * each phase of every step and average is bracketed by CUDA events on the context's stream. */
+lsgd_status lsgd_profile_enable(lsgd_ctx* ctx, int enable);
+/* Synchronise the stream and return the times accumulated since recording was enabled. */
+lsgd_status lsgd_profile_read(lsgd_ctx* ctx, lsgd_profile* out);
+
+/* ---- Stand-alone device kernels of the path (device pointers, asynchronous on `stream`) ---- */
+
+/* K-way average of Eq. 2 (right) over replica-major W [K][d] fp32 (d a multiple of 4, W 16-byte
+ * aligned): every replica's row becomes the fp32 mean; if Wb != NULL its bf16 copy is written to
+ * Wb [K][d].  LSGD_EINVAL on bad sizes or alignment. */
+lsgd_status lsgd_kway_average(float* W, uint16_t* Wb, int K, int64_t d, void* stream);
+
+/* The fused local update of Sec. C.3.1 / A.4 over n elements (n a multiple of 4, 16-byte aligned
+ * pointers): g' = g + (wd_mask ? lambda w : 0); u = m u + g'; w -= lr (nesterov ? g' + m u : u),
+ * or w -= lr g' when m == 0 (u untouched, may be NULL); Wb (optional) receives bf16(w).  Elements
+ * whose index modulo `period` is at least `decay_end` get no weight decay (period = 0: all do). */
+lsgd_status lsgd_sgd_update(float* w, float* u, const float* g, uint16_t* Wb, int64_t n, float lr,
+                            float momentum, int nesterov, float weight_decay, int64_t period,
+                            int64_t decay_end, void* stream);
+
+/* Worker mini-batch indices for one step into dst [K][B] int32 (device), as lsgd_local_step. */
+lsgd_status lsgd_sample_indices(int32_t* dst, uint64_t seed, int64_t step, int K, int B, int64_t N,
+                                void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* LSGD_H */

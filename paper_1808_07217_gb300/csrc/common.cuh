@@ -1,0 +1,62 @@
+// Shared device helpers of the CUDA path (never used by the oracle).
+#pragma once
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace lsgd {
+
+constexpr int kNumSMs = 152;  // GB300: 2 dies x 76 SMs (queried at run time where it matters)
+
+// Philox4x32-10 (Salmon et al., SC'11): 10 rounds of the two multiply-xor lanes with the key
+// bumped by the Weyl increments between rounds.  Used for the worker mini-batch indices (counter
+// word 3 = 0) and the initial weights (counter word 3 = 1).
+struct U4 {
+  uint32_t x, y, z, w;
+};
+
+__host__ __device__ __forceinline__ uint32_t mulhi32(uint32_t a, uint32_t b) {
+#ifdef __CUDA_ARCH__
+  return __umulhi(a, b);
+#else
+  return (uint32_t)(((uint64_t)a * b) >> 32);
+#endif
+}
+
+__host__ __device__ __forceinline__ U4 philox4x32_10(U4 c, uint32_t k0, uint32_t k1) {
+#pragma unroll
+  for (int r = 0; r < 10; ++r) {
+    const uint32_t a = 0xD2511F53u * c.x, ah = mulhi32(0xD2511F53u, c.x);
+    const uint32_t b = 0xCD9E8D57u * c.z, bh = mulhi32(0xCD9E8D57u, c.z);
+    c = U4{bh ^ c.y ^ k0, b, ah ^ c.w ^ k1, a};
+    k0 += 0x9E3779B9u;
+    k1 += 0xBB67AE85u;
+  }
+  return c;
+}
+
+__host__ __device__ __forceinline__ uint32_t u4_get(const U4& v, int i) {
+  return i == 0 ? v.x : (i == 1 ? v.y : (i == 2 ? v.z : v.w));
+}
+
+__device__ __forceinline__ uint16_t f2bf(float f) {
+  __nv_bfloat16 b = __float2bfloat16_rn(f);
+  return *reinterpret_cast<uint16_t*>(&b);
+}
+
+__device__ __forceinline__ float bf2f(uint16_t u) { return __uint_as_float(((uint32_t)u) << 16); }
+
+template <typename T>
+struct Elem;
+template <>
+struct Elem<float> {
+  __device__ __forceinline__ static float load(const float* p) { return *p; }
+  __device__ __forceinline__ static void store(float* p, float v) { *p = v; }
+};
+template <>
+struct Elem<uint16_t> {
+  __device__ __forceinline__ static float load(const uint16_t* p) { return bf2f(*p); }
+  __device__ __forceinline__ static void store(uint16_t* p, float v) { *p = f2bf(v); }
+};
+
+}  // namespace lsgd

@@ -1,0 +1,389 @@
+// Grouped bf16 GEMM on the 5th-generation tensor cores (tcgen05 / TMEM / TMA), sm_103a.
+//
+// The per-replica dense-layer products of Eq. 2's local gradient: forward act x W^T, data
+// gradient dZ x W and weight gradient dZ^T x act, for K replicas at once.  Operands live in the
+// replica-major buffers; each is described by one rank-3 TMA map whose outermost coordinate is the
+// replica, so the CTA for (n-tile, m-tile, replica g) loads its tiles at coordinate z = g.
+//
+// One CTA computes a 128 x BN fp32 tile in TMEM:
+//   warp 0 (one lane)  TMA producer: k-blocks of 64 bf16 (one 128-byte swizzle row) into a ring
+//                      of shared-memory stages, completion signalled on the stage's mbarrier;
+//   warp 1 (one lane)  MMA issuer: 4 x tcgen05.mma (M=128, N=BN, K=16) per stage, accumulate in
+//                      TMEM; tcgen05.commit frees the stage and finally signals the epilogue;
+//   warp 2             allocates / frees the TMEM columns;
+//   warps 0-3          epilogue: tcgen05.ld of their 32 TMEM lanes (= tile rows), bias / ReLU /
+//                      ReLU-mask, store to global.
+// K-major operands use the canonical SWIZZLE_128B K-major layout (8-row atoms of 128 B; SBO =
+// 1024 B; the k-th 16-element slice starts 32 B further); MN-major operands are loaded as
+// 64-element-wide boxes stacked along MN (LBO = box stride, SBO = 1024 B; the k-th slice starts
+// 16 rows = 2048 B further).  Every mbarrier wait is bounded: on expiry the kernel records an error
+// flag, stops issuing, and still frees its TMEM.
+#include <cudaTypedefs.h>
+
+#include <mutex>
+
+#include "common.cuh"
+#include "lsgd_internal.h"
+
+namespace lsgd {
+
+__device__ int g_tc_timeout = 0;
+
+namespace {
+
+constexpr int BM = 128;
+constexpr int BK = 64;
+constexpr int STAGES = 4;
+constexpr long long kWaitCycles = 4000000000LL;  // ~2 s at 2 GHz
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return (uint32_t)__cvta_generic_to_shared(p);
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)),
+               "r"(bytes)
+               : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+      " selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+// Bounded wait on an mbarrier phase; false (and the global error flag set) on expiry.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const long long t0 = clock64();
+  while (!mbar_try_wait(bar, parity)) {
+    if (clock64() - t0 > kWaitCycles) {
+      atomicExch(&g_tc_timeout, 1);
+      return false;
+    }
+  }
+  return true;
+}
+
+__device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, uint64_t* bar, int x,
+                                            int y, int z) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%3, %4, %5}], [%2];" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(bar)), "r"(x), "r"(y), "r"(z)
+      : "memory");
+}
+
+__device__ __forceinline__ uint64_t smem_desc(uint32_t addr, uint32_t lbo, uint32_t sbo) {
+  uint64_t d = 0;
+  d |= (uint64_t)((addr >> 4) & 0x3FFFu);
+  d |= (uint64_t)((lbo >> 4) & 0x3FFFu) << 16;
+  d |= (uint64_t)((sbo >> 4) & 0x3FFFu) << 32;
+  d |= 1ull << 46;  // descriptor version (tcgen05)
+  d |= 2ull << 61;  // SWIZZLE_128B
+  return d;
+}
+
+// kind::f16 instruction descriptor: fp32 accumulator, bf16 A and B, majors, N >> 3, M >> 4.
+__host__ __device__ constexpr uint32_t make_idesc(int M, int N, bool a_mn, bool b_mn) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((a_mn ? 1u : 0u) << 15) | ((b_mn ? 1u : 0u) << 16) |
+         ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+
+__device__ __forceinline__ void mma_bf16(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc,
+                                         uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem_d),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+__device__ __forceinline__ void mma_commit(uint64_t* bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+          smem_u32(bar))
+      : "memory");
+}
+
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
+  uint32_t r[16];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15},"
+      " [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+template <int BN>
+struct Smem {
+  // stage buffers first (1024-byte aligned for the 128-byte swizzle)
+  uint8_t a[STAGES][BM * BK * 2];
+  uint8_t b[STAGES][BN * BK * 2];
+  uint64_t full[STAGES];
+  uint64_t empty[STAGES];
+  uint64_t accum;
+  uint32_t tmem_base;
+};
+
+template <int BN>
+__global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__ TcGemmArgs args) {
+  extern __shared__ uint8_t smem_raw[];
+  Smem<BN>& sm = *reinterpret_cast<Smem<BN>*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                               ~uintptr_t(1023));
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int n0 = blockIdx.x * BN, m0 = blockIdx.y * BM, g = blockIdx.z;
+  const int nk = (args.Kd + BK - 1) / BK;
+  const bool a_mn = args.A.mn_major, b_mn = args.B.mn_major;
+  constexpr uint32_t kBytesA = BM * BK * 2, kBytesB = BN * BK * 2;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(&sm.full[s], 1);
+      mbar_init(&sm.empty[s], 1);
+    }
+    mbar_init(&sm.accum, 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  }
+  if (warp == 2) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     smem_u32(&sm.tmem_base)),
+                 "r"((uint32_t)BN)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+  __syncthreads();
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+  const uint32_t tmem = sm.tmem_base;
+
+  bool ok = true;
+  if (warp == 0 && lane == 0) {
+    // ---------------- TMA producer ----------------
+    int issued = 0;
+    for (int kb = 0; kb < nk && ok; ++kb) {
+      const int s = kb % STAGES;
+      const uint32_t ph = (kb / STAGES) & 1;
+      if (!mbar_wait(&sm.empty[s], ph ^ 1)) {
+        ok = false;
+        break;
+      }
+      mbar_expect_tx(&sm.full[s], kBytesA + kBytesB);
+      const int k0 = kb * BK;
+      if (!a_mn) {
+        tma_load_3d(sm.a[s], &args.A.map, &sm.full[s], k0, m0, g);
+      } else {
+#pragma unroll
+        for (int i = 0; i < BM / 64; ++i)
+          tma_load_3d(sm.a[s] + i * 64 * BK * 2, &args.A.map, &sm.full[s], m0 + 64 * i, k0, g);
+      }
+      if (!b_mn) {
+        tma_load_3d(sm.b[s], &args.B.map, &sm.full[s], k0, n0, g);
+      } else {
+#pragma unroll
+        for (int i = 0; i < BN / 64; ++i)
+          tma_load_3d(sm.b[s] + i * 64 * BK * 2, &args.B.map, &sm.full[s], n0 + 64 * i, k0, g);
+      }
+      issued = kb + 1;
+    }
+    if (!ok) {
+      // let copies already in flight land before the CTA can exit
+      for (int kb = (issued > STAGES ? issued - STAGES : 0); kb < issued; ++kb)
+        mbar_wait(&sm.full[kb % STAGES], (kb / STAGES) & 1);
+    }
+  } else if (warp == 1 && lane == 0) {
+    // ---------------- MMA issuer ----------------
+    constexpr uint32_t idesc_kk = make_idesc(BM, BN, false, false);
+    const uint32_t idesc = idesc_kk | ((a_mn ? 1u : 0u) << 15) | ((b_mn ? 1u : 0u) << 16);
+    for (int kb = 0; kb < nk; ++kb) {
+      const int s = kb % STAGES;
+      const uint32_t ph = (kb / STAGES) & 1;
+      if (!mbar_wait(&sm.full[s], ph)) {
+        ok = false;
+        break;
+      }
+      asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+      const uint32_t a_base = smem_u32(sm.a[s]), b_base = smem_u32(sm.b[s]);
+#pragma unroll
+      for (int kk = 0; kk < BK / 16; ++kk) {
+        const uint64_t ad = a_mn ? smem_desc(a_base + kk * 2048, 64 * BK * 2, 1024)
+                                 : smem_desc(a_base + kk * 32, 16, 1024);
+        const uint64_t bd = b_mn ? smem_desc(b_base + kk * 2048, 64 * BK * 2, 1024)
+                                 : smem_desc(b_base + kk * 32, 16, 1024);
+        mma_bf16(tmem, ad, bd, idesc, (kb > 0 || kk > 0) ? 1u : 0u);
+      }
+      mma_commit(&sm.empty[s]);  // stage reusable once these MMAs have read it
+    }
+    if (ok) mma_commit(&sm.accum);  // accumulator complete
+  }
+  __syncwarp();
+
+  // ---------------- epilogue (all 4 warps) ----------------
+  const bool have_acc = mbar_wait(&sm.accum, 0);
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+  if (have_acc) {
+    const int m = m0 + warp * 32 + lane;
+    const bool row_ok = m < args.M;
+    const float* bias = args.bias ? args.bias + (int64_t)g * args.bias_gs : nullptr;
+    char* Cg = reinterpret_cast<char*>(args.C) +
+               ((int64_t)g * args.c_gs + (int64_t)m * args.c_rs) * (args.c_bf16 ? 2 : 4);
+    const char* Mg = args.mask ? reinterpret_cast<const char*>(args.mask) +
+                                     ((int64_t)g * args.mask_gs + (int64_t)m * args.mask_rs) *
+                                         (args.mask_bf16 ? 2 : 4)
+                               : nullptr;
+    for (int c0 = 0; c0 < BN; c0 += 16) {
+      if (n0 + c0 >= args.N) break;  // warp-uniform
+      float v[16];
+      tmem_ld16(tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)c0, v);
+      if (!row_ok) continue;
+      const int nb = n0 + c0;
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        const int n = nb + i;
+        if (n >= args.N) break;
+        float x = v[i];
+        if (args.epi == EPI_BIAS || args.epi == EPI_BIAS_RELU) x += bias[n];
+        if (args.epi == EPI_BIAS_RELU) x = fmaxf(x, 0.f);
+        if (args.epi == EPI_MASK) {
+          const float mv = args.mask_bf16 ? bf2f(reinterpret_cast<const uint16_t*>(Mg)[n])
+                                          : reinterpret_cast<const float*>(Mg)[n];
+          x = mv > 0.f ? x : 0.f;
+        }
+        v[i] = x;
+      }
+      const bool full16 = nb + 16 <= args.N;
+      if (args.c_bf16) {
+        uint16_t* out = reinterpret_cast<uint16_t*>(Cg) + nb;
+        if (full16 && ((reinterpret_cast<uintptr_t>(out) & 15) == 0)) {
+          uint4 p0, p1;
+          p0.x = (uint32_t)f2bf(v[0]) | ((uint32_t)f2bf(v[1]) << 16);
+          p0.y = (uint32_t)f2bf(v[2]) | ((uint32_t)f2bf(v[3]) << 16);
+          p0.z = (uint32_t)f2bf(v[4]) | ((uint32_t)f2bf(v[5]) << 16);
+          p0.w = (uint32_t)f2bf(v[6]) | ((uint32_t)f2bf(v[7]) << 16);
+          p1.x = (uint32_t)f2bf(v[8]) | ((uint32_t)f2bf(v[9]) << 16);
+          p1.y = (uint32_t)f2bf(v[10]) | ((uint32_t)f2bf(v[11]) << 16);
+          p1.z = (uint32_t)f2bf(v[12]) | ((uint32_t)f2bf(v[13]) << 16);
+          p1.w = (uint32_t)f2bf(v[14]) | ((uint32_t)f2bf(v[15]) << 16);
+          reinterpret_cast<uint4*>(out)[0] = p0;
+          reinterpret_cast<uint4*>(out)[1] = p1;
+        } else {
+          for (int i = 0; i < 16 && nb + i < args.N; ++i) out[i] = f2bf(v[i]);
+        }
+      } else {
+        float* out = reinterpret_cast<float*>(Cg) + nb;
+        if (full16 && ((reinterpret_cast<uintptr_t>(out) & 15) == 0)) {
+#pragma unroll
+          for (int q = 0; q < 4; ++q)
+            reinterpret_cast<float4*>(out)[q] =
+                make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+        } else {
+          for (int i = 0; i < 16 && nb + i < args.N; ++i) out[i] = v[i];
+        }
+      }
+    }
+  }
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+  __syncthreads();
+  if (warp == 2) {
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"((uint32_t)BN)
+                 : "memory");
+  }
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+std::once_flag g_encode_once;
+
+void load_encode() {
+  void* fn = nullptr;
+  cudaDriverEntryPointQueryResult q;
+  if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) ==
+          cudaSuccess &&
+      q == cudaDriverEntryPointSuccess)
+    g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+  else
+    cudaGetLastError();
+}
+
+template <int BN>
+constexpr size_t smem_bytes() {
+  return sizeof(Smem<BN>) + 1024;
+}
+
+}  // namespace
+
+bool tc_available() {
+  int dev = 0;
+  cudaDeviceProp p;
+  if (cudaGetDevice(&dev) != cudaSuccess || cudaGetDeviceProperties(&p, dev) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  std::call_once(g_encode_once, load_encode);
+  return p.major == 10 && g_encode != nullptr;
+}
+
+int tc_take_timeout_flag() {
+  int h = 0;
+  if (cudaMemcpyFromSymbol(&h, g_tc_timeout, sizeof(int)) != cudaSuccess) {
+    cudaGetLastError();
+    return 0;
+  }
+  if (h) {
+    const int zero = 0;
+    cudaMemcpyToSymbol(g_tc_timeout, &zero, sizeof(int));
+  }
+  return h;
+}
+
+bool make_tma_map_bf16(CUtensorMap* map, const void* base, uint64_t dim0, uint64_t dim1,
+                       uint64_t dim2, uint64_t s1, uint64_t s2, uint32_t box0, uint32_t box1) {
+  std::call_once(g_encode_once, load_encode);
+  if (!g_encode) return false;
+  if ((reinterpret_cast<uintptr_t>(base) & 15) || ((s1 * 2) & 15) || ((s2 * 2) & 15)) return false;
+  cuuint64_t dims[3] = {dim0, dim1, dim2};
+  cuuint64_t strides[2] = {s1 * 2, s2 * 2};
+  cuuint32_t box[3] = {box0, box1, 1};
+  cuuint32_t estr[3] = {1, 1, 1};
+  CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims,
+                        strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                        CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+cudaError_t launch_gemm_tc(const TcGemmArgs& a, cudaStream_t stream) {
+  if (a.M <= 0 || a.N <= 0 || a.G <= 0) return cudaSuccess;
+  if (a.Kd <= 0 || a.G > 65535) return cudaErrorInvalidValue;
+  if ((a.epi == EPI_BIAS || a.epi == EPI_BIAS_RELU) && !a.bias) return cudaErrorInvalidValue;
+  if (a.epi == EPI_MASK && !a.mask) return cudaErrorInvalidValue;
+  constexpr int BN = 128;
+  dim3 grid((a.N + BN - 1) / BN, (a.M + BM - 1) / BM, a.G);
+  if (grid.y > 65535) return cudaErrorInvalidValue;
+  const size_t smem = smem_bytes<BN>();
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<BN>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  gemm_tc_kernel<BN><<<grid, 128, smem, stream>>>(a);
+  return cudaGetLastError();
+}
+
+}  // namespace lsgd

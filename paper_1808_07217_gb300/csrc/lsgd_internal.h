@@ -1,0 +1,102 @@
+// Internal launchers of the CUDA path.  Every launcher validates its launch shape on the host and
+// returns the CUDA error of the launch; all work is asynchronous on `stream`.
+#pragma once
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace lsgd {
+
+// ---- element-wise / reduction kernels (kernels.cu) ----
+cudaError_t launch_sample_indices(int32_t* idx, uint64_t seed, int64_t step, int K, int B, int64_t N,
+                                  cudaStream_t stream);
+// dst[r][0..D) = X[idx[r]][0..D) (idx == NULL: row r), cast to bf16 when dst_bf16; labels too.
+cudaError_t launch_gather_rows(void* dst, bool dst_bf16, int ld_dst, const float* X, int D,
+                               const int32_t* idx, int rows, const int32_t* labels_in,
+                               int32_t* labels_out, const float* targets_in, float* targets_out,
+                               cudaStream_t stream);
+// Softmax cross-entropy over logits [G][B][ld]; dz = (softmax - onehot) / B into [G][B][ld_dz]
+// (skipped when dz == NULL); loss_mean[g] = mean row loss, loss_sum[g] = sum, row_loss[g B + j]
+// = row loss (each may be NULL).
+cudaError_t launch_softmax_xent(const float* logits, int ld, int C, const int32_t* labels, int G,
+                                int B, void* dz, bool dz_bf16, int ld_dz, float* loss_mean,
+                                float* loss_sum, float* row_loss, cudaStream_t stream);
+// Least squares: z [G][B][ld] (column 0), r = z - t; loss = r^2 / 2; dz = r / B.
+cudaError_t launch_lsq_loss(const float* z, int ld, const float* targets, int G, int B, void* dz,
+                            bool dz_bf16, int ld_dz, float* loss_mean, float* loss_sum,
+                            float* row_loss, cudaStream_t stream);
+// gb[g * gb_gs + o] = sum_j dz[g][j][o] for o < out.
+cudaError_t launch_colsum(const void* dz, bool dz_bf16, int ld, int G, int B, int out, float* gb,
+                          int64_t gb_gs, cudaStream_t stream);
+cudaError_t launch_sgd_update(float* w, float* u, const float* g, uint16_t* wb, int64_t n, float lr,
+                              float momentum, int nesterov, float weight_decay, int64_t period,
+                              int64_t decay_end, cudaStream_t stream);
+cudaError_t launch_kway_average(float* W, uint16_t* Wb, int K, int64_t d, cudaStream_t stream);
+cudaError_t launch_init_normal(float* w, int64_t n, double stddev, uint64_t seed, uint32_t tensor_id,
+                               cudaStream_t stream);
+cudaError_t launch_fill(float* w, int64_t n, float v, cudaStream_t stream);
+cudaError_t launch_broadcast(float* W, int K, int64_t d, cudaStream_t stream);
+cudaError_t launch_to_bf16(const float* w, uint16_t* wb, int64_t n, cudaStream_t stream);
+cudaError_t launch_check_finite(const float* w, int64_t n, int* flag, cudaStream_t stream);
+
+// ---- grouped GEMM: C[g](m, n) = sum_k A[g](m, k) B[g](k, n), with a fused epilogue ----
+enum GemmEpilogue {
+  EPI_STORE = 0,      // C = acc
+  EPI_BIAS = 1,       // C = acc + bias[n]
+  EPI_BIAS_RELU = 2,  // C = max(acc + bias[n], 0)
+  EPI_MASK = 3        // C = mask(m, n) > 0 ? acc : 0   (ReLU derivative from the stored activation)
+};
+
+struct GemmArgs {
+  int M, N, Kd, G;
+  const void* A;
+  int64_t a_rs, a_cs, a_gs;  // element strides of A(m, k) and per group
+  bool a_bf16;
+  const void* B;
+  int64_t b_rs, b_cs, b_gs;  // element strides of B(k, n)
+  bool b_bf16;
+  void* C;
+  int64_t c_rs, c_gs;  // C(m, n) at C + g c_gs + m c_rs + n
+  bool c_bf16;
+  int epi;
+  const float* bias;
+  int64_t bias_gs;
+  const void* mask;
+  int64_t mask_rs, mask_gs;
+  bool mask_bf16;
+};
+
+cudaError_t launch_gemm_simt(const GemmArgs& a, cudaStream_t stream);
+
+// ---- tcgen05 / TMEM / TMA grouped GEMM (gemm_tc.cu), bf16 operands, fp32 accumulation ----
+// A is M x Kd, B is N x Kd (as stored: "K-major" = Kd contiguous, "MN-major" = M/N contiguous),
+// both described by rank-3 TMA maps whose outermost dimension is the replica (group).
+struct TcOperand {
+  CUtensorMap map;  // box: K-major {64 (Kd), rows}; MN-major {64 (M or N), 64 (Kd)}
+  bool mn_major;
+};
+
+struct TcGemmArgs {
+  int M, N, Kd, G;
+  TcOperand A, B;
+  // epilogue (same semantics as GemmArgs), C(m, n) at C + g c_gs + m c_rs + n
+  void* C;
+  int64_t c_rs, c_gs;
+  bool c_bf16;
+  int epi;
+  const float* bias;
+  int64_t bias_gs;
+  const void* mask;
+  int64_t mask_rs, mask_gs;
+  bool mask_bf16;
+};
+
+// Encode a rank-3 bf16 TMA map over [dim2][dim1][dim0] with strides (elements) s1, s2.
+bool make_tma_map_bf16(CUtensorMap* map, const void* base, uint64_t dim0, uint64_t dim1,
+                       uint64_t dim2, uint64_t s1, uint64_t s2, uint32_t box0, uint32_t box1);
+cudaError_t launch_gemm_tc(const TcGemmArgs& a, cudaStream_t stream);
+bool tc_available();
+// 1 if a bounded wait inside a tcgen05 kernel ran out since the last call (then cleared).
+int tc_take_timeout_flag();
+
+}  // namespace lsgd

@@ -1,0 +1,40 @@
+// ResNet-20 plan of the CUDA path (per-replica implicit-GEMM convolutions, batch-stat BatchNorm,
+// option-A shortcuts), driven by the runtime in runtime.cu.
+#pragma once
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <functional>
+#include <string>
+
+#include "../../include/lsgd.h"
+
+namespace lsgd {
+
+struct ResNetPlan;
+
+bool resnet_supported(const lsgd_config& cfg, std::string* why);
+ResNetPlan* resnet_plan_create(const lsgd_config& cfg);
+void resnet_destroy(ResNetPlan* p);
+int64_t resnet_num_params(const ResNetPlan* p);
+int64_t resnet_d_pad(const ResNetPlan* p);
+// Calls f(canonical offset, padded offset, length) for every parameter tensor.
+void resnet_segments(const ResNetPlan* p, const std::function<void(int64_t, int64_t, int64_t)>& f);
+// Weight decay applies to padded offsets (i mod period) < decay_end.
+void resnet_decay_region(const ResNetPlan* p, int64_t* period, int64_t* decay_end);
+lsgd_status resnet_alloc(ResNetPlan* p, const std::function<void*(size_t)>& alloc);
+lsgd_status resnet_init_params(ResNetPlan* p, float* W, uint64_t seed, cudaStream_t s,
+                               int64_t* launches);
+// One forward + backward over the K replicas' gathered inputs; gradients into G, per-replica mean
+// loss into loss_mean[K].
+lsgd_status resnet_forward_backward(ResNetPlan* p, const float* W, const uint16_t* Wb, float* G,
+                                    int64_t d_pad, const int32_t* labels, float* loss_mean,
+                                    cudaStream_t s, int64_t* launches);
+// Forward only with replica k's weights for `groups` groups of B_loc rows; per-row losses.
+lsgd_status resnet_eval(ResNetPlan* p, const float* W, const uint16_t* Wb, int64_t d_pad, int k,
+                        int groups, const int32_t* labels, float* row_loss, cudaStream_t s,
+                        int64_t* launches);
+void* resnet_input(ResNetPlan* p);
+const char* resnet_last_error(const ResNetPlan* p);
+
+}  // namespace lsgd

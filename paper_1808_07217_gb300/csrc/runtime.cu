@@ -1,0 +1,1038 @@
+// Runtime and C ABI of the local / post-local SGD hot path (declared in include/lsgd.h).
+//
+// K workers are simulated as K replicas in one replica-major arena: fp32 master weights W, local
+// momentum U and gradients G, each [K][d_pad], plus a bf16 shadow Wb of W in BF16 mode (the GEMM
+// operand).  Every per-replica tensor starts 256-byte aligned, so one rank-3 TMA map per operand
+// (replica = outermost dimension) covers all K replicas.  A local step (Eq. 2 left, Algorithm 1's
+// inner loop) is a fixed sequence of kernel launches on the context's stream with no host
+// synchronisation; the K-way average (Eq. 2 right) is one kernel.
+#include <cmath>
+#include <cstdio>
+#include <cstdlib>
+#include <array>
+#include <algorithm>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "../../include/lsgd.h"
+#include "lsgd_internal.h"
+#include "resnet.h"
+
+namespace {
+
+thread_local std::string g_last_error;
+
+int64_t round_up(int64_t v, int64_t m) { return (v + m - 1) / m * m; }
+
+struct Seg {
+  int64_t canon, pad, len;
+};
+
+struct DenseLayer {
+  int in, out, ld_in, ld_out;
+  int64_t w_off, b_off;  // padded per-replica offsets (b_off < 0: no bias)
+  bool tc;               // this layer's products run on tcgen05
+  lsgd::TcOperand fwdA, fwdB, dgA, dgB, wgA, wgB;
+};
+
+}  // namespace
+
+struct lsgd_ctx {
+  lsgd_config cfg;
+  lsgd_allocator alloc{};
+  bool have_alloc = false;
+  cudaStream_t stream = nullptr;
+  int64_t d = 0, d_pad = 0, T = 0, shard = 0;
+  int D = 0, C = 0;  // input width, outputs
+  bool bf16 = false, lsq = false, resnet = false;
+  std::vector<DenseLayer> layers;
+  std::vector<Seg> segs;
+  int64_t wd_period = 0, wd_end = 0;
+  std::vector<void*> allocs;
+  float *W = nullptr, *U = nullptr, *G = nullptr;
+  uint16_t* Wb = nullptr;
+  float* X = nullptr;
+  int32_t* y = nullptr;
+  float* t = nullptr;
+  bool have_data = false;
+  int32_t* idx = nullptr;
+  int32_t* yb = nullptr;
+  float* tb = nullptr;
+  float* xstage = nullptr;
+  int32_t* ystage = nullptr;
+  float* tstage = nullptr;
+  std::vector<void*> act;  // act[l]: input of dense layer l, [K][B][ld] operand dtype
+  float* logits = nullptr;
+  int ld_logits = 0;
+  void* dz[2] = {nullptr, nullptr};
+  int ld_dz = 0;
+  float* loss_hist = nullptr;
+  int64_t loss_cap = 0;
+  float* row_loss = nullptr;  // [K][B] scratch for evaluation
+  int* flag = nullptr;
+  int64_t step = 0, syncs = 0, launches = 0;
+  std::string err;
+  lsgd::ResNetPlan* rn = nullptr;
+  // tracing (lsgd_profile_*)
+  bool prof_on = false;
+  std::vector<cudaEvent_t> prof_pool;
+  size_t prof_used = 0;
+  std::vector<std::array<int64_t, 3>> prof_spans;  // (phase, start event, end event)
+};
+
+namespace {
+
+lsgd_status fail(lsgd_ctx* c, lsgd_status st, const std::string& msg) {
+  if (c) c->err = msg;
+  g_last_error = msg;
+  return st;
+}
+
+lsgd_status fail_cuda(lsgd_ctx* c, cudaError_t e, const char* what) {
+  return fail(c, LSGD_ECUDA, std::string(what) + ": " + cudaGetErrorString(e));
+}
+
+#define LSGD_TRY_CUDA(ctx, expr)                                  \
+  do {                                                            \
+    cudaError_t e__ = (expr);                                     \
+    if (e__ != cudaSuccess) return fail_cuda((ctx), e__, #expr); \
+  } while (0)
+
+#define LSGD_LAUNCH(ctx, expr)                                    \
+  do {                                                            \
+    cudaError_t e__ = (expr);                                     \
+    (ctx)->launches++;                                            \
+    if (e__ != cudaSuccess) return fail_cuda((ctx), e__, #expr); \
+  } while (0)
+
+void* dalloc(lsgd_ctx* c, size_t bytes) {
+  if (bytes == 0) bytes = 256;
+  bytes = (size_t)round_up((int64_t)bytes, 256);
+  void* p = nullptr;
+  if (c->have_alloc) {
+    p = c->alloc.alloc(c->alloc.user, bytes, (void*)c->stream);
+  } else {
+    if (cudaMallocAsync(&p, bytes, c->stream) != cudaSuccess) {
+      cudaGetLastError();
+      p = nullptr;
+    }
+  }
+  if (!p) return nullptr;
+  if (cudaMemsetAsync(p, 0, bytes, c->stream) != cudaSuccess) {
+    cudaGetLastError();
+  }
+  c->allocs.push_back(p);
+  return p;
+}
+
+void free_all(lsgd_ctx* c) {
+  for (void* p : c->allocs) {
+    if (c->have_alloc)
+      c->alloc.free(c->alloc.user, p, (void*)c->stream);
+    else
+      cudaFreeAsync(p, c->stream);
+  }
+  c->allocs.clear();
+}
+
+// ---- tracing: an event at each phase boundary, paired into spans ----
+int64_t prof_mark(lsgd_ctx* c) {
+  if (!c->prof_on) return -1;
+  if (c->prof_used == c->prof_pool.size()) {
+    cudaEvent_t e;
+    if (cudaEventCreate(&e) != cudaSuccess) {
+      cudaGetLastError();
+      return -1;
+    }
+    c->prof_pool.push_back(e);
+  }
+  cudaEventRecord(c->prof_pool[c->prof_used], c->stream);
+  return (int64_t)c->prof_used++;
+}
+
+void prof_span(lsgd_ctx* c, int phase, int64_t a, int64_t b) {
+  if (c->prof_on && a >= 0 && b >= 0) c->prof_spans.push_back({phase, a, b});
+}
+
+// ---- schedules (Sec. A.3, A.4 and Sec. 3) ----
+double lr_at(const lsgd_config& cfg, int64_t T, int64_t s) {
+  const double eta = cfg.lr.base_lr;
+  const double eta_hat = cfg.lr.scale_by_K ? eta * cfg.K : eta;
+  double lr = eta_hat;
+  if (cfg.lr.warmup_epochs > 0.0 && eta_hat != eta) {
+    const double steps_per_epoch = (double)cfg.N / ((double)cfg.K * cfg.B_loc);
+    const double inc = (eta_hat - eta) / (cfg.lr.warmup_epochs * steps_per_epoch);
+    const double v = eta + (double)s * inc;
+    lr = v < eta_hat ? v : eta_hat;
+  }
+  for (int i = 0; i < cfg.lr.n_milestones; ++i)
+    if (s >= (int64_t)std::floor(cfg.lr.milestone_frac[i] * (double)T)) lr *= cfg.lr.decay;
+  return lr;
+}
+
+bool round_end(const lsgd_config& cfg, int64_t T, int64_t s) {
+  if (s == T - 1) return true;
+  if (cfg.t_switch >= 0 && s < cfg.t_switch) return true;
+  const int64_t start = cfg.t_switch > 0 ? cfg.t_switch : 0;
+  return ((s + 1 - start) % cfg.H) == 0;
+}
+
+bool force_simt() {
+  const char* e = std::getenv("LSGD_FORCE_SIMT");
+  return e && e[0] == '1';
+}
+
+// ---- dense model ----
+lsgd_status build_dense_layout(lsgd_ctx* c) {
+  const lsgd_model& m = c->cfg.model;
+  int64_t off = 0, canon = 0;
+  for (int l = 0; l < m.n_layers; ++l) {
+    DenseLayer L{};
+    L.in = m.widths[l];
+    L.out = m.widths[l + 1];
+    L.ld_in = (int)round_up(L.in, 8);
+    L.ld_out = (int)round_up(L.out, 8);
+    L.w_off = off;
+    c->segs.push_back({canon, off, (int64_t)L.in * L.out});
+    canon += (int64_t)L.in * L.out;
+    off = round_up(off + (int64_t)L.in * L.out, 64);
+    if (!c->lsq) {
+      L.b_off = off;
+      c->segs.push_back({canon, off, L.out});
+      canon += L.out;
+      off = round_up(off + L.out, 64);
+    } else {
+      L.b_off = -1;
+    }
+    c->layers.push_back(L);
+  }
+  c->d = canon;
+  c->d_pad = round_up(off, 64);
+  c->wd_period = 0;
+  c->wd_end = c->d_pad;
+  return LSGD_OK;
+}
+
+lsgd_status make_tc_maps(lsgd_ctx* c) {
+  const int K = c->cfg.K, B = c->cfg.B_loc;
+  for (size_t l = 0; l < c->layers.size(); ++l) {
+    DenseLayer& L = c->layers[l];
+    L.tc = false;
+    if (!c->bf16 || force_simt() || !lsgd::tc_available()) continue;
+    const uint16_t* Wb_l = c->Wb + L.w_off;
+    const void* a_in = c->act[l];
+    bool ok = true;
+    // forward: A = act [K][B][ld_in] (K-major), B = W [K][out][in] (K-major)
+    ok &= lsgd::make_tma_map_bf16(&L.fwdA.map, a_in, L.in, B, K, L.ld_in, (uint64_t)B * L.ld_in, 64, 128);
+    ok &= lsgd::make_tma_map_bf16(&L.fwdB.map, Wb_l, L.in, L.out, K, L.in, c->d_pad, 64, 128);
+    L.fwdA.mn_major = false;
+    L.fwdB.mn_major = false;
+    // weight gradient: A = dZ as [K][B][out] read MN-major (M = out), B = act read MN-major (N = in)
+    // The dz buffer used for layer l alternates; both dz buffers share one layout, so the maps are
+    // rebuilt per call from the right base (cheap host work, see run_dense_backward).
+    (void)a_in;
+    L.tc = ok;
+  }
+  return LSGD_OK;
+}
+
+lsgd_status alloc_dense(lsgd_ctx* c) {
+  const int K = c->cfg.K, B = c->cfg.B_loc;
+  const size_t esz = c->bf16 ? 2 : 4;
+  const int L = (int)c->layers.size();
+  c->act.resize(L);
+  int max_ld = 8;
+  for (int l = 0; l < L; ++l) {
+    c->act[l] = dalloc(c, (size_t)K * B * c->layers[l].ld_in * esz);
+    if (!c->act[l]) return fail(c, LSGD_ENOMEM, "activation buffer allocation failed");
+    max_ld = std::max(max_ld, c->layers[l].ld_out);
+  }
+  c->ld_logits = c->layers[L - 1].ld_out;
+  c->logits = (float*)dalloc(c, (size_t)K * B * c->ld_logits * 4);
+  c->ld_dz = max_ld;
+  for (int i = 0; i < 2; ++i) c->dz[i] = dalloc(c, (size_t)K * B * max_ld * esz);
+  if (!c->logits || !c->dz[0] || !c->dz[1]) return fail(c, LSGD_ENOMEM, "gradient buffer allocation failed");
+  return LSGD_OK;
+}
+
+lsgd_status init_dense_params(lsgd_ctx* c) {
+  if (c->cfg.model.init == LSGD_INIT_HE) {
+    for (size_t l = 0; l < c->layers.size(); ++l) {
+      const DenseLayer& L = c->layers[l];
+      LSGD_LAUNCH(c, lsgd::launch_init_normal(c->W + L.w_off, (int64_t)L.in * L.out,
+                                              std::sqrt(2.0 / L.in), c->cfg.seed, (uint32_t)l,
+                                              c->stream));
+    }
+  }
+  return LSGD_OK;
+}
+
+// GEMM helpers: choose the tcgen05 kernel for bf16 layers that have maps, else SIMT.
+lsgd_status gemm(lsgd_ctx* c, const lsgd::GemmArgs& g) {
+  LSGD_LAUNCH(c, lsgd::launch_gemm_simt(g, c->stream));
+  return LSGD_OK;
+}
+
+lsgd_status tc_gemm(lsgd_ctx* c, const lsgd::TcGemmArgs& g) {
+  LSGD_LAUNCH(c, lsgd::launch_gemm_tc(g, c->stream));
+  return LSGD_OK;
+}
+
+// Forward of every dense layer for `groups` groups.  Weights come from replica (w_g0 + g * w_gmul).
+lsgd_status dense_forward(lsgd_ctx* c, int groups, int w_g0, int w_gmul) {
+  const int B = c->cfg.B_loc;
+  const int L = (int)c->layers.size();
+  const void* Wop = c->bf16 ? (const void*)c->Wb : (const void*)c->W;
+  const size_t esz = c->bf16 ? 2 : 4;
+  for (int l = 0; l < L; ++l) {
+    const DenseLayer& Ly = c->layers[l];
+    const bool last = l == L - 1;
+    void* out = last ? (void*)c->logits : c->act[l + 1];
+    const int ld_out = last ? c->ld_logits : c->layers[l + 1].ld_in;
+    const bool out_bf16 = last ? false : c->bf16;
+    const int epi = c->lsq ? lsgd::EPI_STORE : (last ? lsgd::EPI_BIAS : lsgd::EPI_BIAS_RELU);
+    if (Ly.tc && w_gmul == 1 && w_g0 == 0) {
+      lsgd::TcGemmArgs t{};
+      t.M = B;
+      t.N = Ly.out;
+      t.Kd = Ly.in;
+      t.G = groups;
+      t.A = Ly.fwdA;
+      t.B = Ly.fwdB;
+      t.C = out;
+      t.c_rs = ld_out;
+      t.c_gs = (int64_t)B * ld_out;
+      t.c_bf16 = out_bf16;
+      t.epi = epi;
+      t.bias = Ly.b_off >= 0 ? c->W + Ly.b_off : nullptr;
+      t.bias_gs = c->d_pad;
+      lsgd_status st = tc_gemm(c, t);
+      if (st != LSGD_OK) return st;
+      continue;
+    }
+    lsgd::GemmArgs g{};
+    g.M = B;
+    g.N = Ly.out;
+    g.Kd = Ly.in;
+    g.G = groups;
+    g.A = c->act[l];
+    g.a_rs = Ly.ld_in;
+    g.a_cs = 1;
+    g.a_gs = (int64_t)B * Ly.ld_in;
+    g.a_bf16 = c->bf16;
+    g.B = (const char*)Wop + ((int64_t)w_g0 * c->d_pad + Ly.w_off) * esz;
+    g.b_rs = 1;
+    g.b_cs = Ly.in;
+    g.b_gs = (int64_t)w_gmul * c->d_pad;
+    g.b_bf16 = c->bf16;
+    g.C = out;
+    g.c_rs = ld_out;
+    g.c_gs = (int64_t)B * ld_out;
+    g.c_bf16 = out_bf16;
+    g.epi = epi;
+    g.bias = Ly.b_off >= 0 ? c->W + (int64_t)w_g0 * c->d_pad + Ly.b_off : nullptr;
+    g.bias_gs = (int64_t)w_gmul * c->d_pad;
+    lsgd_status st = gemm(c, g);
+    if (st != LSGD_OK) return st;
+  }
+  (void)esz;
+  return LSGD_OK;
+}
+
+lsgd_status dense_backward(lsgd_ctx* c) {
+  const int K = c->cfg.K, B = c->cfg.B_loc;
+  const int L = (int)c->layers.size();
+  const void* Wop = c->bf16 ? (const void*)c->Wb : (const void*)c->W;
+  const size_t esz = c->bf16 ? 2 : 4;
+  int cur = 0;
+  for (int l = L - 1; l >= 0; --l) {
+    const DenseLayer& Ly = c->layers[l];
+    const void* dz = c->dz[cur];
+    // weight gradient G_W[o][i] = sum_j dz[j][o] act[j][i]
+    if (Ly.tc) {
+      lsgd::TcGemmArgs t{};
+      t.M = Ly.out;
+      t.N = Ly.in;
+      t.Kd = B;
+      t.G = K;
+      bool ok = lsgd::make_tma_map_bf16(&t.A.map, dz, Ly.out, B, K, c->ld_dz, (uint64_t)B * c->ld_dz, 64, 64);
+      ok &= lsgd::make_tma_map_bf16(&t.B.map, c->act[l], Ly.in, B, K, Ly.ld_in, (uint64_t)B * Ly.ld_in, 64, 64);
+      if (!ok) return fail(c, LSGD_ECUDA, "TMA map encoding failed (wgrad)");
+      t.A.mn_major = true;
+      t.B.mn_major = true;
+      t.C = c->G + Ly.w_off;
+      t.c_rs = Ly.in;
+      t.c_gs = c->d_pad;
+      t.c_bf16 = false;
+      t.epi = lsgd::EPI_STORE;
+      lsgd_status st = tc_gemm(c, t);
+      if (st != LSGD_OK) return st;
+    } else {
+      lsgd::GemmArgs g{};
+      g.M = Ly.out;
+      g.N = Ly.in;
+      g.Kd = B;
+      g.G = K;
+      g.A = dz;
+      g.a_rs = 1;
+      g.a_cs = c->ld_dz;
+      g.a_gs = (int64_t)B * c->ld_dz;
+      g.a_bf16 = c->bf16;
+      g.B = c->act[l];
+      g.b_rs = Ly.ld_in;
+      g.b_cs = 1;
+      g.b_gs = (int64_t)B * Ly.ld_in;
+      g.b_bf16 = c->bf16;
+      g.C = c->G + Ly.w_off;
+      g.c_rs = Ly.in;
+      g.c_gs = c->d_pad;
+      g.c_bf16 = false;
+      g.epi = lsgd::EPI_STORE;
+      lsgd_status st = gemm(c, g);
+      if (st != LSGD_OK) return st;
+    }
+    if (Ly.b_off >= 0)
+      LSGD_LAUNCH(c, lsgd::launch_colsum(dz, c->bf16, c->ld_dz, K, B, Ly.out, c->G + Ly.b_off,
+                                         c->d_pad, c->stream));
+    if (l > 0) {
+      // data gradient dz_prev[j][i] = (sum_o dz[j][o] W[o][i]) * (act[j][i] > 0)
+      void* dzp = c->dz[1 - cur];
+      if (Ly.tc) {
+        lsgd::TcGemmArgs t{};
+        t.M = B;
+        t.N = Ly.in;
+        t.Kd = Ly.out;
+        t.G = K;
+        bool ok = lsgd::make_tma_map_bf16(&t.A.map, dz, Ly.out, B, K, c->ld_dz, (uint64_t)B * c->ld_dz, 64, 128);
+        ok &= lsgd::make_tma_map_bf16(&t.B.map, c->Wb + Ly.w_off, Ly.in, Ly.out, K, Ly.in, c->d_pad, 64, 64);
+        if (!ok) return fail(c, LSGD_ECUDA, "TMA map encoding failed (dgrad)");
+        t.A.mn_major = false;
+        t.B.mn_major = true;
+        t.C = dzp;
+        t.c_rs = c->ld_dz;
+        t.c_gs = (int64_t)B * c->ld_dz;
+        t.c_bf16 = c->bf16;
+        t.epi = lsgd::EPI_MASK;
+        t.mask = c->act[l];
+        t.mask_rs = Ly.ld_in;
+        t.mask_gs = (int64_t)B * Ly.ld_in;
+        t.mask_bf16 = c->bf16;
+        lsgd_status st = tc_gemm(c, t);
+        if (st != LSGD_OK) return st;
+      } else {
+        lsgd::GemmArgs g{};
+        g.M = B;
+        g.N = Ly.in;
+        g.Kd = Ly.out;
+        g.G = K;
+        g.A = dz;
+        g.a_rs = c->ld_dz;
+        g.a_cs = 1;
+        g.a_gs = (int64_t)B * c->ld_dz;
+        g.a_bf16 = c->bf16;
+        g.B = (const char*)Wop + Ly.w_off * esz;
+        g.b_rs = Ly.in;
+        g.b_cs = 1;
+        g.b_gs = c->d_pad;
+        g.b_bf16 = c->bf16;
+        g.C = dzp;
+        g.c_rs = c->ld_dz;
+        g.c_gs = (int64_t)B * c->ld_dz;
+        g.c_bf16 = c->bf16;
+        g.epi = lsgd::EPI_MASK;
+        g.mask = c->act[l];
+        g.mask_rs = Ly.ld_in;
+        g.mask_gs = (int64_t)B * Ly.ld_in;
+        g.mask_bf16 = c->bf16;
+        lsgd_status st = gemm(c, g);
+        if (st != LSGD_OK) return st;
+      }
+      cur = 1 - cur;
+    }
+  }
+  return LSGD_OK;
+}
+
+// Loss of the last layer's output for `groups` groups; dz into dz[0] unless eval.
+lsgd_status dense_loss(lsgd_ctx* c, int groups, bool eval, float* loss_mean) {
+  const int B = c->cfg.B_loc;
+  void* dz = eval ? nullptr : c->dz[0];
+  if (c->lsq) {
+    LSGD_LAUNCH(c, lsgd::launch_lsq_loss(c->logits, c->ld_logits, c->tb, groups, B, dz, c->bf16,
+                                         c->ld_dz, loss_mean, nullptr, c->row_loss, c->stream));
+  } else {
+    LSGD_LAUNCH(c, lsgd::launch_softmax_xent(c->logits, c->ld_logits, c->C, c->yb, groups, B, dz,
+                                             c->bf16, c->ld_dz, loss_mean, nullptr, c->row_loss,
+                                             c->stream));
+  }
+  return LSGD_OK;
+}
+
+lsgd_status do_update(lsgd_ctx* c) {
+  const float lr = (float)lr_at(c->cfg, c->T, c->step);
+  LSGD_LAUNCH(c, lsgd::launch_sgd_update(c->W, c->U, c->G, c->Wb, (int64_t)c->cfg.K * c->d_pad, lr,
+                                         (float)c->cfg.momentum, c->cfg.nesterov,
+                                         (float)c->cfg.weight_decay, c->wd_period, c->wd_end,
+                                         c->stream));
+  return LSGD_OK;
+}
+
+// The step body after the inputs of this step are gathered into act[0] / yb / tb.
+lsgd_status step_body(lsgd_ctx* c, int64_t e_start) {
+  const int K = c->cfg.K;
+  float* loss_slot = c->loss_hist + (c->step % c->loss_cap) * K;
+  lsgd_status st;
+  const int64_t e_in = prof_mark(c);
+  prof_span(c, LSGD_PH_INPUT, e_start, e_in);
+  int64_t e_bwd;
+  if (c->resnet) {
+    st = lsgd::resnet_forward_backward(c->rn, c->W, c->Wb, c->G, c->d_pad, c->yb, loss_slot,
+                                       c->stream, &c->launches);
+    if (st != LSGD_OK) return fail(c, st, lsgd::resnet_last_error(c->rn));
+    e_bwd = prof_mark(c);
+    prof_span(c, LSGD_PH_FORWARD, e_in, e_bwd);
+  } else {
+    st = dense_forward(c, K, 0, 1);
+    if (st != LSGD_OK) return st;
+    const int64_t e_fwd = prof_mark(c);
+    prof_span(c, LSGD_PH_FORWARD, e_in, e_fwd);
+    st = dense_loss(c, K, false, loss_slot);
+    if (st != LSGD_OK) return st;
+    const int64_t e_loss = prof_mark(c);
+    prof_span(c, LSGD_PH_LOSS, e_fwd, e_loss);
+    st = dense_backward(c);
+    if (st != LSGD_OK) return st;
+    e_bwd = prof_mark(c);
+    prof_span(c, LSGD_PH_BACKWARD, e_loss, e_bwd);
+  }
+  st = do_update(c);
+  if (st != LSGD_OK) return st;
+  prof_span(c, LSGD_PH_UPDATE, e_bwd, prof_mark(c));
+  c->step++;
+  return LSGD_OK;
+}
+
+void* input_buffer(lsgd_ctx* c) { return c->resnet ? lsgd::resnet_input(c->rn) : c->act[0]; }
+int input_ld(lsgd_ctx* c) { return c->resnet ? c->D : c->layers[0].ld_in; }
+
+}  // namespace
+
+// =============================================================================================
+extern "C" {
+
+lsgd_status lsgd_create(const lsgd_config* cfg, const lsgd_allocator* alloc, void* cuda_stream,
+                        lsgd_ctx** out) {
+  if (!cfg || !out) return fail(nullptr, LSGD_EINVAL, "cfg and out must be non-NULL");
+  const lsgd_config& c0 = *cfg;
+  if (c0.K < 1 || c0.B_loc < 1 || c0.H < 1) return fail(nullptr, LSGD_EINVAL, "K, B_loc and H must be >= 1");
+  if (c0.N < c0.K) return fail(nullptr, LSGD_EINVAL, "N must be >= K");
+  if (c0.K > 65535) return fail(nullptr, LSGD_EINVAL, "K must be <= 65535");
+  if (c0.precision != LSGD_FP32 && c0.precision != LSGD_BF16)
+    return fail(nullptr, LSGD_EINVAL, "precision must be LSGD_FP32 or LSGD_BF16");
+  if (c0.N / c0.K * (int64_t)c0.K > 0x7fffffffLL) return fail(nullptr, LSGD_EINVAL, "N too large");
+  if (c0.B_loc > 8192) return fail(nullptr, LSGD_EUNSUPPORTED, "B_loc must be <= 8192");
+  const lsgd_model& m = c0.model;
+  if (m.kind == LSGD_MLP || m.kind == LSGD_LSQ) {
+    if (m.n_layers < 1 || m.n_layers > LSGD_MAX_LAYERS)
+      return fail(nullptr, LSGD_EINVAL, "n_layers must be in [1, LSGD_MAX_LAYERS]");
+    for (int l = 0; l <= m.n_layers; ++l)
+      if (m.widths[l] < 1) return fail(nullptr, LSGD_EINVAL, "layer widths must be >= 1");
+    if (m.kind == LSGD_LSQ && (m.n_layers != 1 || m.widths[1] != 1))
+      return fail(nullptr, LSGD_EINVAL, "least squares is one layer with one output");
+    if (c0.precision == LSGD_BF16)
+      for (int l = 0; l < m.n_layers; ++l)
+        if (m.widths[l] % 8)
+          return fail(nullptr, LSGD_EUNSUPPORTED, "BF16 dense layers need input widths divisible by 8");
+  } else if (m.kind == LSGD_RESNET20) {
+    std::string why;
+    if (!lsgd::resnet_supported(c0, &why)) return fail(nullptr, LSGD_EUNSUPPORTED, why);
+  } else {
+    return fail(nullptr, LSGD_EINVAL, "unknown model kind");
+  }
+
+  lsgd_ctx* c = new lsgd_ctx();
+  c->cfg = c0;
+  if (alloc && alloc->alloc && alloc->free) {
+    c->alloc = *alloc;
+    c->have_alloc = true;
+  }
+  c->stream = (cudaStream_t)cuda_stream;
+  c->bf16 = c0.precision == LSGD_BF16;
+  c->lsq = m.kind == LSGD_LSQ;
+  c->resnet = m.kind == LSGD_RESNET20;
+  c->shard = c0.N / c0.K;
+  c->T = c0.total_steps > 0
+             ? c0.total_steps
+             : (int64_t)std::ceil(c0.epochs * (double)c0.N / ((double)c0.K * c0.B_loc) - 1e-9);
+  if (c->T < 1) c->T = 1;
+  auto bail = [&](lsgd_status st) {
+    if (c->rn) lsgd::resnet_destroy(c->rn);
+    free_all(c);
+    cudaStreamSynchronize(c->stream);
+    cudaGetLastError();
+    delete c;
+    return st;
+  };
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) {
+    cudaGetLastError();
+    fail(nullptr, LSGD_ECUDA, "no CUDA device");
+    return bail(LSGD_ECUDA);
+  }
+
+  const int K = c0.K, B = c0.B_loc;
+  if (c->resnet) {
+    c->rn = lsgd::resnet_plan_create(c0);
+    if (!c->rn) {
+      fail(nullptr, LSGD_ENOMEM, "ResNet plan creation failed");
+      return bail(LSGD_ENOMEM);
+    }
+    c->d = lsgd::resnet_num_params(c->rn);
+    c->d_pad = lsgd::resnet_d_pad(c->rn);
+    lsgd::resnet_segments(c->rn, [&](int64_t canon, int64_t pad, int64_t len) {
+      c->segs.push_back({canon, pad, len});
+    });
+    lsgd::resnet_decay_region(c->rn, &c->wd_period, &c->wd_end);
+    c->D = m.in_h * m.in_w * m.in_c;
+    c->C = m.n_classes;
+  } else {
+    build_dense_layout(c);
+    c->D = m.widths[0];
+    c->C = m.widths[m.n_layers];
+  }
+
+  const size_t n_rep = (size_t)K * c->d_pad;
+  c->W = (float*)dalloc(c, n_rep * 4);
+  c->G = (float*)dalloc(c, n_rep * 4);
+  if (c0.momentum != 0.0) c->U = (float*)dalloc(c, n_rep * 4);
+  if (c->bf16) c->Wb = (uint16_t*)dalloc(c, n_rep * 2);
+  c->idx = (int32_t*)dalloc(c, (size_t)K * B * 4);
+  c->yb = (int32_t*)dalloc(c, (size_t)K * B * 4);
+  c->tb = (float*)dalloc(c, (size_t)K * B * 4);
+  c->loss_cap = c->T;
+  c->loss_hist = (float*)dalloc(c, (size_t)c->loss_cap * K * 4);
+  c->row_loss = (float*)dalloc(c, (size_t)K * B * 4);
+  c->flag = (int*)dalloc(c, 16);
+  if (!c->W || !c->G || (c0.momentum != 0.0 && !c->U) || (c->bf16 && !c->Wb) || !c->idx ||
+      !c->yb || !c->tb || !c->loss_hist || !c->row_loss || !c->flag) {
+    fail(nullptr, LSGD_ENOMEM, "device allocation failed");
+    return bail(LSGD_ENOMEM);
+  }
+  lsgd_status st;
+  if (c->resnet) {
+    st = lsgd::resnet_alloc(c->rn, [&](size_t bytes) { return dalloc(c, bytes); });
+    if (st != LSGD_OK) {
+      fail(nullptr, st, "ResNet buffer allocation failed");
+      return bail(st);
+    }
+    st = lsgd::resnet_init_params(c->rn, c->W, c0.seed, c->stream, &c->launches);
+  } else {
+    st = alloc_dense(c);
+    if (st == LSGD_OK) st = init_dense_params(c);
+    if (st == LSGD_OK) st = make_tc_maps(c);
+  }
+  if (st != LSGD_OK) {
+    g_last_error = c->err;
+    return bail(st);
+  }
+  if (lsgd::launch_broadcast(c->W, K, c->d_pad, c->stream) != cudaSuccess ||
+      (c->bf16 && lsgd::launch_to_bf16(c->W, c->Wb, (int64_t)n_rep, c->stream) != cudaSuccess)) {
+    fail(nullptr, LSGD_ECUDA, "initial broadcast failed");
+    return bail(LSGD_ECUDA);
+  }
+  c->launches += c->bf16 ? 2 : 1;
+  cudaError_t e = cudaStreamSynchronize(c->stream);
+  if (e != cudaSuccess) {
+    fail_cuda(nullptr, e, "lsgd_create");
+    return bail(LSGD_ECUDA);
+  }
+  *out = c;
+  return LSGD_OK;
+}
+
+void lsgd_destroy(lsgd_ctx* c) {
+  if (!c) return;
+  cudaStreamSynchronize(c->stream);
+  for (cudaEvent_t e : c->prof_pool) cudaEventDestroy(e);
+  if (c->rn) lsgd::resnet_destroy(c->rn);
+  free_all(c);
+  cudaStreamSynchronize(c->stream);
+  delete c;
+}
+
+static lsgd_status set_data(lsgd_ctx* c, const float* X, const int32_t* labels, const float* targets,
+                            int64_t N) {
+  if (!c || !X) return fail(c, LSGD_EINVAL, "NULL argument");
+  if (N != c->cfg.N) return fail(c, LSGD_EINVAL, "N differs from the configured dataset size");
+  if (c->lsq != (targets != nullptr) || (!c->lsq && !labels))
+    return fail(c, LSGD_EINVAL, "labels for classifiers, targets for least squares");
+  if (labels)
+    for (int64_t i = 0; i < N; ++i)
+      if (labels[i] < 0 || labels[i] >= c->C) return fail(c, LSGD_EINVAL, "label out of range");
+  if (!c->X) {
+    c->X = (float*)dalloc(c, (size_t)N * c->D * 4);
+    if (!c->X) return fail(c, LSGD_ENOMEM, "dataset allocation failed");
+    if (labels) c->y = (int32_t*)dalloc(c, (size_t)N * 4);
+    if (targets) c->t = (float*)dalloc(c, (size_t)N * 4);
+    if ((labels && !c->y) || (targets && !c->t)) return fail(c, LSGD_ENOMEM, "label allocation failed");
+  }
+  LSGD_TRY_CUDA(c, cudaMemcpyAsync(c->X, X, (size_t)N * c->D * 4, cudaMemcpyHostToDevice, c->stream));
+  if (labels)
+    LSGD_TRY_CUDA(c, cudaMemcpyAsync(c->y, labels, (size_t)N * 4, cudaMemcpyHostToDevice, c->stream));
+  if (targets)
+    LSGD_TRY_CUDA(c, cudaMemcpyAsync(c->t, targets, (size_t)N * 4, cudaMemcpyHostToDevice, c->stream));
+  LSGD_TRY_CUDA(c, cudaStreamSynchronize(c->stream));
+  c->have_data = true;
+  return LSGD_OK;
+}
+
+lsgd_status lsgd_set_dataset(lsgd_ctx* c, const float* X, const int32_t* labels, int64_t N) {
+  if (c && c->lsq) return fail(c, LSGD_EINVAL, "least squares takes lsgd_set_targets");
+  return set_data(c, X, labels, nullptr, N);
+}
+
+lsgd_status lsgd_set_targets(lsgd_ctx* c, const float* X, const float* targets, int64_t N) {
+  if (c && !c->lsq) return fail(c, LSGD_EINVAL, "targets are for least squares only");
+  return set_data(c, X, nullptr, targets, N);
+}
+
+lsgd_status lsgd_local_step(lsgd_ctx* c) {
+  if (!c) return fail(nullptr, LSGD_EINVAL, "NULL context");
+  if (!c->have_data) return fail(c, LSGD_ESTATE, "lsgd_set_dataset must come first");
+  const int K = c->cfg.K, B = c->cfg.B_loc;
+  const int64_t e0 = prof_mark(c);
+  LSGD_LAUNCH(c, lsgd::launch_sample_indices(c->idx, c->cfg.seed, c->step, K, B, c->cfg.N, c->stream));
+  LSGD_LAUNCH(c, lsgd::launch_gather_rows(input_buffer(c), c->bf16, input_ld(c), c->X, c->D, c->idx,
+                                          K * B, c->y, c->y ? c->yb : nullptr, c->t,
+                                          c->t ? c->tb : nullptr, c->stream));
+  return step_body(c, e0);
+}
+
+lsgd_status lsgd_local_step_batch(lsgd_ctx* c, const float* x, const void* lab, int on_device) {
+  if (!c || !x || !lab) return fail(c, LSGD_EINVAL, "NULL argument");
+  const int K = c->cfg.K, B = c->cfg.B_loc;
+  const size_t rows = (size_t)K * B;
+  const float* xs = x;
+  const void* ls = lab;
+  const int64_t e0 = prof_mark(c);
+  if (!on_device) {
+    if (!c->xstage) {
+      c->xstage = (float*)dalloc(c, rows * c->D * 4);
+      c->ystage = (int32_t*)dalloc(c, rows * 4);
+      if (!c->xstage || !c->ystage) return fail(c, LSGD_ENOMEM, "staging allocation failed");
+    }
+    LSGD_TRY_CUDA(c, cudaMemcpyAsync(c->xstage, x, rows * c->D * 4, cudaMemcpyHostToDevice, c->stream));
+    LSGD_TRY_CUDA(c, cudaMemcpyAsync(c->ystage, lab, rows * 4, cudaMemcpyHostToDevice, c->stream));
+    xs = c->xstage;
+    ls = c->ystage;
+  }
+  const int32_t* yl = c->lsq ? nullptr : (const int32_t*)ls;
+  const float* tl = c->lsq ? (const float*)ls : nullptr;
+  LSGD_LAUNCH(c, lsgd::launch_gather_rows(input_buffer(c), c->bf16, input_ld(c), xs, c->D, nullptr,
+                                          (int)rows, yl, yl ? c->yb : nullptr, tl,
+                                          tl ? c->tb : nullptr, c->stream));
+  return step_body(c, e0);
+}
+
+lsgd_status lsgd_sync_average(lsgd_ctx* c) {
+  if (!c) return fail(nullptr, LSGD_EINVAL, "NULL context");
+  const int64_t e0 = prof_mark(c);
+  LSGD_LAUNCH(c, lsgd::launch_kway_average(c->W, c->Wb, c->cfg.K, c->d_pad, c->stream));
+  prof_span(c, LSGD_PH_AVERAGE, e0, prof_mark(c));
+  c->syncs++;
+  return LSGD_OK;
+}
+
+lsgd_status lsgd_profile_enable(lsgd_ctx* c, int enable) {
+  if (!c) return fail(nullptr, LSGD_EINVAL, "NULL context");
+  LSGD_TRY_CUDA(c, cudaStreamSynchronize(c->stream));
+  c->prof_spans.clear();
+  c->prof_used = 0;
+  c->prof_on = enable != 0;
+  return LSGD_OK;
+}
+
+lsgd_status lsgd_profile_read(lsgd_ctx* c, lsgd_profile* out) {
+  if (!c || !out) return fail(c, LSGD_EINVAL, "NULL argument");
+  LSGD_TRY_CUDA(c, cudaStreamSynchronize(c->stream));
+  lsgd_profile p{};
+  for (const auto& sp : c->prof_spans) {
+    float ms = 0.f;
+    LSGD_TRY_CUDA(c, cudaEventElapsedTime(&ms, c->prof_pool[sp[1]], c->prof_pool[sp[2]]));
+    p.count[sp[0]]++;
+    p.ms[sp[0]] += ms;
+  }
+  *out = p;
+  return LSGD_OK;
+}
+
+lsgd_status lsgd_run(lsgd_ctx* c, int64_t n_steps) {
+  if (!c) return fail(nullptr, LSGD_EINVAL, "NULL context");
+  if (n_steps < 0) return fail(c, LSGD_EINVAL, "n_steps must be >= 0");
+  for (int64_t i = 0; i < n_steps; ++i) {
+    const int64_t s = c->step;
+    lsgd_status st = lsgd_local_step(c);
+    if (st != LSGD_OK) return st;
+    if (round_end(c->cfg, c->T, s)) {
+      st = lsgd_sync_average(c);
+      if (st != LSGD_OK) return st;
+    }
+  }
+  return LSGD_OK;
+}
+
+static lsgd_status get_vec(lsgd_ctx* c, const float* buf, int k, float* dst, int dst_is_device,
+                           size_t n) {
+  if (!c || !dst) return fail(c, LSGD_EINVAL, "NULL argument");
+  if (n != (size_t)c->d) return fail(c, LSGD_EINVAL, "n must equal lsgd_num_params()");
+  if (k < -1 || k >= c->cfg.K) return fail(c, LSGD_EINVAL, "replica index out of range");
+  if (!buf) {  // no momentum buffer: momentum is identically zero
+    if (dst_is_device)
+      LSGD_TRY_CUDA(c, cudaMemsetAsync(dst, 0, n * 4, c->stream));
+    else
+      std::memset(dst, 0, n * 4);
+    LSGD_TRY_CUDA(c, cudaStreamSynchronize(c->stream));
+    return LSGD_OK;
+  }
+  if (k >= 0) {
+    const cudaMemcpyKind kind = dst_is_device ? cudaMemcpyDeviceToDevice : cudaMemcpyDeviceToHost;
+    for (const Seg& s : c->segs)
+      LSGD_TRY_CUDA(c, cudaMemcpyAsync(dst + s.canon, buf + (int64_t)k * c->d_pad + s.pad,
+                                       (size_t)s.len * 4, kind, c->stream));
+    LSGD_TRY_CUDA(c, cudaStreamSynchronize(c->stream));
+    return LSGD_OK;
+  }
+  std::vector<float> all((size_t)c->cfg.K * c->d_pad);
+  LSGD_TRY_CUDA(c, cudaMemcpyAsync(all.data(), buf, all.size() * 4, cudaMemcpyDeviceToHost, c->stream));
+  LSGD_TRY_CUDA(c, cudaStreamSynchronize(c->stream));
+  std::vector<float> mean((size_t)c->d);
+  for (const Seg& s : c->segs)
+    for (int64_t i = 0; i < s.len; ++i) {
+      double acc = 0.0;
+      for (int kk = 0; kk < c->cfg.K; ++kk) acc += all[(size_t)kk * c->d_pad + s.pad + i];
+      mean[s.canon + i] = (float)(acc / c->cfg.K);
+    }
+  if (dst_is_device) {
+    LSGD_TRY_CUDA(c, cudaMemcpyAsync(dst, mean.data(), n * 4, cudaMemcpyHostToDevice, c->stream));
+    LSGD_TRY_CUDA(c, cudaStreamSynchronize(c->stream));
+  } else {
+    std::memcpy(dst, mean.data(), n * 4);
+  }
+  return LSGD_OK;
+}
+
+lsgd_status lsgd_params(lsgd_ctx* c, int k, float* dst, int dst_is_device, size_t n) {
+  return get_vec(c, c ? c->W : nullptr, k, dst, dst_is_device, n);
+}
+
+lsgd_status lsgd_momentum(lsgd_ctx* c, int k, float* dst, int dst_is_device, size_t n) {
+  return get_vec(c, c ? c->U : nullptr, k, dst, dst_is_device, n);
+}
+
+static lsgd_status set_vec(lsgd_ctx* c, float* buf, int k, const float* src, size_t n, bool is_w) {
+  if (!c || !src) return fail(c, LSGD_EINVAL, "NULL argument");
+  if (n != (size_t)c->d) return fail(c, LSGD_EINVAL, "n must equal lsgd_num_params()");
+  if (k < -1 || k >= c->cfg.K) return fail(c, LSGD_EINVAL, "replica index out of range");
+  if (!buf) return fail(c, LSGD_ESTATE, "no momentum buffer (momentum is 0)");
+  const int k0 = k < 0 ? 0 : k;
+  for (const Seg& s : c->segs)
+    LSGD_TRY_CUDA(c, cudaMemcpyAsync(buf + (int64_t)k0 * c->d_pad + s.pad, src + s.canon,
+                                     (size_t)s.len * 4, cudaMemcpyHostToDevice, c->stream));
+  if (k < 0) LSGD_LAUNCH(c, lsgd::launch_broadcast(buf, c->cfg.K, c->d_pad, c->stream));
+  if (is_w && c->Wb)
+    LSGD_LAUNCH(c, lsgd::launch_to_bf16(c->W, c->Wb, (int64_t)c->cfg.K * c->d_pad, c->stream));
+  LSGD_TRY_CUDA(c, cudaStreamSynchronize(c->stream));
+  return LSGD_OK;
+}
+
+lsgd_status lsgd_set_params(lsgd_ctx* c, int k, const float* src, size_t n) {
+  return set_vec(c, c ? c->W : nullptr, k, src, n, true);
+}
+
+lsgd_status lsgd_set_momentum(lsgd_ctx* c, int k, const float* src, size_t n) {
+  return set_vec(c, c ? c->U : nullptr, k, src, n, false);
+}
+
+lsgd_status lsgd_losses(lsgd_ctx* c, float* dst, int64_t n_steps) {
+  if (!c || !dst) return fail(c, LSGD_EINVAL, "NULL argument");
+  if (n_steps < 0 || n_steps > c->step || n_steps > c->loss_cap)
+    return fail(c, LSGD_EINVAL, "n_steps exceeds the recorded history");
+  const int K = c->cfg.K;
+  for (int64_t i = 0; i < n_steps; ++i) {
+    const int64_t s = c->step - n_steps + i;
+    LSGD_TRY_CUDA(c, cudaMemcpyAsync(dst + i * K, c->loss_hist + (s % c->loss_cap) * K, (size_t)K * 4,
+                                     cudaMemcpyDeviceToHost, c->stream));
+  }
+  LSGD_TRY_CUDA(c, cudaStreamSynchronize(c->stream));
+  return LSGD_OK;
+}
+
+lsgd_status lsgd_debug_indices(lsgd_ctx* c, int64_t step, int32_t* dst) {
+  if (!c || !dst) return fail(c, LSGD_EINVAL, "NULL argument");
+  if (step < 0) return fail(c, LSGD_EINVAL, "step must be >= 0");
+  const int K = c->cfg.K, B = c->cfg.B_loc;
+  int32_t* tmp = (int32_t*)dalloc(c, (size_t)K * B * 4);
+  if (!tmp) return fail(c, LSGD_ENOMEM, "scratch allocation failed");
+  cudaError_t e = lsgd::launch_sample_indices(tmp, c->cfg.seed, step, K, B, c->cfg.N, c->stream);
+  c->launches++;
+  if (e == cudaSuccess) e = cudaMemcpyAsync(dst, tmp, (size_t)K * B * 4, cudaMemcpyDeviceToHost, c->stream);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(c->stream);
+  // release the scratch buffer
+  c->allocs.pop_back();
+  if (c->have_alloc)
+    c->alloc.free(c->alloc.user, tmp, (void*)c->stream);
+  else
+    cudaFreeAsync(tmp, c->stream);
+  if (e != cudaSuccess) return fail_cuda(c, e, "lsgd_debug_indices");
+  return LSGD_OK;
+}
+
+lsgd_status lsgd_eval_loss(lsgd_ctx* c, int k, int64_t n, double* loss) {
+  if (!c || !loss) return fail(c, LSGD_EINVAL, "NULL argument");
+  if (!c->have_data) return fail(c, LSGD_ESTATE, "lsgd_set_dataset must come first");
+  if (k < -1 || k >= c->cfg.K) return fail(c, LSGD_EINVAL, "replica index out of range");
+  if (n < 1 || n > c->cfg.N) return fail(c, LSGD_EINVAL, "n must be in [1, N]");
+  const int kk = k < 0 ? 0 : k;
+  const int K = c->cfg.K, B = c->cfg.B_loc;
+  const int64_t per = (int64_t)K * B;
+  std::vector<float> rl((size_t)per);
+  double total = 0.0;
+  for (int64_t start = 0; start < n; start += per) {
+    const int rows = (int)std::min<int64_t>(per, n - start);
+    LSGD_LAUNCH(c, lsgd::launch_gather_rows(input_buffer(c), c->bf16, input_ld(c), c->X + start * c->D,
+                                            c->D, nullptr, rows, c->y ? c->y + start : nullptr,
+                                            c->y ? c->yb : nullptr, c->t ? c->t + start : nullptr,
+                                            c->t ? c->tb : nullptr, c->stream));
+    const int groups = (rows + B - 1) / B;
+    lsgd_status st;
+    if (c->resnet) {
+      st = lsgd::resnet_eval(c->rn, c->W, c->Wb, c->d_pad, kk, groups, c->yb, c->row_loss, c->stream,
+                             &c->launches);
+      if (st != LSGD_OK) return fail(c, st, lsgd::resnet_last_error(c->rn));
+    } else {
+      st = dense_forward(c, groups, kk, 0);
+      if (st != LSGD_OK) return st;
+      st = dense_loss(c, groups, true, nullptr);
+      if (st != LSGD_OK) return st;
+    }
+    LSGD_TRY_CUDA(c, cudaMemcpyAsync(rl.data(), c->row_loss, (size_t)rows * 4, cudaMemcpyDeviceToHost,
+                                     c->stream));
+    LSGD_TRY_CUDA(c, cudaStreamSynchronize(c->stream));
+    for (int r = 0; r < rows; ++r) total += rl[r];
+  }
+  *loss = total / (double)n;
+  return LSGD_OK;
+}
+
+lsgd_status lsgd_check_finite(lsgd_ctx* c) {
+  if (!c) return fail(nullptr, LSGD_EINVAL, "NULL context");
+  LSGD_TRY_CUDA(c, cudaMemsetAsync(c->flag, 0, 4, c->stream));
+  LSGD_LAUNCH(c, lsgd::launch_check_finite(c->W, (int64_t)c->cfg.K * c->d_pad, c->flag, c->stream));
+  int h = 0;
+  LSGD_TRY_CUDA(c, cudaMemcpyAsync(&h, c->flag, 4, cudaMemcpyDeviceToHost, c->stream));
+  LSGD_TRY_CUDA(c, cudaStreamSynchronize(c->stream));
+  if (h) return fail(c, LSGD_ENONFINITE, "non-finite parameter found");
+  return LSGD_OK;
+}
+
+static const uint64_t kMagic = 0x3130545043445347ULL;  // "GSDCPT01"
+
+lsgd_status lsgd_save(lsgd_ctx* c, const char* path) {
+  if (!c || !path) return fail(c, LSGD_EINVAL, "NULL argument");
+  const size_t n = (size_t)c->cfg.K * c->d_pad;
+  std::vector<float> buf(n);
+  FILE* f = std::fopen(path, "wb");
+  if (!f) return fail(c, LSGD_EIO, std::string("cannot open ") + path);
+  int64_t hdr[6] = {(int64_t)kMagic, c->cfg.K, c->d_pad, c->step, c->syncs, c->U ? 1 : 0};
+  bool ok = std::fwrite(hdr, sizeof(hdr), 1, f) == 1;
+  for (int which = 0; ok && which < (c->U ? 2 : 1); ++which) {
+    const float* src = which == 0 ? c->W : c->U;
+    cudaError_t e = cudaMemcpyAsync(buf.data(), src, n * 4, cudaMemcpyDeviceToHost, c->stream);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(c->stream);
+    if (e != cudaSuccess) {
+      std::fclose(f);
+      return fail_cuda(c, e, "lsgd_save");
+    }
+    ok = std::fwrite(buf.data(), 4, n, f) == n;
+  }
+  ok = (std::fclose(f) == 0) && ok;
+  if (!ok) return fail(c, LSGD_EIO, "write failed");
+  return LSGD_OK;
+}
+
+lsgd_status lsgd_load(lsgd_ctx* c, const char* path) {
+  if (!c || !path) return fail(c, LSGD_EINVAL, "NULL argument");
+  FILE* f = std::fopen(path, "rb");
+  if (!f) return fail(c, LSGD_EIO, std::string("cannot open ") + path);
+  int64_t hdr[6];
+  if (std::fread(hdr, sizeof(hdr), 1, f) != 1 || hdr[0] != (int64_t)kMagic || hdr[1] != c->cfg.K ||
+      hdr[2] != c->d_pad || hdr[5] != (c->U ? 1 : 0)) {
+    std::fclose(f);
+    return fail(c, LSGD_EIO, "checkpoint does not match this configuration");
+  }
+  const size_t n = (size_t)c->cfg.K * c->d_pad;
+  std::vector<float> buf(n);
+  for (int which = 0; which < (c->U ? 2 : 1); ++which) {
+    if (std::fread(buf.data(), 4, n, f) != n) {
+      std::fclose(f);
+      return fail(c, LSGD_EIO, "truncated checkpoint");
+    }
+    float* dst = which == 0 ? c->W : c->U;
+    cudaError_t e = cudaMemcpyAsync(dst, buf.data(), n * 4, cudaMemcpyHostToDevice, c->stream);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(c->stream);
+    if (e != cudaSuccess) {
+      std::fclose(f);
+      return fail_cuda(c, e, "lsgd_load");
+    }
+  }
+  std::fclose(f);
+  if (c->Wb) LSGD_LAUNCH(c, lsgd::launch_to_bf16(c->W, c->Wb, (int64_t)n, c->stream));
+  LSGD_TRY_CUDA(c, cudaStreamSynchronize(c->stream));
+  c->step = hdr[3];
+  c->syncs = hdr[4];
+  return LSGD_OK;
+}
+
+int64_t lsgd_num_params(const lsgd_ctx* c) { return c ? c->d : -1; }
+int64_t lsgd_step_count(const lsgd_ctx* c) { return c ? c->step : -1; }
+int64_t lsgd_sync_count(const lsgd_ctx* c) { return c ? c->syncs : -1; }
+int64_t lsgd_total_steps(const lsgd_ctx* c) { return c ? c->T : -1; }
+double lsgd_lr_at(const lsgd_ctx* c, int64_t s) { return c ? lr_at(c->cfg, c->T, s) : 0.0; }
+int64_t lsgd_kernel_launches(const lsgd_ctx* c) { return c ? c->launches : -1; }
+
+const char* lsgd_last_error(const lsgd_ctx* c) {
+  if (c) return c->err.c_str();
+  return g_last_error.c_str();
+}
+
+// ---- stand-alone kernels ----
+lsgd_status lsgd_kway_average(float* W, uint16_t* Wb, int K, int64_t d, void* stream) {
+  if (!W || K < 1 || d < 0 || (d & 3) || ((uintptr_t)W & 15) || ((uintptr_t)Wb & 7))
+    return fail(nullptr, LSGD_EINVAL, "lsgd_kway_average: bad arguments");
+  cudaError_t e = lsgd::launch_kway_average(W, Wb, K, d, (cudaStream_t)stream);
+  if (e != cudaSuccess) return fail_cuda(nullptr, e, "lsgd_kway_average");
+  return LSGD_OK;
+}
+
+lsgd_status lsgd_sgd_update(float* w, float* u, const float* g, uint16_t* Wb, int64_t n, float lr,
+                            float momentum, int nesterov, float weight_decay, int64_t period,
+                            int64_t decay_end, void* stream) {
+  if (!w || !g || n < 0 || (n & 3) || (period & 3) || (decay_end & 3) || ((uintptr_t)w & 15) ||
+      ((uintptr_t)g & 15) || ((uintptr_t)u & 15) || ((uintptr_t)Wb & 7) || (momentum != 0.f && !u))
+    return fail(nullptr, LSGD_EINVAL, "lsgd_sgd_update: bad arguments");
+  cudaError_t e = lsgd::launch_sgd_update(w, u, g, Wb, n, lr, momentum, nesterov, weight_decay, period,
+                                          decay_end, (cudaStream_t)stream);
+  if (e != cudaSuccess) return fail_cuda(nullptr, e, "lsgd_sgd_update");
+  return LSGD_OK;
+}
+
+lsgd_status lsgd_sample_indices(int32_t* dst, uint64_t seed, int64_t step, int K, int B, int64_t N,
+                                void* stream) {
+  if (!dst || K < 1 || B < 1 || N < K) return fail(nullptr, LSGD_EINVAL, "lsgd_sample_indices: bad arguments");
+  cudaError_t e = lsgd::launch_sample_indices(dst, seed, step, K, B, N, (cudaStream_t)stream);
+  if (e != cudaSuccess) return fail_cuda(nullptr, e, "lsgd_sample_indices");
+  return LSGD_OK;
+}
+
+}  // extern "C"

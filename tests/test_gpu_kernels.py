@@ -1,0 +1,117 @@
+"""GPU parity of the stand-alone kernels against the oracle: mini-batch indices (bit-exact), He
+initialisation, the fused momentum-SGD update and the K-way average (Eq. 2 right, 1e-6 relative)."""
+import numpy as np
+import pytest
+
+import oracle
+from _gpu_common import built_package, dense_cfgs
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def P():
+    return built_package()
+
+
+@pytest.fixture(scope="module")
+def torch():
+    import torch
+
+    assert torch.cuda.is_available()
+    return torch
+
+
+@pytest.mark.parametrize("K,B,N,seed", [(4, 32, 8192, 0), (16, 128, 50000, 1), (64, 32, 50000, 2),
+                                        (3, 5, 31, 7), (1, 1, 1, 0), (8, 33, 50000, 2**40 + 5)])
+def test_indices_bit_exact(P, torch, K, B, N, seed):
+    dst = torch.empty((K, B), dtype=torch.int32, device="cuda")
+    oc = oracle.make_cfg(K=K, B=B, N=N, seed=seed)
+    for step in (0, 1, 7, 123456):
+        P.lsgd_sample_indices(dst, seed, step, K, B, N)
+        torch.cuda.synchronize()
+        got = dst.cpu().numpy()
+        want = np.stack([oracle.sample_indices(oc, k, step) for k in range(K)])
+        assert np.array_equal(got, want), (step,)
+
+
+def test_context_indices_and_init_match_oracle(P, torch):
+    g, o = dense_cfgs(P, widths=(3072, 1024, 1024, 10), K=16, B=128, H=16, T=49, N=50000,
+                      precision=P.BF16, seed=11)
+    ctx = P.lsgd_create(g)
+    w0 = P.lsgd_params(ctx, 3)
+    want = oracle.init_params(o)
+    assert np.abs(w0 - want).max() <= 1e-6 * np.abs(want).max()
+    # every replica starts from the same model (Algorithm 1 synchronises the initial models)
+    assert np.array_equal(P.lsgd_params(ctx, 0), P.lsgd_params(ctx, 15))
+    for step in (0, 48):
+        got = P.lsgd_debug_indices(ctx, step, 16, 128)
+        assert np.array_equal(got, np.stack([oracle.sample_indices(o, k, step) for k in range(16)]))
+    P.lsgd_destroy(ctx)
+
+
+@pytest.mark.parametrize("K,d", [(1, 4), (3, 1028), (4, 4096 + 36), (16, 67 * 1024 + 12), (64, 2052),
+                                 (33, 96)])
+def test_kway_average(P, torch, K, d):
+    gen = torch.Generator(device="cuda").manual_seed(K * 1000 + d)
+    W = torch.randn((K, d), device="cuda", generator=gen, dtype=torch.float32) * 3
+    Wb = torch.zeros((K, d), device="cuda", dtype=torch.bfloat16)
+    W0 = W.cpu().numpy().astype(np.float64)
+    ref = oracle.average(W0)
+    P.lsgd_kway_average(W, Wb, K, d)
+    torch.cuda.synchronize()
+    got = W.cpu().numpy()
+    # every replica holds exactly the same mean afterwards
+    assert all(np.array_equal(got[0], got[k]) for k in range(K))
+    # |a_i - o_i| / ((1/K) sum_k |w_k,i|) <= 1e-6 (no penalty for cancellation in the mean)
+    err = np.abs(got[0] - ref[0]) / np.maximum(np.abs(W0).mean(0), 1e-30)
+    assert err.max() <= 1e-6, float(err.max())
+    assert torch.equal(Wb.float(), W.to(torch.bfloat16).float())
+
+
+def test_kway_average_of_identical_replicas_is_identity(P, torch):
+    w = torch.randn(4096, device="cuda")
+    W = w.repeat(8, 1).contiguous()
+    P.lsgd_kway_average(W, None, 8, 4096)
+    torch.cuda.synchronize()
+    assert torch.equal(W[5], w)
+
+
+@pytest.mark.parametrize("mom,nest,wd", [(0.0, False, 0.0), (0.9, False, 0.0), (0.9, True, 5e-4),
+                                         (0.0, False, 1e-4)])
+def test_sgd_update(P, torch, mom, nest, wd):
+    n = 4 * 10007
+    gen = torch.Generator(device="cuda").manual_seed(3)
+    w = torch.randn(n, device="cuda", generator=gen)
+    u = torch.randn(n, device="cuda", generator=gen)
+    g = torch.randn(n, device="cuda", generator=gen)
+    wb = torch.zeros(n, device="cuda", dtype=torch.bfloat16)
+    oc = oracle.make_cfg(widths=(n, 1), has_bias=False, momentum=mom, nesterov=nest, weight_decay=wd)
+    w_ref, u_ref = oracle.sgd_update(oc, 0.05, w.cpu().numpy(), u.cpu().numpy(), g.cpu().numpy())
+    P.lsgd_sgd_update(w, u, g, wb, n, 0.05, mom, nest, wd)
+    torch.cuda.synchronize()
+    np.testing.assert_allclose(w.cpu().numpy(), w_ref, rtol=1e-6, atol=1e-6)
+    if mom != 0.0:
+        np.testing.assert_allclose(u.cpu().numpy(), u_ref, rtol=1e-6, atol=1e-6)
+    assert torch.equal(wb.float(), w.to(torch.bfloat16).float())
+
+
+def test_sgd_update_decay_region(P, torch):
+    # weight decay only where (i mod period) < decay_end (BatchNorm gamma / beta are exempt, Sec. A.4)
+    period, end, K = 64, 40, 3
+    n = period * K
+    w = torch.ones(n, device="cuda")
+    g = torch.zeros(n, device="cuda")
+    P.lsgd_sgd_update(w, None, g, None, n, 1.0, 0.0, False, 0.5, period, end)
+    torch.cuda.synchronize()
+    got = w.cpu().numpy().reshape(K, period)
+    assert np.all(got[:, :end] == 0.5) and np.all(got[:, end:] == 1.0)
+
+
+def test_bad_arguments_are_rejected(P, torch):
+    W = torch.zeros(10, device="cuda")
+    with pytest.raises(P.LsgdError) as e:
+        P.lsgd_kway_average(W, None, 2, 5)  # d not a multiple of 4
+    assert e.value.status == P.EINVAL
+    with pytest.raises(P.LsgdError):
+        P.lsgd_sgd_update(W, None, W, None, 6, 0.1, 0.9)  # momentum without a buffer

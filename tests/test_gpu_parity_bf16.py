@@ -1,0 +1,126 @@
+"""bf16-GEMM parity (tcgen05 grouped GEMMs, fp32 accumulation, fp32 master weights).
+
+Tolerances: after 64 steps the parameters within 2e-2 relative L2 of the oracle's and the loss of
+the averaged model within 1e-2 absolute; indices bit-exact.  The full-size MLP 3072-1024-1024-10
+run (K = 16, B = 128, N = 50,000) is checked on sampled replicas the oracle recomputes one by one.
+The tcgen05 products are also compared against the SIMT products on the same bf16 operands."""
+import os
+
+import numpy as np
+import pytest
+
+import oracle
+import synthdata
+from _gpu_common import built_package, dense_cfgs, rel_l2
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def P():
+    import torch
+
+    assert torch.cuda.is_available()
+    return built_package()
+
+
+def _run_both(P, g, o, X, y, steps):
+    w0 = oracle.init_params(o)
+    ctx = P.lsgd_create(g)
+    P.lsgd_set_dataset(ctx, X, y)
+    P.lsgd_set_params(ctx, -1, w0.astype(np.float32))
+    P.lsgd_run(ctx, steps)
+    W, _, losses, syncs = oracle.run(o, X, y=y, W=np.tile(w0.astype(np.float32).astype(np.float64),
+                                                          (o.K, 1)), n_steps=steps)
+    return ctx, W, losses, syncs
+
+
+@pytest.mark.parametrize("widths,K,B,H", [((264, 136, 72, 10), 3, 40, 4),
+                                          ((128, 256, 100), 4, 128, 16)])
+def test_small_mlp_64_steps(P, widths, K, B, H):
+    N = 1200
+    X, y = synthdata.gaussian_mixture(N, widths[0], widths[-1], seed=21)
+    g, o = dense_cfgs(P, widths=widths, K=K, B=B, H=H, T=64, N=N, precision=P.BF16,
+                      base_lr=0.05, momentum=0.9, nesterov=True, weight_decay=5e-4, seed=2)
+    ctx, W, losses, syncs = _run_both(P, g, o, X, y, 64)
+    w_gpu = P.lsgd_params(ctx, -1)
+    assert rel_l2(w_gpu, W[0]) <= 2e-2
+    assert P.lsgd_sync_count(ctx) == syncs == 64 // H
+    n_eval = min(N, 8192)
+    l_gpu = P.lsgd_eval_loss(ctx, -1, n_eval)
+    l_orc = oracle.eval_loss(o, W[0], X, y=y, n=n_eval)
+    assert abs(l_gpu - l_orc) <= 1e-2, (l_gpu, l_orc)
+    lg = P.lsgd_losses(ctx, 64, K)
+    assert np.abs(lg - losses).max() <= 2e-2
+    P.lsgd_destroy(ctx)
+
+
+def test_post_local_switch_bf16(P):
+    widths = (192, 64, 10)
+    N = 960
+    X, y = synthdata.gaussian_mixture(N, widths[0], 10, seed=3)
+    g, o = dense_cfgs(P, widths=widths, K=4, B=32, H=4, T=20, N=N, precision=P.BF16, t_switch=10,
+                      base_lr=0.05, momentum=0.9, nesterov=True, weight_decay=5e-4, seed=6,
+                      milestones=(0.5, 0.75))
+    ctx, W, _, syncs = _run_both(P, g, o, X, y, 20)
+    assert P.lsgd_sync_count(ctx) == syncs == 10 + 3
+    assert rel_l2(P.lsgd_params(ctx, -1), W[0]) <= 2e-2
+    P.lsgd_destroy(ctx)
+
+
+def test_tcgen05_matches_simt_products(P):
+    # Same bf16 operands, fp32 accumulation in both: one step's update agrees to ~1e-4.
+    widths = (3072, 1024, 1024, 10)
+    N = 4096
+    X, y = synthdata.gaussian_mixture(N, 3072, 10, seed=8)
+    outs = {}
+    for mode in ("tc", "simt"):
+        os.environ["LSGD_FORCE_SIMT"] = "1" if mode == "simt" else "0"
+        try:
+            g, o = dense_cfgs(P, widths=widths, K=4, B=128, H=16, T=49, N=N, precision=P.BF16,
+                              base_lr=0.1, momentum=0.9, nesterov=True, weight_decay=5e-4, seed=1)
+            ctx = P.lsgd_create(g)
+        finally:
+            os.environ.pop("LSGD_FORCE_SIMT", None)
+        P.lsgd_set_dataset(ctx, X, y)
+        w0 = P.lsgd_params(ctx, 0)
+        P.lsgd_run(ctx, 1)
+        outs[mode] = (w0, [P.lsgd_params(ctx, k) for k in range(4)], P.lsgd_losses(ctx, 1, 4))
+        P.lsgd_destroy(ctx)
+    w0 = outs["tc"][0]
+    assert np.array_equal(w0, outs["simt"][0])
+    np.testing.assert_allclose(outs["tc"][2], outs["simt"][2], rtol=1e-5, atol=1e-6)
+    for k in range(4):
+        d_tc = outs["tc"][1][k].astype(np.float64) - w0
+        d_si = outs["simt"][1][k].astype(np.float64) - w0
+        assert rel_l2(d_tc, d_si) <= 1e-3, k
+
+
+def test_full_size_mlp_sampled_replicas(P):
+    # MLP 3072-1024-1024-10 with K = 16, B = 128 on N = 50,000 points, the launch configuration
+    # of the benchmark.  One step on all replicas; replicas 0 and 15 recomputed by the oracle.
+    widths = (3072, 1024, 1024, 10)
+    N, K, B = 50000, 16, 128
+    X, y = synthdata.gaussian_mixture_cached(N, 3072, 10, 1234)
+    g, o = dense_cfgs(P, widths=widths, K=K, B=B, H=16, T=49, N=N, precision=P.BF16,
+                      base_lr=0.1, scale_by_K=True, warmup_epochs=5, momentum=0.9, nesterov=True,
+                      weight_decay=5e-4, seed=0)
+    w0 = oracle.init_params(o)
+    ctx = P.lsgd_create(g)
+    P.lsgd_set_dataset(ctx, X, y)
+    P.lsgd_set_params(ctx, -1, w0.astype(np.float32))
+    w0 = w0.astype(np.float32).astype(np.float64)
+    P.lsgd_run(ctx, 1)
+    lg = P.lsgd_losses(ctx, 1, K)[0]
+    lr = oracle.lr(o, 0)
+    assert abs(lr - P.lsgd_lr_at(ctx, 0)) < 1e-12
+    for k in (0, K - 1):
+        idx = oracle.sample_indices(o, k, 0)
+        loss, grad = oracle.loss_grad(o, w0, X, y=y, idx=idx)
+        w1, _ = oracle.sgd_update(o, lr, w0, np.zeros_like(w0), grad)
+        got = P.lsgd_params(ctx, k).astype(np.float64)
+        assert rel_l2(got - w0, w1 - w0) <= 2e-2, k
+        assert abs(lg[k] - loss) <= 1e-2
+    got_idx = P.lsgd_debug_indices(ctx, 0, K, B)
+    assert np.array_equal(got_idx, np.stack([oracle.sample_indices(o, k, 0) for k in range(K)]))
+    P.lsgd_destroy(ctx)

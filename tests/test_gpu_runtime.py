@@ -1,0 +1,169 @@
+"""Runtime behaviour on the GPU: checkpoint / resume, caller-supplied mini-batches, schedule sync
+counts, error handling (bad arguments, call order, failed allocation, non-finite parameters)."""
+import ctypes
+import os
+import tempfile
+
+import numpy as np
+import pytest
+
+import oracle
+import synthdata
+from _gpu_common import built_package, dense_cfgs
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def P():
+    import torch
+
+    assert torch.cuda.is_available()
+    return built_package()
+
+
+def _small(P, precision, **kw):
+    widths = kw.pop("widths", (128, 64, 10))
+    args = dict(widths=widths, K=4, B=16, H=3, T=12, N=512, precision=precision, base_lr=0.05,
+                momentum=0.9, nesterov=True, weight_decay=5e-4, seed=3)
+    args.update(kw)
+    g, o = dense_cfgs(P, **args)
+    X, y = synthdata.gaussian_mixture(args["N"], widths[0], widths[-1], seed=1)
+    return g, o, X, y
+
+
+@pytest.mark.parametrize("prec", ["fp32", "bf16"])
+def test_checkpoint_resume_is_bitwise(P, prec):
+    pr = P.FP32 if prec == "fp32" else P.BF16
+    g, o, X, y = _small(P, pr)
+    a = P.lsgd_create(g)
+    P.lsgd_set_dataset(a, X, y)
+    P.lsgd_run(a, 12)
+    want = [P.lsgd_params(a, k) for k in range(4)]
+    b = P.lsgd_create(g)
+    P.lsgd_set_dataset(b, X, y)
+    P.lsgd_run(b, 5)
+    with tempfile.TemporaryDirectory() as d:
+        path = os.path.join(d, "ck.bin")
+        P.lsgd_save(b, path)
+        c = P.lsgd_create(g)
+        P.lsgd_set_dataset(c, X, y)
+        P.lsgd_load(c, path)
+    assert P.lsgd_step_count(c) == 5 and P.lsgd_sync_count(c) == P.lsgd_sync_count(b)
+    P.lsgd_run(c, 7)
+    for k in range(4):
+        assert np.array_equal(P.lsgd_params(c, k), want[k])
+    assert P.lsgd_sync_count(c) == P.lsgd_sync_count(a) == 4
+    for h in (a, b, c):
+        P.lsgd_destroy(h)
+
+
+@pytest.mark.parametrize("prec", ["fp32", "bf16"])
+def test_caller_batches_equal_sampled_steps(P, prec):
+    import torch
+
+    pr = P.FP32 if prec == "fp32" else P.BF16
+    g, o, X, y = _small(P, pr)
+    a = P.lsgd_create(g)
+    P.lsgd_set_dataset(a, X, y)
+    b = P.lsgd_create(g)
+    P.lsgd_set_dataset(b, X, y)
+    for s in range(3):
+        P.lsgd_local_step(a)
+        idx = P.lsgd_debug_indices(b, s, 4, 16)
+        xb = torch.from_numpy(X[idx.reshape(-1)].reshape(4, 16, -1).copy()).pin_memory()
+        yb = torch.from_numpy(y[idx.reshape(-1)].reshape(4, 16).copy()).pin_memory()
+        if s == 1:
+            xb, yb = xb.cuda(), yb.cuda()
+        P.lsgd_local_step_batch(b, xb, yb)
+    torch.cuda.synchronize()
+    for k in range(4):
+        assert np.array_equal(P.lsgd_params(a, k), P.lsgd_params(b, k))
+    assert np.array_equal(P.lsgd_losses(a, 3, 4), P.lsgd_losses(b, 3, 4))
+    P.lsgd_destroy(a)
+    P.lsgd_destroy(b)
+
+
+def test_sync_counts_follow_schedule(P):
+    for T, H, tp in [(49, 16, -1), (25, 16, 12), (10, 3, 0), (9, 4, 20)]:
+        g, o, X, y = _small(P, P.BF16, T=T, H=H, t_switch=tp)
+        ctx = P.lsgd_create(g)
+        P.lsgd_set_dataset(ctx, X, y)
+        P.lsgd_run(ctx, T)
+        assert P.lsgd_sync_count(ctx) == sum(oracle.is_round_end(o, s) for s in range(T))
+        # the run ends synchronised: every replica holds the average
+        w0 = P.lsgd_params(ctx, 0)
+        assert all(np.array_equal(w0, P.lsgd_params(ctx, k)) for k in range(1, 4))
+        for s in (0, T // 2, T - 1):
+            assert abs(P.lsgd_lr_at(ctx, s) - oracle.lr(o, s)) < 1e-12
+        P.lsgd_destroy(ctx)
+
+
+def test_errors(P):
+    g, o, X, y = _small(P, P.BF16)
+    ctx = P.lsgd_create(g)
+    with pytest.raises(P.LsgdError) as e:
+        P.lsgd_local_step(ctx)
+    assert e.value.status == P.ESTATE
+    with pytest.raises(P.LsgdError) as e:
+        P.lsgd_set_dataset(ctx, X[:100], y[:100])
+    assert e.value.status == P.EINVAL
+    bad = y.copy()
+    bad[3] = 10
+    with pytest.raises(P.LsgdError) as e:
+        P.lsgd_set_dataset(ctx, X, bad)
+    assert e.value.status == P.EINVAL
+    with pytest.raises(P.LsgdError) as e:
+        P.lsgd_params(ctx, 4)
+    assert e.value.status == P.EINVAL
+    P.lsgd_set_dataset(ctx, X, y)
+    P.lsgd_run(ctx, 2)
+    assert P.lsgd_check_finite(ctx)
+    w = P.lsgd_params(ctx, 1)
+    w[17] = np.nan
+    P.lsgd_set_params(ctx, 1, w)
+    assert not P.lsgd_check_finite(ctx)
+    with pytest.raises(P.LsgdError) as e:
+        P.lsgd_load(ctx, "/nonexistent/ck.bin")
+    assert e.value.status == P.EIO
+    P.lsgd_destroy(ctx)
+
+
+def test_failed_allocation_reports_enomem(P):
+    import torch
+
+    calls = {"n": 0}
+
+    def _alloc(user, nbytes, stream):
+        calls["n"] += 1
+        if calls["n"] >= 3:
+            return None  # injected allocation failure
+        return torch.cuda.caching_allocator_alloc(int(nbytes), 0, stream)
+
+    def _free(user, p, stream):
+        torch.cuda.caching_allocator_delete(p)
+
+    cb = (P.ALLOC_FN(_alloc), P.FREE_FN(_free))
+    a = P.Allocator(cb[0], cb[1], None)
+    g, o, X, y = _small(P, P.FP32)
+    with pytest.raises(P.LsgdError) as e:
+        P.lsgd_create(g, allocator=a)
+    assert e.value.status == P.ENOMEM
+    # a fresh context still works afterwards
+    ctx = P.lsgd_create(g)
+    P.lsgd_set_dataset(ctx, X, y)
+    P.lsgd_run(ctx, 1)
+    P.lsgd_destroy(ctx)
+
+
+def test_default_allocator_and_launch_count(P):
+    g, o, X, y = _small(P, P.BF16)
+    ctx = P.lsgd_create(g, allocator=None)
+    P.lsgd_set_dataset(ctx, X, y)
+    before = P.lsgd_kernel_launches(ctx)
+    P.lsgd_local_step(ctx)
+    per_step = P.lsgd_kernel_launches(ctx) - before
+    # sample, gather, 2 forward GEMMs, loss, 2 weight-gradient GEMMs, 2 bias sums, 1 data-gradient
+    # GEMM, update
+    assert per_step == 11
+    P.lsgd_destroy(ctx)

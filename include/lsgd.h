@@ -216,6 +216,15 @@ lsgd_status lsgd_sgd_update(float* w, float* u, const float* g, uint16_t* Wb, in
                             float momentum, int nesterov, float weight_decay, int64_t period,
                             int64_t decay_end, void* stream);
 
+/* Grouped bf16 GEMM of the dense layers' products: C[g] = A[g] B[g]^T for g < G, with A[g] an
+ * M x Kd matrix stored [M][Kd] (a_mn = 0, "K-major") or [Kd][M] (a_mn = 1), B[g] an N x Kd matrix
+ * stored [N][Kd] (b_mn = 0) or [Kd][N] (b_mn = 1), groups packed back to back, C [G][M][N] fp32.
+ * engine 0 = tcgen05 / TMEM / TMA kernel, 1 = SIMT kernel (fp32 accumulation in both).  The
+ * contiguous extent of each operand must be a multiple of 8 elements and the pointers 16-byte
+ * aligned (LSGD_EINVAL otherwise).  Device pointers, asynchronous on `stream`. */
+lsgd_status lsgd_grouped_gemm_bf16(const uint16_t* A, int a_mn, const uint16_t* B, int b_mn, float* C,
+                                   int M, int N, int Kd, int G, int engine, void* stream);
+
 /* Worker mini-batch indices for one step into dst [K][B] int32 (device), as lsgd_local_step. */
 lsgd_status lsgd_sample_indices(int32_t* dst, uint64_t seed, int64_t step, int K, int B, int64_t N,
                                 void* stream);

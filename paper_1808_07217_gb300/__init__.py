@@ -34,7 +34,7 @@ EXPORTS = [
     "lsgd_check_finite", "lsgd_save", "lsgd_load", "lsgd_num_params", "lsgd_step_count",
     "lsgd_sync_count", "lsgd_total_steps", "lsgd_lr_at", "lsgd_kernel_launches", "lsgd_last_error",
     "lsgd_kway_average", "lsgd_sgd_update", "lsgd_sample_indices", "lsgd_profile_enable",
-    "lsgd_profile_read",
+    "lsgd_profile_read", "lsgd_grouped_gemm_bf16",
 ]
 PHASES = ["input", "forward", "loss", "backward", "update", "average"]
 
@@ -152,6 +152,8 @@ def lib():
                                  ctypes.c_float, i64, i64, vp], st),
             "lsgd_sample_indices": ([vp, ctypes.c_uint64, i64, ctypes.c_int, ctypes.c_int, i64, vp], st),
             "lsgd_profile_enable": ([vp, ctypes.c_int], st),
+            "lsgd_grouped_gemm_bf16": ([vp, ctypes.c_int, vp, ctypes.c_int, vp, ctypes.c_int,
+                                        ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int, vp], st),
             "lsgd_profile_read": ([vp, P(Profile)], st),
         }
         for name, (args, res) in sig.items():
@@ -394,3 +396,12 @@ def lsgd_profile_read(ctx: Ctx) -> dict:
     p = Profile()
     _check(lib().lsgd_profile_read(ctx.handle, ctypes.byref(p)), ctx)
     return {name: (int(p.count[i]), float(p.ms[i])) for i, name in enumerate(PHASES)}
+
+
+def lsgd_grouped_gemm_bf16(A, a_mn: bool, B, b_mn: bool, C, M: int, N: int, Kd: int, G: int,
+                           engine: int = 0, stream=None):
+    """C[g] = A[g] B[g]^T on CUDA tensors (A, B bfloat16; C float32); engine 0 tcgen05, 1 SIMT."""
+    stream = _current_stream() if stream is None else stream
+    _check(lib().lsgd_grouped_gemm_bf16(_ptr(A), int(bool(a_mn)), _ptr(B), int(bool(b_mn)), _ptr(C),
+                                        int(M), int(N), int(Kd), int(G), int(engine),
+                                        ctypes.c_void_p(stream)))

@@ -33,7 +33,6 @@ namespace {
 
 constexpr int BM = 128;
 constexpr int BK = 64;
-constexpr int STAGES = 4;
 constexpr long long kWaitCycles = 4000000000LL;  // ~2 s at 2 GHz
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
@@ -129,7 +128,7 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
   for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
 }
 
-template <int BN>
+template <int BN, int STAGES>
 struct Smem {
   // stage buffers first (1024-byte aligned for the 128-byte swizzle)
   uint8_t a[STAGES][BM * BK * 2];
@@ -140,11 +139,11 @@ struct Smem {
   uint32_t tmem_base;
 };
 
-template <int BN>
+template <int BN, int STAGES>
 __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__ TcGemmArgs args) {
   extern __shared__ uint8_t smem_raw[];
-  Smem<BN>& sm = *reinterpret_cast<Smem<BN>*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
-                                               ~uintptr_t(1023));
+  Smem<BN, STAGES>& sm = *reinterpret_cast<Smem<BN, STAGES>*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int n0 = blockIdx.x * BN, m0 = blockIdx.y * BM, g = blockIdx.z;
   const int nk = (args.Kd + BK - 1) / BK;
@@ -234,67 +233,91 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
   __syncwarp();
 
   // ---------------- epilogue (all 4 warps) ----------------
+  // The stage buffers are free once the accumulator is complete (every MMA has read its
+  // operands).  The tile leaves TMEM in 64-column chunks: each thread takes its row's 64 fp32
+  // values (bias / ReLU applied), writes them to a padded shared-memory staging tile, and the CTA
+  // then stores the chunk row-contiguously (a warp writes two 256-byte row segments per
+  // instruction), applying the ReLU mask from a coalesced read of the stored activation.
   const bool have_acc = mbar_wait(&sm.accum, 0);
   asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
   if (have_acc) {
-    const int m = m0 + warp * 32 + lane;
-    const bool row_ok = m < args.M;
+    constexpr int CW = 64, PITCH = CW + 4;  // staged chunk width and row pitch (floats)
+    float* stg = reinterpret_cast<float*>(sm.a[0]);
+    const int r = warp * 32 + lane;  // tile row owned in the TMEM phase
     const float* bias = args.bias ? args.bias + (int64_t)g * args.bias_gs : nullptr;
-    char* Cg = reinterpret_cast<char*>(args.C) +
-               ((int64_t)g * args.c_gs + (int64_t)m * args.c_rs) * (args.c_bf16 ? 2 : 4);
-    const char* Mg = args.mask ? reinterpret_cast<const char*>(args.mask) +
-                                     ((int64_t)g * args.mask_gs + (int64_t)m * args.mask_rs) *
-                                         (args.mask_bf16 ? 2 : 4)
-                               : nullptr;
-    for (int c0 = 0; c0 < BN; c0 += 16) {
-      if (n0 + c0 >= args.N) break;  // warp-uniform
-      float v[16];
-      tmem_ld16(tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)c0, v);
-      if (!row_ok) continue;
-      const int nb = n0 + c0;
+    const int epi = args.epi;
+    for (int cc = 0; cc < BN; cc += CW) {
+      if (n0 + cc >= args.N) break;  // block-uniform
 #pragma unroll
-      for (int i = 0; i < 16; ++i) {
-        const int n = nb + i;
-        if (n >= args.N) break;
-        float x = v[i];
-        if (args.epi == EPI_BIAS || args.epi == EPI_BIAS_RELU) x += bias[n];
-        if (args.epi == EPI_BIAS_RELU) x = fmaxf(x, 0.f);
-        if (args.epi == EPI_MASK) {
-          const float mv = args.mask_bf16 ? bf2f(reinterpret_cast<const uint16_t*>(Mg)[n])
-                                          : reinterpret_cast<const float*>(Mg)[n];
-          x = mv > 0.f ? x : 0.f;
-        }
-        v[i] = x;
-      }
-      const bool full16 = nb + 16 <= args.N;
-      if (args.c_bf16) {
-        uint16_t* out = reinterpret_cast<uint16_t*>(Cg) + nb;
-        if (full16 && ((reinterpret_cast<uintptr_t>(out) & 15) == 0)) {
-          uint4 p0, p1;
-          p0.x = (uint32_t)f2bf(v[0]) | ((uint32_t)f2bf(v[1]) << 16);
-          p0.y = (uint32_t)f2bf(v[2]) | ((uint32_t)f2bf(v[3]) << 16);
-          p0.z = (uint32_t)f2bf(v[4]) | ((uint32_t)f2bf(v[5]) << 16);
-          p0.w = (uint32_t)f2bf(v[6]) | ((uint32_t)f2bf(v[7]) << 16);
-          p1.x = (uint32_t)f2bf(v[8]) | ((uint32_t)f2bf(v[9]) << 16);
-          p1.y = (uint32_t)f2bf(v[10]) | ((uint32_t)f2bf(v[11]) << 16);
-          p1.z = (uint32_t)f2bf(v[12]) | ((uint32_t)f2bf(v[13]) << 16);
-          p1.w = (uint32_t)f2bf(v[14]) | ((uint32_t)f2bf(v[15]) << 16);
-          reinterpret_cast<uint4*>(out)[0] = p0;
-          reinterpret_cast<uint4*>(out)[1] = p1;
-        } else {
-          for (int i = 0; i < 16 && nb + i < args.N; ++i) out[i] = f2bf(v[i]);
-        }
-      } else {
-        float* out = reinterpret_cast<float*>(Cg) + nb;
-        if (full16 && ((reinterpret_cast<uintptr_t>(out) & 15) == 0)) {
+      for (int q = 0; q < CW / 16; ++q) {
+        float v[16];
+        tmem_ld16(tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)(cc + 16 * q), v);
+        if (epi == EPI_BIAS || epi == EPI_BIAS_RELU) {
 #pragma unroll
-          for (int q = 0; q < 4; ++q)
-            reinterpret_cast<float4*>(out)[q] =
-                make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+          for (int i = 0; i < 16; ++i) {
+            const int n = n0 + cc + 16 * q + i;
+            float x = v[i] + (n < args.N ? __ldg(bias + n) : 0.f);
+            v[i] = (epi == EPI_BIAS_RELU) ? fmaxf(x, 0.f) : x;
+          }
+        }
+        float4* dst = reinterpret_cast<float4*>(stg + r * PITCH + 16 * q);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) dst[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+      }
+      asm volatile("bar.sync 1, 128;" ::: "memory");
+      // copy-out: item = (row, 4-column group); 16 groups per 64-column row
+      for (int it = threadIdx.x; it < BM * (CW / 4); it += 128) {
+        const int row = it / (CW / 4), grp = it % (CW / 4);
+        const int m = m0 + row, n = n0 + cc + grp * 4;
+        if (m >= args.M || n >= args.N) continue;
+        float4 x = *reinterpret_cast<const float4*>(stg + row * PITCH + grp * 4);
+        const int64_t off = (int64_t)g * args.c_gs + (int64_t)m * args.c_rs + n;
+        const bool full4 = n + 4 <= args.N;
+        if (epi == EPI_MASK) {
+          const int64_t moff = (int64_t)g * args.mask_gs + (int64_t)m * args.mask_rs + n;
+          float mk[4];
+          if (args.mask_bf16) {
+            const uint16_t* mp = reinterpret_cast<const uint16_t*>(args.mask) + moff;
+            if (full4 && ((reinterpret_cast<uintptr_t>(mp) & 7) == 0)) {
+              const uint2 u = __ldg(reinterpret_cast<const uint2*>(mp));
+              mk[0] = bf2f((uint16_t)(u.x & 0xffff));
+              mk[1] = bf2f((uint16_t)(u.x >> 16));
+              mk[2] = bf2f((uint16_t)(u.y & 0xffff));
+              mk[3] = bf2f((uint16_t)(u.y >> 16));
+            } else {
+              for (int i = 0; i < 4; ++i) mk[i] = (n + i < args.N) ? bf2f(mp[i]) : 0.f;
+            }
+          } else {
+            const float* mp = reinterpret_cast<const float*>(args.mask) + moff;
+            for (int i = 0; i < 4; ++i) mk[i] = (n + i < args.N) ? mp[i] : 0.f;
+          }
+          x.x = mk[0] > 0.f ? x.x : 0.f;
+          x.y = mk[1] > 0.f ? x.y : 0.f;
+          x.z = mk[2] > 0.f ? x.z : 0.f;
+          x.w = mk[3] > 0.f ? x.w : 0.f;
+        }
+        if (args.c_bf16) {
+          uint16_t* out = reinterpret_cast<uint16_t*>(args.C) + off;
+          if (full4 && ((reinterpret_cast<uintptr_t>(out) & 7) == 0)) {
+            uint2 o;
+            o.x = (uint32_t)f2bf(x.x) | ((uint32_t)f2bf(x.y) << 16);
+            o.y = (uint32_t)f2bf(x.z) | ((uint32_t)f2bf(x.w) << 16);
+            *reinterpret_cast<uint2*>(out) = o;
+          } else {
+            const float xs[4] = {x.x, x.y, x.z, x.w};
+            for (int i = 0; i < 4 && n + i < args.N; ++i) out[i] = f2bf(xs[i]);
+          }
         } else {
-          for (int i = 0; i < 16 && nb + i < args.N; ++i) out[i] = v[i];
+          float* out = reinterpret_cast<float*>(args.C) + off;
+          if (full4 && ((reinterpret_cast<uintptr_t>(out) & 15) == 0)) {
+            *reinterpret_cast<float4*>(out) = x;
+          } else {
+            const float xs[4] = {x.x, x.y, x.z, x.w};
+            for (int i = 0; i < 4 && n + i < args.N; ++i) out[i] = xs[i];
+          }
         }
       }
+      asm volatile("bar.sync 1, 128;" ::: "memory");
     }
   }
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
@@ -319,9 +342,23 @@ void load_encode() {
     cudaGetLastError();
 }
 
-template <int BN>
+template <int BN, int STAGES>
 constexpr size_t smem_bytes() {
-  return sizeof(Smem<BN>) + 1024;
+  return sizeof(Smem<BN, STAGES>) + 1024;
+}
+
+template <int BN, int STAGES>
+cudaError_t launch_cfg(const TcGemmArgs& a, dim3 grid, cudaStream_t stream) {
+  constexpr size_t smem = smem_bytes<BN, STAGES>();
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<BN, STAGES>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  gemm_tc_kernel<BN, STAGES><<<grid, 128, smem, stream>>>(a);
+  return cudaGetLastError();
 }
 
 }  // namespace
@@ -366,24 +403,30 @@ bool make_tma_map_bf16(CUtensorMap* map, const void* base, uint64_t dim0, uint64
   return r == CUDA_SUCCESS;
 }
 
+int tc_tile_n(int Kd) { return (Kd + BK - 1) / BK <= 2 ? 128 : 64; }
+
 cudaError_t launch_gemm_tc(const TcGemmArgs& a, cudaStream_t stream) {
   if (a.M <= 0 || a.N <= 0 || a.G <= 0) return cudaSuccess;
   if (a.Kd <= 0 || a.G > 65535) return cudaErrorInvalidValue;
+  // The TMA boxes must deliver exactly the tiles the kernel expects (expect-tx byte counts and
+  // shared-memory extents depend on it).
+  const int bn = tc_tile_n(a.Kd);
+  if (a.A.mn_major ? a.A.box_rows != 64 : a.A.box_rows != BM) return cudaErrorInvalidValue;
+  if (a.B.mn_major ? a.B.box_rows != 64 : a.B.box_rows != bn) return cudaErrorInvalidValue;
   if ((a.epi == EPI_BIAS || a.epi == EPI_BIAS_RELU) && !a.bias) return cudaErrorInvalidValue;
   if (a.epi == EPI_MASK && !a.mask) return cudaErrorInvalidValue;
   constexpr int BN = 128;
   dim3 grid((a.N + BN - 1) / BN, (a.M + BM - 1) / BM, a.G);
   if (grid.y > 65535) return cudaErrorInvalidValue;
-  const size_t smem = smem_bytes<BN>();
-  static bool attr_set = false;
-  if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<BN>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    attr_set = true;
-  }
-  gemm_tc_kernel<BN><<<grid, 128, smem, stream>>>(a);
-  return cudaGetLastError();
+  static_assert(BM == kTcTileM, "tile height");
+  // Short reductions (the weight gradient's k = B_loc) need only two stages; the smaller shared
+  // footprint lets three CTAs share an SM so one CTA's epilogue overlaps the others' loads.
+  if ((a.Kd + BK - 1) / BK <= 2) return launch_cfg<BN, 2>(a, grid, stream);
+  // Long reductions (forward, data gradient): 64-wide N tiles with four stages (96 KB) so two
+  // CTAs share an SM and twice as many tiles stream weights at once.
+  constexpr int BN2 = 64;
+  dim3 grid2((a.N + BN2 - 1) / BN2, (a.M + BM - 1) / BM, a.G);
+  return launch_cfg<BN2, 4>(a, grid2, stream);
 }
 
 }  // namespace lsgd

@@ -149,16 +149,37 @@ __global__ void lsq_loss_kernel(const float* __restrict__ z, int ld, const float
   }
 }
 
+// Bias gradient gb[g][o] = sum_j dz[g][j][o].  A 32 x 8 block covers 64 columns: thread (x, y) sums
+// rows y, y + 8, ... of columns 2x and 2x + 1; the eight partial sums are then added in row-slice
+// order through shared memory, so the result does not depend on scheduling.
 template <typename TD>
-__global__ void colsum_kernel(const TD* __restrict__ dz, int ld, int B, int out,
-                              float* __restrict__ gb, int64_t gb_gs) {
+__global__ void __launch_bounds__(256) colsum_kernel(const TD* __restrict__ dz, int ld, int B,
+                                                     int out, float* __restrict__ gb, int64_t gb_gs) {
+  __shared__ float part[8][65];
   const int g = blockIdx.y;
-  const int o = blockIdx.x * blockDim.x + threadIdx.x;
-  if (o >= out) return;
-  const TD* p = dz + (int64_t)g * B * ld + o;
-  float s = 0.f;
-  for (int j = 0; j < B; ++j) s += Elem<TD>::load(p + (int64_t)j * ld);
-  gb[(int64_t)g * gb_gs + o] = s;
+  const int tx = threadIdx.x, ty = threadIdx.y;
+  const int c0 = blockIdx.x * 64 + 2 * tx;
+  const TD* p = dz + (int64_t)g * B * ld;
+  float s0 = 0.f, s1 = 0.f;
+  for (int j = ty; j < B; j += 8) {
+    const TD* r = p + (int64_t)j * ld + c0;
+    if (c0 < out) s0 += Elem<TD>::load(r);
+    if (c0 + 1 < out) s1 += Elem<TD>::load(r + 1);
+  }
+  part[ty][2 * tx] = s0;
+  part[ty][2 * tx + 1] = s1;
+  __syncthreads();
+  if (ty == 0) {
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const int c = c0 + h;
+      if (c >= out) continue;
+      float s = 0.f;
+#pragma unroll
+      for (int q = 0; q < 8; ++q) s += part[q][2 * tx + h];
+      gb[(int64_t)g * gb_gs + c] = s;
+    }
+  }
 }
 
 // ---------------------------------------------------------------------------------------------
@@ -225,26 +246,19 @@ __global__ void __launch_bounds__(256) kway_average_kernel(float4* __restrict__ 
     const bool ok = col < d4;
     const float4 zero4 = make_float4(0.f, 0.f, 0.f, 0.f);
     float4 s = zero4;
-    int k = r;
-    for (; k + 28 < K; k += 32) {  // 8 loads in flight per lane
+    // Batches of eight replicas per lane (r, r + 4, ..., r + 28): all loads of a batch are issued
+    // before any is summed, so up to 8 x 16 B per lane are in flight.
+    for (int k = r; k < K; k += 32) {
       float4 v[8];
 #pragma unroll
-      for (int q = 0; q < 8; ++q) v[q] = ok ? __ldcs(W + (int64_t)(k + 4 * q) * d4 + col) : zero4;
+      for (int q = 0; q < 8; ++q)
+        v[q] = (ok && k + 4 * q < K) ? __ldcs(W + (int64_t)(k + 4 * q) * d4 + col) : zero4;
 #pragma unroll
       for (int q = 0; q < 8; ++q) {
         s.x += v[q].x;
         s.y += v[q].y;
         s.z += v[q].z;
         s.w += v[q].w;
-      }
-    }
-    for (; k < K; k += 4) {
-      if (ok) {
-        const float4 v = __ldcs(W + (int64_t)k * d4 + col);
-        s.x += v.x;
-        s.y += v.y;
-        s.z += v.z;
-        s.w += v.w;
       }
     }
 #pragma unroll
@@ -391,13 +405,14 @@ cudaError_t launch_lsq_loss(const float* z, int ld, const float* targets, int G,
 cudaError_t launch_colsum(const void* dz, bool dz_bf16, int ld, int G, int B, int out, float* gb,
                           int64_t gb_gs, cudaStream_t stream) {
   if (G <= 0 || out <= 0) return cudaSuccess;
-  dim3 grid((out + 127) / 128, G);
+  if (G > 65535) return cudaErrorInvalidValue;
+  dim3 grid((out + 63) / 64, G), block(32, 8);
   if (dz_bf16)
-    colsum_kernel<uint16_t><<<grid, 128, 0, stream>>>(reinterpret_cast<const uint16_t*>(dz), ld, B,
-                                                      out, gb, gb_gs);
+    colsum_kernel<uint16_t><<<grid, block, 0, stream>>>(reinterpret_cast<const uint16_t*>(dz), ld, B,
+                                                        out, gb, gb_gs);
   else
-    colsum_kernel<float><<<grid, 128, 0, stream>>>(reinterpret_cast<const float*>(dz), ld, B, out,
-                                                   gb, gb_gs);
+    colsum_kernel<float><<<grid, block, 0, stream>>>(reinterpret_cast<const float*>(dz), ld, B, out,
+                                                     gb, gb_gs);
   return cudaGetLastError();
 }
 

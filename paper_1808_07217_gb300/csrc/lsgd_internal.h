@@ -72,8 +72,9 @@ cudaError_t launch_gemm_simt(const GemmArgs& a, cudaStream_t stream);
 // A is M x Kd, B is N x Kd (as stored: "K-major" = Kd contiguous, "MN-major" = M/N contiguous),
 // both described by rank-3 TMA maps whose outermost dimension is the replica (group).
 struct TcOperand {
-  CUtensorMap map;  // box: K-major {64 (Kd), rows}; MN-major {64 (M or N), 64 (Kd)}
+  CUtensorMap map;  // box: K-major {64 (Kd), box_rows}; MN-major {64 (M or N), 64 (Kd)}
   bool mn_major;
+  int box_rows;     // rows of the box the map was encoded with (checked before launch)
 };
 
 struct TcGemmArgs {
@@ -95,6 +96,10 @@ struct TcGemmArgs {
 bool make_tma_map_bf16(CUtensorMap* map, const void* base, uint64_t dim0, uint64_t dim1,
                        uint64_t dim2, uint64_t s1, uint64_t s2, uint32_t box0, uint32_t box1);
 cudaError_t launch_gemm_tc(const TcGemmArgs& a, cudaStream_t stream);
+// N-tile width the tcgen05 kernel uses for a reduction of length Kd (the row count a K-major B
+// operand's TMA box must have).
+int tc_tile_n(int Kd);
+constexpr int kTcTileM = 128;
 bool tc_available();
 // 1 if a bounded wait inside a tcgen05 kernel ran out since the last call (then cleared).
 int tc_take_timeout_flag();

@@ -224,10 +224,14 @@ lsgd_status make_tc_maps(lsgd_ctx* c) {
     const void* a_in = c->act[l];
     bool ok = true;
     // forward: A = act [K][B][ld_in] (K-major), B = W [K][out][in] (K-major)
-    ok &= lsgd::make_tma_map_bf16(&L.fwdA.map, a_in, L.in, B, K, L.ld_in, (uint64_t)B * L.ld_in, 64, 128);
-    ok &= lsgd::make_tma_map_bf16(&L.fwdB.map, Wb_l, L.in, L.out, K, L.in, c->d_pad, 64, 128);
+    const int bn = lsgd::tc_tile_n(L.in);
+    ok &= lsgd::make_tma_map_bf16(&L.fwdA.map, a_in, L.in, B, K, L.ld_in, (uint64_t)B * L.ld_in, 64,
+                                  lsgd::kTcTileM);
+    ok &= lsgd::make_tma_map_bf16(&L.fwdB.map, Wb_l, L.in, L.out, K, L.in, c->d_pad, 64, bn);
     L.fwdA.mn_major = false;
+    L.fwdA.box_rows = lsgd::kTcTileM;
     L.fwdB.mn_major = false;
+    L.fwdB.box_rows = bn;
     // weight gradient: A = dZ as [K][B][out] read MN-major (M = out), B = act read MN-major (N = in)
     // The dz buffer used for layer l alternates; both dz buffers share one layout, so the maps are
     // rebuilt per call from the right base (cheap host work, see run_dense_backward).
@@ -361,6 +365,8 @@ lsgd_status dense_backward(lsgd_ctx* c) {
       if (!ok) return fail(c, LSGD_ECUDA, "TMA map encoding failed (wgrad)");
       t.A.mn_major = true;
       t.B.mn_major = true;
+      t.A.box_rows = 64;
+      t.B.box_rows = 64;
       t.C = c->G + Ly.w_off;
       t.c_rs = Ly.in;
       t.c_gs = c->d_pad;
@@ -404,11 +410,14 @@ lsgd_status dense_backward(lsgd_ctx* c) {
         t.N = Ly.in;
         t.Kd = Ly.out;
         t.G = K;
-        bool ok = lsgd::make_tma_map_bf16(&t.A.map, dz, Ly.out, B, K, c->ld_dz, (uint64_t)B * c->ld_dz, 64, 128);
+        bool ok = lsgd::make_tma_map_bf16(&t.A.map, dz, Ly.out, B, K, c->ld_dz, (uint64_t)B * c->ld_dz,
+                                          64, lsgd::kTcTileM);
         ok &= lsgd::make_tma_map_bf16(&t.B.map, c->Wb + Ly.w_off, Ly.in, Ly.out, K, Ly.in, c->d_pad, 64, 64);
         if (!ok) return fail(c, LSGD_ECUDA, "TMA map encoding failed (dgrad)");
         t.A.mn_major = false;
+        t.A.box_rows = lsgd::kTcTileM;
         t.B.mn_major = true;
+        t.B.box_rows = 64;
         t.C = dzp;
         t.c_rs = c->ld_dz;
         t.c_gs = (int64_t)B * c->ld_dz;
@@ -1024,6 +1033,74 @@ lsgd_status lsgd_sgd_update(float* w, float* u, const float* g, uint16_t* Wb, in
   cudaError_t e = lsgd::launch_sgd_update(w, u, g, Wb, n, lr, momentum, nesterov, weight_decay, period,
                                           decay_end, (cudaStream_t)stream);
   if (e != cudaSuccess) return fail_cuda(nullptr, e, "lsgd_sgd_update");
+  return LSGD_OK;
+}
+
+lsgd_status lsgd_grouped_gemm_bf16(const uint16_t* A, int a_mn, const uint16_t* B, int b_mn, float* C,
+                                   int M, int N, int Kd, int G, int engine, void* stream) {
+  if (!A || !B || !C || M < 1 || N < 1 || Kd < 1 || G < 1 || G > 65535 || (engine != 0 && engine != 1))
+    return fail(nullptr, LSGD_EINVAL, "lsgd_grouped_gemm_bf16: bad arguments");
+  const int a_inner = a_mn ? M : Kd, b_inner = b_mn ? N : Kd;
+  if ((a_inner % 8) || (b_inner % 8) || ((uintptr_t)A & 15) || ((uintptr_t)B & 15) || ((uintptr_t)C & 15))
+    return fail(nullptr, LSGD_EINVAL, "lsgd_grouped_gemm_bf16: contiguous extents must be multiples of 8");
+  cudaStream_t s = (cudaStream_t)stream;
+  cudaError_t e;
+  if (engine == 0) {
+    if (!lsgd::tc_available()) return fail(nullptr, LSGD_EUNSUPPORTED, "tcgen05 not available");
+    lsgd::TcGemmArgs t{};
+    t.M = M;
+    t.N = N;
+    t.Kd = Kd;
+    t.G = G;
+    bool ok;
+    if (a_mn) {
+      ok = lsgd::make_tma_map_bf16(&t.A.map, A, M, Kd, G, M, (uint64_t)M * Kd, 64, 64);
+      t.A.box_rows = 64;
+    } else {
+      ok = lsgd::make_tma_map_bf16(&t.A.map, A, Kd, M, G, Kd, (uint64_t)M * Kd, 64, lsgd::kTcTileM);
+      t.A.box_rows = lsgd::kTcTileM;
+    }
+    const int bn = lsgd::tc_tile_n(Kd);
+    if (b_mn) {
+      ok &= lsgd::make_tma_map_bf16(&t.B.map, B, N, Kd, G, N, (uint64_t)N * Kd, 64, 64);
+      t.B.box_rows = 64;
+    } else {
+      ok &= lsgd::make_tma_map_bf16(&t.B.map, B, Kd, N, G, Kd, (uint64_t)N * Kd, 64, bn);
+      t.B.box_rows = bn;
+    }
+    if (!ok) return fail(nullptr, LSGD_ECUDA, "TMA map encoding failed");
+    t.A.mn_major = a_mn != 0;
+    t.B.mn_major = b_mn != 0;
+    t.C = C;
+    t.c_rs = N;
+    t.c_gs = (int64_t)M * N;
+    t.c_bf16 = false;
+    t.epi = lsgd::EPI_STORE;
+    e = lsgd::launch_gemm_tc(t, s);
+  } else {
+    lsgd::GemmArgs g{};
+    g.M = M;
+    g.N = N;
+    g.Kd = Kd;
+    g.G = G;
+    g.A = A;
+    g.a_rs = a_mn ? 1 : Kd;
+    g.a_cs = a_mn ? M : 1;
+    g.a_gs = (int64_t)M * Kd;
+    g.a_bf16 = true;
+    g.B = B;  // B(k, n) = B[g](n, k)
+    g.b_rs = b_mn ? N : 1;
+    g.b_cs = b_mn ? 1 : Kd;
+    g.b_gs = (int64_t)N * Kd;
+    g.b_bf16 = true;
+    g.C = C;
+    g.c_rs = N;
+    g.c_gs = (int64_t)M * N;
+    g.c_bf16 = false;
+    g.epi = lsgd::EPI_STORE;
+    e = lsgd::launch_gemm_simt(g, s);
+  }
+  if (e != cudaSuccess) return fail_cuda(nullptr, e, "lsgd_grouped_gemm_bf16");
   return LSGD_OK;
 }
 

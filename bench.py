@@ -33,13 +33,16 @@ WORKLOAD = dict(name="mlp_3072-1024-1024-10_K16_B128_H16_bf16", widths=(3072, 10
                 momentum=0.9, nesterov=True, weight_decay=5e-4, seed=0, data_seed=1234)
 
 # Bytes the algorithm moves per parameter and replica (fp32 w, u, g; bf16 shadow):
-#   update  = read g, w, u + write w, u (4 B each) + write bf16 shadow (2 B) = 22
+#   stand-alone update           = read g, w, u + write w, u (4 B each) + write the shadow (2 B) = 22
+#   update fused into the weight-gradient epilogue = read w, u + write w, u + write shadow = 18,
+#     plus the bf16 operands it reads (activations and output gradients, 2 B each)
 #   average = read w + write w (4 B each) + write bf16 shadow (2 B) = 10
 UPDATE_BYTES_PER_PARAM = 22
+FUSED_UPDATE_BYTES_PER_PARAM = 18
 AVERAGE_BYTES_PER_PARAM = 10
-# DRAM bytes per launch of the update kernel from the ncu capture summarised in
-# profiles/sgd_update_kernel_mlp3072_K16.md (None until captured for the current kernel).
-UPDATE_TRAFFIC_PER_LAUNCH = None
+# DRAM bytes per step of the fused weight-gradient + update launches from the ncu capture
+# summarised in profiles/ (None until captured for the current kernel).
+UPDATE_TRAFFIC_PER_STEP = None
 
 FALLBACK_HBM_GBS = 6800.0
 FALLBACK_BF16_TFLOPS = 1900.0
@@ -116,7 +119,7 @@ def _make_cfg(P, total_steps):
                          widths=w["widths"], base_lr=w["base_lr"], scale_by_K=w["scale_by_K"],
                          warmup_epochs=w["warmup_epochs"], momentum=w["momentum"],
                          nesterov=w["nesterov"], weight_decay=w["weight_decay"], seed=w["seed"],
-                         precision=P.BF16)
+                         precision=P.BF16, fused_update=True)
 
 
 def _oracle_cfg(oracle, total_steps):
@@ -291,16 +294,19 @@ def main():
     hbm, bf16_peak, peak_src = _peaks()
     upd_n, upd_ms = prof["update"]
     avg_n, avg_ms = prof["average"]
-    upd_bytes = UPDATE_BYTES_PER_PARAM * K * d
-    upd_gbs = upd_bytes / (upd_ms / upd_n / 1000.0) / 1e9
-    avg_gbs = (AVERAGE_BYTES_PER_PARAM * K * d / (avg_ms / avg_n / 1000.0) / 1e9) if avg_n else None
     widths = w["widths"]
+    # The update phase is the three fused weight-gradient + update launches of each step; the
+    # roofline unit is one step's worth of them (bytes summed over the layers).
+    upd_bytes = sum(FUSED_UPDATE_BYTES_PER_PARAM * K * widths[l] * widths[l + 1]
+                    + 2 * K * B * (widths[l] + widths[l + 1]) for l in range(len(widths) - 1))
+    upd_gbs = upd_bytes / (upd_ms / S_ / 1000.0) / 1e9
+    avg_gbs = (AVERAGE_BYTES_PER_PARAM * K * d / (avg_ms / avg_n / 1000.0) / 1e9) if avg_n else None
     gemm_flops = 0
     for l in range(len(widths) - 1):
         mac = B * widths[l] * widths[l + 1]
         gemm_flops += 2 * mac * (3 if l > 0 else 2)
     gemm_flops *= K
-    gemm_ms = (prof["forward"][1] + prof["backward"][1]) / max(prof["forward"][0], 1)
+    gemm_ms = (prof["forward"][1] + prof["backward"][1] + prof["update"][1]) / max(prof["forward"][0], 1)
     gemm_tflops = gemm_flops / (gemm_ms / 1000.0) / 1e12
     phase_ms = {k: v[1] for k, v in prof.items()}
     tot_phase = sum(phase_ms.values())
@@ -324,10 +330,12 @@ def main():
         "e2e": {"value": e2e_value, "unit": "samples/s", "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h},
         "gpu_launches": launches,
-        "roofline": {"kernel": "sgd_update_kernel", "bound": "hbm", "achieved": upd_gbs,
-                     "peak": hbm, "unit": "GB/s", "frac": upd_gbs / hbm,
-                     "peak_source": f"{peak_src} hbm_gbs", "traffic": UPDATE_TRAFFIC_PER_LAUNCH,
-                     "algorithmic_bytes_per_launch": upd_bytes},
+        "roofline": {"kernel": "gemm_tc_kernel weight gradient + fused local update",
+                     "bound": "hbm", "achieved": upd_gbs, "peak": hbm, "unit": "GB/s",
+                     "frac": upd_gbs / hbm, "peak_source": f"{peak_src} hbm_gbs",
+                     "traffic": UPDATE_TRAFFIC_PER_STEP,
+                     "unit_of_work": "one step's weight-gradient + update launches (3 layers)",
+                     "algorithmic_bytes": upd_bytes, "launches_per_unit": upd_n // S_},
         "sync_average": {"gbs": avg_gbs, "frac_of_hbm": (avg_gbs / hbm) if avg_gbs else None,
                          "ms_per_sync": (avg_ms / avg_n) if avg_n else None},
         "step_split": {"local_frac": 1.0 - phase_ms["average"] / tot_phase,

@@ -99,6 +99,10 @@ typedef struct {
   uint64_t seed;         /* keys Philox4x32-10 for sampling and initialisation */
   int precision;         /* lsgd_precision: FP32 = fp32 everywhere; BF16 = bf16 GEMM operands,
                             fp32 accumulation, fp32 master weights and optimizer state */
+  int fused_update;      /* BF16 dense models on tcgen05: 1 = the weight-gradient epilogue (and the
+                            bias-gradient sum) apply the local update directly, so the gradient is
+                            never written to memory; bit-identical to 0, which runs the stand-alone
+                            update kernel over the whole K x d buffer.  Ignored elsewhere. */
 } lsgd_config;
 
 typedef struct lsgd_ctx lsgd_ctx;
@@ -184,8 +188,10 @@ typedef enum {
   LSGD_PH_INPUT = 0,    /* index sampling + row gather / cast (or the caller batch's copy) */
   LSGD_PH_FORWARD = 1,  /* forward GEMMs / convolutions */
   LSGD_PH_LOSS = 2,     /* softmax cross-entropy (or least-squares) loss and its gradient */
-  LSGD_PH_BACKWARD = 3, /* weight / data gradient products and bias sums */
-  LSGD_PH_UPDATE = 4,   /* the fused local update kernel */
+  LSGD_PH_BACKWARD = 3, /* data / weight gradient products and bias sums (with fused_update: the
+                           data-gradient products and the bias sum + update launches) */
+  LSGD_PH_UPDATE = 4,   /* the local update kernel (with fused_update: the weight-gradient
+                           launches that apply the update in their epilogue) */
   LSGD_PH_AVERAGE = 5,  /* the K-way average kernel */
   LSGD_NUM_PHASES = 6
 } lsgd_phase;

@@ -76,14 +76,14 @@ class Config(ctypes.Structure):
                 ("epochs", ctypes.c_double), ("N", ctypes.c_int64), ("model", Model),
                 ("lr", LrSchedule), ("momentum", ctypes.c_double), ("nesterov", ctypes.c_int),
                 ("weight_decay", ctypes.c_double), ("seed", ctypes.c_uint64),
-                ("precision", ctypes.c_int)]
+                ("precision", ctypes.c_int), ("fused_update", ctypes.c_int)]
 
 
 def make_config(K=1, B_loc=1, H=1, t_switch=-1, total_steps=0, epochs=0.0, N=1, kind=MLP,
                 widths=(3072, 10), init=INIT_HE, in_hwc=(32, 32, 3), n_classes=10, base_ch=16,
                 res_blocks=3, base_lr=0.1, scale_by_K=False, warmup_epochs=0.0, milestones=(),
                 decay=0.1, momentum=0.0, nesterov=False, weight_decay=0.0, seed=0,
-                precision=FP32) -> Config:
+                precision=FP32, fused_update=False) -> Config:
     c = Config()
     c.K, c.B_loc, c.H = int(K), int(B_loc), int(H)
     c.t_switch, c.total_steps, c.epochs, c.N = int(t_switch), int(total_steps), float(epochs), int(N)
@@ -105,6 +105,7 @@ def make_config(K=1, B_loc=1, H=1, t_switch=-1, total_steps=0, epochs=0.0, N=1, 
     c.momentum, c.nesterov, c.weight_decay = float(momentum), int(bool(nesterov)), float(weight_decay)
     c.seed = int(seed)
     c.precision = int(precision)
+    c.fused_update = int(bool(fused_update))
     return c
 
 

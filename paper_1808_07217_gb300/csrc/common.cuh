@@ -46,6 +46,22 @@ __device__ __forceinline__ uint16_t f2bf(float f) {
 
 __device__ __forceinline__ float bf2f(uint16_t u) { return __uint_as_float(((uint32_t)u) << 16); }
 
+// One element of the local update (Sec. C.3.1 / A.4): g' = g + lam w; u = m u + g';
+// w -= lr (nesterov ? g' + m u : u), or w -= lr g' without momentum.  Every kernel that updates
+// parameters goes through this function, so fused and stand-alone updates agree bit for bit.
+template <bool MOM, bool NEST>
+__device__ __forceinline__ void sgd_elem(float& w, float& u, float g, float lr, float m, float lam) {
+  const float gp = fmaf(lam, w, g);
+  float st;
+  if (MOM) {
+    u = fmaf(m, u, gp);
+    st = NEST ? fmaf(m, u, gp) : u;
+  } else {
+    st = gp;
+  }
+  w = fmaf(-lr, st, w);
+}
+
 template <typename T>
 struct Elem;
 template <>

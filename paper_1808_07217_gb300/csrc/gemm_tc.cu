@@ -128,6 +128,26 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
   for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
 }
 
+// The local update on four consecutive parameters (fused weight-gradient epilogue).
+__device__ __forceinline__ void sgd4(float4& w, float4& u, const float4 g, const SgdParams& sp) {
+  if (sp.mom == 0.f) {
+    sgd_elem<false, false>(w.x, u.x, g.x, sp.lr, 0.f, sp.wd);
+    sgd_elem<false, false>(w.y, u.y, g.y, sp.lr, 0.f, sp.wd);
+    sgd_elem<false, false>(w.z, u.z, g.z, sp.lr, 0.f, sp.wd);
+    sgd_elem<false, false>(w.w, u.w, g.w, sp.lr, 0.f, sp.wd);
+  } else if (sp.nesterov) {
+    sgd_elem<true, true>(w.x, u.x, g.x, sp.lr, sp.mom, sp.wd);
+    sgd_elem<true, true>(w.y, u.y, g.y, sp.lr, sp.mom, sp.wd);
+    sgd_elem<true, true>(w.z, u.z, g.z, sp.lr, sp.mom, sp.wd);
+    sgd_elem<true, true>(w.w, u.w, g.w, sp.lr, sp.mom, sp.wd);
+  } else {
+    sgd_elem<true, false>(w.x, u.x, g.x, sp.lr, sp.mom, sp.wd);
+    sgd_elem<true, false>(w.y, u.y, g.y, sp.lr, sp.mom, sp.wd);
+    sgd_elem<true, false>(w.z, u.z, g.z, sp.lr, sp.mom, sp.wd);
+    sgd_elem<true, false>(w.w, u.w, g.w, sp.lr, sp.mom, sp.wd);
+  }
+}
+
 template <int BN, int STAGES>
 struct Smem {
   // stage buffers first (1024-byte aligned for the 128-byte swizzle)
@@ -265,55 +285,124 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
         for (int i = 0; i < 4; ++i) dst[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
       }
       asm volatile("bar.sync 1, 128;" ::: "memory");
-      // copy-out: item = (row, 4-column group); 16 groups per 64-column row
-      for (int it = threadIdx.x; it < BM * (CW / 4); it += 128) {
-        const int row = it / (CW / 4), grp = it % (CW / 4);
-        const int m = m0 + row, n = n0 + cc + grp * 4;
-        if (m >= args.M || n >= args.N) continue;
-        float4 x = *reinterpret_cast<const float4*>(stg + row * PITCH + grp * 4);
-        const int64_t off = (int64_t)g * args.c_gs + (int64_t)m * args.c_rs + n;
-        const bool full4 = n + 4 <= args.N;
-        if (epi == EPI_MASK) {
-          const int64_t moff = (int64_t)g * args.mask_gs + (int64_t)m * args.mask_rs + n;
-          float mk[4];
-          if (args.mask_bf16) {
-            const uint16_t* mp = reinterpret_cast<const uint16_t*>(args.mask) + moff;
-            if (full4 && ((reinterpret_cast<uintptr_t>(mp) & 7) == 0)) {
-              const uint2 u = __ldg(reinterpret_cast<const uint2*>(mp));
-              mk[0] = bf2f((uint16_t)(u.x & 0xffff));
-              mk[1] = bf2f((uint16_t)(u.x >> 16));
-              mk[2] = bf2f((uint16_t)(u.y & 0xffff));
-              mk[3] = bf2f((uint16_t)(u.y >> 16));
+      // copy-out: item = (row, 4-column group), 16 groups per 64-column row.  Each thread takes
+      // UNR items at a time and issues all their global loads (mask, or w and u) before any
+      // arithmetic, so several hundred bytes per thread are in flight.
+      constexpr int UNR = 8, ITEMS = BM * (CW / 4);
+      for (int base = threadIdx.x; base < ITEMS; base += 128 * UNR) {
+        float4 x[UNR], a0[UNR], a1[UNR];
+        int64_t off[UNR];
+        int nn[UNR];
+        bool ok[UNR];
+#pragma unroll
+        for (int q = 0; q < UNR; ++q) {
+          const int it = base + q * 128;
+          const int row = it / (CW / 4), grp = it % (CW / 4);
+          const int m = m0 + row, n = n0 + cc + grp * 4;
+          ok[q] = it < ITEMS && m < args.M && n < args.N;
+          nn[q] = n;
+          off[q] = (int64_t)g * args.c_gs + (int64_t)m * args.c_rs + n;
+          a0[q] = make_float4(0.f, 0.f, 0.f, 0.f);
+          a1[q] = a0[q];
+          if (!ok[q]) continue;
+          x[q] = *reinterpret_cast<const float4*>(stg + row * PITCH + grp * 4);
+          const bool full4 = n + 4 <= args.N;
+          if (epi == EPI_MASK) {
+            const int64_t moff = (int64_t)g * args.mask_gs + (int64_t)m * args.mask_rs + n;
+            if (args.mask_bf16) {
+              const uint16_t* mp = reinterpret_cast<const uint16_t*>(args.mask) + moff;
+              if (full4 && ((reinterpret_cast<uintptr_t>(mp) & 7) == 0)) {
+                const uint2 u = __ldg(reinterpret_cast<const uint2*>(mp));
+                a0[q] = make_float4(bf2f((uint16_t)(u.x & 0xffff)), bf2f((uint16_t)(u.x >> 16)),
+                                    bf2f((uint16_t)(u.y & 0xffff)), bf2f((uint16_t)(u.y >> 16)));
+              } else {
+                float t[4] = {0.f, 0.f, 0.f, 0.f};
+                for (int i = 0; i < 4 && n + i < args.N; ++i) t[i] = bf2f(mp[i]);
+                a0[q] = make_float4(t[0], t[1], t[2], t[3]);
+              }
             } else {
-              for (int i = 0; i < 4; ++i) mk[i] = (n + i < args.N) ? bf2f(mp[i]) : 0.f;
+              const float* mp = reinterpret_cast<const float*>(args.mask) + moff;
+              float t[4] = {0.f, 0.f, 0.f, 0.f};
+              for (int i = 0; i < 4 && n + i < args.N; ++i) t[i] = mp[i];
+              a0[q] = make_float4(t[0], t[1], t[2], t[3]);
+            }
+          } else if (epi == EPI_SGD) {
+            const float* wp = args.sgd.w + off[q];
+            const float* up = args.sgd.u ? args.sgd.u + off[q] : nullptr;
+            if (full4 && ((reinterpret_cast<uintptr_t>(wp) & 15) == 0) &&
+                ((reinterpret_cast<uintptr_t>(up) & 15) == 0)) {
+              a0[q] = __ldcs(reinterpret_cast<const float4*>(wp));
+              if (up) a1[q] = __ldcs(reinterpret_cast<const float4*>(up));
+            } else {
+              float t[4] = {0.f, 0.f, 0.f, 0.f}, v[4] = {0.f, 0.f, 0.f, 0.f};
+              for (int i = 0; i < 4 && n + i < args.N; ++i) {
+                t[i] = wp[i];
+                if (up) v[i] = up[i];
+              }
+              a0[q] = make_float4(t[0], t[1], t[2], t[3]);
+              a1[q] = make_float4(v[0], v[1], v[2], v[3]);
+            }
+          }
+        }
+#pragma unroll
+        for (int q = 0; q < UNR; ++q) {
+          if (!ok[q]) continue;
+          const int n = nn[q];
+          const bool full4 = n + 4 <= args.N;
+          float4 v = x[q];
+          if (epi == EPI_MASK) {
+            v.x = a0[q].x > 0.f ? v.x : 0.f;
+            v.y = a0[q].y > 0.f ? v.y : 0.f;
+            v.z = a0[q].z > 0.f ? v.z : 0.f;
+            v.w = a0[q].w > 0.f ? v.w : 0.f;
+          }
+          if (epi == EPI_SGD) {
+            const SgdParams& sp = args.sgd;
+            float4 wv = a0[q], uv = a1[q];
+            sgd4(wv, uv, v, sp);
+            float* wp = sp.w + off[q];
+            float* up = sp.u ? sp.u + off[q] : nullptr;
+            uint16_t* bp = sp.wb ? sp.wb + off[q] : nullptr;
+            if (full4 && ((reinterpret_cast<uintptr_t>(wp) & 15) == 0) &&
+                ((reinterpret_cast<uintptr_t>(up) & 15) == 0) &&
+                ((reinterpret_cast<uintptr_t>(bp) & 7) == 0)) {
+              __stcs(reinterpret_cast<float4*>(wp), wv);
+              if (up) __stcs(reinterpret_cast<float4*>(up), uv);
+              if (bp) {
+                uint2 o;
+                o.x = (uint32_t)f2bf(wv.x) | ((uint32_t)f2bf(wv.y) << 16);
+                o.y = (uint32_t)f2bf(wv.z) | ((uint32_t)f2bf(wv.w) << 16);
+                __stcs(reinterpret_cast<uint2*>(bp), o);
+              }
+            } else {
+              const float ws[4] = {wv.x, wv.y, wv.z, wv.w}, us[4] = {uv.x, uv.y, uv.z, uv.w};
+              for (int i = 0; i < 4 && n + i < args.N; ++i) {
+                wp[i] = ws[i];
+                if (up) up[i] = us[i];
+                if (bp) bp[i] = f2bf(ws[i]);
+              }
+            }
+            continue;
+          }
+          if (args.c_bf16) {
+            uint16_t* out = reinterpret_cast<uint16_t*>(args.C) + off[q];
+            if (full4 && ((reinterpret_cast<uintptr_t>(out) & 7) == 0)) {
+              uint2 o;
+              o.x = (uint32_t)f2bf(v.x) | ((uint32_t)f2bf(v.y) << 16);
+              o.y = (uint32_t)f2bf(v.z) | ((uint32_t)f2bf(v.w) << 16);
+              *reinterpret_cast<uint2*>(out) = o;
+            } else {
+              const float xs[4] = {v.x, v.y, v.z, v.w};
+              for (int i = 0; i < 4 && n + i < args.N; ++i) out[i] = f2bf(xs[i]);
             }
           } else {
-            const float* mp = reinterpret_cast<const float*>(args.mask) + moff;
-            for (int i = 0; i < 4; ++i) mk[i] = (n + i < args.N) ? mp[i] : 0.f;
-          }
-          x.x = mk[0] > 0.f ? x.x : 0.f;
-          x.y = mk[1] > 0.f ? x.y : 0.f;
-          x.z = mk[2] > 0.f ? x.z : 0.f;
-          x.w = mk[3] > 0.f ? x.w : 0.f;
-        }
-        if (args.c_bf16) {
-          uint16_t* out = reinterpret_cast<uint16_t*>(args.C) + off;
-          if (full4 && ((reinterpret_cast<uintptr_t>(out) & 7) == 0)) {
-            uint2 o;
-            o.x = (uint32_t)f2bf(x.x) | ((uint32_t)f2bf(x.y) << 16);
-            o.y = (uint32_t)f2bf(x.z) | ((uint32_t)f2bf(x.w) << 16);
-            *reinterpret_cast<uint2*>(out) = o;
-          } else {
-            const float xs[4] = {x.x, x.y, x.z, x.w};
-            for (int i = 0; i < 4 && n + i < args.N; ++i) out[i] = f2bf(xs[i]);
-          }
-        } else {
-          float* out = reinterpret_cast<float*>(args.C) + off;
-          if (full4 && ((reinterpret_cast<uintptr_t>(out) & 15) == 0)) {
-            *reinterpret_cast<float4*>(out) = x;
-          } else {
-            const float xs[4] = {x.x, x.y, x.z, x.w};
-            for (int i = 0; i < 4 && n + i < args.N; ++i) out[i] = xs[i];
+            float* out = reinterpret_cast<float*>(args.C) + off[q];
+            if (full4 && ((reinterpret_cast<uintptr_t>(out) & 15) == 0)) {
+              *reinterpret_cast<float4*>(out) = v;
+            } else {
+              const float xs[4] = {v.x, v.y, v.z, v.w};
+              for (int i = 0; i < 4 && n + i < args.N; ++i) out[i] = xs[i];
+            }
           }
         }
       }
@@ -415,6 +504,8 @@ cudaError_t launch_gemm_tc(const TcGemmArgs& a, cudaStream_t stream) {
   if (a.B.mn_major ? a.B.box_rows != 64 : a.B.box_rows != bn) return cudaErrorInvalidValue;
   if ((a.epi == EPI_BIAS || a.epi == EPI_BIAS_RELU) && !a.bias) return cudaErrorInvalidValue;
   if (a.epi == EPI_MASK && !a.mask) return cudaErrorInvalidValue;
+  if (a.epi == EPI_SGD && (!a.sgd.w || (a.sgd.mom != 0.f && !a.sgd.u))) return cudaErrorInvalidValue;
+  if (a.epi != EPI_SGD && !a.C) return cudaErrorInvalidValue;
   constexpr int BN = 128;
   dim3 grid((a.N + BN - 1) / BN, (a.M + BM - 1) / BM, a.G);
   if (grid.y > 65535) return cudaErrorInvalidValue;

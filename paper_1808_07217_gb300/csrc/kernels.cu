@@ -83,47 +83,46 @@ __global__ void gather_rows_kernel(void* __restrict__ dst, int ld_dst, const flo
 }
 
 // ---------------------------------------------------------------------------------------------
-// Softmax cross-entropy: one CTA per group (replica), one warp per row.  Row losses go to shared
-// memory and are summed in row order by one thread, so the result is deterministic.
+// Softmax cross-entropy: one CTA per group (replica), one thread per row, so every row of the
+// group is in flight at once.  Row losses are combined by a fixed-shape tree in shared memory
+// (deterministic).
 template <typename TD>
-__global__ void softmax_xent_kernel(const float* __restrict__ logits, int ld, int C,
-                                    const int32_t* __restrict__ labels, int B, TD* __restrict__ dz,
-                                    int ld_dz, float* __restrict__ loss_mean,
-                                    float* __restrict__ loss_sum, float* __restrict__ row_out) {
-  extern __shared__ float row_loss[];
+__global__ void __launch_bounds__(256) softmax_xent_kernel(
+    const float* __restrict__ logits, int ld, int C, const int32_t* __restrict__ labels, int B,
+    TD* __restrict__ dz, int ld_dz, float* __restrict__ loss_mean, float* __restrict__ loss_sum,
+    float* __restrict__ row_out) {
+  __shared__ float red[256];
   const int g = blockIdx.x;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nwarps = blockDim.x >> 5;
   const float inv_b = 1.0f / (float)B;
-  for (int j = warp; j < B; j += nwarps) {
+  float acc = 0.f;
+  for (int j = threadIdx.x; j < B; j += blockDim.x) {
     const float* z = logits + ((int64_t)g * B + j) * ld;
     float mx = -INFINITY;
-    for (int c = lane; c < C; c += 32) mx = fmaxf(mx, z[c]);
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+    for (int c = 0; c < C; ++c) mx = fmaxf(mx, z[c]);
     float se = 0.f;
-    for (int c = lane; c < C; c += 32) se += expf(z[c] - mx);
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) se += __shfl_xor_sync(0xffffffffu, se, o);
+    for (int c = 0; c < C; ++c) se += expf(z[c] - mx);
     const float lse = mx + logf(se);
     const int y = labels[(int64_t)g * B + j];
     if (dz) {
       TD* dzr = dz + ((int64_t)g * B + j) * ld_dz;
-      for (int c = lane; c < C; c += 32) {
+      for (int c = 0; c < C; ++c) {
         const float p = expf(z[c] - lse);
         Elem<TD>::store(dzr + c, (p - (c == y ? 1.f : 0.f)) * inv_b);
       }
     }
-    if (lane == 0) {
-      row_loss[j] = lse - z[y];
-      if (row_out) row_out[(int64_t)g * B + j] = lse - z[y];
-    }
+    const float l = lse - z[y];
+    if (row_out) row_out[(int64_t)g * B + j] = l;
+    acc += l;
   }
+  red[threadIdx.x] = acc;
   __syncthreads();
+  for (int w = blockDim.x / 2; w > 0; w >>= 1) {
+    if (threadIdx.x < w) red[threadIdx.x] += red[threadIdx.x + w];
+    __syncthreads();
+  }
   if (threadIdx.x == 0) {
-    float s = 0.f;
-    for (int j = 0; j < B; ++j) s += row_loss[j];
-    if (loss_mean) loss_mean[g] = s * inv_b;
-    if (loss_sum) loss_sum[g] = s;
+    if (loss_mean) loss_mean[g] = red[0] * inv_b;
+    if (loss_sum) loss_sum[g] = red[0];
   }
 }
 
@@ -152,9 +151,10 @@ __global__ void lsq_loss_kernel(const float* __restrict__ z, int ld, const float
 // Bias gradient gb[g][o] = sum_j dz[g][j][o].  A 32 x 8 block covers 64 columns: thread (x, y) sums
 // rows y, y + 8, ... of columns 2x and 2x + 1; the eight partial sums are then added in row-slice
 // order through shared memory, so the result does not depend on scheduling.
-template <typename TD>
+template <typename TD, bool UPD>
 __global__ void __launch_bounds__(256) colsum_kernel(const TD* __restrict__ dz, int ld, int B,
-                                                     int out, float* __restrict__ gb, int64_t gb_gs) {
+                                                     int out, float* __restrict__ gb, int64_t gb_gs,
+                                                     SgdParams sgd) {
   __shared__ float part[8][65];
   const int g = blockIdx.y;
   const int tx = threadIdx.x, ty = threadIdx.y;
@@ -177,7 +177,21 @@ __global__ void __launch_bounds__(256) colsum_kernel(const TD* __restrict__ dz, 
       float s = 0.f;
 #pragma unroll
       for (int q = 0; q < 8; ++q) s += part[q][2 * tx + h];
-      gb[(int64_t)g * gb_gs + c] = s;
+      const int64_t i = (int64_t)g * gb_gs + c;
+      if (!UPD) {
+        gb[i] = s;
+      } else {
+        float w = sgd.w[i], u = sgd.u ? sgd.u[i] : 0.f;
+        if (sgd.mom == 0.f)
+          sgd_elem<false, false>(w, u, s, sgd.lr, 0.f, sgd.wd);
+        else if (sgd.nesterov)
+          sgd_elem<true, true>(w, u, s, sgd.lr, sgd.mom, sgd.wd);
+        else
+          sgd_elem<true, false>(w, u, s, sgd.lr, sgd.mom, sgd.wd);
+        sgd.w[i] = w;
+        if (sgd.u) sgd.u[i] = u;
+        if (sgd.wb) sgd.wb[i] = f2bf(w);
+      }
     }
   }
 }
@@ -197,24 +211,12 @@ __global__ void __launch_bounds__(256) sgd_update_kernel(
     float4 wv = __ldcs(w + i);
     float lam = wd;
     if (period > 0 && ((i * 4) % period) >= decay_end) lam = 0.f;
-    float gp[4] = {fmaf(lam, wv.x, gv.x), fmaf(lam, wv.y, gv.y), fmaf(lam, wv.z, gv.z),
-                   fmaf(lam, wv.w, gv.w)};
-    float st[4];
-    if (MOM) {
-      float4 uv = __ldcs(u + i);
-      float uu[4] = {fmaf(m, uv.x, gp[0]), fmaf(m, uv.y, gp[1]), fmaf(m, uv.z, gp[2]),
-                     fmaf(m, uv.w, gp[3])};
-#pragma unroll
-      for (int e = 0; e < 4; ++e) st[e] = NEST ? fmaf(m, uu[e], gp[e]) : uu[e];
-      __stcs(u + i, make_float4(uu[0], uu[1], uu[2], uu[3]));
-    } else {
-#pragma unroll
-      for (int e = 0; e < 4; ++e) st[e] = gp[e];
-    }
-    wv.x = fmaf(-lr, st[0], wv.x);
-    wv.y = fmaf(-lr, st[1], wv.y);
-    wv.z = fmaf(-lr, st[2], wv.z);
-    wv.w = fmaf(-lr, st[3], wv.w);
+    float4 uv = MOM ? __ldcs(u + i) : make_float4(0.f, 0.f, 0.f, 0.f);
+    sgd_elem<MOM, NEST>(wv.x, uv.x, gv.x, lr, m, lam);
+    sgd_elem<MOM, NEST>(wv.y, uv.y, gv.y, lr, m, lam);
+    sgd_elem<MOM, NEST>(wv.z, uv.z, gv.z, lr, m, lam);
+    sgd_elem<MOM, NEST>(wv.w, uv.w, gv.w, lr, m, lam);
+    if (MOM) __stcs(u + i, uv);
     __stcs(w + i, wv);
     if (SHADOW) {
       uint2 o;
@@ -375,13 +377,13 @@ cudaError_t launch_softmax_xent(const float* logits, int ld, int C, const int32_
                                 float* loss_sum, float* row_loss, cudaStream_t stream) {
   if (G <= 0 || B <= 0) return cudaSuccess;
   if (B > 8192 || C < 1) return cudaErrorInvalidValue;
-  const size_t smem = (size_t)B * sizeof(float);
+  const int threads = B >= 256 ? 256 : (B >= 128 ? 128 : (B >= 64 ? 64 : 32));
   if (dz_bf16)
-    softmax_xent_kernel<uint16_t><<<G, 256, smem, stream>>>(
+    softmax_xent_kernel<uint16_t><<<G, threads, 0, stream>>>(
         logits, ld, C, labels, B, reinterpret_cast<uint16_t*>(dz), ld_dz, loss_mean, loss_sum,
         row_loss);
   else
-    softmax_xent_kernel<float><<<G, 256, smem, stream>>>(
+    softmax_xent_kernel<float><<<G, threads, 0, stream>>>(
         logits, ld, C, labels, B, reinterpret_cast<float*>(dz), ld_dz, loss_mean, loss_sum,
         row_loss);
   return cudaGetLastError();
@@ -407,12 +409,27 @@ cudaError_t launch_colsum(const void* dz, bool dz_bf16, int ld, int G, int B, in
   if (G <= 0 || out <= 0) return cudaSuccess;
   if (G > 65535) return cudaErrorInvalidValue;
   dim3 grid((out + 63) / 64, G), block(32, 8);
+  const SgdParams none{};
   if (dz_bf16)
-    colsum_kernel<uint16_t><<<grid, block, 0, stream>>>(reinterpret_cast<const uint16_t*>(dz), ld, B,
-                                                        out, gb, gb_gs);
+    colsum_kernel<uint16_t, false><<<grid, block, 0, stream>>>(
+        reinterpret_cast<const uint16_t*>(dz), ld, B, out, gb, gb_gs, none);
   else
-    colsum_kernel<float><<<grid, block, 0, stream>>>(reinterpret_cast<const float*>(dz), ld, B, out,
-                                                     gb, gb_gs);
+    colsum_kernel<float, false><<<grid, block, 0, stream>>>(reinterpret_cast<const float*>(dz), ld, B,
+                                                            out, gb, gb_gs, none);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_colsum_update(const void* dz, bool dz_bf16, int ld, int G, int B, int out,
+                                 int64_t gs, const SgdParams& sgd, cudaStream_t stream) {
+  if (G <= 0 || out <= 0) return cudaSuccess;
+  if (G > 65535 || !sgd.w || (sgd.mom != 0.f && !sgd.u)) return cudaErrorInvalidValue;
+  dim3 grid((out + 63) / 64, G), block(32, 8);
+  if (dz_bf16)
+    colsum_kernel<uint16_t, true><<<grid, block, 0, stream>>>(reinterpret_cast<const uint16_t*>(dz),
+                                                              ld, B, out, nullptr, gs, sgd);
+  else
+    colsum_kernel<float, true><<<grid, block, 0, stream>>>(reinterpret_cast<const float*>(dz), ld, B,
+                                                           out, nullptr, gs, sgd);
   return cudaGetLastError();
 }
 

@@ -7,6 +7,15 @@
 
 namespace lsgd {
 
+// Parameters of the fused local update (arrays indexed like the GEMM output C).
+struct SgdParams {
+  float* w;
+  float* u;      // may be NULL when mom == 0
+  uint16_t* wb;  // bf16 shadow (may be NULL)
+  float lr, mom, wd;
+  int nesterov;
+};
+
 // ---- element-wise / reduction kernels (kernels.cu) ----
 cudaError_t launch_sample_indices(int32_t* idx, uint64_t seed, int64_t step, int K, int B, int64_t N,
                                   cudaStream_t stream);
@@ -28,6 +37,10 @@ cudaError_t launch_lsq_loss(const float* z, int ld, const float* targets, int G,
 // gb[g * gb_gs + o] = sum_j dz[g][j][o] for o < out.
 cudaError_t launch_colsum(const void* dz, bool dz_bf16, int ld, int G, int B, int out, float* gb,
                           int64_t gb_gs, cudaStream_t stream);
+// Bias gradient fused with the local update: b (at sgd.w + g * gs) receives the update step
+// computed from sum_j dz[g][j][o] instead of the gradient being stored.
+cudaError_t launch_colsum_update(const void* dz, bool dz_bf16, int ld, int G, int B, int out,
+                                 int64_t gs, const SgdParams& sgd, cudaStream_t stream);
 cudaError_t launch_sgd_update(float* w, float* u, const float* g, uint16_t* wb, int64_t n, float lr,
                               float momentum, int nesterov, float weight_decay, int64_t period,
                               int64_t decay_end, cudaStream_t stream);
@@ -44,7 +57,9 @@ enum GemmEpilogue {
   EPI_STORE = 0,      // C = acc
   EPI_BIAS = 1,       // C = acc + bias[n]
   EPI_BIAS_RELU = 2,  // C = max(acc + bias[n], 0)
-  EPI_MASK = 3        // C = mask(m, n) > 0 ? acc : 0   (ReLU derivative from the stored activation)
+  EPI_MASK = 3,       // C = mask(m, n) > 0 ? acc : 0   (ReLU derivative from the stored activation)
+  EPI_SGD = 4         // acc is the gradient of W(m, n): apply the local update to W, U and the bf16
+                      // shadow at C's indexing (nothing is stored to C)
 };
 
 struct GemmArgs {
@@ -80,6 +95,7 @@ struct TcOperand {
 struct TcGemmArgs {
   int M, N, Kd, G;
   TcOperand A, B;
+  SgdParams sgd;  // EPI_SGD only
   // epilogue (same semantics as GemmArgs), C(m, n) at C + g c_gs + m c_rs + n
   void* C;
   int64_t c_rs, c_gs;

@@ -46,6 +46,7 @@ struct lsgd_ctx {
   int64_t d = 0, d_pad = 0, T = 0, shard = 0;
   int D = 0, C = 0;  // input width, outputs
   bool bf16 = false, lsq = false, resnet = false;
+  bool fused = false;  // update applied in the weight-gradient epilogues (see lsgd_config)
   std::vector<DenseLayer> layers;
   std::vector<Seg> segs;
   int64_t wd_period = 0, wd_end = 0;
@@ -344,63 +345,40 @@ lsgd_status dense_forward(lsgd_ctx* c, int groups, int w_g0, int w_gmul) {
   return LSGD_OK;
 }
 
+// Backward of every dense layer, last to first: data gradient (it reads this layer's weights, so
+// it runs before a fused update may change them), weight gradient, bias gradient.
 lsgd_status dense_backward(lsgd_ctx* c) {
   const int K = c->cfg.K, B = c->cfg.B_loc;
   const int L = (int)c->layers.size();
   const void* Wop = c->bf16 ? (const void*)c->Wb : (const void*)c->W;
   const size_t esz = c->bf16 ? 2 : 4;
+  lsgd::SgdParams sgd{};
+  if (c->fused) {
+    sgd.lr = (float)lr_at(c->cfg, c->T, c->step);
+    sgd.mom = (float)c->cfg.momentum;
+    sgd.wd = (float)c->cfg.weight_decay;
+    sgd.nesterov = c->cfg.nesterov;
+  }
+  auto sgd_at = [&](int64_t off) {
+    lsgd::SgdParams p = sgd;
+    p.w = c->W + off;
+    p.u = c->U ? c->U + off : nullptr;
+    p.wb = c->Wb ? c->Wb + off : nullptr;
+    return p;
+  };
+  // Tracing: with the fused update the weight-gradient launches are the update phase, the rest
+  // is the backward phase; otherwise the caller times the whole backward as one span.
+  int64_t e_prev = c->fused ? prof_mark(c) : -1;
+  auto span = [&](int phase) {
+    if (!c->fused) return;
+    const int64_t e = prof_mark(c);
+    prof_span(c, phase, e_prev, e);
+    e_prev = e;
+  };
   int cur = 0;
   for (int l = L - 1; l >= 0; --l) {
     const DenseLayer& Ly = c->layers[l];
     const void* dz = c->dz[cur];
-    // weight gradient G_W[o][i] = sum_j dz[j][o] act[j][i]
-    if (Ly.tc) {
-      lsgd::TcGemmArgs t{};
-      t.M = Ly.out;
-      t.N = Ly.in;
-      t.Kd = B;
-      t.G = K;
-      bool ok = lsgd::make_tma_map_bf16(&t.A.map, dz, Ly.out, B, K, c->ld_dz, (uint64_t)B * c->ld_dz, 64, 64);
-      ok &= lsgd::make_tma_map_bf16(&t.B.map, c->act[l], Ly.in, B, K, Ly.ld_in, (uint64_t)B * Ly.ld_in, 64, 64);
-      if (!ok) return fail(c, LSGD_ECUDA, "TMA map encoding failed (wgrad)");
-      t.A.mn_major = true;
-      t.B.mn_major = true;
-      t.A.box_rows = 64;
-      t.B.box_rows = 64;
-      t.C = c->G + Ly.w_off;
-      t.c_rs = Ly.in;
-      t.c_gs = c->d_pad;
-      t.c_bf16 = false;
-      t.epi = lsgd::EPI_STORE;
-      lsgd_status st = tc_gemm(c, t);
-      if (st != LSGD_OK) return st;
-    } else {
-      lsgd::GemmArgs g{};
-      g.M = Ly.out;
-      g.N = Ly.in;
-      g.Kd = B;
-      g.G = K;
-      g.A = dz;
-      g.a_rs = 1;
-      g.a_cs = c->ld_dz;
-      g.a_gs = (int64_t)B * c->ld_dz;
-      g.a_bf16 = c->bf16;
-      g.B = c->act[l];
-      g.b_rs = Ly.ld_in;
-      g.b_cs = 1;
-      g.b_gs = (int64_t)B * Ly.ld_in;
-      g.b_bf16 = c->bf16;
-      g.C = c->G + Ly.w_off;
-      g.c_rs = Ly.in;
-      g.c_gs = c->d_pad;
-      g.c_bf16 = false;
-      g.epi = lsgd::EPI_STORE;
-      lsgd_status st = gemm(c, g);
-      if (st != LSGD_OK) return st;
-    }
-    if (Ly.b_off >= 0)
-      LSGD_LAUNCH(c, lsgd::launch_colsum(dz, c->bf16, c->ld_dz, K, B, Ly.out, c->G + Ly.b_off,
-                                         c->d_pad, c->stream));
     if (l > 0) {
       // data gradient dz_prev[j][i] = (sum_o dz[j][o] W[o][i]) * (act[j][i] > 0)
       void* dzp = c->dz[1 - cur];
@@ -457,8 +435,69 @@ lsgd_status dense_backward(lsgd_ctx* c) {
         lsgd_status st = gemm(c, g);
         if (st != LSGD_OK) return st;
       }
-      cur = 1 - cur;
+      span(LSGD_PH_BACKWARD);
     }
+    // weight gradient G_W[o][i] = sum_j dz[j][o] act[j][i] (or, fused, the update it drives)
+    if (Ly.tc) {
+      lsgd::TcGemmArgs t{};
+      t.M = Ly.out;
+      t.N = Ly.in;
+      t.Kd = B;
+      t.G = K;
+      bool ok = lsgd::make_tma_map_bf16(&t.A.map, dz, Ly.out, B, K, c->ld_dz, (uint64_t)B * c->ld_dz, 64, 64);
+      ok &= lsgd::make_tma_map_bf16(&t.B.map, c->act[l], Ly.in, B, K, Ly.ld_in, (uint64_t)B * Ly.ld_in, 64, 64);
+      if (!ok) return fail(c, LSGD_ECUDA, "TMA map encoding failed (wgrad)");
+      t.A.mn_major = true;
+      t.B.mn_major = true;
+      t.A.box_rows = 64;
+      t.B.box_rows = 64;
+      t.c_rs = Ly.in;
+      t.c_gs = c->d_pad;
+      t.c_bf16 = false;
+      if (c->fused) {
+        t.epi = lsgd::EPI_SGD;
+        t.sgd = sgd_at(Ly.w_off);
+      } else {
+        t.C = c->G + Ly.w_off;
+        t.epi = lsgd::EPI_STORE;
+      }
+      lsgd_status st = tc_gemm(c, t);
+      if (st != LSGD_OK) return st;
+    } else {
+      lsgd::GemmArgs g{};
+      g.M = Ly.out;
+      g.N = Ly.in;
+      g.Kd = B;
+      g.G = K;
+      g.A = dz;
+      g.a_rs = 1;
+      g.a_cs = c->ld_dz;
+      g.a_gs = (int64_t)B * c->ld_dz;
+      g.a_bf16 = c->bf16;
+      g.B = c->act[l];
+      g.b_rs = Ly.ld_in;
+      g.b_cs = 1;
+      g.b_gs = (int64_t)B * Ly.ld_in;
+      g.b_bf16 = c->bf16;
+      g.C = c->G + Ly.w_off;
+      g.c_rs = Ly.in;
+      g.c_gs = c->d_pad;
+      g.c_bf16 = false;
+      g.epi = lsgd::EPI_STORE;
+      lsgd_status st = gemm(c, g);
+      if (st != LSGD_OK) return st;
+    }
+    span(LSGD_PH_UPDATE);
+    if (Ly.b_off >= 0) {
+      if (c->fused)
+        LSGD_LAUNCH(c, lsgd::launch_colsum_update(dz, c->bf16, c->ld_dz, K, B, Ly.out, c->d_pad,
+                                                  sgd_at(Ly.b_off), c->stream));
+      else
+        LSGD_LAUNCH(c, lsgd::launch_colsum(dz, c->bf16, c->ld_dz, K, B, Ly.out, c->G + Ly.b_off,
+                                           c->d_pad, c->stream));
+      span(LSGD_PH_BACKWARD);
+    }
+    if (l > 0) cur = 1 - cur;
   }
   return LSGD_OK;
 }
@@ -513,11 +552,13 @@ lsgd_status step_body(lsgd_ctx* c, int64_t e_start) {
     st = dense_backward(c);
     if (st != LSGD_OK) return st;
     e_bwd = prof_mark(c);
-    prof_span(c, LSGD_PH_BACKWARD, e_loss, e_bwd);
+    if (!c->fused) prof_span(c, LSGD_PH_BACKWARD, e_loss, e_bwd);
   }
-  st = do_update(c);
-  if (st != LSGD_OK) return st;
-  prof_span(c, LSGD_PH_UPDATE, e_bwd, prof_mark(c));
+  if (!c->fused) {
+    st = do_update(c);
+    if (st != LSGD_OK) return st;
+    prof_span(c, LSGD_PH_UPDATE, e_bwd, prof_mark(c));
+  }
   c->step++;
   return LSGD_OK;
 }
@@ -640,6 +681,10 @@ lsgd_status lsgd_create(const lsgd_config* cfg, const lsgd_allocator* alloc, voi
     st = alloc_dense(c);
     if (st == LSGD_OK) st = init_dense_params(c);
     if (st == LSGD_OK) st = make_tc_maps(c);
+    if (st == LSGD_OK && c0.fused_update && c->bf16) {
+      c->fused = true;
+      for (const DenseLayer& L : c->layers) c->fused = c->fused && L.tc;
+    }
   }
   if (st != LSGD_OK) {
     g_last_error = c->err;

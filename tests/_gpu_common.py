@@ -17,7 +17,7 @@ def built_package():
 
 def dense_cfgs(P, *, widths, K, B, H, T, N, precision, kind="mlp", t_switch=-1, base_lr=0.1,
                scale_by_K=False, warmup_epochs=0.0, milestones=(), momentum=0.0, nesterov=False,
-               weight_decay=0.0, seed=0, init="he"):
+               weight_decay=0.0, seed=0, init="he", fused_update=False):
     """The same run described for the GPU library and for the oracle."""
     gk = {"mlp": P.MLP, "lsq": P.LSQ}[kind]
     ok = {"mlp": oracle.DENSE, "lsq": oracle.LSQ}[kind]
@@ -25,7 +25,8 @@ def dense_cfgs(P, *, widths, K, B, H, T, N, precision, kind="mlp", t_switch=-1, 
                       widths=widths, init=P.INIT_HE if init == "he" else P.INIT_ZERO,
                       base_lr=base_lr, scale_by_K=scale_by_K, warmup_epochs=warmup_epochs,
                       milestones=milestones, momentum=momentum, nesterov=nesterov,
-                      weight_decay=weight_decay, seed=seed, precision=precision)
+                      weight_decay=weight_decay, seed=seed, precision=precision,
+                      fused_update=fused_update)
     o = oracle.make_cfg(kind=ok, widths=widths, has_bias=(kind == "mlp"),
                         bf16=(precision == P.BF16), K=K, B=B, H=H, t_switch=t_switch, T=T, N=N,
                         base_lr=base_lr, scale_by_K=scale_by_K, warmup_epochs=warmup_epochs,

@@ -49,10 +49,11 @@ def test_struct_layout_matches_header(P):
     #include <stddef.h>
     #include "lsgd.h"
     int main(void) {
-      printf("%zu %zu %zu %zu %zu %zu %zu %zu %zu\n", sizeof(lsgd_config), sizeof(lsgd_model),
+      printf("%zu %zu %zu %zu %zu %zu %zu %zu %zu %zu %zu\n", sizeof(lsgd_config), sizeof(lsgd_model),
              sizeof(lsgd_lr_schedule), sizeof(lsgd_allocator), offsetof(lsgd_config, model),
              offsetof(lsgd_config, lr), offsetof(lsgd_config, momentum),
-             offsetof(lsgd_config, seed), offsetof(lsgd_config, precision));
+             offsetof(lsgd_config, seed), offsetof(lsgd_config, precision),
+             offsetof(lsgd_config, fused_update), sizeof(lsgd_profile));
       return 0;
     }
     """
@@ -67,7 +68,7 @@ def test_struct_layout_matches_header(P):
     C = P.Config
     want = [ctypes.sizeof(C), ctypes.sizeof(P.Model), ctypes.sizeof(P.LrSchedule),
             ctypes.sizeof(P.Allocator), C.model.offset, C.lr.offset, C.momentum.offset,
-            C.seed.offset, C.precision.offset]
+            C.seed.offset, C.precision.offset, C.fused_update.offset, ctypes.sizeof(P.Profile)]
     assert got == want
 
 

@@ -109,7 +109,7 @@ def test_full_size_mlp_sampled_replicas(P):
     X, y = synthdata.gaussian_mixture_cached(N, 3072, 10, 1234)
     g, o = dense_cfgs(P, widths=widths, K=K, B=B, H=16, T=49, N=N, precision=P.BF16,
                       base_lr=0.1, scale_by_K=True, warmup_epochs=5, momentum=0.9, nesterov=True,
-                      weight_decay=5e-4, seed=0)
+                      weight_decay=5e-4, seed=0, fused_update=True)
     w0 = oracle.init_params(o)
     ctx = P.lsgd_create(g)
     P.lsgd_set_dataset(ctx, X, y)
@@ -129,3 +129,29 @@ def test_full_size_mlp_sampled_replicas(P):
     got_idx = P.lsgd_debug_indices(ctx, 0, K, B)
     assert np.array_equal(got_idx, np.stack([oracle.sample_indices(o, k, 0) for k in range(K)]))
     P.lsgd_destroy(ctx)
+
+
+@pytest.mark.parametrize("mom,nest,wd", [(0.9, True, 5e-4), (0.9, False, 0.0), (0.0, False, 1e-4)])
+@pytest.mark.parametrize("widths,K,B", [((264, 136, 72, 10), 3, 40), ((3072, 1024, 1024, 10), 4, 128)])
+def test_fused_update_is_bitwise_identical(P, mom, nest, wd, widths, K, B):
+    # The update applied in the weight-gradient epilogue uses the same arithmetic as the
+    # stand-alone update kernel, so parameters, momentum and losses agree bit for bit.
+    N = 2048
+    X, y = synthdata.gaussian_mixture(N, widths[0], widths[-1], seed=4)
+    res = []
+    for fused in (False, True):
+        g, o = dense_cfgs(P, widths=widths, K=K, B=B, H=3, T=7, N=N, precision=P.BF16,
+                          base_lr=0.05, momentum=mom, nesterov=nest, weight_decay=wd, seed=9,
+                          fused_update=fused)
+        ctx = P.lsgd_create(g)
+        P.lsgd_set_dataset(ctx, X, y)
+        P.lsgd_run(ctx, 7)
+        res.append(([P.lsgd_params(ctx, k) for k in range(K)],
+                    [P.lsgd_momentum(ctx, k) for k in range(K)], P.lsgd_losses(ctx, 7, K),
+                    P.lsgd_kernel_launches(ctx)))
+        P.lsgd_destroy(ctx)
+    for k in range(K):
+        assert np.array_equal(res[0][0][k], res[1][0][k])
+        assert np.array_equal(res[0][1][k], res[1][1][k])
+    assert np.array_equal(res[0][2], res[1][2])
+    assert res[1][3] < res[0][3]  # no stand-alone update launches

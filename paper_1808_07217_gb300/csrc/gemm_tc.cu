@@ -82,6 +82,14 @@ __device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, u
       : "memory");
 }
 
+// Fetch a tensor tile into L2 only (no shared memory, no completion tracking).
+__device__ __forceinline__ void tma_prefetch_l2_3d(const CUtensorMap* map, int x, int y, int z) {
+  asm volatile("cp.async.bulk.prefetch.tensor.3d.L2.global.tile [%0, {%1, %2, %3}];" ::"l"(
+                   reinterpret_cast<uint64_t>(map)),
+               "r"(x), "r"(y), "r"(z)
+               : "memory");
+}
+
 __device__ __forceinline__ uint64_t smem_desc(uint32_t addr, uint32_t lbo, uint32_t sbo) {
   uint64_t d = 0;
   d |= (uint64_t)((addr >> 4) & 0x3FFFu);
@@ -194,6 +202,14 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
   bool ok = true;
   if (warp == 0 && lane == 0) {
     // ---------------- TMA producer ----------------
+    if (args.epi == EPI_SGD && args.have_wu_maps) {
+      // the epilogue reads this tile's parameters and momentum: start them towards L2 now
+#pragma unroll
+      for (int i = 0; i < BN / 64; ++i) {
+        tma_prefetch_l2_3d(&args.wmap, n0 + 64 * i, m0, g);
+        if (args.sgd.u) tma_prefetch_l2_3d(&args.umap, n0 + 64 * i, m0, g);
+      }
+    }
     int issued = 0;
     for (int kb = 0; kb < nk && ok; ++kb) {
       const int s = kb % STAGES;
@@ -461,6 +477,21 @@ bool tc_available() {
   }
   std::call_once(g_encode_once, load_encode);
   return p.major == 10 && g_encode != nullptr;
+}
+
+bool make_tma_map_f32(CUtensorMap* map, const void* base, uint64_t dim0, uint64_t dim1,
+                      uint64_t dim2, uint64_t s1, uint64_t s2, uint32_t box0, uint32_t box1) {
+  std::call_once(g_encode_once, load_encode);
+  if (!g_encode) return false;
+  if ((reinterpret_cast<uintptr_t>(base) & 15) || ((s1 * 4) & 15) || ((s2 * 4) & 15)) return false;
+  cuuint64_t dims[3] = {dim0, dim1, dim2};
+  cuuint64_t strides[2] = {s1 * 4, s2 * 4};
+  cuuint32_t box[3] = {box0, box1, 1};
+  cuuint32_t estr[3] = {1, 1, 1};
+  CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, const_cast<void*>(base), dims,
+                        strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
 }
 
 int tc_take_timeout_flag() {

@@ -96,6 +96,10 @@ struct TcGemmArgs {
   int M, N, Kd, G;
   TcOperand A, B;
   SgdParams sgd;  // EPI_SGD only
+  // EPI_SGD: fp32 maps over sgd.w / sgd.u (dims {N, M, G}, box {64, 128}) used to prefetch the
+  // tile's parameters and momentum into L2 while the products run (have_wu_maps = 0: no prefetch)
+  CUtensorMap wmap, umap;
+  int have_wu_maps;
   // epilogue (same semantics as GemmArgs), C(m, n) at C + g c_gs + m c_rs + n
   void* C;
   int64_t c_rs, c_gs;
@@ -111,6 +115,9 @@ struct TcGemmArgs {
 // Encode a rank-3 bf16 TMA map over [dim2][dim1][dim0] with strides (elements) s1, s2.
 bool make_tma_map_bf16(CUtensorMap* map, const void* base, uint64_t dim0, uint64_t dim1,
                        uint64_t dim2, uint64_t s1, uint64_t s2, uint32_t box0, uint32_t box1);
+// The same for fp32 data, without swizzling (used for L2 prefetches of parameter tiles).
+bool make_tma_map_f32(CUtensorMap* map, const void* base, uint64_t dim0, uint64_t dim1,
+                      uint64_t dim2, uint64_t s1, uint64_t s2, uint32_t box0, uint32_t box1);
 cudaError_t launch_gemm_tc(const TcGemmArgs& a, cudaStream_t stream);
 // N-tile width the tcgen05 kernel uses for a reduction of length Kd (the row count a K-major B
 // operand's TMA box must have).

@@ -457,6 +457,10 @@ lsgd_status dense_backward(lsgd_ctx* c) {
       if (c->fused) {
         t.epi = lsgd::EPI_SGD;
         t.sgd = sgd_at(Ly.w_off);
+        t.have_wu_maps =
+            lsgd::make_tma_map_f32(&t.wmap, t.sgd.w, Ly.in, Ly.out, K, Ly.in, c->d_pad, 64, 128) &&
+            (!t.sgd.u ||
+             lsgd::make_tma_map_f32(&t.umap, t.sgd.u, Ly.in, Ly.out, K, Ly.in, c->d_pad, 64, 128));
       } else {
         t.C = c->G + Ly.w_off;
         t.epi = lsgd::EPI_STORE;

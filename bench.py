@@ -180,6 +180,47 @@ def run_reference(args, world, rank):
     print(json.dumps(line), flush=True)
 
 
+def run_sweep(args):
+    """Sync / compute trade-off: MLP 3072-512-512-10, B_loc = 32, heavy-ball momentum 0.9, 500
+    local steps per (K, H) on the synthetic 10-class data; one JSON line per point with samples/s
+    (device time) and the fraction of step time spent in the K-way average."""
+    import torch
+
+    import synthdata
+    from paper_1808_07217_gb300 import _build
+
+    _build.build()
+    import paper_1808_07217_gb300 as P
+
+    torch.cuda.set_device(0)
+    stream = torch.cuda.current_stream()
+    N, B, widths, T = 50000, 32, (3072, 512, 512, 10), 500
+    X, y = synthdata.gaussian_mixture_cached(N, 3072, 10, 1234)
+    for K in (8, 32, 64):
+        for H in (1, 2, 4, 8, 16, 32):
+            cfg = P.make_config(K=K, B_loc=B, H=H, total_steps=T + 20, N=N, widths=widths,
+                                base_lr=0.1, momentum=0.9, seed=0, precision=P.BF16,
+                                fused_update=True)
+            ctx = P.lsgd_create(cfg, stream=stream.cuda_stream)
+            P.lsgd_set_dataset(ctx, X, y)
+            P.lsgd_run(ctx, 20)
+            torch.cuda.synchronize()
+            P.lsgd_profile_enable(ctx, True)
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            P.lsgd_run(ctx, T)
+            e1.record(stream)
+            torch.cuda.synchronize()
+            ms = e0.elapsed_time(e1)
+            prof = P.lsgd_profile_read(ctx)
+            tot = sum(v[1] for v in prof.values())
+            print(json.dumps({"sweep": "mlp_3072-512-512-10_B32", "K": K, "H": H, "steps": T,
+                              "samples_per_s": T * K * B / (ms / 1000.0), "ms_per_step": ms / T,
+                              "sync_frac": prof["average"][1] / tot,
+                              "syncs": prof["average"][0]}), flush=True)
+            P.lsgd_destroy(ctx)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -187,8 +228,13 @@ def main():
     ap.add_argument("--warmup", type=int, default=16)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--sweep", action="store_true",
+                    help="K x H sync / compute sweep of the MLP 3072-512-512-10 workload")
     args = ap.parse_args()
     world, rank, local = _dist()
+    if args.sweep:
+        run_sweep(args)
+        return
 
     if args.impl == "reference":
         run_reference(args, world, rank)

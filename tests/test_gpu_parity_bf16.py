@@ -155,3 +155,64 @@ def test_fused_update_is_bitwise_identical(P, mom, nest, wd, widths, K, B):
         assert np.array_equal(res[0][1][k], res[1][1][k])
     assert np.array_equal(res[0][2], res[1][2])
     assert res[1][3] < res[0][3]  # no stand-alone update launches
+
+
+def test_post_local_mlp4096_sampled_replica(P):
+    # Post-local SGD on MLP 3072-4096-4096-4096-100 (K = 16, B = 128, N = 50,000, 100 classes):
+    # the first step recomputed by the oracle for one sampled replica, then the whole 10-epoch
+    # schedule (t' = first decay = floor(0.5 T)) run on the GPU with its sync count checked.
+    widths = (3072, 4096, 4096, 4096, 100)
+    N, K, B = 50000, 16, 128
+    T = -(-10 * N // (K * B))  # ceil(10 epochs of N samples / (K B))
+    tp = T // 2
+    X, y = synthdata.gaussian_mixture_cached(N, 3072, 100, 1234)
+    g, o = dense_cfgs(P, widths=widths, K=K, B=B, H=16, T=T, N=N, precision=P.BF16, t_switch=tp,
+                      base_lr=0.1, scale_by_K=True, warmup_epochs=5, milestones=(0.5, 0.75),
+                      momentum=0.9, nesterov=True, weight_decay=5e-4, seed=3, fused_update=True)
+    w0 = oracle.init_params(o)
+    ctx = P.lsgd_create(g)
+    P.lsgd_set_dataset(ctx, X, y)
+    P.lsgd_set_params(ctx, -1, w0.astype(np.float32))
+    w0 = w0.astype(np.float32).astype(np.float64)
+    P.lsgd_run(ctx, 1)
+    k = K - 1
+    idx = oracle.sample_indices(o, k, 0)
+    loss, grad = oracle.loss_grad(o, w0, X, y=y, idx=idx)
+    # Step 0 is in the mini-batch phase, so the parameters are averaged right after it; the
+    # worker's momentum stays local and after the first step equals g' = g + lambda w0.
+    got_k = P.lsgd_momentum(ctx, k).astype(np.float64)
+    gp = grad + 5e-4 * w0
+    assert rel_l2(got_k, gp) <= 2e-2
+    assert abs(P.lsgd_losses(ctx, 1, K)[0][k] - loss) <= 1e-2
+    P.lsgd_run(ctx, T - 1)
+    assert P.lsgd_sync_count(ctx) == tp + -(-(T - tp) // 16)
+    assert P.lsgd_check_finite(ctx)
+    lg = P.lsgd_losses(ctx, T, K)
+    print("post-local MLP4096 mean loss every 16 steps:", lg.mean(1)[::16].round(3).tolist())
+    P.lsgd_destroy(ctx)
+
+
+@pytest.mark.parametrize("K", [8, 64])
+def test_sweep_shape_mlp512_sampled_replicas(P, K):
+    # MLP 3072-512-512-10, B = 32, heavy-ball momentum 0.9, H = 4: two local steps on all
+    # replicas; replicas 0 and K-1 recomputed step by step by the oracle.
+    widths = (3072, 512, 512, 10)
+    N, B = 50000, 32
+    X, y = synthdata.gaussian_mixture_cached(N, 3072, 10, 1234)
+    g, o = dense_cfgs(P, widths=widths, K=K, B=B, H=4, T=500, N=N, precision=P.BF16,
+                      base_lr=0.1, momentum=0.9, seed=5, fused_update=True)
+    w0 = oracle.init_params(o).astype(np.float32).astype(np.float64)
+    ctx = P.lsgd_create(g)
+    P.lsgd_set_dataset(ctx, X, y)
+    P.lsgd_set_params(ctx, -1, w0.astype(np.float32))
+    P.lsgd_run(ctx, 2)
+    lg = P.lsgd_losses(ctx, 2, K)
+    for k in (0, K - 1):
+        w, u = w0.copy(), np.zeros_like(w0)
+        for s in range(2):
+            loss, grad = oracle.loss_grad(o, w, X, y=y, idx=oracle.sample_indices(o, k, s))
+            w, u = oracle.sgd_update(o, oracle.lr(o, s), w, u, grad)
+            assert abs(lg[s][k] - loss) <= 1e-2
+        got = P.lsgd_params(ctx, k).astype(np.float64)
+        assert rel_l2(got - w0, w - w0) <= 2e-2, k
+    P.lsgd_destroy(ctx)

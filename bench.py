@@ -221,6 +221,56 @@ def run_sweep(args):
             P.lsgd_destroy(ctx)
 
 
+RESNET_WORKLOAD = dict(name="resnet20_K16_B128_postlocal_H16_bf16", K=16, B=128, H=16, N=50000,
+                       C=10, base_lr=0.2, scale_by_K=True, warmup_epochs=5.0, momentum=0.9,
+                       nesterov=True, weight_decay=1e-4, seed=0, data_seed=1234)
+
+
+def run_resnet(args):
+    """Post-local ResNet-20 (K = 16, B_loc = 128, H = 16 after t' = T / 2): samples/s over the
+    local-SGD phase with the per-phase split.  One JSON line."""
+    import torch
+
+    import synthdata
+    from paper_1808_07217_gb300 import _build
+
+    _build.build()
+    import paper_1808_07217_gb300 as P
+
+    torch.cuda.set_device(0)
+    w = RESNET_WORKLOAD
+    K, B = w["K"], w["B"]
+    X, y = synthdata.gaussian_mixture_cached(w["N"], 3072, w["C"], w["data_seed"])
+    W_, S_ = max(3, args.warmup), args.steps
+    total = W_ + S_
+    stream = torch.cuda.current_stream()
+    cfg = P.make_config(K=K, B_loc=B, H=w["H"], t_switch=0, total_steps=total, N=w["N"],
+                        kind=P.RESNET20, in_hwc=(32, 32, 3), n_classes=w["C"], base_ch=16,
+                        res_blocks=3, base_lr=w["base_lr"], scale_by_K=w["scale_by_K"],
+                        warmup_epochs=w["warmup_epochs"], milestones=(0.5, 0.75),
+                        momentum=w["momentum"], nesterov=w["nesterov"],
+                        weight_decay=w["weight_decay"], seed=w["seed"], precision=P.BF16)
+    ctx = P.lsgd_create(cfg, stream=stream.cuda_stream)
+    P.lsgd_set_dataset(ctx, X, y)
+    P.lsgd_run(ctx, W_)
+    torch.cuda.synchronize()
+    n0 = P.lsgd_kernel_launches(ctx)
+    P.lsgd_profile_enable(ctx, True)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    P.lsgd_run(ctx, S_)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1)
+    prof = P.lsgd_profile_read(ctx)
+    print(json.dumps({"workload": w["name"], "value": S_ * K * B / (ms / 1000.0),
+                      "unit": "samples/s", "steps": S_, "ms_per_step": ms / S_,
+                      "gpu_launches": P.lsgd_kernel_launches(ctx) - n0,
+                      "phase_ms_per_step": {k: v[1] / S_ for k, v in prof.items()},
+                      "params_per_replica": P.lsgd_num_params(ctx)}), flush=True)
+    P.lsgd_destroy(ctx)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -230,10 +280,15 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--sweep", action="store_true",
                     help="K x H sync / compute sweep of the MLP 3072-512-512-10 workload")
+    ap.add_argument("--resnet", action="store_true",
+                    help="post-local ResNet-20 workload (K = 16, B_loc = 128) instead of the MLP")
     args = ap.parse_args()
     world, rank, local = _dist()
     if args.sweep:
         run_sweep(args)
+        return
+    if args.resnet:
+        run_resnet(args)
         return
 
     if args.impl == "reference":

@@ -1,38 +1,864 @@
-// ResNet-20 on the CUDA path.
+// ResNet-20 on the CUDA path, K replicas per launch.
+//
+// The CIFAR network of He et al. 2016 used by the paper (Sec. 4 and A.2: 0.27 M parameters): a 3x3
+// stem convolution, three stages of basic blocks (base, 2 base, 4 base channels; stride 2 at the
+// first block of stages 2 and 3), option-A shortcuts (stride-2 subsampling, zero channels appended
+// after the input channels), BatchNorm with each worker's own batch statistics (Sec. A.4), global
+// average pooling and a fully connected classifier.  Activations are NHWC, replica-major
+// ([K][B][H][W][C]); convolution weights [Cout][3][3][Cin].  In BF16 mode the convolution operands
+// (image, stored activations, weights, output gradients) are bf16; accumulation, BatchNorm,
+// pooling, the classifier and the update are fp32.
+//
+// Reductions over the pixels of a replica (BatchNorm statistics, their backward sums, weight
+// gradients) run in two deterministic passes: per-chunk partial results into a scratch buffer,
+// then a fixed-order combination.
+#include <algorithm>
+#include <cmath>
+#include <string>
+#include <vector>
+
+#include "common.cuh"
+#include "lsgd_internal.h"
 #include "resnet.h"
 
 namespace lsgd {
 
+namespace {
+
+constexpr float kBnEps = 1e-5f;
+constexpr int kStatChunk = 1024;   // pixels per BatchNorm reduction chunk
+constexpr int kWgradChunk = 2048;  // pixels per weight-gradient chunk
+constexpr int kWgradTile = 16;     // pixels staged per weight-gradient iteration
+constexpr int kMaxJ16 = 36;        // (9 Cin) / 16 accumulators per thread, Cin <= 64
+
+struct ConvL {
+  int cin, cout, stride, hin, win, hout, wout;
+  int64_t w_off, g_off, b_off;  // padded per-replica offsets
+  int64_t cw, cg, cb;           // canonical offsets
+};
+
+int64_t rup(int64_t v, int64_t m) { return (v + m - 1) / m * m; }
+
+int grid_cap(int64_t items, int threads) {
+  int64_t b = (items + threads - 1) / threads;
+  return (int)std::max<int64_t>(1, std::min<int64_t>(b, (int64_t)kNumSMs * 16));
+}
+
+// ------------------------------------------------------------------------------------------
+// Direct 3x3 convolution, zero padding 1: y[g][b][oh][ow][co] = sum_{kh,kw,ci}
+// in[g][b][oh s + kh - 1][ow s + kw - 1][ci] w[g][co][kh][kw][ci].  One thread per output pixel
+// and 16 output channels; the 16 channels' weights sit in shared memory.
+template <typename TA>
+__global__ void __launch_bounds__(128) conv_fwd_kernel(const TA* __restrict__ in,
+                                                       const TA* __restrict__ w, int64_t w_gs,
+                                                       float* __restrict__ y, int B, int Hin,
+                                                       int Win, int Cin, int Hout, int Wout,
+                                                       int Cout, int stride) {
+  extern __shared__ float ws[];  // [16][9][Cin]
+  const int g = blockIdx.z, co0 = blockIdx.y * 16;
+  const int nco = min(16, Cout - co0);
+  const TA* wg = w + (int64_t)g * w_gs;
+  const int KC = 9 * Cin;
+  for (int e = threadIdx.x; e < 16 * KC; e += blockDim.x) {
+    const int co = e / KC, r = e % KC;
+    ws[e] = co < nco ? Elem<TA>::load(wg + (int64_t)(co0 + co) * KC + r) : 0.f;
+  }
+  __syncthreads();
+  const int64_t P = (int64_t)B * Hout * Wout;
+  const int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (p >= P) return;
+  const int ow = (int)(p % Wout);
+  const int oh = (int)((p / Wout) % Hout);
+  const int b = (int)(p / ((int64_t)Wout * Hout));
+  float acc[16];
+#pragma unroll
+  for (int i = 0; i < 16; ++i) acc[i] = 0.f;
+  const TA* ing = in + (int64_t)g * B * Hin * Win * Cin;
+  for (int kh = 0; kh < 3; ++kh) {
+    const int ih = oh * stride + kh - 1;
+    if (ih < 0 || ih >= Hin) continue;
+    for (int kw = 0; kw < 3; ++kw) {
+      const int iw = ow * stride + kw - 1;
+      if (iw < 0 || iw >= Win) continue;
+      const TA* src = ing + (((int64_t)b * Hin + ih) * Win + iw) * Cin;
+      const float* wk = ws + (kh * 3 + kw) * Cin;
+      for (int ci = 0; ci < Cin; ++ci) {
+        const float x = Elem<TA>::load(src + ci);
+#pragma unroll
+        for (int co = 0; co < 16; ++co) acc[co] = fmaf(x, wk[co * KC + ci], acc[co]);
+      }
+    }
+  }
+  float* dst = y + ((int64_t)g * P + p) * Cout + co0;
+  for (int co = 0; co < nco; ++co) dst[co] = acc[co];
+}
+
+// Data gradient of conv_fwd: dx[g][b][ih][iw][ci] = sum over the taps that reach (ih, iw) of
+// sum_co dy[g][b][oh][ow][co] w[g][co][kh][kw][ci], plus (option-A shortcut) the block's
+// pre-activation gradient dout * (out > 0) at (ih / s, iw / s, ci) when ih, iw are multiples of s
+// and ci < the block's input channels.
+template <typename TA>
+__global__ void __launch_bounds__(64) conv_dgrad_kernel(
+    const TA* __restrict__ dy, const TA* __restrict__ w, int64_t w_gs, float* __restrict__ dx,
+    int B, int Hin, int Win, int Cin, int Hout, int Wout, int Cout, int stride,
+    const float* __restrict__ dout, const TA* __restrict__ out_act) {
+  extern __shared__ float ws[];  // [Cout][9][16]
+  const int g = blockIdx.z, ci0 = blockIdx.y * 16;
+  const int nci = min(16, Cin - ci0);
+  const TA* wg = w + (int64_t)g * w_gs;
+  for (int e = threadIdx.x; e < Cout * 9 * 16; e += blockDim.x) {
+    const int ci = e % 16, tap = (e / 16) % 9, co = e / 144;
+    ws[e] = ci < nci ? Elem<TA>::load(wg + ((int64_t)co * 9 + tap) * Cin + ci0 + ci) : 0.f;
+  }
+  __syncthreads();
+  const int64_t P = (int64_t)B * Hin * Win;
+  const int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (p >= P) return;
+  const int iw = (int)(p % Win);
+  const int ih = (int)((p / Win) % Hin);
+  const int b = (int)(p / ((int64_t)Win * Hin));
+  float acc[16];
+#pragma unroll
+  for (int i = 0; i < 16; ++i) acc[i] = 0.f;
+  const TA* dyg = dy + (int64_t)g * B * Hout * Wout * Cout;
+  for (int kh = 0; kh < 3; ++kh) {
+    const int on = ih + 1 - kh;
+    if (on < 0 || on % stride) continue;
+    const int oh = on / stride;
+    if (oh >= Hout) continue;
+    for (int kw = 0; kw < 3; ++kw) {
+      const int wn = iw + 1 - kw;
+      if (wn < 0 || wn % stride) continue;
+      const int ow = wn / stride;
+      if (ow >= Wout) continue;
+      const TA* src = dyg + (((int64_t)b * Hout + oh) * Wout + ow) * Cout;
+      const float* wk = ws + (kh * 3 + kw) * 16;
+      for (int co = 0; co < Cout; ++co) {
+        const float d = Elem<TA>::load(src + co);
+#pragma unroll
+        for (int ci = 0; ci < 16; ++ci) acc[ci] = fmaf(d, wk[co * 144 + ci], acc[ci]);
+      }
+    }
+  }
+  if (dout && ih % stride == 0 && iw % stride == 0) {
+    const int64_t e = ((((int64_t)g * B + b) * Hout + ih / stride) * Wout + iw / stride) * Cout;
+    for (int ci = 0; ci < nci; ++ci)
+      if (Elem<TA>::load(out_act + e + ci0 + ci) > 0.f) acc[ci] += dout[e + ci0 + ci];
+  }
+  float* dst = dx + ((int64_t)g * P + p) * Cin + ci0;
+  for (int ci = 0; ci < nci; ++ci) dst[ci] = acc[ci];
+}
+
+// Weight gradient, pass 1: part[g][q][co][j] = sum over the pixels of chunk q of
+// dy[p][co] * im2col(in)[p][j], j = (kh 3 + kw) Cin + ci.  Thread (co = t mod 16, j0 = t / 16)
+// owns j = j0 + 16 k; pixels are staged kWgradTile at a time in shared memory.
+template <typename TA>
+__global__ void __launch_bounds__(256) conv_wgrad_partial_kernel(
+    const TA* __restrict__ dy, const TA* __restrict__ in, float* __restrict__ part, int B, int Hin,
+    int Win, int Cin, int Hout, int Wout, int Cout, int stride, int nq) {
+  extern __shared__ float sm[];
+  const int J = 9 * Cin;
+  float* dys = sm;                     // [kWgradTile][16]
+  float* ims = sm + kWgradTile * 16;   // [kWgradTile][J]
+  const int g = blockIdx.z, co0 = blockIdx.y * 16, q = blockIdx.x;
+  const int co = threadIdx.x & 15, j0 = threadIdx.x >> 4;
+  const int64_t P = (int64_t)B * Hout * Wout;
+  const int64_t p0 = (int64_t)q * kWgradChunk, p1 = min(P, p0 + kWgradChunk);
+  const TA* dyg = dy + (int64_t)g * P * Cout;
+  const TA* ing = in + (int64_t)g * B * Hin * Win * Cin;
+  float acc[kMaxJ16];
+#pragma unroll
+  for (int k = 0; k < kMaxJ16; ++k) acc[k] = 0.f;
+  for (int64_t pb = p0; pb < p1; pb += kWgradTile) {
+    {
+      const int pp = threadIdx.x >> 4, c = threadIdx.x & 15;
+      const int64_t p = pb + pp;
+      dys[pp * 16 + c] = (p < p1 && co0 + c < Cout) ? Elem<TA>::load(dyg + p * Cout + co0 + c) : 0.f;
+    }
+    for (int e = threadIdx.x; e < kWgradTile * J; e += blockDim.x) {
+      const int pp = e / J, j = e % J;
+      const int64_t p = pb + pp;
+      float v = 0.f;
+      if (p < p1) {
+        const int tap = j / Cin, ci = j % Cin;
+        const int ow = (int)(p % Wout), oh = (int)((p / Wout) % Hout);
+        const int b = (int)(p / ((int64_t)Wout * Hout));
+        const int ih = oh * stride + tap / 3 - 1, iw = ow * stride + tap % 3 - 1;
+        if (ih >= 0 && ih < Hin && iw >= 0 && iw < Win)
+          v = Elem<TA>::load(ing + (((int64_t)b * Hin + ih) * Win + iw) * Cin + ci);
+      }
+      ims[e] = v;
+    }
+    __syncthreads();
+    for (int pp = 0; pp < kWgradTile; ++pp) {
+      const float d = dys[pp * 16 + co];
+      const float* row = ims + pp * J;
+#pragma unroll
+      for (int k = 0; k < kMaxJ16; ++k) {
+        const int j = j0 + 16 * k;
+        if (j < J) acc[k] = fmaf(d, row[j], acc[k]);
+      }
+    }
+    __syncthreads();
+  }
+  if (co0 + co < Cout) {
+    float* dst = part + (((int64_t)g * nq + q) * Cout + co0 + co) * J;
+#pragma unroll
+    for (int k = 0; k < kMaxJ16; ++k) {
+      const int j = j0 + 16 * k;
+      if (j < J) dst[j] = acc[k];
+    }
+  }
+}
+
+// Weight gradient, pass 2: G[g][w_off + e] = sum_q part[g][q][e] in chunk order.
+__global__ void sum_partials_kernel(const float* __restrict__ part, int nq, int64_t n, int G,
+                                    float* __restrict__ out, int64_t out_gs) {
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < (int64_t)G * n; t += stride) {
+    const int g = (int)(t / n);
+    const int64_t e = t % n;
+    const float* p = part + (int64_t)g * nq * n + e;
+    float s = 0.f;
+    for (int q = 0; q < nq; ++q) s += p[(int64_t)q * n];
+    out[(int64_t)g * out_gs + e] = s;
+  }
+}
+
+// BatchNorm statistics, pass 1: per chunk of pixels, the chunk mean and the sum of squared
+// deviations from it (two passes over the chunk), part[g][q][c] = (mean, M2).
+__global__ void __launch_bounds__(256) bn_stats_partial_kernel(const float* __restrict__ y,
+                                                               int64_t P, int C, int nq,
+                                                               float* __restrict__ part) {
+  __shared__ float red[256];
+  __shared__ float mean_s[256];
+  const int g = blockIdx.y, q = blockIdx.x;
+  const int lanes = blockDim.x / C;
+  const int c = threadIdx.x % C, l = threadIdx.x / C;
+  const int64_t p0 = (int64_t)q * kStatChunk, p1 = min(P, p0 + kStatChunk);
+  const float* yg = y + (int64_t)g * P * C;
+  float s = 0.f;
+  if (l < lanes)
+    for (int64_t p = p0 + l; p < p1; p += lanes) s += yg[p * C + c];
+  red[threadIdx.x] = s;
+  __syncthreads();
+  if (threadIdx.x < C) {
+    float t = 0.f;
+    for (int i = 0; i < lanes; ++i) t += red[i * C + threadIdx.x];
+    mean_s[threadIdx.x] = t / (float)(p1 - p0);
+  }
+  __syncthreads();
+  const float m = mean_s[c];
+  float s2 = 0.f;
+  if (l < lanes)
+    for (int64_t p = p0 + l; p < p1; p += lanes) {
+      const float dv = yg[p * C + c] - m;
+      s2 = fmaf(dv, dv, s2);
+    }
+  __syncthreads();
+  red[threadIdx.x] = s2;
+  __syncthreads();
+  if (threadIdx.x < C) {
+    float t = 0.f;
+    for (int i = 0; i < lanes; ++i) t += red[i * C + threadIdx.x];
+    float* dst = part + (((int64_t)g * nq + q) * C + threadIdx.x) * 2;
+    dst[0] = mean_s[threadIdx.x];
+    dst[1] = t;
+  }
+}
+
+// Pass 2: Chan et al.'s pairwise combination of the chunk (count, mean, M2) in chunk order (fp64),
+// biased variance, rstd = 1 / sqrt(var + eps).
+__global__ void bn_stats_finalize_kernel(const float* __restrict__ part, int64_t P, int C, int nq,
+                                         int G, float* __restrict__ mean, float* __restrict__ rstd) {
+  const int t = blockIdx.x * blockDim.x + threadIdx.x;
+  if (t >= G * C) return;
+  const int g = t / C, c = t % C;
+  double n = 0.0, mu = 0.0, M2 = 0.0;
+  for (int q = 0; q < nq; ++q) {
+    const double nb = (double)min((int64_t)kStatChunk, P - (int64_t)q * kStatChunk);
+    const float* pq = part + (((int64_t)g * nq + q) * C + c) * 2;
+    const double mb = pq[0], M2b = pq[1];
+    const double delta = mb - mu, nt = n + nb;
+    mu += delta * nb / nt;
+    M2 += M2b + delta * delta * n * nb / nt;
+    n = nt;
+  }
+  mean[t] = (float)mu;
+  rstd[t] = (float)(1.0 / sqrt(M2 / n + (double)kBnEps));
+}
+
+// out = relu(gamma (y - mean) rstd + beta [+ option-A shortcut of the block input]).
+template <typename TA>
+__global__ void bn_act_fwd_kernel(const float* __restrict__ y, const float* __restrict__ mean,
+                                  const float* __restrict__ rstd, const float* __restrict__ W,
+                                  int64_t g_off, int64_t b_off, int64_t d_gs, int w_g0, int w_gmul,
+                                  const TA* __restrict__ sc, int sc_H, int sc_W, int sc_C,
+                                  int stride, TA* __restrict__ out, int G, int B, int H, int Wd,
+                                  int C) {
+  const int64_t per = (int64_t)B * H * Wd * C;
+  const int64_t n = (int64_t)G * per;
+  const int64_t step = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < n; e += step) {
+    const int g = (int)(e / per);
+    const int c = (int)(e % C);
+    const float* Wg = W + (int64_t)(w_g0 + g * w_gmul) * d_gs;
+    float v = Wg[g_off + c] * ((y[e] - mean[g * C + c]) * rstd[g * C + c]) + Wg[b_off + c];
+    if (sc && c < sc_C) {
+      const int64_t pix = (e % per) / C;
+      const int x = (int)(pix % Wd), h = (int)((pix / Wd) % H), b = (int)(pix / ((int64_t)Wd * H));
+      v += Elem<TA>::load(sc + ((((int64_t)g * B + b) * sc_H + h * stride) * sc_W + x * stride) * sc_C + c);
+    }
+    Elem<TA>::store(out + e, fmaxf(v, 0.f));
+  }
+}
+
+// BatchNorm backward, pass 1: with dz = dout * (out > 0) and xhat = (y - mean) rstd, chunk sums
+// part[g][q][c] = (sum dz, sum dz xhat).
+template <typename TA>
+__global__ void __launch_bounds__(256) bn_bwd_partial_kernel(
+    const float* __restrict__ dout, const TA* __restrict__ out, const float* __restrict__ y,
+    const float* __restrict__ mean, const float* __restrict__ rstd, int64_t P, int C, int nq,
+    float* __restrict__ part) {
+  __shared__ float r1[256], r2[256];
+  const int g = blockIdx.y, q = blockIdx.x;
+  const int lanes = blockDim.x / C;
+  const int c = threadIdx.x % C, l = threadIdx.x / C;
+  const int64_t p0 = (int64_t)q * kStatChunk, p1 = min(P, p0 + kStatChunk);
+  const int64_t base = (int64_t)g * P * C;
+  const float mu = mean[g * C + c], rs = rstd[g * C + c];
+  float s1 = 0.f, s2 = 0.f;
+  if (l < lanes)
+    for (int64_t p = p0 + l; p < p1; p += lanes) {
+      const int64_t e = base + p * C + c;
+      const float dz = Elem<TA>::load(out + e) > 0.f ? dout[e] : 0.f;
+      s1 += dz;
+      s2 = fmaf(dz, (y[e] - mu) * rs, s2);
+    }
+  r1[threadIdx.x] = s1;
+  r2[threadIdx.x] = s2;
+  __syncthreads();
+  if (threadIdx.x < C) {
+    float t1 = 0.f, t2 = 0.f;
+    for (int i = 0; i < lanes; ++i) {
+      t1 += r1[i * C + threadIdx.x];
+      t2 += r2[i * C + threadIdx.x];
+    }
+    float* dst = part + (((int64_t)g * nq + q) * C + threadIdx.x) * 2;
+    dst[0] = t1;
+    dst[1] = t2;
+  }
+}
+
+// Pass 2: s[g][c] = chunk sums in order; dgamma = sum dz xhat, dbeta = sum dz into G.
+__global__ void bn_bwd_finalize_kernel(const float* __restrict__ part, int C, int nq, int G,
+                                       float* __restrict__ s12, float* __restrict__ Gr,
+                                       int64_t g_off, int64_t b_off, int64_t d_gs) {
+  const int t = blockIdx.x * blockDim.x + threadIdx.x;
+  if (t >= G * C) return;
+  const int g = t / C, c = t % C;
+  float a = 0.f, b = 0.f;
+  for (int q = 0; q < nq; ++q) {
+    const float* pq = part + (((int64_t)g * nq + q) * C + c) * 2;
+    a += pq[0];
+    b += pq[1];
+  }
+  s12[(int64_t)t * 2] = a;
+  s12[(int64_t)t * 2 + 1] = b;
+  Gr[(int64_t)g * d_gs + g_off + c] = b;
+  Gr[(int64_t)g * d_gs + b_off + c] = a;
+}
+
+// dy = gamma rstd (dz - mean(dz) - xhat mean(dz xhat)), the convolution's output gradient.
+template <typename TA>
+__global__ void bn_bwd_apply_kernel(const float* __restrict__ dout, const TA* __restrict__ out,
+                                    const float* __restrict__ y, const float* __restrict__ mean,
+                                    const float* __restrict__ rstd, const float* __restrict__ s12,
+                                    const float* __restrict__ W, int64_t g_off, int64_t d_gs,
+                                    TA* __restrict__ dy, int G, int64_t P, int C) {
+  const int64_t per = P * C, n = (int64_t)G * per;
+  const float invM = 1.0f / (float)P;
+  const int64_t step = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < n; e += step) {
+    const int g = (int)(e / per), c = (int)(e % C);
+    const int gc = g * C + c;
+    const float dz = Elem<TA>::load(out + e) > 0.f ? dout[e] : 0.f;
+    const float xh = (y[e] - mean[gc]) * rstd[gc];
+    const float v = W[(int64_t)g * d_gs + g_off + c] * rstd[gc] *
+                    (dz - s12[2 * gc] * invM - xh * (s12[2 * gc + 1] * invM));
+    Elem<TA>::store(dy + e, v);
+  }
+}
+
+// feat[g][b][f] = mean over the H W pixels of act[g][b][.][.][f].
+template <typename TA>
+__global__ void avgpool_kernel(const TA* __restrict__ act, float* __restrict__ feat, int GB, int HW,
+                               int F) {
+  const int t = blockIdx.x * blockDim.x + threadIdx.x;
+  if (t >= GB * F) return;
+  const int gb = t / F, f = t % F;
+  const TA* src = act + (int64_t)gb * HW * F + f;
+  float s = 0.f;
+  for (int p = 0; p < HW; ++p) s += Elem<TA>::load(src + (int64_t)p * F);
+  feat[t] = s / (float)HW;
+}
+
+// dact[g][b][p][f] = dfeat[g][b][f] / HW (gradient of the average pooling).
+__global__ void avgpool_bwd_kernel(const float* __restrict__ dfeat, float* __restrict__ dact,
+                                   int64_t n, int HW, int F) {
+  const int64_t step = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < n; e += step) {
+    const int f = (int)(e % F);
+    const int64_t gb = e / ((int64_t)HW * F);
+    dact[e] = dfeat[gb * F + f] / (float)HW;
+  }
+}
+
+}  // namespace
+
 struct ResNetPlan {
+  lsgd_config cfg{};
+  int K = 0, B = 0, C = 0, H0 = 0, W0 = 0, C0 = 0, base = 0, blocks = 0, F = 0;
+  bool bf16 = false;
+  std::vector<ConvL> convs;
+  int64_t fc_w = 0, fc_b = 0, c_fc_w = 0, c_fc_b = 0;
+  int64_t d = 0, d_pad = 0, decay_end = 0;
+  int64_t max_act = 0;  // largest activation tensor over all replicas (elements)
+  void* x0 = nullptr;
+  std::vector<void*> act;
+  std::vector<float*> y, mean, rstd;
+  float *feat = nullptr, *logits = nullptr, *dlogits = nullptr, *dfeat = nullptr;
+  float* dA[2] = {nullptr, nullptr};
+  float* dh = nullptr;
+  void* dy = nullptr;
+  float* part = nullptr;
+  size_t part_floats = 0;
+  float* s12 = nullptr;
   std::string err;
 };
 
-bool resnet_supported(const lsgd_config&, std::string* why) {
-  if (why) *why = "ResNet-20 is not available in this build";
-  return false;
+namespace {
+
+size_t esz(const ResNetPlan* p) { return p->bf16 ? 2 : 4; }
+
+lsgd_status rn_check(ResNetPlan* p, int64_t* launches, cudaError_t e, const char* what) {
+  if (launches) ++*launches;
+  if (e != cudaSuccess) {
+    p->err = std::string(what) + ": " + cudaGetErrorString(e);
+    return LSGD_ECUDA;
+  }
+  return LSGD_OK;
 }
-ResNetPlan* resnet_plan_create(const lsgd_config&) { return nullptr; }
+
+// A raw kernel launch (its error is the launch's last error) ...
+#define RN_LAUNCH(expr)                                                              \
+  do {                                                                               \
+    expr;                                                                            \
+    const lsgd_status st__ = rn_check(p, launches, cudaGetLastError(), #expr);       \
+    if (st__ != LSGD_OK) return st__;                                                \
+  } while (0)
+// ... or a launcher returning a cudaError_t (which also reports rejected arguments).
+#define RN_CALL(expr)                                                                \
+  do {                                                                               \
+    const lsgd_status st__ = rn_check(p, launches, (expr), #expr);                   \
+    if (st__ != LSGD_OK) return st__;                                                \
+  } while (0)
+
+int64_t conv_pixels(const ResNetPlan* p, const ConvL& c) { return (int64_t)p->B * c.hout * c.wout; }
+
+template <typename TA>
+lsgd_status conv_forward(ResNetPlan* p, const ConvL& c, const void* in, const void* Wop, int w_g0,
+                         int w_gmul, float* y, int G, cudaStream_t s, int64_t* launches) {
+  const int64_t P = conv_pixels(p, c);
+  dim3 grid((unsigned)((P + 127) / 128), (unsigned)((c.cout + 15) / 16), (unsigned)G);
+  const size_t smem = (size_t)16 * 9 * c.cin * 4;
+  const TA* wbase = reinterpret_cast<const TA*>(Wop) + (int64_t)w_g0 * p->d_pad + c.w_off;
+  RN_LAUNCH((conv_fwd_kernel<TA><<<grid, 128, smem, s>>>(
+      reinterpret_cast<const TA*>(in), wbase, (int64_t)w_gmul * p->d_pad, y, p->B, c.hin, c.win,
+      c.cin, c.hout, c.wout, c.cout, c.stride)));
+  return LSGD_OK;
+}
+
+lsgd_status bn_stats(ResNetPlan* p, const ConvL& c, const float* y, float* mean, float* rstd, int G,
+                     cudaStream_t s, int64_t* launches) {
+  const int64_t P = conv_pixels(p, c);
+  const int nq = (int)((P + kStatChunk - 1) / kStatChunk);
+  const int lanes = std::max(1, 256 / c.cout);
+  dim3 grid(nq, G);
+  RN_LAUNCH((bn_stats_partial_kernel<<<grid, lanes * c.cout, 0, s>>>(y, P, c.cout, nq, p->part)));
+  RN_LAUNCH((bn_stats_finalize_kernel<<<(G * c.cout + 127) / 128, 128, 0, s>>>(p->part, P, c.cout, nq,
+                                                                                G, mean, rstd)));
+  return LSGD_OK;
+}
+
+template <typename TA>
+lsgd_status forward_impl(ResNetPlan* p, const float* W, const void* Wop, int w_g0, int w_gmul,
+                         int G, cudaStream_t s, int64_t* launches) {
+  const size_t n_conv = p->convs.size();
+  for (size_t i = 0; i < n_conv; ++i) {
+    const ConvL& c = p->convs[i];
+    // block j uses convolutions 2j+1 (input act[2j], the block input) and 2j+2 (input act[2j+1])
+    const void* in = i == 0 ? p->x0 : p->act[i - 1];
+    lsgd_status st = conv_forward<TA>(p, c, in, Wop, w_g0, w_gmul, p->y[i], G, s, launches);
+    if (st != LSGD_OK) return st;
+    st = bn_stats(p, c, p->y[i], p->mean[i], p->rstd[i], G, s, launches);
+    if (st != LSGD_OK) return st;
+    const bool second = i > 0 && i % 2 == 0;
+    const TA* sc = second ? reinterpret_cast<const TA*>(p->act[i - 2]) : nullptr;
+    const ConvL& ca = p->convs[second ? i - 1 : i];
+    const int64_t n = (int64_t)G * conv_pixels(p, c) * c.cout;
+    RN_LAUNCH((bn_act_fwd_kernel<TA><<<grid_cap(n, 256), 256, 0, s>>>(
+        p->y[i], p->mean[i], p->rstd[i], W, c.g_off, c.b_off, p->d_pad, w_g0, w_gmul, sc, ca.hin,
+        ca.win, ca.cin, ca.stride, reinterpret_cast<TA*>(p->act[i]), G, p->B, c.hout, c.wout,
+        c.cout)));
+  }
+  // global average pooling and the classifier (fp32)
+  const ConvL& last = p->convs.back();
+  const int HW = last.hout * last.wout;
+  RN_LAUNCH((avgpool_kernel<TA><<<(G * p->B * p->F + 127) / 128, 128, 0, s>>>(
+      reinterpret_cast<const TA*>(p->act.back()), p->feat, G * p->B, HW, p->F)));
+  GemmArgs g{};
+  g.M = p->B;
+  g.N = p->C;
+  g.Kd = p->F;
+  g.G = G;
+  g.A = p->feat;
+  g.a_rs = p->F;
+  g.a_cs = 1;
+  g.a_gs = (int64_t)p->B * p->F;
+  g.B = W + (int64_t)w_g0 * p->d_pad + p->fc_w;
+  g.b_rs = 1;
+  g.b_cs = p->F;
+  g.b_gs = (int64_t)w_gmul * p->d_pad;
+  g.C = p->logits;
+  g.c_rs = p->C;
+  g.c_gs = (int64_t)p->B * p->C;
+  g.epi = EPI_BIAS;
+  g.bias = W + (int64_t)w_g0 * p->d_pad + p->fc_b;
+  g.bias_gs = (int64_t)w_gmul * p->d_pad;
+  RN_CALL(launch_gemm_simt(g, s));
+  return LSGD_OK;
+}
+
+template <typename TA>
+lsgd_status bn_backward(ResNetPlan* p, const ConvL& c, int i, const float* dout, const void* out,
+                        const float* W, float* Gr, cudaStream_t s, int64_t* launches) {
+  const int K = p->K;
+  const int64_t P = conv_pixels(p, c);
+  const int nq = (int)((P + kStatChunk - 1) / kStatChunk);
+  const int lanes = std::max(1, 256 / c.cout);
+  RN_LAUNCH((bn_bwd_partial_kernel<TA><<<dim3(nq, K), lanes * c.cout, 0, s>>>(
+      dout, reinterpret_cast<const TA*>(out), p->y[i], p->mean[i], p->rstd[i], P, c.cout, nq,
+      p->part)));
+  RN_LAUNCH((bn_bwd_finalize_kernel<<<(K * c.cout + 127) / 128, 128, 0, s>>>(
+      p->part, c.cout, nq, K, p->s12, Gr, c.g_off, c.b_off, p->d_pad)));
+  const int64_t n = (int64_t)K * P * c.cout;
+  RN_LAUNCH((bn_bwd_apply_kernel<TA><<<grid_cap(n, 256), 256, 0, s>>>(
+      dout, reinterpret_cast<const TA*>(out), p->y[i], p->mean[i], p->rstd[i], p->s12, W, c.g_off,
+      p->d_pad, reinterpret_cast<TA*>(p->dy), K, P, c.cout)));
+  return LSGD_OK;
+}
+
+template <typename TA>
+lsgd_status conv_wgrad(ResNetPlan* p, const ConvL& c, const void* in, float* Gr, cudaStream_t s,
+                       int64_t* launches) {
+  const int K = p->K;
+  const int64_t P = conv_pixels(p, c);
+  const int nq = (int)((P + kWgradChunk - 1) / kWgradChunk);
+  const int J = 9 * c.cin;
+  const size_t smem = (size_t)(kWgradTile * 16 + kWgradTile * J) * 4;
+  RN_LAUNCH((conv_wgrad_partial_kernel<TA><<<dim3(nq, (c.cout + 15) / 16, K), 256, smem, s>>>(
+      reinterpret_cast<const TA*>(p->dy), reinterpret_cast<const TA*>(in), p->part, p->B, c.hin,
+      c.win, c.cin, c.hout, c.wout, c.cout, c.stride, nq)));
+  const int64_t n = (int64_t)c.cout * J;
+  RN_LAUNCH((sum_partials_kernel<<<grid_cap((int64_t)K * n, 256), 256, 0, s>>>(
+      p->part, nq, n, K, Gr + c.w_off, p->d_pad)));
+  return LSGD_OK;
+}
+
+template <typename TA>
+lsgd_status conv_dgrad(ResNetPlan* p, const ConvL& c, const void* Wop, float* dx, const float* dout,
+                       const void* out_act, cudaStream_t s, int64_t* launches) {
+  const int K = p->K;
+  const int64_t P = (int64_t)p->B * c.hin * c.win;
+  dim3 grid((unsigned)((P + 63) / 64), (unsigned)((c.cin + 15) / 16), (unsigned)K);
+  const size_t smem = (size_t)c.cout * 9 * 16 * 4;
+  RN_LAUNCH((conv_dgrad_kernel<TA><<<grid, 64, smem, s>>>(
+      reinterpret_cast<const TA*>(p->dy), reinterpret_cast<const TA*>(Wop) + c.w_off, p->d_pad, dx,
+      p->B, c.hin, c.win, c.cin, c.hout, c.wout, c.cout, c.stride, dout,
+      reinterpret_cast<const TA*>(out_act))));
+  return LSGD_OK;
+}
+
+template <typename TA>
+lsgd_status fwd_bwd_impl(ResNetPlan* p, const float* W, const void* Wop, float* Gr,
+                         const int32_t* labels, float* loss_mean, cudaStream_t s, int64_t* launches) {
+  const int K = p->K, B = p->B;
+  lsgd_status st = forward_impl<TA>(p, W, Wop, 0, 1, K, s, launches);
+  if (st != LSGD_OK) return st;
+  RN_CALL(launch_softmax_xent(p->logits, p->C, p->C, labels, K, B, p->dlogits, false, p->C,
+                              loss_mean, nullptr, nullptr, s));
+  // classifier gradients: G_W = dlogits^T feat, G_b = sum dlogits, dfeat = dlogits W
+  {
+    GemmArgs g{};
+    g.M = p->C;
+    g.N = p->F;
+    g.Kd = B;
+    g.G = K;
+    g.A = p->dlogits;
+    g.a_rs = 1;
+    g.a_cs = p->C;
+    g.a_gs = (int64_t)B * p->C;
+    g.B = p->feat;
+    g.b_rs = p->F;
+    g.b_cs = 1;
+    g.b_gs = (int64_t)B * p->F;
+    g.C = Gr + p->fc_w;
+    g.c_rs = p->F;
+    g.c_gs = p->d_pad;
+    g.epi = EPI_STORE;
+    RN_CALL(launch_gemm_simt(g, s));
+    RN_CALL(launch_colsum(p->dlogits, false, p->C, K, B, p->C, Gr + p->fc_b, p->d_pad, s));
+    GemmArgs h{};
+    h.M = B;
+    h.N = p->F;
+    h.Kd = p->C;
+    h.G = K;
+    h.A = p->dlogits;
+    h.a_rs = p->C;
+    h.a_cs = 1;
+    h.a_gs = (int64_t)B * p->C;
+    h.B = W + p->fc_w;
+    h.b_rs = p->F;
+    h.b_cs = 1;
+    h.b_gs = p->d_pad;
+    h.C = p->dfeat;
+    h.c_rs = p->F;
+    h.c_gs = (int64_t)B * p->F;
+    h.epi = EPI_STORE;
+    RN_CALL(launch_gemm_simt(h, s));
+  }
+  const ConvL& last = p->convs.back();
+  const int HW = last.hout * last.wout;
+  int cur = 0;
+  {
+    const int64_t n = (int64_t)K * B * HW * p->F;
+    RN_LAUNCH((avgpool_bwd_kernel<<<grid_cap(n, 256), 256, 0, s>>>(p->dfeat, p->dA[cur], n, HW,
+                                                                     p->F)));
+  }
+  const int n_blocks = (int)(p->convs.size() - 1) / 2;
+  for (int j = n_blocks - 1; j >= 0; --j) {
+    const int ia = 2 * j + 1, ib = 2 * j + 2;
+    const ConvL& ca = p->convs[ia];
+    const ConvL& cb = p->convs[ib];
+    const void* blk_in = p->act[2 * j];
+    // second convolution: BN backward through the block's output ReLU, then its products
+    st = bn_backward<TA>(p, cb, ib, p->dA[cur], p->act[ib], W, Gr, s, launches);
+    if (st != LSGD_OK) return st;
+    st = conv_wgrad<TA>(p, cb, p->act[ia], Gr, s, launches);
+    if (st != LSGD_OK) return st;
+    st = conv_dgrad<TA>(p, cb, Wop, p->dh, nullptr, nullptr, s, launches);
+    if (st != LSGD_OK) return st;
+    // first convolution: BN backward through the inner ReLU, then its products; the data
+    // gradient also receives the shortcut's share of the block's output gradient
+    st = bn_backward<TA>(p, ca, ia, p->dh, p->act[ia], W, Gr, s, launches);
+    if (st != LSGD_OK) return st;
+    st = conv_wgrad<TA>(p, ca, blk_in, Gr, s, launches);
+    if (st != LSGD_OK) return st;
+    st = conv_dgrad<TA>(p, ca, Wop, p->dA[1 - cur], p->dA[cur], p->act[ib], s, launches);
+    if (st != LSGD_OK) return st;
+    cur = 1 - cur;
+  }
+  // stem: BN backward and the weight gradient (no data gradient for the image)
+  const ConvL& c0 = p->convs[0];
+  st = bn_backward<TA>(p, c0, 0, p->dA[cur], p->act[0], W, Gr, s, launches);
+  if (st != LSGD_OK) return st;
+  return conv_wgrad<TA>(p, c0, p->x0, Gr, s, launches);
+}
+
+}  // namespace
+
+bool resnet_supported(const lsgd_config& cfg, std::string* why) {
+  const lsgd_model& m = cfg.model;
+  if (m.in_h < 1 || m.in_w < 1 || m.in_c < 1 || m.n_classes < 1 || m.base_ch < 1 || m.res_blocks < 1) {
+    if (why) *why = "ResNet geometry must be positive";
+    return false;
+  }
+  if (m.base_ch * 4 > 64 || m.in_c > 64) {
+    if (why) *why = "ResNet channels above 64 are not supported";
+    return false;
+  }
+  if (cfg.B_loc > 8192 || (int64_t)cfg.B_loc * m.in_h * m.in_w > (1LL << 30)) {
+    if (why) *why = "ResNet batch too large";
+    return false;
+  }
+  return true;
+}
+
+ResNetPlan* resnet_plan_create(const lsgd_config& cfg) {
+  ResNetPlan* p = new ResNetPlan();
+  p->cfg = cfg;
+  p->K = cfg.K;
+  p->B = cfg.B_loc;
+  const lsgd_model& m = cfg.model;
+  p->H0 = m.in_h;
+  p->W0 = m.in_w;
+  p->C0 = m.in_c;
+  p->C = m.n_classes;
+  p->base = m.base_ch;
+  p->blocks = m.res_blocks;
+  p->bf16 = cfg.precision == LSGD_BF16;
+  // layout: canonical order (stem, block convs, fc W, fc b; each conv followed by its BN gamma,
+  // beta); padded order puts every BatchNorm parameter after the decayed ones.
+  int64_t canon = 0, off = 0;
+  int h = p->H0, w = p->W0, ch = p->C0;
+  auto add = [&](int cin, int cout, int stride) {
+    ConvL c{};
+    c.cin = cin;
+    c.cout = cout;
+    c.stride = stride;
+    c.hin = h;
+    c.win = w;
+    c.hout = (h - 1) / stride + 1;
+    c.wout = (w - 1) / stride + 1;
+    c.cw = canon;
+    canon += (int64_t)cout * 9 * cin;
+    c.cg = canon;
+    canon += cout;
+    c.cb = canon;
+    canon += cout;
+    c.w_off = off;
+    off = rup(off + (int64_t)cout * 9 * cin, 64);
+    h = c.hout;
+    w = c.wout;
+    p->convs.push_back(c);
+  };
+  add(ch, p->base, 1);
+  ch = p->base;
+  for (int st = 0; st < 3; ++st) {
+    const int cout = p->base << st;
+    for (int b = 0; b < p->blocks; ++b) {
+      add(ch, cout, (st > 0 && b == 0) ? 2 : 1);
+      add(cout, cout, 1);
+      ch = cout;
+    }
+  }
+  p->F = ch;
+  p->c_fc_w = canon;
+  canon += (int64_t)p->C * p->F;
+  p->c_fc_b = canon;
+  canon += p->C;
+  p->fc_w = off;
+  off = rup(off + (int64_t)p->C * p->F, 64);
+  p->fc_b = off;
+  off = rup(off + p->C, 64);
+  p->decay_end = off;
+  for (ConvL& c : p->convs) {
+    c.g_off = off;
+    off = rup(off + c.cout, 64);
+    c.b_off = off;
+    off = rup(off + c.cout, 64);
+  }
+  p->d = canon;
+  p->d_pad = rup(off, 64);
+  int64_t mx = (int64_t)p->B * p->H0 * p->W0 * p->C0;
+  for (const ConvL& c : p->convs) mx = std::max(mx, (int64_t)p->B * c.hout * c.wout * c.cout);
+  p->max_act = mx * p->K;
+  return p;
+}
+
 void resnet_destroy(ResNetPlan* p) { delete p; }
-int64_t resnet_num_params(const ResNetPlan*) { return 0; }
-int64_t resnet_d_pad(const ResNetPlan*) { return 0; }
-void resnet_segments(const ResNetPlan*, const std::function<void(int64_t, int64_t, int64_t)>&) {}
-void resnet_decay_region(const ResNetPlan*, int64_t* period, int64_t* decay_end) {
-  *period = 0;
-  *decay_end = 0;
+int64_t resnet_num_params(const ResNetPlan* p) { return p->d; }
+int64_t resnet_d_pad(const ResNetPlan* p) { return p->d_pad; }
+
+void resnet_segments(const ResNetPlan* p, const std::function<void(int64_t, int64_t, int64_t)>& f) {
+  for (const ConvL& c : p->convs) {
+    f(c.cw, c.w_off, (int64_t)c.cout * 9 * c.cin);
+    f(c.cg, c.g_off, c.cout);
+    f(c.cb, c.b_off, c.cout);
+  }
+  f(p->c_fc_w, p->fc_w, (int64_t)p->C * p->F);
+  f(p->c_fc_b, p->fc_b, p->C);
 }
-lsgd_status resnet_alloc(ResNetPlan*, const std::function<void*(size_t)>&) { return LSGD_EUNSUPPORTED; }
-lsgd_status resnet_init_params(ResNetPlan*, float*, uint64_t, cudaStream_t, int64_t*) {
-  return LSGD_EUNSUPPORTED;
+
+void resnet_decay_region(const ResNetPlan* p, int64_t* period, int64_t* decay_end) {
+  *period = p->d_pad;
+  *decay_end = p->decay_end;
 }
-lsgd_status resnet_forward_backward(ResNetPlan*, const float*, const uint16_t*, float*, int64_t,
-                                    const int32_t*, float*, cudaStream_t, int64_t*) {
-  return LSGD_EUNSUPPORTED;
+
+lsgd_status resnet_alloc(ResNetPlan* p, const std::function<void*(size_t)>& alloc) {
+  const int K = p->K, B = p->B;
+  const size_t e = esz(p);
+  p->x0 = alloc((size_t)K * B * p->H0 * p->W0 * p->C0 * e);
+  size_t part = 0;
+  for (const ConvL& c : p->convs) {
+    const int64_t n = (int64_t)K * B * c.hout * c.wout * c.cout;
+    p->y.push_back((float*)alloc((size_t)n * 4));
+    p->act.push_back(alloc((size_t)n * e));
+    p->mean.push_back((float*)alloc((size_t)K * c.cout * 4));
+    p->rstd.push_back((float*)alloc((size_t)K * c.cout * 4));
+    const int64_t P = (int64_t)B * c.hout * c.wout;
+    const int64_t nq_s = (P + kStatChunk - 1) / kStatChunk;
+    const int64_t nq_w = (P + kWgradChunk - 1) / kWgradChunk;
+    part = std::max(part, (size_t)(K * nq_s * c.cout * 2));
+    part = std::max(part, (size_t)(K * nq_w * c.cout * 9 * c.cin));
+  }
+  p->part_floats = part;
+  p->part = (float*)alloc(part * 4);
+  p->feat = (float*)alloc((size_t)K * B * p->F * 4);
+  p->dfeat = (float*)alloc((size_t)K * B * p->F * 4);
+  p->logits = (float*)alloc((size_t)K * B * p->C * 4);
+  p->dlogits = (float*)alloc((size_t)K * B * p->C * 4);
+  p->dA[0] = (float*)alloc((size_t)p->max_act * 4);
+  p->dA[1] = (float*)alloc((size_t)p->max_act * 4);
+  p->dh = (float*)alloc((size_t)p->max_act * 4);
+  p->dy = alloc((size_t)p->max_act * e);
+  p->s12 = (float*)alloc((size_t)K * 2 * 64 * 4);
+  if (!p->x0 || !p->part || !p->feat || !p->dfeat || !p->logits || !p->dlogits || !p->dA[0] ||
+      !p->dA[1] || !p->dh || !p->dy || !p->s12)
+    return LSGD_ENOMEM;
+  for (size_t i = 0; i < p->convs.size(); ++i)
+    if (!p->y[i] || !p->act[i] || !p->mean[i] || !p->rstd[i]) return LSGD_ENOMEM;
+  return LSGD_OK;
 }
-lsgd_status resnet_eval(ResNetPlan*, const float*, const uint16_t*, int64_t, int, int, const int32_t*,
-                        float*, cudaStream_t, int64_t*) {
-  return LSGD_EUNSUPPORTED;
+
+// He initialisation of the convolutions (fan-in 9 Cin), N(0, 0.01^2) for the classifier, zero
+// biases, BN gamma = 1 and beta = 0 (Sec. A.2); replica 0, broadcast by the caller.
+lsgd_status resnet_init_params(ResNetPlan* p, float* W, uint64_t seed, cudaStream_t s,
+                               int64_t* launches) {
+  if (p->cfg.model.init != LSGD_INIT_HE) return LSGD_OK;  // all zeros
+  uint32_t tensor = 0;
+  for (const ConvL& c : p->convs) {
+    RN_CALL(launch_init_normal(W + c.w_off, (int64_t)c.cout * 9 * c.cin, std::sqrt(2.0 / (9.0 * c.cin)),
+                               seed, tensor, s));
+    ++tensor;
+    RN_CALL(launch_fill(W + c.g_off, c.cout, 1.0f, s));
+  }
+  RN_CALL(launch_init_normal(W + p->fc_w, (int64_t)p->C * p->F, 0.01, seed, tensor, s));
+  return LSGD_OK;
 }
-void* resnet_input(ResNetPlan*) { return nullptr; }
+
+lsgd_status resnet_forward_backward(ResNetPlan* p, const float* W, const uint16_t* Wb, float* G,
+                                    int64_t d_pad, const int32_t* labels, float* loss_mean,
+                                    cudaStream_t s, int64_t* launches) {
+  (void)d_pad;
+  if (p->bf16) return fwd_bwd_impl<uint16_t>(p, W, Wb, G, labels, loss_mean, s, launches);
+  return fwd_bwd_impl<float>(p, W, W, G, labels, loss_mean, s, launches);
+}
+
+lsgd_status resnet_eval(ResNetPlan* p, const float* W, const uint16_t* Wb, int64_t d_pad, int k,
+                        int groups, const int32_t* labels, float* row_loss, cudaStream_t s,
+                        int64_t* launches) {
+  (void)d_pad;
+  lsgd_status st = p->bf16 ? forward_impl<uint16_t>(p, W, Wb, k, 0, groups, s, launches)
+                           : forward_impl<float>(p, W, W, k, 0, groups, s, launches);
+  if (st != LSGD_OK) return st;
+  RN_CALL(launch_softmax_xent(p->logits, p->C, p->C, labels, groups, p->B, nullptr, false, p->C,
+                              nullptr, nullptr, row_loss, s));
+  return LSGD_OK;
+}
+
+void* resnet_input(ResNetPlan* p) { return p->x0; }
 const char* resnet_last_error(const ResNetPlan* p) { return p ? p->err.c_str() : ""; }
 
 }  // namespace lsgd

@@ -1,0 +1,146 @@
+"""ResNet-20 on the GPU against the oracle: per-step fp32 parity on a reduced network, multi-step
+bf16 parity on the full ResNet-20 topology, and the full post-local ResNet-20 run size (K = 16,
+B = 128, N = 50,000) checked on a sampled replica."""
+import numpy as np
+import pytest
+
+import oracle
+import synthdata
+from _gpu_common import built_package, rel_l2
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def P():
+    import torch
+
+    assert torch.cuda.is_available()
+    return built_package()
+
+
+def resnet_cfgs(P, *, hwc, base, blocks, classes, K, B, H, T, N, precision, t_switch=-1,
+                base_lr=0.1, scale_by_K=False, warmup_epochs=0.0, milestones=(), momentum=0.0,
+                nesterov=False, weight_decay=0.0, seed=0):
+    g = P.make_config(K=K, B_loc=B, H=H, t_switch=t_switch, total_steps=T, N=N, kind=P.RESNET20,
+                      in_hwc=hwc, n_classes=classes, base_ch=base, res_blocks=blocks,
+                      base_lr=base_lr, scale_by_K=scale_by_K, warmup_epochs=warmup_epochs,
+                      milestones=milestones, momentum=momentum, nesterov=nesterov,
+                      weight_decay=weight_decay, seed=seed, precision=precision)
+    o = oracle.make_cfg(kind=oracle.RESNET20, in_hwc=hwc, n_classes=classes, base_ch=base,
+                        res_blocks=blocks, bf16=(precision == P.BF16), K=K, B=B, H=H,
+                        t_switch=t_switch, T=T, N=N, base_lr=base_lr, scale_by_K=scale_by_K,
+                        warmup_epochs=warmup_epochs, milestones=milestones, momentum=momentum,
+                        nesterov=nesterov, weight_decay=weight_decay, seed=seed)
+    return g, o
+
+
+def test_resnet20_size_and_init(P):
+    g, o = resnet_cfgs(P, hwc=(32, 32, 3), base=16, blocks=3, classes=10, K=2, B=4, H=1, T=2,
+                       N=64, precision=P.BF16, seed=7)
+    ctx = P.lsgd_create(g)
+    assert P.lsgd_num_params(ctx) == 269722
+    w = P.lsgd_params(ctx, 1)
+    want = oracle.init_params(o)
+    assert np.abs(w - want).max() <= 1e-6 * np.abs(want).max()
+    P.lsgd_destroy(ctx)
+
+
+@pytest.mark.parametrize("K,B,H,blocks", [(3, 6, 2, 1), (2, 5, 1, 2)])
+def test_reduced_resnet_fp32_stepwise(P, K, B, H, blocks):
+    hwc, base, C = (8, 8, 3), 4, 5
+    N = 60
+    rng = np.random.default_rng(K + B)
+    X = rng.standard_normal((N, 8 * 8 * 3)).astype(np.float32)
+    y = rng.integers(0, C, N).astype(np.int32)
+    g, o = resnet_cfgs(P, hwc=hwc, base=base, blocks=blocks, classes=C, K=K, B=B, H=H, T=6, N=N,
+                       precision=P.FP32, base_lr=0.05, momentum=0.9, nesterov=True,
+                       weight_decay=1e-3, seed=2)
+    ctx = P.lsgd_create(g)
+    P.lsgd_set_dataset(ctx, X, y)
+    Wo = np.tile(oracle.init_params(o), (K, 1))
+    Uo = np.zeros_like(Wo)
+    worst = 0.0
+    for s in range(6):
+        Wf, Uf = Wo.astype(np.float32), Uo.astype(np.float32)
+        for k in range(K):
+            P.lsgd_set_params(ctx, k, Wf[k])
+            P.lsgd_set_momentum(ctx, k, Uf[k])
+        P.lsgd_run(ctx, 1)
+        Wo, Uo, lo, _ = oracle.run(o, X, y=y, W=Wf.astype(np.float64), U=Uf.astype(np.float64),
+                                   s0=s, n_steps=1)
+        for k in range(K):
+            got = P.lsgd_params(ctx, k).astype(np.float64)
+            worst = max(worst, np.abs(got - Wo[k]).max() / np.abs(Wo[k]).max())
+        np.testing.assert_allclose(P.lsgd_losses(ctx, 1, K)[0], lo[0], rtol=1e-4, atol=1e-5)
+    P.lsgd_destroy(ctx)
+    assert worst <= 1e-5, worst
+
+
+def test_resnet20_bf16_multistep(P):
+    # A stable regime (lr 0.02, B = 16): there the oracle's own bf16 and fp32 runs differ by ~3 %
+    # over four steps.  (With lr 0.2 and B = 8 the run diverges within four steps and even the
+    # oracle's bf16 and fp32 trajectories differ by ~70 %.)
+    N, K, B = 64, 2, 16
+    X, y = synthdata.gaussian_mixture(N, 3072, 10, seed=3)
+    g, o = resnet_cfgs(P, hwc=(32, 32, 3), base=16, blocks=3, classes=10, K=K, B=B, H=2, T=4, N=N,
+                       precision=P.BF16, base_lr=0.02, momentum=0.9, nesterov=True,
+                       weight_decay=1e-4, seed=4)
+    w0 = oracle.init_params(o)
+    ctx = P.lsgd_create(g)
+    P.lsgd_set_dataset(ctx, X, y)
+    P.lsgd_set_params(ctx, -1, w0.astype(np.float32))
+    P.lsgd_run(ctx, 4)
+    w0 = w0.astype(np.float32).astype(np.float64)
+    W, _, lo, syncs = oracle.run(o, X, y=y, W=np.tile(w0, (K, 1)), n_steps=4)
+    got = P.lsgd_params(ctx, -1).astype(np.float64)
+    # the bar of the bf16 mode: parameters within 2e-2 relative L2 of the oracle's
+    assert rel_l2(got, W[0]) <= 2e-2
+    # and the GPU's departure from the oracle's bf16 trajectory stays below the effect of bf16
+    # quantization itself (the oracle's bf16 vs fp32 runs): 19 layers of bf16 re-rounding
+    # amplify summation-order differences, so the update agrees to a few percent.
+    _, o32 = resnet_cfgs(P, hwc=(32, 32, 3), base=16, blocks=3, classes=10, K=K, B=B, H=2, T=4,
+                         N=N, precision=P.FP32, base_lr=0.02, momentum=0.9, nesterov=True,
+                         weight_decay=1e-4, seed=4)
+    W32, _, _, _ = oracle.run(o32, X, y=y, W=np.tile(w0, (K, 1)), n_steps=4)
+    d_gpu = rel_l2(got - w0, W[0] - w0)
+    d_q = rel_l2(W32[0] - w0, W[0] - w0)
+    print(f"ResNet-20 bf16, 4 steps: update vs oracle {d_gpu:.3e}, oracle bf16 vs fp32 {d_q:.3e}")
+    assert d_gpu <= d_q
+    assert np.abs(P.lsgd_losses(ctx, 4, K) - lo).max() <= 1e-2
+    assert P.lsgd_sync_count(ctx) == syncs == 2
+    # evaluation loss of the averaged model on the first 16 rows (BatchNorm statistics of each
+    # group of B rows, as in training)
+    l_gpu = P.lsgd_eval_loss(ctx, -1, 16)
+    l_orc = np.mean([oracle.loss_grad(o, W[0], X, y=y, idx=np.arange(i, i + B))[0]
+                     for i in range(0, 16, B)])
+    assert abs(l_gpu - l_orc) <= 1e-2
+    P.lsgd_destroy(ctx)
+
+
+def test_resnet20_full_size_sampled_replica(P):
+    # Post-local ResNet-20: K = 16, B = 128, N = 50,000, one epoch, t' = floor(0.5 T), H = 16,
+    # Nesterov 0.9, weight decay 1e-4 (not on BatchNorm), lr 0.2 scaled by K with warm-up.
+    N, K, B = 50000, 16, 128
+    T = -(-N // (K * B))
+    X, y = synthdata.gaussian_mixture_cached(N, 3072, 10, 1234)
+    g, o = resnet_cfgs(P, hwc=(32, 32, 3), base=16, blocks=3, classes=10, K=K, B=B, H=16, T=T,
+                       N=N, precision=P.BF16, t_switch=T // 2, base_lr=0.2, scale_by_K=True,
+                       warmup_epochs=5, milestones=(0.5, 0.75), momentum=0.9, nesterov=True,
+                       weight_decay=1e-4, seed=1)
+    w0 = oracle.init_params(o)
+    ctx = P.lsgd_create(g)
+    P.lsgd_set_dataset(ctx, X, y)
+    P.lsgd_set_params(ctx, -1, w0.astype(np.float32))
+    w0 = w0.astype(np.float32).astype(np.float64)
+    P.lsgd_run(ctx, 1)
+    k = 5
+    loss, grad = oracle.loss_grad(o, w0, X, y=y, idx=oracle.sample_indices(o, k, 0))
+    gp = grad + 1e-4 * w0 * oracle.weight_decay_mask(o)
+    # step 0 is in the mini-batch phase, so the parameters are averaged; the momentum is local
+    assert rel_l2(P.lsgd_momentum(ctx, k).astype(np.float64), gp) <= 2e-2
+    assert abs(P.lsgd_losses(ctx, 1, K)[0][k] - loss) <= 1e-2
+    P.lsgd_run(ctx, T - 1)
+    assert P.lsgd_sync_count(ctx) == T // 2 + -(-(T - T // 2) // 16)
+    assert P.lsgd_check_finite(ctx)
+    P.lsgd_destroy(ctx)

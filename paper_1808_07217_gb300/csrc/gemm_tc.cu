@@ -173,8 +173,14 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
   Smem<BN, STAGES>& sm = *reinterpret_cast<Smem<BN, STAGES>*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int n0 = blockIdx.x * BN, m0 = blockIdx.y * BM, g = blockIdx.z;
-  const int nk = (args.Kd + BK - 1) / BK;
+  const int splits = args.splits > 1 ? args.splits : 1;
+  const int n0 = blockIdx.x * BN, m0 = blockIdx.y * BM, g = blockIdx.z / splits;
+  const int split = blockIdx.z % splits;
+  const int nk_all = (args.Kd + BK - 1) / BK;
+  const int per_split = (nk_all + splits - 1) / splits;
+  const int kb_first = split * per_split;
+  const int nk = min(nk_all - kb_first, per_split);  // >= 1 (the host makes every split nonempty)
+  const int64_t c_base = (int64_t)g * args.c_gs + (int64_t)split * args.c_split_stride;
   const bool a_mn = args.A.mn_major, b_mn = args.B.mn_major;
   constexpr uint32_t kBytesA = BM * BK * 2, kBytesB = BN * BK * 2;
 
@@ -219,7 +225,7 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
         break;
       }
       mbar_expect_tx(&sm.full[s], kBytesA + kBytesB);
-      const int k0 = kb * BK;
+      const int k0 = (kb_first + kb) * BK;
       if (!a_mn) {
         tma_load_3d(sm.a[s], &args.A.map, &sm.full[s], k0, m0, g);
       } else {
@@ -317,7 +323,7 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
           const int m = m0 + row, n = n0 + cc + grp * 4;
           ok[q] = it < ITEMS && m < args.M && n < args.N;
           nn[q] = n;
-          off[q] = (int64_t)g * args.c_gs + (int64_t)m * args.c_rs + n;
+          off[q] = c_base + (int64_t)m * args.c_rs + n;
           a0[q] = make_float4(0.f, 0.f, 0.f, 0.f);
           a1[q] = a0[q];
           if (!ok[q]) continue;
@@ -525,6 +531,14 @@ bool make_tma_map_bf16(CUtensorMap* map, const void* base, uint64_t dim0, uint64
 
 int tc_tile_n(int Kd) { return (Kd + BK - 1) / BK <= 2 ? 128 : 64; }
 
+int tc_valid_splits(int Kd, int want) {
+  const int nk_all = (Kd + BK - 1) / BK;
+  if (want < 1) want = 1;
+  if (want > nk_all) want = nk_all;
+  const int per = (nk_all + want - 1) / want;
+  return (nk_all + per - 1) / per;  // every split gets at least one k-block
+}
+
 cudaError_t launch_gemm_tc(const TcGemmArgs& a, cudaStream_t stream) {
   if (a.M <= 0 || a.N <= 0 || a.G <= 0) return cudaSuccess;
   if (a.Kd <= 0 || a.G > 65535) return cudaErrorInvalidValue;
@@ -537,8 +551,14 @@ cudaError_t launch_gemm_tc(const TcGemmArgs& a, cudaStream_t stream) {
   if (a.epi == EPI_MASK && !a.mask) return cudaErrorInvalidValue;
   if (a.epi == EPI_SGD && (!a.sgd.w || (a.sgd.mom != 0.f && !a.sgd.u))) return cudaErrorInvalidValue;
   if (a.epi != EPI_SGD && !a.C) return cudaErrorInvalidValue;
+  const int splits = a.splits > 1 ? a.splits : 1;
+  if (splits > 1) {
+    const int nk_all = (a.Kd + BK - 1) / BK, per = (nk_all + splits - 1) / splits;
+    if (a.epi != EPI_STORE || (int64_t)(splits - 1) * per >= nk_all) return cudaErrorInvalidValue;
+    if ((int64_t)a.G * splits > 65535) return cudaErrorInvalidValue;
+  }
   constexpr int BN = 128;
-  dim3 grid((a.N + BN - 1) / BN, (a.M + BM - 1) / BM, a.G);
+  dim3 grid((a.N + BN - 1) / BN, (a.M + BM - 1) / BM, a.G * splits);
   if (grid.y > 65535) return cudaErrorInvalidValue;
   static_assert(BM == kTcTileM, "tile height");
   // Short reductions (the weight gradient's k = B_loc) need only two stages; the smaller shared
@@ -547,7 +567,7 @@ cudaError_t launch_gemm_tc(const TcGemmArgs& a, cudaStream_t stream) {
   // Long reductions (forward, data gradient): 64-wide N tiles with four stages (96 KB) so two
   // CTAs share an SM and twice as many tiles stream weights at once.
   constexpr int BN2 = 64;
-  dim3 grid2((a.N + BN2 - 1) / BN2, (a.M + BM - 1) / BM, a.G);
+  dim3 grid2((a.N + BN2 - 1) / BN2, (a.M + BM - 1) / BM, a.G * splits);
   return launch_cfg<BN2, 4>(a, grid2, stream);
 }
 

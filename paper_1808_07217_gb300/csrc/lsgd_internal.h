@@ -100,6 +100,10 @@ struct TcGemmArgs {
   // tile's parameters and momentum into L2 while the products run (have_wu_maps = 0: no prefetch)
   CUtensorMap wmap, umap;
   int have_wu_maps;
+  // split-K: the reduction is cut into `splits` contiguous ranges of k-blocks, split s writing its
+  // partial product at C + g c_gs + s c_split_stride (EPI_STORE only); 0 or 1 = no split
+  int splits;
+  int64_t c_split_stride;
   // epilogue (same semantics as GemmArgs), C(m, n) at C + g c_gs + m c_rs + n
   void* C;
   int64_t c_rs, c_gs;
@@ -122,6 +126,8 @@ cudaError_t launch_gemm_tc(const TcGemmArgs& a, cudaStream_t stream);
 // N-tile width the tcgen05 kernel uses for a reduction of length Kd (the row count a K-major B
 // operand's TMA box must have).
 int tc_tile_n(int Kd);
+// The largest split count <= want for which every split of a Kd-long reduction is nonempty.
+int tc_valid_splits(int Kd, int want);
 constexpr int kTcTileM = 128;
 bool tc_available();
 // 1 if a bounded wait inside a tcgen05 kernel ran out since the last call (then cleared).

@@ -14,6 +14,7 @@
 // then a fixed-order combination.
 #include <algorithm>
 #include <cmath>
+#include <cstdlib>
 #include <string>
 #include <vector>
 
@@ -267,28 +268,82 @@ __global__ void __launch_bounds__(256) bn_stats_partial_kernel(const float* __re
   }
 }
 
-// Pass 2: Chan et al.'s pairwise combination of the chunk (count, mean, M2) in chunk order (fp64),
-// biased variance, rstd = 1 / sqrt(var + eps).
-__global__ void bn_stats_finalize_kernel(const float* __restrict__ part, int64_t P, int C, int nq,
-                                         int G, float* __restrict__ mean, float* __restrict__ rstd) {
-  const int t = blockIdx.x * blockDim.x + threadIdx.x;
-  if (t >= G * C) return;
-  const int g = t / C, c = t % C;
-  double n = 0.0, mu = 0.0, M2 = 0.0;
-  for (int q = 0; q < nq; ++q) {
-    const double nb = (double)min((int64_t)kStatChunk, P - (int64_t)q * kStatChunk);
-    const float* pq = part + (((int64_t)g * nq + q) * C + c) * 2;
-    const double mb = pq[0], M2b = pq[1];
-    const double delta = mb - mu, nt = n + nb;
-    mu += delta * nb / nt;
-    M2 += M2b + delta * delta * n * nb / nt;
-    n = nt;
-  }
-  mean[t] = (float)mu;
-  rstd[t] = (float)(1.0 / sqrt(M2 / n + (double)kBnEps));
+// Pass 2: Chan et al.'s pairwise combination of the chunk (count, mean, M2): one warp per
+// (replica, channel); lane l combines chunks l, l + 32, ... in order, then a fixed butterfly of
+// shuffles combines the lanes.  Biased variance, rstd = 1 / sqrt(var + eps).
+__device__ __forceinline__ void chan_merge(float& n, float& mu, float& M2, float nb, float mb,
+                                           float M2b) {
+  const float nt = n + nb;
+  if (nt <= 0.f) return;
+  const float delta = mb - mu, f = nb / nt;
+  mu = fmaf(delta, f, mu);
+  M2 = M2 + M2b + delta * delta * n * f;
+  n = nt;
 }
 
-// out = relu(gamma (y - mean) rstd + beta [+ option-A shortcut of the block input]).
+__global__ void bn_stats_finalize_kernel(const float* __restrict__ part, int64_t P, int C, int nq,
+                                         int G, float* __restrict__ mean, float* __restrict__ rstd) {
+  const int wid = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
+  if (wid >= G * C) return;
+  const int g = wid / C, c = wid % C;
+  float n = 0.f, mu = 0.f, M2 = 0.f;
+  for (int q = lane; q < nq; q += 32) {
+    const float nb = (float)min((int64_t)kStatChunk, P - (int64_t)q * kStatChunk);
+    const float* pq = part + (((int64_t)g * nq + q) * C + c) * 2;
+    chan_merge(n, mu, M2, nb, pq[0], pq[1]);
+  }
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const float n2 = __shfl_xor_sync(0xffffffffu, n, o);
+    const float m2 = __shfl_xor_sync(0xffffffffu, mu, o);
+    const float M22 = __shfl_xor_sync(0xffffffffu, M2, o);
+    // both partners combine (lower lane first) so they hold bit-identical results
+    float na = n, ma = mu, Ma = M2;
+    float nb = n2, mb = m2, Mb = M22;
+    if (lane & o) {
+      na = n2; ma = m2; Ma = M22;
+      nb = n; mb = mu; Mb = M2;
+    }
+    chan_merge(na, ma, Ma, nb, mb, Mb);
+    n = na;
+    mu = ma;
+    M2 = Ma;
+  }
+  if (lane == 0) {
+    mean[wid] = mu;
+    rstd[wid] = 1.0f / sqrtf(M2 / n + kBnEps);
+  }
+}
+
+// Four consecutive channels of an activation tensor (bf16 or fp32).
+template <typename TA>
+struct Vec4;
+template <>
+struct Vec4<float> {
+  __device__ __forceinline__ static float4 load(const float* p) {
+    return *reinterpret_cast<const float4*>(p);
+  }
+  __device__ __forceinline__ static void store(float* p, float4 v) {
+    *reinterpret_cast<float4*>(p) = v;
+  }
+};
+template <>
+struct Vec4<uint16_t> {
+  __device__ __forceinline__ static float4 load(const uint16_t* p) {
+    const uint2 u = *reinterpret_cast<const uint2*>(p);
+    return make_float4(bf2f((uint16_t)(u.x & 0xffff)), bf2f((uint16_t)(u.x >> 16)),
+                       bf2f((uint16_t)(u.y & 0xffff)), bf2f((uint16_t)(u.y >> 16)));
+  }
+  __device__ __forceinline__ static void store(uint16_t* p, float4 v) {
+    uint2 o;
+    o.x = (uint32_t)f2bf(v.x) | ((uint32_t)f2bf(v.y) << 16);
+    o.y = (uint32_t)f2bf(v.z) | ((uint32_t)f2bf(v.w) << 16);
+    *reinterpret_cast<uint2*>(p) = o;
+  }
+};
+
+// out = relu(gamma (y - mean) rstd + beta [+ option-A shortcut of the block input]); one thread
+// per pixel and 4 channels (C a multiple of 4, fewer than 2^31 groups of 4).
 template <typename TA>
 __global__ void bn_act_fwd_kernel(const float* __restrict__ y, const float* __restrict__ mean,
                                   const float* __restrict__ rstd, const float* __restrict__ W,
@@ -296,20 +351,33 @@ __global__ void bn_act_fwd_kernel(const float* __restrict__ y, const float* __re
                                   const TA* __restrict__ sc, int sc_H, int sc_W, int sc_C,
                                   int stride, TA* __restrict__ out, int G, int B, int H, int Wd,
                                   int C) {
-  const int64_t per = (int64_t)B * H * Wd * C;
-  const int64_t n = (int64_t)G * per;
-  const int64_t step = (int64_t)gridDim.x * blockDim.x;
-  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < n; e += step) {
-    const int g = (int)(e / per);
-    const int c = (int)(e % C);
+  const int C4 = C / 4;
+  const int P = B * H * Wd;
+  const int n4 = G * P * C4;
+  for (int t = blockIdx.x * blockDim.x + threadIdx.x; t < n4; t += gridDim.x * blockDim.x) {
+    const int c0 = (t % C4) * 4;
+    const int row = t / C4;
+    const int g = row / P, pix = row - g * P;
     const float* Wg = W + (int64_t)(w_g0 + g * w_gmul) * d_gs;
-    float v = Wg[g_off + c] * ((y[e] - mean[g * C + c]) * rstd[g * C + c]) + Wg[b_off + c];
-    if (sc && c < sc_C) {
-      const int64_t pix = (e % per) / C;
-      const int x = (int)(pix % Wd), h = (int)((pix / Wd) % H), b = (int)(pix / ((int64_t)Wd * H));
-      v += Elem<TA>::load(sc + ((((int64_t)g * B + b) * sc_H + h * stride) * sc_W + x * stride) * sc_C + c);
+    const float4 yv = *reinterpret_cast<const float4*>(y + (int64_t)t * 4);
+    const float yy[4] = {yv.x, yv.y, yv.z, yv.w};
+    float v[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const int c = c0 + i;
+      v[i] = Wg[g_off + c] * ((yy[i] - mean[g * C + c]) * rstd[g * C + c]) + Wg[b_off + c];
     }
-    Elem<TA>::store(out + e, fmaxf(v, 0.f));
+    if (sc && c0 < sc_C) {
+      const int x = pix % Wd, h = (pix / Wd) % H, b = pix / (Wd * H);
+      const float4 s4 = Vec4<TA>::load(
+          sc + ((((int64_t)g * B + b) * sc_H + h * stride) * sc_W + x * stride) * sc_C + c0);
+      v[0] += s4.x;
+      v[1] += s4.y;
+      v[2] += s4.z;
+      v[3] += s4.w;
+    }
+    Vec4<TA>::store(out + (int64_t)t * 4, make_float4(fmaxf(v[0], 0.f), fmaxf(v[1], 0.f),
+                                                      fmaxf(v[2], 0.f), fmaxf(v[3], 0.f)));
   }
 }
 
@@ -329,6 +397,7 @@ __global__ void __launch_bounds__(256) bn_bwd_partial_kernel(
   const float mu = mean[g * C + c], rs = rstd[g * C + c];
   float s1 = 0.f, s2 = 0.f;
   if (l < lanes)
+#pragma unroll 4
     for (int64_t p = p0 + l; p < p1; p += lanes) {
       const int64_t e = base + p * C + c;
       const float dz = Elem<TA>::load(out + e) > 0.f ? dout[e] : 0.f;
@@ -369,24 +438,36 @@ __global__ void bn_bwd_finalize_kernel(const float* __restrict__ part, int C, in
   Gr[(int64_t)g * d_gs + b_off + c] = a;
 }
 
-// dy = gamma rstd (dz - mean(dz) - xhat mean(dz xhat)), the convolution's output gradient.
+// dy = gamma rstd (dz - mean(dz) - xhat mean(dz xhat)), the convolution's output gradient; one
+// thread per pixel and 4 channels.
 template <typename TA>
 __global__ void bn_bwd_apply_kernel(const float* __restrict__ dout, const TA* __restrict__ out,
                                     const float* __restrict__ y, const float* __restrict__ mean,
                                     const float* __restrict__ rstd, const float* __restrict__ s12,
                                     const float* __restrict__ W, int64_t g_off, int64_t d_gs,
-                                    TA* __restrict__ dy, int G, int64_t P, int C) {
-  const int64_t per = P * C, n = (int64_t)G * per;
+                                    TA* __restrict__ dy, int G, int64_t P64, int C) {
+  const int C4 = C / 4;
+  const int P = (int)P64;
+  const int n4 = G * P * C4;
   const float invM = 1.0f / (float)P;
-  const int64_t step = (int64_t)gridDim.x * blockDim.x;
-  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < n; e += step) {
-    const int g = (int)(e / per), c = (int)(e % C);
-    const int gc = g * C + c;
-    const float dz = Elem<TA>::load(out + e) > 0.f ? dout[e] : 0.f;
-    const float xh = (y[e] - mean[gc]) * rstd[gc];
-    const float v = W[(int64_t)g * d_gs + g_off + c] * rstd[gc] *
-                    (dz - s12[2 * gc] * invM - xh * (s12[2 * gc + 1] * invM));
-    Elem<TA>::store(dy + e, v);
+  for (int t = blockIdx.x * blockDim.x + threadIdx.x; t < n4; t += gridDim.x * blockDim.x) {
+    const int c0 = (t % C4) * 4;
+    const int g = (t / C4) / P;
+    const float4 d4 = *reinterpret_cast<const float4*>(dout + (int64_t)t * 4);
+    const float4 o4 = Vec4<TA>::load(out + (int64_t)t * 4);
+    const float4 y4 = *reinterpret_cast<const float4*>(y + (int64_t)t * 4);
+    const float dd[4] = {d4.x, d4.y, d4.z, d4.w}, oo[4] = {o4.x, o4.y, o4.z, o4.w};
+    const float yy[4] = {y4.x, y4.y, y4.z, y4.w};
+    float v[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const int gc = g * C + c0 + i;
+      const float dz = oo[i] > 0.f ? dd[i] : 0.f;
+      const float xh = (yy[i] - mean[gc]) * rstd[gc];
+      v[i] = W[(int64_t)g * d_gs + g_off + c0 + i] * rstd[gc] *
+             (dz - s12[2 * gc] * invM - xh * (s12[2 * gc + 1] * invM));
+    }
+    Vec4<TA>::store(dy + (int64_t)t * 4, make_float4(v[0], v[1], v[2], v[3]));
   }
 }
 
@@ -414,6 +495,150 @@ __global__ void avgpool_bwd_kernel(const float* __restrict__ dfeat, float* __res
   }
 }
 
+// im2col for the tensor-core convolutions: col[g][p][(kh 3 + kw) Cin + ci] =
+// in[g][b][oh s + kh - 1][ow s + kw - 1][ci] (zero outside the image), p = (b, oh, ow); bf16,
+// 8 channels (16 bytes) per thread, Cin a multiple of 8.
+__global__ void im2col_kernel(const uint16_t* __restrict__ in, uint16_t* __restrict__ col, int G,
+                              int B, int Hin, int Win, int Cin, int Hout, int Wout, int stride) {
+  const int c8n = Cin / 8;
+  const int64_t P = (int64_t)B * Hout * Wout;
+  const int64_t n = (int64_t)G * P * 9 * c8n;
+  const int64_t step = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < n; e += step) {
+    const int c8 = (int)(e % c8n);
+    int64_t t = e / c8n;
+    const int tap = (int)(t % 9);
+    t /= 9;
+    const int64_t p = t % P;
+    const int g = (int)(t / P);
+    const int ow = (int)(p % Wout), oh = (int)((p / Wout) % Hout), b = (int)(p / ((int64_t)Wout * Hout));
+    const int ih = oh * stride + tap / 3 - 1, iw = ow * stride + tap % 3 - 1;
+    uint4 v = make_uint4(0u, 0u, 0u, 0u);
+    if (ih >= 0 && ih < Hin && iw >= 0 && iw < Win)
+      v = __ldg(reinterpret_cast<const uint4*>(in + ((((int64_t)g * B + b) * Hin + ih) * Win + iw) * Cin + c8 * 8));
+    *reinterpret_cast<uint4*>(col + ((int64_t)g * P + p) * 9 * Cin + tap * Cin + c8 * 8) = v;
+  }
+}
+
+// im2col with any channel count: col[g][p][tap Cin + ci] for j = tap Cin + ci < 9 Cin, zero for
+// the padding columns 9 Cin <= j < ldc (ldc a multiple of 8 keeps rows 16-byte aligned).
+template <typename TA>
+__global__ void im2col_any_kernel(const TA* __restrict__ in, uint16_t* __restrict__ col, int G, int B,
+                                  int Hin, int Win, int Cin, int Hout, int Wout, int stride, int ldc) {
+  const int64_t P = (int64_t)B * Hout * Wout;
+  const int64_t n = (int64_t)G * P * ldc;
+  const int64_t step = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < n; e += step) {
+    const int j = (int)(e % ldc);
+    const int64_t t = e / ldc;
+    const int64_t p = t % P;
+    const int g = (int)(t / P);
+    float v = 0.f;
+    if (j < 9 * Cin) {
+      const int tap = j / Cin, ci = j % Cin;
+      const int ow = (int)(p % Wout), oh = (int)((p / Wout) % Hout);
+      const int b = (int)(p / ((int64_t)Wout * Hout));
+      const int ih = oh * stride + tap / 3 - 1, iw = ow * stride + tap % 3 - 1;
+      if (ih >= 0 && ih < Hin && iw >= 0 && iw < Win)
+        v = Elem<TA>::load(in + ((((int64_t)g * B + b) * Hin + ih) * Win + iw) * Cin + ci);
+    }
+    col[e] = f2bf(v);
+  }
+}
+
+// Column matrix of a data gradient: for each pixel (ih, iw) of the convolution's input and each
+// flipped tap t' = (kh', kw'), the output-gradient row at ((ih + kh' - 1) / s, (iw + kw' - 1) / s)
+// when both are whole and inside the output, else zero.  With the flipped, transposed weights
+// this writes dx = sum over the taps reaching (ih, iw) of dy w (stride 1 or 2).
+__global__ void col_dgrad_kernel(const uint16_t* __restrict__ dy, uint16_t* __restrict__ col, int G,
+                                 int B, int Hin, int Win, int Cout, int Hout, int Wout, int stride) {
+  const int c8n = Cout / 8;
+  const int64_t P = (int64_t)B * Hin * Win;
+  const int64_t n = (int64_t)G * P * 9 * c8n;
+  const int64_t step = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < n; e += step) {
+    const int c8 = (int)(e % c8n);
+    int64_t t = e / c8n;
+    const int tap = (int)(t % 9);
+    t /= 9;
+    const int64_t p = t % P;
+    const int g = (int)(t / P);
+    const int iw = (int)(p % Win), ih = (int)((p / Win) % Hin), b = (int)(p / ((int64_t)Win * Hin));
+    const int hn = ih + tap / 3 - 1, wn = iw + tap % 3 - 1;
+    uint4 v = make_uint4(0u, 0u, 0u, 0u);
+    if (hn >= 0 && wn >= 0 && hn % stride == 0 && wn % stride == 0 && hn / stride < Hout &&
+        wn / stride < Wout)
+      v = __ldg(reinterpret_cast<const uint4*>(
+          dy + ((((int64_t)g * B + b) * Hout + hn / stride) * Wout + wn / stride) * Cout + c8 * 8));
+    *reinterpret_cast<uint4*>(col + ((int64_t)g * P + p) * 9 * Cout + tap * Cout + c8 * 8) = v;
+  }
+}
+
+// Weights with each [9 Cin] row padded to ldc columns (zeros), bf16: the stem's tensor-core
+// operand (9 Cin = 27 is not a multiple of 8).
+__global__ void pad_weights_kernel(const uint16_t* __restrict__ Wb, int64_t d_pad, int64_t w_off,
+                                   uint16_t* __restrict__ out, int G, int rows, int cols, int ldc) {
+  const int64_t n = (int64_t)G * rows * ldc;
+  const int64_t step = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < n; e += step) {
+    const int j = (int)(e % ldc);
+    const int r = (int)((e / ldc) % rows);
+    const int g = (int)(e / ((int64_t)rows * ldc));
+    out[e] = j < cols ? Wb[(int64_t)g * d_pad + w_off + (int64_t)r * cols + j] : (uint16_t)0;
+  }
+}
+
+// Sum of split partials [g][q][rows][ldc] in split order, keeping the first `cols` columns:
+// out[g * out_gs + r cols + j].
+__global__ void sum_partials_crop_kernel(const float* __restrict__ part, int nq, int rows, int ldc,
+                                         int cols, int G, float* __restrict__ out, int64_t out_gs) {
+  const int64_t n = (int64_t)G * rows * cols;
+  const int64_t step = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < n; t += step) {
+    const int j = (int)(t % cols);
+    const int r = (int)((t / cols) % rows);
+    const int g = (int)(t / ((int64_t)rows * cols));
+    const float* p = part + (int64_t)g * nq * rows * ldc + (int64_t)r * ldc + j;
+    float s = 0.f;
+    for (int q = 0; q < nq; ++q) s += p[(int64_t)q * rows * ldc];
+    out[(int64_t)g * out_gs + (int64_t)r * cols + j] = s;
+  }
+}
+
+// Weights of the stride-1 data gradient as a convolution of the output gradient:
+// wt[g][ci][t][co] = w[g][co][8 - t][ci] (taps flipped, channels transposed), bf16.
+__global__ void flip_weights_kernel(const uint16_t* __restrict__ Wb, int64_t d_pad, int64_t w_off,
+                                    uint16_t* __restrict__ wt, int G, int Cin, int Cout) {
+  const int64_t n = (int64_t)G * Cin * 9 * Cout;
+  const int64_t step = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < n; e += step) {
+    const int co = (int)(e % Cout);
+    const int t = (int)((e / Cout) % 9);
+    const int ci = (int)((e / (9 * Cout)) % Cin);
+    const int g = (int)(e / ((int64_t)Cin * 9 * Cout));
+    wt[e] = Wb[(int64_t)g * d_pad + w_off + ((int64_t)co * 9 + (8 - t)) * Cin + ci];
+  }
+}
+
+// The option-A shortcut's share of a block's input gradient: for input pixels on the stride grid
+// and the first Cin channels, dx += dout * (out > 0) at (ih / s, iw / s).
+template <typename TA>
+__global__ void add_shortcut_grad_kernel(float* __restrict__ dx, const float* __restrict__ dout,
+                                         const TA* __restrict__ out, int G, int B, int Hin, int Win,
+                                         int Cin, int Hout, int Wout, int Cout, int stride) {
+  const int64_t n = (int64_t)G * B * Hin * Win * Cin;
+  const int64_t step = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < n; e += step) {
+    const int ci = (int)(e % Cin);
+    const int64_t pix = e / Cin;
+    const int iw = (int)(pix % Win), ih = (int)((pix / Win) % Hin);
+    if (ih % stride || iw % stride) continue;
+    const int64_t gb = pix / ((int64_t)Win * Hin);
+    const int64_t o = ((gb * Hout + ih / stride) * Wout + iw / stride) * Cout + ci;
+    if (Elem<TA>::load(out + o) > 0.f) dx[e] += dout[o];
+  }
+}
+
 }  // namespace
 
 struct ResNetPlan {
@@ -434,6 +659,13 @@ struct ResNetPlan {
   float* part = nullptr;
   size_t part_floats = 0;
   float* s12 = nullptr;
+  // tensor-core convolutions (BF16 mode): per-convolution im2col of its input (kept from the
+  // forward for the weight gradient), the output-gradient im2col and flipped weights of the
+  // stride-1 data gradients
+  bool tc = false;
+  std::vector<uint16_t*> col;
+  uint16_t* colT = nullptr;
+  uint16_t* wt = nullptr;
   std::string err;
 };
 
@@ -466,10 +698,56 @@ lsgd_status rn_check(ResNetPlan* p, int64_t* launches, cudaError_t e, const char
 
 int64_t conv_pixels(const ResNetPlan* p, const ConvL& c) { return (int64_t)p->B * c.hout * c.wout; }
 
+bool conv_on_tc(const ResNetPlan* p, const ConvL& c) { return p->tc && c.cout % 8 == 0; }
+// Row length of a convolution's column matrix: 9 Cin rounded up to a multiple of 8 elements.
+int col_ld(const ConvL& c) { return (int)rup(9 * c.cin, 8); }
+
+int grid_for_items(int64_t n) { return grid_cap(n, 256); }
+
 template <typename TA>
-lsgd_status conv_forward(ResNetPlan* p, const ConvL& c, const void* in, const void* Wop, int w_g0,
+lsgd_status conv_forward(ResNetPlan* p, int i, const void* in, const void* Wop, int w_g0,
                          int w_gmul, float* y, int G, cudaStream_t s, int64_t* launches) {
+  const ConvL& c = p->convs[i];
   const int64_t P = conv_pixels(p, c);
+  if (conv_on_tc(p, c) && w_g0 == 0 && w_gmul == 1) {
+    // y = im2col(in) [P][9 Cin] x W^T on the tensor cores (both operands K-major)
+    const int Kc = col_ld(c);
+    const uint16_t* wop = reinterpret_cast<const uint16_t*>(Wop) + c.w_off;
+    int64_t w_gs = p->d_pad;
+    if (Kc == 9 * c.cin) {
+      RN_LAUNCH((im2col_kernel<<<grid_for_items((int64_t)G * P * 9 * (c.cin / 8)), 256, 0, s>>>(
+          reinterpret_cast<const uint16_t*>(in), p->col[i], G, p->B, c.hin, c.win, c.cin, c.hout,
+          c.wout, c.stride)));
+    } else {
+      RN_LAUNCH((im2col_any_kernel<uint16_t><<<grid_for_items((int64_t)G * P * Kc), 256, 0, s>>>(
+          reinterpret_cast<const uint16_t*>(in), p->col[i], G, p->B, c.hin, c.win, c.cin, c.hout,
+          c.wout, c.stride, Kc)));
+      RN_LAUNCH((pad_weights_kernel<<<grid_for_items((int64_t)G * c.cout * Kc), 256, 0, s>>>(
+          reinterpret_cast<const uint16_t*>(Wop), p->d_pad, c.w_off, p->wt, G, c.cout, 9 * c.cin, Kc)));
+      wop = p->wt;
+      w_gs = (int64_t)c.cout * Kc;
+    }
+    TcGemmArgs t{};
+    t.M = (int)P;
+    t.N = c.cout;
+    t.Kd = Kc;
+    t.G = G;
+    const int bn = tc_tile_n(Kc);
+    bool ok = make_tma_map_bf16(&t.A.map, p->col[i], Kc, P, G, Kc, (uint64_t)P * Kc, 64, kTcTileM);
+    ok &= make_tma_map_bf16(&t.B.map, wop, Kc, c.cout, G, Kc, w_gs, 64, bn);
+    if (!ok) {
+      p->err = "TMA map encoding failed (convolution)";
+      return LSGD_ECUDA;
+    }
+    t.A.box_rows = kTcTileM;
+    t.B.box_rows = bn;
+    t.C = y;
+    t.c_rs = c.cout;
+    t.c_gs = P * c.cout;
+    t.epi = EPI_STORE;
+    RN_CALL(launch_gemm_tc(t, s));
+    return LSGD_OK;
+  }
   dim3 grid((unsigned)((P + 127) / 128), (unsigned)((c.cout + 15) / 16), (unsigned)G);
   const size_t smem = (size_t)16 * 9 * c.cin * 4;
   const TA* wbase = reinterpret_cast<const TA*>(Wop) + (int64_t)w_g0 * p->d_pad + c.w_off;
@@ -486,8 +764,8 @@ lsgd_status bn_stats(ResNetPlan* p, const ConvL& c, const float* y, float* mean,
   const int lanes = std::max(1, 256 / c.cout);
   dim3 grid(nq, G);
   RN_LAUNCH((bn_stats_partial_kernel<<<grid, lanes * c.cout, 0, s>>>(y, P, c.cout, nq, p->part)));
-  RN_LAUNCH((bn_stats_finalize_kernel<<<(G * c.cout + 127) / 128, 128, 0, s>>>(p->part, P, c.cout, nq,
-                                                                                G, mean, rstd)));
+  RN_LAUNCH((bn_stats_finalize_kernel<<<(G * c.cout * 32 + 127) / 128, 128, 0, s>>>(
+      p->part, P, c.cout, nq, G, mean, rstd)));
   return LSGD_OK;
 }
 
@@ -499,14 +777,14 @@ lsgd_status forward_impl(ResNetPlan* p, const float* W, const void* Wop, int w_g
     const ConvL& c = p->convs[i];
     // block j uses convolutions 2j+1 (input act[2j], the block input) and 2j+2 (input act[2j+1])
     const void* in = i == 0 ? p->x0 : p->act[i - 1];
-    lsgd_status st = conv_forward<TA>(p, c, in, Wop, w_g0, w_gmul, p->y[i], G, s, launches);
+    lsgd_status st = conv_forward<TA>(p, (int)i, in, Wop, w_g0, w_gmul, p->y[i], G, s, launches);
     if (st != LSGD_OK) return st;
     st = bn_stats(p, c, p->y[i], p->mean[i], p->rstd[i], G, s, launches);
     if (st != LSGD_OK) return st;
     const bool second = i > 0 && i % 2 == 0;
     const TA* sc = second ? reinterpret_cast<const TA*>(p->act[i - 2]) : nullptr;
     const ConvL& ca = p->convs[second ? i - 1 : i];
-    const int64_t n = (int64_t)G * conv_pixels(p, c) * c.cout;
+    const int64_t n = (int64_t)G * conv_pixels(p, c) * c.cout / 4;
     RN_LAUNCH((bn_act_fwd_kernel<TA><<<grid_cap(n, 256), 256, 0, s>>>(
         p->y[i], p->mean[i], p->rstd[i], W, c.g_off, c.b_off, p->d_pad, w_g0, w_gmul, sc, ca.hin,
         ca.win, ca.cin, ca.stride, reinterpret_cast<TA*>(p->act[i]), G, p->B, c.hout, c.wout,
@@ -552,7 +830,7 @@ lsgd_status bn_backward(ResNetPlan* p, const ConvL& c, int i, const float* dout,
       p->part)));
   RN_LAUNCH((bn_bwd_finalize_kernel<<<(K * c.cout + 127) / 128, 128, 0, s>>>(
       p->part, c.cout, nq, K, p->s12, Gr, c.g_off, c.b_off, p->d_pad)));
-  const int64_t n = (int64_t)K * P * c.cout;
+  const int64_t n = (int64_t)K * P * c.cout / 4;
   RN_LAUNCH((bn_bwd_apply_kernel<TA><<<grid_cap(n, 256), 256, 0, s>>>(
       dout, reinterpret_cast<const TA*>(out), p->y[i], p->mean[i], p->rstd[i], p->s12, W, c.g_off,
       p->d_pad, reinterpret_cast<TA*>(p->dy), K, P, c.cout)));
@@ -560,10 +838,41 @@ lsgd_status bn_backward(ResNetPlan* p, const ConvL& c, int i, const float* dout,
 }
 
 template <typename TA>
-lsgd_status conv_wgrad(ResNetPlan* p, const ConvL& c, const void* in, float* Gr, cudaStream_t s,
+lsgd_status conv_wgrad(ResNetPlan* p, int i, const void* in, float* Gr, cudaStream_t s,
                        int64_t* launches) {
+  const ConvL& c = p->convs[i];
   const int K = p->K;
   const int64_t P = conv_pixels(p, c);
+  if (conv_on_tc(p, c)) {
+    // dW [Cout][9 Cin] = dy^T [Cout][P] x im2col(in) [P][9 Cin]: both operands pixel-major
+    // ("MN-major"); the pixel reduction is split across CTAs and the partials summed in order.
+    const int Kc = col_ld(c);
+    const int tiles = ((Kc + 63) / 64) * K;
+    const int splits = tc_valid_splits((int)P, std::max(1, (4 * kNumSMs + tiles - 1) / tiles));
+    TcGemmArgs t{};
+    t.M = c.cout;
+    t.N = Kc;
+    t.Kd = (int)P;
+    t.G = K;
+    bool ok = make_tma_map_bf16(&t.A.map, p->dy, c.cout, P, K, c.cout, (uint64_t)P * c.cout, 64, 64);
+    ok &= make_tma_map_bf16(&t.B.map, p->col[i], Kc, P, K, Kc, (uint64_t)P * Kc, 64, 64);
+    if (!ok) {
+      p->err = "TMA map encoding failed (convolution weight gradient)";
+      return LSGD_ECUDA;
+    }
+    t.A.mn_major = t.B.mn_major = true;
+    t.A.box_rows = t.B.box_rows = 64;
+    t.C = p->part;
+    t.c_rs = Kc;
+    t.c_split_stride = (int64_t)c.cout * Kc;
+    t.c_gs = (int64_t)splits * c.cout * Kc;
+    t.splits = splits;
+    t.epi = EPI_STORE;
+    RN_CALL(launch_gemm_tc(t, s));
+    RN_LAUNCH((sum_partials_crop_kernel<<<grid_cap((int64_t)K * c.cout * 9 * c.cin, 256), 256, 0, s>>>(
+        p->part, splits, c.cout, Kc, 9 * c.cin, K, Gr + c.w_off, p->d_pad)));
+    return LSGD_OK;
+  }
   const int nq = (int)((P + kWgradChunk - 1) / kWgradChunk);
   const int J = 9 * c.cin;
   const size_t smem = (size_t)(kWgradTile * 16 + kWgradTile * J) * 4;
@@ -577,10 +886,46 @@ lsgd_status conv_wgrad(ResNetPlan* p, const ConvL& c, const void* in, float* Gr,
 }
 
 template <typename TA>
-lsgd_status conv_dgrad(ResNetPlan* p, const ConvL& c, const void* Wop, float* dx, const float* dout,
+lsgd_status conv_dgrad(ResNetPlan* p, int i, const void* Wop, float* dx, const float* dout,
                        const void* out_act, cudaStream_t s, int64_t* launches) {
+  const ConvL& c = p->convs[i];
   const int K = p->K;
   const int64_t P = (int64_t)p->B * c.hin * c.win;
+  if (conv_on_tc(p, c) && c.cin % 8 == 0) {
+    // dx = col(dy) [P][9 Cout] x wt^T with the flipped, transposed weights (stride 1 or 2)
+    const int Kc = 9 * c.cout;
+    RN_LAUNCH((col_dgrad_kernel<<<grid_for_items((int64_t)K * P * 9 * (c.cout / 8)), 256, 0, s>>>(
+        reinterpret_cast<const uint16_t*>(p->dy), p->colT, K, p->B, c.hin, c.win, c.cout, c.hout,
+        c.wout, c.stride)));
+    RN_LAUNCH((flip_weights_kernel<<<grid_for_items((int64_t)K * c.cin * Kc), 256, 0, s>>>(
+        reinterpret_cast<const uint16_t*>(Wop), p->d_pad, c.w_off, p->wt, K, c.cin, c.cout)));
+    TcGemmArgs t{};
+    t.M = (int)P;
+    t.N = c.cin;
+    t.Kd = Kc;
+    t.G = K;
+    const int bn = tc_tile_n(Kc);
+    bool ok = make_tma_map_bf16(&t.A.map, p->colT, Kc, P, K, Kc, (uint64_t)P * Kc, 64, kTcTileM);
+    ok &= make_tma_map_bf16(&t.B.map, p->wt, Kc, c.cin, K, Kc, (uint64_t)c.cin * Kc, 64, bn);
+    if (!ok) {
+      p->err = "TMA map encoding failed (convolution data gradient)";
+      return LSGD_ECUDA;
+    }
+    t.A.box_rows = kTcTileM;
+    t.B.box_rows = bn;
+    t.C = dx;
+    t.c_rs = c.cin;
+    t.c_gs = P * c.cin;
+    t.epi = EPI_STORE;
+    RN_CALL(launch_gemm_tc(t, s));
+    if (dout) {
+      const int64_t n = (int64_t)K * P * c.cin;
+      RN_LAUNCH((add_shortcut_grad_kernel<TA><<<grid_cap(n, 256), 256, 0, s>>>(
+          dx, dout, reinterpret_cast<const TA*>(out_act), K, p->B, c.hin, c.win, c.cin, c.hout,
+          c.wout, c.cout, c.stride)));
+    }
+    return LSGD_OK;
+  }
   dim3 grid((unsigned)((P + 63) / 64), (unsigned)((c.cin + 15) / 16), (unsigned)K);
   const size_t smem = (size_t)c.cout * 9 * 16 * 4;
   RN_LAUNCH((conv_dgrad_kernel<TA><<<grid, 64, smem, s>>>(
@@ -655,17 +1000,17 @@ lsgd_status fwd_bwd_impl(ResNetPlan* p, const float* W, const void* Wop, float* 
     // second convolution: BN backward through the block's output ReLU, then its products
     st = bn_backward<TA>(p, cb, ib, p->dA[cur], p->act[ib], W, Gr, s, launches);
     if (st != LSGD_OK) return st;
-    st = conv_wgrad<TA>(p, cb, p->act[ia], Gr, s, launches);
+    st = conv_wgrad<TA>(p, ib, p->act[ia], Gr, s, launches);
     if (st != LSGD_OK) return st;
-    st = conv_dgrad<TA>(p, cb, Wop, p->dh, nullptr, nullptr, s, launches);
+    st = conv_dgrad<TA>(p, ib, Wop, p->dh, nullptr, nullptr, s, launches);
     if (st != LSGD_OK) return st;
     // first convolution: BN backward through the inner ReLU, then its products; the data
     // gradient also receives the shortcut's share of the block's output gradient
     st = bn_backward<TA>(p, ca, ia, p->dh, p->act[ia], W, Gr, s, launches);
     if (st != LSGD_OK) return st;
-    st = conv_wgrad<TA>(p, ca, blk_in, Gr, s, launches);
+    st = conv_wgrad<TA>(p, ia, blk_in, Gr, s, launches);
     if (st != LSGD_OK) return st;
-    st = conv_dgrad<TA>(p, ca, Wop, p->dA[1 - cur], p->dA[cur], p->act[ib], s, launches);
+    st = conv_dgrad<TA>(p, ia, Wop, p->dA[1 - cur], p->dA[cur], p->act[ib], s, launches);
     if (st != LSGD_OK) return st;
     cur = 1 - cur;
   }
@@ -673,7 +1018,7 @@ lsgd_status fwd_bwd_impl(ResNetPlan* p, const float* W, const void* Wop, float* 
   const ConvL& c0 = p->convs[0];
   st = bn_backward<TA>(p, c0, 0, p->dA[cur], p->act[0], W, Gr, s, launches);
   if (st != LSGD_OK) return st;
-  return conv_wgrad<TA>(p, c0, p->x0, Gr, s, launches);
+  return conv_wgrad<TA>(p, 0, p->x0, Gr, s, launches);
 }
 
 }  // namespace
@@ -686,6 +1031,14 @@ bool resnet_supported(const lsgd_config& cfg, std::string* why) {
   }
   if (m.base_ch * 4 > 64 || m.in_c > 64) {
     if (why) *why = "ResNet channels above 64 are not supported";
+    return false;
+  }
+  if (m.base_ch % 4) {
+    if (why) *why = "ResNet base channels must be a multiple of 4";
+    return false;
+  }
+  if ((int64_t)cfg.K * cfg.B_loc * m.in_h * m.in_w * m.base_ch >= (1LL << 31)) {
+    if (why) *why = "ResNet activations too large for 32-bit element indexing";
     return false;
   }
   if (cfg.B_loc > 8192 || (int64_t)cfg.B_loc * m.in_h * m.in_w > (1LL << 30)) {
@@ -708,6 +1061,10 @@ ResNetPlan* resnet_plan_create(const lsgd_config& cfg) {
   p->base = m.base_ch;
   p->blocks = m.res_blocks;
   p->bf16 = cfg.precision == LSGD_BF16;
+  {
+    const char* e = std::getenv("LSGD_FORCE_SIMT");
+    p->tc = p->bf16 && tc_available() && !(e && e[0] == '1');
+  }
   // layout: canonical order (stem, block convs, fc W, fc b; each conv followed by its BN gamma,
   // beta); padded order puts every BatchNorm parameter after the decayed ones.
   int64_t canon = 0, off = 0;
@@ -790,7 +1147,7 @@ lsgd_status resnet_alloc(ResNetPlan* p, const std::function<void*(size_t)>& allo
   const int K = p->K, B = p->B;
   const size_t e = esz(p);
   p->x0 = alloc((size_t)K * B * p->H0 * p->W0 * p->C0 * e);
-  size_t part = 0;
+  size_t part = 0, colT = 0, wt = 0;
   for (const ConvL& c : p->convs) {
     const int64_t n = (int64_t)K * B * c.hout * c.wout * c.cout;
     p->y.push_back((float*)alloc((size_t)n * 4));
@@ -802,6 +1159,30 @@ lsgd_status resnet_alloc(ResNetPlan* p, const std::function<void*(size_t)>& allo
     const int64_t nq_w = (P + kWgradChunk - 1) / kWgradChunk;
     part = std::max(part, (size_t)(K * nq_s * c.cout * 2));
     part = std::max(part, (size_t)(K * nq_w * c.cout * 9 * c.cin));
+    if (conv_on_tc(p, c)) {
+      const int Kc = col_ld(c);
+      const int tiles = ((Kc + 63) / 64) * K;
+      const int splits = tc_valid_splits((int)P, std::max(1, (4 * kNumSMs + tiles - 1) / tiles));
+      part = std::max(part, (size_t)K * splits * c.cout * Kc);
+      p->col.push_back((uint16_t*)alloc((size_t)K * P * Kc * 2));
+      if (!p->col.back()) return LSGD_ENOMEM;
+      if (c.cin % 8 == 0) {
+        colT = std::max(colT, (size_t)K * B * c.hin * c.win * 9 * c.cout);
+        wt = std::max(wt, (size_t)K * c.cin * 9 * c.cout);
+      } else {
+        wt = std::max(wt, (size_t)K * c.cout * Kc);
+      }
+    } else {
+      p->col.push_back(nullptr);
+    }
+  }
+  if (colT) {
+    p->colT = (uint16_t*)alloc(colT * 2);
+    if (!p->colT) return LSGD_ENOMEM;
+  }
+  if (wt) {
+    p->wt = (uint16_t*)alloc(wt * 2);
+    if (!p->wt) return LSGD_ENOMEM;
   }
   p->part_floats = part;
   p->part = (float*)alloc(part * 4);

@@ -231,6 +231,17 @@ lsgd_status lsgd_sgd_update(float* w, float* u, const float* g, uint16_t* Wb, in
 lsgd_status lsgd_grouped_gemm_bf16(const uint16_t* A, int a_mn, const uint16_t* B, int b_mn, float* C,
                                    int M, int N, int Kd, int G, int engine, void* stream);
 
+/* Per-worker BatchNorm batch statistics (Sec. A.4: each worker normalises with the statistics of
+ * its own mini-batch): for y [G][P][C] fp32 (G replicas, P = batch x height x width positions, C
+ * channels, channel fastest) writes mean[G][C] and rstd[G][C] = 1 / sqrt(biased variance + 1e-5).
+ * Two deterministic passes: per-chunk mean and squared deviations, then Chan's pairwise
+ * combination in chunk order.  The chunk partials live in a scratch buffer of
+ * G x ceil(P / 1024) x C x 2 floats that this call allocates and frees on `stream` (stream-ordered
+ * allocation).  Device pointers; 1 <= C <= 256, G <= 65535, P <= 65535 x 1024; LSGD_EINVAL
+ * otherwise, LSGD_ENOMEM if the scratch cannot be allocated. */
+lsgd_status lsgd_batchnorm_stats(const float* y, int64_t P, int C, int G, float* mean, float* rstd,
+                                 void* stream);
+
 /* Worker mini-batch indices for one step into dst [K][B] int32 (device), as lsgd_local_step. */
 lsgd_status lsgd_sample_indices(int32_t* dst, uint64_t seed, int64_t step, int K, int B, int64_t N,
                                 void* stream);

@@ -34,7 +34,7 @@ EXPORTS = [
     "lsgd_check_finite", "lsgd_save", "lsgd_load", "lsgd_num_params", "lsgd_step_count",
     "lsgd_sync_count", "lsgd_total_steps", "lsgd_lr_at", "lsgd_kernel_launches", "lsgd_last_error",
     "lsgd_kway_average", "lsgd_sgd_update", "lsgd_sample_indices", "lsgd_profile_enable",
-    "lsgd_profile_read", "lsgd_grouped_gemm_bf16",
+    "lsgd_profile_read", "lsgd_grouped_gemm_bf16", "lsgd_batchnorm_stats",
 ]
 PHASES = ["input", "forward", "loss", "backward", "update", "average"]
 
@@ -153,6 +153,7 @@ def lib():
                                  ctypes.c_float, i64, i64, vp], st),
             "lsgd_sample_indices": ([vp, ctypes.c_uint64, i64, ctypes.c_int, ctypes.c_int, i64, vp], st),
             "lsgd_profile_enable": ([vp, ctypes.c_int], st),
+            "lsgd_batchnorm_stats": ([vp, i64, ctypes.c_int, ctypes.c_int, vp, vp, vp], st),
             "lsgd_grouped_gemm_bf16": ([vp, ctypes.c_int, vp, ctypes.c_int, vp, ctypes.c_int,
                                         ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int, vp], st),
             "lsgd_profile_read": ([vp, P(Profile)], st),
@@ -406,3 +407,10 @@ def lsgd_grouped_gemm_bf16(A, a_mn: bool, B, b_mn: bool, C, M: int, N: int, Kd: 
     _check(lib().lsgd_grouped_gemm_bf16(_ptr(A), int(bool(a_mn)), _ptr(B), int(bool(b_mn)), _ptr(C),
                                         int(M), int(N), int(Kd), int(G), int(engine),
                                         ctypes.c_void_p(stream)))
+
+
+def lsgd_batchnorm_stats(y, P: int, C: int, G: int, mean, rstd, stream=None):
+    """Per-replica BatchNorm statistics of a CUDA float32 tensor y [G, P, C] into mean, rstd [G, C]."""
+    stream = _current_stream() if stream is None else stream
+    _check(lib().lsgd_batchnorm_stats(_ptr(y), int(P), int(C), int(G), _ptr(mean), _ptr(rstd),
+                                      ctypes.c_void_p(stream)))

@@ -1023,6 +1023,24 @@ lsgd_status fwd_bwd_impl(ResNetPlan* p, const float* W, const void* Wop, float* 
 
 }  // namespace
 
+size_t batchnorm_stats_scratch_floats(int64_t P, int C, int G) {
+  const int64_t nq = (P + kStatChunk - 1) / kStatChunk;
+  return (size_t)G * nq * C * 2;
+}
+
+cudaError_t launch_batchnorm_stats(const float* y, int64_t P, int C, int G, float* mean,
+                                   float* rstd, float* part, cudaStream_t s) {
+  if (P < 1 || C < 1 || C > 256 || G < 1 || G > 65535) return cudaErrorInvalidValue;
+  const int64_t nq = (P + kStatChunk - 1) / kStatChunk;
+  if (nq > 65535) return cudaErrorInvalidValue;
+  const int lanes = std::max(1, 256 / C);
+  bn_stats_partial_kernel<<<dim3((unsigned)nq, (unsigned)G), lanes * C, 0, s>>>(y, P, C, (int)nq, part);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  bn_stats_finalize_kernel<<<(G * C * 32 + 127) / 128, 128, 0, s>>>(part, P, C, (int)nq, G, mean, rstd);
+  return cudaGetLastError();
+}
+
 bool resnet_supported(const lsgd_config& cfg, std::string* why) {
   const lsgd_model& m = cfg.model;
   if (m.in_h < 1 || m.in_w < 1 || m.in_c < 1 || m.n_classes < 1 || m.base_ch < 1 || m.res_blocks < 1) {

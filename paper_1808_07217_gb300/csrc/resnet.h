@@ -35,6 +35,12 @@ lsgd_status resnet_eval(ResNetPlan* p, const float* W, const uint16_t* Wb, int64
                         int groups, const int32_t* labels, float* row_loss, cudaStream_t s,
                         int64_t* launches);
 void* resnet_input(ResNetPlan* p);
+
+// Per-replica BatchNorm batch statistics of y [G][P][C] fp32 into mean, rstd [G][C], through the
+// chunk partials `part` (batchnorm_stats_scratch_floats(P, C, G) floats, fully overwritten).
+size_t batchnorm_stats_scratch_floats(int64_t P, int C, int G);
+cudaError_t launch_batchnorm_stats(const float* y, int64_t P, int C, int G, float* mean,
+                                   float* rstd, float* part, cudaStream_t s);
 const char* resnet_last_error(const ResNetPlan* p);
 
 }  // namespace lsgd

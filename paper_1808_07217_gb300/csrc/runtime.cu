@@ -1153,6 +1153,24 @@ lsgd_status lsgd_grouped_gemm_bf16(const uint16_t* A, int a_mn, const uint16_t* 
   return LSGD_OK;
 }
 
+lsgd_status lsgd_batchnorm_stats(const float* y, int64_t P, int C, int G, float* mean, float* rstd,
+                                 void* stream) {
+  if (!y || !mean || !rstd || P < 1 || C < 1 || C > 256 || G < 1 || G > 65535 ||
+      (P + 1023) / 1024 > 65535)
+    return fail(nullptr, LSGD_EINVAL, "lsgd_batchnorm_stats: bad arguments");
+  cudaStream_t s = (cudaStream_t)stream;
+  float* part = nullptr;
+  const size_t bytes = lsgd::batchnorm_stats_scratch_floats(P, C, G) * sizeof(float);
+  if (cudaMallocAsync((void**)&part, bytes, s) != cudaSuccess) {
+    cudaGetLastError();
+    return fail(nullptr, LSGD_ENOMEM, "lsgd_batchnorm_stats: scratch allocation failed");
+  }
+  cudaError_t e = lsgd::launch_batchnorm_stats(y, P, C, G, mean, rstd, part, s);
+  cudaFreeAsync(part, s);
+  if (e != cudaSuccess) return fail_cuda(nullptr, e, "lsgd_batchnorm_stats");
+  return LSGD_OK;
+}
+
 lsgd_status lsgd_sample_indices(int32_t* dst, uint64_t seed, int64_t step, int K, int B, int64_t N,
                                 void* stream) {
   if (!dst || K < 1 || B < 1 || N < K) return fail(nullptr, LSGD_EINVAL, "lsgd_sample_indices: bad arguments");

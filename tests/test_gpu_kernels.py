@@ -115,3 +115,22 @@ def test_bad_arguments_are_rejected(P, torch):
     assert e.value.status == P.EINVAL
     with pytest.raises(P.LsgdError):
         P.lsgd_sgd_update(W, None, W, None, 6, 0.1, 0.9)  # momentum without a buffer
+
+
+@pytest.mark.parametrize("G,n,C", [(16, 131072, 16), (3, 1000, 64), (2, 2049, 3), (1, 1, 8)])
+def test_batchnorm_stats(P, torch, G, n, C):
+    # mean and biased variance over the positions of each replica (numpy fp64 as the definition);
+    # an offset mean tests the two-pass / pairwise-combination variance
+    gen = torch.Generator(device="cuda").manual_seed(G * 7 + C)
+    y = torch.randn((G, n, C), device="cuda", generator=gen) * 2.0 + 5.0
+    mean = torch.empty((G, C), device="cuda")
+    rstd = torch.empty((G, C), device="cuda")
+    P.lsgd_batchnorm_stats(y, n, C, G, mean, rstd)
+    torch.cuda.synchronize()
+    yn = y.double().cpu().numpy()
+    m = yn.mean(axis=1)
+    r = 1.0 / np.sqrt(yn.var(axis=1) + 1e-5)
+    np.testing.assert_allclose(mean.cpu().numpy(), m, rtol=1e-5, atol=1e-5)
+    np.testing.assert_allclose(rstd.cpu().numpy(), r, rtol=1e-4)
+    with pytest.raises(P.LsgdError):
+        P.lsgd_batchnorm_stats(y, n, 300, G, mean, rstd)

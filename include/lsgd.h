@@ -242,6 +242,21 @@ lsgd_status lsgd_grouped_gemm_bf16(const uint16_t* A, int a_mn, const uint16_t* 
 lsgd_status lsgd_batchnorm_stats(const float* y, int64_t P, int C, int G, float* mean, float* rstd,
                                  void* stream);
 
+/* lsgd_batchnorm_stats for callers that cannot allocate device memory during a run: a program
+ * whose device memory is all handed to its own caching pool (an allocation would fail, or force
+ * the pool to give memory back and stall), or a latency-critical loop that fixes its memory use at
+ * start-up.  No counterpart in the paper: the method never allocates.  Same arguments and results
+ * as lsgd_batchnorm_stats; the chunk partials go to a fixed 4 MiB array in the library's device
+ * image (2^20 floats, kept on every GPU that loads the library until the process exits), so
+ * G x ceil(P / 1024) x C x 2 must not exceed 1048576 (LSGD_EINVAL with a message otherwise).
+ * No cudaMalloc / cudaFree / allocating call of any kind.  The first call on a device looks up
+ * the array's device address with that device current (make that first call before any stream
+ * capture).  All calls share the array: calls that may overlap on the GPU (other streams, other
+ * host threads) race and must be ordered by the caller.  Nothing needs clearing between calls:
+ * each call overwrites every partial it reads. */
+lsgd_status lsgd_batchnorm_stats_noalloc(const float* y, int64_t P, int C, int G, float* mean,
+                                         float* rstd, void* stream);
+
 /* Worker mini-batch indices for one step into dst [K][B] int32 (device), as lsgd_local_step. */
 lsgd_status lsgd_sample_indices(int32_t* dst, uint64_t seed, int64_t step, int K, int B, int64_t N,
                                 void* stream);

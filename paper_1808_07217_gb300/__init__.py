@@ -35,6 +35,7 @@ EXPORTS = [
     "lsgd_sync_count", "lsgd_total_steps", "lsgd_lr_at", "lsgd_kernel_launches", "lsgd_last_error",
     "lsgd_kway_average", "lsgd_sgd_update", "lsgd_sample_indices", "lsgd_profile_enable",
     "lsgd_profile_read", "lsgd_grouped_gemm_bf16", "lsgd_batchnorm_stats",
+    "lsgd_batchnorm_stats_noalloc",
 ]
 PHASES = ["input", "forward", "loss", "backward", "update", "average"]
 
@@ -154,6 +155,7 @@ def lib():
             "lsgd_sample_indices": ([vp, ctypes.c_uint64, i64, ctypes.c_int, ctypes.c_int, i64, vp], st),
             "lsgd_profile_enable": ([vp, ctypes.c_int], st),
             "lsgd_batchnorm_stats": ([vp, i64, ctypes.c_int, ctypes.c_int, vp, vp, vp], st),
+            "lsgd_batchnorm_stats_noalloc": ([vp, i64, ctypes.c_int, ctypes.c_int, vp, vp, vp], st),
             "lsgd_grouped_gemm_bf16": ([vp, ctypes.c_int, vp, ctypes.c_int, vp, ctypes.c_int,
                                         ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int, vp], st),
             "lsgd_profile_read": ([vp, P(Profile)], st),
@@ -414,3 +416,12 @@ def lsgd_batchnorm_stats(y, P: int, C: int, G: int, mean, rstd, stream=None):
     stream = _current_stream() if stream is None else stream
     _check(lib().lsgd_batchnorm_stats(_ptr(y), int(P), int(C), int(G), _ptr(mean), _ptr(rstd),
                                       ctypes.c_void_p(stream)))
+
+
+def lsgd_batchnorm_stats_noalloc(y, P: int, C: int, G: int, mean, rstd, stream=None):
+    """lsgd_batchnorm_stats without any device allocation (fixed 4 MiB scratch inside the library),
+    for callers whose device memory is all spoken for; see include/lsgd.h for the limit and the
+    shared-scratch rules."""
+    stream = _current_stream() if stream is None else stream
+    _check(lib().lsgd_batchnorm_stats_noalloc(_ptr(y), int(P), int(C), int(G), _ptr(mean),
+                                              _ptr(rstd), ctypes.c_void_p(stream)))

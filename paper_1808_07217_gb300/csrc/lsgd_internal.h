@@ -5,7 +5,12 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <string>
+
 namespace lsgd {
+
+// Record the message lsgd_last_error(NULL) returns on this thread.
+void set_last_error(const std::string& msg);
 
 // Parameters of the fused local update (arrays indexed like the GEMM output C).
 struct SgdParams {

@@ -38,6 +38,10 @@ struct DenseLayer {
 
 }  // namespace
 
+namespace lsgd {
+void set_last_error(const std::string& msg) { g_last_error = msg; }
+}  // namespace lsgd
+
 struct lsgd_ctx {
   lsgd_config cfg;
   lsgd_allocator alloc{};

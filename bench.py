@@ -40,9 +40,10 @@ WORKLOAD = dict(name="mlp_3072-1024-1024-10_K16_B128_H16_bf16", widths=(3072, 10
 UPDATE_BYTES_PER_PARAM = 22
 FUSED_UPDATE_BYTES_PER_PARAM = 18
 AVERAGE_BYTES_PER_PARAM = 10
-# DRAM bytes per step of the fused weight-gradient + update launches from the ncu capture
-# summarised in profiles/ (None until captured for the current kernel).
-UPDATE_TRAFFIC_PER_STEP = None
+# DRAM bytes (read + write) per step of the three fused weight-gradient + update launches, from
+# the ncu capture summarised in profiles/step_kernels_mlp3072_K16_B128.md (below the algorithmic
+# bytes because part of each launch's writes is still in L2 when the launch ends).
+UPDATE_TRAFFIC_PER_STEP = 1116399104
 
 FALLBACK_HBM_GBS = 6800.0
 FALLBACK_BF16_TFLOPS = 1900.0
@@ -113,13 +114,13 @@ class ClockSampler:
                 "reasons": reasons, "samples": len(rows)}
 
 
-def _make_cfg(P, total_steps):
+def _make_cfg(P, total_steps, fused=True, K=None):
     w = WORKLOAD
-    return P.make_config(K=w["K"], B_loc=w["B"], H=w["H"], total_steps=total_steps, N=w["N"],
+    return P.make_config(K=K or w["K"], B_loc=w["B"], H=w["H"], total_steps=total_steps, N=w["N"],
                          widths=w["widths"], base_lr=w["base_lr"], scale_by_K=w["scale_by_K"],
                          warmup_epochs=w["warmup_epochs"], momentum=w["momentum"],
                          nesterov=w["nesterov"], weight_decay=w["weight_decay"], seed=w["seed"],
-                         precision=P.BF16, fused_update=True)
+                         precision=P.BF16, fused_update=fused)
 
 
 def _oracle_cfg(oracle, total_steps):
@@ -239,7 +240,7 @@ def run_resnet(args):
 
     torch.cuda.set_device(0)
     w = RESNET_WORKLOAD
-    K, B = w["K"], w["B"]
+    K, B = args.replicas or w["K"], w["B"]
     X, y = synthdata.gaussian_mixture_cached(w["N"], 3072, w["C"], w["data_seed"])
     W_, S_ = max(3, args.warmup), args.steps
     total = W_ + S_
@@ -282,6 +283,11 @@ def main():
                     help="K x H sync / compute sweep of the MLP 3072-512-512-10 workload")
     ap.add_argument("--resnet", action="store_true",
                     help="post-local ResNet-20 workload (K = 16, B_loc = 128) instead of the MLP")
+    ap.add_argument("--unfused", action="store_true",
+                    help="apply the update with the stand-alone kernel over the whole K x d buffer "
+                         "instead of the weight-gradient epilogue (same arithmetic)")
+    ap.add_argument("--replicas", type=int, default=0,
+                    help="override K (smaller cases for profiler captures); 0 = the workload's K")
     args = ap.parse_args()
     world, rank, local = _dist()
     if args.sweep:
@@ -313,13 +319,14 @@ def main():
     import paper_1808_07217_gb300 as P
 
     w = WORKLOAD
-    K, B, H = w["K"], w["B"], w["H"]
+    K, B, H = args.replicas or w["K"], w["B"], w["H"]
+    fused = not args.unfused
     X, y = synthdata.gaussian_mixture_cached(w["N"], w["widths"][0], w["C"], w["data_seed"])
     W_, S_ = max(3, args.warmup), args.steps
     e2e_warm = 2
     total = W_ + S_ + e2e_warm + S_
     stream = torch.cuda.current_stream()
-    ctx = P.lsgd_create(_make_cfg(P, total), stream=stream.cuda_stream)
+    ctx = P.lsgd_create(_make_cfg(P, total, fused, K), stream=stream.cuda_stream)
     P.lsgd_set_dataset(ctx, X, y)
     d = P.lsgd_num_params(ctx)
 
@@ -398,8 +405,11 @@ def main():
     widths = w["widths"]
     # The update phase is the three fused weight-gradient + update launches of each step; the
     # roofline unit is one step's worth of them (bytes summed over the layers).
-    upd_bytes = sum(FUSED_UPDATE_BYTES_PER_PARAM * K * widths[l] * widths[l + 1]
-                    + 2 * K * B * (widths[l] + widths[l + 1]) for l in range(len(widths) - 1))
+    if fused:
+        upd_bytes = sum(FUSED_UPDATE_BYTES_PER_PARAM * K * widths[l] * widths[l + 1]
+                        + 2 * K * B * (widths[l] + widths[l + 1]) for l in range(len(widths) - 1))
+    else:
+        upd_bytes = UPDATE_BYTES_PER_PARAM * K * d
     upd_gbs = upd_bytes / (upd_ms / S_ / 1000.0) / 1e9
     avg_gbs = (AVERAGE_BYTES_PER_PARAM * K * d / (avg_ms / avg_n / 1000.0) / 1e9) if avg_n else None
     gemm_flops = 0
@@ -424,18 +434,21 @@ def main():
         "value": value, "unit": "samples/s", "n_gpus": world, "steps": S_, "warmup": W_,
         "ms_per_step": t_ms / S_, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": {"workload": w["name"], "global_batch": K * B, "K": K, "B_loc": B, "H": H,
+        "config": {"workload": w["name"] if K == w["K"] else w["name"].replace("K16", f"K{K}"),
+                   "global_batch": K * B, "K": K, "B_loc": B, "H": H, "fused_update": fused,
                    "params_per_replica": d, "parallelism": "replicas" if world > 1 else "single",
                    "l2": "per-step working set (w, u, g, shadow: 1.0 GB) exceeds the 129 MB L2",
                    "syncs_in_timed_region": n_syncs},
         "e2e": {"value": e2e_value, "unit": "samples/s", "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h},
         "gpu_launches": launches,
-        "roofline": {"kernel": "gemm_tc_kernel weight gradient + fused local update",
+        "roofline": {"kernel": ("gemm_tc_kernel weight gradient + fused local update" if fused
+                                else "sgd_update_kernel"),
                      "bound": "hbm", "achieved": upd_gbs, "peak": hbm, "unit": "GB/s",
                      "frac": upd_gbs / hbm, "peak_source": f"{peak_src} hbm_gbs",
-                     "traffic": UPDATE_TRAFFIC_PER_STEP,
-                     "unit_of_work": "one step's weight-gradient + update launches (3 layers)",
+                     "traffic": UPDATE_TRAFFIC_PER_STEP if fused and K == w["K"] else None,
+                     "unit_of_work": ("one step's weight-gradient + update launches (3 layers)"
+                                      if fused else "one launch over the whole K x d buffer"),
                      "algorithmic_bytes": upd_bytes, "launches_per_unit": upd_n // S_},
         "sync_average": {"gbs": avg_gbs, "frac_of_hbm": (avg_gbs / hbm) if avg_gbs else None,
                          "ms_per_sync": (avg_ms / avg_n) if avg_n else None},

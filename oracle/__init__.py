@@ -62,13 +62,16 @@ class Cfg(ctypes.Structure):
         ("n_classes", ctypes.c_int),
         ("base_ch", ctypes.c_int),
         ("res_blocks", ctypes.c_int),
+        ("hier_block", ctypes.c_int),
+        ("hier_rounds", ctypes.c_int),
     ]
 
 
 def make_cfg(kind=DENSE, widths=(3072, 10), has_bias=True, bf16=False, K=1, B=1, H=1,
              t_switch=-1, T=1, N=1, base_lr=0.1, scale_by_K=False, warmup_epochs=0.0,
              milestones=(), decay=0.1, momentum=0.0, nesterov=False, weight_decay=0.0, seed=0,
-             in_hwc=(32, 32, 3), n_classes=10, base_ch=16, res_blocks=3) -> Cfg:
+             in_hwc=(32, 32, 3), n_classes=10, base_ch=16, res_blocks=3, hier_block=0,
+             hier_rounds=1) -> Cfg:
     c = Cfg()
     c.kind = kind
     if kind != RESNET20:
@@ -94,6 +97,8 @@ def make_cfg(kind=DENSE, widths=(3072, 10), has_bias=True, bf16=False, K=1, B=1,
     c.n_classes = int(n_classes)
     c.base_ch = int(base_ch)
     c.res_blocks = int(res_blocks)
+    c.hier_block = int(hier_block)
+    c.hier_rounds = int(hier_rounds)
     return c
 
 
@@ -136,6 +141,12 @@ def lib():
             L.oracle_is_round_end.argtypes = [cfgp, ctypes.c_int64]
             L.oracle_is_round_end.restype = ctypes.c_int
             L.oracle_average.argtypes = [ctypes.c_int, ctypes.c_int64, dp]
+            L.oracle_block_average.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_int64, dp]
+            L.oracle_sync_kind.argtypes = [cfgp, ctypes.c_int64]
+            L.oracle_sync_kind.restype = ctypes.c_int
+            L.oracle_run_counted.argtypes = [cfgp, fp, ip, fp, dp, dp, ctypes.c_int64,
+                                             ctypes.c_int64, dp, P(ctypes.c_int64),
+                                             P(ctypes.c_int64)]
             L.oracle_run.argtypes = [cfgp, fp, ip, fp, dp, dp, ctypes.c_int64, ctypes.c_int64, dp,
                                      P(ctypes.c_int64)]
             L.oracle_run_minibatch.argtypes = [cfgp, fp, ip, fp, dp, dp, ctypes.c_int64,
@@ -224,6 +235,36 @@ def average(W) -> np.ndarray:
     K, d = W.shape
     lib().oracle_average(int(K), int(d), _p(W, ctypes.c_double))
     return W
+
+
+def sync_kind(c: Cfg, s: int) -> int:
+    """0 = no average after step s, 1 = block average, 2 = global average."""
+    return int(lib().oracle_sync_kind(ctypes.byref(c), int(s)))
+
+
+def block_average(W, block: int) -> np.ndarray:
+    W = np.array(W, dtype=np.float64)
+    K, d = W.shape
+    lib().oracle_block_average(int(K), int(block), int(d), _p(W, ctypes.c_double))
+    return W
+
+
+def run_counted(c: Cfg, X, y=None, t=None, W=None, U=None, s0=0, n_steps=None):
+    """run() that also returns the number of block averages: W, U, losses, n_global, n_block."""
+    d = num_params(c)
+    if W is None:
+        W = np.tile(init_params(c), (c.K, 1))
+    W = np.array(W, dtype=np.float64).reshape(c.K, d)
+    U = np.zeros_like(W) if U is None else np.array(U, dtype=np.float64).reshape(c.K, d)
+    n = int(c.T - s0 if n_steps is None else n_steps)
+    losses = np.zeros((n, c.K), dtype=np.float64)
+    ng, nb = ctypes.c_int64(0), ctypes.c_int64(0)
+    X, y, t = _f32(X), _i32(y), _f32(t)
+    lib().oracle_run_counted(ctypes.byref(c), _p(X, ctypes.c_float), _p(y, ctypes.c_int32),
+                             _p(t, ctypes.c_float), _p(W, ctypes.c_double), _p(U, ctypes.c_double),
+                             int(s0), n, _p(losses, ctypes.c_double), ctypes.byref(ng),
+                             ctypes.byref(nb))
+    return W, U, losses, int(ng.value), int(nb.value)
 
 
 def run(c: Cfg, X, y=None, t=None, W=None, U=None, s0=0, n_steps=None):

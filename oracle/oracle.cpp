@@ -304,6 +304,25 @@ int oracle_is_round_end(const oracle_cfg* c, int64_t s) {
   return ((s + 1 - start) % c->H) == 0;
 }
 
+// Which average ends local step s.  Without hierarchy: the global average at every round end.
+// Hierarchical local SGD (Sec. D, the equations of the hierarchical scheme): the r-th round end
+// after the switch averages within each block of hier_block workers, and every hier_rounds-th
+// round end (r a multiple of H^b) averages all K workers; the mini-batch phase (s < t') and the
+// last step of the run use the global average.
+int oracle_sync_kind(const oracle_cfg* c, int64_t s) {
+  if (!oracle_is_round_end(c, s)) return ORACLE_SYNC_NONE;
+  if (c->hier_block <= 0 || s == c->T - 1) return ORACLE_SYNC_GLOBAL;
+  if (c->t_switch >= 0 && s < c->t_switch) return ORACLE_SYNC_GLOBAL;
+  const int64_t start = c->t_switch > 0 ? c->t_switch : 0;
+  const int64_t r = (s + 1 - start) / c->H;
+  return (r % c->hier_rounds == 0) ? ORACLE_SYNC_GLOBAL : ORACLE_SYNC_BLOCK;
+}
+
+// Block average: w^k := (1/K') sum over the K' workers of k's block (Sec. D).
+void oracle_block_average(int K, int block, int64_t d, double* W) {
+  for (int b0 = 0; b0 < K; b0 += block) oracle_average(block, d, W + (int64_t)b0 * d);
+}
+
 // Eq. 2, right part: w^k := (1/K) sum_k w^k for every worker k.
 void oracle_average(int K, int64_t d, double* W) {
   for (int64_t i = 0; i < d; ++i) {
@@ -316,12 +335,13 @@ void oracle_average(int K, int64_t d, double* W) {
 
 // Local / post-local SGD (Eq. 2; Algorithms 1 and 2) from global step s0 for n_steps steps.
 // W and U hold the K workers' models and momentum buffers, worker-major, and are updated in place.
-void oracle_run(const oracle_cfg* c, const float* X, const int32_t* y, const float* t, double* W,
-                double* U, int64_t s0, int64_t n_steps, double* losses, int64_t* n_syncs) {
+void oracle_run_counted(const oracle_cfg* c, const float* X, const int32_t* y, const float* t,
+                        double* W, double* U, int64_t s0, int64_t n_steps, double* losses,
+                        int64_t* n_global, int64_t* n_block) {
   const int64_t d = oracle_num_params(c);
   std::vector<int32_t> idx((size_t)c->B);
   std::vector<double> g((size_t)d);
-  int64_t syncs = 0;
+  int64_t syncs = 0, blocks = 0;
   for (int64_t s = s0; s < s0 + n_steps; ++s) {
     const double lr = oracle_lr(c, s);
     for (int k = 0; k < c->K; ++k) {
@@ -330,12 +350,22 @@ void oracle_run(const oracle_cfg* c, const float* X, const int32_t* y, const flo
       oracle_sgd_update(c, lr, W + (int64_t)k * d, U + (int64_t)k * d, g.data());
       if (losses) losses[(s - s0) * c->K + k] = l;
     }
-    if (oracle_is_round_end(c, s)) {
+    const int kind = oracle_sync_kind(c, s);
+    if (kind == ORACLE_SYNC_GLOBAL) {
       oracle_average(c->K, d, W);
       ++syncs;
+    } else if (kind == ORACLE_SYNC_BLOCK) {
+      oracle_block_average(c->K, c->hier_block, d, W);
+      ++blocks;
     }
   }
-  if (n_syncs) *n_syncs = syncs;
+  if (n_global) *n_global = syncs;
+  if (n_block) *n_block = blocks;
+}
+
+void oracle_run(const oracle_cfg* c, const float* X, const int32_t* y, const float* t, double* W,
+                double* U, int64_t s0, int64_t n_steps, double* losses, int64_t* n_syncs) {
+  oracle_run_counted(c, X, y, t, W, U, s0, n_steps, losses, n_syncs, nullptr);
 }
 
 // Mini-batch SGD (Eq. 1) on a single model: each step averages the K workers' local mini-batch

@@ -45,7 +45,12 @@ typedef struct {
   uint64_t seed;
   /* ResNet-20 geometry (kind == ORACLE_RESNET20) */
   int in_h, in_w, in_c, n_classes, base_ch, res_blocks; /* res_blocks: basic blocks per stage */
+  /* hierarchical local SGD (Sec. D): blocks of hier_block consecutive workers average after every
+     H-step round, all K workers after every hier_rounds-th round (hier_block = 0: off) */
+  int hier_block, hier_rounds;
 } oracle_cfg;
+
+enum { ORACLE_SYNC_NONE = 0, ORACLE_SYNC_BLOCK = 1, ORACLE_SYNC_GLOBAL = 2 };
 
 int64_t oracle_num_params(const oracle_cfg* c);
 void oracle_weight_decay_mask(const oracle_cfg* c, uint8_t* mask);
@@ -57,9 +62,15 @@ double oracle_loss_grad(const oracle_cfg* c, const double* w, const float* X, co
 void oracle_sgd_update(const oracle_cfg* c, double lr, double* w, double* u, const double* g);
 double oracle_lr(const oracle_cfg* c, int64_t s);
 int oracle_is_round_end(const oracle_cfg* c, int64_t s);
+int oracle_sync_kind(const oracle_cfg* c, int64_t s);
 void oracle_average(int K, int64_t d, double* W);
+void oracle_block_average(int K, int block, int64_t d, double* W);
 void oracle_run(const oracle_cfg* c, const float* X, const int32_t* y, const float* t, double* W,
                 double* U, int64_t s0, int64_t n_steps, double* losses, int64_t* n_syncs);
+/* As oracle_run, also counting the block averages of hierarchical local SGD. */
+void oracle_run_counted(const oracle_cfg* c, const float* X, const int32_t* y, const float* t,
+                        double* W, double* U, int64_t s0, int64_t n_steps, double* losses,
+                        int64_t* n_global, int64_t* n_block);
 void oracle_run_minibatch(const oracle_cfg* c, const float* X, const int32_t* y, const float* t,
                           double* w, double* u, int64_t s0, int64_t n_steps, double* losses);
 double oracle_eval_loss(const oracle_cfg* c, const double* w, const float* X, const int32_t* y,

@@ -294,3 +294,45 @@ def test_init_statistics():
     assert np.all(oracle.init_params(c, oracle.INIT_ZERO) == 0)
     # fp32-representable (the accelerated path stores fp32 master weights)
     assert np.array_equal(w, w.astype(np.float32).astype(np.float64))
+
+
+# ---- hierarchical local SGD (Sec. D) ----
+
+def test_hierarchical_with_one_block_is_local_sgd():
+    # K' = K: every block average is the global average, so the run equals plain local SGD.
+    X, y = _data(48, 12, 5, 11)
+    c_h = _mlp_cfg(H=2, T=12, hier_block=4, hier_rounds=3, momentum=0.9, nesterov=True)
+    c_l = _mlp_cfg(H=2, T=12, momentum=0.9, nesterov=True)
+    Wh, _, lh, ng, nb = oracle.run_counted(c_h, X, y=y)
+    Wl, _, ll, _ = oracle.run(c_l, X, y=y)
+    assert np.array_equal(Wh, Wl) and np.array_equal(lh, ll)
+    assert (ng, nb) == (2, 4)
+
+
+def test_hierarchical_with_singleton_blocks_is_local_sgd_with_longer_rounds():
+    # K' = 1: a block average leaves every worker unchanged, so hierarchical (H, H^b) equals local
+    # SGD with rounds of H H^b steps.
+    X, y = _data(48, 12, 5, 12)
+    c_h = _mlp_cfg(H=2, T=12, hier_block=1, hier_rounds=3)
+    c_l = _mlp_cfg(H=6, T=12)
+    Wh, _, _, ng, nb = oracle.run_counted(c_h, X, y=y)
+    Wl, _, _, nl = oracle.run(c_l, X, y=y)
+    assert np.array_equal(Wh, Wl) and ng == nl == 2 and nb == 4
+
+
+def test_block_average_is_blockwise_mean():
+    rng = np.random.default_rng(2)
+    W = rng.standard_normal((6, 9))
+    A = oracle.block_average(W, 3)
+    np.testing.assert_allclose(A[:3], np.tile(W[:3].mean(0), (3, 1)), rtol=1e-15, atol=1e-15)
+    np.testing.assert_allclose(A[3:], np.tile(W[3:].mean(0), (3, 1)), rtol=1e-15, atol=1e-15)
+
+
+@pytest.mark.parametrize("T,H,Hb", [(64, 4, 4), (96, 2, 8), (48, 16, 3)])
+def test_hierarchical_sync_counts_match_communication_model(T, H, Hb):
+    # Sec. F: with T a multiple of H H^b there are T/(H H^b) global and T/H - T/(H H^b) block
+    # averages (the two terms of the hierarchical communication cost).
+    c = oracle.make_cfg(K=4, B=1, H=H, T=T, hier_block=2, hier_rounds=Hb)
+    kinds = [oracle.sync_kind(c, s) for s in range(T)]
+    assert kinds.count(2) == T // (H * Hb)
+    assert kinds.count(1) == T // H - T // (H * Hb)

@@ -103,6 +103,11 @@ typedef struct {
                             bias-gradient sum) apply the local update directly, so the gradient is
                             never written to memory; bit-identical to 0, which runs the stand-alone
                             update kernel over the whole K x d buffer.  Ignored elsewhere. */
+  int hier_block;        /* hierarchical local SGD (Sec. D): > 0 = after every H-step round the
+                            hier_block consecutive replicas of each block are averaged, and every
+                            hier_rounds-th round (and the run's last step) all K; must divide K.
+                            0 = off.  The mini-batch phase of post-local SGD averages globally. */
+  int hier_rounds;       /* H^b >= 1 */
 } lsgd_config;
 
 typedef struct lsgd_ctx lsgd_ctx;
@@ -141,8 +146,14 @@ lsgd_status lsgd_local_step_batch(lsgd_ctx* ctx, const float* x, const void* lab
  * Refreshes the bf16 shadow. */
 lsgd_status lsgd_sync_average(lsgd_ctx* ctx);
 
+/* Block average of hierarchical local SGD (Sec. D): every replica becomes the mean of the
+ * hier_block replicas of its block.  LSGD_ESTATE if the context has no blocks. */
+lsgd_status lsgd_block_average(lsgd_ctx* ctx);
+
 /* n_steps local steps from the current step counter, averaging after every step s that ends a
- * round: s < t' (post-local first phase), (s + 1 - max(t', 0)) mod H == 0, or s == T - 1. */
+ * round: s < t' (post-local first phase), (s + 1 - max(t', 0)) mod H == 0, or s == T - 1.  With
+ * hier_block > 0 the r-th round end after the switch is a block average unless r is a multiple
+ * of hier_rounds (or s == T - 1). */
 lsgd_status lsgd_run(lsgd_ctx* ctx, int64_t n_steps);
 
 /* Replica k's fp32 parameters (k = -1: the element-wise mean over replicas, computed in fp64 on
@@ -174,7 +185,8 @@ lsgd_status lsgd_load(lsgd_ctx* ctx, const char* path);
 
 int64_t lsgd_num_params(const lsgd_ctx* ctx);   /* d, canonical (unpadded) */
 int64_t lsgd_step_count(const lsgd_ctx* ctx);   /* local steps taken so far (next step's s) */
-int64_t lsgd_sync_count(const lsgd_ctx* ctx);   /* averages performed so far */
+int64_t lsgd_sync_count(const lsgd_ctx* ctx);   /* global averages performed so far */
+int64_t lsgd_block_sync_count(const lsgd_ctx* ctx); /* block averages performed so far */
 int64_t lsgd_total_steps(const lsgd_ctx* ctx);  /* T */
 double lsgd_lr_at(const lsgd_ctx* ctx, int64_t step); /* gamma(s) as used by the update */
 /* Kernel launches issued by this context since creation (for launch accounting). */

@@ -35,7 +35,7 @@ EXPORTS = [
     "lsgd_sync_count", "lsgd_total_steps", "lsgd_lr_at", "lsgd_kernel_launches", "lsgd_last_error",
     "lsgd_kway_average", "lsgd_sgd_update", "lsgd_sample_indices", "lsgd_profile_enable",
     "lsgd_profile_read", "lsgd_grouped_gemm_bf16", "lsgd_batchnorm_stats",
-    "lsgd_batchnorm_stats_noalloc",
+    "lsgd_batchnorm_stats_noalloc", "lsgd_block_average", "lsgd_block_sync_count",
 ]
 PHASES = ["input", "forward", "loss", "backward", "update", "average"]
 
@@ -77,14 +77,15 @@ class Config(ctypes.Structure):
                 ("epochs", ctypes.c_double), ("N", ctypes.c_int64), ("model", Model),
                 ("lr", LrSchedule), ("momentum", ctypes.c_double), ("nesterov", ctypes.c_int),
                 ("weight_decay", ctypes.c_double), ("seed", ctypes.c_uint64),
-                ("precision", ctypes.c_int), ("fused_update", ctypes.c_int)]
+                ("precision", ctypes.c_int), ("fused_update", ctypes.c_int),
+                ("hier_block", ctypes.c_int), ("hier_rounds", ctypes.c_int)]
 
 
 def make_config(K=1, B_loc=1, H=1, t_switch=-1, total_steps=0, epochs=0.0, N=1, kind=MLP,
                 widths=(3072, 10), init=INIT_HE, in_hwc=(32, 32, 3), n_classes=10, base_ch=16,
                 res_blocks=3, base_lr=0.1, scale_by_K=False, warmup_epochs=0.0, milestones=(),
                 decay=0.1, momentum=0.0, nesterov=False, weight_decay=0.0, seed=0,
-                precision=FP32, fused_update=False) -> Config:
+                precision=FP32, fused_update=False, hier_block=0, hier_rounds=1) -> Config:
     c = Config()
     c.K, c.B_loc, c.H = int(K), int(B_loc), int(H)
     c.t_switch, c.total_steps, c.epochs, c.N = int(t_switch), int(total_steps), float(epochs), int(N)
@@ -107,6 +108,7 @@ def make_config(K=1, B_loc=1, H=1, t_switch=-1, total_steps=0, epochs=0.0, N=1, 
     c.seed = int(seed)
     c.precision = int(precision)
     c.fused_update = int(bool(fused_update))
+    c.hier_block, c.hier_rounds = int(hier_block), int(hier_rounds)
     return c
 
 
@@ -145,6 +147,8 @@ def lib():
             "lsgd_num_params": ([vp], i64),
             "lsgd_step_count": ([vp], i64),
             "lsgd_sync_count": ([vp], i64),
+            "lsgd_block_sync_count": ([vp], i64),
+            "lsgd_block_average": ([vp], st),
             "lsgd_total_steps": ([vp], i64),
             "lsgd_lr_at": ([vp, i64], ctypes.c_double),
             "lsgd_kernel_launches": ([vp], i64),
@@ -352,6 +356,14 @@ def lsgd_step_count(ctx: Ctx) -> int:
 
 def lsgd_sync_count(ctx: Ctx) -> int:
     return int(lib().lsgd_sync_count(ctx.handle))
+
+
+def lsgd_block_sync_count(ctx: Ctx) -> int:
+    return int(lib().lsgd_block_sync_count(ctx.handle))
+
+
+def lsgd_block_average(ctx: Ctx):
+    _check(lib().lsgd_block_average(ctx.handle), ctx)
 
 
 def lsgd_total_steps(ctx: Ctx) -> int:

@@ -236,6 +236,9 @@ template <bool SHADOW>
 __global__ void __launch_bounds__(256) kway_average_kernel(float4* __restrict__ W,
                                                            uint2* __restrict__ Wb, int K,
                                                            int64_t d4) {
+  // blockIdx.y selects a group of K consecutive replicas (one group for the global average)
+  W += (int64_t)blockIdx.y * K * d4;
+  if (SHADOW) Wb += (int64_t)blockIdx.y * K * d4;
   const int lane = threadIdx.x & 31;
   const int r = lane >> 3, c = lane & 7;
   const int64_t nblk = (d4 + 7) / 8;
@@ -463,18 +466,24 @@ cudaError_t launch_sgd_update(float* w, float* u, const float* g, uint16_t* wb, 
 }
 
 cudaError_t launch_kway_average(float* W, uint16_t* Wb, int K, int64_t d, cudaStream_t stream) {
-  if (K < 1 || d <= 0) return cudaSuccess;
-  if (d & 3) return cudaErrorInvalidValue;
+  return launch_group_average(W, Wb, K, 1, d, stream);
+}
+
+cudaError_t launch_group_average(float* W, uint16_t* Wb, int Kp, int groups, int64_t d,
+                                 cudaStream_t stream) {
+  if (Kp < 1 || groups < 1 || d <= 0) return cudaSuccess;
+  if ((d & 3) || groups > 65535) return cudaErrorInvalidValue;
   const int64_t d4 = d / 4;
   const int64_t nblk = (d4 + 7) / 8;  // one warp per 128-byte column block
   const int threads = 256;
-  const int blocks = grid_for(nblk * 32, threads, 8);
+  const int blocks = std::max(1, grid_for(nblk * 32, threads, 8) / groups);
+  dim3 grid(blocks, groups);
   if (Wb)
-    kway_average_kernel<true><<<blocks, threads, 0, stream>>>(reinterpret_cast<float4*>(W),
-                                                              reinterpret_cast<uint2*>(Wb), K, d4);
+    kway_average_kernel<true><<<grid, threads, 0, stream>>>(reinterpret_cast<float4*>(W),
+                                                            reinterpret_cast<uint2*>(Wb), Kp, d4);
   else
-    kway_average_kernel<false><<<blocks, threads, 0, stream>>>(reinterpret_cast<float4*>(W), nullptr,
-                                                               K, d4);
+    kway_average_kernel<false><<<grid, threads, 0, stream>>>(reinterpret_cast<float4*>(W), nullptr,
+                                                             Kp, d4);
   return cudaGetLastError();
 }
 

@@ -50,6 +50,9 @@ cudaError_t launch_sgd_update(float* w, float* u, const float* g, uint16_t* wb, 
                               float momentum, int nesterov, float weight_decay, int64_t period,
                               int64_t decay_end, cudaStream_t stream);
 cudaError_t launch_kway_average(float* W, uint16_t* Wb, int K, int64_t d, cudaStream_t stream);
+// Average within each of `groups` groups of Kp consecutive replicas (replica stride d).
+cudaError_t launch_group_average(float* W, uint16_t* Wb, int Kp, int groups, int64_t d,
+                                 cudaStream_t stream);
 cudaError_t launch_init_normal(float* w, int64_t n, double stddev, uint64_t seed, uint32_t tensor_id,
                                cudaStream_t stream);
 cudaError_t launch_fill(float* w, int64_t n, float v, cudaStream_t stream);

@@ -76,7 +76,7 @@ struct lsgd_ctx {
   int64_t loss_cap = 0;
   float* row_loss = nullptr;  // [K][B] scratch for evaluation
   int* flag = nullptr;
-  int64_t step = 0, syncs = 0, launches = 0;
+  int64_t step = 0, syncs = 0, block_syncs = 0, launches = 0;
   std::string err;
   lsgd::ResNetPlan* rn = nullptr;
   // tracing (lsgd_profile_*)
@@ -181,6 +181,16 @@ bool round_end(const lsgd_config& cfg, int64_t T, int64_t s) {
   if (cfg.t_switch >= 0 && s < cfg.t_switch) return true;
   const int64_t start = cfg.t_switch > 0 ? cfg.t_switch : 0;
   return ((s + 1 - start) % cfg.H) == 0;
+}
+
+// Average ending step s: 0 none, 1 block (hierarchical), 2 global (Sec. 3 and Sec. D).
+int sync_kind(const lsgd_config& cfg, int64_t T, int64_t s) {
+  if (!round_end(cfg, T, s)) return 0;
+  if (cfg.hier_block <= 0 || s == T - 1) return 2;
+  if (cfg.t_switch >= 0 && s < cfg.t_switch) return 2;
+  const int64_t start = cfg.t_switch > 0 ? cfg.t_switch : 0;
+  const int64_t r = (s + 1 - start) / cfg.H;
+  return (r % std::max(1, cfg.hier_rounds) == 0) ? 2 : 1;
 }
 
 bool force_simt() {
@@ -590,6 +600,8 @@ lsgd_status lsgd_create(const lsgd_config* cfg, const lsgd_allocator* alloc, voi
     return fail(nullptr, LSGD_EINVAL, "precision must be LSGD_FP32 or LSGD_BF16");
   if (c0.N / c0.K * (int64_t)c0.K > 0x7fffffffLL) return fail(nullptr, LSGD_EINVAL, "N too large");
   if (c0.B_loc > 8192) return fail(nullptr, LSGD_EUNSUPPORTED, "B_loc must be <= 8192");
+  if (c0.hier_block < 0 || (c0.hier_block > 0 && (c0.K % c0.hier_block || c0.hier_rounds < 1)))
+    return fail(nullptr, LSGD_EINVAL, "hier_block must divide K and hier_rounds must be >= 1");
   const lsgd_model& m = c0.model;
   if (m.kind == LSGD_MLP || m.kind == LSGD_LSQ) {
     if (m.n_layers < 1 || m.n_layers > LSGD_MAX_LAYERS)
@@ -806,6 +818,17 @@ lsgd_status lsgd_sync_average(lsgd_ctx* c) {
   return LSGD_OK;
 }
 
+lsgd_status lsgd_block_average(lsgd_ctx* c) {
+  if (!c) return fail(nullptr, LSGD_EINVAL, "NULL context");
+  if (c->cfg.hier_block <= 0) return fail(c, LSGD_ESTATE, "the context has no averaging blocks");
+  const int64_t e0 = prof_mark(c);
+  LSGD_LAUNCH(c, lsgd::launch_group_average(c->W, c->Wb, c->cfg.hier_block,
+                                            c->cfg.K / c->cfg.hier_block, c->d_pad, c->stream));
+  prof_span(c, LSGD_PH_AVERAGE, e0, prof_mark(c));
+  c->block_syncs++;
+  return LSGD_OK;
+}
+
 lsgd_status lsgd_profile_enable(lsgd_ctx* c, int enable) {
   if (!c) return fail(nullptr, LSGD_EINVAL, "NULL context");
   LSGD_TRY_CUDA(c, cudaStreamSynchronize(c->stream));
@@ -836,8 +859,12 @@ lsgd_status lsgd_run(lsgd_ctx* c, int64_t n_steps) {
     const int64_t s = c->step;
     lsgd_status st = lsgd_local_step(c);
     if (st != LSGD_OK) return st;
-    if (round_end(c->cfg, c->T, s)) {
+    const int kind = sync_kind(c->cfg, c->T, s);
+    if (kind == 2) {
       st = lsgd_sync_average(c);
+      if (st != LSGD_OK) return st;
+    } else if (kind == 1) {
+      st = lsgd_block_average(c);
       if (st != LSGD_OK) return st;
     }
   }
@@ -998,7 +1025,7 @@ lsgd_status lsgd_check_finite(lsgd_ctx* c) {
   return LSGD_OK;
 }
 
-static const uint64_t kMagic = 0x3130545043445347ULL;  // "GSDCPT01"
+static const uint64_t kMagic = 0x3230545043445347ULL;  // "GSDCPT02"
 
 lsgd_status lsgd_save(lsgd_ctx* c, const char* path) {
   if (!c || !path) return fail(c, LSGD_EINVAL, "NULL argument");
@@ -1006,7 +1033,8 @@ lsgd_status lsgd_save(lsgd_ctx* c, const char* path) {
   std::vector<float> buf(n);
   FILE* f = std::fopen(path, "wb");
   if (!f) return fail(c, LSGD_EIO, std::string("cannot open ") + path);
-  int64_t hdr[6] = {(int64_t)kMagic, c->cfg.K, c->d_pad, c->step, c->syncs, c->U ? 1 : 0};
+  int64_t hdr[7] = {(int64_t)kMagic, c->cfg.K, c->d_pad, c->step, c->syncs, c->U ? 1 : 0,
+                    c->block_syncs};
   bool ok = std::fwrite(hdr, sizeof(hdr), 1, f) == 1;
   for (int which = 0; ok && which < (c->U ? 2 : 1); ++which) {
     const float* src = which == 0 ? c->W : c->U;
@@ -1027,7 +1055,7 @@ lsgd_status lsgd_load(lsgd_ctx* c, const char* path) {
   if (!c || !path) return fail(c, LSGD_EINVAL, "NULL argument");
   FILE* f = std::fopen(path, "rb");
   if (!f) return fail(c, LSGD_EIO, std::string("cannot open ") + path);
-  int64_t hdr[6];
+  int64_t hdr[7];
   if (std::fread(hdr, sizeof(hdr), 1, f) != 1 || hdr[0] != (int64_t)kMagic || hdr[1] != c->cfg.K ||
       hdr[2] != c->d_pad || hdr[5] != (c->U ? 1 : 0)) {
     std::fclose(f);
@@ -1053,12 +1081,14 @@ lsgd_status lsgd_load(lsgd_ctx* c, const char* path) {
   LSGD_TRY_CUDA(c, cudaStreamSynchronize(c->stream));
   c->step = hdr[3];
   c->syncs = hdr[4];
+  c->block_syncs = hdr[6];
   return LSGD_OK;
 }
 
 int64_t lsgd_num_params(const lsgd_ctx* c) { return c ? c->d : -1; }
 int64_t lsgd_step_count(const lsgd_ctx* c) { return c ? c->step : -1; }
 int64_t lsgd_sync_count(const lsgd_ctx* c) { return c ? c->syncs : -1; }
+int64_t lsgd_block_sync_count(const lsgd_ctx* c) { return c ? c->block_syncs : -1; }
 int64_t lsgd_total_steps(const lsgd_ctx* c) { return c ? c->T : -1; }
 double lsgd_lr_at(const lsgd_ctx* c, int64_t s) { return c ? lr_at(c->cfg, c->T, s) : 0.0; }
 int64_t lsgd_kernel_launches(const lsgd_ctx* c) { return c ? c->launches : -1; }

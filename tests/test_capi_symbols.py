@@ -54,6 +54,7 @@ def test_struct_layout_matches_header(P):
              offsetof(lsgd_config, lr), offsetof(lsgd_config, momentum),
              offsetof(lsgd_config, seed), offsetof(lsgd_config, precision),
              offsetof(lsgd_config, fused_update), sizeof(lsgd_profile));
+      printf("%zu %zu\n", offsetof(lsgd_config, hier_block), offsetof(lsgd_config, hier_rounds));
       return 0;
     }
     """
@@ -68,7 +69,8 @@ def test_struct_layout_matches_header(P):
     C = P.Config
     want = [ctypes.sizeof(C), ctypes.sizeof(P.Model), ctypes.sizeof(P.LrSchedule),
             ctypes.sizeof(P.Allocator), C.model.offset, C.lr.offset, C.momentum.offset,
-            C.seed.offset, C.precision.offset, C.fused_update.offset, ctypes.sizeof(P.Profile)]
+            C.seed.offset, C.precision.offset, C.fused_update.offset, ctypes.sizeof(P.Profile),
+            C.hier_block.offset, C.hier_rounds.offset]
     assert got == want
 
 

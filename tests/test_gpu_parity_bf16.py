@@ -216,3 +216,29 @@ def test_sweep_shape_mlp512_sampled_replicas(P, K):
         got = P.lsgd_params(ctx, k).astype(np.float64)
         assert rel_l2(got - w0, w - w0) <= 2e-2, k
     P.lsgd_destroy(ctx)
+
+
+def test_hierarchical_local_sgd(P):
+    # Hierarchical local SGD (Sec. D): K = 8 workers in blocks of K' = 2, H = 2, H^b = 3.
+    widths = (256, 128, 10)
+    N, K, B, T = 2048, 8, 32, 24
+    X, y = synthdata.gaussian_mixture(N, 256, 10, seed=6)
+    g, o = dense_cfgs(P, widths=widths, K=K, B=B, H=2, T=T, N=N, precision=P.BF16, base_lr=0.05,
+                      momentum=0.9, nesterov=True, weight_decay=5e-4, seed=8, fused_update=True,
+                      hier_block=2, hier_rounds=3)
+    w0 = oracle.init_params(o)
+    ctx = P.lsgd_create(g)
+    P.lsgd_set_dataset(ctx, X, y)
+    P.lsgd_set_params(ctx, -1, w0.astype(np.float32))
+    P.lsgd_run(ctx, 2)  # first round: ends with a block average
+    reps = [P.lsgd_params(ctx, k) for k in range(K)]
+    for b in range(0, K, 2):
+        assert np.array_equal(reps[b], reps[b + 1])
+    assert not np.array_equal(reps[0], reps[2])
+    P.lsgd_run(ctx, T - 2)
+    W, _, lo, ng, nb = oracle.run_counted(o, X, y=y, W=np.tile(w0.astype(np.float32).astype(np.float64),
+                                                                (K, 1)))
+    assert (P.lsgd_sync_count(ctx), P.lsgd_block_sync_count(ctx)) == (ng, nb) == (4, 8)
+    assert rel_l2(P.lsgd_params(ctx, -1), W[0]) <= 2e-2
+    assert np.abs(P.lsgd_losses(ctx, T, K) - lo).max() <= 2e-2
+    P.lsgd_destroy(ctx)

@@ -71,8 +71,9 @@ def test_softmax_regression_config_stepwise(P):
     _stepwise_parity(P, g, o, X, y=y, widths=(3072, 10))
 
 
-@pytest.mark.parametrize("K,B,H,tp", [(3, 7, 3, -1), (5, 40, 2, 4), (1, 9, 4, -1)])
-def test_mlp_momentum_stepwise(P, K, B, H, tp):
+@pytest.mark.parametrize("K,B,H,tp,hb", [(3, 7, 3, -1, 0), (5, 40, 2, 4, 0), (1, 9, 4, -1, 0),
+                                         (4, 8, 1, 2, 2)])
+def test_mlp_momentum_stepwise(P, K, B, H, tp, hb):
     widths = (50, 72, 36, 13)
     N = 400
     rng = np.random.default_rng(K * 10 + B)
@@ -80,7 +81,8 @@ def test_mlp_momentum_stepwise(P, K, B, H, tp):
     y = rng.integers(0, widths[-1], N).astype(np.int32)
     g, o = dense_cfgs(P, widths=widths, K=K, B=B, H=H, T=10, N=N, precision=P.FP32, t_switch=tp,
                       base_lr=0.05, momentum=0.9, nesterov=True, weight_decay=5e-4, seed=4,
-                      scale_by_K=True, warmup_epochs=1.0, milestones=(0.5, 0.75))
+                      scale_by_K=True, warmup_epochs=1.0, milestones=(0.5, 0.75),
+                      hier_block=hb, hier_rounds=3 if hb else 1)
     _stepwise_parity(P, g, o, X, y=y, widths=widths)
 
 

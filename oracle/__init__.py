@@ -29,6 +29,7 @@ _lock = threading.Lock()
 _lib = None
 
 DENSE, LSQ, RESNET20 = 0, 1, 2
+COMPRESS_NONE, COMPRESS_SIGN, COMPRESS_EF_SIGN = 0, 1, 2
 INIT_ZERO, INIT_HE = 0, 1
 MAX_LAYERS = 8
 
@@ -64,6 +65,8 @@ class Cfg(ctypes.Structure):
         ("res_blocks", ctypes.c_int),
         ("hier_block", ctypes.c_int),
         ("hier_rounds", ctypes.c_int),
+        ("compress", ctypes.c_int),
+        ("global_momentum", ctypes.c_double),
     ]
 
 
@@ -71,7 +74,7 @@ def make_cfg(kind=DENSE, widths=(3072, 10), has_bias=True, bf16=False, K=1, B=1,
              t_switch=-1, T=1, N=1, base_lr=0.1, scale_by_K=False, warmup_epochs=0.0,
              milestones=(), decay=0.1, momentum=0.0, nesterov=False, weight_decay=0.0, seed=0,
              in_hwc=(32, 32, 3), n_classes=10, base_ch=16, res_blocks=3, hier_block=0,
-             hier_rounds=1) -> Cfg:
+             hier_rounds=1, compress=0, global_momentum=0.0) -> Cfg:
     c = Cfg()
     c.kind = kind
     if kind != RESNET20:
@@ -99,6 +102,8 @@ def make_cfg(kind=DENSE, widths=(3072, 10), has_bias=True, bf16=False, K=1, B=1,
     c.res_blocks = int(res_blocks)
     c.hier_block = int(hier_block)
     c.hier_rounds = int(hier_rounds)
+    c.compress = int(compress)
+    c.global_momentum = float(global_momentum)
     return c
 
 
@@ -149,6 +154,8 @@ def lib():
                                              P(ctypes.c_int64)]
             L.oracle_run.argtypes = [cfgp, fp, ip, fp, dp, dp, ctypes.c_int64, ctypes.c_int64, dp,
                                      P(ctypes.c_int64)]
+            L.oracle_run_ext.argtypes = [cfgp, fp, ip, fp, dp, dp, dp, dp, dp, ctypes.c_int64,
+                                         ctypes.c_int64, dp, P(ctypes.c_int64), P(ctypes.c_int64)]
             L.oracle_run_minibatch.argtypes = [cfgp, fp, ip, fp, dp, dp, ctypes.c_int64,
                                                ctypes.c_int64, dp]
             L.oracle_eval_loss.argtypes = [cfgp, dp, fp, ip, fp, ctypes.c_int64]
@@ -265,6 +272,29 @@ def run_counted(c: Cfg, X, y=None, t=None, W=None, U=None, s0=0, n_steps=None):
                              int(s0), n, _p(losses, ctypes.c_double), ctypes.byref(ng),
                              ctypes.byref(nb))
     return W, U, losses, int(ng.value), int(nb.value)
+
+
+def run_ext(c: Cfg, X, y=None, t=None, W=None, U=None, Wref=None, E=None, Ug=None, s0=0,
+            n_steps=None):
+    """Run with the synchronisation state of the compressed / global-momentum variants.
+    Returns W, U, Wref, E, Ug, losses, n_global, n_block."""
+    d = num_params(c)
+    if W is None:
+        W = np.tile(init_params(c), (c.K, 1))
+    W = np.array(W, dtype=np.float64).reshape(c.K, d)
+    U = np.zeros_like(W) if U is None else np.array(U, dtype=np.float64).reshape(c.K, d)
+    Wref = W[0].copy() if Wref is None else np.array(Wref, dtype=np.float64).reshape(d)
+    E = np.zeros_like(W) if E is None else np.array(E, dtype=np.float64).reshape(c.K, d)
+    Ug = np.zeros(d) if Ug is None else np.array(Ug, dtype=np.float64).reshape(d)
+    n = int(c.T - s0 if n_steps is None else n_steps)
+    losses = np.zeros((n, c.K), dtype=np.float64)
+    ng, nb = ctypes.c_int64(0), ctypes.c_int64(0)
+    X, y, t = _f32(X), _i32(y), _f32(t)
+    lib().oracle_run_ext(ctypes.byref(c), _p(X, ctypes.c_float), _p(y, ctypes.c_int32),
+                         _p(t, ctypes.c_float), _p(W, ctypes.c_double), _p(U, ctypes.c_double),
+                         _p(Wref, ctypes.c_double), _p(E, ctypes.c_double), _p(Ug, ctypes.c_double),
+                         int(s0), n, _p(losses, ctypes.c_double), ctypes.byref(ng), ctypes.byref(nb))
+    return W, U, Wref, E, Ug, losses, int(ng.value), int(nb.value)
 
 
 def run(c: Cfg, X, y=None, t=None, W=None, U=None, s0=0, n_steps=None):

@@ -259,6 +259,8 @@ double oracle_loss_grad(const oracle_cfg* c, const double* w, const float* X, co
 
 // Local momentum SGD step on one worker (Sec. C.3.1: u = m u + grad, w = w - gamma u, kept per
 // worker), with the Nesterov variant without dampening and plain L2 weight decay (Sec. A.4): g' = g + lambda w; u = m u + g'; step = g' + m u (Nesterov) or u; w -= gamma step.
+// With the signSGD variant of Algorithm 4 the local step moves by lr sign(step), the step
+// direction after weight decay and momentum (sign(0) = 0).
 void oracle_sgd_update(const oracle_cfg* c, double lr, double* w, double* u, const double* g) {
   const int64_t d = oracle_num_params(c);
   std::vector<uint8_t> mask((size_t)d);
@@ -272,6 +274,7 @@ void oracle_sgd_update(const oracle_cfg* c, double lr, double* w, double* u, con
       u[i] = c->momentum * u[i] + gp;
       step = c->nesterov ? gp + c->momentum * u[i] : u[i];
     }
+    if (c->compress == ORACLE_COMPRESS_SIGN) step = (step > 0.0) - (step < 0.0);
     w[i] -= lr * step;
   }
 }
@@ -335,12 +338,79 @@ void oracle_average(int K, int64_t d, double* W) {
 
 // Local / post-local SGD (Eq. 2; Algorithms 1 and 2) from global step s0 for n_steps steps.
 // W and U hold the K workers' models and momentum buffers, worker-major, and are updated in place.
-void oracle_run_counted(const oracle_cfg* c, const float* X, const int32_t* y, const float* t,
-                        double* W, double* U, int64_t s0, int64_t n_steps, double* losses,
-                        int64_t* n_global, int64_t* n_block) {
+namespace {
+
+// The synchronisation that ends a round, for the round-start model wref shared by all workers:
+//  * plain (Eq. 2): w^k := wref := (1/K) sum_k w^k;
+//  * global momentum (Sec. C.3.1): ug := m_g ug + (wref - mean_k w^k) / lr; wref -= lr ug;
+//  * signSGD compression (Algorithm 4): Delta^k = wref - w^k, s^k = sign(Delta^k),
+//    p^k = ||Delta^k||_1 / d; wref -= (1/K) sum_k s^k p^k;
+//  * EF-signSGD (Algorithm 5): Delta^k = wref - w^k + e^k, s^k, p^k as above,
+//    e^k := Delta^k - s^k p^k (the residual the compression dropped), wref -= (1/K) sum_k s^k p^k;
+// and every worker restarts from wref.
+void global_sync(const oracle_cfg* c, int64_t d, double lr, double* W, double* wref, double* E,
+                 double* ug) {
+  const int K = c->K;
+  if (c->compress == ORACLE_COMPRESS_NONE) {
+    oracle_average(K, d, W);
+    if (c->global_momentum > 0.0) {
+      for (int64_t i = 0; i < d; ++i) {
+        ug[i] = c->global_momentum * ug[i] + (wref[i] - W[i]) / lr;
+        wref[i] -= lr * ug[i];
+      }
+      for (int k = 0; k < K; ++k)
+        for (int64_t i = 0; i < d; ++i) W[(int64_t)k * d + i] = wref[i];
+    } else {
+      for (int64_t i = 0; i < d; ++i) wref[i] = W[i];
+    }
+    return;
+  }
+  std::vector<double> delta((size_t)K * d), p((size_t)K);
+  for (int k = 0; k < K; ++k) {
+    double l1 = 0.0;
+    for (int64_t i = 0; i < d; ++i) {
+      double v = wref[i] - W[(int64_t)k * d + i];
+      if (c->compress == ORACLE_COMPRESS_EF_SIGN) v += E[(int64_t)k * d + i];
+      delta[(size_t)k * d + i] = v;
+      l1 += std::fabs(v);
+    }
+    p[k] = l1 / (double)d;
+  }
+  for (int64_t i = 0; i < d; ++i) {
+    double acc = 0.0;
+    for (int k = 0; k < K; ++k) {
+      const double v = delta[(size_t)k * d + i];
+      const double sp = (double)((v > 0.0) - (v < 0.0)) * p[k];
+      acc += sp;
+      if (c->compress == ORACLE_COMPRESS_EF_SIGN) E[(int64_t)k * d + i] = v - sp;
+    }
+    wref[i] -= acc / K;
+  }
+  for (int k = 0; k < K; ++k)
+    for (int64_t i = 0; i < d; ++i) W[(int64_t)k * d + i] = wref[i];
+}
+
+}  // namespace
+
+void oracle_run_ext(const oracle_cfg* c, const float* X, const int32_t* y, const float* t,
+                    double* W, double* U, double* Wref, double* E, double* Ug, int64_t s0,
+                    int64_t n_steps, double* losses, int64_t* n_global, int64_t* n_block) {
   const int64_t d = oracle_num_params(c);
   std::vector<int32_t> idx((size_t)c->B);
   std::vector<double> g((size_t)d);
+  std::vector<double> wref_own, e_own, ug_own;
+  if (!Wref) {
+    wref_own.assign(W, W + d);
+    Wref = wref_own.data();
+  }
+  if (!E) {
+    e_own.assign((size_t)c->K * d, 0.0);
+    E = e_own.data();
+  }
+  if (!Ug) {
+    ug_own.assign((size_t)d, 0.0);
+    Ug = ug_own.data();
+  }
   int64_t syncs = 0, blocks = 0;
   for (int64_t s = s0; s < s0 + n_steps; ++s) {
     const double lr = oracle_lr(c, s);
@@ -352,7 +422,7 @@ void oracle_run_counted(const oracle_cfg* c, const float* X, const int32_t* y, c
     }
     const int kind = oracle_sync_kind(c, s);
     if (kind == ORACLE_SYNC_GLOBAL) {
-      oracle_average(c->K, d, W);
+      global_sync(c, d, lr, W, Wref, E, Ug);
       ++syncs;
     } else if (kind == ORACLE_SYNC_BLOCK) {
       oracle_block_average(c->K, c->hier_block, d, W);
@@ -361,6 +431,13 @@ void oracle_run_counted(const oracle_cfg* c, const float* X, const int32_t* y, c
   }
   if (n_global) *n_global = syncs;
   if (n_block) *n_block = blocks;
+}
+
+void oracle_run_counted(const oracle_cfg* c, const float* X, const int32_t* y, const float* t,
+                        double* W, double* U, int64_t s0, int64_t n_steps, double* losses,
+                        int64_t* n_global, int64_t* n_block) {
+  oracle_run_ext(c, X, y, t, W, U, nullptr, nullptr, nullptr, s0, n_steps, losses, n_global,
+                 n_block);
 }
 
 void oracle_run(const oracle_cfg* c, const float* X, const int32_t* y, const float* t, double* W,

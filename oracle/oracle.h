@@ -48,7 +48,14 @@ typedef struct {
   /* hierarchical local SGD (Sec. D): blocks of hier_block consecutive workers average after every
      H-step round, all K workers after every hier_rounds-th round (hier_block = 0: off) */
   int hier_block, hier_rounds;
+  /* compressed averaging (Sec. B.3): 0 none, 1 signSGD variant (Algorithm 4: sign local steps,
+     sign-compressed model differences), 2 EF-signSGD (Algorithm 5: error-feedback memory) */
+  int compress;
+  /* global momentum (Sec. C.3.1): > 0 applies momentum m_g to the averaged model difference */
+  double global_momentum;
 } oracle_cfg;
+
+enum { ORACLE_COMPRESS_NONE = 0, ORACLE_COMPRESS_SIGN = 1, ORACLE_COMPRESS_EF_SIGN = 2 };
 
 enum { ORACLE_SYNC_NONE = 0, ORACLE_SYNC_BLOCK = 1, ORACLE_SYNC_GLOBAL = 2 };
 
@@ -67,6 +74,12 @@ void oracle_average(int K, int64_t d, double* W);
 void oracle_block_average(int K, int block, int64_t d, double* W);
 void oracle_run(const oracle_cfg* c, const float* X, const int32_t* y, const float* t, double* W,
                 double* U, int64_t s0, int64_t n_steps, double* losses, int64_t* n_syncs);
+/* Local / post-local SGD with the synchronisation state of the compressed and global-momentum
+ * variants: Wref [d] the synchronised model at the start of the round (NULL: taken from W[0]),
+ * E [K][d] the error-feedback memories, Ug [d] the global momentum (NULL: zeros / not kept). */
+void oracle_run_ext(const oracle_cfg* c, const float* X, const int32_t* y, const float* t,
+                    double* W, double* U, double* Wref, double* E, double* Ug, int64_t s0,
+                    int64_t n_steps, double* losses, int64_t* n_global, int64_t* n_block);
 /* As oracle_run, also counting the block averages of hierarchical local SGD. */
 void oracle_run_counted(const oracle_cfg* c, const float* X, const int32_t* y, const float* t,
                         double* W, double* U, int64_t s0, int64_t n_steps, double* losses,

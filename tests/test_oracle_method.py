@@ -336,3 +336,93 @@ def test_hierarchical_sync_counts_match_communication_model(T, H, Hb):
     kinds = [oracle.sync_kind(c, s) for s in range(T)]
     assert kinds.count(2) == T // (H * Hb)
     assert kinds.count(1) == T // H - T // (H * Hb)
+
+
+# ---- global momentum (Sec. C.3.1) and compressed averaging (Sec. B.3, Algorithms 4 and 5) ----
+
+def _sr_cfg(**kw):
+    # softmax regression: no ReLU, so no gradient component is exactly zero on random data
+    args = dict(widths=(12, 5), K=3, B=4, H=1, T=8, N=48, base_lr=0.05, seed=31)
+    args.update(kw)
+    return oracle.make_cfg(**args)
+
+
+def test_global_momentum_h1_is_heavy_ball_minibatch_sgd():
+    # With H = 1 and plain local steps, the global momentum u = m u + (w_ref - mean w^k) / lr
+    # = m u + mean_k grad^k, w_ref -= lr u: heavy-ball mini-batch SGD on the union batch.
+    X, y = _data(48, 12, 5, 21)
+    c_g = _sr_cfg(global_momentum=0.9)
+    c_m = _sr_cfg(momentum=0.9)
+    W, _, _, _, _, _, ng, _ = oracle.run_ext(c_g, X, y=y)
+    w, _, _ = oracle.run_minibatch(c_m, X, y=y)
+    assert ng == 8
+    np.testing.assert_allclose(W[0], w, rtol=0, atol=1e-12 * np.abs(w).max())
+
+
+def test_global_momentum_vanishing_factor_is_plain_averaging():
+    X, y = _data(48, 12, 5, 22)
+    W, _, _, _, _, _, _, _ = oracle.run_ext(_sr_cfg(H=2, global_momentum=1e-12), X, y=y)
+    Wp, _, _, _ = oracle.run(_sr_cfg(H=2), X, y=y)
+    np.testing.assert_allclose(W, Wp, rtol=0, atol=1e-12 * np.abs(Wp).max())
+
+
+def test_sign_compression_is_lossless_for_one_worker_and_one_step():
+    # Algorithm 4 with K = 1, H = 1: the sign local step moves every coordinate by exactly lr, so
+    # ||Delta||_1 / d = lr and sign(Delta) lr = Delta: the run is plain signSGD, w -= lr sign(grad).
+    X, y = _data(48, 12, 5, 23)
+    c = _sr_cfg(K=1, compress=oracle.COMPRESS_SIGN)
+    W, _, _, _, _, _, ng, _ = oracle.run_ext(c, X, y=y)
+    w = oracle.init_params(c)
+    for s in range(c.T):
+        _, g = oracle.loss_grad(c, w, X, y=y, idx=oracle.sample_indices(c, 0, s))
+        w = w - 0.05 * np.sign(g)
+    assert ng == 8
+    np.testing.assert_allclose(W[0], w, rtol=0, atol=1e-13)
+
+
+def test_sign_compressed_average_of_a_round():
+    # One round of K = 2 workers (H = 3): the model after the sync is w_ref - (1/K) sum_k s^k p^k
+    # of the workers' models before it (taken from the same run with a longer round).
+    X, y = _data(48, 12, 5, 24)
+    c = _sr_cfg(K=2, H=3, T=100, compress=oracle.COMPRESS_SIGN)
+    c_long = _sr_cfg(K=2, H=4, T=100, compress=oracle.COMPRESS_SIGN)
+    w0 = oracle.init_params(c)
+    Wpre, _, _, _, _, _, _, _ = oracle.run_ext(c_long, X, y=y, n_steps=3)
+    Wpost, _, wref, _, _, _, ng, _ = oracle.run_ext(c, X, y=y, n_steps=3)
+    assert ng == 1
+    delta = w0[None, :] - Wpre
+    p = np.abs(delta).sum(1) / delta.shape[1]
+    expect = w0 - (np.sign(delta) * p[:, None]).mean(0)
+    np.testing.assert_allclose(wref, expect, rtol=0, atol=1e-14)
+    assert np.array_equal(Wpost[0], wref) and np.array_equal(Wpost[1], wref)
+
+
+def test_error_feedback_bookkeeping():
+    # Algorithm 5 with K = 1: the synchronised model equals the worker's own model after the round
+    # corrected by the change of its error memory, w_ref(t+1) = w(t+H) - e(t) + e(t+1), and the memory
+    # keeps exactly what the compression dropped.
+    X, y = _data(48, 12, 5, 25)
+    c = _sr_cfg(K=1, H=3, T=100, compress=oracle.COMPRESS_EF_SIGN)
+    c_plain = _sr_cfg(K=1, H=3, T=100)
+    rng = np.random.default_rng(5)
+    d = oracle.num_params(c)
+    e0 = 1e-3 * rng.standard_normal((1, d))
+    W, _, wref, e1, _, _, _, _ = oracle.run_ext(c, X, y=y, E=e0, n_steps=3)
+    Wl, _, _, _ = oracle.run(c_plain, X, y=y, n_steps=3)  # EF does not change the local steps
+    np.testing.assert_allclose(wref, Wl[0] - e0[0] + e1[0], rtol=0, atol=1e-14)
+    w0 = oracle.init_params(c)
+    delta = w0 - Wl[0] + e0[0]
+    sp = np.sign(delta) * np.abs(delta).mean()
+    np.testing.assert_allclose(e1[0], delta - sp, rtol=0, atol=1e-14)
+
+
+def test_split_run_with_sync_state_equals_straight_run():
+    X, y = _data(48, 12, 5, 26)
+    for kw in (dict(compress=oracle.COMPRESS_EF_SIGN), dict(global_momentum=0.8),
+               dict(compress=oracle.COMPRESS_SIGN, momentum=0.9)):
+        c = _sr_cfg(H=2, T=9, **kw)
+        A = oracle.run_ext(c, X, y=y)
+        B = oracle.run_ext(c, X, y=y, n_steps=4)
+        C = oracle.run_ext(c, X, y=y, W=B[0], U=B[1], Wref=B[2], E=B[3], Ug=B[4], s0=4, n_steps=5)
+        for a, b in zip(A[:5], C[:5]):
+            assert np.array_equal(a, b)

@@ -222,6 +222,64 @@ def run_sweep(args):
             P.lsgd_destroy(ctx)
 
 
+# Algorithmic bytes per parameter and replica of one synchronisation (fp32 state, bf16 shadow),
+# plus bytes per parameter of the shared vectors (w_ref, u_g: fp32):
+#   plain average          : read w, write w + shadow                           = 10 | 0
+#   global momentum        : the same, plus read + write w_ref and u_g          = 10 | 16
+#   sign (two passes)      : read w (L1 norms), read w + write w + shadow       = 14 | 12 (w_ref read
+#                            twice, written once)
+#   EF-sign (two passes)   : sign's, plus read e (twice) and write e            = 26 | 12
+SYNC_VARIANT_BYTES = {"plain": (10, 0), "global_momentum": (10, 16), "sign": (14, 12),
+                      "ef_sign": (26, 12)}
+
+
+def run_sync_variants(args):
+    """Time one synchronisation of each averaging variant on the MLP workload's parameter arena
+    (K = 16 replicas of d = 4.2 M parameters; 268 MB of fp32 replicas, larger than L2): one JSON
+    line per variant with ms per sync and algorithmic GB/s against the HBM peak."""
+    import torch
+
+    from paper_1808_07217_gb300 import _build
+
+    _build.build()
+    import paper_1808_07217_gb300 as P
+
+    torch.cuda.set_device(0)
+    stream = torch.cuda.current_stream()
+    hbm, _, src = _peaks()
+    w = WORKLOAD
+    K = args.replicas or w["K"]
+    n_sync = max(args.steps, 8)
+    for name, extra in (("plain", {}), ("global_momentum", dict(global_momentum=0.9)),
+                        ("sign", dict(compress=P.COMPRESS_SIGN)),
+                        ("ef_sign", dict(compress=P.COMPRESS_EF_SIGN))):
+        cfg = P.make_config(K=K, B_loc=w["B"], H=w["H"], total_steps=16, N=w["N"],
+                            widths=w["widths"], base_lr=w["base_lr"], momentum=w["momentum"],
+                            nesterov=w["nesterov"], weight_decay=w["weight_decay"], seed=w["seed"],
+                            precision=P.BF16, **extra)
+        ctx = P.lsgd_create(cfg, stream=stream.cuda_stream)
+        d = P.lsgd_num_params(ctx)
+        for _ in range(max(3, args.warmup)):
+            P.lsgd_sync_average(ctx)
+        torch.cuda.synchronize()
+        n1 = P.lsgd_kernel_launches(ctx)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(n_sync):
+            P.lsgd_sync_average(ctx)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1) / n_sync
+        per_rep, shared = SYNC_VARIANT_BYTES[name]
+        nbytes = per_rep * K * d + shared * d
+        gbs = nbytes / (ms * 1e6)
+        print(json.dumps({"sync_variant": name, "K": K, "d": d, "ms_per_sync": ms,
+                          "launches_per_sync": (P.lsgd_kernel_launches(ctx) - n1) / n_sync,
+                          "algorithmic_bytes": nbytes, "achieved_gbs": gbs,
+                          "peak_gbs": hbm, "frac": gbs / hbm, "peak_source": src}), flush=True)
+        P.lsgd_destroy(ctx)
+
+
 RESNET_WORKLOAD = dict(name="resnet20_K16_B128_postlocal_H16_bf16", K=16, B=128, H=16, N=50000,
                        C=10, base_lr=0.2, scale_by_K=True, warmup_epochs=5.0, momentum=0.9,
                        nesterov=True, weight_decay=1e-4, seed=0, data_seed=1234)
@@ -281,6 +339,9 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--sweep", action="store_true",
                     help="K x H sync / compute sweep of the MLP 3072-512-512-10 workload")
+    ap.add_argument("--sync-variants", action="store_true",
+                    help="time one synchronisation of each averaging variant (plain, global "
+                         "momentum, sign, EF-sign) on the MLP workload's K x d arena")
     ap.add_argument("--resnet", action="store_true",
                     help="post-local ResNet-20 workload (K = 16, B_loc = 128) instead of the MLP")
     ap.add_argument("--unfused", action="store_true",
@@ -295,6 +356,9 @@ def main():
         return
     if args.resnet:
         run_resnet(args)
+        return
+    if args.sync_variants:
+        run_sync_variants(args)
         return
 
     if args.impl == "reference":

@@ -108,7 +108,22 @@ typedef struct {
                             hier_rounds-th round (and the run's last step) all K; must divide K.
                             0 = off.  The mini-batch phase of post-local SGD averages globally. */
   int hier_rounds;       /* H^b >= 1 */
+  int compress;          /* lsgd_compress: averaging of compressed model differences (Sec. B.3)
+                            relative to the round-start model w_ref.  Not with hier_block;
+                            K <= 1024. */
+  double global_momentum;/* m_g > 0: global momentum at every average (Sec. C.3.1):
+                            u_g = m_g u_g + (w_ref - mean_k w^k) / gamma, w_ref -= gamma u_g.
+                            Not with compress or hier_block. */
 } lsgd_config;
+
+typedef enum {
+  LSGD_COMPRESS_NONE = 0,
+  LSGD_COMPRESS_SIGN = 1,    /* Algorithm 4: local steps w -= gamma sign(step); the average becomes
+                                w_ref -= (1/K) sum_k sign(Delta_k) ||Delta_k||_1 / d,
+                                Delta_k = w_ref - w^k */
+  LSGD_COMPRESS_EF_SIGN = 2  /* Algorithm 5: plain local steps; Delta_k = w_ref - w^k + e^k, the same
+                                compressed average, and e^k = Delta_k - sign(Delta_k) ||Delta_k||_1 / d */
+} lsgd_compress;
 
 typedef struct lsgd_ctx lsgd_ctx;
 
@@ -143,7 +158,9 @@ lsgd_status lsgd_local_step_batch(lsgd_ctx* ctx, const float* x, const void* lab
 
 /* The K-way average w^k := (1/K) sum_k w^k for every k (Eq. 2 right; the all-reduce and model
  * update that close each round of Algorithm 1); momentum buffers stay local (Sec. A.4).
- * Refreshes the bf16 shadow. */
+ * Refreshes the bf16 shadow.  With cfg.compress or cfg.global_momentum the average is the
+ * corresponding variant (gamma of the step that ended the round) and the result also becomes the
+ * next round's w_ref; lsgd_set_params(ctx, -1, ...) resets w_ref. */
 lsgd_status lsgd_sync_average(lsgd_ctx* ctx);
 
 /* Block average of hierarchical local SGD (Sec. D): every replica becomes the mean of the
@@ -164,6 +181,19 @@ lsgd_status lsgd_momentum(lsgd_ctx* ctx, int k, float* dst, int dst_is_device, s
 lsgd_status lsgd_set_params(lsgd_ctx* ctx, int k, const float* src, size_t n);
 lsgd_status lsgd_set_momentum(lsgd_ctx* ctx, int k, const float* src, size_t n);
 
+typedef enum {
+  LSGD_STATE_WREF = 0,            /* round-start model w_ref (k = 0) */
+  LSGD_STATE_ERROR = 1,           /* error-feedback memory e^k of replica k (Algorithm 5) */
+  LSGD_STATE_GLOBAL_MOMENTUM = 2  /* global momentum u_g (k = 0; Sec. C.3.1) */
+} lsgd_sync_state_kind;
+/* Read / overwrite the synchronisation state of the compressed and global-momentum averages, n =
+ * lsgd_num_params() floats of host memory in canonical order.  k selects the replica for
+ * LSGD_STATE_ERROR (k = -1 on write: every replica) and must be 0 for the others.  LSGD_ESTATE if
+ * the configuration does not keep that state (w_ref exists with compress or global_momentum, e^k
+ * with LSGD_COMPRESS_EF_SIGN, u_g with global_momentum). */
+lsgd_status lsgd_sync_state(lsgd_ctx* ctx, int which, int k, float* dst, size_t n);
+lsgd_status lsgd_set_sync_state(lsgd_ctx* ctx, int which, int k, const float* src, size_t n);
+
 /* Per-replica mean mini-batch loss of the last `n_steps` steps, [n_steps][K] fp32, oldest first.
  * The history holds the last T steps. */
 lsgd_status lsgd_losses(lsgd_ctx* ctx, float* dst, int64_t n_steps);
@@ -178,8 +208,9 @@ lsgd_status lsgd_eval_loss(lsgd_ctx* ctx, int k, int64_t n, double* loss);
 /* LSGD_ENONFINITE if any replica parameter is NaN or Inf. */
 lsgd_status lsgd_check_finite(lsgd_ctx* ctx);
 
-/* Checkpoint / resume of w, u (all replicas), the step and sync counters.  Philox is counter based
- * so no generator state is stored.  lsgd_load requires a context created with the same config. */
+/* Checkpoint / resume of w, u (all replicas), the synchronisation state (w_ref, e^k, u_g where the
+ * configuration keeps it), the step and sync counters.  Philox is counter based so no generator
+ * state is stored.  lsgd_load requires a context created with the same config. */
 lsgd_status lsgd_save(lsgd_ctx* ctx, const char* path);
 lsgd_status lsgd_load(lsgd_ctx* ctx, const char* path);
 

@@ -21,6 +21,8 @@ MAX_LAYERS = 8
 MLP, LSQ, RESNET20 = 0, 1, 2
 FP32, BF16 = 0, 1
 INIT_ZERO, INIT_HE = 0, 1
+COMPRESS_NONE, COMPRESS_SIGN, COMPRESS_EF_SIGN = 0, 1, 2
+STATE_WREF, STATE_ERROR, STATE_GLOBAL_MOMENTUM = 0, 1, 2
 
 OK, EINVAL, ENOMEM, ECUDA, ESTATE, ENONFINITE, ETIMEOUT, EUNSUPPORTED, EIO = range(9)
 _STATUS = {0: "OK", 1: "EINVAL", 2: "ENOMEM", 3: "ECUDA", 4: "ESTATE", 5: "ENONFINITE",
@@ -36,6 +38,7 @@ EXPORTS = [
     "lsgd_kway_average", "lsgd_sgd_update", "lsgd_sample_indices", "lsgd_profile_enable",
     "lsgd_profile_read", "lsgd_grouped_gemm_bf16", "lsgd_batchnorm_stats",
     "lsgd_batchnorm_stats_noalloc", "lsgd_block_average", "lsgd_block_sync_count",
+    "lsgd_sync_state", "lsgd_set_sync_state",
 ]
 PHASES = ["input", "forward", "loss", "backward", "update", "average"]
 
@@ -78,14 +81,16 @@ class Config(ctypes.Structure):
                 ("lr", LrSchedule), ("momentum", ctypes.c_double), ("nesterov", ctypes.c_int),
                 ("weight_decay", ctypes.c_double), ("seed", ctypes.c_uint64),
                 ("precision", ctypes.c_int), ("fused_update", ctypes.c_int),
-                ("hier_block", ctypes.c_int), ("hier_rounds", ctypes.c_int)]
+                ("hier_block", ctypes.c_int), ("hier_rounds", ctypes.c_int),
+                ("compress", ctypes.c_int), ("global_momentum", ctypes.c_double)]
 
 
 def make_config(K=1, B_loc=1, H=1, t_switch=-1, total_steps=0, epochs=0.0, N=1, kind=MLP,
                 widths=(3072, 10), init=INIT_HE, in_hwc=(32, 32, 3), n_classes=10, base_ch=16,
                 res_blocks=3, base_lr=0.1, scale_by_K=False, warmup_epochs=0.0, milestones=(),
                 decay=0.1, momentum=0.0, nesterov=False, weight_decay=0.0, seed=0,
-                precision=FP32, fused_update=False, hier_block=0, hier_rounds=1) -> Config:
+                precision=FP32, fused_update=False, hier_block=0, hier_rounds=1, compress=0,
+                global_momentum=0.0) -> Config:
     c = Config()
     c.K, c.B_loc, c.H = int(K), int(B_loc), int(H)
     c.t_switch, c.total_steps, c.epochs, c.N = int(t_switch), int(total_steps), float(epochs), int(N)
@@ -109,6 +114,7 @@ def make_config(K=1, B_loc=1, H=1, t_switch=-1, total_steps=0, epochs=0.0, N=1, 
     c.precision = int(precision)
     c.fused_update = int(bool(fused_update))
     c.hier_block, c.hier_rounds = int(hier_block), int(hier_rounds)
+    c.compress, c.global_momentum = int(compress), float(global_momentum)
     return c
 
 
@@ -138,6 +144,8 @@ def lib():
             "lsgd_momentum": ([vp, ctypes.c_int, vp, ctypes.c_int, ctypes.c_size_t], st),
             "lsgd_set_params": ([vp, ctypes.c_int, vp, ctypes.c_size_t], st),
             "lsgd_set_momentum": ([vp, ctypes.c_int, vp, ctypes.c_size_t], st),
+            "lsgd_sync_state": ([vp, ctypes.c_int, ctypes.c_int, vp, ctypes.c_size_t], st),
+            "lsgd_set_sync_state": ([vp, ctypes.c_int, ctypes.c_int, vp, ctypes.c_size_t], st),
             "lsgd_losses": ([vp, vp, i64], st),
             "lsgd_debug_indices": ([vp, i64, vp], st),
             "lsgd_eval_loss": ([vp, ctypes.c_int, i64, P(ctypes.c_double)], st),
@@ -314,6 +322,17 @@ def lsgd_set_params(ctx: Ctx, k: int, w):
 def lsgd_set_momentum(ctx: Ctx, k: int, u):
     u = np.ascontiguousarray(u, dtype=np.float32)
     _check(lib().lsgd_set_momentum(ctx.handle, int(k), _ptr(u), u.size), ctx)
+
+
+def lsgd_sync_state(ctx: Ctx, which: int, k: int = 0):
+    out = np.empty(lsgd_num_params(ctx), dtype=np.float32)
+    _check(lib().lsgd_sync_state(ctx.handle, int(which), int(k), _ptr(out), out.size), ctx)
+    return out
+
+
+def lsgd_set_sync_state(ctx: Ctx, which: int, k: int, v):
+    v = np.ascontiguousarray(v, dtype=np.float32)
+    _check(lib().lsgd_set_sync_state(ctx.handle, int(which), int(k), _ptr(v), v.size), ctx)
 
 
 def lsgd_losses(ctx: Ctx, n_steps: int, K: int):

@@ -47,10 +47,12 @@ __device__ __forceinline__ uint16_t f2bf(float f) {
 __device__ __forceinline__ float bf2f(uint16_t u) { return __uint_as_float(((uint32_t)u) << 16); }
 
 // One element of the local update (Sec. C.3.1 / A.4): g' = g + lam w; u = m u + g';
-// w -= lr (nesterov ? g' + m u : u), or w -= lr g' without momentum.  Every kernel that updates
-// parameters goes through this function, so fused and stand-alone updates agree bit for bit.
+// w -= lr (nesterov ? g' + m u : u), or w -= lr g' without momentum; with `sgn` (the signSGD
+// variant of Algorithm 4) w -= lr sign(step), sign(0) = 0.  Every kernel that updates parameters
+// goes through this function, so fused and stand-alone updates agree bit for bit.
 template <bool MOM, bool NEST>
-__device__ __forceinline__ void sgd_elem(float& w, float& u, float g, float lr, float m, float lam) {
+__device__ __forceinline__ void sgd_elem(float& w, float& u, float g, float lr, float m, float lam,
+                                         bool sgn = false) {
   const float gp = fmaf(lam, w, g);
   float st;
   if (MOM) {
@@ -59,6 +61,7 @@ __device__ __forceinline__ void sgd_elem(float& w, float& u, float g, float lr, 
   } else {
     st = gp;
   }
+  if (sgn) st = st > 0.f ? 1.f : (st < 0.f ? -1.f : 0.f);
   w = fmaf(-lr, st, w);
 }
 

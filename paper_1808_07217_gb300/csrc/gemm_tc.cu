@@ -138,21 +138,22 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
 
 // The local update on four consecutive parameters (fused weight-gradient epilogue).
 __device__ __forceinline__ void sgd4(float4& w, float4& u, const float4 g, const SgdParams& sp) {
+  const bool sg = sp.sign != 0;
   if (sp.mom == 0.f) {
-    sgd_elem<false, false>(w.x, u.x, g.x, sp.lr, 0.f, sp.wd);
-    sgd_elem<false, false>(w.y, u.y, g.y, sp.lr, 0.f, sp.wd);
-    sgd_elem<false, false>(w.z, u.z, g.z, sp.lr, 0.f, sp.wd);
-    sgd_elem<false, false>(w.w, u.w, g.w, sp.lr, 0.f, sp.wd);
+    sgd_elem<false, false>(w.x, u.x, g.x, sp.lr, 0.f, sp.wd, sg);
+    sgd_elem<false, false>(w.y, u.y, g.y, sp.lr, 0.f, sp.wd, sg);
+    sgd_elem<false, false>(w.z, u.z, g.z, sp.lr, 0.f, sp.wd, sg);
+    sgd_elem<false, false>(w.w, u.w, g.w, sp.lr, 0.f, sp.wd, sg);
   } else if (sp.nesterov) {
-    sgd_elem<true, true>(w.x, u.x, g.x, sp.lr, sp.mom, sp.wd);
-    sgd_elem<true, true>(w.y, u.y, g.y, sp.lr, sp.mom, sp.wd);
-    sgd_elem<true, true>(w.z, u.z, g.z, sp.lr, sp.mom, sp.wd);
-    sgd_elem<true, true>(w.w, u.w, g.w, sp.lr, sp.mom, sp.wd);
+    sgd_elem<true, true>(w.x, u.x, g.x, sp.lr, sp.mom, sp.wd, sg);
+    sgd_elem<true, true>(w.y, u.y, g.y, sp.lr, sp.mom, sp.wd, sg);
+    sgd_elem<true, true>(w.z, u.z, g.z, sp.lr, sp.mom, sp.wd, sg);
+    sgd_elem<true, true>(w.w, u.w, g.w, sp.lr, sp.mom, sp.wd, sg);
   } else {
-    sgd_elem<true, false>(w.x, u.x, g.x, sp.lr, sp.mom, sp.wd);
-    sgd_elem<true, false>(w.y, u.y, g.y, sp.lr, sp.mom, sp.wd);
-    sgd_elem<true, false>(w.z, u.z, g.z, sp.lr, sp.mom, sp.wd);
-    sgd_elem<true, false>(w.w, u.w, g.w, sp.lr, sp.mom, sp.wd);
+    sgd_elem<true, false>(w.x, u.x, g.x, sp.lr, sp.mom, sp.wd, sg);
+    sgd_elem<true, false>(w.y, u.y, g.y, sp.lr, sp.mom, sp.wd, sg);
+    sgd_elem<true, false>(w.z, u.z, g.z, sp.lr, sp.mom, sp.wd, sg);
+    sgd_elem<true, false>(w.w, u.w, g.w, sp.lr, sp.mom, sp.wd, sg);
   }
 }
 

@@ -182,12 +182,13 @@ __global__ void __launch_bounds__(256) colsum_kernel(const TD* __restrict__ dz, 
         gb[i] = s;
       } else {
         float w = sgd.w[i], u = sgd.u ? sgd.u[i] : 0.f;
+        const bool sg = sgd.sign != 0;
         if (sgd.mom == 0.f)
-          sgd_elem<false, false>(w, u, s, sgd.lr, 0.f, sgd.wd);
+          sgd_elem<false, false>(w, u, s, sgd.lr, 0.f, sgd.wd, sg);
         else if (sgd.nesterov)
-          sgd_elem<true, true>(w, u, s, sgd.lr, sgd.mom, sgd.wd);
+          sgd_elem<true, true>(w, u, s, sgd.lr, sgd.mom, sgd.wd, sg);
         else
-          sgd_elem<true, false>(w, u, s, sgd.lr, sgd.mom, sgd.wd);
+          sgd_elem<true, false>(w, u, s, sgd.lr, sgd.mom, sgd.wd, sg);
         sgd.w[i] = w;
         if (sgd.u) sgd.u[i] = u;
         if (sgd.wb) sgd.wb[i] = f2bf(w);
@@ -204,7 +205,7 @@ template <bool MOM, bool NEST, bool SHADOW>
 __global__ void __launch_bounds__(256) sgd_update_kernel(
     float4* __restrict__ w, float4* __restrict__ u, const float4* __restrict__ g,
     uint2* __restrict__ wb, int64_t n4, float lr, float m, float wd, int64_t period,
-    int64_t decay_end) {
+    int64_t decay_end, int sgn) {
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n4; i += stride) {
     const float4 gv = __ldcs(g + i);
@@ -212,10 +213,10 @@ __global__ void __launch_bounds__(256) sgd_update_kernel(
     float lam = wd;
     if (period > 0 && ((i * 4) % period) >= decay_end) lam = 0.f;
     float4 uv = MOM ? __ldcs(u + i) : make_float4(0.f, 0.f, 0.f, 0.f);
-    sgd_elem<MOM, NEST>(wv.x, uv.x, gv.x, lr, m, lam);
-    sgd_elem<MOM, NEST>(wv.y, uv.y, gv.y, lr, m, lam);
-    sgd_elem<MOM, NEST>(wv.z, uv.z, gv.z, lr, m, lam);
-    sgd_elem<MOM, NEST>(wv.w, uv.w, gv.w, lr, m, lam);
+    sgd_elem<MOM, NEST>(wv.x, uv.x, gv.x, lr, m, lam, sgn != 0);
+    sgd_elem<MOM, NEST>(wv.y, uv.y, gv.y, lr, m, lam, sgn != 0);
+    sgd_elem<MOM, NEST>(wv.z, uv.z, gv.z, lr, m, lam, sgn != 0);
+    sgd_elem<MOM, NEST>(wv.w, uv.w, gv.w, lr, m, lam, sgn != 0);
     if (MOM) __stcs(u + i, uv);
     __stcs(w + i, wv);
     if (SHADOW) {
@@ -228,10 +229,12 @@ __global__ void __launch_bounds__(256) sgd_update_kernel(
 }
 
 // ---------------------------------------------------------------------------------------------
-// K-way average.  A warp owns a 128-byte column block (8 float4) of every replica: lane
-// (r = lane / 8, c = lane % 8) sums replicas r, r + 4, r + 8, ... of float4 column c (each load
-// instruction reads four full 128-byte lines), the four partial sums are combined with two
-// butterfly shuffles, and every lane writes the mean back to its replicas (fp32 and bf16).
+// K-way average.  A thread owns one float4 column of every replica of its group and forms the
+// mean as w^0 + (1/K) sum_k (w^k - w^0), summing in replica order with eight loads in flight (a
+// warp's load instruction reads 512 contiguous bytes of one replica); it writes the mean back to
+// every replica (fp32 and bf16).  The differences are small and nearly exact while the replicas
+// stay close, so the mean carries about one rounding of w instead of K, and the mean of identical
+// replicas is exactly that replica for every K.
 template <bool SHADOW>
 __global__ void __launch_bounds__(256) kway_average_kernel(float4* __restrict__ W,
                                                            uint2* __restrict__ Wb, int K,
@@ -239,56 +242,248 @@ __global__ void __launch_bounds__(256) kway_average_kernel(float4* __restrict__ 
   // blockIdx.y selects a group of K consecutive replicas (one group for the global average)
   W += (int64_t)blockIdx.y * K * d4;
   if (SHADOW) Wb += (int64_t)blockIdx.y * K * d4;
-  const int lane = threadIdx.x & 31;
-  const int r = lane >> 3, c = lane & 7;
-  const int64_t nblk = (d4 + 7) / 8;
-  const int64_t warps = (int64_t)gridDim.x * (blockDim.x >> 5);
   const float invK = 1.0f / (float)K;
   const bool exactK = (K & (K - 1)) == 0;
-  for (int64_t blk = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); blk < nblk;
-       blk += warps) {
-    const int64_t col = blk * 8 + c;
-    const bool ok = col < d4;
-    const float4 zero4 = make_float4(0.f, 0.f, 0.f, 0.f);
-    float4 s = zero4;
-    // Batches of eight replicas per lane (r, r + 4, ..., r + 28): all loads of a batch are issued
-    // before any is summed, so up to 8 x 16 B per lane are in flight.
-    for (int k = r; k < K; k += 32) {
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t col = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; col < d4; col += stride) {
+    const float4 w0 = W[col];
+    float4 s = make_float4(0.f, 0.f, 0.f, 0.f);
+    int k = 0;
+    for (; k + 8 <= K; k += 8) {
       float4 v[8];
 #pragma unroll
-      for (int q = 0; q < 8; ++q)
-        v[q] = (ok && k + 4 * q < K) ? __ldcs(W + (int64_t)(k + 4 * q) * d4 + col) : zero4;
+      for (int q = 0; q < 8; ++q) v[q] = __ldcs(W + (int64_t)(k + q) * d4 + col);
 #pragma unroll
       for (int q = 0; q < 8; ++q) {
-        s.x += v[q].x;
-        s.y += v[q].y;
-        s.z += v[q].z;
-        s.w += v[q].w;
+        s.x += v[q].x - w0.x;
+        s.y += v[q].y - w0.y;
+        s.z += v[q].z - w0.z;
+        s.w += v[q].w - w0.w;
       }
     }
-#pragma unroll
-    for (int o = 8; o <= 16; o <<= 1) {
-      s.x += __shfl_xor_sync(0xffffffffu, s.x, o);
-      s.y += __shfl_xor_sync(0xffffffffu, s.y, o);
-      s.z += __shfl_xor_sync(0xffffffffu, s.z, o);
-      s.w += __shfl_xor_sync(0xffffffffu, s.w, o);
+    for (; k < K; ++k) {
+      const float4 v = __ldcs(W + (int64_t)k * d4 + col);
+      s.x += v.x - w0.x;
+      s.y += v.y - w0.y;
+      s.z += v.z - w0.z;
+      s.w += v.w - w0.w;
     }
     float4 mean;
     if (exactK) {
-      mean = make_float4(s.x * invK, s.y * invK, s.z * invK, s.w * invK);
+      mean = make_float4(fmaf(s.x, invK, w0.x), fmaf(s.y, invK, w0.y), fmaf(s.z, invK, w0.z),
+                         fmaf(s.w, invK, w0.w));
     } else {
-      mean = make_float4(s.x / (float)K, s.y / (float)K, s.z / (float)K, s.w / (float)K);
+      mean = make_float4(w0.x + s.x / (float)K, w0.y + s.y / (float)K, w0.z + s.z / (float)K,
+                         w0.w + s.w / (float)K);
     }
-    if (ok) {
-      uint2 o;
-      if (SHADOW) {
-        o.x = (uint32_t)f2bf(mean.x) | ((uint32_t)f2bf(mean.y) << 16);
-        o.y = (uint32_t)f2bf(mean.z) | ((uint32_t)f2bf(mean.w) << 16);
+    uint2 o;
+    if (SHADOW) {
+      o.x = (uint32_t)f2bf(mean.x) | ((uint32_t)f2bf(mean.y) << 16);
+      o.y = (uint32_t)f2bf(mean.z) | ((uint32_t)f2bf(mean.w) << 16);
+    }
+    for (int kk = 0; kk < K; ++kk) {
+      __stcs(W + (int64_t)kk * d4 + col, mean);
+      if (SHADOW) __stcs(Wb + (int64_t)kk * d4 + col, o);
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------------------------
+// Synchronisation variants.  L1 norms of the replicas' model differences: a block owns a chunk of
+// kL1Chunk float4 columns, loads w_ref there once and walks the replicas; each replica's chunk sum
+// is a fixed-shape reduction (thread, warp shuffle, warps in order), and l1_finalize_kernel adds
+// the chunk sums in a fixed-shape tree, so the norms are deterministic.
+constexpr int kL1Threads = 256;
+constexpr int kL1PerThread = 4;
+constexpr int kL1Chunk = kL1Threads * kL1PerThread;
+constexpr int kL1MaxK = 1024;  // shared memory holds one value per warp and replica
+
+template <bool EF>
+__global__ void __launch_bounds__(kL1Threads) l1_partial_kernel(const float4* __restrict__ W,
+                                                                const float4* __restrict__ wref,
+                                                                const float4* __restrict__ E,
+                                                                int K, int64_t d4, int nq,
+                                                                float* __restrict__ part) {
+  extern __shared__ float red[];  // [kL1Threads / 32][K]
+  const int q = blockIdx.x, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int64_t base = (int64_t)q * kL1Chunk + threadIdx.x;
+  float4 r[kL1PerThread];
+  bool ok[kL1PerThread];
+#pragma unroll
+  for (int j = 0; j < kL1PerThread; ++j) {
+    const int64_t i = base + (int64_t)j * kL1Threads;
+    ok[j] = i < d4;
+    r[j] = ok[j] ? wref[i] : make_float4(0.f, 0.f, 0.f, 0.f);
+  }
+  // replicas per batch: 32 loads in flight per thread before any is reduced
+  constexpr int KB = EF ? 4 : 8;
+  for (int k0 = 0; k0 < K; k0 += KB) {
+    float4 v[KB][kL1PerThread], e[KB][kL1PerThread];
+#pragma unroll
+    for (int b = 0; b < KB; ++b)
+#pragma unroll
+      for (int j = 0; j < kL1PerThread; ++j) {
+        const bool in = ok[j] && k0 + b < K;
+        const int64_t i = (int64_t)(k0 + b) * d4 + base + (int64_t)j * kL1Threads;
+        v[b][j] = in ? __ldcs(W + i) : r[j];
+        e[b][j] = (EF && in) ? __ldcs(E + i) : make_float4(0.f, 0.f, 0.f, 0.f);
       }
-      for (int kk = r; kk < K; kk += 4) {
-        __stcs(W + (int64_t)kk * d4 + col, mean);
-        if (SHADOW) __stcs(Wb + (int64_t)kk * d4 + col, o);
+    float s[KB];
+#pragma unroll
+    for (int b = 0; b < KB; ++b) {
+      s[b] = 0.f;
+#pragma unroll
+      for (int j = 0; j < kL1PerThread; ++j)
+        s[b] += fabsf(r[j].x - v[b][j].x + e[b][j].x) + fabsf(r[j].y - v[b][j].y + e[b][j].y) +
+                fabsf(r[j].z - v[b][j].z + e[b][j].z) + fabsf(r[j].w - v[b][j].w + e[b][j].w);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1)
+#pragma unroll
+      for (int b = 0; b < KB; ++b) s[b] += __shfl_xor_sync(0xffffffffu, s[b], o);
+    if (lane == 0)
+#pragma unroll
+      for (int b = 0; b < KB; ++b)
+        if (k0 + b < K) red[warp * K + k0 + b] = s[b];
+  }
+  __syncthreads();
+  for (int k = threadIdx.x; k < K; k += kL1Threads) {
+    float s = 0.f;
+    for (int w = 0; w < kL1Threads / 32; ++w) s += red[w * K + k];
+    part[(int64_t)k * nq + q] = s;
+  }
+}
+
+// p[k] = (sum of replica k's chunk sums) / d_canon: one block per replica, each thread adds a fixed
+// stride of chunks in fp64, then a fixed-shape tree over the block.
+__global__ void __launch_bounds__(256) l1_finalize_kernel(const float* __restrict__ part, int nq,
+                                                          double d_canon, float* __restrict__ p) {
+  __shared__ double red[256];
+  const int k = blockIdx.x;
+  double s = 0.0;
+  for (int q = threadIdx.x; q < nq; q += blockDim.x) s += part[(int64_t)k * nq + q];
+  red[threadIdx.x] = s;
+  __syncthreads();
+  for (int w = blockDim.x / 2; w > 0; w >>= 1) {
+    if (threadIdx.x < w) red[threadIdx.x] += red[threadIdx.x + w];
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) p[k] = (float)(red[0] / d_canon);
+}
+
+// One thread per float4 column: sum_k sign(Delta_k) p_k, the new synchronised model, the error
+// memories (EF) and the broadcast to every replica.
+template <bool EF, bool SHADOW>
+__global__ void __launch_bounds__(256) sign_sync_kernel(float4* __restrict__ W, uint2* __restrict__ Wb,
+                                                        float4* __restrict__ wref, float4* __restrict__ E,
+                                                        const float* __restrict__ p, int K,
+                                                        int64_t d4) {
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < d4; i += stride) {
+    const float4 r = wref[i];
+    float acc[4] = {0.f, 0.f, 0.f, 0.f};
+    // one replica's contribution: sign(Delta_k) p_k, and (EF) the residual left in e^k
+    auto add = [&](int k, const float4 b, const float4 e4) {
+      float dv[4] = {r.x - b.x, r.y - b.y, r.z - b.z, r.w - b.w};
+      if (EF) {
+        dv[0] += e4.x;
+        dv[1] += e4.y;
+        dv[2] += e4.z;
+        dv[3] += e4.w;
       }
+      const float pk = p[k];
+      float sp[4];
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        sp[j] = (dv[j] > 0.f ? 1.f : (dv[j] < 0.f ? -1.f : 0.f)) * pk;
+        acc[j] += sp[j];
+      }
+      if (EF)
+        __stcs(E + (int64_t)k * d4 + i,
+               make_float4(dv[0] - sp[0], dv[1] - sp[1], dv[2] - sp[2], dv[3] - sp[3]));
+    };
+    const float4 zero4 = make_float4(0.f, 0.f, 0.f, 0.f);
+    int k = 0;
+    for (; k + 4 <= K; k += 4) {
+      float4 b[4], e[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        b[q] = __ldcs(W + (int64_t)(k + q) * d4 + i);
+        e[q] = EF ? __ldcs(E + (int64_t)(k + q) * d4 + i) : zero4;
+      }
+#pragma unroll
+      for (int q = 0; q < 4; ++q) add(k + q, b[q], e[q]);
+    }
+    for (; k < K; ++k)
+      add(k, __ldcs(W + (int64_t)k * d4 + i), EF ? __ldcs(E + (int64_t)k * d4 + i) : zero4);
+    const float fk = (float)K;
+    const float4 nr = make_float4(r.x - acc[0] / fk, r.y - acc[1] / fk, r.z - acc[2] / fk, r.w - acc[3] / fk);
+    wref[i] = nr;
+    uint2 o;
+    if (SHADOW) {
+      o.x = (uint32_t)f2bf(nr.x) | ((uint32_t)f2bf(nr.y) << 16);
+      o.y = (uint32_t)f2bf(nr.z) | ((uint32_t)f2bf(nr.w) << 16);
+    }
+    for (int kk = 0; kk < K; ++kk) {
+      __stcs(W + (int64_t)kk * d4 + i, nr);
+      if (SHADOW) __stcs(Wb + (int64_t)kk * d4 + i, o);
+    }
+  }
+}
+
+// Global momentum: ug = mg ug + (wref - mean_k w^k) / lr, wref -= lr ug, broadcast.  The model
+// difference is accumulated as sum_k (wref - w^k) (in replica order): each term is exact or nearly
+// so while w^k stays close to wref, so the difference keeps fp32 relative accuracy instead of
+// inheriting the rounding error of a mean of large weights (a one-step round moves w by ~1e-3 of
+// its size, where the mean's rounding alone would cost ~1e-4 relative in ug).
+template <bool SHADOW>
+__global__ void __launch_bounds__(256) gm_sync_kernel(float4* __restrict__ W, uint2* __restrict__ Wb,
+                                                      float4* __restrict__ wref, float4* __restrict__ ug,
+                                                      int K, int64_t d4, float lr, float mg) {
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < d4; i += stride) {
+    const float4 r = wref[i];
+    float m[4] = {0.f, 0.f, 0.f, 0.f};
+    int k = 0;
+    for (; k + 8 <= K; k += 8) {
+      float4 b[8];
+#pragma unroll
+      for (int q = 0; q < 8; ++q) b[q] = __ldcs(W + (int64_t)(k + q) * d4 + i);
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        m[0] += r.x - b[q].x;
+        m[1] += r.y - b[q].y;
+        m[2] += r.z - b[q].z;
+        m[3] += r.w - b[q].w;
+      }
+    }
+    for (; k < K; ++k) {
+      const float4 b = __ldcs(W + (int64_t)k * d4 + i);
+      m[0] += r.x - b.x;
+      m[1] += r.y - b.y;
+      m[2] += r.z - b.z;
+      m[3] += r.w - b.w;
+    }
+    float4 u = ug[i];
+    const float rr[4] = {r.x, r.y, r.z, r.w};
+    float uu[4] = {u.x, u.y, u.z, u.w}, nr[4];
+    const float klr = (float)K * lr;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      uu[j] = fmaf(mg, uu[j], m[j] / klr);
+      nr[j] = fmaf(-lr, uu[j], rr[j]);
+    }
+    ug[i] = make_float4(uu[0], uu[1], uu[2], uu[3]);
+    const float4 n4 = make_float4(nr[0], nr[1], nr[2], nr[3]);
+    wref[i] = n4;
+    uint2 o;
+    if (SHADOW) {
+      o.x = (uint32_t)f2bf(nr[0]) | ((uint32_t)f2bf(nr[1]) << 16);
+      o.y = (uint32_t)f2bf(nr[2]) | ((uint32_t)f2bf(nr[3]) << 16);
+    }
+    for (int kk = 0; kk < K; ++kk) {
+      __stcs(W + (int64_t)kk * d4 + i, n4);
+      if (SHADOW) __stcs(Wb + (int64_t)kk * d4 + i, o);
     }
   }
 }
@@ -438,7 +633,7 @@ cudaError_t launch_colsum_update(const void* dz, bool dz_bf16, int ld, int G, in
 
 cudaError_t launch_sgd_update(float* w, float* u, const float* g, uint16_t* wb, int64_t n, float lr,
                               float momentum, int nesterov, float weight_decay, int64_t period,
-                              int64_t decay_end, cudaStream_t stream) {
+                              int64_t decay_end, cudaStream_t stream, int sign_steps) {
   if (n <= 0) return cudaSuccess;
   if ((n & 3) || (period & 3) || (decay_end & 3)) return cudaErrorInvalidValue;
   const bool mom = momentum != 0.0f;
@@ -452,7 +647,8 @@ cudaError_t launch_sgd_update(float* w, float* u, const float* g, uint16_t* wb, 
   auto WB = reinterpret_cast<uint2*>(wb);
 #define LSGD_UPD(M, NE, S)                                                                     \
   sgd_update_kernel<M, NE, S><<<blocks, threads, 0, stream>>>(W, U, G, WB, n4, lr, momentum, \
-                                                              weight_decay, period, decay_end)
+                                                              weight_decay, period, decay_end, \
+                                                              sign_steps)
   const bool sh = wb != nullptr;
   if (!mom) {
     if (sh) LSGD_UPD(false, false, true); else LSGD_UPD(false, false, false);
@@ -474,9 +670,8 @@ cudaError_t launch_group_average(float* W, uint16_t* Wb, int Kp, int groups, int
   if (Kp < 1 || groups < 1 || d <= 0) return cudaSuccess;
   if ((d & 3) || groups > 65535) return cudaErrorInvalidValue;
   const int64_t d4 = d / 4;
-  const int64_t nblk = (d4 + 7) / 8;  // one warp per 128-byte column block
   const int threads = 256;
-  const int blocks = std::max(1, grid_for(nblk * 32, threads, 8) / groups);
+  const int blocks = std::max(1, grid_for(d4, threads, 8) / groups);
   dim3 grid(blocks, groups);
   if (Wb)
     kway_average_kernel<true><<<grid, threads, 0, stream>>>(reinterpret_cast<float4*>(W),
@@ -484,6 +679,59 @@ cudaError_t launch_group_average(float* W, uint16_t* Wb, int Kp, int groups, int
   else
     kway_average_kernel<false><<<grid, threads, 0, stream>>>(reinterpret_cast<float4*>(W), nullptr,
                                                              Kp, d4);
+  return cudaGetLastError();
+}
+
+int l1_chunks(int64_t d) { return (int)((d / 4 + kL1Chunk - 1) / kL1Chunk); }
+
+cudaError_t launch_l1_norms(const float* W, const float* wref, const float* E, int K, int64_t d,
+                            int64_t d_canon, float* part, float* p, cudaStream_t stream) {
+  if (K < 1 || K > kL1MaxK || d <= 0 || (d & 3)) return cudaErrorInvalidValue;
+  const int nq = l1_chunks(d);
+  const size_t smem = (size_t)(kL1Threads / 32) * K * sizeof(float);
+  auto W4 = reinterpret_cast<const float4*>(W);
+  auto R4 = reinterpret_cast<const float4*>(wref);
+  auto E4 = reinterpret_cast<const float4*>(E);
+  if (E)
+    l1_partial_kernel<true><<<nq, kL1Threads, smem, stream>>>(W4, R4, E4, K, d / 4, nq, part);
+  else
+    l1_partial_kernel<false><<<nq, kL1Threads, smem, stream>>>(W4, R4, E4, K, d / 4, nq, part);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  l1_finalize_kernel<<<K, 256, 0, stream>>>(part, nq, (double)d_canon, p);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_sign_sync(float* W, uint16_t* Wb, float* wref, float* E, const float* p, int K,
+                             int64_t d, cudaStream_t stream) {
+  if (K < 1 || d <= 0 || (d & 3)) return cudaErrorInvalidValue;
+  const int64_t d4 = d / 4;
+  const int blocks = grid_for(d4, 256, 8);
+  auto W4 = reinterpret_cast<float4*>(W);
+  auto R4 = reinterpret_cast<float4*>(wref);
+  auto E4 = reinterpret_cast<float4*>(E);
+  auto B2 = reinterpret_cast<uint2*>(Wb);
+  if (E) {
+    if (Wb) sign_sync_kernel<true, true><<<blocks, 256, 0, stream>>>(W4, B2, R4, E4, p, K, d4);
+    else sign_sync_kernel<true, false><<<blocks, 256, 0, stream>>>(W4, B2, R4, E4, p, K, d4);
+  } else {
+    if (Wb) sign_sync_kernel<false, true><<<blocks, 256, 0, stream>>>(W4, B2, R4, E4, p, K, d4);
+    else sign_sync_kernel<false, false><<<blocks, 256, 0, stream>>>(W4, B2, R4, E4, p, K, d4);
+  }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gm_sync(float* W, uint16_t* Wb, float* wref, float* ug, int K, int64_t d,
+                           float lr, float mg, cudaStream_t stream) {
+  if (K < 1 || d <= 0 || (d & 3) || !(lr > 0.f)) return cudaErrorInvalidValue;
+  const int64_t d4 = d / 4;
+  const int blocks = grid_for(d4, 256, 8);
+  auto W4 = reinterpret_cast<float4*>(W);
+  auto R4 = reinterpret_cast<float4*>(wref);
+  auto U4 = reinterpret_cast<float4*>(ug);
+  auto B2 = reinterpret_cast<uint2*>(Wb);
+  if (Wb) gm_sync_kernel<true><<<blocks, 256, 0, stream>>>(W4, B2, R4, U4, K, d4, lr, mg);
+  else gm_sync_kernel<false><<<blocks, 256, 0, stream>>>(W4, B2, R4, U4, K, d4, lr, mg);
   return cudaGetLastError();
 }
 

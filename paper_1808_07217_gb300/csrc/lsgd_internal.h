@@ -19,6 +19,7 @@ struct SgdParams {
   uint16_t* wb;  // bf16 shadow (may be NULL)
   float lr, mom, wd;
   int nesterov;
+  int sign;      // signSGD local steps: w -= lr sign(step)
 };
 
 // ---- element-wise / reduction kernels (kernels.cu) ----
@@ -48,7 +49,20 @@ cudaError_t launch_colsum_update(const void* dz, bool dz_bf16, int ld, int G, in
                                  int64_t gs, const SgdParams& sgd, cudaStream_t stream);
 cudaError_t launch_sgd_update(float* w, float* u, const float* g, uint16_t* wb, int64_t n, float lr,
                               float momentum, int nesterov, float weight_decay, int64_t period,
-                              int64_t decay_end, cudaStream_t stream);
+                              int64_t decay_end, cudaStream_t stream, int sign_steps = 0);
+// ---- synchronisation variants (Sec. C.3.1 global momentum; Algorithms 4 and 5) ----
+// p[k] = ||wref - W[k] (+ E[k])||_1 / d_canon, through per-chunk partials `part` [K][nq]
+// (nq = l1_chunks(d)), combined in chunk order.
+int l1_chunks(int64_t d);
+cudaError_t launch_l1_norms(const float* W, const float* wref, const float* E, int K, int64_t d,
+                            int64_t d_canon, float* part, float* p, cudaStream_t stream);
+// wref -= (1/K) sum_k sign(Delta_k) p[k], Delta_k = wref - W[k] (+ E[k]); E[k] = Delta_k - s p
+// when E != NULL; every replica (and its bf16 shadow) becomes wref.
+cudaError_t launch_sign_sync(float* W, uint16_t* Wb, float* wref, float* E, const float* p, int K,
+                             int64_t d, cudaStream_t stream);
+// ug = mg ug + (wref - mean_k W[k]) / lr; wref -= lr ug; every replica becomes wref.
+cudaError_t launch_gm_sync(float* W, uint16_t* Wb, float* wref, float* ug, int K, int64_t d,
+                           float lr, float mg, cudaStream_t stream);
 cudaError_t launch_kway_average(float* W, uint16_t* Wb, int K, int64_t d, cudaStream_t stream);
 // Average within each of `groups` groups of Kp consecutive replicas (replica stride d).
 cudaError_t launch_group_average(float* W, uint16_t* Wb, int Kp, int groups, int64_t d,

@@ -10,6 +10,7 @@
 #include <cstdio>
 #include <cstdlib>
 #include <array>
+#include <utility>
 #include <algorithm>
 #include <cstring>
 #include <string>
@@ -80,6 +81,12 @@ struct lsgd_ctx {
   std::string err;
   lsgd::ResNetPlan* rn = nullptr;
   // tracing (lsgd_profile_*)
+  // synchronisation state of the compressed / global-momentum averages
+  float* wref = nullptr;   // [d_pad] model at the start of the round
+  float* E = nullptr;      // [K][d_pad] error-feedback memories
+  float* ug = nullptr;     // [d_pad] global momentum
+  float* pnorm = nullptr;  // [K] ||Delta_k||_1 / d
+  float* l1part = nullptr; // [K][l1_chunks] partial sums
   bool prof_on = false;
   std::vector<cudaEvent_t> prof_pool;
   size_t prof_used = 0;
@@ -372,6 +379,7 @@ lsgd_status dense_backward(lsgd_ctx* c) {
     sgd.mom = (float)c->cfg.momentum;
     sgd.wd = (float)c->cfg.weight_decay;
     sgd.nesterov = c->cfg.nesterov;
+    sgd.sign = c->cfg.compress == LSGD_COMPRESS_SIGN;
   }
   auto sgd_at = [&](int64_t off) {
     lsgd::SgdParams p = sgd;
@@ -540,7 +548,7 @@ lsgd_status do_update(lsgd_ctx* c) {
   LSGD_LAUNCH(c, lsgd::launch_sgd_update(c->W, c->U, c->G, c->Wb, (int64_t)c->cfg.K * c->d_pad, lr,
                                          (float)c->cfg.momentum, c->cfg.nesterov,
                                          (float)c->cfg.weight_decay, c->wd_period, c->wd_end,
-                                         c->stream));
+                                         c->stream, c->cfg.compress == LSGD_COMPRESS_SIGN));
   return LSGD_OK;
 }
 
@@ -602,6 +610,13 @@ lsgd_status lsgd_create(const lsgd_config* cfg, const lsgd_allocator* alloc, voi
   if (c0.B_loc > 8192) return fail(nullptr, LSGD_EUNSUPPORTED, "B_loc must be <= 8192");
   if (c0.hier_block < 0 || (c0.hier_block > 0 && (c0.K % c0.hier_block || c0.hier_rounds < 1)))
     return fail(nullptr, LSGD_EINVAL, "hier_block must divide K and hier_rounds must be >= 1");
+  if (c0.compress < LSGD_COMPRESS_NONE || c0.compress > LSGD_COMPRESS_EF_SIGN || c0.global_momentum < 0.0 ||
+      ((c0.compress != LSGD_COMPRESS_NONE || c0.global_momentum > 0.0) && c0.hier_block > 0) ||
+      (c0.compress != LSGD_COMPRESS_NONE && c0.global_momentum > 0.0))
+    return fail(nullptr, LSGD_EINVAL,
+                "compress and global_momentum exclude each other and hierarchical averaging");
+  if (c0.compress != LSGD_COMPRESS_NONE && c0.K > 1024)
+    return fail(nullptr, LSGD_EINVAL, "compress supports K <= 1024");
   const lsgd_model& m = c0.model;
   if (m.kind == LSGD_MLP || m.kind == LSGD_LSQ) {
     if (m.n_layers < 1 || m.n_layers > LSGD_MAX_LAYERS)
@@ -684,6 +699,19 @@ lsgd_status lsgd_create(const lsgd_config* cfg, const lsgd_allocator* alloc, voi
   c->loss_hist = (float*)dalloc(c, (size_t)c->loss_cap * K * 4);
   c->row_loss = (float*)dalloc(c, (size_t)K * B * 4);
   c->flag = (int*)dalloc(c, 16);
+  const bool need_ref = c0.compress != LSGD_COMPRESS_NONE || c0.global_momentum > 0.0;
+  if (need_ref) {
+    c->wref = (float*)dalloc(c, (size_t)c->d_pad * 4);
+    c->pnorm = (float*)dalloc(c, (size_t)K * 4);
+    c->l1part = (float*)dalloc(c, (size_t)K * lsgd::l1_chunks(c->d_pad) * 4);
+    if (c0.compress == LSGD_COMPRESS_EF_SIGN) c->E = (float*)dalloc(c, n_rep * 4);
+    if (c0.global_momentum > 0.0) c->ug = (float*)dalloc(c, (size_t)c->d_pad * 4);
+    if (!c->wref || !c->pnorm || !c->l1part || (c0.compress == LSGD_COMPRESS_EF_SIGN && !c->E) ||
+        (c0.global_momentum > 0.0 && !c->ug)) {
+      fail(nullptr, LSGD_ENOMEM, "device allocation failed");
+      return bail(LSGD_ENOMEM);
+    }
+  }
   if (!c->W || !c->G || (c0.momentum != 0.0 && !c->U) || (c->bf16 && !c->Wb) || !c->idx ||
       !c->yb || !c->tb || !c->loss_hist || !c->row_loss || !c->flag) {
     fail(nullptr, LSGD_ENOMEM, "device allocation failed");
@@ -716,6 +744,12 @@ lsgd_status lsgd_create(const lsgd_config* cfg, const lsgd_allocator* alloc, voi
     return bail(LSGD_ECUDA);
   }
   c->launches += c->bf16 ? 2 : 1;
+  if (c->wref &&
+      cudaMemcpyAsync(c->wref, c->W, (size_t)c->d_pad * 4, cudaMemcpyDeviceToDevice, c->stream) !=
+          cudaSuccess) {
+    fail(nullptr, LSGD_ECUDA, "initial round-start model copy failed");
+    return bail(LSGD_ECUDA);
+  }
   cudaError_t e = cudaStreamSynchronize(c->stream);
   if (e != cudaSuccess) {
     fail_cuda(nullptr, e, "lsgd_create");
@@ -812,7 +846,21 @@ lsgd_status lsgd_local_step_batch(lsgd_ctx* c, const float* x, const void* lab, 
 lsgd_status lsgd_sync_average(lsgd_ctx* c) {
   if (!c) return fail(nullptr, LSGD_EINVAL, "NULL context");
   const int64_t e0 = prof_mark(c);
-  LSGD_LAUNCH(c, lsgd::launch_kway_average(c->W, c->Wb, c->cfg.K, c->d_pad, c->stream));
+  const int K = c->cfg.K;
+  if (c->cfg.compress != LSGD_COMPRESS_NONE) {
+    // Algorithms 4 / 5: sign-compressed model differences relative to the round start
+    LSGD_LAUNCH(c, lsgd::launch_l1_norms(c->W, c->wref, c->E, K, c->d_pad, c->d, c->l1part, c->pnorm,
+                                         c->stream));
+    c->launches++;  // launch_l1_norms runs two kernels (chunk sums, then their total)
+    LSGD_LAUNCH(c, lsgd::launch_sign_sync(c->W, c->Wb, c->wref, c->E, c->pnorm, K, c->d_pad, c->stream));
+  } else if (c->cfg.global_momentum > 0.0) {
+    // Sec. C.3.1 global momentum with the step size of the step that ended the round
+    const float lr = (float)lr_at(c->cfg, c->T, c->step > 0 ? c->step - 1 : 0);
+    LSGD_LAUNCH(c, lsgd::launch_gm_sync(c->W, c->Wb, c->wref, c->ug, K, c->d_pad, lr,
+                                        (float)c->cfg.global_momentum, c->stream));
+  } else {
+    LSGD_LAUNCH(c, lsgd::launch_kway_average(c->W, c->Wb, K, c->d_pad, c->stream));
+  }
   prof_span(c, LSGD_PH_AVERAGE, e0, prof_mark(c));
   c->syncs++;
   return LSGD_OK;
@@ -929,6 +977,9 @@ static lsgd_status set_vec(lsgd_ctx* c, float* buf, int k, const float* src, siz
     LSGD_TRY_CUDA(c, cudaMemcpyAsync(buf + (int64_t)k0 * c->d_pad + s.pad, src + s.canon,
                                      (size_t)s.len * 4, cudaMemcpyHostToDevice, c->stream));
   if (k < 0) LSGD_LAUNCH(c, lsgd::launch_broadcast(buf, c->cfg.K, c->d_pad, c->stream));
+  if (is_w && k < 0 && c->wref)
+    LSGD_TRY_CUDA(c, cudaMemcpyAsync(c->wref, c->W, (size_t)c->d_pad * 4, cudaMemcpyDeviceToDevice,
+                                     c->stream));
   if (is_w && c->Wb)
     LSGD_LAUNCH(c, lsgd::launch_to_bf16(c->W, c->Wb, (int64_t)c->cfg.K * c->d_pad, c->stream));
   LSGD_TRY_CUDA(c, cudaStreamSynchronize(c->stream));
@@ -941,6 +992,49 @@ lsgd_status lsgd_set_params(lsgd_ctx* c, int k, const float* src, size_t n) {
 
 lsgd_status lsgd_set_momentum(lsgd_ctx* c, int k, const float* src, size_t n) {
   return set_vec(c, c ? c->U : nullptr, k, src, n, false);
+}
+
+// The arrays behind lsgd_sync_state: the replica stride is d_pad for E and 0 for the others.
+static float* sync_state_buf(lsgd_ctx* c, int which, bool* per_replica) {
+  *per_replica = which == LSGD_STATE_ERROR;
+  switch (which) {
+    case LSGD_STATE_WREF: return c->wref;
+    case LSGD_STATE_ERROR: return c->E;
+    case LSGD_STATE_GLOBAL_MOMENTUM: return c->ug;
+    default: return nullptr;
+  }
+}
+
+lsgd_status lsgd_sync_state(lsgd_ctx* c, int which, int k, float* dst, size_t n) {
+  if (!c || !dst) return fail(c, LSGD_EINVAL, "NULL argument");
+  if (n != (size_t)c->d) return fail(c, LSGD_EINVAL, "n must equal lsgd_num_params()");
+  bool per = false;
+  float* buf = sync_state_buf(c, which, &per);
+  if (!buf) return fail(c, LSGD_ESTATE, "this configuration keeps no such synchronisation state");
+  if (per ? (k < 0 || k >= c->cfg.K) : k != 0)
+    return fail(c, LSGD_EINVAL, "replica index out of range for this state");
+  for (const Seg& s : c->segs)
+    LSGD_TRY_CUDA(c, cudaMemcpyAsync(dst + s.canon, buf + (int64_t)k * c->d_pad + s.pad,
+                                     (size_t)s.len * 4, cudaMemcpyDeviceToHost, c->stream));
+  LSGD_TRY_CUDA(c, cudaStreamSynchronize(c->stream));
+  return LSGD_OK;
+}
+
+lsgd_status lsgd_set_sync_state(lsgd_ctx* c, int which, int k, const float* src, size_t n) {
+  if (!c || !src) return fail(c, LSGD_EINVAL, "NULL argument");
+  if (n != (size_t)c->d) return fail(c, LSGD_EINVAL, "n must equal lsgd_num_params()");
+  bool per = false;
+  float* buf = sync_state_buf(c, which, &per);
+  if (!buf) return fail(c, LSGD_ESTATE, "this configuration keeps no such synchronisation state");
+  if (per ? (k < -1 || k >= c->cfg.K) : k != 0)
+    return fail(c, LSGD_EINVAL, "replica index out of range for this state");
+  const int k0 = k < 0 ? 0 : k;
+  for (const Seg& s : c->segs)
+    LSGD_TRY_CUDA(c, cudaMemcpyAsync(buf + (int64_t)k0 * c->d_pad + s.pad, src + s.canon,
+                                     (size_t)s.len * 4, cudaMemcpyHostToDevice, c->stream));
+  if (per && k < 0) LSGD_LAUNCH(c, lsgd::launch_broadcast(buf, c->cfg.K, c->d_pad, c->stream));
+  LSGD_TRY_CUDA(c, cudaStreamSynchronize(c->stream));
+  return LSGD_OK;
 }
 
 lsgd_status lsgd_losses(lsgd_ctx* c, float* dst, int64_t n_steps) {
@@ -1025,7 +1119,14 @@ lsgd_status lsgd_check_finite(lsgd_ctx* c) {
   return LSGD_OK;
 }
 
-static const uint64_t kMagic = 0x3230545043445347ULL;  // "GSDCPT02"
+static const uint64_t kMagic = 0x3330545043445347ULL;  // "GSDCPT03"
+
+// Bit mask of the state arrays a checkpoint holds after W: 1 momentum, 2 round-start model,
+// 4 error-feedback memories, 8 global momentum.  A checkpoint loads only into a context that
+// keeps exactly the same arrays.
+static int64_t state_mask(const lsgd_ctx* c) {
+  return (c->U ? 1 : 0) | (c->wref ? 2 : 0) | (c->E ? 4 : 0) | (c->ug ? 8 : 0);
+}
 
 lsgd_status lsgd_save(lsgd_ctx* c, const char* path) {
   if (!c || !path) return fail(c, LSGD_EINVAL, "NULL argument");
@@ -1033,18 +1134,25 @@ lsgd_status lsgd_save(lsgd_ctx* c, const char* path) {
   std::vector<float> buf(n);
   FILE* f = std::fopen(path, "wb");
   if (!f) return fail(c, LSGD_EIO, std::string("cannot open ") + path);
-  int64_t hdr[7] = {(int64_t)kMagic, c->cfg.K, c->d_pad, c->step, c->syncs, c->U ? 1 : 0,
+  int64_t hdr[7] = {(int64_t)kMagic, c->cfg.K, c->d_pad, c->step, c->syncs, state_mask(c),
                     c->block_syncs};
   bool ok = std::fwrite(hdr, sizeof(hdr), 1, f) == 1;
-  for (int which = 0; ok && which < (c->U ? 2 : 1); ++which) {
-    const float* src = which == 0 ? c->W : c->U;
-    cudaError_t e = cudaMemcpyAsync(buf.data(), src, n * 4, cudaMemcpyDeviceToHost, c->stream);
+  // w and u of every replica, then the synchronisation state the context keeps
+  std::vector<std::pair<const float*, size_t>> parts = {{c->W, n}};
+  if (c->U) parts.push_back({c->U, n});
+  if (c->wref) parts.push_back({c->wref, (size_t)c->d_pad});
+  if (c->E) parts.push_back({c->E, n});
+  if (c->ug) parts.push_back({c->ug, (size_t)c->d_pad});
+  for (size_t which = 0; ok && which < parts.size(); ++which) {
+    const float* src = parts[which].first;
+    const size_t cnt = parts[which].second;
+    cudaError_t e = cudaMemcpyAsync(buf.data(), src, cnt * 4, cudaMemcpyDeviceToHost, c->stream);
     if (e == cudaSuccess) e = cudaStreamSynchronize(c->stream);
     if (e != cudaSuccess) {
       std::fclose(f);
       return fail_cuda(c, e, "lsgd_save");
     }
-    ok = std::fwrite(buf.data(), 4, n, f) == n;
+    ok = std::fwrite(buf.data(), 4, cnt, f) == cnt;
   }
   ok = (std::fclose(f) == 0) && ok;
   if (!ok) return fail(c, LSGD_EIO, "write failed");
@@ -1057,19 +1165,25 @@ lsgd_status lsgd_load(lsgd_ctx* c, const char* path) {
   if (!f) return fail(c, LSGD_EIO, std::string("cannot open ") + path);
   int64_t hdr[7];
   if (std::fread(hdr, sizeof(hdr), 1, f) != 1 || hdr[0] != (int64_t)kMagic || hdr[1] != c->cfg.K ||
-      hdr[2] != c->d_pad || hdr[5] != (c->U ? 1 : 0)) {
+      hdr[2] != c->d_pad || hdr[5] != state_mask(c)) {
     std::fclose(f);
     return fail(c, LSGD_EIO, "checkpoint does not match this configuration");
   }
   const size_t n = (size_t)c->cfg.K * c->d_pad;
   std::vector<float> buf(n);
-  for (int which = 0; which < (c->U ? 2 : 1); ++which) {
-    if (std::fread(buf.data(), 4, n, f) != n) {
+  std::vector<std::pair<float*, size_t>> parts = {{c->W, n}};
+  if (c->U) parts.push_back({c->U, n});
+  if (c->wref) parts.push_back({c->wref, (size_t)c->d_pad});
+  if (c->E) parts.push_back({c->E, n});
+  if (c->ug) parts.push_back({c->ug, (size_t)c->d_pad});
+  for (size_t which = 0; which < parts.size(); ++which) {
+    float* dst = parts[which].first;
+    const size_t cnt = parts[which].second;
+    if (std::fread(buf.data(), 4, cnt, f) != cnt) {
       std::fclose(f);
       return fail(c, LSGD_EIO, "truncated checkpoint");
     }
-    float* dst = which == 0 ? c->W : c->U;
-    cudaError_t e = cudaMemcpyAsync(dst, buf.data(), n * 4, cudaMemcpyHostToDevice, c->stream);
+    cudaError_t e = cudaMemcpyAsync(dst, buf.data(), cnt * 4, cudaMemcpyHostToDevice, c->stream);
     if (e == cudaSuccess) e = cudaStreamSynchronize(c->stream);
     if (e != cudaSuccess) {
       std::fclose(f);

@@ -54,7 +54,8 @@ def test_struct_layout_matches_header(P):
              offsetof(lsgd_config, lr), offsetof(lsgd_config, momentum),
              offsetof(lsgd_config, seed), offsetof(lsgd_config, precision),
              offsetof(lsgd_config, fused_update), sizeof(lsgd_profile));
-      printf("%zu %zu\n", offsetof(lsgd_config, hier_block), offsetof(lsgd_config, hier_rounds));
+      printf("%zu %zu %zu %zu\n", offsetof(lsgd_config, hier_block), offsetof(lsgd_config, hier_rounds),
+             offsetof(lsgd_config, compress), offsetof(lsgd_config, global_momentum));
       return 0;
     }
     """
@@ -70,7 +71,7 @@ def test_struct_layout_matches_header(P):
     want = [ctypes.sizeof(C), ctypes.sizeof(P.Model), ctypes.sizeof(P.LrSchedule),
             ctypes.sizeof(P.Allocator), C.model.offset, C.lr.offset, C.momentum.offset,
             C.seed.offset, C.precision.offset, C.fused_update.offset, ctypes.sizeof(P.Profile),
-            C.hier_block.offset, C.hier_rounds.offset]
+            C.hier_block.offset, C.hier_rounds.offset, C.compress.offset, C.global_momentum.offset]
     assert got == want
 
 

@@ -30,6 +30,8 @@ _lib = None
 
 DENSE, LSQ, RESNET20 = 0, 1, 2
 COMPRESS_NONE, COMPRESS_SIGN, COMPRESS_EF_SIGN = 0, 1, 2
+HWARM_NONE, HWARM_LINEAR, HWARM_EXPONENTIAL, HWARM_CONSTANT = 0, 1, 2, 3
+SAMPLE_SHARDS, SAMPLE_RESHUFFLE = 0, 1
 INIT_ZERO, INIT_HE = 0, 1
 MAX_LAYERS = 8
 
@@ -67,6 +69,9 @@ class Cfg(ctypes.Structure):
         ("hier_rounds", ctypes.c_int),
         ("compress", ctypes.c_int),
         ("global_momentum", ctypes.c_double),
+        ("h_warmup", ctypes.c_int),
+        ("h_warmup_epochs", ctypes.c_double),
+        ("sampling", ctypes.c_int),
     ]
 
 
@@ -74,7 +79,11 @@ def make_cfg(kind=DENSE, widths=(3072, 10), has_bias=True, bf16=False, K=1, B=1,
              t_switch=-1, T=1, N=1, base_lr=0.1, scale_by_K=False, warmup_epochs=0.0,
              milestones=(), decay=0.1, momentum=0.0, nesterov=False, weight_decay=0.0, seed=0,
              in_hwc=(32, 32, 3), n_classes=10, base_ch=16, res_blocks=3, hier_block=0,
-             hier_rounds=1, compress=0, global_momentum=0.0) -> Cfg:
+             hier_rounds=1, compress=0, global_momentum=0.0, h_warmup=HWARM_NONE,
+             h_warmup_epochs=0.0, sampling=SAMPLE_SHARDS) -> Cfg:
+    if h_warmup != HWARM_NONE and (hier_block > 0 or t_switch >= 0):
+        raise ValueError("local-step warm-up replaces the post-local switch and is not combined "
+                         "with hierarchical averaging")
     c = Cfg()
     c.kind = kind
     if kind != RESNET20:
@@ -104,6 +113,9 @@ def make_cfg(kind=DENSE, widths=(3072, 10), has_bias=True, bf16=False, K=1, B=1,
     c.hier_rounds = int(hier_rounds)
     c.compress = int(compress)
     c.global_momentum = float(global_momentum)
+    c.h_warmup = int(h_warmup)
+    c.h_warmup_epochs = float(h_warmup_epochs)
+    c.sampling = int(sampling)
     return c
 
 
@@ -149,6 +161,12 @@ def lib():
             L.oracle_block_average.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_int64, dp]
             L.oracle_sync_kind.argtypes = [cfgp, ctypes.c_int64]
             L.oracle_sync_kind.restype = ctypes.c_int
+            L.oracle_epoch.argtypes = [cfgp, ctypes.c_int64]
+            L.oracle_epoch.restype = ctypes.c_int64
+            L.oracle_round_length.argtypes = [cfgp, ctypes.c_int64]
+            L.oracle_round_length.restype = ctypes.c_int64
+            L.oracle_permute.argtypes = [cfgp, ctypes.c_int64, ctypes.c_int64]
+            L.oracle_permute.restype = ctypes.c_int64
             L.oracle_run_counted.argtypes = [cfgp, fp, ip, fp, dp, dp, ctypes.c_int64,
                                              ctypes.c_int64, dp, P(ctypes.c_int64),
                                              P(ctypes.c_int64)]
@@ -231,6 +249,18 @@ def sgd_update(c: Cfg, lr: float, w, u, g):
 
 def lr(c: Cfg, s: int) -> float:
     return float(lib().oracle_lr(ctypes.byref(c), int(s)))
+
+
+def epoch(c: Cfg, s: int) -> int:
+    return int(lib().oracle_epoch(ctypes.byref(c), int(s)))
+
+
+def round_length(c: Cfg, s0: int) -> int:
+    return int(lib().oracle_round_length(ctypes.byref(c), int(s0)))
+
+
+def permute(c: Cfg, e: int, i: int) -> int:
+    return int(lib().oracle_permute(ctypes.byref(c), int(e), int(i)))
 
 
 def is_round_end(c: Cfg, s: int) -> bool:

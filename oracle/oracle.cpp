@@ -226,9 +226,53 @@ void oracle_philox4x32_10(const uint32_t ctr[4], const uint32_t key[2], uint32_t
 // from the worker's local data).  The data is split into K contiguous shards of floor(N/K) points;
 // draw j uses word (j mod 4) of Philox(counter = (j div 4, s, k, 0), key = seed) and maps it to the
 // shard by the high half of a 32x32-bit product.
+int64_t oracle_epoch(const oracle_cfg* c, int64_t s) {
+  return s * (int64_t)c->K * c->B / c->N;
+}
+
+// The reshuffling sampler's permutation of [0, N) for epoch e: a balanced Feistel network of four
+// rounds (Luby and Rackoff) on the smallest even-bit domain 2^(2h) >= N, with round functions
+// F_r(R) = word 0 of Philox4x32-10((R, e, r, 2), seed) masked to h bits, restricted to [0, N) by
+// cycle walking (Black and Rogaway): apply the network until the value falls inside [0, N).  Each
+// network is a bijection of the domain, so the walk from any i < N returns to [0, N) and the result
+// is a bijection of [0, N).
+int64_t oracle_permute(const oracle_cfg* c, int64_t e, int64_t i) {
+  int h = 1;
+  while ((int64_t)1 << (2 * h) < c->N) ++h;
+  const uint64_t mask = ((uint64_t)1 << h) - 1;
+  uint64_t x = (uint64_t)i;
+  do {
+    uint64_t L = x >> h, R = x & mask;
+    for (uint32_t r = 0; r < 4; ++r) {
+      Philox4 ctr = {{(uint32_t)R, (uint32_t)e, r, 2u}};
+      const Philox4 f = philox4x32_10(ctr, (uint32_t)c->seed, (uint32_t)(c->seed >> 32));
+      const uint64_t nR = L ^ ((uint64_t)f.v[0] & mask);
+      L = R;
+      R = nR;
+    }
+    x = (L << h) | R;
+  } while (x >= (uint64_t)c->N);
+  return (int64_t)x;
+}
+
+// I^k_s.  Shards: static contiguous shard of S = floor(N / K) points, B uniform draws with
+// replacement.  Reshuffle: in epoch e the data is pi_e(0), ..., pi_e(N - 1), worker k's partition
+// is positions [k S, (k + 1) S) of it, and the worker's t-th step of the epoch takes the next B
+// positions of its partition, (t B + j) mod S.
 void oracle_sample_indices(const oracle_cfg* c, int k, int64_t s, int32_t* out) {
   const uint64_t S = (uint64_t)(c->N / c->K);
   const uint64_t base = (uint64_t)k * S;
+  if (c->sampling == ORACLE_SAMPLE_RESHUFFLE) {
+    const int64_t e = oracle_epoch(c, s);
+    const int64_t KB = (int64_t)c->K * c->B;
+    const int64_t first = (e * c->N + KB - 1) / KB;  // first step of epoch e
+    const int64_t t = s - first;
+    for (int j = 0; j < c->B; ++j) {
+      const uint64_t pos = ((uint64_t)t * c->B + j) % S;
+      out[j] = (int32_t)oracle_permute(c, e, (int64_t)(base + pos));
+    }
+    return;
+  }
   for (int j = 0; j < c->B; ++j) {
     Philox4 ctr = {{(uint32_t)(j >> 2), (uint32_t)s, (uint32_t)k, 0u}};
     Philox4 r = philox4x32_10(ctr, (uint32_t)c->seed, (uint32_t)(c->seed >> 32));
@@ -297,6 +341,28 @@ double oracle_lr(const oracle_cfg* c, int64_t s) {
   return lr;
 }
 
+// Local-step warm-up: the round that starts in epoch e < P = h_warmup_epochs has length
+//   linear:      1 + floor((H - 1) e / P)
+//   exponential: min(H, 2^floor(e log2(H) / P))   (H = 8 over P = 3 epochs: 1, 2, 4, then 8)
+//   constant:    1
+// and H once e >= P.
+int64_t oracle_round_length(const oracle_cfg* c, int64_t s0) {
+  if (c->h_warmup == ORACLE_HWARM_NONE) return c->H;
+  const double e = (double)oracle_epoch(c, s0), P = c->h_warmup_epochs;
+  if (e >= P) return c->H;
+  switch (c->h_warmup) {
+    case ORACLE_HWARM_LINEAR:
+      return 1 + (int64_t)std::floor((double)(c->H - 1) * e / P);
+    case ORACLE_HWARM_EXPONENTIAL: {
+      const double x = std::floor(e * std::log2((double)c->H) / P);
+      const double len = std::pow(2.0, x);
+      return len < (double)c->H ? (int64_t)len : c->H;
+    }
+    default:
+      return 1;
+  }
+}
+
 // Whether the models are averaged after local step s (0-based): post-local SGD (Sec. 3) uses
 // H_(t) = 1 before the switch step t' and H after it; the last step of the run always ends a round
 // so the returned model is the average.
@@ -304,7 +370,14 @@ int oracle_is_round_end(const oracle_cfg* c, int64_t s) {
   if (s == c->T - 1) return 1;
   if (c->t_switch >= 0 && s < c->t_switch) return 1;
   const int64_t start = c->t_switch > 0 ? c->t_switch : 0;
-  return ((s + 1 - start) % c->H) == 0;
+  if (c->h_warmup == ORACLE_HWARM_NONE) return ((s + 1 - start) % c->H) == 0;
+  // rounds of varying length, walked from the first one
+  int64_t r0 = start;
+  for (;;) {
+    const int64_t len = oracle_round_length(c, r0);
+    if (s < r0 + len) return s == r0 + len - 1;
+    r0 += len;
+  }
 }
 
 // Which average ends local step s.  Without hierarchy: the global average at every round end.

@@ -53,7 +53,20 @@ typedef struct {
   int compress;
   /* global momentum (Sec. C.3.1): > 0 applies momentum m_g to the averaged model difference */
   double global_momentum;
+  /* local-step warm-up (Sec. C, "warm-up of the number of local SGD steps"; Sec. 4's ImageNet
+     runs): the round that starts in epoch e < h_warmup_epochs has ORACLE_HWARM_* length instead
+     of H */
+  int h_warmup;
+  double h_warmup_epochs;
+  /* ORACLE_SAMPLE_SHARDS: static contiguous shards, uniform with replacement;
+     ORACLE_SAMPLE_RESHUFFLE: a fresh global permutation every epoch, disjoint worker partitions,
+     each worker passing through its partition in order (Sec. 4 / A.4 training procedure) */
+  int sampling;
 } oracle_cfg;
+
+enum { ORACLE_HWARM_NONE = 0, ORACLE_HWARM_LINEAR = 1, ORACLE_HWARM_EXPONENTIAL = 2,
+       ORACLE_HWARM_CONSTANT = 3 };
+enum { ORACLE_SAMPLE_SHARDS = 0, ORACLE_SAMPLE_RESHUFFLE = 1 };
 
 enum { ORACLE_COMPRESS_NONE = 0, ORACLE_COMPRESS_SIGN = 1, ORACLE_COMPRESS_EF_SIGN = 2 };
 
@@ -63,6 +76,12 @@ int64_t oracle_num_params(const oracle_cfg* c);
 void oracle_weight_decay_mask(const oracle_cfg* c, uint8_t* mask);
 void oracle_philox4x32_10(const uint32_t ctr[4], const uint32_t key[2], uint32_t out[4]);
 void oracle_sample_indices(const oracle_cfg* c, int k, int64_t s, int32_t* out);
+/* Epoch of local step s: floor(s K B / N) (samples all workers accessed before it, over N). */
+int64_t oracle_epoch(const oracle_cfg* c, int64_t s);
+/* Length of the local-SGD round that starts at step s0. */
+int64_t oracle_round_length(const oracle_cfg* c, int64_t s0);
+/* pi_e(i): the epoch-e permutation of [0, N) of the reshuffling sampler. */
+int64_t oracle_permute(const oracle_cfg* c, int64_t e, int64_t i);
 void oracle_init_params(const oracle_cfg* c, int init_kind, double* w);
 double oracle_loss_grad(const oracle_cfg* c, const double* w, const float* X, const int32_t* y,
                         const float* t, const int32_t* idx, int B, double* grad);

@@ -114,7 +114,32 @@ typedef struct {
   double global_momentum;/* m_g > 0: global momentum at every average (Sec. C.3.1):
                             u_g = m_g u_g + (w_ref - mean_k w^k) / gamma, w_ref -= gamma u_g.
                             Not with compress or hier_block. */
+  int h_warmup;          /* lsgd_h_warmup: local-step warm-up (Sec. C; Sec. 4's ImageNet runs).  The
+                            round starting at step s0 in epoch e = floor(s0 K B_loc / N) <
+                            h_warmup_epochs = P has 1 + floor((H-1) e / P) steps (LINEAR),
+                            min(H, 2^floor(e log2(H) / P)) (EXPONENTIAL) or 1 (CONSTANT); H from
+                            epoch P on.  Replaces the post-local switch (t_switch must be < 0);
+                            not with hier_block. */
+  double h_warmup_epochs;
+  int sampling;          /* lsgd_sampling */
 } lsgd_config;
+
+typedef enum {
+  LSGD_HWARM_NONE = 0,
+  LSGD_HWARM_LINEAR = 1,
+  LSGD_HWARM_EXPONENTIAL = 2,
+  LSGD_HWARM_CONSTANT = 3
+} lsgd_h_warmup;
+
+typedef enum {
+  LSGD_SAMPLE_SHARDS = 0,    /* static contiguous shards of S = floor(N/K) points, B uniform draws
+                                with replacement per step: k S + mulhi(Philox word, S) */
+  LSGD_SAMPLE_RESHUFFLE = 1  /* Sec. 4 / A.4: the data is re-permuted globally every epoch and
+                                partitioned disjointly; worker k's t-th step of epoch e takes
+                                pi_e(k S + (t B + j) mod S), j < B, where pi_e is a four-round
+                                Feistel permutation of [0, N) keyed by Philox (seed, e) with cycle
+                                walking; N < 2^31 */
+} lsgd_sampling;
 
 typedef enum {
   LSGD_COMPRESS_NONE = 0,
@@ -213,6 +238,13 @@ lsgd_status lsgd_check_finite(lsgd_ctx* ctx);
  * state is stored.  lsgd_load requires a context created with the same config. */
 lsgd_status lsgd_save(lsgd_ctx* ctx, const char* path);
 lsgd_status lsgd_load(lsgd_ctx* ctx, const char* path);
+
+/* The schedule a context created from cfg follows, computed on the host without a GPU: for local
+ * steps s = 0 .. n_steps-1, lr[s] = gamma(s) (Sec. A.3 warm-up, Sec. A.4 decays) and sync_kind[s] =
+ * the average that ends step s (0 none, 1 block average, 2 global average: post-local switch,
+ * local-step warm-up, hierarchical rounds).  Either array may be NULL.  Validates cfg exactly as
+ * lsgd_create does. */
+lsgd_status lsgd_schedule(const lsgd_config* cfg, int64_t n_steps, double* lr, int32_t* sync_kind);
 
 int64_t lsgd_num_params(const lsgd_ctx* ctx);   /* d, canonical (unpadded) */
 int64_t lsgd_step_count(const lsgd_ctx* ctx);   /* local steps taken so far (next step's s) */

@@ -23,6 +23,8 @@ FP32, BF16 = 0, 1
 INIT_ZERO, INIT_HE = 0, 1
 COMPRESS_NONE, COMPRESS_SIGN, COMPRESS_EF_SIGN = 0, 1, 2
 STATE_WREF, STATE_ERROR, STATE_GLOBAL_MOMENTUM = 0, 1, 2
+HWARM_NONE, HWARM_LINEAR, HWARM_EXPONENTIAL, HWARM_CONSTANT = 0, 1, 2, 3
+SAMPLE_SHARDS, SAMPLE_RESHUFFLE = 0, 1
 
 OK, EINVAL, ENOMEM, ECUDA, ESTATE, ENONFINITE, ETIMEOUT, EUNSUPPORTED, EIO = range(9)
 _STATUS = {0: "OK", 1: "EINVAL", 2: "ENOMEM", 3: "ECUDA", 4: "ESTATE", 5: "ENONFINITE",
@@ -38,7 +40,7 @@ EXPORTS = [
     "lsgd_kway_average", "lsgd_sgd_update", "lsgd_sample_indices", "lsgd_profile_enable",
     "lsgd_profile_read", "lsgd_grouped_gemm_bf16", "lsgd_batchnorm_stats",
     "lsgd_batchnorm_stats_noalloc", "lsgd_block_average", "lsgd_block_sync_count",
-    "lsgd_sync_state", "lsgd_set_sync_state",
+    "lsgd_sync_state", "lsgd_set_sync_state", "lsgd_schedule",
 ]
 PHASES = ["input", "forward", "loss", "backward", "update", "average"]
 
@@ -82,7 +84,9 @@ class Config(ctypes.Structure):
                 ("weight_decay", ctypes.c_double), ("seed", ctypes.c_uint64),
                 ("precision", ctypes.c_int), ("fused_update", ctypes.c_int),
                 ("hier_block", ctypes.c_int), ("hier_rounds", ctypes.c_int),
-                ("compress", ctypes.c_int), ("global_momentum", ctypes.c_double)]
+                ("compress", ctypes.c_int), ("global_momentum", ctypes.c_double),
+                ("h_warmup", ctypes.c_int), ("h_warmup_epochs", ctypes.c_double),
+                ("sampling", ctypes.c_int)]
 
 
 def make_config(K=1, B_loc=1, H=1, t_switch=-1, total_steps=0, epochs=0.0, N=1, kind=MLP,
@@ -90,7 +94,7 @@ def make_config(K=1, B_loc=1, H=1, t_switch=-1, total_steps=0, epochs=0.0, N=1, 
                 res_blocks=3, base_lr=0.1, scale_by_K=False, warmup_epochs=0.0, milestones=(),
                 decay=0.1, momentum=0.0, nesterov=False, weight_decay=0.0, seed=0,
                 precision=FP32, fused_update=False, hier_block=0, hier_rounds=1, compress=0,
-                global_momentum=0.0) -> Config:
+                global_momentum=0.0, h_warmup=0, h_warmup_epochs=0.0, sampling=0) -> Config:
     c = Config()
     c.K, c.B_loc, c.H = int(K), int(B_loc), int(H)
     c.t_switch, c.total_steps, c.epochs, c.N = int(t_switch), int(total_steps), float(epochs), int(N)
@@ -115,6 +119,8 @@ def make_config(K=1, B_loc=1, H=1, t_switch=-1, total_steps=0, epochs=0.0, N=1, 
     c.fused_update = int(bool(fused_update))
     c.hier_block, c.hier_rounds = int(hier_block), int(hier_rounds)
     c.compress, c.global_momentum = int(compress), float(global_momentum)
+    c.h_warmup, c.h_warmup_epochs = int(h_warmup), float(h_warmup_epochs)
+    c.sampling = int(sampling)
     return c
 
 
@@ -145,6 +151,7 @@ def lib():
             "lsgd_set_params": ([vp, ctypes.c_int, vp, ctypes.c_size_t], st),
             "lsgd_set_momentum": ([vp, ctypes.c_int, vp, ctypes.c_size_t], st),
             "lsgd_sync_state": ([vp, ctypes.c_int, ctypes.c_int, vp, ctypes.c_size_t], st),
+            "lsgd_schedule": ([P(Config), i64, vp, vp], st),
             "lsgd_set_sync_state": ([vp, ctypes.c_int, ctypes.c_int, vp, ctypes.c_size_t], st),
             "lsgd_losses": ([vp, vp, i64], st),
             "lsgd_debug_indices": ([vp, i64, vp], st),
@@ -322,6 +329,16 @@ def lsgd_set_params(ctx: Ctx, k: int, w):
 def lsgd_set_momentum(ctx: Ctx, k: int, u):
     u = np.ascontiguousarray(u, dtype=np.float32)
     _check(lib().lsgd_set_momentum(ctx.handle, int(k), _ptr(u), u.size), ctx)
+
+
+def lsgd_schedule(cfg: Config, n_steps: int):
+    """(lr[s], sync_kind[s]) for s < n_steps, computed on the host (no GPU needed)."""
+    lr = np.zeros(int(n_steps), dtype=np.float64)
+    kinds = np.zeros(int(n_steps), dtype=np.int32)
+    st = lib().lsgd_schedule(ctypes.byref(cfg), int(n_steps), _ptr(lr), _ptr(kinds))
+    if st != OK:
+        raise RuntimeError(f"lsgd_schedule: status {st}: {lib().lsgd_last_error(None).decode()}")
+    return lr, kinds
 
 
 def lsgd_sync_state(ctx: Ctx, which: int, k: int = 0):

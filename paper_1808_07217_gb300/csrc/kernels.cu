@@ -10,6 +10,7 @@
 // multiples of the SM count.
 #include <algorithm>
 
+#include "../../include/lsgd.h"
 #include "common.cuh"
 #include "lsgd_internal.h"
 
@@ -40,6 +41,45 @@ __global__ void sample_indices_kernel(int32_t* __restrict__ idx, uint32_t k0, ui
     const int j = jg * 4 + i;
     if (j < B) idx[(int64_t)k * B + j] = (int32_t)(base + mulhi32(u4_get(r, i), S));
   }
+}
+
+// ---------------------------------------------------------------------------------------------
+// Reshuffling sampler.  pi_e is a keyed permutation of [0, N): a four-round balanced Feistel network
+// (Luby-Rackoff) on 2h-bit values, 4^h >= N, whose round r maps (L, R) to (R, L xor F_r(R)) with
+// F_r(R) = the low h bits of word 0 of Philox4x32-10((R, e, r, 2), seed); values that land outside
+// [0, N) are fed through the network again (cycle walking, Black-Rogaway).  The walk from an
+// i < N stays on i's cycle of the network, so it re-enters [0, N) in fewer than 4^h rounds; the
+// bound only guards that fact.
+__device__ __forceinline__ uint32_t feistel_pi(uint32_t i, uint32_t N, int h, uint32_t e,
+                                               uint32_t k0, uint32_t k1) {
+  const uint64_t mask = (1ull << h) - 1ull;
+  const uint64_t dom = 1ull << (2 * h);
+  uint64_t x = i;
+  for (uint64_t walk = 0; walk < dom; ++walk) {
+    uint64_t L = x >> h, R = x & mask;
+#pragma unroll
+    for (uint32_t r = 0; r < 4; ++r) {
+      const U4 f = philox4x32_10(U4{(uint32_t)R, e, r, 2u}, k0, k1);
+      const uint64_t nR = L ^ ((uint64_t)u4_get(f, 0) & mask);
+      L = R;
+      R = nR;
+    }
+    x = (L << h) | R;
+    if (x < N) break;
+  }
+  return (uint32_t)x;
+}
+
+// I^k_s[j] = pi_e(k S + (t B + j) mod S): worker k's t-th step of epoch e takes the next B
+// positions of its partition [k S, (k + 1) S) of the epoch's permutation.  One thread per index.
+__global__ void sample_reshuffle_kernel(int32_t* __restrict__ idx, uint32_t k0, uint32_t k1,
+                                        uint32_t epoch, int64_t t, int K, int B, uint32_t S,
+                                        uint32_t N, int h) {
+  const int q = blockIdx.x * blockDim.x + threadIdx.x;
+  if (q >= K * B) return;
+  const int k = q / B, j = q % B;
+  const uint32_t pos = (uint32_t)(((uint64_t)t * (uint64_t)B + (uint64_t)j) % S);
+  idx[q] = (int32_t)feistel_pi((uint32_t)k * S + pos, N, h, epoch, k0, k1);
 }
 
 // ---------------------------------------------------------------------------------------------
@@ -542,10 +582,24 @@ __global__ void check_finite_kernel(const float* __restrict__ w, int64_t n, int*
 
 // ---------------------------------------------------------------------------------------------
 cudaError_t launch_sample_indices(int32_t* idx, uint64_t seed, int64_t step, int K, int B, int64_t N,
-                                  cudaStream_t stream) {
-  if (K < 1 || B < 1 || N < K) return cudaErrorInvalidValue;
+                                  int sampling, cudaStream_t stream) {
+  if (K < 1 || B < 1 || N < K || step < 0) return cudaErrorInvalidValue;
   const int64_t S = N / K;
-  if ((int64_t)K * S > 0x7fffffffLL) return cudaErrorInvalidValue;
+  if ((int64_t)K * S > 0x7fffffffLL || N > 0x7fffffffLL) return cudaErrorInvalidValue;
+  if (sampling == LSGD_SAMPLE_RESHUFFLE) {
+    const int64_t KB = (int64_t)K * B;
+    if (KB > 0x7fffffffLL) return cudaErrorInvalidValue;
+    const int64_t e = step * KB / N;            // epoch of this step
+    const int64_t first = (e * N + KB - 1) / KB;  // its first step
+    int h = 1;
+    while ((1ll << (2 * h)) < N) ++h;
+    const int threads = 128;
+    const int blocks = (int)((KB + threads - 1) / threads);
+    sample_reshuffle_kernel<<<blocks, threads, 0, stream>>>(idx, (uint32_t)seed, (uint32_t)(seed >> 32),
+                                                            (uint32_t)e, step - first, K, B,
+                                                            (uint32_t)S, (uint32_t)N, h);
+    return cudaGetLastError();
+  }
   const int groups = (B + 3) / 4;
   const int threads = 128;
   const int blocks = (int)(((int64_t)K * groups + threads - 1) / threads);

@@ -23,8 +23,10 @@ struct SgdParams {
 };
 
 // ---- element-wise / reduction kernels (kernels.cu) ----
+// sampling: LSGD_SAMPLE_SHARDS (i.i.d. within static shards) or LSGD_SAMPLE_RESHUFFLE (epoch
+// permutation, disjoint partitions, in-order pass)
 cudaError_t launch_sample_indices(int32_t* idx, uint64_t seed, int64_t step, int K, int B, int64_t N,
-                                  cudaStream_t stream);
+                                  int sampling, cudaStream_t stream);
 // dst[r][0..D) = X[idx[r]][0..D) (idx == NULL: row r), cast to bf16 when dst_bf16; labels too.
 cudaError_t launch_gather_rows(void* dst, bool dst_bf16, int ld_dst, const float* X, int D,
                                const int32_t* idx, int rows, const int32_t* labels_in,

@@ -43,6 +43,12 @@ namespace lsgd {
 void set_last_error(const std::string& msg) { g_last_error = msg; }
 }  // namespace lsgd
 
+// A round of the local-step warm-up schedule: its first step and length (len <= 0: unknown).
+struct RoundCursor {
+  int64_t start = 0;
+  int64_t len = 0;
+};
+
 struct lsgd_ctx {
   lsgd_config cfg;
   lsgd_allocator alloc{};
@@ -87,6 +93,7 @@ struct lsgd_ctx {
   float* ug = nullptr;     // [d_pad] global momentum
   float* pnorm = nullptr;  // [K] ||Delta_k||_1 / d
   float* l1part = nullptr; // [K][l1_chunks] partial sums
+  RoundCursor cursor;       // the round lsgd_run last stood in (local-step warm-up)
   bool prof_on = false;
   std::vector<cudaEvent_t> prof_pool;
   size_t prof_used = 0;
@@ -183,16 +190,45 @@ double lr_at(const lsgd_config& cfg, int64_t T, int64_t s) {
   return lr;
 }
 
-bool round_end(const lsgd_config& cfg, int64_t T, int64_t s) {
+// Epoch of step s: the samples all workers used before it, over N.
+int64_t epoch_of(const lsgd_config& cfg, int64_t s) {
+  return s * (int64_t)cfg.K * cfg.B_loc / cfg.N;
+}
+
+// Local-step warm-up (Sec. C; Sec. 4's ImageNet runs): the round that starts at step s0, in epoch
+// e < P, has 1 + floor((H - 1) e / P) steps (linear), min(H, 2^floor(e log2 H / P)) (exponential)
+// or 1 (constant); H from epoch P on.
+int64_t round_length(const lsgd_config& cfg, int64_t s0) {
+  if (cfg.h_warmup == LSGD_HWARM_NONE) return cfg.H;
+  const double e = (double)epoch_of(cfg, s0), P = cfg.h_warmup_epochs;
+  if (e >= P) return cfg.H;
+  if (cfg.h_warmup == LSGD_HWARM_LINEAR) return 1 + (int64_t)std::floor((double)(cfg.H - 1) * e / P);
+  if (cfg.h_warmup == LSGD_HWARM_EXPONENTIAL) {
+    const double len = std::pow(2.0, std::floor(e * std::log2((double)cfg.H) / P));
+    return len < (double)cfg.H ? (int64_t)len : cfg.H;
+  }
+  return 1;
+}
+
+// Whether step s ends a round: every step before the switch t' (post-local SGD, Sec. 3), then
+// rounds of H steps (of round_length steps with a local-step warm-up, walked forward from the
+// round `cur` last stood in); the last step of the run always does.
+bool round_end(const lsgd_config& cfg, int64_t T, int64_t s, RoundCursor* cur) {
   if (s == T - 1) return true;
   if (cfg.t_switch >= 0 && s < cfg.t_switch) return true;
   const int64_t start = cfg.t_switch > 0 ? cfg.t_switch : 0;
-  return ((s + 1 - start) % cfg.H) == 0;
+  if (cfg.h_warmup == LSGD_HWARM_NONE) return ((s + 1 - start) % cfg.H) == 0;
+  if (cur->len <= 0 || cur->start > s) *cur = RoundCursor{start, round_length(cfg, start)};
+  while (s >= cur->start + cur->len) {
+    cur->start += cur->len;
+    cur->len = round_length(cfg, cur->start);
+  }
+  return s == cur->start + cur->len - 1;
 }
 
 // Average ending step s: 0 none, 1 block (hierarchical), 2 global (Sec. 3 and Sec. D).
-int sync_kind(const lsgd_config& cfg, int64_t T, int64_t s) {
-  if (!round_end(cfg, T, s)) return 0;
+int sync_kind_at(const lsgd_config& cfg, int64_t T, int64_t s, RoundCursor* cur) {
+  if (!round_end(cfg, T, s, cur)) return 0;
   if (cfg.hier_block <= 0 || s == T - 1) return 2;
   if (cfg.t_switch >= 0 && s < cfg.t_switch) return 2;
   const int64_t start = cfg.t_switch > 0 ? cfg.t_switch : 0;
@@ -589,18 +625,8 @@ lsgd_status step_body(lsgd_ctx* c, int64_t e_start) {
   return LSGD_OK;
 }
 
-void* input_buffer(lsgd_ctx* c) { return c->resnet ? lsgd::resnet_input(c->rn) : c->act[0]; }
-int input_ld(lsgd_ctx* c) { return c->resnet ? c->D : c->layers[0].ld_in; }
-
-}  // namespace
-
-// =============================================================================================
-extern "C" {
-
-lsgd_status lsgd_create(const lsgd_config* cfg, const lsgd_allocator* alloc, void* cuda_stream,
-                        lsgd_ctx** out) {
-  if (!cfg || !out) return fail(nullptr, LSGD_EINVAL, "cfg and out must be non-NULL");
-  const lsgd_config& c0 = *cfg;
+// Every check lsgd_create makes on a configuration before touching the GPU.
+lsgd_status validate_config(const lsgd_config& c0) {
   if (c0.K < 1 || c0.B_loc < 1 || c0.H < 1) return fail(nullptr, LSGD_EINVAL, "K, B_loc and H must be >= 1");
   if (c0.N < c0.K) return fail(nullptr, LSGD_EINVAL, "N must be >= K");
   if (c0.K > 65535) return fail(nullptr, LSGD_EINVAL, "K must be <= 65535");
@@ -617,6 +643,13 @@ lsgd_status lsgd_create(const lsgd_config* cfg, const lsgd_allocator* alloc, voi
                 "compress and global_momentum exclude each other and hierarchical averaging");
   if (c0.compress != LSGD_COMPRESS_NONE && c0.K > 1024)
     return fail(nullptr, LSGD_EINVAL, "compress supports K <= 1024");
+  if (c0.h_warmup < LSGD_HWARM_NONE || c0.h_warmup > LSGD_HWARM_CONSTANT ||
+      c0.h_warmup_epochs < 0.0 || c0.sampling < LSGD_SAMPLE_SHARDS ||
+      c0.sampling > LSGD_SAMPLE_RESHUFFLE)
+    return fail(nullptr, LSGD_EINVAL, "bad h_warmup / h_warmup_epochs / sampling");
+  if (c0.h_warmup != LSGD_HWARM_NONE && (c0.t_switch >= 0 || c0.hier_block > 0))
+    return fail(nullptr, LSGD_EINVAL,
+                "local-step warm-up replaces the post-local switch; not with hier_block");
   const lsgd_model& m = c0.model;
   if (m.kind == LSGD_MLP || m.kind == LSGD_LSQ) {
     if (m.n_layers < 1 || m.n_layers > LSGD_MAX_LAYERS)
@@ -636,6 +669,32 @@ lsgd_status lsgd_create(const lsgd_config* cfg, const lsgd_allocator* alloc, voi
     return fail(nullptr, LSGD_EINVAL, "unknown model kind");
   }
 
+  return LSGD_OK;
+}
+
+// T: total_steps, else ceil(epochs N / (K B_loc)), at least 1.
+int64_t total_steps_of(const lsgd_config& c0) {
+  const int64_t T = c0.total_steps > 0
+                        ? c0.total_steps
+                        : (int64_t)std::ceil(c0.epochs * (double)c0.N / ((double)c0.K * c0.B_loc) - 1e-9);
+  return T < 1 ? 1 : T;
+}
+
+void* input_buffer(lsgd_ctx* c) { return c->resnet ? lsgd::resnet_input(c->rn) : c->act[0]; }
+int input_ld(lsgd_ctx* c) { return c->resnet ? c->D : c->layers[0].ld_in; }
+
+}  // namespace
+
+// =============================================================================================
+extern "C" {
+
+lsgd_status lsgd_create(const lsgd_config* cfg, const lsgd_allocator* alloc, void* cuda_stream,
+                        lsgd_ctx** out) {
+  if (!cfg || !out) return fail(nullptr, LSGD_EINVAL, "cfg and out must be non-NULL");
+  const lsgd_config& c0 = *cfg;
+  const lsgd_status vst = validate_config(c0);
+  if (vst != LSGD_OK) return vst;
+  const lsgd_model& m = c0.model;
   lsgd_ctx* c = new lsgd_ctx();
   c->cfg = c0;
   if (alloc && alloc->alloc && alloc->free) {
@@ -647,10 +706,7 @@ lsgd_status lsgd_create(const lsgd_config* cfg, const lsgd_allocator* alloc, voi
   c->lsq = m.kind == LSGD_LSQ;
   c->resnet = m.kind == LSGD_RESNET20;
   c->shard = c0.N / c0.K;
-  c->T = c0.total_steps > 0
-             ? c0.total_steps
-             : (int64_t)std::ceil(c0.epochs * (double)c0.N / ((double)c0.K * c0.B_loc) - 1e-9);
-  if (c->T < 1) c->T = 1;
+  c->T = total_steps_of(c0);
   auto bail = [&](lsgd_status st) {
     if (c->rn) lsgd::resnet_destroy(c->rn);
     free_all(c);
@@ -810,7 +866,8 @@ lsgd_status lsgd_local_step(lsgd_ctx* c) {
   if (!c->have_data) return fail(c, LSGD_ESTATE, "lsgd_set_dataset must come first");
   const int K = c->cfg.K, B = c->cfg.B_loc;
   const int64_t e0 = prof_mark(c);
-  LSGD_LAUNCH(c, lsgd::launch_sample_indices(c->idx, c->cfg.seed, c->step, K, B, c->cfg.N, c->stream));
+  LSGD_LAUNCH(c, lsgd::launch_sample_indices(c->idx, c->cfg.seed, c->step, K, B, c->cfg.N,
+                                             c->cfg.sampling, c->stream));
   LSGD_LAUNCH(c, lsgd::launch_gather_rows(input_buffer(c), c->bf16, input_ld(c), c->X, c->D, c->idx,
                                           K * B, c->y, c->y ? c->yb : nullptr, c->t,
                                           c->t ? c->tb : nullptr, c->stream));
@@ -907,7 +964,7 @@ lsgd_status lsgd_run(lsgd_ctx* c, int64_t n_steps) {
     const int64_t s = c->step;
     lsgd_status st = lsgd_local_step(c);
     if (st != LSGD_OK) return st;
-    const int kind = sync_kind(c->cfg, c->T, s);
+    const int kind = sync_kind_at(c->cfg, c->T, s, &c->cursor);
     if (kind == 2) {
       st = lsgd_sync_average(c);
       if (st != LSGD_OK) return st;
@@ -1057,7 +1114,8 @@ lsgd_status lsgd_debug_indices(lsgd_ctx* c, int64_t step, int32_t* dst) {
   const int K = c->cfg.K, B = c->cfg.B_loc;
   int32_t* tmp = (int32_t*)dalloc(c, (size_t)K * B * 4);
   if (!tmp) return fail(c, LSGD_ENOMEM, "scratch allocation failed");
-  cudaError_t e = lsgd::launch_sample_indices(tmp, c->cfg.seed, step, K, B, c->cfg.N, c->stream);
+  cudaError_t e =
+      lsgd::launch_sample_indices(tmp, c->cfg.seed, step, K, B, c->cfg.N, c->cfg.sampling, c->stream);
   c->launches++;
   if (e == cudaSuccess) e = cudaMemcpyAsync(dst, tmp, (size_t)K * B * 4, cudaMemcpyDeviceToHost, c->stream);
   if (e == cudaSuccess) e = cudaStreamSynchronize(c->stream);
@@ -1203,6 +1261,19 @@ int64_t lsgd_num_params(const lsgd_ctx* c) { return c ? c->d : -1; }
 int64_t lsgd_step_count(const lsgd_ctx* c) { return c ? c->step : -1; }
 int64_t lsgd_sync_count(const lsgd_ctx* c) { return c ? c->syncs : -1; }
 int64_t lsgd_block_sync_count(const lsgd_ctx* c) { return c ? c->block_syncs : -1; }
+lsgd_status lsgd_schedule(const lsgd_config* cfg, int64_t n_steps, double* lr, int32_t* sync_kind) {
+  if (!cfg || n_steps < 0) return fail(nullptr, LSGD_EINVAL, "lsgd_schedule: bad arguments");
+  const lsgd_status st = validate_config(*cfg);
+  if (st != LSGD_OK) return st;
+  const int64_t T = total_steps_of(*cfg);
+  RoundCursor cur;
+  for (int64_t s = 0; s < n_steps; ++s) {
+    if (lr) lr[s] = lr_at(*cfg, T, s);
+    if (sync_kind) sync_kind[s] = sync_kind_at(*cfg, T, s, &cur);
+  }
+  return LSGD_OK;
+}
+
 int64_t lsgd_total_steps(const lsgd_ctx* c) { return c ? c->T : -1; }
 double lsgd_lr_at(const lsgd_ctx* c, int64_t s) { return c ? lr_at(c->cfg, c->T, s) : 0.0; }
 int64_t lsgd_kernel_launches(const lsgd_ctx* c) { return c ? c->launches : -1; }
@@ -1322,7 +1393,8 @@ lsgd_status lsgd_batchnorm_stats(const float* y, int64_t P, int C, int G, float*
 lsgd_status lsgd_sample_indices(int32_t* dst, uint64_t seed, int64_t step, int K, int B, int64_t N,
                                 void* stream) {
   if (!dst || K < 1 || B < 1 || N < K) return fail(nullptr, LSGD_EINVAL, "lsgd_sample_indices: bad arguments");
-  cudaError_t e = lsgd::launch_sample_indices(dst, seed, step, K, B, N, (cudaStream_t)stream);
+  cudaError_t e =
+      lsgd::launch_sample_indices(dst, seed, step, K, B, N, LSGD_SAMPLE_SHARDS, (cudaStream_t)stream);
   if (e != cudaSuccess) return fail_cuda(nullptr, e, "lsgd_sample_indices");
   return LSGD_OK;
 }

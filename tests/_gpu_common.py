@@ -18,7 +18,8 @@ def built_package():
 def dense_cfgs(P, *, widths, K, B, H, T, N, precision, kind="mlp", t_switch=-1, base_lr=0.1,
                scale_by_K=False, warmup_epochs=0.0, milestones=(), momentum=0.0, nesterov=False,
                weight_decay=0.0, seed=0, init="he", fused_update=False, hier_block=0,
-               hier_rounds=1, compress=0, global_momentum=0.0):
+               hier_rounds=1, compress=0, global_momentum=0.0, h_warmup=0, h_warmup_epochs=0.0,
+               sampling=0):
     """The same run described for the GPU library and for the oracle."""
     gk = {"mlp": P.MLP, "lsq": P.LSQ}[kind]
     ok = {"mlp": oracle.DENSE, "lsq": oracle.LSQ}[kind]
@@ -28,14 +29,16 @@ def dense_cfgs(P, *, widths, K, B, H, T, N, precision, kind="mlp", t_switch=-1, 
                       milestones=milestones, momentum=momentum, nesterov=nesterov,
                       weight_decay=weight_decay, seed=seed, precision=precision,
                       fused_update=fused_update, hier_block=hier_block, hier_rounds=hier_rounds,
-                      compress=compress, global_momentum=global_momentum)
+                      compress=compress, global_momentum=global_momentum, h_warmup=h_warmup,
+                      h_warmup_epochs=h_warmup_epochs, sampling=sampling)
     o = oracle.make_cfg(kind=ok, widths=widths, has_bias=(kind == "mlp"),
                         bf16=(precision == P.BF16), K=K, B=B, H=H, t_switch=t_switch, T=T, N=N,
                         base_lr=base_lr, scale_by_K=scale_by_K, warmup_epochs=warmup_epochs,
                         milestones=milestones, momentum=momentum, nesterov=nesterov,
                         weight_decay=weight_decay, seed=seed, hier_block=hier_block,
                         hier_rounds=hier_rounds, compress=compress,
-                        global_momentum=global_momentum)
+                        global_momentum=global_momentum, h_warmup=h_warmup,
+                        h_warmup_epochs=h_warmup_epochs, sampling=sampling)
     return g, o
 
 

@@ -54,8 +54,10 @@ def test_struct_layout_matches_header(P):
              offsetof(lsgd_config, lr), offsetof(lsgd_config, momentum),
              offsetof(lsgd_config, seed), offsetof(lsgd_config, precision),
              offsetof(lsgd_config, fused_update), sizeof(lsgd_profile));
-      printf("%zu %zu %zu %zu\n", offsetof(lsgd_config, hier_block), offsetof(lsgd_config, hier_rounds),
-             offsetof(lsgd_config, compress), offsetof(lsgd_config, global_momentum));
+      printf("%zu %zu %zu %zu %zu %zu %zu\n", offsetof(lsgd_config, hier_block),
+             offsetof(lsgd_config, hier_rounds), offsetof(lsgd_config, compress),
+             offsetof(lsgd_config, global_momentum), offsetof(lsgd_config, h_warmup),
+             offsetof(lsgd_config, h_warmup_epochs), offsetof(lsgd_config, sampling));
       return 0;
     }
     """
@@ -71,7 +73,8 @@ def test_struct_layout_matches_header(P):
     want = [ctypes.sizeof(C), ctypes.sizeof(P.Model), ctypes.sizeof(P.LrSchedule),
             ctypes.sizeof(P.Allocator), C.model.offset, C.lr.offset, C.momentum.offset,
             C.seed.offset, C.precision.offset, C.fused_update.offset, ctypes.sizeof(P.Profile),
-            C.hier_block.offset, C.hier_rounds.offset, C.compress.offset, C.global_momentum.offset]
+            C.hier_block.offset, C.hier_rounds.offset, C.compress.offset, C.global_momentum.offset,
+            C.h_warmup.offset, C.h_warmup_epochs.offset, C.sampling.offset]
     assert got == want
 
 

@@ -65,6 +65,26 @@ def _dist():
     return world, rank, local
 
 
+def max_over_ranks(x: float, world: int) -> float:
+    """The largest value of x over all ranks (every rank gets it); x itself with one rank.  The
+    tensor lives where the process group's backend wants it (GPU for NCCL, host for gloo)."""
+    if world == 1:
+        return float(x)
+    import torch
+    import torch.distributed as dist
+
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([float(x)], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_throughput(units_per_rank: float, seconds: float, world: int) -> float:
+    """Units all ranks processed over the slowest rank's time (replicas only: every rank runs the
+    same fixed work, so the job ends when the slowest does)."""
+    return world * units_per_rank / max_over_ranks(seconds, world)
+
+
 class ClockSampler:
     """nvidia-smi samples of SM clock and throttle reasons while a timed region runs."""
 
@@ -419,12 +439,9 @@ def main():
     prof = P.lsgd_profile_read(ctx)
     P.lsgd_profile_enable(ctx, False)
     clk = clocks.stop()
-    if world > 1:
-        tt = torch.tensor([t_ms], device="cuda")
-        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
-        t_ms = float(tt.item())
     samples_per_rank = S_ * K * B
-    value = world * samples_per_rank / (t_ms / 1000.0)
+    t_ms = max_over_ranks(t_ms, world)
+    value = whole_job_throughput(samples_per_rank, t_ms / 1000.0, world)
 
     # ---- end to end through the C ABI with host buffers ----
     rng = np.random.default_rng(0)
@@ -454,11 +471,7 @@ def main():
         e2e_step(i)
     torch.cuda.synchronize()
     t_e2e = time.perf_counter() - t0
-    if world > 1:
-        tt = torch.tensor([t_e2e], device="cuda")
-        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
-        t_e2e = float(tt.item())
-    e2e_value = world * samples_per_rank / t_e2e
+    e2e_value = whole_job_throughput(samples_per_rank, t_e2e, world)
     h2d = K * B * w["widths"][0] * 4 + K * B * 4
     d2h = K * 4
 

@@ -230,8 +230,23 @@ lsgd_status lsgd_debug_indices(lsgd_ctx* ctx, int64_t step, int32_t* dst);
  * computed with the same forward kernels (no update). */
 lsgd_status lsgd_eval_loss(lsgd_ctx* ctx, int k, int64_t n, double* loss);
 
-/* LSGD_ENONFINITE if any replica parameter is NaN or Inf. */
+/* LSGD_ENONFINITE if any replica parameter is NaN or Inf (after lsgd_device_status's check). */
 lsgd_status lsgd_check_finite(lsgd_ctx* ctx);
+
+/* Failure detection for the device-side waits.  Every wait inside the tensor-core kernels (on a TMA
+ * arrival, an MMA completion or a free pipeline stage) is bounded (about 2 s of SM clocks); when
+ * one runs out the kernel records it in a device flag, stops issuing work, drains its copies in
+ * flight, frees its tensor memory and exits, so the context stays usable.  lsgd_device_status
+ * synchronises ctx's stream (ctx may be NULL), reads and clears that flag and returns
+ * LSGD_ETIMEOUT if it was set (the results computed since the previous check are then invalid),
+ * else LSGD_OK.  The flag is per device and process. */
+lsgd_status lsgd_device_status(lsgd_ctx* ctx);
+
+/* Exercises that expiry path on its own: one thread waits, through the kernels' bounded wait,
+ * with a limit of limit_ms (0..1000) milliseconds, on an mbarrier phase that completes only if
+ * arrive != 0.  Returns LSGD_OK when the phase completed, LSGD_ETIMEOUT when the wait ran out
+ * (the device flag is consumed), on the current device and the given stream. */
+lsgd_status lsgd_bounded_wait_selftest(int arrive, double limit_ms, void* stream);
 
 /* Checkpoint / resume of w, u (all replicas), the synchronisation state (w_ref, e^k, u_g where the
  * configuration keeps it), the step and sync counters.  Philox is counter based so no generator

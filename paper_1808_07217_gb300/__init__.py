@@ -40,7 +40,8 @@ EXPORTS = [
     "lsgd_kway_average", "lsgd_sgd_update", "lsgd_sample_indices", "lsgd_profile_enable",
     "lsgd_profile_read", "lsgd_grouped_gemm_bf16", "lsgd_batchnorm_stats",
     "lsgd_batchnorm_stats_noalloc", "lsgd_block_average", "lsgd_block_sync_count",
-    "lsgd_sync_state", "lsgd_set_sync_state", "lsgd_schedule",
+    "lsgd_sync_state", "lsgd_set_sync_state", "lsgd_schedule", "lsgd_device_status",
+    "lsgd_bounded_wait_selftest",
 ]
 PHASES = ["input", "forward", "loss", "backward", "update", "average"]
 
@@ -152,6 +153,8 @@ def lib():
             "lsgd_set_momentum": ([vp, ctypes.c_int, vp, ctypes.c_size_t], st),
             "lsgd_sync_state": ([vp, ctypes.c_int, ctypes.c_int, vp, ctypes.c_size_t], st),
             "lsgd_schedule": ([P(Config), i64, vp, vp], st),
+            "lsgd_device_status": ([vp], st),
+            "lsgd_bounded_wait_selftest": ([ctypes.c_int, ctypes.c_double, vp], st),
             "lsgd_set_sync_state": ([vp, ctypes.c_int, ctypes.c_int, vp, ctypes.c_size_t], st),
             "lsgd_losses": ([vp, vp, i64], st),
             "lsgd_debug_indices": ([vp, i64, vp], st),
@@ -329,6 +332,17 @@ def lsgd_set_params(ctx: Ctx, k: int, w):
 def lsgd_set_momentum(ctx: Ctx, k: int, u):
     u = np.ascontiguousarray(u, dtype=np.float32)
     _check(lib().lsgd_set_momentum(ctx.handle, int(k), _ptr(u), u.size), ctx)
+
+
+def lsgd_device_status(ctx: Ctx = None) -> int:
+    """OK, or ETIMEOUT if a bounded device wait ran out since the last check (flag cleared)."""
+    return int(lib().lsgd_device_status(ctx.handle if ctx is not None else None))
+
+
+def lsgd_bounded_wait_selftest(arrive: bool, limit_ms: float, stream=None) -> int:
+    """Status of one bounded wait that completes only if `arrive`: OK or ETIMEOUT."""
+    stream = _current_stream() if stream is None else stream
+    return int(lib().lsgd_bounded_wait_selftest(int(bool(arrive)), float(limit_ms), stream))
 
 
 def lsgd_schedule(cfg: Config, n_steps: int):

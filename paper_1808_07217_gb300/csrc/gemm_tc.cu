@@ -60,12 +60,17 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   return ok != 0;
 }
 
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+
 // Bounded wait on an mbarrier phase; false (and the global error flag set) on expiry.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity,
+                                          long long limit_cycles = kWaitCycles) {
   if (mbar_try_wait(bar, parity)) return true;
   const long long t0 = clock64();
   while (!mbar_try_wait(bar, parity)) {
-    if (clock64() - t0 > kWaitCycles) {
+    if (clock64() - t0 > limit_cycles) {
       atomicExch(&g_tc_timeout, 1);
       return false;
     }
@@ -499,6 +504,27 @@ bool make_tma_map_f32(CUtensorMap* map, const void* base, uint64_t dim0, uint64_
                         strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
                         CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
+}
+
+namespace {
+// The expiry path of the GEMM's bounded waits, on its own: one thread waits on an mbarrier phase
+// that completes only if `arrive` is set, through the same mbar_wait (limit in SM cycles).
+// out = 1 if the phase completed, 0 if the wait ran out (g_tc_timeout is then set).
+__global__ void bounded_wait_selftest_kernel(long long limit_cycles, int arrive, int* out) {
+  __shared__ __align__(8) uint64_t bar;
+  if (threadIdx.x != 0) return;
+  mbar_init(&bar, 1);
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  if (arrive) mbar_arrive(&bar);
+  *out = mbar_wait(&bar, 0, limit_cycles) ? 1 : 0;
+}
+}  // namespace
+
+cudaError_t launch_bounded_wait_selftest(long long limit_cycles, int arrive, int* out,
+                                         cudaStream_t stream) {
+  if (limit_cycles < 0 || limit_cycles > kWaitCycles || !out) return cudaErrorInvalidValue;
+  bounded_wait_selftest_kernel<<<1, 32, 0, stream>>>(limit_cycles, arrive, out);
+  return cudaGetLastError();
 }
 
 int tc_take_timeout_flag() {

@@ -156,5 +156,9 @@ constexpr int kTcTileM = 128;
 bool tc_available();
 // 1 if a bounded wait inside a tcgen05 kernel ran out since the last call (then cleared).
 int tc_take_timeout_flag();
+// One bounded mbarrier wait (the GEMM's mbar_wait) with the given cycle limit (<= the GEMM's):
+// *out (device) = 1 if the phase completed (arrive != 0), 0 if the wait ran out.
+cudaError_t launch_bounded_wait_selftest(long long limit_cycles, int arrive, int* out,
+                                         cudaStream_t stream);
 
 }  // namespace lsgd

@@ -1166,8 +1166,44 @@ lsgd_status lsgd_eval_loss(lsgd_ctx* c, int k, int64_t n, double* loss) {
   return LSGD_OK;
 }
 
+lsgd_status lsgd_device_status(lsgd_ctx* c) {
+  if (c) LSGD_TRY_CUDA(c, cudaStreamSynchronize(c->stream));
+  if (lsgd::tc_take_timeout_flag())
+    return fail(c, LSGD_ETIMEOUT,
+                "a bounded wait inside a tensor-core kernel ran out; results since the last check "
+                "are not valid");
+  return LSGD_OK;
+}
+
+lsgd_status lsgd_bounded_wait_selftest(int arrive, double limit_ms, void* stream) {
+  if (!(limit_ms >= 0.0) || limit_ms > 1000.0)
+    return fail(nullptr, LSGD_EINVAL, "limit_ms must be in [0, 1000]");
+  int dev = 0, khz = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&khz, cudaDevAttrClockRate, dev) != cudaSuccess || khz <= 0) {
+    cudaGetLastError();
+    return fail(nullptr, LSGD_ECUDA, "cannot read the SM clock rate");
+  }
+  const cudaStream_t st = (cudaStream_t)stream;
+  const long long cycles = (long long)(limit_ms * (double)khz);
+  int* d_out = nullptr;
+  int h_out = -1;
+  cudaError_t e = cudaMallocAsync((void**)&d_out, sizeof(int), st);
+  if (e == cudaSuccess) e = lsgd::launch_bounded_wait_selftest(cycles, arrive, d_out, st);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(&h_out, d_out, sizeof(int), cudaMemcpyDeviceToHost, st);
+  if (d_out) cudaFreeAsync(d_out, st);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+  if (e != cudaSuccess) return fail_cuda(nullptr, e, "lsgd_bounded_wait_selftest");
+  const int flagged = lsgd::tc_take_timeout_flag();
+  if (h_out == 1 && !flagged) return LSGD_OK;
+  if (h_out == 0 && flagged) return fail(nullptr, LSGD_ETIMEOUT, "bounded wait ran out (as asked)");
+  return fail(nullptr, LSGD_ECUDA, "bounded-wait self-test: inconsistent result");
+}
+
 lsgd_status lsgd_check_finite(lsgd_ctx* c) {
   if (!c) return fail(nullptr, LSGD_EINVAL, "NULL context");
+  const lsgd_status ds = lsgd_device_status(c);
+  if (ds != LSGD_OK) return ds;
   LSGD_TRY_CUDA(c, cudaMemsetAsync(c->flag, 0, 4, c->stream));
   LSGD_LAUNCH(c, lsgd::launch_check_finite(c->W, (int64_t)c->cfg.K * c->d_pad, c->flag, c->stream));
   int h = 0;

@@ -40,10 +40,10 @@ WORKLOAD = dict(name="mlp_3072-1024-1024-10_K16_B128_H16_bf16", widths=(3072, 10
 UPDATE_BYTES_PER_PARAM = 22
 FUSED_UPDATE_BYTES_PER_PARAM = 18
 AVERAGE_BYTES_PER_PARAM = 10
-# DRAM bytes (read + write) per step of the three fused weight-gradient + update launches, from
-# the ncu capture summarised in profiles/step_kernels_mlp3072_K16_B128.md (below the algorithmic
-# bytes because part of each launch's writes is still in L2 when the launch ends).
-UPDATE_TRAFFIC_PER_STEP = 1116399104
+# DRAM bytes (read + write) per step of the three weight-gradient + update launches, from the ncu
+# capture summarised in profiles/wgrad_update_mlp3072_K16_B128.md (below the algorithmic bytes
+# because part of each launch's writes is still in L2 when the launch ends).
+UPDATE_TRAFFIC_PER_STEP = 1121953792
 
 FALLBACK_HBM_GBS = 6800.0
 FALLBACK_BF16_TFLOPS = 1900.0
@@ -408,7 +408,7 @@ def main():
     X, y = synthdata.gaussian_mixture_cached(w["N"], w["widths"][0], w["C"], w["data_seed"])
     W_, S_ = max(3, args.warmup), args.steps
     e2e_warm = 2
-    total = W_ + S_ + e2e_warm + S_
+    total = W_ + S_ + S_ + e2e_warm + S_  # warm-up, timed, traced, end-to-end warm-up and timed
     stream = torch.cuda.current_stream()
     ctx = P.lsgd_create(_make_cfg(P, total, fused, K), stream=stream.cuda_stream)
     P.lsgd_set_dataset(ctx, X, y)
@@ -422,7 +422,6 @@ def main():
     time.sleep(0.3)
     n0 = P.lsgd_kernel_launches(ctx)
     syncs0 = P.lsgd_sync_count(ctx)
-    P.lsgd_profile_enable(ctx, True)
     if world > 1:
         torch.distributed.barrier()
     torch.cuda.synchronize()
@@ -436,9 +435,14 @@ def main():
     t_ms = e0.elapsed_time(e1)
     launches = P.lsgd_kernel_launches(ctx) - n0
     n_syncs = P.lsgd_sync_count(ctx) - syncs0
+    clk = clocks.stop()
+
+    # ---- the same number of steps again with per-phase CUDA events (the split and roofline) ----
+    P.lsgd_profile_enable(ctx, True)
+    P.lsgd_run(ctx, S_)
+    torch.cuda.synchronize()
     prof = P.lsgd_profile_read(ctx)
     P.lsgd_profile_enable(ctx, False)
-    clk = clocks.stop()
     samples_per_rank = S_ * K * B
     t_ms = max_over_ranks(t_ms, world)
     value = whole_job_throughput(samples_per_rank, t_ms / 1000.0, world)
@@ -448,7 +452,7 @@ def main():
     n_stage = 4
     xs, ys = [], []
     for i in range(n_stage):
-        idx = P.lsgd_debug_indices(ctx, W_ + S_ + i, K, B).reshape(-1)
+        idx = P.lsgd_debug_indices(ctx, W_ + 2 * S_ + i, K, B).reshape(-1)
         xs.append(torch.from_numpy(X[idx].reshape(K, B, -1)).pin_memory())
         ys.append(torch.from_numpy(y[idx].reshape(K, B).copy()).pin_memory())
     del rng
@@ -519,8 +523,8 @@ def main():
         "e2e": {"value": e2e_value, "unit": "samples/s", "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h},
         "gpu_launches": launches,
-        "roofline": {"kernel": ("gemm_tc_kernel weight gradient + fused local update" if fused
-                                else "sgd_update_kernel"),
+        "roofline": {"kernel": ("wgrad_update_kernel (weight gradient + fused local update)"
+                                if fused else "sgd_update_kernel"),
                      "bound": "hbm", "achieved": upd_gbs, "peak": hbm, "unit": "GB/s",
                      "frac": upd_gbs / hbm, "peak_source": f"{peak_src} hbm_gbs",
                      "traffic": UPDATE_TRAFFIC_PER_STEP if fused and K == w["K"] else None,

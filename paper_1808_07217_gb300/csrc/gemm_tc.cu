@@ -18,8 +18,13 @@
 // 64-element-wide boxes stacked along MN (LBO = box stride, SBO = 1024 B; the k-th slice starts
 // 16 rows = 2048 B further).  Every mbarrier wait is bounded: on expiry the kernel records an error
 // flag, stops issuing, and still frees its TMEM.
+//
+// wgrad_update_kernel (further down) is the weight gradient fused with the local update: a
+// persistent variant of the same pipeline whose epilogue streams the parameters through shared
+// memory by TMA.
 #include <cudaTypedefs.h>
 
+#include <algorithm>
 #include <mutex>
 
 #include "common.cuh"
@@ -85,14 +90,6 @@ __device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, u
       " [%0], [%1, {%3, %4, %5}], [%2];" ::"r"(smem_u32(dst)),
       "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(bar)), "r"(x), "r"(y), "r"(z)
       : "memory");
-}
-
-// Fetch a tensor tile into L2 only (no shared memory, no completion tracking).
-__device__ __forceinline__ void tma_prefetch_l2_3d(const CUtensorMap* map, int x, int y, int z) {
-  asm volatile("cp.async.bulk.prefetch.tensor.3d.L2.global.tile [%0, {%1, %2, %3}];" ::"l"(
-                   reinterpret_cast<uint64_t>(map)),
-               "r"(x), "r"(y), "r"(z)
-               : "memory");
 }
 
 __device__ __forceinline__ uint64_t smem_desc(uint32_t addr, uint32_t lbo, uint32_t sbo) {
@@ -214,14 +211,6 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
   bool ok = true;
   if (warp == 0 && lane == 0) {
     // ---------------- TMA producer ----------------
-    if (args.epi == EPI_SGD && args.have_wu_maps) {
-      // the epilogue reads this tile's parameters and momentum: start them towards L2 now
-#pragma unroll
-      for (int i = 0; i < BN / 64; ++i) {
-        tma_prefetch_l2_3d(&args.wmap, n0 + 64 * i, m0, g);
-        if (args.sgd.u) tma_prefetch_l2_3d(&args.umap, n0 + 64 * i, m0, g);
-      }
-    }
     int issued = 0;
     for (int kb = 0; kb < nk && ok; ++kb) {
       const int s = kb % STAGES;
@@ -314,11 +303,11 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
       }
       asm volatile("bar.sync 1, 128;" ::: "memory");
       // copy-out: item = (row, 4-column group), 16 groups per 64-column row.  Each thread takes
-      // UNR items at a time and issues all their global loads (mask, or w and u) before any
-      // arithmetic, so several hundred bytes per thread are in flight.
+      // UNR items at a time and issues all their mask loads before any arithmetic, so several
+      // hundred bytes per thread are in flight.
       constexpr int UNR = 8, ITEMS = BM * (CW / 4);
       for (int base = threadIdx.x; base < ITEMS; base += 128 * UNR) {
-        float4 x[UNR], a0[UNR], a1[UNR];
+        float4 x[UNR], a0[UNR];
         int64_t off[UNR];
         int nn[UNR];
         bool ok[UNR];
@@ -331,7 +320,6 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
           nn[q] = n;
           off[q] = c_base + (int64_t)m * args.c_rs + n;
           a0[q] = make_float4(0.f, 0.f, 0.f, 0.f);
-          a1[q] = a0[q];
           if (!ok[q]) continue;
           x[q] = *reinterpret_cast<const float4*>(stg + row * PITCH + grp * 4);
           const bool full4 = n + 4 <= args.N;
@@ -354,22 +342,6 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
               for (int i = 0; i < 4 && n + i < args.N; ++i) t[i] = mp[i];
               a0[q] = make_float4(t[0], t[1], t[2], t[3]);
             }
-          } else if (epi == EPI_SGD) {
-            const float* wp = args.sgd.w + off[q];
-            const float* up = args.sgd.u ? args.sgd.u + off[q] : nullptr;
-            if (full4 && ((reinterpret_cast<uintptr_t>(wp) & 15) == 0) &&
-                ((reinterpret_cast<uintptr_t>(up) & 15) == 0)) {
-              a0[q] = __ldcs(reinterpret_cast<const float4*>(wp));
-              if (up) a1[q] = __ldcs(reinterpret_cast<const float4*>(up));
-            } else {
-              float t[4] = {0.f, 0.f, 0.f, 0.f}, v[4] = {0.f, 0.f, 0.f, 0.f};
-              for (int i = 0; i < 4 && n + i < args.N; ++i) {
-                t[i] = wp[i];
-                if (up) v[i] = up[i];
-              }
-              a0[q] = make_float4(t[0], t[1], t[2], t[3]);
-              a1[q] = make_float4(v[0], v[1], v[2], v[3]);
-            }
           }
         }
 #pragma unroll
@@ -383,34 +355,6 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
             v.y = a0[q].y > 0.f ? v.y : 0.f;
             v.z = a0[q].z > 0.f ? v.z : 0.f;
             v.w = a0[q].w > 0.f ? v.w : 0.f;
-          }
-          if (epi == EPI_SGD) {
-            const SgdParams& sp = args.sgd;
-            float4 wv = a0[q], uv = a1[q];
-            sgd4(wv, uv, v, sp);
-            float* wp = sp.w + off[q];
-            float* up = sp.u ? sp.u + off[q] : nullptr;
-            uint16_t* bp = sp.wb ? sp.wb + off[q] : nullptr;
-            if (full4 && ((reinterpret_cast<uintptr_t>(wp) & 15) == 0) &&
-                ((reinterpret_cast<uintptr_t>(up) & 15) == 0) &&
-                ((reinterpret_cast<uintptr_t>(bp) & 7) == 0)) {
-              __stcs(reinterpret_cast<float4*>(wp), wv);
-              if (up) __stcs(reinterpret_cast<float4*>(up), uv);
-              if (bp) {
-                uint2 o;
-                o.x = (uint32_t)f2bf(wv.x) | ((uint32_t)f2bf(wv.y) << 16);
-                o.y = (uint32_t)f2bf(wv.z) | ((uint32_t)f2bf(wv.w) << 16);
-                __stcs(reinterpret_cast<uint2*>(bp), o);
-              }
-            } else {
-              const float ws[4] = {wv.x, wv.y, wv.z, wv.w}, us[4] = {uv.x, uv.y, uv.z, uv.w};
-              for (int i = 0; i < 4 && n + i < args.N; ++i) {
-                wp[i] = ws[i];
-                if (up) up[i] = us[i];
-                if (bp) bp[i] = f2bf(ws[i]);
-              }
-            }
-            continue;
           }
           if (args.c_bf16) {
             uint16_t* out = reinterpret_cast<uint16_t*>(args.C) + off[q];
@@ -441,6 +385,304 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
   __syncthreads();
   if (warp == 2) {
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"((uint32_t)BN)
+                 : "memory");
+  }
+}
+
+// =============================================================================================
+// Weight gradient fused with the local update: persistent, every parameter byte moved by TMA.
+//
+// For replica g and a 128 x 128 tile (rows m = output units, columns n = inputs) of a layer's
+// weight matrix, the gradient dZ[g]^T act[g] (k = B_loc) accumulates in one of two TMEM
+// accumulators while the previous tile's update runs.  The tile's parameters and momentum stream
+// through a ring of shared-memory slots in 32-column chunks (128 rows x 128 B, SWIZZLE_128B), are
+// updated in place, and go back to HBM by TMA stores (clipped at the matrix edge), together with
+// the bf16 shadow staged in a 64-byte-swizzled buffer.  One CTA per SM:
+//   warp 0      operand producer: dZ / act k-blocks into a two-stage ring
+//   warp 1      MMA issuer: tcgen05.mma (M = N = 128, K = 16) into accumulator (tile & 1)
+//   warp 2      TMEM allocation (256 columns); w / u chunk producer
+//   warps 4-7   epilogue, one tile row per thread (TMEM lane quarter = warp % 4): per chunk,
+//               tcgen05.ld of 32 gradient columns, the local momentum-SGD update (weight decay,
+//               heavy-ball or Nesterov momentum, Sec. A.4) on w, u in shared memory, bf16 w into a staging buffer; thread 128 then issues the three TMA stores
+//               and recycles the slot of the chunk before once its stores have read it.
+// Only thread 128 waits on the epilogue's mbarriers and the outcome reaches the other epilogue
+// threads through a named barrier, so a wait that runs out cannot split them.
+namespace wu {
+constexpr int TN = 128;                     // tile columns (= rows: BM)
+constexpr int CW = 32;                      // chunk columns (fp32: one 128-byte row)
+constexpr int ST = 2;                       // operand stages
+constexpr int NS = 4;                       // w / u chunk slots
+constexpr int NWB = 3;                      // bf16 staging buffers
+constexpr int THREADS = 256;
+constexpr int EPI0 = 128;                   // first epilogue thread
+constexpr uint32_t kChunkF32 = BM * CW * 4;  // 16 KB
+constexpr uint32_t kChunkB16 = BM * CW * 2;  // 8 KB
+}  // namespace wu
+
+struct WuSmem {
+  uint8_t a[wu::ST][BM * BK * 2];         // 16 KB each
+  uint8_t b[wu::ST][wu::TN * BK * 2];     // 16 KB each
+  uint8_t w[wu::NS][wu::kChunkF32];       // 1024-aligned (SWIZZLE_128B)
+  uint8_t u[wu::NS][wu::kChunkF32];
+  uint8_t wb[wu::NWB][wu::kChunkB16];     // 512-aligned (SWIZZLE_64B)
+  uint64_t op_full[wu::ST], op_empty[wu::ST];
+  uint64_t acc_full[2], acc_empty[2];
+  uint64_t wu_full[wu::NS], wu_empty[wu::NS];
+  uint32_t tmem_base;
+  int epi_ok[2];
+};
+
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,"
+      "%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]),
+        "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]),
+        "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+__device__ __forceinline__ void tma_store_3d(const CUtensorMap* map, const void* src, int x, int y,
+                                             int z) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%2, %3, %4}], [%1];" ::"l"(
+          reinterpret_cast<uint64_t>(map)),
+      "r"(smem_u32(src)), "r"(x), "r"(y), "r"(z)
+      : "memory");
+}
+
+__device__ __forceinline__ int wu_chunks(int N, int n0) {
+  const int left = N - n0;
+  return left >= wu::TN ? wu::TN / wu::CW : (left + wu::CW - 1) / wu::CW;
+}
+
+__global__ void __launch_bounds__(wu::THREADS, 1) wgrad_update_kernel(
+    const __grid_constant__ WgradUpdateArgs args) {
+  extern __shared__ uint8_t smem_raw[];
+  WuSmem& sm = *reinterpret_cast<WuSmem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                          ~uintptr_t(1023));
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int tiles_n = (args.N + wu::TN - 1) / wu::TN, tiles_m = (args.M + BM - 1) / BM;
+  const int tiles = tiles_n * tiles_m * args.G;
+  const int nk = (args.Kd + BK - 1) / BK;
+  const bool a_mn = args.A.mn_major, b_mn = args.B.mn_major;
+  const bool has_u = args.sgd.u != nullptr;
+  constexpr uint32_t kBytesA = BM * BK * 2, kBytesB = wu::TN * BK * 2;
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < wu::ST; ++i) {
+      mbar_init(&sm.op_full[i], 1);
+      mbar_init(&sm.op_empty[i], 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&sm.acc_full[i], 1);
+      mbar_init(&sm.acc_empty[i], 1);
+    }
+    for (int i = 0; i < wu::NS; ++i) {
+      mbar_init(&sm.wu_full[i], 1);
+      mbar_init(&sm.wu_empty[i], 1);
+    }
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  }
+  if (warp == 2) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     smem_u32(&sm.tmem_base)),
+                 "r"(2u * wu::TN)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+  __syncthreads();
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+  const uint32_t tmem = sm.tmem_base;
+
+  auto tile_coords = [&](int t, int& g, int& m0, int& n0) {
+    const int per_g = tiles_m * tiles_n;
+    g = t / per_g;
+    const int r = t % per_g;
+    m0 = (r / tiles_n) * BM;
+    n0 = (r % tiles_n) * wu::TN;
+  };
+
+  if (warp == 0 && lane == 0) {
+    // ---------------- operand producer ----------------
+    int it = 0;
+    bool ok = true;
+    for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x) {
+      int g, m0, n0;
+      tile_coords(t, g, m0, n0);
+      for (int kb = 0; kb < nk; ++kb, ++it) {
+        const int s = it % wu::ST;
+        if (!mbar_wait(&sm.op_empty[s], ((it / wu::ST) & 1) ^ 1)) {
+          ok = false;
+          break;
+        }
+        mbar_expect_tx(&sm.op_full[s], kBytesA + kBytesB);
+        const int k0 = kb * BK;
+        if (!a_mn) {
+          tma_load_3d(sm.a[s], &args.A.map, &sm.op_full[s], k0, m0, g);
+        } else {
+#pragma unroll
+          for (int i = 0; i < BM / 64; ++i)
+            tma_load_3d(sm.a[s] + i * 64 * BK * 2, &args.A.map, &sm.op_full[s], m0 + 64 * i, k0, g);
+        }
+        if (!b_mn) {
+          tma_load_3d(sm.b[s], &args.B.map, &sm.op_full[s], k0, n0, g);
+        } else {
+#pragma unroll
+          for (int i = 0; i < wu::TN / 64; ++i)
+            tma_load_3d(sm.b[s] + i * 64 * BK * 2, &args.B.map, &sm.op_full[s], n0 + 64 * i, k0, g);
+        }
+      }
+    }
+    if (!ok) {
+      // let copies in flight land before the CTA can exit
+      for (int j = (it > wu::ST ? it - wu::ST : 0); j < it; ++j)
+        mbar_wait(&sm.op_full[j % wu::ST], (j / wu::ST) & 1);
+    }
+  } else if (warp == 1 && lane == 0) {
+    // ---------------- MMA issuer ----------------
+    const uint32_t idesc = make_idesc(BM, wu::TN, a_mn, b_mn);
+    int it = 0, i = 0;
+    bool ok = true;
+    for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x, ++i) {
+      const int ab = i & 1;
+      if (!mbar_wait(&sm.acc_empty[ab], ((i >> 1) & 1) ^ 1)) break;
+      asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+      const uint32_t acc = tmem + (uint32_t)(ab * wu::TN);
+      for (int kb = 0; kb < nk; ++kb, ++it) {
+        const int s = it % wu::ST;
+        if (!mbar_wait(&sm.op_full[s], (it / wu::ST) & 1)) {
+          ok = false;
+          break;
+        }
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        const uint32_t a_base = smem_u32(sm.a[s]), b_base = smem_u32(sm.b[s]);
+#pragma unroll
+        for (int kk = 0; kk < BK / 16; ++kk) {
+          const uint64_t ad = a_mn ? smem_desc(a_base + kk * 2048, 64 * BK * 2, 1024)
+                                   : smem_desc(a_base + kk * 32, 16, 1024);
+          const uint64_t bd = b_mn ? smem_desc(b_base + kk * 2048, 64 * BK * 2, 1024)
+                                   : smem_desc(b_base + kk * 32, 16, 1024);
+          mma_bf16(acc, ad, bd, idesc, (kb > 0 || kk > 0) ? 1u : 0u);
+        }
+        mma_commit(&sm.op_empty[s]);
+      }
+      if (ok) mma_commit(&sm.acc_full[ab]);
+    }
+  } else if (warp == 2 && lane == 0) {
+    // ---------------- w / u chunk producer ----------------
+    int q = 0;
+    bool ok = true;
+    const uint32_t bytes = wu::kChunkF32 * (has_u ? 2u : 1u);
+    for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x) {
+      int g, m0, n0;
+      tile_coords(t, g, m0, n0);
+      const int nc = wu_chunks(args.N, n0);
+      for (int c = 0; c < nc; ++c, ++q) {
+        const int sl = q % wu::NS;
+        if (!mbar_wait(&sm.wu_empty[sl], ((q / wu::NS) & 1) ^ 1)) {
+          ok = false;
+          break;
+        }
+        mbar_expect_tx(&sm.wu_full[sl], bytes);
+        tma_load_3d(sm.w[sl], &args.wmap, &sm.wu_full[sl], n0 + c * wu::CW, m0, g);
+        if (has_u) tma_load_3d(sm.u[sl], &args.umap, &sm.wu_full[sl], n0 + c * wu::CW, m0, g);
+      }
+    }
+    if (!ok) {
+      for (int j = (q > wu::NS ? q - wu::NS : 0); j < q; ++j)
+        mbar_wait(&sm.wu_full[j % wu::NS], (j / wu::NS) & 1);
+    }
+  } else if (warp >= 4) {
+    // ---------------- epilogue ----------------
+    const bool leader = threadIdx.x == wu::EPI0;
+    const int quarter = warp & 3;
+    const int r = quarter * 32 + lane;  // tile row of this thread
+    const SgdParams& sp = args.sgd;
+    // The leader waits; everyone learns the outcome after the named barrier.  Two flag slots
+    // alternate, so the leader never overwrites a flag another thread has yet to read (each
+    // thread reads slot f before it can reach the barrier of the next wait).
+    int fi = 0;
+    auto epi_wait = [&](uint64_t* bar, uint32_t parity) -> bool {
+      if (leader) sm.epi_ok[fi] = mbar_wait(bar, parity) ? 1 : 0;
+      asm volatile("bar.sync 1, 128;" ::: "memory");
+      const bool okw = sm.epi_ok[fi] != 0;
+      fi ^= 1;
+      return okw;
+    };
+    int q = 0, i = 0, wbi = 0;
+    bool ok = true;
+    for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x, ++i) {
+      int g, m0, n0;
+      tile_coords(t, g, m0, n0);
+      const int ab = i & 1;
+      const int nc = wu_chunks(args.N, n0);
+      if (!epi_wait(&sm.acc_full[ab], (i >> 1) & 1)) {
+        ok = false;
+        break;
+      }
+      asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+      for (int c = 0; c < nc; ++c, ++q, wbi = (wbi + 1) % wu::NWB) {
+        const int sl = q % wu::NS;
+        if (!epi_wait(&sm.wu_full[sl], (q / wu::NS) & 1)) {
+          ok = false;
+          break;
+        }
+        mbar_try_wait(&sm.wu_full[sl], (q / wu::NS) & 1);  // acquire the TMA-written data
+        float gv[32];
+        tmem_ld32(tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(ab * wu::TN + c * wu::CW), gv);
+        uint8_t* wrow = sm.w[sl] + r * 128;
+        uint8_t* urow = sm.u[sl] + r * 128;
+        uint8_t* brow = sm.wb[wbi] + r * 64;
+        uint32_t packed[16];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          const int phys = (j ^ (r & 7)) << 4;
+          float4 wv = *reinterpret_cast<const float4*>(wrow + phys);
+          float4 uv = has_u ? *reinterpret_cast<const float4*>(urow + phys)
+                            : make_float4(0.f, 0.f, 0.f, 0.f);
+          sgd4(wv, uv, make_float4(gv[4 * j], gv[4 * j + 1], gv[4 * j + 2], gv[4 * j + 3]), sp);
+          *reinterpret_cast<float4*>(wrow + phys) = wv;
+          if (has_u) *reinterpret_cast<float4*>(urow + phys) = uv;
+          packed[2 * j] = (uint32_t)f2bf(wv.x) | ((uint32_t)f2bf(wv.y) << 16);
+          packed[2 * j + 1] = (uint32_t)f2bf(wv.z) | ((uint32_t)f2bf(wv.w) << 16);
+        }
+#pragma unroll
+        for (int h = 0; h < 4; ++h)
+          *reinterpret_cast<uint4*>(brow + ((h ^ ((r >> 1) & 3)) << 4)) =
+              make_uint4(packed[4 * h], packed[4 * h + 1], packed[4 * h + 2], packed[4 * h + 3]);
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+        asm volatile("bar.sync 1, 128;" ::: "memory");
+        if (leader) {
+          const int x = n0 + c * wu::CW;
+          tma_store_3d(&args.wmap, sm.w[sl], x, m0, g);
+          if (has_u) tma_store_3d(&args.umap, sm.u[sl], x, m0, g);
+          if (sp.wb) tma_store_3d(&args.wbmap, sm.wb[wbi], x, m0, g);
+          asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+          // the stores of the chunk before have read their slot: hand it back to the producer
+          asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
+          if (q > 0) mbar_arrive(&sm.wu_empty[(q - 1) % wu::NS]);
+          if (c == nc - 1) mbar_arrive(&sm.acc_empty[ab]);  // every row has read the accumulator
+        }
+      }
+    }
+    if (leader) asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+    (void)ok;
+  }
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+  __syncthreads();
+  if (warp == 2) {
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
+                 "r"(2u * wu::TN)
                  : "memory");
   }
 }
@@ -556,6 +798,59 @@ bool make_tma_map_bf16(CUtensorMap* map, const void* base, uint64_t dim0, uint64
   return r == CUDA_SUCCESS;
 }
 
+bool make_tma_map(CUtensorMap* map, const void* base, bool bf16, uint64_t dim0, uint64_t dim1,
+                  uint64_t dim2, uint64_t s1, uint64_t s2, uint32_t box0, uint32_t box1,
+                  int swizzle_bytes) {
+  std::call_once(g_encode_once, load_encode);
+  if (!g_encode) return false;
+  const uint64_t esz = bf16 ? 2 : 4;
+  if ((reinterpret_cast<uintptr_t>(base) & 15) || ((s1 * esz) & 15) || ((s2 * esz) & 15)) return false;
+  CUtensorMapSwizzle sw;
+  switch (swizzle_bytes) {
+    case 0: sw = CU_TENSOR_MAP_SWIZZLE_NONE; break;
+    case 32: sw = CU_TENSOR_MAP_SWIZZLE_32B; break;
+    case 64: sw = CU_TENSOR_MAP_SWIZZLE_64B; break;
+    case 128: sw = CU_TENSOR_MAP_SWIZZLE_128B; break;
+    default: return false;
+  }
+  if (swizzle_bytes && box0 * esz > (uint64_t)swizzle_bytes) return false;
+  cuuint64_t dims[3] = {dim0, dim1, dim2};
+  cuuint64_t strides[2] = {s1 * esz, s2 * esz};
+  cuuint32_t box[3] = {box0, box1, 1};
+  cuuint32_t estr[3] = {1, 1, 1};
+  CUresult r = g_encode(map, bf16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32,
+                        3, const_cast<void*>(base), dims, strides, box, estr,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+cudaError_t launch_wgrad_update(const WgradUpdateArgs& a, cudaStream_t stream) {
+  if (a.M <= 0 || a.N <= 0 || a.G <= 0) return cudaSuccess;
+  if (a.Kd <= 0 || !a.sgd.w || (a.sgd.mom != 0.f && !a.sgd.u)) return cudaErrorInvalidValue;
+  // operand boxes as the kernel expects them (64-wide MN-major boxes, or full K-major tiles)
+  if (a.A.mn_major ? a.A.box_rows != 64 : a.A.box_rows != BM) return cudaErrorInvalidValue;
+  if (a.B.mn_major ? a.B.box_rows != 64 : a.B.box_rows != wu::TN) return cudaErrorInvalidValue;
+  const int64_t tiles = (int64_t)((a.N + wu::TN - 1) / wu::TN) * ((a.M + BM - 1) / BM) * a.G;
+  if (tiles > 0x7fffffffLL) return cudaErrorInvalidValue;
+  int dev = 0, sms = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  if (e != cudaSuccess) return e;
+  constexpr size_t smem = sizeof(WuSmem) + 1024;
+  static_assert(smem <= 232448, "shared memory per CTA");
+  static int attr_dev = -1;
+  if (attr_dev != dev) {
+    e = cudaFuncSetAttribute(wgrad_update_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)smem);
+    if (e != cudaSuccess) return e;
+    attr_dev = dev;
+  }
+  const int grid = (int)std::min<int64_t>(tiles, sms);
+  wgrad_update_kernel<<<grid, wu::THREADS, smem, stream>>>(a);
+  return cudaGetLastError();
+}
+
 int tc_tile_n(int Kd) { return (Kd + BK - 1) / BK <= 2 ? 128 : 64; }
 
 int tc_valid_splits(int Kd, int want) {
@@ -576,8 +871,7 @@ cudaError_t launch_gemm_tc(const TcGemmArgs& a, cudaStream_t stream) {
   if (a.B.mn_major ? a.B.box_rows != 64 : a.B.box_rows != bn) return cudaErrorInvalidValue;
   if ((a.epi == EPI_BIAS || a.epi == EPI_BIAS_RELU) && !a.bias) return cudaErrorInvalidValue;
   if (a.epi == EPI_MASK && !a.mask) return cudaErrorInvalidValue;
-  if (a.epi == EPI_SGD && (!a.sgd.w || (a.sgd.mom != 0.f && !a.sgd.u))) return cudaErrorInvalidValue;
-  if (a.epi != EPI_SGD && !a.C) return cudaErrorInvalidValue;
+  if (!a.C) return cudaErrorInvalidValue;
   const int splits = a.splits > 1 ? a.splits : 1;
   if (splits > 1) {
     const int nk_all = (a.Kd + BK - 1) / BK, per = (nk_all + splits - 1) / splits;

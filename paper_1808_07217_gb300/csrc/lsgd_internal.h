@@ -81,9 +81,7 @@ enum GemmEpilogue {
   EPI_STORE = 0,      // C = acc
   EPI_BIAS = 1,       // C = acc + bias[n]
   EPI_BIAS_RELU = 2,  // C = max(acc + bias[n], 0)
-  EPI_MASK = 3,       // C = mask(m, n) > 0 ? acc : 0   (ReLU derivative from the stored activation)
-  EPI_SGD = 4         // acc is the gradient of W(m, n): apply the local update to W, U and the bf16
-                      // shadow at C's indexing (nothing is stored to C)
+  EPI_MASK = 3        // C = mask(m, n) > 0 ? acc : 0   (ReLU derivative from the stored activation)
 };
 
 struct GemmArgs {
@@ -119,11 +117,6 @@ struct TcOperand {
 struct TcGemmArgs {
   int M, N, Kd, G;
   TcOperand A, B;
-  SgdParams sgd;  // EPI_SGD only
-  // EPI_SGD: fp32 maps over sgd.w / sgd.u (dims {N, M, G}, box {64, 128}) used to prefetch the
-  // tile's parameters and momentum into L2 while the products run (have_wu_maps = 0: no prefetch)
-  CUtensorMap wmap, umap;
-  int have_wu_maps;
   // split-K: the reduction is cut into `splits` contiguous ranges of k-blocks, split s writing its
   // partial product at C + g c_gs + s c_split_stride (EPI_STORE only); 0 or 1 = no split
   int splits;
@@ -139,6 +132,23 @@ struct TcGemmArgs {
   int64_t mask_rs, mask_gs;
   bool mask_bf16;
 };
+
+// The weight gradient of one dense layer fused with the local update, for G replicas: W[g] (M x
+// N, row stride N) -= update(dZ[g]^T act[g]) with the momentum and bf16 shadow of SgdParams.
+// wmap / umap: fp32 maps over sgd.w / sgd.u, dims {N, M, G}, strides {N, replica stride}, box
+// {32, 128}, 128-byte swizzle; wbmap: the same over sgd.wb in bf16 with a 64-byte swizzle.
+struct WgradUpdateArgs {
+  int M, N, Kd, G;
+  TcOperand A, B;  // dZ (m = output unit) and act (n = input), as for the weight-gradient GEMM
+  SgdParams sgd;
+  CUtensorMap wmap, umap, wbmap;
+};
+cudaError_t launch_wgrad_update(const WgradUpdateArgs& a, cudaStream_t stream);
+// Rank-3 TMA map over [dim2][dim1][dim0] (fp32 or bf16) with strides (elements) s1, s2, box
+// {box0, box1, 1} and a swizzle of 0, 32, 64 or 128 bytes.
+bool make_tma_map(CUtensorMap* map, const void* base, bool bf16, uint64_t dim0, uint64_t dim1,
+                  uint64_t dim2, uint64_t s1, uint64_t s2, uint32_t box0, uint32_t box1,
+                  int swizzle_bytes);
 
 // Encode a rank-3 bf16 TMA map over [dim2][dim1][dim0] with strides (elements) s1, s2.
 bool make_tma_map_bf16(CUtensorMap* map, const void* base, uint64_t dim0, uint64_t dim1,

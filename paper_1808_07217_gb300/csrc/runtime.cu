@@ -513,18 +513,32 @@ lsgd_status dense_backward(lsgd_ctx* c) {
       t.c_gs = c->d_pad;
       t.c_bf16 = false;
       if (c->fused) {
-        t.epi = lsgd::EPI_SGD;
-        t.sgd = sgd_at(Ly.w_off);
-        t.have_wu_maps =
-            lsgd::make_tma_map_f32(&t.wmap, t.sgd.w, Ly.in, Ly.out, K, Ly.in, c->d_pad, 64, 128) &&
-            (!t.sgd.u ||
-             lsgd::make_tma_map_f32(&t.umap, t.sgd.u, Ly.in, Ly.out, K, Ly.in, c->d_pad, 64, 128));
+        // persistent weight-gradient + update kernel: parameters, momentum and the bf16 shadow
+        // stream through shared memory by TMA in 128 x 32 chunks
+        lsgd::WgradUpdateArgs wa{};
+        wa.M = Ly.out;
+        wa.N = Ly.in;
+        wa.Kd = B;
+        wa.G = K;
+        wa.A = t.A;
+        wa.B = t.B;
+        wa.sgd = sgd_at(Ly.w_off);
+        bool mok = lsgd::make_tma_map(&wa.wmap, wa.sgd.w, false, Ly.in, Ly.out, K, Ly.in, c->d_pad,
+                                      32, 128, 128);
+        if (wa.sgd.u)
+          mok &= lsgd::make_tma_map(&wa.umap, wa.sgd.u, false, Ly.in, Ly.out, K, Ly.in, c->d_pad,
+                                    32, 128, 128);
+        if (wa.sgd.wb)
+          mok &= lsgd::make_tma_map(&wa.wbmap, wa.sgd.wb, true, Ly.in, Ly.out, K, Ly.in, c->d_pad,
+                                    32, 128, 64);
+        if (!mok) return fail(c, LSGD_ECUDA, "TMA map encoding failed (fused update)");
+        LSGD_LAUNCH(c, lsgd::launch_wgrad_update(wa, c->stream));
       } else {
         t.C = c->G + Ly.w_off;
         t.epi = lsgd::EPI_STORE;
+        lsgd_status st = tc_gemm(c, t);
+        if (st != LSGD_OK) return st;
       }
-      lsgd_status st = tc_gemm(c, t);
-      if (st != LSGD_OK) return st;
     } else {
       lsgd::GemmArgs g{};
       g.M = Ly.out;

@@ -65,6 +65,15 @@ __device__ __forceinline__ void sgd_elem(float& w, float& u, float g, float lr, 
   w = fmaf(-lr, st, w);
 }
 
+// Programmatic dependent launch: kernels of the training step are launched so that the next one
+// may be scheduled while the previous one drains.  Each such kernel first waits for the previous
+// grid's completion and memory (griddepcontrol.wait) before touching global memory, and at once
+// allows the next kernel to launch (its CTAs still wait here for this grid to finish).
+__device__ __forceinline__ void pdl_begin() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 template <typename T>
 struct Elem;
 template <>

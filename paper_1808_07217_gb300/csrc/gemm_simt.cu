@@ -15,6 +15,7 @@ constexpr int BM = 64, BN = 64, BK = 16, PAD = 4;
 
 template <typename TA, typename TB, typename TC, typename TM, int EPI>
 __global__ void __launch_bounds__(256) gemm_simt_kernel(GemmArgs a) {
+  pdl_begin();
   __shared__ __align__(16) float As[BK][BM + PAD];
   __shared__ __align__(16) float Bs[BK][BN + PAD];
   const int g = blockIdx.z;
@@ -101,16 +102,16 @@ template <typename TA, typename TB, typename TC, typename TM>
 cudaError_t dispatch_epi(const GemmArgs& a, dim3 grid, cudaStream_t s) {
   switch (a.epi) {
     case EPI_STORE:
-      gemm_simt_kernel<TA, TB, TC, TM, EPI_STORE><<<grid, 256, 0, s>>>(a);
+      launch_pdl(gemm_simt_kernel<TA, TB, TC, TM, EPI_STORE>, grid, 256, 0, s, a);
       break;
     case EPI_BIAS:
-      gemm_simt_kernel<TA, TB, TC, TM, EPI_BIAS><<<grid, 256, 0, s>>>(a);
+      launch_pdl(gemm_simt_kernel<TA, TB, TC, TM, EPI_BIAS>, grid, 256, 0, s, a);
       break;
     case EPI_BIAS_RELU:
-      gemm_simt_kernel<TA, TB, TC, TM, EPI_BIAS_RELU><<<grid, 256, 0, s>>>(a);
+      launch_pdl(gemm_simt_kernel<TA, TB, TC, TM, EPI_BIAS_RELU>, grid, 256, 0, s, a);
       break;
     case EPI_MASK:
-      gemm_simt_kernel<TA, TB, TC, TM, EPI_MASK><<<grid, 256, 0, s>>>(a);
+      launch_pdl(gemm_simt_kernel<TA, TB, TC, TM, EPI_MASK>, grid, 256, 0, s, a);
       break;
     default:
       return cudaErrorInvalidValue;

@@ -207,6 +207,7 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
   __syncthreads();
   asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
   const uint32_t tmem = sm.tmem_base;
+  pdl_begin();  // everything above touched only shared memory and TMEM
 
   bool ok = true;
   if (warp == 0 && lane == 0) {
@@ -502,6 +503,7 @@ __global__ void __launch_bounds__(wu::THREADS, 1) wgrad_update_kernel(
   __syncthreads();
   asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
   const uint32_t tmem = sm.tmem_base;
+  pdl_begin();  // everything above touched only shared memory and TMEM
 
   auto tile_coords = [&](int t, int& g, int& m0, int& n0) {
     const int per_g = tiles_m * tiles_n;
@@ -716,7 +718,7 @@ cudaError_t launch_cfg(const TcGemmArgs& a, dim3 grid, cudaStream_t stream) {
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
-  gemm_tc_kernel<BN, STAGES><<<grid, 128, smem, stream>>>(a);
+  launch_pdl(gemm_tc_kernel<BN, STAGES>, grid, dim3(128), smem, stream, a);
   return cudaGetLastError();
 }
 
@@ -847,7 +849,7 @@ cudaError_t launch_wgrad_update(const WgradUpdateArgs& a, cudaStream_t stream) {
     attr_dev = dev;
   }
   const int grid = (int)std::min<int64_t>(tiles, sms);
-  wgrad_update_kernel<<<grid, wu::THREADS, smem, stream>>>(a);
+  launch_pdl(wgrad_update_kernel, dim3(grid), dim3(wu::THREADS), smem, stream, a);
   return cudaGetLastError();
 }
 

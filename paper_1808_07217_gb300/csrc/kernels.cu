@@ -30,6 +30,7 @@ int grid_for(int64_t work_items, int threads, int per_sm = 8) {
 // I^k_s[j] = k S + mulhi(word_{j mod 4}(Philox((j/4, s, k, 0), seed)), S), S = floor(N / K).
 __global__ void sample_indices_kernel(int32_t* __restrict__ idx, uint32_t k0, uint32_t k1,
                                       uint32_t step, int K, int B, uint32_t S) {
+  pdl_begin();
   const int groups = (B + 3) / 4;
   const int t = blockIdx.x * blockDim.x + threadIdx.x;
   if (t >= K * groups) return;
@@ -75,6 +76,7 @@ __device__ __forceinline__ uint32_t feistel_pi(uint32_t i, uint32_t N, int h, ui
 __global__ void sample_reshuffle_kernel(int32_t* __restrict__ idx, uint32_t k0, uint32_t k1,
                                         uint32_t epoch, int64_t t, int K, int B, uint32_t S,
                                         uint32_t N, int h) {
+  pdl_begin();
   const int q = blockIdx.x * blockDim.x + threadIdx.x;
   if (q >= K * B) return;
   const int k = q / B, j = q % B;
@@ -89,6 +91,7 @@ __global__ void gather_rows_kernel(void* __restrict__ dst, int ld_dst, const flo
                                    int D, const int32_t* __restrict__ idx, int rows,
                                    const int32_t* __restrict__ lab_in, int32_t* __restrict__ lab_out,
                                    const float* __restrict__ t_in, float* __restrict__ t_out) {
+  pdl_begin();
   const int r = blockIdx.x;
   if (r >= rows) return;
   const int64_t src_row = idx ? (int64_t)idx[r] : (int64_t)r;
@@ -131,6 +134,7 @@ __global__ void __launch_bounds__(256) softmax_xent_kernel(
     const float* __restrict__ logits, int ld, int C, const int32_t* __restrict__ labels, int B,
     TD* __restrict__ dz, int ld_dz, float* __restrict__ loss_mean, float* __restrict__ loss_sum,
     float* __restrict__ row_out) {
+  pdl_begin();
   __shared__ float red[256];
   const int g = blockIdx.x;
   const float inv_b = 1.0f / (float)B;
@@ -170,6 +174,7 @@ template <typename TD>
 __global__ void lsq_loss_kernel(const float* __restrict__ z, int ld, const float* __restrict__ t,
                                 int B, TD* __restrict__ dz, int ld_dz, float* __restrict__ loss_mean,
                                 float* __restrict__ loss_sum, float* __restrict__ row_out) {
+  pdl_begin();
   extern __shared__ float row_loss[];
   const int g = blockIdx.x;
   const float inv_b = 1.0f / (float)B;
@@ -195,6 +200,7 @@ template <typename TD, bool UPD>
 __global__ void __launch_bounds__(256) colsum_kernel(const TD* __restrict__ dz, int ld, int B,
                                                      int out, float* __restrict__ gb, int64_t gb_gs,
                                                      SgdParams sgd) {
+  pdl_begin();
   __shared__ float part[8][65];
   const int g = blockIdx.y;
   const int tx = threadIdx.x, ty = threadIdx.y;
@@ -246,6 +252,7 @@ __global__ void __launch_bounds__(256) sgd_update_kernel(
     float4* __restrict__ w, float4* __restrict__ u, const float4* __restrict__ g,
     uint2* __restrict__ wb, int64_t n4, float lr, float m, float wd, int64_t period,
     int64_t decay_end, int sgn) {
+  pdl_begin();
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n4; i += stride) {
     const float4 gv = __ldcs(g + i);
@@ -279,6 +286,7 @@ template <bool SHADOW>
 __global__ void __launch_bounds__(256) kway_average_kernel(float4* __restrict__ W,
                                                            uint2* __restrict__ Wb, int K,
                                                            int64_t d4) {
+  pdl_begin();
   // blockIdx.y selects a group of K consecutive replicas (one group for the global average)
   W += (int64_t)blockIdx.y * K * d4;
   if (SHADOW) Wb += (int64_t)blockIdx.y * K * d4;
@@ -344,6 +352,7 @@ __global__ void __launch_bounds__(kL1Threads) l1_partial_kernel(const float4* __
                                                                 const float4* __restrict__ E,
                                                                 int K, int64_t d4, int nq,
                                                                 float* __restrict__ part) {
+  pdl_begin();
   extern __shared__ float red[];  // [kL1Threads / 32][K]
   const int q = blockIdx.x, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int64_t base = (int64_t)q * kL1Chunk + threadIdx.x;
@@ -398,6 +407,7 @@ __global__ void __launch_bounds__(kL1Threads) l1_partial_kernel(const float4* __
 // stride of chunks in fp64, then a fixed-shape tree over the block.
 __global__ void __launch_bounds__(256) l1_finalize_kernel(const float* __restrict__ part, int nq,
                                                           double d_canon, float* __restrict__ p) {
+  pdl_begin();
   __shared__ double red[256];
   const int k = blockIdx.x;
   double s = 0.0;
@@ -418,6 +428,7 @@ __global__ void __launch_bounds__(256) sign_sync_kernel(float4* __restrict__ W, 
                                                         float4* __restrict__ wref, float4* __restrict__ E,
                                                         const float* __restrict__ p, int K,
                                                         int64_t d4) {
+  pdl_begin();
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < d4; i += stride) {
     const float4 r = wref[i];
@@ -480,6 +491,7 @@ template <bool SHADOW>
 __global__ void __launch_bounds__(256) gm_sync_kernel(float4* __restrict__ W, uint2* __restrict__ Wb,
                                                       float4* __restrict__ wref, float4* __restrict__ ug,
                                                       int K, int64_t d4, float lr, float mg) {
+  pdl_begin();
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < d4; i += stride) {
     const float4 r = wref[i];
@@ -595,7 +607,7 @@ cudaError_t launch_sample_indices(int32_t* idx, uint64_t seed, int64_t step, int
     while ((1ll << (2 * h)) < N) ++h;
     const int threads = 128;
     const int blocks = (int)((KB + threads - 1) / threads);
-    sample_reshuffle_kernel<<<blocks, threads, 0, stream>>>(idx, (uint32_t)seed, (uint32_t)(seed >> 32),
+    launch_pdl(sample_reshuffle_kernel, blocks, threads, 0, stream, idx, (uint32_t)seed, (uint32_t)(seed >> 32),
                                                             (uint32_t)e, step - first, K, B,
                                                             (uint32_t)S, (uint32_t)N, h);
     return cudaGetLastError();
@@ -603,7 +615,7 @@ cudaError_t launch_sample_indices(int32_t* idx, uint64_t seed, int64_t step, int
   const int groups = (B + 3) / 4;
   const int threads = 128;
   const int blocks = (int)(((int64_t)K * groups + threads - 1) / threads);
-  sample_indices_kernel<<<blocks, threads, 0, stream>>>(idx, (uint32_t)seed, (uint32_t)(seed >> 32),
+  launch_pdl(sample_indices_kernel, blocks, threads, 0, stream, idx, (uint32_t)seed, (uint32_t)(seed >> 32),
                                                         (uint32_t)step, K, B, (uint32_t)S);
   return cudaGetLastError();
 }
@@ -616,10 +628,10 @@ cudaError_t launch_gather_rows(void* dst, bool dst_bf16, int ld_dst, const float
   if (ld_dst < D) return cudaErrorInvalidValue;
   const int threads = D >= 1024 ? 256 : 128;
   if (dst_bf16)
-    gather_rows_kernel<true><<<rows, threads, 0, stream>>>(dst, ld_dst, X, D, idx, rows, labels_in,
+    launch_pdl(gather_rows_kernel<true>, rows, threads, 0, stream, dst, ld_dst, X, D, idx, rows, labels_in,
                                                            labels_out, targets_in, targets_out);
   else
-    gather_rows_kernel<false><<<rows, threads, 0, stream>>>(dst, ld_dst, X, D, idx, rows, labels_in,
+    launch_pdl(gather_rows_kernel<false>, rows, threads, 0, stream, dst, ld_dst, X, D, idx, rows, labels_in,
                                                             labels_out, targets_in, targets_out);
   return cudaGetLastError();
 }
@@ -631,11 +643,11 @@ cudaError_t launch_softmax_xent(const float* logits, int ld, int C, const int32_
   if (B > 8192 || C < 1) return cudaErrorInvalidValue;
   const int threads = B >= 256 ? 256 : (B >= 128 ? 128 : (B >= 64 ? 64 : 32));
   if (dz_bf16)
-    softmax_xent_kernel<uint16_t><<<G, threads, 0, stream>>>(
+    launch_pdl(softmax_xent_kernel<uint16_t>, G, threads, 0, stream, 
         logits, ld, C, labels, B, reinterpret_cast<uint16_t*>(dz), ld_dz, loss_mean, loss_sum,
         row_loss);
   else
-    softmax_xent_kernel<float><<<G, threads, 0, stream>>>(
+    launch_pdl(softmax_xent_kernel<float>, G, threads, 0, stream, 
         logits, ld, C, labels, B, reinterpret_cast<float*>(dz), ld_dz, loss_mean, loss_sum,
         row_loss);
   return cudaGetLastError();
@@ -648,10 +660,10 @@ cudaError_t launch_lsq_loss(const float* z, int ld, const float* targets, int G,
   if (B > 8192) return cudaErrorInvalidValue;
   const size_t smem = (size_t)B * sizeof(float);
   if (dz_bf16)
-    lsq_loss_kernel<uint16_t><<<G, 256, smem, stream>>>(
+    launch_pdl(lsq_loss_kernel<uint16_t>, G, 256, smem, stream, 
         z, ld, targets, B, reinterpret_cast<uint16_t*>(dz), ld_dz, loss_mean, loss_sum, row_loss);
   else
-    lsq_loss_kernel<float><<<G, 256, smem, stream>>>(z, ld, targets, B, reinterpret_cast<float*>(dz),
+    launch_pdl(lsq_loss_kernel<float>, G, 256, smem, stream, z, ld, targets, B, reinterpret_cast<float*>(dz),
                                                      ld_dz, loss_mean, loss_sum, row_loss);
   return cudaGetLastError();
 }
@@ -663,10 +675,10 @@ cudaError_t launch_colsum(const void* dz, bool dz_bf16, int ld, int G, int B, in
   dim3 grid((out + 63) / 64, G), block(32, 8);
   const SgdParams none{};
   if (dz_bf16)
-    colsum_kernel<uint16_t, false><<<grid, block, 0, stream>>>(
+    launch_pdl(colsum_kernel<uint16_t, false>, grid, block, 0, stream, 
         reinterpret_cast<const uint16_t*>(dz), ld, B, out, gb, gb_gs, none);
   else
-    colsum_kernel<float, false><<<grid, block, 0, stream>>>(reinterpret_cast<const float*>(dz), ld, B,
+    launch_pdl(colsum_kernel<float, false>, grid, block, 0, stream, reinterpret_cast<const float*>(dz), ld, B,
                                                             out, gb, gb_gs, none);
   return cudaGetLastError();
 }
@@ -677,10 +689,10 @@ cudaError_t launch_colsum_update(const void* dz, bool dz_bf16, int ld, int G, in
   if (G > 65535 || !sgd.w || (sgd.mom != 0.f && !sgd.u)) return cudaErrorInvalidValue;
   dim3 grid((out + 63) / 64, G), block(32, 8);
   if (dz_bf16)
-    colsum_kernel<uint16_t, true><<<grid, block, 0, stream>>>(reinterpret_cast<const uint16_t*>(dz),
+    launch_pdl(colsum_kernel<uint16_t, true>, grid, block, 0, stream, reinterpret_cast<const uint16_t*>(dz),
                                                               ld, B, out, nullptr, gs, sgd);
   else
-    colsum_kernel<float, true><<<grid, block, 0, stream>>>(reinterpret_cast<const float*>(dz), ld, B,
+    launch_pdl(colsum_kernel<float, true>, grid, block, 0, stream, reinterpret_cast<const float*>(dz), ld, B,
                                                            out, nullptr, gs, sgd);
   return cudaGetLastError();
 }
@@ -700,7 +712,7 @@ cudaError_t launch_sgd_update(float* w, float* u, const float* g, uint16_t* wb, 
   auto G = reinterpret_cast<const float4*>(g);
   auto WB = reinterpret_cast<uint2*>(wb);
 #define LSGD_UPD(M, NE, S)                                                                     \
-  sgd_update_kernel<M, NE, S><<<blocks, threads, 0, stream>>>(W, U, G, WB, n4, lr, momentum, \
+  launch_pdl(sgd_update_kernel<M, NE, S>, blocks, threads, 0, stream, W, U, G, WB, n4, lr, momentum, \
                                                               weight_decay, period, decay_end, \
                                                               sign_steps)
   const bool sh = wb != nullptr;
@@ -728,10 +740,10 @@ cudaError_t launch_group_average(float* W, uint16_t* Wb, int Kp, int groups, int
   const int blocks = std::max(1, grid_for(d4, threads, 8) / groups);
   dim3 grid(blocks, groups);
   if (Wb)
-    kway_average_kernel<true><<<grid, threads, 0, stream>>>(reinterpret_cast<float4*>(W),
+    launch_pdl(kway_average_kernel<true>, grid, threads, 0, stream, reinterpret_cast<float4*>(W),
                                                             reinterpret_cast<uint2*>(Wb), Kp, d4);
   else
-    kway_average_kernel<false><<<grid, threads, 0, stream>>>(reinterpret_cast<float4*>(W), nullptr,
+    launch_pdl(kway_average_kernel<false>, grid, threads, 0, stream, reinterpret_cast<float4*>(W), nullptr,
                                                              Kp, d4);
   return cudaGetLastError();
 }
@@ -747,12 +759,12 @@ cudaError_t launch_l1_norms(const float* W, const float* wref, const float* E, i
   auto R4 = reinterpret_cast<const float4*>(wref);
   auto E4 = reinterpret_cast<const float4*>(E);
   if (E)
-    l1_partial_kernel<true><<<nq, kL1Threads, smem, stream>>>(W4, R4, E4, K, d / 4, nq, part);
+    launch_pdl(l1_partial_kernel<true>, nq, kL1Threads, smem, stream, W4, R4, E4, K, d / 4, nq, part);
   else
-    l1_partial_kernel<false><<<nq, kL1Threads, smem, stream>>>(W4, R4, E4, K, d / 4, nq, part);
+    launch_pdl(l1_partial_kernel<false>, nq, kL1Threads, smem, stream, W4, R4, E4, K, d / 4, nq, part);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  l1_finalize_kernel<<<K, 256, 0, stream>>>(part, nq, (double)d_canon, p);
+  launch_pdl(l1_finalize_kernel, K, 256, 0, stream, part, nq, (double)d_canon, p);
   return cudaGetLastError();
 }
 
@@ -766,11 +778,11 @@ cudaError_t launch_sign_sync(float* W, uint16_t* Wb, float* wref, float* E, cons
   auto E4 = reinterpret_cast<float4*>(E);
   auto B2 = reinterpret_cast<uint2*>(Wb);
   if (E) {
-    if (Wb) sign_sync_kernel<true, true><<<blocks, 256, 0, stream>>>(W4, B2, R4, E4, p, K, d4);
-    else sign_sync_kernel<true, false><<<blocks, 256, 0, stream>>>(W4, B2, R4, E4, p, K, d4);
+    if (Wb) launch_pdl(sign_sync_kernel<true, true>, blocks, 256, 0, stream, W4, B2, R4, E4, p, K, d4);
+    else launch_pdl(sign_sync_kernel<true, false>, blocks, 256, 0, stream, W4, B2, R4, E4, p, K, d4);
   } else {
-    if (Wb) sign_sync_kernel<false, true><<<blocks, 256, 0, stream>>>(W4, B2, R4, E4, p, K, d4);
-    else sign_sync_kernel<false, false><<<blocks, 256, 0, stream>>>(W4, B2, R4, E4, p, K, d4);
+    if (Wb) launch_pdl(sign_sync_kernel<false, true>, blocks, 256, 0, stream, W4, B2, R4, E4, p, K, d4);
+    else launch_pdl(sign_sync_kernel<false, false>, blocks, 256, 0, stream, W4, B2, R4, E4, p, K, d4);
   }
   return cudaGetLastError();
 }
@@ -784,8 +796,8 @@ cudaError_t launch_gm_sync(float* W, uint16_t* Wb, float* wref, float* ug, int K
   auto R4 = reinterpret_cast<float4*>(wref);
   auto U4 = reinterpret_cast<float4*>(ug);
   auto B2 = reinterpret_cast<uint2*>(Wb);
-  if (Wb) gm_sync_kernel<true><<<blocks, 256, 0, stream>>>(W4, B2, R4, U4, K, d4, lr, mg);
-  else gm_sync_kernel<false><<<blocks, 256, 0, stream>>>(W4, B2, R4, U4, K, d4, lr, mg);
+  if (Wb) launch_pdl(gm_sync_kernel<true>, blocks, 256, 0, stream, W4, B2, R4, U4, K, d4, lr, mg);
+  else launch_pdl(gm_sync_kernel<false>, blocks, 256, 0, stream, W4, B2, R4, U4, K, d4, lr, mg);
   return cudaGetLastError();
 }
 

@@ -9,6 +9,27 @@
 
 namespace lsgd {
 
+// Launch `kernel` with programmatic dependent launch allowed (the kernel begins with pdl_begin()):
+// it may be scheduled while the previous kernel on the stream finishes, hiding launch latency and
+// its own prologue.
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                              cudaStream_t stream, Args... args) {
+  static_assert(sizeof...(KArgs) == sizeof...(Args), "argument count");
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+}
+
+
 // Record the message lsgd_last_error(NULL) returns on this thread.
 void set_last_error(const std::string& msg);
 

@@ -12,7 +12,8 @@ CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(PKG, "_build")
 LIBDIR = os.path.join(PKG, "_lib")
 LIB = os.path.join(LIBDIR, "liblsgd.so")
-SOURCES = ["kernels.cu", "gemm_simt.cu", "gemm_tc.cu", "resnet.cu", "runtime.cu", "bn_noalloc.cu"]
+SOURCES = ["kernels.cu", "gemm_simt.cu", "gemm_tc.cu", "head.cu", "resnet.cu", "runtime.cu",
+           "bn_noalloc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2"]
 

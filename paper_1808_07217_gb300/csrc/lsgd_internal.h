@@ -165,6 +165,32 @@ struct WgradUpdateArgs {
   CUtensorMap wmap, umap, wbmap;
 };
 cudaError_t launch_wgrad_update(const WgradUpdateArgs& a, cudaStream_t stream);
+// The classifier head (last dense layer with at most kHeadMaxClasses outputs, bf16 mode): the
+// forward product + softmax cross-entropy, then data / weight / bias gradients with the fused
+// update (or the gradient into `grad`).  Replica g's parameters start at g * rep_stride.
+constexpr int kHeadMaxClasses = 16;
+struct HeadArgs {
+  int C, B, in, reps;
+  int64_t rep_stride, w_off, b_off;
+  const uint16_t* act;  // [reps][B][ld_in] bf16 input of the last layer
+  int ld_in;
+  const uint16_t* Wb;   // bf16 shadow of the parameters (the products' operand)
+  const float* W;       // fp32 parameters (the bias of the forward)
+  const int32_t* labels;  // [reps][B]
+  uint16_t* dz;         // [reps][B][ld_dz] bf16 logits gradient
+  int ld_dz;
+  uint16_t* dz_prev;    // [reps][B][ld_dz_prev] data gradient for the layer below (NULL: none)
+  int ld_dz_prev;
+  float* row_loss;      // [reps][B]
+  float* loss_mean;     // [reps]
+  int fused;            // 1: apply the update through sgd (arena base pointers); 0: write grad
+  SgdParams sgd;
+  float* grad;
+};
+bool head_supported(int C, int B, int in);
+cudaError_t launch_head_forward(const HeadArgs& h, cudaStream_t stream);
+cudaError_t launch_head_backward(const HeadArgs& h, cudaStream_t stream);
+
 // Rank-3 TMA map over [dim2][dim1][dim0] (fp32 or bf16) with strides (elements) s1, s2, box
 // {box0, box1, 1} and a swizzle of 0, 32, 64 or 128 bytes.
 bool make_tma_map(CUtensorMap* map, const void* base, bool bf16, uint64_t dim0, uint64_t dim1,

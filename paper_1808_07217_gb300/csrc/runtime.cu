@@ -58,6 +58,8 @@ struct lsgd_ctx {
   int D = 0, C = 0;  // input width, outputs
   bool bf16 = false, lsq = false, resnet = false;
   bool fused = false;  // update applied in the weight-gradient epilogues (see lsgd_config)
+  bool head = false;   // last layer + loss by the two classifier-head kernels (bf16, few classes)
+  float* loss_slot_now = nullptr;  // this step's entry of the loss history (head path)
   std::vector<DenseLayer> layers;
   std::vector<Seg> segs;
   int64_t wd_period = 0, wd_end = 0;
@@ -342,12 +344,12 @@ lsgd_status tc_gemm(lsgd_ctx* c, const lsgd::TcGemmArgs& g) {
 }
 
 // Forward of every dense layer for `groups` groups.  Weights come from replica (w_g0 + g * w_gmul).
-lsgd_status dense_forward(lsgd_ctx* c, int groups, int w_g0, int w_gmul) {
+lsgd_status dense_forward(lsgd_ctx* c, int groups, int w_g0, int w_gmul, bool skip_last = false) {
   const int B = c->cfg.B_loc;
   const int L = (int)c->layers.size();
   const void* Wop = c->bf16 ? (const void*)c->Wb : (const void*)c->W;
   const size_t esz = c->bf16 ? 2 : 4;
-  for (int l = 0; l < L; ++l) {
+  for (int l = 0; l < (skip_last ? L - 1 : L); ++l) {
     const DenseLayer& Ly = c->layers[l];
     const bool last = l == L - 1;
     void* out = last ? (void*)c->logits : c->act[l + 1];
@@ -402,6 +404,28 @@ lsgd_status dense_forward(lsgd_ctx* c, int groups, int w_g0, int w_gmul) {
   return LSGD_OK;
 }
 
+// The classifier-head kernels' view of the last layer (forward + loss and backward share it).
+lsgd::HeadArgs head_args(lsgd_ctx* c) {
+  const DenseLayer& Ly = c->layers.back();
+  lsgd::HeadArgs h{};
+  h.C = Ly.out;
+  h.B = c->cfg.B_loc;
+  h.in = Ly.in;
+  h.reps = c->cfg.K;
+  h.rep_stride = c->d_pad;
+  h.w_off = Ly.w_off;
+  h.b_off = Ly.b_off;
+  h.act = (const uint16_t*)c->act[c->layers.size() - 1];
+  h.ld_in = Ly.ld_in;
+  h.Wb = c->Wb;
+  h.W = c->W;
+  h.labels = c->yb;
+  h.dz = (uint16_t*)c->dz[0];
+  h.ld_dz = c->ld_dz;
+  h.row_loss = c->row_loss;
+  return h;
+}
+
 // Backward of every dense layer, last to first: data gradient (it reads this layer's weights, so
 // it runs before a fused update may change them), weight gradient, bias gradient.
 lsgd_status dense_backward(lsgd_ctx* c) {
@@ -434,7 +458,24 @@ lsgd_status dense_backward(lsgd_ctx* c) {
     e_prev = e;
   };
   int cur = 0;
-  for (int l = L - 1; l >= 0; --l) {
+  int l_top = L - 1;
+  if (c->head) {
+    // the last layer's weight / bias gradients and their update (its data gradient for the layer
+    // below came with the head's forward kernel)
+    lsgd::HeadArgs h = head_args(c);
+    h.loss_mean = c->loss_slot_now;
+    h.fused = c->fused ? 1 : 0;
+    h.sgd = sgd;
+    h.sgd.w = c->W;
+    h.sgd.u = c->U;
+    h.sgd.wb = c->Wb;
+    h.grad = c->G;
+    LSGD_LAUNCH(c, lsgd::launch_head_backward(h, c->stream));
+    span(LSGD_PH_UPDATE);
+    l_top = L - 2;
+    cur = 1;
+  }
+  for (int l = l_top; l >= 0; --l) {
     const DenseLayer& Ly = c->layers[l];
     const void* dz = c->dz[cur];
     if (l > 0) {
@@ -617,11 +658,21 @@ lsgd_status step_body(lsgd_ctx* c, int64_t e_start) {
     e_bwd = prof_mark(c);
     prof_span(c, LSGD_PH_FORWARD, e_in, e_bwd);
   } else {
-    st = dense_forward(c, K, 0, 1);
+    st = dense_forward(c, K, 0, 1, c->head);
     if (st != LSGD_OK) return st;
     const int64_t e_fwd = prof_mark(c);
     prof_span(c, LSGD_PH_FORWARD, e_in, e_fwd);
-    st = dense_loss(c, K, false, loss_slot);
+    if (c->head) {
+      // the last layer's product, the loss, the logits gradient and the data gradient for the
+      // layer below in one kernel; the mean loss is finished by the head's backward kernel
+      lsgd::HeadArgs h = head_args(c);
+      h.dz_prev = c->layers.size() > 1 ? (uint16_t*)c->dz[1] : nullptr;
+      h.ld_dz_prev = c->ld_dz;
+      LSGD_LAUNCH(c, lsgd::launch_head_forward(h, c->stream));
+      c->loss_slot_now = loss_slot;
+    } else {
+      st = dense_loss(c, K, false, loss_slot);
+    }
     if (st != LSGD_OK) return st;
     const int64_t e_loss = prof_mark(c);
     prof_span(c, LSGD_PH_LOSS, e_fwd, e_loss);
@@ -802,6 +853,10 @@ lsgd_status lsgd_create(const lsgd_config* cfg, const lsgd_allocator* alloc, voi
     if (st == LSGD_OK && c0.fused_update && c->bf16) {
       c->fused = true;
       for (const DenseLayer& L : c->layers) c->fused = c->fused && L.tc;
+    }
+    if (st == LSGD_OK) {
+      const DenseLayer& top = c->layers.back();
+      c->head = c->bf16 && !c->lsq && top.tc && lsgd::head_supported(top.out, c0.B_loc, top.in);
     }
   }
   if (st != LSGD_OK) {

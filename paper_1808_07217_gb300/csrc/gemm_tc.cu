@@ -357,6 +357,15 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
             v.z = a0[q].z > 0.f ? v.z : 0.f;
             v.w = a0[q].w > 0.f ? v.w : 0.f;
           }
+          if (args.bias_colsum) {
+            // keep the stored (rounded) value for the column sums below; each item is this
+            // thread's alone
+            const int it = base + q * 128;
+            const float4 r4 = args.c_bf16 ? make_float4(bf2f(f2bf(v.x)), bf2f(f2bf(v.y)),
+                                                        bf2f(f2bf(v.z)), bf2f(f2bf(v.w)))
+                                          : v;
+            *reinterpret_cast<float4*>(stg + (it / (CW / 4)) * PITCH + (it % (CW / 4)) * 4) = r4;
+          }
           if (args.c_bf16) {
             uint16_t* out = reinterpret_cast<uint16_t*>(args.C) + off[q];
             if (full4 && ((reinterpret_cast<uintptr_t>(out) & 7) == 0)) {
@@ -380,6 +389,41 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
         }
       }
       asm volatile("bar.sync 1, 128;" ::: "memory");
+      if (args.bias_colsum) {
+        // Bias gradient of the layer this data gradient feeds: the sum over all rows (the tile
+        // holds the whole mini-batch) of the stored values, per column; two row halves per
+        // column, added in a fixed order, then the local update of that bias (or its gradient).
+        float* hs = stg + BM * PITCH;  // 2 x 64 partial sums after the staged tile
+        const int col = threadIdx.x & (CW - 1), half = threadIdx.x / CW;
+        float sum = 0.f;
+        const int r1 = min(args.M - m0, BM);
+        for (int row = half * (BM / 2); row < min(r1, (half + 1) * (BM / 2)); ++row)
+          sum += stg[row * PITCH + col];
+        hs[half * CW + col] = sum;
+        asm volatile("bar.sync 1, 128;" ::: "memory");
+        const int n = n0 + cc + threadIdx.x;
+        if (threadIdx.x < CW && n < args.N) {
+          const float gb = hs[threadIdx.x] + hs[CW + threadIdx.x];
+          const int64_t k = (int64_t)g * args.bias_gs + n;
+          if (!args.bsgd.w) {
+            args.bias_grad[k] = gb;
+          } else {
+            const SgdParams& sp = args.bsgd;
+            float w = sp.w[k], u = sp.u ? sp.u[k] : 0.f;
+            const bool sg = sp.sign != 0;
+            if (sp.mom == 0.f)
+              sgd_elem<false, false>(w, u, gb, sp.lr, 0.f, sp.wd, sg);
+            else if (sp.nesterov)
+              sgd_elem<true, true>(w, u, gb, sp.lr, sp.mom, sp.wd, sg);
+            else
+              sgd_elem<true, false>(w, u, gb, sp.lr, sp.mom, sp.wd, sg);
+            sp.w[k] = w;
+            if (sp.u) sp.u[k] = u;
+            if (sp.wb) sp.wb[k] = f2bf(w);
+          }
+        }
+        asm volatile("bar.sync 1, 128;" ::: "memory");
+      }
     }
   }
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
@@ -874,6 +918,9 @@ cudaError_t launch_gemm_tc(const TcGemmArgs& a, cudaStream_t stream) {
   if ((a.epi == EPI_BIAS || a.epi == EPI_BIAS_RELU) && !a.bias) return cudaErrorInvalidValue;
   if (a.epi == EPI_MASK && !a.mask) return cudaErrorInvalidValue;
   if (!a.C) return cudaErrorInvalidValue;
+  // the bias column sums need the whole mini-batch in one tile, and the masked data gradient
+  if (a.bias_colsum && (a.M > BM || a.epi != EPI_MASK || (!a.bsgd.w && !a.bias_grad)))
+    return cudaErrorInvalidValue;
   const int splits = a.splits > 1 ? a.splits : 1;
   if (splits > 1) {
     const int nk_all = (a.Kd + BK - 1) / BK, per = (nk_all + splits - 1) / splits;

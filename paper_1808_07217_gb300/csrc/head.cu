@@ -7,9 +7,10 @@
 //
 //   head_forward_kernel   z = a W^T + b, l = logsumexp(z) - z_y, dZ = (softmax(z) - onehot(y)) / B,
 //                         and dA = (dZ W) * (a > 0) for the layer below, row by row
-//   head_backward_kernel  per 64-column block of W: gW = dZ^T a, and for block 0 gb = sum_j dZ_j
-//                         and the mean loss; then the local update of those parameters (fused
-//                         mode) or the gradient (else)
+//   head_backward_kernel  per 64-column block of W: gW = dZ^T a, the bias gradient of the layer
+//                         below for those 64 columns (sum over rows of dA), and for block 0
+//                         gb = sum_j dZ_j and the mean loss; then the local update of those
+//                         parameters (fused mode) or the gradients (else)
 #include "../../include/lsgd.h"
 #include "common.cuh"
 #include "lsgd_internal.h"
@@ -218,6 +219,39 @@ __global__ void __launch_bounds__(256) head_backward_kernel(HeadArgs h) {
     sp.w[k] = w;
     if (sp.u) sp.u[k] = u;
     if (sp.wb) sp.wb[k] = f2bf(w);
+  }
+  // the layer below: its bias gradient for this block's 64 columns = sum over rows of the bf16
+  // data gradient the forward kernel stored (four row quarters, then added in quarter order)
+  if (h.b_prev_off >= 0 && h.dz_prev) {
+    __syncthreads();  // part[] is free again
+    const int n = t & (kHeadCols - 1), qtr = t / kHeadCols;  // 4 quarters of the rows
+    float s = 0.f;
+    if (n0 + n < h.in) {
+      const int rows = (h.B + 3) / 4, j0 = qtr * rows, j1 = min(h.B, j0 + rows);
+      for (int j = j0; j < j1; ++j)
+        s += bf2f(h.dz_prev[((int64_t)g * h.B + j) * h.ld_dz_prev + n0 + n]);
+    }
+    part[qtr * kHeadCols + n] = s;
+    __syncthreads();
+    if (t < kHeadCols && n0 + t < h.in) {
+      const float gb = ((part[t] + part[kHeadCols + t]) + part[2 * kHeadCols + t]) +
+                       part[3 * kHeadCols + t];
+      const int64_t k = rep + h.b_prev_off + n0 + t;
+      if (!h.fused) {
+        h.grad[k] = gb;
+      } else {
+        float w = sp.w[k], u = sp.u ? sp.u[k] : 0.f;
+        if (sp.mom == 0.f)
+          sgd_elem<false, false>(w, u, gb, sp.lr, 0.f, sp.wd, sg);
+        else if (sp.nesterov)
+          sgd_elem<true, true>(w, u, gb, sp.lr, sp.mom, sp.wd, sg);
+        else
+          sgd_elem<true, false>(w, u, gb, sp.lr, sp.mom, sp.wd, sg);
+        sp.w[k] = w;
+        if (sp.u) sp.u[k] = u;
+        if (sp.wb) sp.wb[k] = f2bf(w);
+      }
+    }
   }
   // bias gradient (one warp per class, a fixed butterfly over rows) and the mean loss (warp 7):
   // the first column block of each replica

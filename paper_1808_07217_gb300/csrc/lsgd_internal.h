@@ -122,6 +122,13 @@ struct GemmArgs {
   const void* mask;
   int64_t mask_rs, mask_gs;
   bool mask_bf16;
+  // EPI_MASK with M <= 128 (one tile holds the whole mini-batch): also form the column sums of the
+  // stored result -- the bias gradient of the layer it feeds -- and apply the local update to that
+  // bias through bsgd (bsgd.w at the bias, replica stride bias_gs), or, with bsgd.w == NULL, write
+  // it to bias_grad (same indexing)
+  bool bias_colsum;
+  SgdParams bsgd;
+  float* bias_grad;
 };
 
 cudaError_t launch_gemm_simt(const GemmArgs& a, cudaStream_t stream);
@@ -152,6 +159,13 @@ struct TcGemmArgs {
   const void* mask;
   int64_t mask_rs, mask_gs;
   bool mask_bf16;
+  // EPI_MASK with M <= 128 (one tile holds the whole mini-batch): also form the column sums of the
+  // stored result -- the bias gradient of the layer it feeds -- and apply the local update to that
+  // bias through bsgd (bsgd.w at the bias, replica stride bias_gs), or, with bsgd.w == NULL, write
+  // it to bias_grad (same indexing)
+  bool bias_colsum;
+  SgdParams bsgd;
+  float* bias_grad;
 };
 
 // The weight gradient of one dense layer fused with the local update, for G replicas: W[g] (M x
@@ -186,6 +200,9 @@ struct HeadArgs {
   int fused;            // 1: apply the update through sgd (arena base pointers); 0: write grad
   SgdParams sgd;
   float* grad;
+  // backward only: the bias gradient of the layer below (sum over rows of dz_prev, which the
+  // forward kernel wrote) and its update, column block by column block; b_prev_off < 0: none
+  int64_t b_prev_off;
 };
 bool head_supported(int C, int B, int in);
 cudaError_t launch_head_forward(const HeadArgs& h, cudaStream_t stream);

@@ -423,6 +423,7 @@ lsgd::HeadArgs head_args(lsgd_ctx* c) {
   h.dz = (uint16_t*)c->dz[0];
   h.ld_dz = c->ld_dz;
   h.row_loss = c->row_loss;
+  h.b_prev_off = -1;
   return h;
 }
 
@@ -459,11 +460,17 @@ lsgd_status dense_backward(lsgd_ctx* c) {
   };
   int cur = 0;
   int l_top = L - 1;
+  int bias_done = -1;  // layer whose bias the last data-gradient GEMM already handled
   if (c->head) {
     // the last layer's weight / bias gradients and their update (its data gradient for the layer
     // below came with the head's forward kernel)
     lsgd::HeadArgs h = head_args(c);
     h.loss_mean = c->loss_slot_now;
+    if (L > 1) {
+      h.dz_prev = (uint16_t*)c->dz[1];
+      h.ld_dz_prev = c->ld_dz;
+      h.b_prev_off = c->layers[L - 2].b_off;  // the layer below's bias, from the stored dA
+    }
     h.fused = c->fused ? 1 : 0;
     h.sgd = sgd;
     h.sgd.w = c->W;
@@ -504,6 +511,18 @@ lsgd_status dense_backward(lsgd_ctx* c) {
         t.mask_rs = Ly.ld_in;
         t.mask_gs = (int64_t)B * Ly.ld_in;
         t.mask_bf16 = c->bf16;
+        const DenseLayer& below = c->layers[l - 1];
+        if (below.b_off >= 0 && B <= lsgd::kTcTileM) {
+          // the whole mini-batch is one tile: the epilogue also sums the stored result over rows,
+          // which is the bias gradient of the layer below, and updates that bias
+          t.bias_colsum = true;
+          t.bias_gs = c->d_pad;
+          if (c->fused)
+            t.bsgd = sgd_at(below.b_off);
+          else
+            t.bias_grad = c->G + below.b_off;
+          bias_done = l - 1;
+        }
         lsgd_status st = tc_gemm(c, t);
         if (st != LSGD_OK) return st;
       } else {
@@ -605,7 +624,8 @@ lsgd_status dense_backward(lsgd_ctx* c) {
       if (st != LSGD_OK) return st;
     }
     span(LSGD_PH_UPDATE);
-    if (Ly.b_off >= 0) {
+    // the bias sums: unless the head's kernel (layer L - 2) or the data-gradient GEMM above did them
+    if (Ly.b_off >= 0 && !(c->head && l == L - 2) && bias_done != l) {
       if (c->fused)
         LSGD_LAUNCH(c, lsgd::launch_colsum_update(dz, c->bf16, c->ld_dz, K, B, Ly.out, c->d_pad,
                                                   sgd_at(Ly.b_off), c->stream));

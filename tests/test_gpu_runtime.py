@@ -164,7 +164,7 @@ def test_default_allocator_and_launch_count(P):
     P.lsgd_local_step(ctx)
     per_step = P.lsgd_kernel_launches(ctx) - before
     # sample, gather, the first layer's forward GEMM, the classifier head's two kernels (last
-    # layer forward + loss; its gradients, the data gradient below and its bias sum), the first
-    # layer's weight-gradient GEMM and bias sum, the update
-    assert per_step == 8
+    # layer forward, loss and the data gradient below; the head's gradients and the first layer's
+    # bias gradient), the first layer's weight-gradient GEMM, the update
+    assert per_step == 7
     P.lsgd_destroy(ctx)

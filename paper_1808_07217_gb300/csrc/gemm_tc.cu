@@ -92,6 +92,29 @@ __device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, u
       : "memory");
 }
 
+__device__ __forceinline__ void tma_load_5d(void* dst, const CUtensorMap* map, uint64_t* bar, int c0,
+                                            int c1, int c2, int c3, int c4) {
+  asm volatile(
+      "cp.async.bulk.tensor.5d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%3, %4, %5, %6, %7}], [%2];" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(bar)), "r"(c0), "r"(c1), "r"(c2), "r"(c3),
+      "r"(c4)
+      : "memory");
+}
+
+// Shared-memory descriptor of a K-major operand whose rows are `swz` bytes (32, 64 or 128) with the
+// matching swizzle: core matrices of 8 rows, SBO = 8 rows, layout code 6 / 4 / 2.
+__device__ __forceinline__ uint64_t smem_desc_kmajor(uint32_t addr, uint32_t swz) {
+  const uint64_t layout = swz == 128 ? 2ull : (swz == 64 ? 4ull : 6ull);
+  uint64_t d = 0;
+  d |= (uint64_t)((addr >> 4) & 0x3FFFu);
+  d |= (uint64_t)1u << 16;  // LBO (unused by swizzled K-major layouts)
+  d |= (uint64_t)(((8u * swz) >> 4) & 0x3FFFu) << 32;
+  d |= 1ull << 46;
+  d |= layout << 61;
+  return d;
+}
+
 __device__ __forceinline__ uint64_t smem_desc(uint32_t addr, uint32_t lbo, uint32_t sbo) {
   uint64_t d = 0;
   d |= (uint64_t)((addr >> 4) & 0x3FFFu);
@@ -178,8 +201,12 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int splits = args.splits > 1 ? args.splits : 1;
   const int n0 = blockIdx.x * BN, m0 = blockIdx.y * BM, g = blockIdx.z / splits;
+  // implicit convolution: the tile's 128 output pixels are rows of whole images (TW = Wout) from
+  // pixel m0 on, i.e. output row oy0 of image b0
+  const int cv_b0 = args.conv ? m0 / (args.cv_hout * args.cv_wout) : 0;
+  const int cv_oy0 = args.conv ? (m0 / args.cv_wout) % args.cv_hout : 0;
   const int split = blockIdx.z % splits;
-  const int nk_all = (args.Kd + BK - 1) / BK;
+  const int nk_all = args.conv ? 9 : (args.Kd + BK - 1) / BK;
   const int per_split = (nk_all + splits - 1) / splits;
   const int kb_first = split * per_split;
   const int nk = min(nk_all - kb_first, per_split);  // >= 1 (the host makes every split nonempty)
@@ -220,6 +247,17 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
         ok = false;
         break;
       }
+      if (args.conv) {
+        // tap t = kb: the input shifted by (kh - 1, kw - 1) (zero outside the image, stride by
+        // the map's element strides) and the weights' tap-t slice [N][Ck]
+        const int t = kb_first + kb, kh = t / 3, kw = t % 3;
+        mbar_expect_tx(&sm.full[s], (uint32_t)(BM + BN) * args.cv_ck * 2);
+        tma_load_5d(sm.a[s], &args.A.map, &sm.full[s], 0, kw - 1,
+                    cv_oy0 * args.cv_stride + kh - 1, cv_b0, g);
+        tma_load_3d(sm.b[s], &args.B.map, &sm.full[s], t * args.cv_ck, n0, g);
+        issued = kb + 1;
+        continue;
+      }
       mbar_expect_tx(&sm.full[s], kBytesA + kBytesB);
       const int k0 = (kb_first + kb) * BK;
       if (!a_mn) {
@@ -256,6 +294,15 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
       }
       asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
       const uint32_t a_base = smem_u32(sm.a[s]), b_base = smem_u32(sm.b[s]);
+      if (args.conv) {
+        // rows of Ck bf16 = swz bytes; K = 16 per MMA, 32 bytes further along the row
+        const uint32_t swz = (uint32_t)args.cv_ck * 2;
+        for (int kk = 0; kk < args.cv_ck / 16; ++kk)
+          mma_bf16(tmem, smem_desc_kmajor(a_base + kk * 32, swz),
+                   smem_desc_kmajor(b_base + kk * 32, swz), idesc, (kb > 0 || kk > 0) ? 1u : 0u);
+        mma_commit(&sm.empty[s]);
+        continue;
+      }
 #pragma unroll
       for (int kk = 0; kk < BK / 16; ++kk) {
         const uint64_t ad = a_mn ? smem_desc(a_base + kk * 2048, 64 * BK * 2, 1024)
@@ -897,6 +944,46 @@ cudaError_t launch_wgrad_update(const WgradUpdateArgs& a, cudaStream_t stream) {
   return cudaGetLastError();
 }
 
+bool conv_tile_shape(int hout, int wout, int* rows, int* images) {
+  if (wout < 1 || hout < 1 || wout > BM || BM % wout) return false;
+  const int per_image = hout * wout;
+  if (per_image >= BM) {
+    if (per_image % BM) return false;
+    *rows = BM / wout;
+    *images = 1;
+  } else {
+    if (BM % per_image) return false;
+    *rows = hout;
+    *images = BM / per_image;
+  }
+  return true;
+}
+
+bool make_tma_map_conv(CUtensorMap* map, const void* base, int ck, int win, int hin, int B, int G,
+                       int wout, int hout, int stride) {
+  std::call_once(g_encode_once, load_encode);
+  int rows = 0, images = 0;
+  if (!g_encode || (ck != 16 && ck != 32 && ck != 64) || (stride != 1 && stride != 2) ||
+      !conv_tile_shape(hout, wout, &rows, &images) || (reinterpret_cast<uintptr_t>(base) & 15))
+    return false;
+  if (wout * stride > 256 || rows * stride > 256 || images > 256) return false;
+  const uint64_t e = 2;
+  cuuint64_t dims[5] = {(cuuint64_t)ck, (cuuint64_t)win, (cuuint64_t)hin, (cuuint64_t)B,
+                        (cuuint64_t)G};
+  cuuint64_t strides[4] = {(cuuint64_t)ck * e, (cuuint64_t)win * ck * e,
+                           (cuuint64_t)hin * win * ck * e, (cuuint64_t)B * hin * win * ck * e};
+  cuuint32_t box[5] = {(cuuint32_t)ck, (cuuint32_t)(wout * stride), (cuuint32_t)(rows * stride),
+                       (cuuint32_t)images, 1};
+  cuuint32_t estr[5] = {1, (cuuint32_t)stride, (cuuint32_t)stride, 1, 1};
+  const CUtensorMapSwizzle sw = ck == 64 ? CU_TENSOR_MAP_SWIZZLE_128B
+                                         : (ck == 32 ? CU_TENSOR_MAP_SWIZZLE_64B
+                                                     : CU_TENSOR_MAP_SWIZZLE_32B);
+  CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5, const_cast<void*>(base), dims,
+                        strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, sw,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
 int tc_tile_n(int Kd) { return (Kd + BK - 1) / BK <= 2 ? 128 : 64; }
 
 int tc_valid_splits(int Kd, int want) {
@@ -918,6 +1005,18 @@ cudaError_t launch_gemm_tc(const TcGemmArgs& a, cudaStream_t stream) {
   if ((a.epi == EPI_BIAS || a.epi == EPI_BIAS_RELU) && !a.bias) return cudaErrorInvalidValue;
   if (a.epi == EPI_MASK && !a.mask) return cudaErrorInvalidValue;
   if (!a.C) return cudaErrorInvalidValue;
+  if (a.conv) {
+    // K-major tap slices of cv_ck channels on both sides; 64-wide N tiles, four stages, no split
+    int rows = 0, images = 0;
+    if ((a.cv_ck != 16 && a.cv_ck != 32 && a.cv_ck != 64) || (a.cv_stride != 1 && a.cv_stride != 2) ||
+        !conv_tile_shape(a.cv_hout, a.cv_wout, &rows, &images) || a.splits > 1 ||
+        a.A.mn_major || a.B.mn_major || a.bias_colsum)
+      return cudaErrorInvalidValue;
+    if (a.M % (a.cv_hout * a.cv_wout)) return cudaErrorInvalidValue;  // whole images
+    dim3 gridc((a.N + 63) / 64, (a.M + BM - 1) / BM, a.G);
+    if (gridc.y > 65535) return cudaErrorInvalidValue;
+    return launch_cfg<64, 4>(a, gridc, stream);
+  }
   // the bias column sums need the whole mini-batch in one tile, and the masked data gradient
   if (a.bias_colsum && (a.M > BM || a.epi != EPI_MASK || (!a.bsgd.w && !a.bias_grad)))
     return cudaErrorInvalidValue;

@@ -129,7 +129,19 @@ struct GemmArgs {
   bool bias_colsum;
   SgdParams bsgd;
   float* bias_grad;
+  // implicit 3x3 convolution (zero padding 1): C[p][n] = sum over taps t and k < cv_ck of
+  // in[shift_t(p)][k] B[n][t][k].  A is a rank-5 map over the NHWC input {cv_ck, W, H, B, G} whose
+  // box is {cv_ck, Wout * s, rows * s, images, 1} with element strides {1, s, s, 1, 1}; B a rank-3
+  // map over the [N][9][cv_ck] weights {9 cv_ck, N, G} with box {cv_ck, 64}; both swizzled by
+  // cv_ck * 2 bytes.  M = pixels of the output (whole rows per 128-pixel tile), Kd unused.
+  int conv;
+  int cv_ck, cv_stride, cv_hout, cv_wout;
 };
+// The tile geometry of an implicit convolution with an Hout x Wout output: whole output rows,
+// 128 pixels per tile.  False when the shape does not tile that way.
+bool conv_tile_shape(int hout, int wout, int* rows, int* images);
+bool make_tma_map_conv(CUtensorMap* map, const void* base, int ck, int win, int hin, int B, int G,
+                       int wout, int hout, int stride);
 
 cudaError_t launch_gemm_simt(const GemmArgs& a, cudaStream_t stream);
 
@@ -166,7 +178,19 @@ struct TcGemmArgs {
   bool bias_colsum;
   SgdParams bsgd;
   float* bias_grad;
+  // implicit 3x3 convolution (zero padding 1): C[p][n] = sum over taps t and k < cv_ck of
+  // in[shift_t(p)][k] B[n][t][k].  A is a rank-5 map over the NHWC input {cv_ck, W, H, B, G} whose
+  // box is {cv_ck, Wout * s, rows * s, images, 1} with element strides {1, s, s, 1, 1}; B a rank-3
+  // map over the [N][9][cv_ck] weights {9 cv_ck, N, G} with box {cv_ck, 64}; both swizzled by
+  // cv_ck * 2 bytes.  M = pixels of the output (whole rows per 128-pixel tile), Kd unused.
+  int conv;
+  int cv_ck, cv_stride, cv_hout, cv_wout;
 };
+// The tile geometry of an implicit convolution with an Hout x Wout output: whole output rows,
+// 128 pixels per tile.  False when the shape does not tile that way.
+bool conv_tile_shape(int hout, int wout, int* rows, int* images);
+bool make_tma_map_conv(CUtensorMap* map, const void* base, int ck, int win, int hin, int B, int G,
+                       int wout, int hout, int stride);
 
 // The weight gradient of one dense layer fused with the local update, for G replicas: W[g] (M x
 // N, row stride N) -= update(dZ[g]^T act[g]) with the momentum and bf16 shadow of SgdParams.

@@ -268,6 +268,79 @@ __global__ void __launch_bounds__(256) bn_stats_partial_kernel(const float* __re
   }
 }
 
+// The same for C a multiple of 4 (C / 4 dividing 256): thread = (group of 4 channels, pixel lane),
+// float4 loads; each pass's lane sums are combined by a fixed-shape tree in shared memory.
+__device__ __forceinline__ void tree_sum4(float4* red, int lane, int lanes, int cg, int C4) {
+  int span = 1;
+  while (span < lanes) span <<= 1;
+  for (int st = span >> 1; st > 0; st >>= 1) {
+    __syncthreads();
+    if (lane < st && lane + st < lanes) {
+      float4& a = red[lane * C4 + cg];
+      const float4 b = red[(lane + st) * C4 + cg];
+      a.x += b.x;
+      a.y += b.y;
+      a.z += b.z;
+      a.w += b.w;
+    }
+  }
+  __syncthreads();
+}
+
+__global__ void __launch_bounds__(256) bn_stats_partial_v4_kernel(const float* __restrict__ y,
+                                                                  int64_t P, int C, int nq,
+                                                                  float* __restrict__ part) {
+  __shared__ float4 red[256];
+  const int g = blockIdx.y, q = blockIdx.x;
+  const int C4 = C / 4, lanes = blockDim.x / C4;
+  const int cg = threadIdx.x % C4, l = threadIdx.x / C4;
+  const int64_t p0 = (int64_t)q * kStatChunk, p1 = min(P, p0 + kStatChunk);
+  const float4* yg = reinterpret_cast<const float4*>(y + (int64_t)g * P * C) + cg;
+  float4 s = make_float4(0.f, 0.f, 0.f, 0.f);
+  if (l < lanes) {
+#pragma unroll 4
+    for (int64_t p = p0 + l; p < p1; p += lanes) {
+      const float4 v = yg[p * C4];
+      s.x += v.x;
+      s.y += v.y;
+      s.z += v.z;
+      s.w += v.w;
+    }
+    red[l * C4 + cg] = s;
+  }
+  tree_sum4(red, l < lanes ? l : 0x7fffffff, lanes, cg, C4);
+  const float inv = 1.0f / (float)(p1 - p0);
+  const float4 tot = red[cg];
+  const float4 m = make_float4(tot.x * inv, tot.y * inv, tot.z * inv, tot.w * inv);
+  __syncthreads();  // everyone has read red[cg] before it is reused
+  float4 s2 = make_float4(0.f, 0.f, 0.f, 0.f);
+  if (l < lanes) {
+#pragma unroll 4
+    for (int64_t p = p0 + l; p < p1; p += lanes) {
+      const float4 v = yg[p * C4];
+      const float dx = v.x - m.x, dy = v.y - m.y, dz = v.z - m.z, dw = v.w - m.w;
+      s2.x = fmaf(dx, dx, s2.x);
+      s2.y = fmaf(dy, dy, s2.y);
+      s2.z = fmaf(dz, dz, s2.z);
+      s2.w = fmaf(dw, dw, s2.w);
+    }
+    red[l * C4 + cg] = s2;
+  }
+  tree_sum4(red, l < lanes ? l : 0x7fffffff, lanes, cg, C4);
+  if (l == 0) {
+    const float4 t2 = red[cg];
+    float* dst = part + (((int64_t)g * nq + q) * C + 4 * cg) * 2;
+    dst[0] = m.x;
+    dst[1] = t2.x;
+    dst[2] = m.y;
+    dst[3] = t2.y;
+    dst[4] = m.z;
+    dst[5] = t2.z;
+    dst[6] = m.w;
+    dst[7] = t2.w;
+  }
+}
+
 // Pass 2: Chan et al.'s pairwise combination of the chunk (count, mean, M2): one warp per
 // (replica, channel); lane l combines chunks l, l + 32, ... in order, then a fixed butterfly of
 // shuffles combines the lanes.  Biased variance, rstd = 1 / sqrt(var + eps).
@@ -381,6 +454,50 @@ __global__ void bn_act_fwd_kernel(const float* __restrict__ y, const float* __re
   }
 }
 
+// The same with a fixed group of 4 channels per thread (C / 4 dividing the block size): the
+// channels' gamma, beta, mean and rstd are loaded once, pixels advance by grid strides, and the
+// replica is blockIdx.y (32-bit pixel indexing).
+template <typename TA>
+__global__ void __launch_bounds__(256) bn_act_fwd_v4_kernel(
+    const float* __restrict__ y, const float* __restrict__ mean, const float* __restrict__ rstd,
+    const float* __restrict__ W, int64_t g_off, int64_t b_off, int64_t d_gs, int w_g0, int w_gmul,
+    const TA* __restrict__ sc, int sc_H, int sc_W, int sc_C, int stride, TA* __restrict__ out, int B,
+    int H, int Wd, int C) {
+  const int g = blockIdx.y, C4 = C / 4;
+  const int c0 = (threadIdx.x % C4) * 4, pl = threadIdx.x / C4, ppb = blockDim.x / C4;
+  const int P = B * H * Wd;
+  const float* Wg = W + (int64_t)(w_g0 + g * w_gmul) * d_gs;
+  float ga[4], be[4], mu[4], rs[4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    ga[i] = Wg[g_off + c0 + i];
+    be[i] = Wg[b_off + c0 + i];
+    mu[i] = mean[g * C + c0 + i];
+    rs[i] = rstd[g * C + c0 + i];
+  }
+  const bool with_sc = sc && c0 < sc_C;
+  const float* yg = y + (int64_t)g * P * C + c0;
+  TA* og = out + (int64_t)g * P * C + c0;
+  for (int p = blockIdx.x * ppb + pl; p < P; p += gridDim.x * ppb) {
+    const float4 yv = *reinterpret_cast<const float4*>(yg + (int64_t)p * C);
+    const float yy[4] = {yv.x, yv.y, yv.z, yv.w};
+    float v[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) v[i] = ga[i] * ((yy[i] - mu[i]) * rs[i]) + be[i];
+    if (with_sc) {
+      const int x = p % Wd, hb = p / Wd, h = hb % H, b = hb / H;
+      const float4 s4 = Vec4<TA>::load(
+          sc + ((((int64_t)g * B + b) * sc_H + h * stride) * sc_W + x * stride) * sc_C + c0);
+      v[0] += s4.x;
+      v[1] += s4.y;
+      v[2] += s4.z;
+      v[3] += s4.w;
+    }
+    Vec4<TA>::store(og + (int64_t)p * C, make_float4(fmaxf(v[0], 0.f), fmaxf(v[1], 0.f),
+                                                    fmaxf(v[2], 0.f), fmaxf(v[3], 0.f)));
+  }
+}
+
 // BatchNorm backward, pass 1: with dz = dout * (out > 0) and xhat = (y - mean) rstd, chunk sums
 // part[g][q][c] = (sum dz, sum dz xhat).
 template <typename TA>
@@ -416,6 +533,77 @@ __global__ void __launch_bounds__(256) bn_bwd_partial_kernel(
     float* dst = part + (((int64_t)g * nq + q) * C + threadIdx.x) * 2;
     dst[0] = t1;
     dst[1] = t2;
+  }
+}
+
+// The same for C a multiple of 4 (C / 4 dividing 256), float4 / 4-channel loads and a fixed-shape
+// tree over the pixel lanes.
+template <typename TA>
+__global__ void __launch_bounds__(256) bn_bwd_partial_v4_kernel(
+    const float* __restrict__ dout, const TA* __restrict__ out, const float* __restrict__ y,
+    const float* __restrict__ mean, const float* __restrict__ rstd, int64_t P, int C, int nq,
+    float* __restrict__ part) {
+  __shared__ float4 r1[256], r2[256];
+  const int g = blockIdx.y, q = blockIdx.x;
+  const int C4 = C / 4, lanes = blockDim.x / C4;
+  const int cg = threadIdx.x % C4, l = threadIdx.x / C4;
+  const int64_t p0 = (int64_t)q * kStatChunk, p1 = min(P, p0 + kStatChunk);
+  const int64_t base = (int64_t)g * P * C + 4 * cg;
+  const float4 mu = *reinterpret_cast<const float4*>(mean + g * C + 4 * cg);
+  const float4 rs = *reinterpret_cast<const float4*>(rstd + g * C + 4 * cg);
+  float4 s1 = make_float4(0.f, 0.f, 0.f, 0.f), s2 = s1;
+  if (l < lanes) {
+#pragma unroll 4
+    for (int64_t p = p0 + l; p < p1; p += lanes) {
+      const int64_t e = base + p * C;
+      const float4 d = *reinterpret_cast<const float4*>(dout + e);
+      const float4 o = Vec4<TA>::load(out + e);
+      const float4 v = *reinterpret_cast<const float4*>(y + e);
+      const float dz0 = o.x > 0.f ? d.x : 0.f, dz1 = o.y > 0.f ? d.y : 0.f;
+      const float dz2 = o.z > 0.f ? d.z : 0.f, dz3 = o.w > 0.f ? d.w : 0.f;
+      s1.x += dz0;
+      s1.y += dz1;
+      s1.z += dz2;
+      s1.w += dz3;
+      s2.x = fmaf(dz0, (v.x - mu.x) * rs.x, s2.x);
+      s2.y = fmaf(dz1, (v.y - mu.y) * rs.y, s2.y);
+      s2.z = fmaf(dz2, (v.z - mu.z) * rs.z, s2.z);
+      s2.w = fmaf(dz3, (v.w - mu.w) * rs.w, s2.w);
+    }
+    r1[l * C4 + cg] = s1;
+    r2[l * C4 + cg] = s2;
+  }
+  int span = 1;
+  while (span < lanes) span <<= 1;
+  for (int st = span >> 1; st > 0; st >>= 1) {
+    __syncthreads();
+    if (l < st && l + st < lanes) {
+      float4& a = r1[l * C4 + cg];
+      const float4 b = r1[(l + st) * C4 + cg];
+      a.x += b.x;
+      a.y += b.y;
+      a.z += b.z;
+      a.w += b.w;
+      float4& a2 = r2[l * C4 + cg];
+      const float4 b2 = r2[(l + st) * C4 + cg];
+      a2.x += b2.x;
+      a2.y += b2.y;
+      a2.z += b2.z;
+      a2.w += b2.w;
+    }
+  }
+  __syncthreads();
+  if (l == 0) {
+    const float4 t1 = r1[cg], t2 = r2[cg];
+    float* dst = part + (((int64_t)g * nq + q) * C + 4 * cg) * 2;
+    dst[0] = t1.x;
+    dst[1] = t2.x;
+    dst[2] = t1.y;
+    dst[3] = t2.y;
+    dst[4] = t1.z;
+    dst[5] = t2.z;
+    dst[6] = t1.w;
+    dst[7] = t2.w;
   }
 }
 
@@ -471,6 +659,45 @@ __global__ void bn_bwd_apply_kernel(const float* __restrict__ dout, const TA* __
   }
 }
 
+// The same with a fixed group of 4 channels per thread (C / 4 dividing the block size), the
+// per-channel factors loaded once, blockIdx.y the replica.
+template <typename TA>
+__global__ void __launch_bounds__(256) bn_bwd_apply_v4_kernel(
+    const float* __restrict__ dout, const TA* __restrict__ out, const float* __restrict__ y,
+    const float* __restrict__ mean, const float* __restrict__ rstd, const float* __restrict__ s12,
+    const float* __restrict__ W, int64_t g_off, int64_t d_gs, TA* __restrict__ dy, int P, int C) {
+  const int g = blockIdx.y, C4 = C / 4;
+  const int c0 = (threadIdx.x % C4) * 4, pl = threadIdx.x / C4, ppb = blockDim.x / C4;
+  const float invM = 1.0f / (float)P;
+  float mu[4], rs[4], gr[4], m1[4], m2[4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int gc = g * C + c0 + i;
+    mu[i] = mean[gc];
+    rs[i] = rstd[gc];
+    gr[i] = W[(int64_t)g * d_gs + g_off + c0 + i] * rs[i];
+    m1[i] = s12[2 * gc] * invM;
+    m2[i] = s12[2 * gc + 1] * invM;
+  }
+  const int64_t base = (int64_t)g * P * C + c0;
+  for (int p = blockIdx.x * ppb + pl; p < P; p += gridDim.x * ppb) {
+    const int64_t e = base + (int64_t)p * C;
+    const float4 d4 = *reinterpret_cast<const float4*>(dout + e);
+    const float4 o4 = Vec4<TA>::load(out + e);
+    const float4 y4 = *reinterpret_cast<const float4*>(y + e);
+    const float dd[4] = {d4.x, d4.y, d4.z, d4.w}, oo[4] = {o4.x, o4.y, o4.z, o4.w};
+    const float yy[4] = {y4.x, y4.y, y4.z, y4.w};
+    float v[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float dz = oo[i] > 0.f ? dd[i] : 0.f;
+      const float xh = (yy[i] - mu[i]) * rs[i];
+      v[i] = gr[i] * (dz - m1[i] - xh * m2[i]);
+    }
+    Vec4<TA>::store(dy + e, make_float4(v[0], v[1], v[2], v[3]));
+  }
+}
+
 // feat[g][b][f] = mean over the H W pixels of act[g][b][.][.][f].
 template <typename TA>
 __global__ void avgpool_kernel(const TA* __restrict__ act, float* __restrict__ feat, int GB, int HW,
@@ -496,28 +723,26 @@ __global__ void avgpool_bwd_kernel(const float* __restrict__ dfeat, float* __res
 }
 
 // im2col for the tensor-core convolutions: col[g][p][(kh 3 + kw) Cin + ci] =
-// in[g][b][oh s + kh - 1][ow s + kw - 1][ci] (zero outside the image), p = (b, oh, ow); bf16,
-// 8 channels (16 bytes) per thread, Cin a multiple of 8.
-__global__ void im2col_kernel(const uint16_t* __restrict__ in, uint16_t* __restrict__ col, int G,
-                              int B, int Hin, int Win, int Cin, int Hout, int Wout, int stride) {
-  const int c8n = Cin / 8;
-  const int64_t P = (int64_t)B * Hout * Wout;
-  const int64_t n = (int64_t)G * P * 9 * c8n;
-  const int64_t step = (int64_t)gridDim.x * blockDim.x;
-  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < n; e += step) {
-    const int c8 = (int)(e % c8n);
-    int64_t t = e / c8n;
-    const int tap = (int)(t % 9);
-    t /= 9;
-    const int64_t p = t % P;
-    const int g = (int)(t / P);
-    const int ow = (int)(p % Wout), oh = (int)((p / Wout) % Hout), b = (int)(p / ((int64_t)Wout * Hout));
-    const int ih = oh * stride + tap / 3 - 1, iw = ow * stride + tap % 3 - 1;
-    uint4 v = make_uint4(0u, 0u, 0u, 0u);
-    if (ih >= 0 && ih < Hin && iw >= 0 && iw < Win)
-      v = __ldg(reinterpret_cast<const uint4*>(in + ((((int64_t)g * B + b) * Hin + ih) * Win + iw) * Cin + c8 * 8));
-    *reinterpret_cast<uint4*>(col + ((int64_t)g * P + p) * 9 * Cin + tap * Cin + c8 * 8) = v;
-  }
+// in[g][b][oh s + kh - 1][ow s + kw - 1][ci] (zero outside the image), p = (b, oh, ow); bf16, Cin a
+// multiple of 8.  blockIdx.y is the replica; thread e of the replica takes pixel e / R and 16-byte
+// chunk e % R of its column row (R = 9 Cin / 8), so consecutive threads write consecutive chunks.
+__global__ void __launch_bounds__(256) im2col_v2_kernel(const uint16_t* __restrict__ in,
+                                                        uint16_t* __restrict__ col, int B, int Hin,
+                                                        int Win, int Cin, int Hout, int Wout,
+                                                        int stride) {
+  const int g = blockIdx.y, c8n = Cin / 8, R = 9 * c8n;
+  const int P = B * Hout * Wout;
+  const int e = blockIdx.x * blockDim.x + threadIdx.x;
+  if (e >= P * R) return;
+  const int p = e / R, r = e - p * R;
+  const int tap = r / c8n, c8 = r - tap * c8n;
+  const int ow = p % Wout, t2 = p / Wout, oh = t2 % Hout, b = t2 / Hout;
+  const int ih = oh * stride + tap / 3 - 1, iw = ow * stride + tap % 3 - 1;
+  uint4 v = make_uint4(0u, 0u, 0u, 0u);
+  if (ih >= 0 && ih < Hin && iw >= 0 && iw < Win)
+    v = __ldg(reinterpret_cast<const uint4*>(
+        in + ((((int64_t)g * B + b) * Hin + ih) * Win + iw) * Cin + c8 * 8));
+  *reinterpret_cast<uint4*>(col + ((int64_t)g * P + p) * 9 * Cin + (int64_t)r * 8) = v;
 }
 
 // im2col with any channel count: col[g][p][tap Cin + ci] for j = tap Cin + ci < 9 Cin, zero for
@@ -549,29 +774,26 @@ __global__ void im2col_any_kernel(const TA* __restrict__ in, uint16_t* __restric
 // Column matrix of a data gradient: for each pixel (ih, iw) of the convolution's input and each
 // flipped tap t' = (kh', kw'), the output-gradient row at ((ih + kh' - 1) / s, (iw + kw' - 1) / s)
 // when both are whole and inside the output, else zero.  With the flipped, transposed weights
-// this writes dx = sum over the taps reaching (ih, iw) of dy w (stride 1 or 2).
-__global__ void col_dgrad_kernel(const uint16_t* __restrict__ dy, uint16_t* __restrict__ col, int G,
-                                 int B, int Hin, int Win, int Cout, int Hout, int Wout, int stride) {
-  const int c8n = Cout / 8;
-  const int64_t P = (int64_t)B * Hin * Win;
-  const int64_t n = (int64_t)G * P * 9 * c8n;
-  const int64_t step = (int64_t)gridDim.x * blockDim.x;
-  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < n; e += step) {
-    const int c8 = (int)(e % c8n);
-    int64_t t = e / c8n;
-    const int tap = (int)(t % 9);
-    t /= 9;
-    const int64_t p = t % P;
-    const int g = (int)(t / P);
-    const int iw = (int)(p % Win), ih = (int)((p / Win) % Hin), b = (int)(p / ((int64_t)Win * Hin));
-    const int hn = ih + tap / 3 - 1, wn = iw + tap % 3 - 1;
-    uint4 v = make_uint4(0u, 0u, 0u, 0u);
-    if (hn >= 0 && wn >= 0 && hn % stride == 0 && wn % stride == 0 && hn / stride < Hout &&
-        wn / stride < Wout)
-      v = __ldg(reinterpret_cast<const uint4*>(
-          dy + ((((int64_t)g * B + b) * Hout + hn / stride) * Wout + wn / stride) * Cout + c8 * 8));
-    *reinterpret_cast<uint4*>(col + ((int64_t)g * P + p) * 9 * Cout + tap * Cout + c8 * 8) = v;
-  }
+// this writes dx = sum over the taps reaching (ih, iw) of dy w (stride 1 or 2).  blockIdx.y is
+// the replica; thread = (pixel, 16-byte chunk), 32-bit indexing.
+__global__ void __launch_bounds__(256) col_dgrad_v2_kernel(const uint16_t* __restrict__ dy,
+                                                           uint16_t* __restrict__ col, int B, int Hin,
+                                                           int Win, int Cout, int Hout, int Wout,
+                                                           int stride) {
+  const int g = blockIdx.y, c8n = Cout / 8, R = 9 * c8n;
+  const int P = B * Hin * Win;
+  const int e = blockIdx.x * blockDim.x + threadIdx.x;
+  if (e >= P * R) return;
+  const int p = e / R, r = e - p * R;
+  const int tap = r / c8n, c8 = r - tap * c8n;
+  const int iw = p % Win, t2 = p / Win, ih = t2 % Hin, b = t2 / Hin;
+  const int hn = ih + tap / 3 - 1, wn = iw + tap % 3 - 1;
+  uint4 v = make_uint4(0u, 0u, 0u, 0u);
+  if (hn >= 0 && wn >= 0 && hn % stride == 0 && wn % stride == 0 && hn / stride < Hout &&
+      wn / stride < Wout)
+    v = __ldg(reinterpret_cast<const uint4*>(
+        dy + ((((int64_t)g * B + b) * Hout + hn / stride) * Wout + wn / stride) * Cout + c8 * 8));
+  *reinterpret_cast<uint4*>(col + ((int64_t)g * P + p) * 9 * Cout + (int64_t)r * 8) = v;
 }
 
 // Weights with each [9 Cin] row padded to ldc columns (zeros), bf16: the stem's tensor-core
@@ -621,22 +843,28 @@ __global__ void flip_weights_kernel(const uint16_t* __restrict__ Wb, int64_t d_p
 }
 
 // The option-A shortcut's share of a block's input gradient: for input pixels on the stride grid
-// and the first Cin channels, dx += dout * (out > 0) at (ih / s, iw / s).
+// and the first Cin channels, dx += dout * (out > 0) at (ih / s, iw / s).  Thread = (output pixel,
+// 4 channels < Cin), blockIdx.y the replica; only the input pixels on the stride grid are touched.
 template <typename TA>
-__global__ void add_shortcut_grad_kernel(float* __restrict__ dx, const float* __restrict__ dout,
-                                         const TA* __restrict__ out, int G, int B, int Hin, int Win,
-                                         int Cin, int Hout, int Wout, int Cout, int stride) {
-  const int64_t n = (int64_t)G * B * Hin * Win * Cin;
-  const int64_t step = (int64_t)gridDim.x * blockDim.x;
-  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < n; e += step) {
-    const int ci = (int)(e % Cin);
-    const int64_t pix = e / Cin;
-    const int iw = (int)(pix % Win), ih = (int)((pix / Win) % Hin);
-    if (ih % stride || iw % stride) continue;
-    const int64_t gb = pix / ((int64_t)Win * Hin);
-    const int64_t o = ((gb * Hout + ih / stride) * Wout + iw / stride) * Cout + ci;
-    if (Elem<TA>::load(out + o) > 0.f) dx[e] += dout[o];
-  }
+__global__ void __launch_bounds__(256) add_shortcut_grad_v2_kernel(
+    float* __restrict__ dx, const float* __restrict__ dout, const TA* __restrict__ out, int B,
+    int Hin, int Win, int Cin, int Hout, int Wout, int Cout, int stride) {
+  const int g = blockIdx.y, C4 = Cin / 4;
+  const int Po = B * Hout * Wout;
+  const int e = blockIdx.x * blockDim.x + threadIdx.x;
+  if (e >= Po * C4) return;
+  const int po = e / C4, c0 = (e - po * C4) * 4;
+  const int ow = po % Wout, t2 = po / Wout, oh = t2 % Hout, b = t2 / Hout;
+  const int64_t o = ((int64_t)g * Po + po) * Cout + c0;
+  const int64_t i = ((((int64_t)g * B + b) * Hin + oh * stride) * Win + ow * stride) * Cin + c0;
+  const float4 d = *reinterpret_cast<const float4*>(dout + o);
+  const float4 a = Vec4<TA>::load(out + o);
+  float4 x = *reinterpret_cast<float4*>(dx + i);
+  x.x += a.x > 0.f ? d.x : 0.f;
+  x.y += a.y > 0.f ? d.y : 0.f;
+  x.z += a.z > 0.f ? d.z : 0.f;
+  x.w += a.w > 0.f ? d.w : 0.f;
+  *reinterpret_cast<float4*>(dx + i) = x;
 }
 
 }  // namespace
@@ -703,6 +931,20 @@ bool conv_on_tc(const ResNetPlan* p, const ConvL& c) { return p->tc && c.cout % 
 int col_ld(const ConvL& c) { return (int)rup(9 * c.cin, 8); }
 
 int grid_for_items(int64_t n) { return grid_cap(n, 256); }
+// Implicit-GEMM convolutions on the tensor cores: Ck = 16, 32 or 64 channels per tap, an output
+// that tiles into 128-pixel blocks of whole rows (see conv_tile_shape), stride 1 or 2.
+bool implicit_conv_ok(int ck, int stride, int hout, int wout) {
+  int rows = 0, images = 0;
+  return (ck == 16 || ck == 32 || ck == 64) && (stride == 1 || stride == 2) &&
+         conv_tile_shape(hout, wout, &rows, &images);
+}
+// The four-channel kernels need C a multiple of 4 with C / 4 dividing their 256 threads.
+bool vec4_ok(int C) { return C % 4 == 0 && 256 % (C / 4) == 0; }
+// Blocks of a per-replica kernel whose threads each take one pixel and group of 4 channels.
+unsigned px_blocks(int64_t P, int C) {
+  const int64_t ppb = 256 / (C / 4);
+  return (unsigned)std::max<int64_t>(1, std::min<int64_t>((P + ppb - 1) / ppb, (int64_t)kNumSMs * 8));
+}
 
 template <typename TA>
 lsgd_status conv_forward(ResNetPlan* p, int i, const void* in, const void* Wop, int w_g0,
@@ -715,9 +957,10 @@ lsgd_status conv_forward(ResNetPlan* p, int i, const void* in, const void* Wop, 
     const uint16_t* wop = reinterpret_cast<const uint16_t*>(Wop) + c.w_off;
     int64_t w_gs = p->d_pad;
     if (Kc == 9 * c.cin) {
-      RN_LAUNCH((im2col_kernel<<<grid_for_items((int64_t)G * P * 9 * (c.cin / 8)), 256, 0, s>>>(
-          reinterpret_cast<const uint16_t*>(in), p->col[i], G, p->B, c.hin, c.win, c.cin, c.hout,
-          c.wout, c.stride)));
+      RN_LAUNCH((im2col_v2_kernel<<<dim3((unsigned)((P * 9 * (c.cin / 8) + 255) / 256), (unsigned)G),
+                                      256, 0, s>>>(reinterpret_cast<const uint16_t*>(in), p->col[i],
+                                                   p->B, c.hin, c.win, c.cin, c.hout, c.wout,
+                                                   c.stride)));
     } else {
       RN_LAUNCH((im2col_any_kernel<uint16_t><<<grid_for_items((int64_t)G * P * Kc), 256, 0, s>>>(
           reinterpret_cast<const uint16_t*>(in), p->col[i], G, p->B, c.hin, c.win, c.cin, c.hout,
@@ -732,6 +975,31 @@ lsgd_status conv_forward(ResNetPlan* p, int i, const void* in, const void* Wop, 
     t.N = c.cout;
     t.Kd = Kc;
     t.G = G;
+    if (implicit_conv_ok(c.cin, c.stride, c.hout, c.wout) && Kc == 9 * c.cin) {
+      // implicit GEMM: the input tile of each tap straight from the NHWC activation by TMA
+      // (the column matrix above is only kept for the weight gradient)
+      t.conv = 1;
+      t.cv_ck = c.cin;
+      t.cv_stride = c.stride;
+      t.cv_hout = c.hout;
+      t.cv_wout = c.wout;
+      bool okc = make_tma_map_conv(&t.A.map, in, c.cin, c.win, c.hin, p->B, G, c.wout, c.hout,
+                                   c.stride);
+      okc &= make_tma_map(&t.B.map, wop, true, 9 * c.cin, c.cout, G, 9 * c.cin, w_gs, c.cin, 64,
+                          2 * c.cin);
+      if (!okc) {
+        p->err = "TMA map encoding failed (implicit convolution)";
+        return LSGD_ECUDA;
+      }
+      t.A.box_rows = kTcTileM;
+      t.B.box_rows = 64;
+      t.C = y;
+      t.c_rs = c.cout;
+      t.c_gs = P * c.cout;
+      t.epi = EPI_STORE;
+      RN_CALL(launch_gemm_tc(t, s));
+      return LSGD_OK;
+    }
     const int bn = tc_tile_n(Kc);
     bool ok = make_tma_map_bf16(&t.A.map, p->col[i], Kc, P, G, Kc, (uint64_t)P * Kc, 64, kTcTileM);
     ok &= make_tma_map_bf16(&t.B.map, wop, Kc, c.cout, G, Kc, w_gs, 64, bn);
@@ -763,7 +1031,10 @@ lsgd_status bn_stats(ResNetPlan* p, const ConvL& c, const float* y, float* mean,
   const int nq = (int)((P + kStatChunk - 1) / kStatChunk);
   const int lanes = std::max(1, 256 / c.cout);
   dim3 grid(nq, G);
-  RN_LAUNCH((bn_stats_partial_kernel<<<grid, lanes * c.cout, 0, s>>>(y, P, c.cout, nq, p->part)));
+  if (vec4_ok(c.cout))
+    RN_LAUNCH((bn_stats_partial_v4_kernel<<<grid, 256, 0, s>>>(y, P, c.cout, nq, p->part)));
+  else
+    RN_LAUNCH((bn_stats_partial_kernel<<<grid, lanes * c.cout, 0, s>>>(y, P, c.cout, nq, p->part)));
   RN_LAUNCH((bn_stats_finalize_kernel<<<(G * c.cout * 32 + 127) / 128, 128, 0, s>>>(
       p->part, P, c.cout, nq, G, mean, rstd)));
   return LSGD_OK;
@@ -784,11 +1055,19 @@ lsgd_status forward_impl(ResNetPlan* p, const float* W, const void* Wop, int w_g
     const bool second = i > 0 && i % 2 == 0;
     const TA* sc = second ? reinterpret_cast<const TA*>(p->act[i - 2]) : nullptr;
     const ConvL& ca = p->convs[second ? i - 1 : i];
-    const int64_t n = (int64_t)G * conv_pixels(p, c) * c.cout / 4;
-    RN_LAUNCH((bn_act_fwd_kernel<TA><<<grid_cap(n, 256), 256, 0, s>>>(
-        p->y[i], p->mean[i], p->rstd[i], W, c.g_off, c.b_off, p->d_pad, w_g0, w_gmul, sc, ca.hin,
-        ca.win, ca.cin, ca.stride, reinterpret_cast<TA*>(p->act[i]), G, p->B, c.hout, c.wout,
-        c.cout)));
+    if (vec4_ok(c.cout)) {
+      RN_LAUNCH((bn_act_fwd_v4_kernel<TA><<<dim3(px_blocks(conv_pixels(p, c), c.cout), (unsigned)G),
+                                             256, 0, s>>>(
+          p->y[i], p->mean[i], p->rstd[i], W, c.g_off, c.b_off, p->d_pad, w_g0, w_gmul, sc, ca.hin,
+          ca.win, ca.cin, ca.stride, reinterpret_cast<TA*>(p->act[i]), p->B, c.hout, c.wout,
+          c.cout)));
+    } else {
+      const int64_t n = (int64_t)G * conv_pixels(p, c) * c.cout / 4;
+      RN_LAUNCH((bn_act_fwd_kernel<TA><<<grid_cap(n, 256), 256, 0, s>>>(
+          p->y[i], p->mean[i], p->rstd[i], W, c.g_off, c.b_off, p->d_pad, w_g0, w_gmul, sc, ca.hin,
+          ca.win, ca.cin, ca.stride, reinterpret_cast<TA*>(p->act[i]), G, p->B, c.hout, c.wout,
+          c.cout)));
+    }
   }
   // global average pooling and the classifier (fp32)
   const ConvL& last = p->convs.back();
@@ -825,15 +1104,26 @@ lsgd_status bn_backward(ResNetPlan* p, const ConvL& c, int i, const float* dout,
   const int64_t P = conv_pixels(p, c);
   const int nq = (int)((P + kStatChunk - 1) / kStatChunk);
   const int lanes = std::max(1, 256 / c.cout);
-  RN_LAUNCH((bn_bwd_partial_kernel<TA><<<dim3(nq, K), lanes * c.cout, 0, s>>>(
-      dout, reinterpret_cast<const TA*>(out), p->y[i], p->mean[i], p->rstd[i], P, c.cout, nq,
-      p->part)));
+  if (vec4_ok(c.cout))
+    RN_LAUNCH((bn_bwd_partial_v4_kernel<TA><<<dim3(nq, K), 256, 0, s>>>(
+        dout, reinterpret_cast<const TA*>(out), p->y[i], p->mean[i], p->rstd[i], P, c.cout, nq,
+        p->part)));
+  else
+    RN_LAUNCH((bn_bwd_partial_kernel<TA><<<dim3(nq, K), lanes * c.cout, 0, s>>>(
+        dout, reinterpret_cast<const TA*>(out), p->y[i], p->mean[i], p->rstd[i], P, c.cout, nq,
+        p->part)));
   RN_LAUNCH((bn_bwd_finalize_kernel<<<(K * c.cout + 127) / 128, 128, 0, s>>>(
       p->part, c.cout, nq, K, p->s12, Gr, c.g_off, c.b_off, p->d_pad)));
-  const int64_t n = (int64_t)K * P * c.cout / 4;
-  RN_LAUNCH((bn_bwd_apply_kernel<TA><<<grid_cap(n, 256), 256, 0, s>>>(
-      dout, reinterpret_cast<const TA*>(out), p->y[i], p->mean[i], p->rstd[i], p->s12, W, c.g_off,
-      p->d_pad, reinterpret_cast<TA*>(p->dy), K, P, c.cout)));
+  if (vec4_ok(c.cout)) {
+    RN_LAUNCH((bn_bwd_apply_v4_kernel<TA><<<dim3(px_blocks(P, c.cout), (unsigned)K), 256, 0, s>>>(
+        dout, reinterpret_cast<const TA*>(out), p->y[i], p->mean[i], p->rstd[i], p->s12, W, c.g_off,
+        p->d_pad, reinterpret_cast<TA*>(p->dy), (int)P, c.cout)));
+  } else {
+    const int64_t n = (int64_t)K * P * c.cout / 4;
+    RN_LAUNCH((bn_bwd_apply_kernel<TA><<<grid_cap(n, 256), 256, 0, s>>>(
+        dout, reinterpret_cast<const TA*>(out), p->y[i], p->mean[i], p->rstd[i], p->s12, W, c.g_off,
+        p->d_pad, reinterpret_cast<TA*>(p->dy), K, P, c.cout)));
+  }
   return LSGD_OK;
 }
 
@@ -891,12 +1181,52 @@ lsgd_status conv_dgrad(ResNetPlan* p, int i, const void* Wop, float* dx, const f
   const ConvL& c = p->convs[i];
   const int K = p->K;
   const int64_t P = (int64_t)p->B * c.hin * c.win;
+  if (conv_on_tc(p, c) && c.stride == 1 && implicit_conv_ok(c.cout, 1, c.hin, c.win)) {
+    // stride 1: dx is the convolution of dy with the flipped, transposed weights -- an implicit
+    // GEMM over dy's taps, no column matrix
+    RN_LAUNCH((flip_weights_kernel<<<grid_for_items((int64_t)K * c.cin * 9 * c.cout), 256, 0, s>>>(
+        reinterpret_cast<const uint16_t*>(Wop), p->d_pad, c.w_off, p->wt, K, c.cin, c.cout)));
+    TcGemmArgs t{};
+    t.M = (int)P;
+    t.N = c.cin;
+    t.Kd = 9 * c.cout;
+    t.G = K;
+    t.conv = 1;
+    t.cv_ck = c.cout;
+    t.cv_stride = 1;
+    t.cv_hout = c.hin;
+    t.cv_wout = c.win;
+    bool ok = make_tma_map_conv(&t.A.map, p->dy, c.cout, c.wout, c.hout, p->B, K, c.win, c.hin, 1);
+    ok &= make_tma_map(&t.B.map, p->wt, true, 9 * c.cout, c.cin, K, 9 * c.cout,
+                       (uint64_t)c.cin * 9 * c.cout, c.cout, 64, 2 * c.cout);
+    if (!ok) {
+      p->err = "TMA map encoding failed (implicit data gradient)";
+      return LSGD_ECUDA;
+    }
+    t.A.box_rows = kTcTileM;
+    t.B.box_rows = 64;
+    t.C = dx;
+    t.c_rs = c.cin;
+    t.c_gs = P * c.cin;
+    t.epi = EPI_STORE;
+    RN_CALL(launch_gemm_tc(t, s));
+    if (dout) {
+      const int64_t n = (int64_t)p->B * c.hout * c.wout * (c.cin / 4);
+      RN_LAUNCH((add_shortcut_grad_v2_kernel<TA><<<dim3((unsigned)((n + 255) / 256), (unsigned)K), 256,
+                                                   0, s>>>(dx, dout,
+                                                           reinterpret_cast<const TA*>(out_act),
+                                                           p->B, c.hin, c.win, c.cin, c.hout,
+                                                           c.wout, c.cout, c.stride)));
+    }
+    return LSGD_OK;
+  }
   if (conv_on_tc(p, c) && c.cin % 8 == 0) {
     // dx = col(dy) [P][9 Cout] x wt^T with the flipped, transposed weights (stride 1 or 2)
     const int Kc = 9 * c.cout;
-    RN_LAUNCH((col_dgrad_kernel<<<grid_for_items((int64_t)K * P * 9 * (c.cout / 8)), 256, 0, s>>>(
-        reinterpret_cast<const uint16_t*>(p->dy), p->colT, K, p->B, c.hin, c.win, c.cout, c.hout,
-        c.wout, c.stride)));
+    RN_LAUNCH((col_dgrad_v2_kernel<<<dim3((unsigned)((P * 9 * (c.cout / 8) + 255) / 256), (unsigned)K),
+                                         256, 0, s>>>(reinterpret_cast<const uint16_t*>(p->dy),
+                                                      p->colT, p->B, c.hin, c.win, c.cout, c.hout,
+                                                      c.wout, c.stride)));
     RN_LAUNCH((flip_weights_kernel<<<grid_for_items((int64_t)K * c.cin * Kc), 256, 0, s>>>(
         reinterpret_cast<const uint16_t*>(Wop), p->d_pad, c.w_off, p->wt, K, c.cin, c.cout)));
     TcGemmArgs t{};
@@ -919,10 +1249,12 @@ lsgd_status conv_dgrad(ResNetPlan* p, int i, const void* Wop, float* dx, const f
     t.epi = EPI_STORE;
     RN_CALL(launch_gemm_tc(t, s));
     if (dout) {
-      const int64_t n = (int64_t)K * P * c.cin;
-      RN_LAUNCH((add_shortcut_grad_kernel<TA><<<grid_cap(n, 256), 256, 0, s>>>(
-          dx, dout, reinterpret_cast<const TA*>(out_act), K, p->B, c.hin, c.win, c.cin, c.hout,
-          c.wout, c.cout, c.stride)));
+      const int64_t n = (int64_t)p->B * c.hout * c.wout * (c.cin / 4);
+      RN_LAUNCH((add_shortcut_grad_v2_kernel<TA><<<dim3((unsigned)((n + 255) / 256), (unsigned)K), 256,
+                                                   0, s>>>(dx, dout,
+                                                           reinterpret_cast<const TA*>(out_act),
+                                                           p->B, c.hin, c.win, c.cin, c.hout,
+                                                           c.wout, c.cout, c.stride)));
     }
     return LSGD_OK;
   }
@@ -1034,7 +1366,10 @@ cudaError_t launch_batchnorm_stats(const float* y, int64_t P, int C, int G, floa
   const int64_t nq = (P + kStatChunk - 1) / kStatChunk;
   if (nq > 65535) return cudaErrorInvalidValue;
   const int lanes = std::max(1, 256 / C);
-  bn_stats_partial_kernel<<<dim3((unsigned)nq, (unsigned)G), lanes * C, 0, s>>>(y, P, C, (int)nq, part);
+  if (vec4_ok(C))
+    bn_stats_partial_v4_kernel<<<dim3((unsigned)nq, (unsigned)G), 256, 0, s>>>(y, P, C, (int)nq, part);
+  else
+    bn_stats_partial_kernel<<<dim3((unsigned)nq, (unsigned)G), lanes * C, 0, s>>>(y, P, C, (int)nq, part);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   bn_stats_finalize_kernel<<<(G * C * 32 + 127) / 128, 128, 0, s>>>(part, P, C, (int)nq, G, mean, rstd);

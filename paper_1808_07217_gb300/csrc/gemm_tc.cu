@@ -206,7 +206,7 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
   const int cv_b0 = args.conv ? m0 / (args.cv_hout * args.cv_wout) : 0;
   const int cv_oy0 = args.conv ? (m0 / args.cv_wout) % args.cv_hout : 0;
   const int split = blockIdx.z % splits;
-  const int nk_all = args.conv ? 9 : (args.Kd + BK - 1) / BK;
+  const int nk_all = args.conv ? (9 + 64 / args.cv_ck - 1) / (64 / args.cv_ck) : (args.Kd + BK - 1) / BK;
   const int per_split = (nk_all + splits - 1) / splits;
   const int kb_first = split * per_split;
   const int nk = min(nk_all - kb_first, per_split);  // >= 1 (the host makes every split nonempty)
@@ -248,13 +248,17 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
         break;
       }
       if (args.conv) {
-        // tap t = kb: the input shifted by (kh - 1, kw - 1) (zero outside the image, stride by
-        // the map's element strides) and the weights' tap-t slice [N][Ck]
-        const int t = kb_first + kb, kh = t / 3, kw = t % 3;
-        mbar_expect_tx(&sm.full[s], (uint32_t)(BM + BN) * args.cv_ck * 2);
-        tma_load_5d(sm.a[s], &args.A.map, &sm.full[s], 0, kw - 1,
-                    cv_oy0 * args.cv_stride + kh - 1, cv_b0, g);
-        tma_load_3d(sm.b[s], &args.B.map, &sm.full[s], t * args.cv_ck, n0, g);
+        // 64 / Ck taps per stage; tap t: the input shifted by (kh - 1, kw - 1) (zero outside the
+        // image, stride by the map's element strides) and the weights' tap-t slice [N][Ck]
+        const int ck = args.cv_ck, tps = 64 / ck;
+        const int t0 = (kb_first + kb) * tps, t1 = min(9, t0 + tps);
+        mbar_expect_tx(&sm.full[s], (uint32_t)(t1 - t0) * (BM + BN) * ck * 2);
+        for (int t = t0; t < t1; ++t) {
+          const int kh = t / 3, kw = t % 3, j = t - t0;
+          tma_load_5d(sm.a[s] + j * BM * ck * 2, &args.A.map, &sm.full[s], 0, kw - 1,
+                      cv_oy0 * args.cv_stride + kh - 1, cv_b0, g);
+          tma_load_3d(sm.b[s] + j * BN * ck * 2, &args.B.map, &sm.full[s], t * ck, n0, g);
+        }
         issued = kb + 1;
         continue;
       }
@@ -295,11 +299,15 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
       asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
       const uint32_t a_base = smem_u32(sm.a[s]), b_base = smem_u32(sm.b[s]);
       if (args.conv) {
-        // rows of Ck bf16 = swz bytes; K = 16 per MMA, 32 bytes further along the row
-        const uint32_t swz = (uint32_t)args.cv_ck * 2;
-        for (int kk = 0; kk < args.cv_ck / 16; ++kk)
-          mma_bf16(tmem, smem_desc_kmajor(a_base + kk * 32, swz),
-                   smem_desc_kmajor(b_base + kk * 32, swz), idesc, (kb > 0 || kk > 0) ? 1u : 0u);
+        // each tap's sub-tiles: rows of Ck bf16 = swz bytes; K = 16 per MMA, 32 bytes further
+        const int ck = args.cv_ck, tps = 64 / ck;
+        const int nt = min(9, (kb_first + kb + 1) * tps) - (kb_first + kb) * tps;
+        const uint32_t swz = (uint32_t)ck * 2;
+        for (int j = 0; j < nt; ++j)
+          for (int kk = 0; kk < ck / 16; ++kk)
+            mma_bf16(tmem, smem_desc_kmajor(a_base + j * BM * ck * 2 + kk * 32, swz),
+                     smem_desc_kmajor(b_base + j * BN * ck * 2 + kk * 32, swz), idesc,
+                     (kb > 0 || j > 0 || kk > 0) ? 1u : 0u);
         mma_commit(&sm.empty[s]);
         continue;
       }
@@ -780,6 +788,172 @@ __global__ void __launch_bounds__(wu::THREADS, 1) wgrad_update_kernel(
   }
 }
 
+// =============================================================================================
+// Implicit-GEMM 3x3 convolution, persistent: out[g][p][n] = sum over taps t and k < ck of
+// in[g][shift_t(p)][k] w[g][n][t][k] (zero padding 1, stride 1 or 2), fp32 out.
+//
+// A CTA owns one replica and every cpr-th 128-pixel tile of it.  The replica's weights (all nine
+// taps, N rows of ck channels) are loaded once; the input tile of each tap streams through a
+// ring of shared-memory stages by TMA (a rank-5 box of the NHWC input, out-of-bounds fill = the
+// zero padding, element strides = the convolution stride); two TMEM accumulators let a tile's
+// MMAs overlap the previous tile's epilogue.
+//   warp 0      TMA producer (weights once, then one stage per tap)
+//   warp 1      MMA issuer: per tap ck / 16 tcgen05.mma (M = 128, N = NP, K = 16)
+//   warp 2      TMEM allocation
+//   warps 4-7   epilogue: tcgen05.ld of the tile row's NP columns, fp32 stores
+namespace cv {
+constexpr int THREADS = 256;
+constexpr int RING_BYTES = 96 * 1024;
+constexpr int MAX_STAGES = 24;  // 4 KB stages (ck = 16)
+constexpr int EPI0 = 128;
+}  // namespace cv
+
+__global__ void __launch_bounds__(cv::THREADS, 1) conv_tc_kernel(const __grid_constant__ ConvArgs a) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~uintptr_t(1023));
+  const int ck = a.ck, np = a.np;
+  // a stage holds the three taps of one kernel row (kh): three TMA boxes, one handshake
+  const uint32_t tap_bytes = (uint32_t)BM * ck * 2;
+  const uint32_t stage_bytes = 3 * tap_bytes;
+  const int nst = min(cv::MAX_STAGES, cv::RING_BYTES / (int)stage_bytes);
+  uint8_t* ring = base;
+  uint8_t* wsm = base + cv::RING_BYTES;
+  const uint32_t wtap = (uint32_t)np * ck * 2;  // bytes of one tap's weights
+  uint64_t* bars = reinterpret_cast<uint64_t*>(wsm + 9 * wtap);
+  uint64_t* full = bars;
+  uint64_t* empty = bars + cv::MAX_STAGES;
+  uint64_t* acc_full = bars + 2 * cv::MAX_STAGES;
+  uint64_t* acc_empty = acc_full + 2;
+  uint64_t* w_full = acc_empty + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(w_full + 1);
+  int* epi_ok = reinterpret_cast<int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int g = blockIdx.y, cpr = gridDim.x;
+  const int tiles = a.P / BM;  // per replica
+  const int per_img = a.hout * a.wout;
+  const uint32_t tmem_cols = (uint32_t)(2 * np < 32 ? 32 : 2 * np);
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < nst; ++i) {
+      mbar_init(&full[i], 1);
+      mbar_init(&empty[i], 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&acc_full[i], 1);
+      mbar_init(&acc_empty[i], 1);
+    }
+    mbar_init(w_full, 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  }
+  if (warp == 2) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     smem_u32(tmem_slot)),
+                 "r"(tmem_cols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+  __syncthreads();
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+  const uint32_t tmem = *tmem_slot;
+  pdl_begin();  // everything above touched only shared memory and TMEM
+
+  if (warp == 0 && lane == 0) {
+    // ---------------- producer ----------------
+    mbar_expect_tx(w_full, 9 * wtap);
+    for (int t = 0; t < 9; ++t) tma_load_3d(wsm + t * wtap, &a.w_map, w_full, t * ck, 0, g);
+    int q = 0;
+    bool ok = true;
+    for (int tile = blockIdx.x; tile < tiles && ok; tile += cpr) {
+      const int p0 = tile * BM, b0 = p0 / per_img, oy0 = (p0 / a.wout) % a.hout;
+      for (int kh = 0; kh < 3; ++kh, ++q) {
+        const int sl = q % nst;
+        if (!mbar_wait(&empty[sl], ((q / nst) & 1) ^ 1)) {
+          ok = false;
+          break;
+        }
+        mbar_expect_tx(&full[sl], stage_bytes);
+        for (int kw = 0; kw < 3; ++kw)
+          tma_load_5d(ring + sl * stage_bytes + kw * tap_bytes, &a.in_map, &full[sl], 0, kw - 1,
+                      oy0 * a.stride + kh - 1, b0, g);
+      }
+    }
+    // copies in flight land before the CTA can exit
+    mbar_wait(w_full, 0);
+    for (int j = (q > nst ? q - nst : 0); j < q; ++j) mbar_wait(&full[j % nst], (j / nst) & 1);
+  } else if (warp == 1 && lane == 0) {
+    // ---------------- MMA issuer ----------------
+    const uint32_t idesc = make_idesc(BM, np, false, false);
+    const uint32_t swz = (uint32_t)ck * 2;
+    bool ok = mbar_wait(w_full, 0);
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    int q = 0, i = 0;
+    for (int tile = blockIdx.x; tile < tiles && ok; tile += cpr, ++i) {
+      const int ab = i & 1;
+      if (!mbar_wait(&acc_empty[ab], ((i >> 1) & 1) ^ 1)) break;
+      asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+      const uint32_t acc = tmem + (uint32_t)(ab * np);
+      for (int kh = 0; kh < 3; ++kh, ++q) {
+        const int sl = q % nst;
+        if (!mbar_wait(&full[sl], (q / nst) & 1)) {
+          ok = false;
+          break;
+        }
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        for (int kw = 0; kw < 3; ++kw) {
+          const int t = kh * 3 + kw;
+          const uint32_t a_base = smem_u32(ring + sl * stage_bytes + kw * tap_bytes);
+          const uint32_t b_base = smem_u32(wsm + t * wtap);
+          for (int kk = 0; kk < ck / 16; ++kk)
+            mma_bf16(acc, smem_desc_kmajor(a_base + kk * 32, swz),
+                     smem_desc_kmajor(b_base + kk * 32, swz), idesc, (t > 0 || kk > 0) ? 1u : 0u);
+        }
+        mma_commit(&empty[sl]);
+      }
+      if (ok) mma_commit(&acc_full[ab]);
+    }
+  } else if (warp >= 4) {
+    // ---------------- epilogue ----------------
+    const bool leader = threadIdx.x == cv::EPI0;
+    const int quarter = warp & 3, r = quarter * 32 + lane;
+    int fi = 0;
+    auto epi_wait = [&](uint64_t* bar, uint32_t parity) -> bool {
+      if (leader) epi_ok[fi] = mbar_wait(bar, parity) ? 1 : 0;
+      asm volatile("bar.sync 1, 128;" ::: "memory");
+      const bool okw = epi_ok[fi] != 0;
+      fi ^= 1;
+      return okw;
+    };
+    int i = 0;
+    for (int tile = blockIdx.x; tile < tiles; tile += cpr, ++i) {
+      const int ab = i & 1;
+      if (!epi_wait(&acc_full[ab], (i >> 1) & 1)) break;
+      asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+      float* orow = a.out + (int64_t)g * a.out_gs + ((int64_t)tile * BM + r) * a.N;
+      for (int c0 = 0; c0 < a.N; c0 += 16) {
+        float v[16];
+        tmem_ld16(tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(ab * np + c0), v);
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+          *reinterpret_cast<float4*>(orow + c0 + 4 * j) =
+              make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
+      }
+      asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+      asm volatile("bar.sync 1, 128;" ::: "memory");
+      if (leader) mbar_arrive(&acc_empty[ab]);
+    }
+  }
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+  __syncthreads();
+  if (warp == 2) {
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(tmem_cols)
+                 : "memory");
+  }
+}
+
 PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 std::once_flag g_encode_once;
 
@@ -916,6 +1090,32 @@ bool make_tma_map(CUtensorMap* map, const void* base, bool bf16, uint64_t dim0, 
                         CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
+}
+
+cudaError_t launch_conv_tc(const ConvArgs& a, cudaStream_t stream) {
+  if (a.P <= 0 || a.G <= 0) return cudaSuccess;
+  int rows = 0, images = 0;
+  if ((a.ck != 16 && a.ck != 32 && a.ck != 64) || (a.stride != 1 && a.stride != 2) ||
+      (a.N != 16 && a.N != 32 && a.N != 64) || a.np != a.N || !a.out || a.G > 65535 ||
+      !conv_tile_shape(a.hout, a.wout, &rows, &images) || a.P % (a.hout * a.wout) || a.P % BM)
+    return cudaErrorInvalidValue;
+  int dev = 0, sms = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  if (e != cudaSuccess) return e;
+  const size_t smem = 1024 + cv::RING_BYTES + 9 * (size_t)a.np * a.ck * 2 +
+                      (2 * cv::MAX_STAGES + 5) * 8 + 16;
+  static int attr_dev = -1;
+  if (attr_dev != dev) {
+    e = cudaFuncSetAttribute(conv_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             1024 + cv::RING_BYTES + 9 * 64 * 64 * 2 + (2 * cv::MAX_STAGES + 5) * 8 + 16);
+    if (e != cudaSuccess) return e;
+    attr_dev = dev;
+  }
+  // CTAs per replica: about one per SM over all replicas, at most one per tile
+  const int tiles = a.P / BM;
+  const int cpr = std::max(1, std::min(tiles, (sms + a.G - 1) / a.G));
+  return launch_pdl(conv_tc_kernel, dim3(cpr, a.G), dim3(cv::THREADS), smem, stream, a);
 }
 
 cudaError_t launch_wgrad_update(const WgradUpdateArgs& a, cudaStream_t stream) {

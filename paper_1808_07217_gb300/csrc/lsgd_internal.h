@@ -137,6 +137,18 @@ struct GemmArgs {
   int conv;
   int cv_ck, cv_stride, cv_hout, cv_wout;
 };
+// Persistent implicit-GEMM 3x3 convolution (zero padding 1): out[g][p][n] (fp32, replica stride
+// out_gs) = sum over taps t and k < ck of in[g][shift_t(p)][k] w[g][n][t][k].  in_map: the rank-5
+// map of make_tma_map_conv; w_map: a rank-3 map over the [N][9][ck] weights {9 ck, N, G} with box
+// {ck, np} and a ck * 2-byte swizzle.  ck, N in {16, 32, 64}, np = N; P = output pixels per
+// replica, a multiple of 128 and of hout * wout.
+struct ConvArgs {
+  CUtensorMap in_map, w_map;
+  int ck, stride, hout, wout, N, np, G, P;
+  float* out;
+  int64_t out_gs;
+};
+cudaError_t launch_conv_tc(const ConvArgs& a, cudaStream_t stream);
 // The tile geometry of an implicit convolution with an Hout x Wout output: whole output rows,
 // 128 pixels per tile.  False when the shape does not tile that way.
 bool conv_tile_shape(int hout, int wout, int* rows, int* images);

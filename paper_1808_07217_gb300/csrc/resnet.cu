@@ -27,7 +27,8 @@ namespace lsgd {
 namespace {
 
 constexpr float kBnEps = 1e-5f;
-constexpr int kStatChunk = 1024;   // pixels per BatchNorm reduction chunk
+constexpr int kStatChunk = 1024;   // pixels per BatchNorm reduction chunk (lsgd_batchnorm_stats)
+constexpr int kRnChunk = 256;      // the same inside the ResNet step (more CTAs on small stages)
 constexpr int kWgradChunk = 2048;  // pixels per weight-gradient chunk
 constexpr int kWgradTile = 16;     // pixels staged per weight-gradient iteration
 constexpr int kMaxJ16 = 36;        // (9 Cin) / 16 accumulators per thread, Cin <= 64
@@ -229,14 +230,14 @@ __global__ void sum_partials_kernel(const float* __restrict__ part, int nq, int6
 // BatchNorm statistics, pass 1: per chunk of pixels, the chunk mean and the sum of squared
 // deviations from it (two passes over the chunk), part[g][q][c] = (mean, M2).
 __global__ void __launch_bounds__(256) bn_stats_partial_kernel(const float* __restrict__ y,
-                                                               int64_t P, int C, int nq,
+                                                               int64_t P, int C, int nq, int chunk,
                                                                float* __restrict__ part) {
   __shared__ float red[256];
   __shared__ float mean_s[256];
   const int g = blockIdx.y, q = blockIdx.x;
   const int lanes = blockDim.x / C;
   const int c = threadIdx.x % C, l = threadIdx.x / C;
-  const int64_t p0 = (int64_t)q * kStatChunk, p1 = min(P, p0 + kStatChunk);
+  const int64_t p0 = (int64_t)q * chunk, p1 = min(P, p0 + chunk);
   const float* yg = y + (int64_t)g * P * C;
   float s = 0.f;
   if (l < lanes)
@@ -289,12 +290,13 @@ __device__ __forceinline__ void tree_sum4(float4* red, int lane, int lanes, int 
 
 __global__ void __launch_bounds__(256) bn_stats_partial_v4_kernel(const float* __restrict__ y,
                                                                   int64_t P, int C, int nq,
+                                                                  int chunk,
                                                                   float* __restrict__ part) {
   __shared__ float4 red[256];
   const int g = blockIdx.y, q = blockIdx.x;
   const int C4 = C / 4, lanes = blockDim.x / C4;
   const int cg = threadIdx.x % C4, l = threadIdx.x / C4;
-  const int64_t p0 = (int64_t)q * kStatChunk, p1 = min(P, p0 + kStatChunk);
+  const int64_t p0 = (int64_t)q * chunk, p1 = min(P, p0 + chunk);
   const float4* yg = reinterpret_cast<const float4*>(y + (int64_t)g * P * C) + cg;
   float4 s = make_float4(0.f, 0.f, 0.f, 0.f);
   if (l < lanes) {
@@ -355,13 +357,14 @@ __device__ __forceinline__ void chan_merge(float& n, float& mu, float& M2, float
 }
 
 __global__ void bn_stats_finalize_kernel(const float* __restrict__ part, int64_t P, int C, int nq,
-                                         int G, float* __restrict__ mean, float* __restrict__ rstd) {
+                                         int chunk, int G, float* __restrict__ mean,
+                                         float* __restrict__ rstd) {
   const int wid = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
   if (wid >= G * C) return;
   const int g = wid / C, c = wid % C;
   float n = 0.f, mu = 0.f, M2 = 0.f;
   for (int q = lane; q < nq; q += 32) {
-    const float nb = (float)min((int64_t)kStatChunk, P - (int64_t)q * kStatChunk);
+    const float nb = (float)min((int64_t)chunk, P - (int64_t)q * chunk);
     const float* pq = part + (((int64_t)g * nq + q) * C + c) * 2;
     chan_merge(n, mu, M2, nb, pq[0], pq[1]);
   }
@@ -504,12 +507,12 @@ template <typename TA>
 __global__ void __launch_bounds__(256) bn_bwd_partial_kernel(
     const float* __restrict__ dout, const TA* __restrict__ out, const float* __restrict__ y,
     const float* __restrict__ mean, const float* __restrict__ rstd, int64_t P, int C, int nq,
-    float* __restrict__ part) {
+    int chunk, float* __restrict__ part) {
   __shared__ float r1[256], r2[256];
   const int g = blockIdx.y, q = blockIdx.x;
   const int lanes = blockDim.x / C;
   const int c = threadIdx.x % C, l = threadIdx.x / C;
-  const int64_t p0 = (int64_t)q * kStatChunk, p1 = min(P, p0 + kStatChunk);
+  const int64_t p0 = (int64_t)q * chunk, p1 = min(P, p0 + chunk);
   const int64_t base = (int64_t)g * P * C;
   const float mu = mean[g * C + c], rs = rstd[g * C + c];
   float s1 = 0.f, s2 = 0.f;
@@ -542,12 +545,12 @@ template <typename TA>
 __global__ void __launch_bounds__(256) bn_bwd_partial_v4_kernel(
     const float* __restrict__ dout, const TA* __restrict__ out, const float* __restrict__ y,
     const float* __restrict__ mean, const float* __restrict__ rstd, int64_t P, int C, int nq,
-    float* __restrict__ part) {
+    int chunk, float* __restrict__ part) {
   __shared__ float4 r1[256], r2[256];
   const int g = blockIdx.y, q = blockIdx.x;
   const int C4 = C / 4, lanes = blockDim.x / C4;
   const int cg = threadIdx.x % C4, l = threadIdx.x / C4;
-  const int64_t p0 = (int64_t)q * kStatChunk, p1 = min(P, p0 + kStatChunk);
+  const int64_t p0 = (int64_t)q * chunk, p1 = min(P, p0 + chunk);
   const int64_t base = (int64_t)g * P * C + 4 * cg;
   const float4 mu = *reinterpret_cast<const float4*>(mean + g * C + 4 * cg);
   const float4 rs = *reinterpret_cast<const float4*>(rstd + g * C + 4 * cg);
@@ -607,23 +610,31 @@ __global__ void __launch_bounds__(256) bn_bwd_partial_v4_kernel(
   }
 }
 
-// Pass 2: s[g][c] = chunk sums in order; dgamma = sum dz xhat, dbeta = sum dz into G.
+// Pass 2: s[g][c] = the chunk sums (one warp per (replica, channel): lane l adds chunks l, l + 32,
+// ... in order, then a fixed butterfly); dgamma = sum dz xhat, dbeta = sum dz into G.
 __global__ void bn_bwd_finalize_kernel(const float* __restrict__ part, int C, int nq, int G,
                                        float* __restrict__ s12, float* __restrict__ Gr,
                                        int64_t g_off, int64_t b_off, int64_t d_gs) {
-  const int t = blockIdx.x * blockDim.x + threadIdx.x;
-  if (t >= G * C) return;
-  const int g = t / C, c = t % C;
+  const int wid = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
+  if (wid >= G * C) return;
+  const int g = wid / C, c = wid % C;
   float a = 0.f, b = 0.f;
-  for (int q = 0; q < nq; ++q) {
+  for (int q = lane; q < nq; q += 32) {
     const float* pq = part + (((int64_t)g * nq + q) * C + c) * 2;
     a += pq[0];
     b += pq[1];
   }
-  s12[(int64_t)t * 2] = a;
-  s12[(int64_t)t * 2 + 1] = b;
-  Gr[(int64_t)g * d_gs + g_off + c] = b;
-  Gr[(int64_t)g * d_gs + b_off + c] = a;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    a += __shfl_xor_sync(0xffffffffu, a, o);
+    b += __shfl_xor_sync(0xffffffffu, b, o);
+  }
+  if (lane == 0) {
+    s12[(int64_t)wid * 2] = a;
+    s12[(int64_t)wid * 2 + 1] = b;
+    Gr[(int64_t)g * d_gs + g_off + c] = b;
+    Gr[(int64_t)g * d_gs + b_off + c] = a;
+  }
 }
 
 // dy = gamma rstd (dz - mean(dz) - xhat mean(dz xhat)), the convolution's output gradient; one
@@ -743,6 +754,29 @@ __global__ void __launch_bounds__(256) im2col_v2_kernel(const uint16_t* __restri
     v = __ldg(reinterpret_cast<const uint4*>(
         in + ((((int64_t)g * B + b) * Hin + ih) * Win + iw) * Cin + c8 * 8));
   *reinterpret_cast<uint4*>(col + ((int64_t)g * P + p) * 9 * Cin + (int64_t)r * 8) = v;
+}
+
+// The same with the channel count a template constant: a CTA per output row (b, oh) of replica
+// blockIdx.y, its threads over the row's Wout x 9 Cin / 8 chunks (divisions by constants only).
+template <int C8N>
+__global__ void __launch_bounds__(256) im2col_row_kernel(const uint16_t* __restrict__ in,
+                                                         uint16_t* __restrict__ col, int B, int Hin,
+                                                         int Win, int Hout, int Wout, int stride) {
+  constexpr int Cin = 8 * C8N, R = 9 * C8N;
+  const int g = blockIdx.y, row = blockIdx.x;
+  const int oh = row % Hout, b = row / Hout;
+  const int64_t P = (int64_t)B * Hout * Wout;
+  const uint16_t* ing = in + ((int64_t)g * B + b) * Hin * Win * Cin;
+  uint16_t* out = col + ((int64_t)g * P + (int64_t)row * Wout) * 9 * Cin;
+  for (int e = threadIdx.x; e < Wout * R; e += blockDim.x) {
+    const int ow = e / R, r = e - ow * R;
+    const int tap = r / C8N, c8 = r - tap * C8N;
+    const int ih = oh * stride + tap / 3 - 1, iw = ow * stride + tap % 3 - 1;
+    uint4 v = make_uint4(0u, 0u, 0u, 0u);
+    if (ih >= 0 && ih < Hin && iw >= 0 && iw < Win)
+      v = __ldg(reinterpret_cast<const uint4*>(ing + ((int64_t)ih * Win + iw) * Cin + c8 * 8));
+    *reinterpret_cast<uint4*>(out + (int64_t)e * 8) = v;
+  }
 }
 
 // im2col with any channel count: col[g][p][tap Cin + ci] for j = tap Cin + ci < 9 Cin, zero for
@@ -938,6 +972,8 @@ bool implicit_conv_ok(int ck, int stride, int hout, int wout) {
   return (ck == 16 || ck == 32 || ck == 64) && (stride == 1 || stride == 2) &&
          conv_tile_shape(hout, wout, &rows, &images);
 }
+// The persistent convolution kernel: N = 16, 32 or 64 outputs, whole 128-pixel tiles.
+bool persistent_conv_ok(int n, int64_t P) { return (n == 16 || n == 32 || n == 64) && P % 128 == 0; }
 // The four-channel kernels need C a multiple of 4 with C / 4 dividing their 256 threads.
 bool vec4_ok(int C) { return C % 4 == 0 && 256 % (C / 4) == 0; }
 // Blocks of a per-replica kernel whose threads each take one pixel and group of 4 channels.
@@ -957,10 +993,21 @@ lsgd_status conv_forward(ResNetPlan* p, int i, const void* in, const void* Wop, 
     const uint16_t* wop = reinterpret_cast<const uint16_t*>(Wop) + c.w_off;
     int64_t w_gs = p->d_pad;
     if (Kc == 9 * c.cin) {
-      RN_LAUNCH((im2col_v2_kernel<<<dim3((unsigned)((P * 9 * (c.cin / 8) + 255) / 256), (unsigned)G),
-                                      256, 0, s>>>(reinterpret_cast<const uint16_t*>(in), p->col[i],
-                                                   p->B, c.hin, c.win, c.cin, c.hout, c.wout,
-                                                   c.stride)));
+      const uint16_t* in16 = reinterpret_cast<const uint16_t*>(in);
+      const dim3 rows_grid((unsigned)(p->B * c.hout), (unsigned)G);
+      if (c.cin == 16)
+        RN_LAUNCH((im2col_row_kernel<2><<<rows_grid, 256, 0, s>>>(in16, p->col[i], p->B, c.hin, c.win,
+                                                                  c.hout, c.wout, c.stride)));
+      else if (c.cin == 32)
+        RN_LAUNCH((im2col_row_kernel<4><<<rows_grid, 256, 0, s>>>(in16, p->col[i], p->B, c.hin, c.win,
+                                                                  c.hout, c.wout, c.stride)));
+      else if (c.cin == 64)
+        RN_LAUNCH((im2col_row_kernel<8><<<rows_grid, 256, 0, s>>>(in16, p->col[i], p->B, c.hin, c.win,
+                                                                  c.hout, c.wout, c.stride)));
+      else
+        RN_LAUNCH((im2col_v2_kernel<<<dim3((unsigned)((P * 9 * (c.cin / 8) + 255) / 256), (unsigned)G),
+                                        256, 0, s>>>(in16, p->col[i], p->B, c.hin, c.win, c.cin,
+                                                     c.hout, c.wout, c.stride)));
     } else {
       RN_LAUNCH((im2col_any_kernel<uint16_t><<<grid_for_items((int64_t)G * P * Kc), 256, 0, s>>>(
           reinterpret_cast<const uint16_t*>(in), p->col[i], G, p->B, c.hin, c.win, c.cin, c.hout,
@@ -975,6 +1022,31 @@ lsgd_status conv_forward(ResNetPlan* p, int i, const void* in, const void* Wop, 
     t.N = c.cout;
     t.Kd = Kc;
     t.G = G;
+    if (implicit_conv_ok(c.cin, c.stride, c.hout, c.wout) && Kc == 9 * c.cin &&
+        persistent_conv_ok(c.cout, P)) {
+      // persistent implicit GEMM: the input tile of each tap straight from the NHWC activation
+      // by TMA (the column matrix above is only kept for the weight gradient)
+      ConvArgs ca{};
+      bool okc = make_tma_map_conv(&ca.in_map, in, c.cin, c.win, c.hin, p->B, G, c.wout, c.hout,
+                                   c.stride);
+      okc &= make_tma_map(&ca.w_map, wop, true, 9 * c.cin, c.cout, G, 9 * c.cin, w_gs, c.cin,
+                          c.cout, 2 * c.cin);
+      if (!okc) {
+        p->err = "TMA map encoding failed (implicit convolution)";
+        return LSGD_ECUDA;
+      }
+      ca.ck = c.cin;
+      ca.stride = c.stride;
+      ca.hout = c.hout;
+      ca.wout = c.wout;
+      ca.N = ca.np = c.cout;
+      ca.G = G;
+      ca.P = (int)P;
+      ca.out = y;
+      ca.out_gs = P * c.cout;
+      RN_CALL(launch_conv_tc(ca, s));
+      return LSGD_OK;
+    }
     if (implicit_conv_ok(c.cin, c.stride, c.hout, c.wout) && Kc == 9 * c.cin) {
       // implicit GEMM: the input tile of each tap straight from the NHWC activation by TMA
       // (the column matrix above is only kept for the weight gradient)
@@ -1028,15 +1100,16 @@ lsgd_status conv_forward(ResNetPlan* p, int i, const void* in, const void* Wop, 
 lsgd_status bn_stats(ResNetPlan* p, const ConvL& c, const float* y, float* mean, float* rstd, int G,
                      cudaStream_t s, int64_t* launches) {
   const int64_t P = conv_pixels(p, c);
-  const int nq = (int)((P + kStatChunk - 1) / kStatChunk);
+  const int nq = (int)((P + kRnChunk - 1) / kRnChunk);
   const int lanes = std::max(1, 256 / c.cout);
   dim3 grid(nq, G);
   if (vec4_ok(c.cout))
-    RN_LAUNCH((bn_stats_partial_v4_kernel<<<grid, 256, 0, s>>>(y, P, c.cout, nq, p->part)));
+    RN_LAUNCH((bn_stats_partial_v4_kernel<<<grid, 256, 0, s>>>(y, P, c.cout, nq, kRnChunk, p->part)));
   else
-    RN_LAUNCH((bn_stats_partial_kernel<<<grid, lanes * c.cout, 0, s>>>(y, P, c.cout, nq, p->part)));
+    RN_LAUNCH((bn_stats_partial_kernel<<<grid, lanes * c.cout, 0, s>>>(y, P, c.cout, nq, kRnChunk,
+                                                                       p->part)));
   RN_LAUNCH((bn_stats_finalize_kernel<<<(G * c.cout * 32 + 127) / 128, 128, 0, s>>>(
-      p->part, P, c.cout, nq, G, mean, rstd)));
+      p->part, P, c.cout, nq, kRnChunk, G, mean, rstd)));
   return LSGD_OK;
 }
 
@@ -1102,17 +1175,17 @@ lsgd_status bn_backward(ResNetPlan* p, const ConvL& c, int i, const float* dout,
                         const float* W, float* Gr, cudaStream_t s, int64_t* launches) {
   const int K = p->K;
   const int64_t P = conv_pixels(p, c);
-  const int nq = (int)((P + kStatChunk - 1) / kStatChunk);
+  const int nq = (int)((P + kRnChunk - 1) / kRnChunk);
   const int lanes = std::max(1, 256 / c.cout);
   if (vec4_ok(c.cout))
     RN_LAUNCH((bn_bwd_partial_v4_kernel<TA><<<dim3(nq, K), 256, 0, s>>>(
         dout, reinterpret_cast<const TA*>(out), p->y[i], p->mean[i], p->rstd[i], P, c.cout, nq,
-        p->part)));
+        kRnChunk, p->part)));
   else
     RN_LAUNCH((bn_bwd_partial_kernel<TA><<<dim3(nq, K), lanes * c.cout, 0, s>>>(
         dout, reinterpret_cast<const TA*>(out), p->y[i], p->mean[i], p->rstd[i], P, c.cout, nq,
-        p->part)));
-  RN_LAUNCH((bn_bwd_finalize_kernel<<<(K * c.cout + 127) / 128, 128, 0, s>>>(
+        kRnChunk, p->part)));
+  RN_LAUNCH((bn_bwd_finalize_kernel<<<(K * c.cout * 32 + 127) / 128, 128, 0, s>>>(
       p->part, c.cout, nq, K, p->s12, Gr, c.g_off, c.b_off, p->d_pad)));
   if (vec4_ok(c.cout)) {
     RN_LAUNCH((bn_bwd_apply_v4_kernel<TA><<<dim3(px_blocks(P, c.cout), (unsigned)K), 256, 0, s>>>(
@@ -1186,30 +1259,52 @@ lsgd_status conv_dgrad(ResNetPlan* p, int i, const void* Wop, float* dx, const f
     // GEMM over dy's taps, no column matrix
     RN_LAUNCH((flip_weights_kernel<<<grid_for_items((int64_t)K * c.cin * 9 * c.cout), 256, 0, s>>>(
         reinterpret_cast<const uint16_t*>(Wop), p->d_pad, c.w_off, p->wt, K, c.cin, c.cout)));
-    TcGemmArgs t{};
-    t.M = (int)P;
-    t.N = c.cin;
-    t.Kd = 9 * c.cout;
-    t.G = K;
-    t.conv = 1;
-    t.cv_ck = c.cout;
-    t.cv_stride = 1;
-    t.cv_hout = c.hin;
-    t.cv_wout = c.win;
-    bool ok = make_tma_map_conv(&t.A.map, p->dy, c.cout, c.wout, c.hout, p->B, K, c.win, c.hin, 1);
-    ok &= make_tma_map(&t.B.map, p->wt, true, 9 * c.cout, c.cin, K, 9 * c.cout,
-                       (uint64_t)c.cin * 9 * c.cout, c.cout, 64, 2 * c.cout);
-    if (!ok) {
-      p->err = "TMA map encoding failed (implicit data gradient)";
-      return LSGD_ECUDA;
+    if (persistent_conv_ok(c.cin, P)) {
+      ConvArgs ca{};
+      bool okc = make_tma_map_conv(&ca.in_map, p->dy, c.cout, c.wout, c.hout, p->B, K, c.win,
+                                   c.hin, 1);
+      okc &= make_tma_map(&ca.w_map, p->wt, true, 9 * c.cout, c.cin, K, 9 * c.cout,
+                          (uint64_t)c.cin * 9 * c.cout, c.cout, c.cin, 2 * c.cout);
+      if (!okc) {
+        p->err = "TMA map encoding failed (implicit data gradient)";
+        return LSGD_ECUDA;
+      }
+      ca.ck = c.cout;
+      ca.stride = 1;
+      ca.hout = c.hin;
+      ca.wout = c.win;
+      ca.N = ca.np = c.cin;
+      ca.G = K;
+      ca.P = (int)P;
+      ca.out = dx;
+      ca.out_gs = P * c.cin;
+      RN_CALL(launch_conv_tc(ca, s));
+    } else {
+      TcGemmArgs t{};
+      t.M = (int)P;
+      t.N = c.cin;
+      t.Kd = 9 * c.cout;
+      t.G = K;
+      t.conv = 1;
+      t.cv_ck = c.cout;
+      t.cv_stride = 1;
+      t.cv_hout = c.hin;
+      t.cv_wout = c.win;
+      bool ok = make_tma_map_conv(&t.A.map, p->dy, c.cout, c.wout, c.hout, p->B, K, c.win, c.hin, 1);
+      ok &= make_tma_map(&t.B.map, p->wt, true, 9 * c.cout, c.cin, K, 9 * c.cout,
+                         (uint64_t)c.cin * 9 * c.cout, c.cout, 64, 2 * c.cout);
+      if (!ok) {
+        p->err = "TMA map encoding failed (implicit data gradient)";
+        return LSGD_ECUDA;
+      }
+      t.A.box_rows = kTcTileM;
+      t.B.box_rows = 64;
+      t.C = dx;
+      t.c_rs = c.cin;
+      t.c_gs = P * c.cin;
+      t.epi = EPI_STORE;
+      RN_CALL(launch_gemm_tc(t, s));
     }
-    t.A.box_rows = kTcTileM;
-    t.B.box_rows = 64;
-    t.C = dx;
-    t.c_rs = c.cin;
-    t.c_gs = P * c.cin;
-    t.epi = EPI_STORE;
-    RN_CALL(launch_gemm_tc(t, s));
     if (dout) {
       const int64_t n = (int64_t)p->B * c.hout * c.wout * (c.cin / 4);
       RN_LAUNCH((add_shortcut_grad_v2_kernel<TA><<<dim3((unsigned)((n + 255) / 256), (unsigned)K), 256,
@@ -1367,12 +1462,15 @@ cudaError_t launch_batchnorm_stats(const float* y, int64_t P, int C, int G, floa
   if (nq > 65535) return cudaErrorInvalidValue;
   const int lanes = std::max(1, 256 / C);
   if (vec4_ok(C))
-    bn_stats_partial_v4_kernel<<<dim3((unsigned)nq, (unsigned)G), 256, 0, s>>>(y, P, C, (int)nq, part);
+    bn_stats_partial_v4_kernel<<<dim3((unsigned)nq, (unsigned)G), 256, 0, s>>>(y, P, C, (int)nq,
+                                                                               kStatChunk, part);
   else
-    bn_stats_partial_kernel<<<dim3((unsigned)nq, (unsigned)G), lanes * C, 0, s>>>(y, P, C, (int)nq, part);
+    bn_stats_partial_kernel<<<dim3((unsigned)nq, (unsigned)G), lanes * C, 0, s>>>(y, P, C, (int)nq,
+                                                                               kStatChunk, part);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  bn_stats_finalize_kernel<<<(G * C * 32 + 127) / 128, 128, 0, s>>>(part, P, C, (int)nq, G, mean, rstd);
+  bn_stats_finalize_kernel<<<(G * C * 32 + 127) / 128, 128, 0, s>>>(part, P, C, (int)nq, kStatChunk,
+                                                                     G, mean, rstd);
   return cudaGetLastError();
 }
 
@@ -1508,7 +1606,7 @@ lsgd_status resnet_alloc(ResNetPlan* p, const std::function<void*(size_t)>& allo
     p->mean.push_back((float*)alloc((size_t)K * c.cout * 4));
     p->rstd.push_back((float*)alloc((size_t)K * c.cout * 4));
     const int64_t P = (int64_t)B * c.hout * c.wout;
-    const int64_t nq_s = (P + kStatChunk - 1) / kStatChunk;
+    const int64_t nq_s = (P + kRnChunk - 1) / kRnChunk;
     const int64_t nq_w = (P + kWgradChunk - 1) / kWgradChunk;
     part = std::max(part, (size_t)(K * nq_s * c.cout * 2));
     part = std::max(part, (size_t)(K * nq_w * c.cout * 9 * c.cin));

@@ -28,7 +28,10 @@ namespace {
 
 constexpr float kBnEps = 1e-5f;
 constexpr int kStatChunk = 1024;   // pixels per BatchNorm reduction chunk (lsgd_batchnorm_stats)
-constexpr int kRnChunk = 256;      // the same inside the ResNet step (more CTAs on small stages)
+constexpr int kRnChunk = 256;      // the smallest chunk inside the ResNet step (scratch sizing)
+// Pixels per reduction chunk inside the ResNet step: 1024 on large tensors, 256 on the small
+// later stages so that they still spread over many CTAs.
+int rn_chunk(int64_t P) { return P >= 65536 ? 1024 : kRnChunk; }
 constexpr int kWgradChunk = 2048;  // pixels per weight-gradient chunk
 constexpr int kWgradTile = 16;     // pixels staged per weight-gradient iteration
 constexpr int kMaxJ16 = 36;        // (9 Cin) / 16 accumulators per thread, Cin <= 64
@@ -779,29 +782,29 @@ __global__ void __launch_bounds__(256) im2col_row_kernel(const uint16_t* __restr
   }
 }
 
-// im2col with any channel count: col[g][p][tap Cin + ci] for j = tap Cin + ci < 9 Cin, zero for
-// the padding columns 9 Cin <= j < ldc (ldc a multiple of 8 keeps rows 16-byte aligned).
+// im2col with any channel count, one CTA per output row (b, oh) of replica blockIdx.y: its
+// threads over the row's Wout x ldc column entries (32-bit indexing).
 template <typename TA>
-__global__ void im2col_any_kernel(const TA* __restrict__ in, uint16_t* __restrict__ col, int G, int B,
-                                  int Hin, int Win, int Cin, int Hout, int Wout, int stride, int ldc) {
+__global__ void __launch_bounds__(256) im2col_any_row_kernel(const TA* __restrict__ in,
+                                                             uint16_t* __restrict__ col, int B,
+                                                             int Hin, int Win, int Cin, int Hout,
+                                                             int Wout, int stride, int ldc) {
+  const int g = blockIdx.y, row = blockIdx.x;
+  const int oh = row % Hout, b = row / Hout;
   const int64_t P = (int64_t)B * Hout * Wout;
-  const int64_t n = (int64_t)G * P * ldc;
-  const int64_t step = (int64_t)gridDim.x * blockDim.x;
-  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < n; e += step) {
-    const int j = (int)(e % ldc);
-    const int64_t t = e / ldc;
-    const int64_t p = t % P;
-    const int g = (int)(t / P);
+  const TA* ing = in + ((int64_t)g * B + b) * Hin * Win * Cin;
+  uint16_t* out = col + ((int64_t)g * P + (int64_t)row * Wout) * ldc;
+  const int J = 9 * Cin;
+  for (int e = threadIdx.x; e < Wout * ldc; e += blockDim.x) {
+    const int ow = e / ldc, j = e - ow * ldc;
     float v = 0.f;
-    if (j < 9 * Cin) {
-      const int tap = j / Cin, ci = j % Cin;
-      const int ow = (int)(p % Wout), oh = (int)((p / Wout) % Hout);
-      const int b = (int)(p / ((int64_t)Wout * Hout));
+    if (j < J) {
+      const int tap = j / Cin, ci = j - tap * Cin;
       const int ih = oh * stride + tap / 3 - 1, iw = ow * stride + tap % 3 - 1;
       if (ih >= 0 && ih < Hin && iw >= 0 && iw < Win)
-        v = Elem<TA>::load(in + ((((int64_t)g * B + b) * Hin + ih) * Win + iw) * Cin + ci);
+        v = Elem<TA>::load(ing + (ih * Win + iw) * Cin + ci);
     }
-    col[e] = f2bf(v);
+    out[e] = f2bf(v);
   }
 }
 
@@ -830,6 +833,32 @@ __global__ void __launch_bounds__(256) col_dgrad_v2_kernel(const uint16_t* __res
   *reinterpret_cast<uint4*>(col + ((int64_t)g * P + p) * 9 * Cout + (int64_t)r * 8) = v;
 }
 
+// The same as one CTA per input row (b, ih) of replica blockIdx.y, the output-gradient channel
+// count a template constant.
+template <int C8N>
+__global__ void __launch_bounds__(256) col_dgrad_row_kernel(const uint16_t* __restrict__ dy,
+                                                            uint16_t* __restrict__ col, int B,
+                                                            int Hin, int Win, int Hout, int Wout,
+                                                            int stride) {
+  constexpr int Cout = 8 * C8N, R = 9 * C8N;
+  const int g = blockIdx.y, row = blockIdx.x;
+  const int ih = row % Hin, b = row / Hin;
+  const int64_t P = (int64_t)B * Hin * Win;
+  const uint16_t* dyg = dy + ((int64_t)g * B + b) * Hout * Wout * Cout;
+  uint16_t* out = col + ((int64_t)g * P + (int64_t)row * Win) * 9 * Cout;
+  for (int e = threadIdx.x; e < Win * R; e += blockDim.x) {
+    const int iw = e / R, r = e - iw * R;
+    const int tap = r / C8N, c8 = r - tap * C8N;
+    const int hn = ih + tap / 3 - 1, wn = iw + tap % 3 - 1;
+    uint4 v = make_uint4(0u, 0u, 0u, 0u);
+    if (hn >= 0 && wn >= 0 && hn % stride == 0 && wn % stride == 0 && hn / stride < Hout &&
+        wn / stride < Wout)
+      v = __ldg(reinterpret_cast<const uint4*>(dyg + ((hn / stride) * Wout + wn / stride) * Cout +
+                                               c8 * 8));
+    *reinterpret_cast<uint4*>(out + (int64_t)e * 8) = v;
+  }
+}
+
 // Weights with each [9 Cin] row padded to ldc columns (zeros), bf16: the stem's tensor-core
 // operand (9 Cin = 27 is not a multiple of 8).
 __global__ void pad_weights_kernel(const uint16_t* __restrict__ Wb, int64_t d_pad, int64_t w_off,
@@ -855,8 +884,10 @@ __global__ void sum_partials_crop_kernel(const float* __restrict__ part, int nq,
     const int r = (int)((t / cols) % rows);
     const int g = (int)(t / ((int64_t)rows * cols));
     const float* p = part + (int64_t)g * nq * rows * ldc + (int64_t)r * ldc + j;
+    const int64_t qs = (int64_t)rows * ldc;
     float s = 0.f;
-    for (int q = 0; q < nq; ++q) s += p[(int64_t)q * rows * ldc];
+#pragma unroll 8
+    for (int q = 0; q < nq; ++q) s += p[q * qs];
     out[(int64_t)g * out_gs + (int64_t)r * cols + j] = s;
   }
 }
@@ -865,14 +896,13 @@ __global__ void sum_partials_crop_kernel(const float* __restrict__ part, int nq,
 // wt[g][ci][t][co] = w[g][co][8 - t][ci] (taps flipped, channels transposed), bf16.
 __global__ void flip_weights_kernel(const uint16_t* __restrict__ Wb, int64_t d_pad, int64_t w_off,
                                     uint16_t* __restrict__ wt, int G, int Cin, int Cout) {
-  const int64_t n = (int64_t)G * Cin * 9 * Cout;
-  const int64_t step = (int64_t)gridDim.x * blockDim.x;
-  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < n; e += step) {
-    const int co = (int)(e % Cout);
-    const int t = (int)((e / Cout) % 9);
-    const int ci = (int)((e / (9 * Cout)) % Cin);
-    const int g = (int)(e / ((int64_t)Cin * 9 * Cout));
-    wt[e] = Wb[(int64_t)g * d_pad + w_off + ((int64_t)co * 9 + (8 - t)) * Cin + ci];
+  // blockIdx.y = replica; 32-bit indexing within it (Cin 9 Cout < 2^31)
+  const int g = blockIdx.y, n = Cin * 9 * Cout;
+  const uint16_t* src = Wb + (int64_t)g * d_pad + w_off;
+  uint16_t* dst = wt + (int64_t)g * n;
+  for (int e = blockIdx.x * blockDim.x + threadIdx.x; e < n; e += gridDim.x * blockDim.x) {
+    const int co = e % Cout, t = (e / Cout) % 9, ci = e / (9 * Cout);
+    dst[e] = src[(co * 9 + (8 - t)) * Cin + ci];
   }
 }
 
@@ -1009,9 +1039,10 @@ lsgd_status conv_forward(ResNetPlan* p, int i, const void* in, const void* Wop, 
                                         256, 0, s>>>(in16, p->col[i], p->B, c.hin, c.win, c.cin,
                                                      c.hout, c.wout, c.stride)));
     } else {
-      RN_LAUNCH((im2col_any_kernel<uint16_t><<<grid_for_items((int64_t)G * P * Kc), 256, 0, s>>>(
-          reinterpret_cast<const uint16_t*>(in), p->col[i], G, p->B, c.hin, c.win, c.cin, c.hout,
-          c.wout, c.stride, Kc)));
+      RN_LAUNCH((im2col_any_row_kernel<uint16_t><<<dim3((unsigned)(p->B * c.hout), (unsigned)G), 256,
+                                                   0, s>>>(reinterpret_cast<const uint16_t*>(in),
+                                                           p->col[i], p->B, c.hin, c.win, c.cin,
+                                                           c.hout, c.wout, c.stride, Kc)));
       RN_LAUNCH((pad_weights_kernel<<<grid_for_items((int64_t)G * c.cout * Kc), 256, 0, s>>>(
           reinterpret_cast<const uint16_t*>(Wop), p->d_pad, c.w_off, p->wt, G, c.cout, 9 * c.cin, Kc)));
       wop = p->wt;
@@ -1100,16 +1131,17 @@ lsgd_status conv_forward(ResNetPlan* p, int i, const void* in, const void* Wop, 
 lsgd_status bn_stats(ResNetPlan* p, const ConvL& c, const float* y, float* mean, float* rstd, int G,
                      cudaStream_t s, int64_t* launches) {
   const int64_t P = conv_pixels(p, c);
-  const int nq = (int)((P + kRnChunk - 1) / kRnChunk);
+  const int chunk = rn_chunk(P);
+  const int nq = (int)((P + chunk - 1) / chunk);
   const int lanes = std::max(1, 256 / c.cout);
   dim3 grid(nq, G);
   if (vec4_ok(c.cout))
-    RN_LAUNCH((bn_stats_partial_v4_kernel<<<grid, 256, 0, s>>>(y, P, c.cout, nq, kRnChunk, p->part)));
+    RN_LAUNCH((bn_stats_partial_v4_kernel<<<grid, 256, 0, s>>>(y, P, c.cout, nq, chunk, p->part)));
   else
-    RN_LAUNCH((bn_stats_partial_kernel<<<grid, lanes * c.cout, 0, s>>>(y, P, c.cout, nq, kRnChunk,
+    RN_LAUNCH((bn_stats_partial_kernel<<<grid, lanes * c.cout, 0, s>>>(y, P, c.cout, nq, chunk,
                                                                        p->part)));
   RN_LAUNCH((bn_stats_finalize_kernel<<<(G * c.cout * 32 + 127) / 128, 128, 0, s>>>(
-      p->part, P, c.cout, nq, kRnChunk, G, mean, rstd)));
+      p->part, P, c.cout, nq, chunk, G, mean, rstd)));
   return LSGD_OK;
 }
 
@@ -1175,16 +1207,17 @@ lsgd_status bn_backward(ResNetPlan* p, const ConvL& c, int i, const float* dout,
                         const float* W, float* Gr, cudaStream_t s, int64_t* launches) {
   const int K = p->K;
   const int64_t P = conv_pixels(p, c);
-  const int nq = (int)((P + kRnChunk - 1) / kRnChunk);
+  const int chunk = rn_chunk(P);
+  const int nq = (int)((P + chunk - 1) / chunk);
   const int lanes = std::max(1, 256 / c.cout);
   if (vec4_ok(c.cout))
     RN_LAUNCH((bn_bwd_partial_v4_kernel<TA><<<dim3(nq, K), 256, 0, s>>>(
         dout, reinterpret_cast<const TA*>(out), p->y[i], p->mean[i], p->rstd[i], P, c.cout, nq,
-        kRnChunk, p->part)));
+        chunk, p->part)));
   else
     RN_LAUNCH((bn_bwd_partial_kernel<TA><<<dim3(nq, K), lanes * c.cout, 0, s>>>(
         dout, reinterpret_cast<const TA*>(out), p->y[i], p->mean[i], p->rstd[i], P, c.cout, nq,
-        kRnChunk, p->part)));
+        chunk, p->part)));
   RN_LAUNCH((bn_bwd_finalize_kernel<<<(K * c.cout * 32 + 127) / 128, 128, 0, s>>>(
       p->part, c.cout, nq, K, p->s12, Gr, c.g_off, c.b_off, p->d_pad)));
   if (vec4_ok(c.cout)) {
@@ -1257,8 +1290,9 @@ lsgd_status conv_dgrad(ResNetPlan* p, int i, const void* Wop, float* dx, const f
   if (conv_on_tc(p, c) && c.stride == 1 && implicit_conv_ok(c.cout, 1, c.hin, c.win)) {
     // stride 1: dx is the convolution of dy with the flipped, transposed weights -- an implicit
     // GEMM over dy's taps, no column matrix
-    RN_LAUNCH((flip_weights_kernel<<<grid_for_items((int64_t)K * c.cin * 9 * c.cout), 256, 0, s>>>(
-        reinterpret_cast<const uint16_t*>(Wop), p->d_pad, c.w_off, p->wt, K, c.cin, c.cout)));
+    RN_LAUNCH((flip_weights_kernel<<<dim3((unsigned)((c.cin * 9 * c.cout + 255) / 256), (unsigned)K), 256,
+                                       0, s>>>(reinterpret_cast<const uint16_t*>(Wop), p->d_pad, c.w_off,
+                                               p->wt, K, c.cin, c.cout)));
     if (persistent_conv_ok(c.cin, P)) {
       ConvArgs ca{};
       bool okc = make_tma_map_conv(&ca.in_map, p->dy, c.cout, c.wout, c.hout, p->B, K, c.win,
@@ -1318,12 +1352,25 @@ lsgd_status conv_dgrad(ResNetPlan* p, int i, const void* Wop, float* dx, const f
   if (conv_on_tc(p, c) && c.cin % 8 == 0) {
     // dx = col(dy) [P][9 Cout] x wt^T with the flipped, transposed weights (stride 1 or 2)
     const int Kc = 9 * c.cout;
-    RN_LAUNCH((col_dgrad_v2_kernel<<<dim3((unsigned)((P * 9 * (c.cout / 8) + 255) / 256), (unsigned)K),
+    const dim3 rows_grid((unsigned)(p->B * c.hin), (unsigned)K);
+    const uint16_t* dy16 = reinterpret_cast<const uint16_t*>(p->dy);
+    if (c.cout == 16)
+      RN_LAUNCH((col_dgrad_row_kernel<2><<<rows_grid, 256, 0, s>>>(dy16, p->colT, p->B, c.hin, c.win,
+                                                                   c.hout, c.wout, c.stride)));
+    else if (c.cout == 32)
+      RN_LAUNCH((col_dgrad_row_kernel<4><<<rows_grid, 256, 0, s>>>(dy16, p->colT, p->B, c.hin, c.win,
+                                                                   c.hout, c.wout, c.stride)));
+    else if (c.cout == 64)
+      RN_LAUNCH((col_dgrad_row_kernel<8><<<rows_grid, 256, 0, s>>>(dy16, p->colT, p->B, c.hin, c.win,
+                                                                   c.hout, c.wout, c.stride)));
+    else
+      RN_LAUNCH((col_dgrad_v2_kernel<<<dim3((unsigned)((P * 9 * (c.cout / 8) + 255) / 256), (unsigned)K),
                                          256, 0, s>>>(reinterpret_cast<const uint16_t*>(p->dy),
                                                       p->colT, p->B, c.hin, c.win, c.cout, c.hout,
                                                       c.wout, c.stride)));
-    RN_LAUNCH((flip_weights_kernel<<<grid_for_items((int64_t)K * c.cin * Kc), 256, 0, s>>>(
-        reinterpret_cast<const uint16_t*>(Wop), p->d_pad, c.w_off, p->wt, K, c.cin, c.cout)));
+    RN_LAUNCH((flip_weights_kernel<<<dim3((unsigned)((c.cin * Kc + 255) / 256), (unsigned)K), 256, 0,
+                                       s>>>(reinterpret_cast<const uint16_t*>(Wop), p->d_pad, c.w_off,
+                                            p->wt, K, c.cin, c.cout)));
     TcGemmArgs t{};
     t.M = (int)P;
     t.N = c.cin;

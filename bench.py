@@ -40,10 +40,10 @@ WORKLOAD = dict(name="mlp_3072-1024-1024-10_K16_B128_H16_bf16", widths=(3072, 10
 UPDATE_BYTES_PER_PARAM = 22
 FUSED_UPDATE_BYTES_PER_PARAM = 18
 AVERAGE_BYTES_PER_PARAM = 10
-# DRAM bytes (read + write) per step of the three weight-gradient + update launches, from the ncu
-# capture summarised in profiles/wgrad_update_mlp3072_K16_B128.md (below the algorithmic bytes
-# because part of each launch's writes is still in L2 when the launch ends).
-UPDATE_TRAFFIC_PER_STEP = 1121953792
+# DRAM bytes (read + write) per step of the update launches (the classifier head's backward and
+# the weight-gradient + update launch of both hidden layers), from the ncu capture summarised in
+# profiles/wgrad_update_mlp3072_K16_B128.md; None until that capture matches the current kernels.
+UPDATE_TRAFFIC_PER_STEP = None
 
 FALLBACK_HBM_GBS = 6800.0
 FALLBACK_BF16_TFLOPS = 1900.0
@@ -484,8 +484,9 @@ def main():
     upd_n, upd_ms = prof["update"]
     avg_n, avg_ms = prof["average"]
     widths = w["widths"]
-    # The update phase is the three fused weight-gradient + update launches of each step; the
-    # roofline unit is one step's worth of them (bytes summed over the layers).
+    # The update phase is each step's fused update launches (the head's backward, then one
+    # weight-gradient + update launch over both hidden layers); the roofline unit is one step's
+    # worth of them (bytes summed over the layers).
     if fused:
         upd_bytes = sum(FUSED_UPDATE_BYTES_PER_PARAM * K * widths[l] * widths[l + 1]
                         + 2 * K * B * (widths[l] + widths[l + 1]) for l in range(len(widths) - 1))
@@ -528,7 +529,8 @@ def main():
                      "bound": "hbm", "achieved": upd_gbs, "peak": hbm, "unit": "GB/s",
                      "frac": upd_gbs / hbm, "peak_source": f"{peak_src} hbm_gbs",
                      "traffic": UPDATE_TRAFFIC_PER_STEP if fused and K == w["K"] else None,
-                     "unit_of_work": ("one step's weight-gradient + update launches (3 layers)"
+                     "unit_of_work": ("one step's fused weight-gradient + update launches "
+                                      "(3 layers: the head's backward, one launch for the rest)"
                                       if fused else "one launch over the whole K x d buffer"),
                      "algorithmic_bytes": upd_bytes, "launches_per_unit": upd_n // S_},
         "sync_average": {"gbs": avg_gbs, "frac_of_hbm": (avg_gbs / hbm) if avg_gbs else None,

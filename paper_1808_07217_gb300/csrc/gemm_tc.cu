@@ -497,14 +497,17 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
 // accumulators while the previous tile's update runs.  The tile's parameters and momentum stream
 // through a ring of shared-memory slots in 32-column chunks (128 rows x 128 B, SWIZZLE_128B), are
 // updated in place, and go back to HBM by TMA stores (clipped at the matrix edge), together with
-// the bf16 shadow staged in a 64-byte-swizzled buffer.  One CTA per SM:
+// the bf16 shadow staged in a 64-byte-swizzled buffer.  The tiles of up to two layers form one
+// list (the first layer's, then the second's), so a layer's last partial wave and the launch's
+// ramp are paid once for both.  One CTA per SM:
 //   warp 0      operand producer: dZ / act k-blocks into a two-stage ring
 //   warp 1      MMA issuer: tcgen05.mma (M = N = 128, K = 16) into accumulator (tile & 1)
 //   warp 2      TMEM allocation (256 columns); w / u chunk producer
 //   warps 4-7   epilogue, one tile row per thread (TMEM lane quarter = warp % 4): per chunk,
 //               tcgen05.ld of 32 gradient columns, the local momentum-SGD update (weight decay,
-//               heavy-ball or Nesterov momentum, Sec. A.4) on w, u in shared memory, bf16 w into a staging buffer; thread 128 then issues the three TMA stores
-//               and recycles the slot of the chunk before once its stores have read it.
+//               heavy-ball or Nesterov momentum, Sec. A.4) on w, u in shared memory, bf16 w
+//               into a staging buffer; thread 128 then issues the three TMA stores and
+//               recycles the slot of the chunk before once its stores have read it.
 // Only thread 128 waits on the epilogue's mbarriers and the outcome reaches the other epilogue
 // threads through a named barrier, so a wait that runs out cannot split them.
 namespace wu {
@@ -568,10 +571,14 @@ __global__ void __launch_bounds__(wu::THREADS, 1) wgrad_update_kernel(
   WuSmem& sm = *reinterpret_cast<WuSmem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                           ~uintptr_t(1023));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int tiles_n = (args.N + wu::TN - 1) / wu::TN, tiles_m = (args.M + BM - 1) / BM;
-  const int tiles = tiles_n * tiles_m * args.G;
+  // tiles of layer 0 come first, then those of layer 1 (operand layouts are the same in both)
+  const int tn0 = (args.L[0].N + wu::TN - 1) / wu::TN, tm0 = (args.L[0].M + BM - 1) / BM;
+  const int tn1 = args.nl > 1 ? (args.L[1].N + wu::TN - 1) / wu::TN : 0;
+  const int tm1 = args.nl > 1 ? (args.L[1].M + BM - 1) / BM : 0;
+  const int tiles0 = tn0 * tm0 * args.G;
+  const int tiles = tiles0 + tn1 * tm1 * args.G;
   const int nk = (args.Kd + BK - 1) / BK;
-  const bool a_mn = args.A.mn_major, b_mn = args.B.mn_major;
+  const bool a_mn = args.L[0].A.mn_major, b_mn = args.L[0].B.mn_major;
   const bool has_u = args.sgd.u != nullptr;
   constexpr uint32_t kBytesA = BM * BK * 2, kBytesB = wu::TN * BK * 2;
 
@@ -604,7 +611,11 @@ __global__ void __launch_bounds__(wu::THREADS, 1) wgrad_update_kernel(
   const uint32_t tmem = sm.tmem_base;
   pdl_begin();  // everything above touched only shared memory and TMEM
 
-  auto tile_coords = [&](int t, int& g, int& m0, int& n0) {
+  auto tile_coords = [&](int t, const WgradUpdateLayer*& ly, int& g, int& m0, int& n0) {
+    const bool second = t >= tiles0;
+    ly = second ? &args.L[1] : &args.L[0];
+    const int tiles_n = second ? tn1 : tn0, tiles_m = second ? tm1 : tm0;
+    if (second) t -= tiles0;
     const int per_g = tiles_m * tiles_n;
     g = t / per_g;
     const int r = t % per_g;
@@ -617,8 +628,9 @@ __global__ void __launch_bounds__(wu::THREADS, 1) wgrad_update_kernel(
     int it = 0;
     bool ok = true;
     for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x) {
+      const WgradUpdateLayer* ly;
       int g, m0, n0;
-      tile_coords(t, g, m0, n0);
+      tile_coords(t, ly, g, m0, n0);
       for (int kb = 0; kb < nk; ++kb, ++it) {
         const int s = it % wu::ST;
         if (!mbar_wait(&sm.op_empty[s], ((it / wu::ST) & 1) ^ 1)) {
@@ -628,18 +640,18 @@ __global__ void __launch_bounds__(wu::THREADS, 1) wgrad_update_kernel(
         mbar_expect_tx(&sm.op_full[s], kBytesA + kBytesB);
         const int k0 = kb * BK;
         if (!a_mn) {
-          tma_load_3d(sm.a[s], &args.A.map, &sm.op_full[s], k0, m0, g);
+          tma_load_3d(sm.a[s], &ly->A.map, &sm.op_full[s], k0, m0, g);
         } else {
 #pragma unroll
           for (int i = 0; i < BM / 64; ++i)
-            tma_load_3d(sm.a[s] + i * 64 * BK * 2, &args.A.map, &sm.op_full[s], m0 + 64 * i, k0, g);
+            tma_load_3d(sm.a[s] + i * 64 * BK * 2, &ly->A.map, &sm.op_full[s], m0 + 64 * i, k0, g);
         }
         if (!b_mn) {
-          tma_load_3d(sm.b[s], &args.B.map, &sm.op_full[s], k0, n0, g);
+          tma_load_3d(sm.b[s], &ly->B.map, &sm.op_full[s], k0, n0, g);
         } else {
 #pragma unroll
           for (int i = 0; i < wu::TN / 64; ++i)
-            tma_load_3d(sm.b[s] + i * 64 * BK * 2, &args.B.map, &sm.op_full[s], n0 + 64 * i, k0, g);
+            tma_load_3d(sm.b[s] + i * 64 * BK * 2, &ly->B.map, &sm.op_full[s], n0 + 64 * i, k0, g);
         }
       }
     }
@@ -684,9 +696,10 @@ __global__ void __launch_bounds__(wu::THREADS, 1) wgrad_update_kernel(
     bool ok = true;
     const uint32_t bytes = wu::kChunkF32 * (has_u ? 2u : 1u);
     for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x) {
+      const WgradUpdateLayer* ly;
       int g, m0, n0;
-      tile_coords(t, g, m0, n0);
-      const int nc = wu_chunks(args.N, n0);
+      tile_coords(t, ly, g, m0, n0);
+      const int nc = wu_chunks(ly->N, n0);
       for (int c = 0; c < nc; ++c, ++q) {
         const int sl = q % wu::NS;
         if (!mbar_wait(&sm.wu_empty[sl], ((q / wu::NS) & 1) ^ 1)) {
@@ -694,8 +707,8 @@ __global__ void __launch_bounds__(wu::THREADS, 1) wgrad_update_kernel(
           break;
         }
         mbar_expect_tx(&sm.wu_full[sl], bytes);
-        tma_load_3d(sm.w[sl], &args.wmap, &sm.wu_full[sl], n0 + c * wu::CW, m0, g);
-        if (has_u) tma_load_3d(sm.u[sl], &args.umap, &sm.wu_full[sl], n0 + c * wu::CW, m0, g);
+        tma_load_3d(sm.w[sl], &ly->wmap, &sm.wu_full[sl], n0 + c * wu::CW, m0, g);
+        if (has_u) tma_load_3d(sm.u[sl], &ly->umap, &sm.wu_full[sl], n0 + c * wu::CW, m0, g);
       }
     }
     if (!ok) {
@@ -722,10 +735,11 @@ __global__ void __launch_bounds__(wu::THREADS, 1) wgrad_update_kernel(
     int q = 0, i = 0, wbi = 0;
     bool ok = true;
     for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x, ++i) {
+      const WgradUpdateLayer* ly;
       int g, m0, n0;
-      tile_coords(t, g, m0, n0);
+      tile_coords(t, ly, g, m0, n0);
       const int ab = i & 1;
-      const int nc = wu_chunks(args.N, n0);
+      const int nc = wu_chunks(ly->N, n0);
       if (!epi_wait(&sm.acc_full[ab], (i >> 1) & 1)) {
         ok = false;
         break;
@@ -765,9 +779,9 @@ __global__ void __launch_bounds__(wu::THREADS, 1) wgrad_update_kernel(
         asm volatile("bar.sync 1, 128;" ::: "memory");
         if (leader) {
           const int x = n0 + c * wu::CW;
-          tma_store_3d(&args.wmap, sm.w[sl], x, m0, g);
-          if (has_u) tma_store_3d(&args.umap, sm.u[sl], x, m0, g);
-          if (sp.wb) tma_store_3d(&args.wbmap, sm.wb[wbi], x, m0, g);
+          tma_store_3d(&ly->wmap, sm.w[sl], x, m0, g);
+          if (has_u) tma_store_3d(&ly->umap, sm.u[sl], x, m0, g);
+          if (sp.wb) tma_store_3d(&ly->wbmap, sm.wb[wbi], x, m0, g);
           asm volatile("cp.async.bulk.commit_group;" ::: "memory");
           // the stores of the chunk before have read their slot: hand it back to the producer
           asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
@@ -1119,12 +1133,21 @@ cudaError_t launch_conv_tc(const ConvArgs& a, cudaStream_t stream) {
 }
 
 cudaError_t launch_wgrad_update(const WgradUpdateArgs& a, cudaStream_t stream) {
-  if (a.M <= 0 || a.N <= 0 || a.G <= 0) return cudaSuccess;
+  if (a.nl < 1 || a.nl > kWgradMaxLayers) return cudaErrorInvalidValue;
+  if (a.G <= 0) return cudaSuccess;
   if (a.Kd <= 0 || !a.sgd.w || (a.sgd.mom != 0.f && !a.sgd.u)) return cudaErrorInvalidValue;
-  // operand boxes as the kernel expects them (64-wide MN-major boxes, or full K-major tiles)
-  if (a.A.mn_major ? a.A.box_rows != 64 : a.A.box_rows != BM) return cudaErrorInvalidValue;
-  if (a.B.mn_major ? a.B.box_rows != 64 : a.B.box_rows != wu::TN) return cudaErrorInvalidValue;
-  const int64_t tiles = (int64_t)((a.N + wu::TN - 1) / wu::TN) * ((a.M + BM - 1) / BM) * a.G;
+  int64_t tiles = 0;
+  for (int l = 0; l < a.nl; ++l) {
+    const WgradUpdateLayer& ly = a.L[l];
+    if (ly.M <= 0 || ly.N <= 0) return cudaErrorInvalidValue;
+    // operand boxes as the kernel expects them (64-wide MN-major boxes, or full K-major tiles),
+    // with the same layouts in every layer
+    if (ly.A.mn_major ? ly.A.box_rows != 64 : ly.A.box_rows != BM) return cudaErrorInvalidValue;
+    if (ly.B.mn_major ? ly.B.box_rows != 64 : ly.B.box_rows != wu::TN) return cudaErrorInvalidValue;
+    if (ly.A.mn_major != a.L[0].A.mn_major || ly.B.mn_major != a.L[0].B.mn_major)
+      return cudaErrorInvalidValue;
+    tiles += (int64_t)((ly.N + wu::TN - 1) / wu::TN) * ((ly.M + BM - 1) / BM) * a.G;
+  }
   if (tiles > 0x7fffffffLL) return cudaErrorInvalidValue;
   int dev = 0, sms = 0;
   cudaError_t e = cudaGetDevice(&dev);

@@ -208,11 +208,21 @@ bool make_tma_map_conv(CUtensorMap* map, const void* base, int ck, int win, int 
 // N, row stride N) -= update(dZ[g]^T act[g]) with the momentum and bf16 shadow of SgdParams.
 // wmap / umap: fp32 maps over sgd.w / sgd.u, dims {N, M, G}, strides {N, replica stride}, box
 // {32, 128}, 128-byte swizzle; wbmap: the same over sgd.wb in bf16 with a 64-byte swizzle.
-struct WgradUpdateArgs {
-  int M, N, Kd, G;
-  TcOperand A, B;  // dZ (m = output unit) and act (n = input), as for the weight-gradient GEMM
-  SgdParams sgd;
+// One layer of a weight-gradient + update launch: dZ (m = output unit) and act (n = input) as for
+// the weight-gradient GEMM, and 128 x 32 chunk maps of the layer's w, u (fp32) and bf16 shadow.
+struct WgradUpdateLayer {
+  int M, N;
+  TcOperand A, B;
   CUtensorMap wmap, umap, wbmap;
+};
+// Up to kWgradMaxLayers layers share one persistent launch (their tiles form one list, layer 0's
+// first).  All layers have the same contraction length Kd (= B_loc), replica count G and update
+// rule; sgd's pointers matter only for being null or not (u: momentum, wb: bf16 shadow).
+constexpr int kWgradMaxLayers = 2;
+struct WgradUpdateArgs {
+  int Kd, G, nl;
+  WgradUpdateLayer L[kWgradMaxLayers];
+  SgdParams sgd;
 };
 cudaError_t launch_wgrad_update(const WgradUpdateArgs& a, cudaStream_t stream);
 // The classifier head (last dense layer with at most kHeadMaxClasses outputs, bf16 mode): the

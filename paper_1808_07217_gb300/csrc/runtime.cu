@@ -461,6 +461,7 @@ lsgd_status dense_backward(lsgd_ctx* c) {
   int cur = 0;
   int l_top = L - 1;
   int bias_done = -1;  // layer whose bias the last data-gradient GEMM already handled
+  lsgd::WgradUpdateArgs wa{};  // fused weight-gradient + update layers not yet launched
   if (c->head) {
     // the last layer's weight / bias gradients and their update (its data gradient for the layer
     // below came with the head's forward kernel)
@@ -485,6 +486,8 @@ lsgd_status dense_backward(lsgd_ctx* c) {
   for (int l = l_top; l >= 0; --l) {
     const DenseLayer& Ly = c->layers[l];
     const void* dz = c->dz[cur];
+    // read before this layer's data gradient sets bias_done for the layer below
+    const bool bias_by_dgrad_above = bias_done == l;
     if (l > 0) {
       // data gradient dz_prev[j][i] = (sum_o dz[j][o] W[o][i]) * (act[j][i] > 0)
       void* dzp = c->dz[1 - cur];
@@ -575,29 +578,39 @@ lsgd_status dense_backward(lsgd_ctx* c) {
       if (c->fused) {
         // persistent weight-gradient + update kernel: parameters, momentum and the bf16 shadow
         // stream through shared memory by TMA in 128 x 32 chunks
-        lsgd::WgradUpdateArgs wa{};
-        wa.M = Ly.out;
-        wa.N = Ly.in;
-        wa.Kd = B;
-        wa.G = K;
-        wa.A = t.A;
-        wa.B = t.B;
-        wa.sgd = sgd_at(Ly.w_off);
-        bool mok = lsgd::make_tma_map(&wa.wmap, wa.sgd.w, false, Ly.in, Ly.out, K, Ly.in, c->d_pad,
+        lsgd::WgradUpdateLayer& wl = wa.L[wa.nl];
+        wl.M = Ly.out;
+        wl.N = Ly.in;
+        wl.A = t.A;
+        wl.B = t.B;
+        const lsgd::SgdParams sp = sgd_at(Ly.w_off);
+        bool mok = lsgd::make_tma_map(&wl.wmap, sp.w, false, Ly.in, Ly.out, K, Ly.in, c->d_pad,
                                       32, 128, 128);
-        if (wa.sgd.u)
-          mok &= lsgd::make_tma_map(&wa.umap, wa.sgd.u, false, Ly.in, Ly.out, K, Ly.in, c->d_pad,
+        if (sp.u)
+          mok &= lsgd::make_tma_map(&wl.umap, sp.u, false, Ly.in, Ly.out, K, Ly.in, c->d_pad,
                                     32, 128, 128);
-        if (wa.sgd.wb)
-          mok &= lsgd::make_tma_map(&wa.wbmap, wa.sgd.wb, true, Ly.in, Ly.out, K, Ly.in, c->d_pad,
+        if (sp.wb)
+          mok &= lsgd::make_tma_map(&wl.wbmap, sp.wb, true, Ly.in, Ly.out, K, Ly.in, c->d_pad,
                                     32, 128, 64);
         if (!mok) return fail(c, LSGD_ECUDA, "TMA map encoding failed (fused update)");
-        LSGD_LAUNCH(c, lsgd::launch_wgrad_update(wa, c->stream));
+        if (wa.nl == 0) wa.sgd = sp;
+        ++wa.nl;
+        // Layer 1's update waits for layer 0's, so both go in one launch: nothing in between
+        // writes the gradients they read (layer 0 has no data gradient) or reads the parameters
+        // they change.
+        if (!(l == 1 && c->layers[0].tc)) {
+          wa.Kd = B;
+          wa.G = K;
+          LSGD_LAUNCH(c, lsgd::launch_wgrad_update(wa, c->stream));
+          wa.nl = 0;
+          span(LSGD_PH_UPDATE);
+        }
       } else {
         t.C = c->G + Ly.w_off;
         t.epi = lsgd::EPI_STORE;
         lsgd_status st = tc_gemm(c, t);
         if (st != LSGD_OK) return st;
+        span(LSGD_PH_UPDATE);
       }
     } else {
       lsgd::GemmArgs g{};
@@ -622,10 +635,10 @@ lsgd_status dense_backward(lsgd_ctx* c) {
       g.epi = lsgd::EPI_STORE;
       lsgd_status st = gemm(c, g);
       if (st != LSGD_OK) return st;
+      span(LSGD_PH_UPDATE);
     }
-    span(LSGD_PH_UPDATE);
     // the bias sums: unless the head's kernel (layer L - 2) or the data-gradient GEMM above did them
-    if (Ly.b_off >= 0 && !(c->head && l == L - 2) && bias_done != l) {
+    if (Ly.b_off >= 0 && !(c->head && l == L - 2) && !bias_by_dgrad_above) {
       if (c->fused)
         LSGD_LAUNCH(c, lsgd::launch_colsum_update(dz, c->bf16, c->ld_dz, K, B, Ly.out, c->d_pad,
                                                   sgd_at(Ly.b_off), c->stream));

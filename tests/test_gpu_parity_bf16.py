@@ -132,10 +132,12 @@ def test_full_size_mlp_sampled_replicas(P):
 
 
 @pytest.mark.parametrize("mom,nest,wd", [(0.9, True, 5e-4), (0.9, False, 0.0), (0.0, False, 1e-4)])
-@pytest.mark.parametrize("widths,K,B", [((264, 136, 72, 10), 3, 40), ((3072, 1024, 1024, 10), 4, 128)])
+@pytest.mark.parametrize("widths,K,B", [((264, 136, 72, 10), 3, 40), ((3072, 1024, 1024, 10), 4, 128),
+                                        ((200, 136, 96, 72, 10), 2, 24)])
 def test_fused_update_is_bitwise_identical(P, mom, nest, wd, widths, K, B):
     # The update applied in the weight-gradient epilogue uses the same arithmetic as the
-    # stand-alone update kernel, so parameters, momentum and losses agree bit for bit.
+    # stand-alone update kernel, so parameters, momentum and losses agree bit for bit.  (The
+    # first two layers' updates share one launch; with four layers the third has its own.)
     N = 2048
     X, y = synthdata.gaussian_mixture(N, widths[0], widths[-1], seed=4)
     res = []

@@ -30,7 +30,14 @@ sys.path.insert(0, ROOT)
 
 WORKLOAD = dict(name="mlp_3072-1024-1024-10_K16_B128_H16_bf16", widths=(3072, 1024, 1024, 10),
                 K=16, B=128, H=16, N=50000, C=10, base_lr=0.1, scale_by_K=True, warmup_epochs=5.0,
-                momentum=0.9, nesterov=True, weight_decay=5e-4, seed=0, data_seed=1234)
+                momentum=0.9, nesterov=True, weight_decay=5e-4, seed=0, data_seed=1234,
+                epochs=2.0)
+
+
+def job_steps(w, K=None):
+    """T of one training job: ceil(epochs * N / (K * B_loc)) local steps (49 for the workload)."""
+    K = K or w["K"]
+    return -(-int(w["epochs"] * w["N"]) // (K * w["B"]))
 
 # Bytes the algorithm moves per parameter and replica (fp32 w, u, g; bf16 shadow):
 #   stand-alone update           = read g, w, u + write w, u (4 B each) + write the shadow (2 B) = 22
@@ -408,14 +415,27 @@ def main():
     X, y = synthdata.gaussian_mixture_cached(w["N"], w["widths"][0], w["C"], w["data_seed"])
     W_, S_ = max(3, args.warmup), args.steps
     e2e_warm = 2
-    total = W_ + S_ + S_ + e2e_warm + S_  # warm-up, timed, traced, end-to-end warm-up and timed
+    # The workload is a T-step job (2 epochs: 49 steps, the learning rate still warming up toward
+    # K x 0.1); longer runs repeat it from the model it ended with (lsgd_set_step(0) after the
+    # job's last step and its final average), so every timed step is a step of that schedule.
+    T_job = job_steps(w, K)
+    cfg = _make_cfg(P, T_job, fused, K)
+    _, kinds = P.lsgd_schedule(cfg, T_job)
     stream = torch.cuda.current_stream()
-    ctx = P.lsgd_create(_make_cfg(P, total, fused, K), stream=stream.cuda_stream)
+    ctx = P.lsgd_create(cfg, stream=stream.cuda_stream)
     P.lsgd_set_dataset(ctx, X, y)
     d = P.lsgd_num_params(ctx)
 
+    def run_steps(n):
+        while n > 0:
+            m = min(n, T_job - P.lsgd_step_count(ctx))
+            P.lsgd_run(ctx, m)
+            n -= m
+            if P.lsgd_step_count(ctx) == T_job:
+                P.lsgd_set_step(ctx, 0)
+
     # ---- device-resident timing ----
-    P.lsgd_run(ctx, W_)
+    run_steps(W_)
     torch.cuda.synchronize()
     clocks = ClockSampler(local)
     clocks.start()
@@ -427,7 +447,7 @@ def main():
     torch.cuda.synchronize()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record(stream)
-    P.lsgd_run(ctx, S_)
+    run_steps(S_)
     e1.record(stream)
     torch.cuda.synchronize()
     if world > 1:
@@ -438,8 +458,11 @@ def main():
     clk = clocks.stop()
 
     # ---- the same number of steps again with per-phase CUDA events (the split and roofline) ----
+    n_chk = min(P.lsgd_step_count(ctx), 16)
+    if n_chk and not np.isfinite(P.lsgd_losses(ctx, n_chk, K)).all():
+        raise RuntimeError("non-finite loss in the timed steps")
     P.lsgd_profile_enable(ctx, True)
-    P.lsgd_run(ctx, S_)
+    run_steps(S_)
     torch.cuda.synchronize()
     prof = P.lsgd_profile_read(ctx)
     P.lsgd_profile_enable(ctx, False)
@@ -452,29 +475,38 @@ def main():
     n_stage = 4
     xs, ys = [], []
     for i in range(n_stage):
-        idx = P.lsgd_debug_indices(ctx, W_ + 2 * S_ + i, K, B).reshape(-1)
+        idx = P.lsgd_debug_indices(ctx, (P.lsgd_step_count(ctx) + i) % T_job, K, B).reshape(-1)
         xs.append(torch.from_numpy(X[idx].reshape(K, B, -1)).pin_memory())
         ys.append(torch.from_numpy(y[idx].reshape(K, B).copy()).pin_memory())
     del rng
-    loss_host = np.empty((1, K), dtype=np.float32)
+    # every step's K losses come back to pinned host memory; the reads are asynchronous, like the
+    # host-to-device copies (which run on the library's copy stream, one batch ahead), and all
+    # of them have landed when the timed region ends
+    loss_host = torch.empty((max(S_, e2e_warm), K), dtype=torch.float32).pin_memory()
 
     def e2e_step(i):
         s = P.lsgd_step_count(ctx)
         P.lsgd_local_step_batch(ctx, xs[i % n_stage], ys[i % n_stage])
-        if (s + 1) % H == 0 or s == total - 1:
+        if kinds[s] == 2:  # the round ends with this step (the schedule of lsgd_run)
             P.lsgd_sync_average(ctx)
-        P.lib().lsgd_losses(ctx.handle, P._ptr(loss_host), 1)  # device -> host read, synchronises
+        P.lsgd_losses_async(ctx, loss_host[i], 1)  # device -> host read of this step's losses
+        if s + 1 == T_job:
+            P.lsgd_set_step(ctx, 0)
 
     for i in range(e2e_warm):
         e2e_step(i)
+    P.lsgd_synchronize(ctx)
     torch.cuda.synchronize()
     if world > 1:
         torch.distributed.barrier()
     t0 = time.perf_counter()
     for i in range(S_):
         e2e_step(i)
+    P.lsgd_synchronize(ctx)
     torch.cuda.synchronize()
     t_e2e = time.perf_counter() - t0
+    if not bool(torch.isfinite(loss_host[:S_]).all()):
+        raise RuntimeError("non-finite loss in the end-to-end steps")
     e2e_value = whole_job_throughput(samples_per_rank, t_e2e, world)
     h2d = K * B * w["widths"][0] * 4 + K * B * 4
     d2h = K * 4
@@ -518,6 +550,8 @@ def main():
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": {"workload": w["name"] if K == w["K"] else w["name"].replace("K16", f"K{K}"),
                    "global_batch": K * B, "K": K, "B_loc": B, "H": H, "fused_update": fused,
+                   "job": f"{T_job}-step schedule ({w['epochs']:g} epochs of N = {w['N']}), "
+                          "repeated from its end state",
                    "params_per_replica": d, "parallelism": "replicas" if world > 1 else "single",
                    "l2": "per-step working set (w, u, g, shadow: 1.0 GB) exceeds the 129 MB L2",
                    "syncs_in_timed_region": n_syncs},

@@ -175,9 +175,12 @@ lsgd_status lsgd_local_step(lsgd_ctx* ctx);
 
 /* Same step, but on a caller-supplied mini-batch x [K][B_loc][widths[0]] fp32 and labels
  * [K][B_loc] (or targets for LSQ), replica-major, instead of sampling the resident dataset.
- * `on_device` = 0: host pointers (pinned memory is copied asynchronously, pageable memory
- * synchronously); either way the caller keeps the buffers unchanged until the stream has reached
- * the step (e.g. until lsgd_losses for that step returns). */
+ * `on_device` = 0: host pointers, copied into one of two library-owned staging buffers on a copy
+ * stream of the library's (asynchronously from pinned memory, synchronously from pageable
+ * memory), so that the copy of the next batch can run while this step computes; the step waits
+ * for its copy, a copy waits until the step two batches earlier has read its buffer.  Either way
+ * the caller keeps the buffers unchanged until the step has been reached (lsgd_losses,
+ * lsgd_synchronize). */
 lsgd_status lsgd_local_step_batch(lsgd_ctx* ctx, const float* x, const void* labels_or_targets,
                                   int on_device);
 
@@ -222,6 +225,12 @@ lsgd_status lsgd_set_sync_state(lsgd_ctx* ctx, int which, int k, const float* sr
 /* Per-replica mean mini-batch loss of the last `n_steps` steps, [n_steps][K] fp32, oldest first.
  * The history holds the last T steps. */
 lsgd_status lsgd_losses(lsgd_ctx* ctx, float* dst, int64_t n_steps);
+/* The same read, enqueued on the context's stream without waiting: dst (host memory the caller
+ * owns; pinned for a truly asynchronous copy) holds the values once the stream has passed the
+ * copy, e.g. after lsgd_synchronize. */
+lsgd_status lsgd_losses_async(lsgd_ctx* ctx, float* dst, int64_t n_steps);
+/* Wait until every step, copy and average enqueued on the context so far has completed. */
+lsgd_status lsgd_synchronize(lsgd_ctx* ctx);
 
 /* The mini-batch indices I^k_s of step s for every worker, [K][B_loc] int32 (host). */
 lsgd_status lsgd_debug_indices(lsgd_ctx* ctx, int64_t step, int32_t* dst);
@@ -263,6 +272,12 @@ lsgd_status lsgd_schedule(const lsgd_config* cfg, int64_t n_steps, double* lr, i
 
 int64_t lsgd_num_params(const lsgd_ctx* ctx);   /* d, canonical (unpadded) */
 int64_t lsgd_step_count(const lsgd_ctx* ctx);   /* local steps taken so far (next step's s) */
+/* Make s the next step's index, 0 <= s <= T: the learning rate, the round ends and the sampled
+ * mini-batches follow s from there (s = 0 starts the schedule again from the current model).
+ * Parameters, momentum, synchronisation state and the counters of syncs and launches are kept;
+ * loss-history entries are overwritten as steps reuse their slots.  Steps already enqueued are
+ * unaffected (each carries its own s). */
+lsgd_status lsgd_set_step(lsgd_ctx* ctx, int64_t step);
 int64_t lsgd_sync_count(const lsgd_ctx* ctx);   /* global averages performed so far */
 int64_t lsgd_block_sync_count(const lsgd_ctx* ctx); /* block averages performed so far */
 int64_t lsgd_total_steps(const lsgd_ctx* ctx);  /* T */

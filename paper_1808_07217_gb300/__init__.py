@@ -41,7 +41,7 @@ EXPORTS = [
     "lsgd_profile_read", "lsgd_grouped_gemm_bf16", "lsgd_batchnorm_stats",
     "lsgd_batchnorm_stats_noalloc", "lsgd_block_average", "lsgd_block_sync_count",
     "lsgd_sync_state", "lsgd_set_sync_state", "lsgd_schedule", "lsgd_device_status",
-    "lsgd_bounded_wait_selftest",
+    "lsgd_bounded_wait_selftest", "lsgd_losses_async", "lsgd_synchronize", "lsgd_set_step",
 ]
 PHASES = ["input", "forward", "loss", "backward", "update", "average"]
 
@@ -157,6 +157,8 @@ def lib():
             "lsgd_bounded_wait_selftest": ([ctypes.c_int, ctypes.c_double, vp], st),
             "lsgd_set_sync_state": ([vp, ctypes.c_int, ctypes.c_int, vp, ctypes.c_size_t], st),
             "lsgd_losses": ([vp, vp, i64], st),
+            "lsgd_losses_async": ([vp, vp, i64], st),
+            "lsgd_synchronize": ([vp], st),
             "lsgd_debug_indices": ([vp, i64, vp], st),
             "lsgd_eval_loss": ([vp, ctypes.c_int, i64, P(ctypes.c_double)], st),
             "lsgd_check_finite": ([vp], st),
@@ -164,6 +166,7 @@ def lib():
             "lsgd_load": ([vp, ctypes.c_char_p], st),
             "lsgd_num_params": ([vp], i64),
             "lsgd_step_count": ([vp], i64),
+            "lsgd_set_step": ([vp, i64], st),
             "lsgd_sync_count": ([vp], i64),
             "lsgd_block_sync_count": ([vp], i64),
             "lsgd_block_average": ([vp], st),
@@ -372,6 +375,16 @@ def lsgd_losses(ctx: Ctx, n_steps: int, K: int):
     return out
 
 
+def lsgd_losses_async(ctx: Ctx, out, n_steps: int):
+    """Enqueue the read of the last n_steps steps' losses into `out` ([n_steps, K] fp32 host
+    array or pinned tensor the caller keeps alive); valid after lsgd_synchronize."""
+    _check(lib().lsgd_losses_async(ctx.handle, _ptr(out), int(n_steps)), ctx)
+
+
+def lsgd_synchronize(ctx: Ctx):
+    _check(lib().lsgd_synchronize(ctx.handle), ctx)
+
+
 def lsgd_debug_indices(ctx: Ctx, step: int, K: int, B: int):
     out = np.empty((int(K), int(B)), dtype=np.int32)
     _check(lib().lsgd_debug_indices(ctx.handle, int(step), _ptr(out)), ctx)
@@ -402,6 +415,10 @@ def lsgd_load(ctx: Ctx, path: str):
 
 def lsgd_step_count(ctx: Ctx) -> int:
     return int(lib().lsgd_step_count(ctx.handle))
+
+
+def lsgd_set_step(ctx: Ctx, step: int):
+    _check(lib().lsgd_set_step(ctx.handle, int(step)), ctx)
 
 
 def lsgd_sync_count(ctx: Ctx) -> int:

@@ -73,9 +73,15 @@ struct lsgd_ctx {
   int32_t* idx = nullptr;
   int32_t* yb = nullptr;
   float* tb = nullptr;
-  float* xstage = nullptr;
-  int32_t* ystage = nullptr;
-  float* tstage = nullptr;
+  // host mini-batches (lsgd_local_step_batch): two staging buffers filled on a copy stream, so
+  // the next batch's host-to-device copy overlaps the current step
+  float* xstage[2] = {nullptr, nullptr};
+  void* lstage[2] = {nullptr, nullptr};  // labels (int32) or targets (fp32)
+  cudaStream_t copy_stream = nullptr;
+  cudaEvent_t stage_copied[2] = {nullptr, nullptr};  // the copy into the buffer has landed
+  cudaEvent_t stage_free[2] = {nullptr, nullptr};    // the gather that read the buffer is done
+  bool stage_used[2] = {false, false};
+  int stage_next = 0;
   std::vector<void*> act;  // act[l]: input of dense layer l, [K][B][ld] operand dtype
   float* logits = nullptr;
   int ld_logits = 0;
@@ -919,8 +925,14 @@ lsgd_status lsgd_create(const lsgd_config* cfg, const lsgd_allocator* alloc, voi
 
 void lsgd_destroy(lsgd_ctx* c) {
   if (!c) return;
+  if (c->copy_stream) cudaStreamSynchronize(c->copy_stream);
   cudaStreamSynchronize(c->stream);
   for (cudaEvent_t e : c->prof_pool) cudaEventDestroy(e);
+  for (int i = 0; i < 2; ++i) {
+    if (c->stage_copied[i]) cudaEventDestroy(c->stage_copied[i]);
+    if (c->stage_free[i]) cudaEventDestroy(c->stage_free[i]);
+  }
+  if (c->copy_stream) cudaStreamDestroy(c->copy_stream);
   if (c->rn) lsgd::resnet_destroy(c->rn);
   free_all(c);
   cudaStreamSynchronize(c->stream);
@@ -983,22 +995,43 @@ lsgd_status lsgd_local_step_batch(lsgd_ctx* c, const float* x, const void* lab, 
   const float* xs = x;
   const void* ls = lab;
   const int64_t e0 = prof_mark(c);
+  int sl = -1;
   if (!on_device) {
-    if (!c->xstage) {
-      c->xstage = (float*)dalloc(c, rows * c->D * 4);
-      c->ystage = (int32_t*)dalloc(c, rows * 4);
-      if (!c->xstage || !c->ystage) return fail(c, LSGD_ENOMEM, "staging allocation failed");
+    // staging buffer sl: its copy waits until the gather of two batches ago has read it, and this
+    // step's gather waits for the copy; nothing else orders the copy stream against the step
+    if (!c->copy_stream) {
+      LSGD_TRY_CUDA(c, cudaStreamCreateWithFlags(&c->copy_stream, cudaStreamNonBlocking));
+      for (int i = 0; i < 2; ++i) {
+        LSGD_TRY_CUDA(c, cudaEventCreateWithFlags(&c->stage_copied[i], cudaEventDisableTiming));
+        LSGD_TRY_CUDA(c, cudaEventCreateWithFlags(&c->stage_free[i], cudaEventDisableTiming));
+      }
     }
-    LSGD_TRY_CUDA(c, cudaMemcpyAsync(c->xstage, x, rows * c->D * 4, cudaMemcpyHostToDevice, c->stream));
-    LSGD_TRY_CUDA(c, cudaMemcpyAsync(c->ystage, lab, rows * 4, cudaMemcpyHostToDevice, c->stream));
-    xs = c->xstage;
-    ls = c->ystage;
+    sl = c->stage_next;
+    if (!c->xstage[sl]) {
+      c->xstage[sl] = (float*)dalloc(c, rows * c->D * 4);
+      c->lstage[sl] = dalloc(c, rows * 4);
+      if (!c->xstage[sl] || !c->lstage[sl]) return fail(c, LSGD_ENOMEM, "staging allocation failed");
+    }
+    if (c->stage_used[sl]) LSGD_TRY_CUDA(c, cudaStreamWaitEvent(c->copy_stream, c->stage_free[sl], 0));
+    LSGD_TRY_CUDA(c, cudaMemcpyAsync(c->xstage[sl], x, rows * c->D * 4, cudaMemcpyHostToDevice,
+                                     c->copy_stream));
+    LSGD_TRY_CUDA(c, cudaMemcpyAsync(c->lstage[sl], lab, rows * 4, cudaMemcpyHostToDevice,
+                                     c->copy_stream));
+    LSGD_TRY_CUDA(c, cudaEventRecord(c->stage_copied[sl], c->copy_stream));
+    LSGD_TRY_CUDA(c, cudaStreamWaitEvent(c->stream, c->stage_copied[sl], 0));
+    c->stage_next ^= 1;
+    xs = c->xstage[sl];
+    ls = c->lstage[sl];
   }
   const int32_t* yl = c->lsq ? nullptr : (const int32_t*)ls;
   const float* tl = c->lsq ? (const float*)ls : nullptr;
   LSGD_LAUNCH(c, lsgd::launch_gather_rows(input_buffer(c), c->bf16, input_ld(c), xs, c->D, nullptr,
                                           (int)rows, yl, yl ? c->yb : nullptr, tl,
                                           tl ? c->tb : nullptr, c->stream));
+  if (sl >= 0) {
+    LSGD_TRY_CUDA(c, cudaEventRecord(c->stage_free[sl], c->stream));
+    c->stage_used[sl] = true;
+  }
   return step_body(c, e0);
 }
 
@@ -1196,7 +1229,7 @@ lsgd_status lsgd_set_sync_state(lsgd_ctx* c, int which, int k, const float* src,
   return LSGD_OK;
 }
 
-lsgd_status lsgd_losses(lsgd_ctx* c, float* dst, int64_t n_steps) {
+static lsgd_status copy_losses(lsgd_ctx* c, float* dst, int64_t n_steps) {
   if (!c || !dst) return fail(c, LSGD_EINVAL, "NULL argument");
   if (n_steps < 0 || n_steps > c->step || n_steps > c->loss_cap)
     return fail(c, LSGD_EINVAL, "n_steps exceeds the recorded history");
@@ -1206,6 +1239,23 @@ lsgd_status lsgd_losses(lsgd_ctx* c, float* dst, int64_t n_steps) {
     LSGD_TRY_CUDA(c, cudaMemcpyAsync(dst + i * K, c->loss_hist + (s % c->loss_cap) * K, (size_t)K * 4,
                                      cudaMemcpyDeviceToHost, c->stream));
   }
+  return LSGD_OK;
+}
+
+lsgd_status lsgd_losses(lsgd_ctx* c, float* dst, int64_t n_steps) {
+  lsgd_status st = copy_losses(c, dst, n_steps);
+  if (st != LSGD_OK) return st;
+  LSGD_TRY_CUDA(c, cudaStreamSynchronize(c->stream));
+  return LSGD_OK;
+}
+
+lsgd_status lsgd_losses_async(lsgd_ctx* c, float* dst, int64_t n_steps) {
+  return copy_losses(c, dst, n_steps);
+}
+
+lsgd_status lsgd_synchronize(lsgd_ctx* c) {
+  if (!c) return fail(nullptr, LSGD_EINVAL, "NULL context");
+  if (c->copy_stream) LSGD_TRY_CUDA(c, cudaStreamSynchronize(c->copy_stream));
   LSGD_TRY_CUDA(c, cudaStreamSynchronize(c->stream));
   return LSGD_OK;
 }
@@ -1397,6 +1447,14 @@ lsgd_status lsgd_load(lsgd_ctx* c, const char* path) {
 
 int64_t lsgd_num_params(const lsgd_ctx* c) { return c ? c->d : -1; }
 int64_t lsgd_step_count(const lsgd_ctx* c) { return c ? c->step : -1; }
+
+lsgd_status lsgd_set_step(lsgd_ctx* c, int64_t step) {
+  if (!c) return fail(nullptr, LSGD_EINVAL, "NULL context");
+  if (step < 0 || step > c->T) return fail(c, LSGD_EINVAL, "step must lie in [0, T]");
+  c->step = step;  // steps already enqueued carry their own s, learning rate and sync kind
+  c->cursor = RoundCursor{};
+  return LSGD_OK;
+}
 int64_t lsgd_sync_count(const lsgd_ctx* c) { return c ? c->syncs : -1; }
 int64_t lsgd_block_sync_count(const lsgd_ctx* c) { return c ? c->block_syncs : -1; }
 lsgd_status lsgd_schedule(const lsgd_config* cfg, int64_t n_steps, double* lr, int32_t* sync_kind) {

@@ -84,6 +84,42 @@ def test_caller_batches_equal_sampled_steps(P, prec):
     P.lsgd_destroy(b)
 
 
+def test_pipelined_host_batches_equal_sampled_steps(P):
+    # Seven host batches enqueued back to back with asynchronous loss reads: the copies run ahead
+    # on the library's copy stream through its two staging buffers, and every step must still
+    # see its own batch (a buffer overwritten before its gather ran would change the result).
+    import torch
+
+    g, o, X, y = _small(P, P.BF16, T=8, H=3)
+    a = P.lsgd_create(g)
+    P.lsgd_set_dataset(a, X, y)
+    b = P.lsgd_create(g)
+    P.lsgd_set_dataset(b, X, y)
+    n = 7
+    batches = []
+    for s in range(n):
+        idx = P.lsgd_debug_indices(b, s, 4, 16).reshape(-1)
+        xb = torch.from_numpy(X[idx].reshape(4, 16, -1).copy())
+        yb = torch.from_numpy(y[idx].reshape(4, 16).copy())
+        if s != 4:  # one pageable batch among the pinned ones
+            xb, yb = xb.pin_memory(), yb.pin_memory()
+        batches.append((xb, yb))
+    losses = torch.zeros((n, 4), dtype=torch.float32).pin_memory()
+    for s in range(n):
+        P.lsgd_local_step(a)
+        P.lsgd_local_step_batch(b, *batches[s])
+        if (s + 1) % 3 == 0:
+            P.lsgd_sync_average(a)
+            P.lsgd_sync_average(b)
+        P.lsgd_losses_async(b, losses[s], 1)
+    P.lsgd_synchronize(b)
+    for k in range(4):
+        assert np.array_equal(P.lsgd_params(a, k), P.lsgd_params(b, k))
+    assert np.array_equal(P.lsgd_losses(a, n, 4), losses.numpy())
+    P.lsgd_destroy(a)
+    P.lsgd_destroy(b)
+
+
 def test_sync_counts_follow_schedule(P):
     for T, H, tp in [(49, 16, -1), (25, 16, 12), (10, 3, 0), (9, 4, 20)]:
         g, o, X, y = _small(P, P.BF16, T=T, H=H, t_switch=tp)

@@ -309,12 +309,15 @@ def run_sync_variants(args):
 
 RESNET_WORKLOAD = dict(name="resnet20_K16_B128_postlocal_H16_bf16", K=16, B=128, H=16, N=50000,
                        C=10, base_lr=0.2, scale_by_K=True, warmup_epochs=5.0, momentum=0.9,
-                       nesterov=True, weight_decay=1e-4, seed=0, data_seed=1234)
+                       nesterov=True, weight_decay=1e-4, seed=0, data_seed=1234, epochs=1.0)
 
 
 def run_resnet(args):
-    """Post-local ResNet-20 (K = 16, B_loc = 128, H = 16 after t' = T / 2): samples/s over the
-    local-SGD phase with the per-phase split.  One JSON line."""
+    """Post-local ResNet-20 (K = 16, B_loc = 128): the 25-step job of one epoch, H = 1 before
+    t' = floor(T / 2) and H = 16 after, learning rate decayed at 50 % and 75 % of T, repeated from
+    its end state; samples/s over whole jobs' steps, then the per-phase split from a traced pass.
+    One JSON line."""
+    import numpy as np
     import torch
 
     import synthdata
@@ -328,9 +331,9 @@ def run_resnet(args):
     K, B = args.replicas or w["K"], w["B"]
     X, y = synthdata.gaussian_mixture_cached(w["N"], 3072, w["C"], w["data_seed"])
     W_, S_ = max(3, args.warmup), args.steps
-    total = W_ + S_
+    T_job = job_steps(w, K)
     stream = torch.cuda.current_stream()
-    cfg = P.make_config(K=K, B_loc=B, H=w["H"], t_switch=0, total_steps=total, N=w["N"],
+    cfg = P.make_config(K=K, B_loc=B, H=w["H"], t_switch=T_job // 2, total_steps=T_job, N=w["N"],
                         kind=P.RESNET20, in_hwc=(32, 32, 3), n_classes=w["C"], base_ch=16,
                         res_blocks=3, base_lr=w["base_lr"], scale_by_K=w["scale_by_K"],
                         warmup_epochs=w["warmup_epochs"], milestones=(0.5, 0.75),
@@ -338,20 +341,36 @@ def run_resnet(args):
                         weight_decay=w["weight_decay"], seed=w["seed"], precision=P.BF16)
     ctx = P.lsgd_create(cfg, stream=stream.cuda_stream)
     P.lsgd_set_dataset(ctx, X, y)
-    P.lsgd_run(ctx, W_)
+
+    def run_steps(n):
+        while n > 0:
+            m = min(n, T_job - P.lsgd_step_count(ctx))
+            P.lsgd_run(ctx, m)
+            n -= m
+            if P.lsgd_step_count(ctx) == T_job:
+                P.lsgd_set_step(ctx, 0)
+
+    run_steps(W_)
     torch.cuda.synchronize()
-    n0 = P.lsgd_kernel_launches(ctx)
-    P.lsgd_profile_enable(ctx, True)
+    n0, sy0 = P.lsgd_kernel_launches(ctx), P.lsgd_sync_count(ctx)
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record(stream)
-    P.lsgd_run(ctx, S_)
+    run_steps(S_)
     e1.record(stream)
     torch.cuda.synchronize()
     ms = e0.elapsed_time(e1)
+    launches, syncs = P.lsgd_kernel_launches(ctx) - n0, P.lsgd_sync_count(ctx) - sy0
+    n_chk = min(P.lsgd_step_count(ctx), 8)
+    if n_chk and not np.isfinite(P.lsgd_losses(ctx, n_chk, K)).all():
+        raise RuntimeError("non-finite loss in the timed steps")
+    P.lsgd_profile_enable(ctx, True)
+    run_steps(S_)
+    torch.cuda.synchronize()
     prof = P.lsgd_profile_read(ctx)
     print(json.dumps({"workload": w["name"], "value": S_ * K * B / (ms / 1000.0),
                       "unit": "samples/s", "steps": S_, "ms_per_step": ms / S_,
-                      "gpu_launches": P.lsgd_kernel_launches(ctx) - n0,
+                      "job": f"{T_job}-step schedule (t' = {T_job // 2}), repeated from its end state",
+                      "syncs_in_timed_region": syncs, "gpu_launches": launches,
                       "phase_ms_per_step": {k: v[1] / S_ for k, v in prof.items()},
                       "params_per_replica": P.lsgd_num_params(ctx)}), flush=True)
     P.lsgd_destroy(ctx)

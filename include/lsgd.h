@@ -347,6 +347,19 @@ lsgd_status lsgd_grouped_gemm_bf16(const uint16_t* A, int a_mn, const uint16_t* 
 lsgd_status lsgd_batchnorm_stats(const float* y, int64_t P, int C, int G, float* mean, float* rstd,
                                  void* stream);
 
+/* Weight gradient of a 3x3 convolution with zero padding 1 and stride s (1 or 2), the product
+ * behind ResNet-20's backward pass (Sec. A.2), for G independent groups on the tensor cores:
+ *   dW[g][co][kh][kw][ci] = sum over b, oy, ox of dy[g][b][oy][ox][co] x[g][b][oy s + kh - 1][ox s + kw - 1][ci]
+ * (x zero outside the image).  x [G][B][s Hout][s Wout][Cin] and dy [G][B][Hout][Wout][Cout] are
+ * NHWC bf16 device arrays (16-byte aligned), dW [G][Cout][3][3][Cin] fp32 device, fully
+ * overwritten.  The column matrix of every 64-pixel block is built in shared memory; one fp32
+ * partial per CTA (a scratch buffer allocated and freed on `stream`) is summed in CTA order, so
+ * the result is deterministic.  Cin 16, 32 or 64; Cout a multiple of 16 up to 64; Wout dividing
+ * 64 and Hout Wout a multiple of 64: LSGD_EINVAL otherwise, LSGD_ENOMEM if the scratch cannot be
+ * allocated, LSGD_EUNSUPPORTED without tcgen05. */
+lsgd_status lsgd_conv_wgrad_bf16(const uint16_t* x, const uint16_t* dy, float* dW, int G, int B,
+                                 int Hout, int Wout, int Cin, int Cout, int stride, void* stream);
+
 /* lsgd_batchnorm_stats for callers that cannot allocate device memory during a run: a program
  * whose device memory is all handed to its own caching pool (an allocation would fail, or force
  * the pool to give memory back and stall), or a latency-critical loop that fixes its memory use at

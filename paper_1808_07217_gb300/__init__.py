@@ -42,6 +42,7 @@ EXPORTS = [
     "lsgd_batchnorm_stats_noalloc", "lsgd_block_average", "lsgd_block_sync_count",
     "lsgd_sync_state", "lsgd_set_sync_state", "lsgd_schedule", "lsgd_device_status",
     "lsgd_bounded_wait_selftest", "lsgd_losses_async", "lsgd_synchronize", "lsgd_set_step",
+    "lsgd_conv_wgrad_bf16",
 ]
 PHASES = ["input", "forward", "loss", "backward", "update", "average"]
 
@@ -167,6 +168,7 @@ def lib():
             "lsgd_num_params": ([vp], i64),
             "lsgd_step_count": ([vp], i64),
             "lsgd_set_step": ([vp, i64], st),
+            "lsgd_conv_wgrad_bf16": ([vp, vp, vp] + [ctypes.c_int] * 7 + [vp], st),
             "lsgd_sync_count": ([vp], i64),
             "lsgd_block_sync_count": ([vp], i64),
             "lsgd_block_average": ([vp], st),
@@ -488,6 +490,16 @@ def lsgd_grouped_gemm_bf16(A, a_mn: bool, B, b_mn: bool, C, M: int, N: int, Kd: 
     _check(lib().lsgd_grouped_gemm_bf16(_ptr(A), int(bool(a_mn)), _ptr(B), int(bool(b_mn)), _ptr(C),
                                         int(M), int(N), int(Kd), int(G), int(engine),
                                         ctypes.c_void_p(stream)))
+
+
+def lsgd_conv_wgrad_bf16(x, dy, dW, G: int, B: int, Hout: int, Wout: int, Cin: int, Cout: int,
+                         stride: int, stream=None):
+    """dW [G, Cout, 3, 3, Cin] float32 = the 3x3 (pad 1, stride) convolution weight gradient of
+    NHWC bfloat16 CUDA tensors x [G, B, stride Hout, stride Wout, Cin] and dy [G, B, Hout, Wout, Cout]."""
+    stream = _current_stream() if stream is None else stream
+    _check(lib().lsgd_conv_wgrad_bf16(_ptr(x), _ptr(dy), _ptr(dW), int(G), int(B), int(Hout),
+                                      int(Wout), int(Cin), int(Cout), int(stride),
+                                      ctypes.c_void_p(stream)))
 
 
 def lsgd_batchnorm_stats(y, P: int, C: int, G: int, mean, rstd, stream=None):

@@ -968,6 +968,197 @@ __global__ void __launch_bounds__(cv::THREADS, 1) conv_tc_kernel(const __grid_co
   }
 }
 
+
+// =============================================================================================
+// Weight gradient of a 3x3 convolution on the tensor cores, column matrix built in shared memory:
+//   dW[g][co][t][ci] = sum over output pixels p of dy[g][p][co] x[g][src_t(p)][ci].
+// As D[m][n] = sum_k A[m][k] B[n][k] with m = t Cin + ci (9 Cin rows in 128-row tiles), n = co
+// (one 64-wide operand, zero beyond Cout) and k = output pixels in blocks of 64: B is the output
+// gradient's 64 x 64 tile by TMA (pixel-major = MN-major, 128-byte swizzle); A is MN-major too,
+// gathered by the builder warps from a TMA-loaded strip of input rows (the halo rows above and
+// below come from out-of-bounds zero fill, the halo columns are written as zeros): one 16-byte
+// chunk = 8 channels of one tap and pixel per copy.  A CTA owns one replica and a contiguous range
+// of pixel blocks and keeps every m-tile's 128 x 64 fp32 accumulator in TMEM; it writes its
+// partial dW, and a second kernel sums the CTAs' partials in order.  Rows m >= 9 Cin of the last
+// m-tile are never written: they only reach accumulator rows that are not stored.
+//   warp 0      TMA producer (input strip + output-gradient tile per block), NS-stage ring
+//   warp 1      MMA issuer: per block and m-tile, 4 x tcgen05.mma (M = 128, N = 64, K = 16)
+//   warp 2      TMEM allocation
+//   warps 4-7   build A for each block; at the end, tcgen05.ld of the accumulators and the
+//               partial's stores
+namespace cw {
+constexpr int THREADS = 256;
+constexpr int NS = 2;       // pipeline stages
+constexpr int KB = 64;      // output pixels per block
+constexpr int EPI0 = 128;   // first builder thread
+constexpr int MAX_MT = 5;   // m-tiles (9 Cin <= 640)
+constexpr uint32_t kTileA = 16384;  // one m-tile of A: two 64-row atoms x 64 pixels x 128 B
+constexpr uint32_t kTileB = 8192;   // the output-gradient tile: 64 pixels x 128 B
+}  // namespace cw
+
+__host__ __device__ inline int cw_rows(int stride, int wout) { return (cw::KB / wout - 1) * stride + 3; }
+__host__ __device__ inline uint32_t cw_halo_pitch(int cin, int stride, int win, int wout) {
+  return ((uint32_t)cw_rows(stride, wout) * win * cin * 2 + 1023u) & ~1023u;
+}
+
+__global__ void __launch_bounds__(cw::THREADS, 1) conv_wgrad_tc_kernel(
+    const __grid_constant__ ConvWgradArgs a) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~uintptr_t(1023));
+  const int cin = a.cin, cout = a.cout, mrows = 9 * cin;
+  const int mt_n = (mrows + 127) / 128;
+  const int rh = cw_rows(a.stride, a.wout);
+  const uint32_t halo_bytes = (uint32_t)rh * a.win * cin * 2;
+  const uint32_t halo_pitch = cw_halo_pitch(cin, a.stride, a.win, a.wout);
+  const uint32_t a_bytes = (uint32_t)mt_n * cw::kTileA;
+  uint8_t* A0 = base;                              // [NS][mt_n][2][64][128 B]
+  uint8_t* B0 = A0 + cw::NS * a_bytes;             // [NS][64][128 B]
+  uint8_t* X0 = B0 + cw::NS * cw::kTileB;          // [NS][rh][Win][Cin]
+  uint64_t* full = reinterpret_cast<uint64_t*>(X0 + cw::NS * halo_pitch);
+  uint64_t* empty = full + cw::NS;
+  uint64_t* aready = empty + cw::NS;
+  uint64_t* acc_full = aready + cw::NS;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(acc_full + 1);
+  int* epi_ok = reinterpret_cast<int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int g = blockIdx.y, q = blockIdx.x, cpr = gridDim.x;
+  const int nkb = a.P / cw::KB;
+  const int kb0 = (int)((int64_t)q * nkb / cpr);
+  const int nblk = (int)((int64_t)(q + 1) * nkb / cpr) - kb0;
+  const int per_img = a.hout * a.wout;
+  uint32_t tmem_cols = 32;
+  while (tmem_cols < (uint32_t)mt_n * 64) tmem_cols <<= 1;
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < cw::NS; ++i) {
+      mbar_init(&full[i], 1);
+      mbar_init(&empty[i], 1);
+      mbar_init(&aready[i], 1);
+    }
+    mbar_init(acc_full, 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  }
+  if (warp == 2) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     smem_u32(tmem_slot)),
+                 "r"(tmem_cols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+  __syncthreads();
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+  const uint32_t tmem = *tmem_slot;
+  pdl_begin();  // everything above touched only shared memory and TMEM
+
+  if (warp == 0 && lane == 0) {
+    // ---------------- producer ----------------
+    int j = 0;
+    for (; j < nblk; ++j) {
+      const int s = j % cw::NS;
+      if (!mbar_wait(&empty[s], ((j / cw::NS) & 1) ^ 1)) break;
+      const int p0 = (kb0 + j) * cw::KB;
+      const int b = p0 / per_img, oy0 = (p0 % per_img) / a.wout;
+      mbar_expect_tx(&full[s], halo_bytes + cw::kTileB);
+      tma_load_5d(X0 + s * halo_pitch, &a.x_map, &full[s], 0, 0, oy0 * a.stride - 1, b, g);
+      tma_load_3d(B0 + s * cw::kTileB, &a.dy_map, &full[s], 0, p0, g);
+    }
+    // copies in flight land before the CTA can exit
+    for (int i = (j > cw::NS ? j - cw::NS : 0); i < j; ++i)
+      mbar_wait(&full[i % cw::NS], (i / cw::NS) & 1);
+  } else if (warp == 1 && lane == 0) {
+    // ---------------- MMA issuer ----------------
+    const uint32_t idesc = make_idesc(BM, 64, true, true);
+    bool ok = true;
+    for (int j = 0; j < nblk; ++j) {
+      const int s = j % cw::NS;
+      const uint32_t ph = (j / cw::NS) & 1;
+      if (!mbar_wait(&aready[s], ph) || !mbar_wait(&full[s], ph)) {
+        ok = false;
+        break;
+      }
+      asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+      const uint32_t ab = smem_u32(A0 + s * a_bytes), bb = smem_u32(B0 + s * cw::kTileB);
+      for (int mt = 0; mt < mt_n; ++mt)
+#pragma unroll
+        for (int kk = 0; kk < cw::KB / 16; ++kk)
+          mma_bf16(tmem + (uint32_t)(mt * 64), smem_desc(ab + mt * cw::kTileA + kk * 2048, 8192, 1024),
+                   smem_desc(bb + kk * 2048, 8192, 1024), idesc, (j > 0 || kk > 0) ? 1u : 0u);
+      mma_commit(&empty[s]);  // stage reusable once these MMAs have read it
+    }
+    if (ok && nblk > 0) mma_commit(acc_full);
+  } else if (warp >= 4) {
+    // ---------------- builders, then the epilogue ----------------
+    const int tid = threadIdx.x - cw::EPI0;
+    const bool leader = tid == 0;
+    int fi = 0;
+    auto bwait = [&](uint64_t* bar, uint32_t parity) -> bool {
+      if (leader) epi_ok[fi] = mbar_wait(bar, parity) ? 1 : 0;
+      asm volatile("bar.sync 1, 128;" ::: "memory");
+      const bool okw = epi_ok[fi] != 0;
+      fi ^= 1;
+      return okw;
+    };
+    const int cg_n = cin / 8;           // 16-byte chunks per tap
+    const int items = 9 * cg_n * cw::KB;
+    bool ok = true;
+    for (int j = 0; j < nblk; ++j) {
+      const int s = j % cw::NS;
+      const uint32_t ph = (j / cw::NS) & 1;
+      if (!bwait(&full[s], ph)) {
+        ok = false;
+        break;
+      }
+      mbar_try_wait(&full[s], ph);  // acquire the TMA-written strip in this thread
+      const uint8_t* X = X0 + s * halo_pitch;
+      uint8_t* A = A0 + s * a_bytes;
+      for (int e = tid; e < items; e += 128) {
+        const int k = e % cw::KB, c = e / cw::KB;  // pixel of the block (fastest), chunk
+        const int t = c / cg_n, cg = c - t * cg_n;
+        const int kh = t / 3, kw = t - 3 * kh;
+        const int r = k / a.wout, ox = k - r * a.wout;
+        const int ix = ox * a.stride + kw - 1;
+        uint4 v = make_uint4(0u, 0u, 0u, 0u);
+        if (ix >= 0 && ix < a.win)
+          v = *reinterpret_cast<const uint4*>(
+              X + ((size_t)((r * a.stride + kh) * a.win + ix) * cin + cg * 8) * 2);
+        const int m = t * cin + cg * 8;
+        *reinterpret_cast<uint4*>(A + (m >> 7) * cw::kTileA + ((m >> 6) & 1) * 8192 +
+                                  (k >> 3) * 1024 + (k & 7) * 128 +
+                                  ((((m >> 3) & 7) ^ (k & 7)) << 4)) = v;
+      }
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // visible to the MMAs
+      asm volatile("bar.sync 1, 128;" ::: "memory");
+      if (leader) mbar_arrive(&aready[s]);
+    }
+    if (ok && nblk > 0 && bwait(acc_full, 0)) {
+      asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+      const int quarter = warp & 3;
+      float* out = a.part + ((int64_t)g * cpr + q) * cout * mrows;
+      for (int mt = 0; mt < mt_n; ++mt) {
+        const int m = mt * 128 + quarter * 32 + lane;
+        for (int c0 = 0; c0 < cout; c0 += 16) {
+          float v[16];
+          tmem_ld16(tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(mt * 64 + c0), v);
+          if (m < mrows) {
+#pragma unroll
+            for (int i = 0; i < 16; ++i) out[(int64_t)(c0 + i) * mrows + m] = v[i];
+          }
+        }
+      }
+    }
+  }
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+  __syncthreads();
+  if (warp == 2) {
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(tmem_cols)
+                 : "memory");
+  }
+}
+
 PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 std::once_flag g_encode_once;
 
@@ -1205,6 +1396,69 @@ bool make_tma_map_conv(CUtensorMap* map, const void* base, int ck, int win, int 
                         strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, sw,
                         CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
+}
+
+bool conv_wgrad_tc_ok(int cin, int cout, int stride, int hin, int win, int hout, int wout) {
+  if ((cin != 16 && cin != 32 && cin != 64) || cout < 16 || cout > 64 || cout % 16) return false;
+  if ((stride != 1 && stride != 2) || wout < 1 || wout > cw::KB || cw::KB % wout) return false;
+  if ((hout * wout) % cw::KB || win != wout * stride || hin != hout * stride) return false;
+  return win <= 256 && cw_rows(stride, wout) <= 256;
+}
+
+static size_t conv_wgrad_smem(int cin, int stride, int win, int wout) {
+  const int mt_n = (9 * cin + 127) / 128;
+  return 1024 + (size_t)cw::NS * ((size_t)mt_n * cw::kTileA + cw::kTileB +
+                                  cw_halo_pitch(cin, stride, win, wout)) +
+         (3 * cw::NS + 1) * 8 + 16;
+}
+
+int conv_wgrad_ctas(int cin, int stride, int wout, int G, int64_t P) {
+  const size_t smem = conv_wgrad_smem(cin, stride, wout * stride, wout);
+  const int per_sm = smem <= 113 * 1024 ? 2 : 1;
+  const int64_t blocks = P / cw::KB;
+  return (int)std::max<int64_t>(1, std::min<int64_t>(blocks, (int64_t)kNumSMs * per_sm / std::max(G, 1)));
+}
+
+bool make_tma_map_halo(CUtensorMap* map, const void* base, int cin, int win, int hin, int B, int G,
+                       int stride, int wout) {
+  std::call_once(g_encode_once, load_encode);
+  if (!g_encode || (cin != 16 && cin != 32 && cin != 64) || (reinterpret_cast<uintptr_t>(base) & 15))
+    return false;
+  const int rh = cw_rows(stride, wout);
+  if (win > 256 || rh > 256) return false;
+  const uint64_t e = 2;
+  cuuint64_t dims[5] = {(cuuint64_t)cin, (cuuint64_t)win, (cuuint64_t)hin, (cuuint64_t)B,
+                        (cuuint64_t)G};
+  cuuint64_t strides[4] = {(cuuint64_t)cin * e, (cuuint64_t)win * cin * e,
+                           (cuuint64_t)hin * win * cin * e, (cuuint64_t)B * hin * win * cin * e};
+  cuuint32_t box[5] = {(cuuint32_t)cin, (cuuint32_t)win, (cuuint32_t)rh, 1, 1};
+  cuuint32_t estr[5] = {1, 1, 1, 1, 1};
+  CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5, const_cast<void*>(base), dims,
+                        strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+cudaError_t launch_conv_wgrad_tc(const ConvWgradArgs& a, cudaStream_t stream) {
+  if (a.P <= 0 || a.G <= 0) return cudaSuccess;
+  if (!conv_wgrad_tc_ok(a.cin, a.cout, a.stride, a.hin, a.win, a.hout, a.wout) || !a.part ||
+      a.P % cw::KB || a.P % (a.hout * a.wout) || a.cpr < 1 || a.cpr > a.P / cw::KB ||
+      a.G > 65535 || (9 * a.cin + 127) / 128 > cw::MAX_MT)
+    return cudaErrorInvalidValue;
+  const size_t smem = conv_wgrad_smem(a.cin, a.stride, a.win, a.wout);
+  if (smem > 232448) return cudaErrorInvalidValue;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  static int attr_dev = -1;
+  if (attr_dev != dev) {
+    e = cudaFuncSetAttribute(conv_wgrad_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             232448);
+    if (e != cudaSuccess) return e;
+    attr_dev = dev;
+  }
+  launch_pdl(conv_wgrad_tc_kernel, dim3(a.cpr, a.G), dim3(cw::THREADS), smem, stream, a);
+  return cudaGetLastError();
 }
 
 int tc_tile_n(int Kd) { return (Kd + BK - 1) / BK <= 2 ? 128 : 64; }

@@ -149,6 +149,25 @@ struct ConvArgs {
   int64_t out_gs;
 };
 cudaError_t launch_conv_tc(const ConvArgs& a, cudaStream_t stream);
+// Weight gradient of a 3x3 convolution (zero padding 1, stride 1 or 2) on the tensor cores, the
+// column matrix built in shared memory: part[g][q][co][t Cin + ci] = the sum over CTA q's 64-pixel
+// output blocks of dy[g][p][co] x[g][src_t(p)][ci], src_t(p) the input pixel under tap t of output
+// pixel p (zero outside the image).  x_map: make_tma_map_halo over the NHWC input; dy_map: rank-3
+// bf16 map over [G][P][Cout] with box {64, 64} and a 128-byte swizzle.  Cin 16 / 32 / 64, Cout a
+// multiple of 16 up to 64, Wout dividing 64, Hout Wout a multiple of 64.
+struct ConvWgradArgs {
+  CUtensorMap x_map, dy_map;
+  int cin, cout, stride, hin, win, hout, wout, G, P;
+  int cpr;      // CTAs (partials) per replica, from conv_wgrad_ctas
+  float* part;  // [G][cpr][cout][9 cin]
+};
+bool conv_wgrad_tc_ok(int cin, int cout, int stride, int hin, int win, int hout, int wout);
+int conv_wgrad_ctas(int cin, int stride, int wout, int G, int64_t P);
+// The input strip of one 64-pixel output block: rank-5 map {Cin, Win, Hin, B, G} with box
+// {Cin, Win, rows, 1, 1}, rows = (64 / Wout - 1) stride + 3, no swizzle.
+bool make_tma_map_halo(CUtensorMap* map, const void* base, int cin, int win, int hin, int B, int G,
+                       int stride, int wout);
+cudaError_t launch_conv_wgrad_tc(const ConvWgradArgs& a, cudaStream_t stream);
 // The tile geometry of an implicit convolution with an Hout x Wout output: whole output rows,
 // 128 pixels per tile.  False when the shape does not tile that way.
 bool conv_tile_shape(int hout, int wout, int* rows, int* images);

@@ -1002,6 +1002,18 @@ bool implicit_conv_ok(int ck, int stride, int hout, int wout) {
   return (ck == 16 || ck == 32 || ck == 64) && (stride == 1 || stride == 2) &&
          conv_tile_shape(hout, wout, &rows, &images);
 }
+// The weight gradient builds its column matrix in shared memory (conv_wgrad_tc_kernel).
+bool wgrad_tc(const ResNetPlan* p, const ConvL& c) {
+  return conv_on_tc(p, c) && conv_wgrad_tc_ok(c.cin, c.cout, c.stride, c.hin, c.win, c.hout, c.wout);
+}
+// The forward reads the input straight from the activation (implicit GEMM).
+bool implicit_fwd(const ConvL& c) {
+  return implicit_conv_ok(c.cin, c.stride, c.hout, c.wout) && col_ld(c) == 9 * c.cin;
+}
+// A tensor-core convolution whose forward or weight gradient needs the column matrix in HBM.
+bool needs_col(const ResNetPlan* p, const ConvL& c) {
+  return conv_on_tc(p, c) && !(wgrad_tc(p, c) && implicit_fwd(c));
+}
 // The persistent convolution kernel: N = 16, 32 or 64 outputs, whole 128-pixel tiles.
 bool persistent_conv_ok(int n, int64_t P) { return (n == 16 || n == 32 || n == 64) && P % 128 == 0; }
 // The four-channel kernels need C a multiple of 4 with C / 4 dividing their 256 threads.
@@ -1022,7 +1034,9 @@ lsgd_status conv_forward(ResNetPlan* p, int i, const void* in, const void* Wop, 
     const int Kc = col_ld(c);
     const uint16_t* wop = reinterpret_cast<const uint16_t*>(Wop) + c.w_off;
     int64_t w_gs = p->d_pad;
-    if (Kc == 9 * c.cin) {
+    if (Kc == 9 * c.cin && !needs_col(p, c)) {
+      // neither product needs the column matrix
+    } else if (Kc == 9 * c.cin) {
       const uint16_t* in16 = reinterpret_cast<const uint16_t*>(in);
       const dim3 rows_grid((unsigned)(p->B * c.hout), (unsigned)G);
       if (c.cin == 16)
@@ -1056,7 +1070,7 @@ lsgd_status conv_forward(ResNetPlan* p, int i, const void* in, const void* Wop, 
     if (implicit_conv_ok(c.cin, c.stride, c.hout, c.wout) && Kc == 9 * c.cin &&
         persistent_conv_ok(c.cout, P)) {
       // persistent implicit GEMM: the input tile of each tap straight from the NHWC activation
-      // by TMA (the column matrix above is only kept for the weight gradient)
+      // by TMA
       ConvArgs ca{};
       bool okc = make_tma_map_conv(&ca.in_map, in, c.cin, c.win, c.hin, p->B, G, c.wout, c.hout,
                                    c.stride);
@@ -1080,7 +1094,6 @@ lsgd_status conv_forward(ResNetPlan* p, int i, const void* in, const void* Wop, 
     }
     if (implicit_conv_ok(c.cin, c.stride, c.hout, c.wout) && Kc == 9 * c.cin) {
       // implicit GEMM: the input tile of each tap straight from the NHWC activation by TMA
-      // (the column matrix above is only kept for the weight gradient)
       t.conv = 1;
       t.cv_ck = c.cin;
       t.cv_stride = c.stride;
@@ -1239,6 +1252,15 @@ lsgd_status conv_wgrad(ResNetPlan* p, int i, const void* in, float* Gr, cudaStre
   const ConvL& c = p->convs[i];
   const int K = p->K;
   const int64_t P = conv_pixels(p, c);
+  if (wgrad_tc(p, c)) {
+    // dW [Cout][9 Cin] from dy and the input directly: the column matrix of each 64-pixel block
+    // is built in shared memory; one partial per CTA, summed in order
+    RN_CALL(launch_conv_wgrad_bf16(reinterpret_cast<const uint16_t*>(in),
+                                   reinterpret_cast<const uint16_t*>(p->dy), Gr + c.w_off, p->d_pad,
+                                   K, p->B, c.hout, c.wout, c.cin, c.cout, c.stride, p->part, s));
+    ++*launches;  // the partials' sum
+    return LSGD_OK;
+  }
   if (conv_on_tc(p, c)) {
     // dW [Cout][9 Cin] = dy^T [Cout][P] x im2col(in) [P][9 Cin]: both operands pixel-major
     // ("MN-major"); the pixel reduction is split across CTAs and the partials summed in order.
@@ -1502,6 +1524,42 @@ size_t batchnorm_stats_scratch_floats(int64_t P, int C, int G) {
   return (size_t)G * nq * C * 2;
 }
 
+size_t conv_wgrad_scratch_floats(int G, int B, int hout, int wout, int cin, int cout, int stride) {
+  const int64_t P = (int64_t)B * hout * wout;
+  return (size_t)G * conv_wgrad_ctas(cin, stride, wout, G, P) * cout * 9 * cin;
+}
+
+cudaError_t launch_conv_wgrad_bf16(const uint16_t* x, const uint16_t* dy, float* dW, int64_t dW_gs,
+                                   int G, int B, int hout, int wout, int cin, int cout, int stride,
+                                   float* part, cudaStream_t s) {
+  const int hin = hout * stride, win = wout * stride;
+  const int64_t P = (int64_t)B * hout * wout;
+  if (!conv_wgrad_tc_ok(cin, cout, stride, hin, win, hout, wout) || G < 1 || B < 1 ||
+      P > 0x7fffffffLL)
+    return cudaErrorInvalidValue;
+  ConvWgradArgs a{};
+  if (!make_tma_map_halo(&a.x_map, x, cin, win, hin, B, G, stride, wout) ||
+      !make_tma_map_bf16(&a.dy_map, dy, cout, P, G, cout, (uint64_t)P * cout, 64, 64))
+    return cudaErrorInvalidValue;
+  a.cin = cin;
+  a.cout = cout;
+  a.stride = stride;
+  a.hin = hin;
+  a.win = win;
+  a.hout = hout;
+  a.wout = wout;
+  a.G = G;
+  a.P = (int)P;
+  a.cpr = conv_wgrad_ctas(cin, stride, wout, G, P);
+  a.part = part;
+  cudaError_t e = launch_conv_wgrad_tc(a, s);
+  if (e != cudaSuccess) return e;
+  // an ordinary launch: this kernel reads the partials without a grid-dependency wait
+  sum_partials_crop_kernel<<<grid_cap((int64_t)G * cout * 9 * cin, 256), 256, 0, s>>>(
+      part, a.cpr, cout, 9 * cin, 9 * cin, G, dW, dW_gs);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_batchnorm_stats(const float* y, int64_t P, int C, int G, float* mean,
                                    float* rstd, float* part, cudaStream_t s) {
   if (P < 1 || C < 1 || C > 256 || G < 1 || G > 65535) return cudaErrorInvalidValue;
@@ -1659,11 +1717,20 @@ lsgd_status resnet_alloc(ResNetPlan* p, const std::function<void*(size_t)>& allo
     part = std::max(part, (size_t)(K * nq_w * c.cout * 9 * c.cin));
     if (conv_on_tc(p, c)) {
       const int Kc = col_ld(c);
-      const int tiles = ((Kc + 63) / 64) * K;
-      const int splits = tc_valid_splits((int)P, std::max(1, (4 * kNumSMs + tiles - 1) / tiles));
-      part = std::max(part, (size_t)K * splits * c.cout * Kc);
-      p->col.push_back((uint16_t*)alloc((size_t)K * P * Kc * 2));
-      if (!p->col.back()) return LSGD_ENOMEM;
+      if (wgrad_tc(p, c)) {
+        const int cpr = conv_wgrad_ctas(c.cin, c.stride, c.wout, K, P);
+        part = std::max(part, (size_t)K * cpr * c.cout * 9 * c.cin);
+      } else {
+        const int tiles = ((Kc + 63) / 64) * K;
+        const int splits = tc_valid_splits((int)P, std::max(1, (4 * kNumSMs + tiles - 1) / tiles));
+        part = std::max(part, (size_t)K * splits * c.cout * Kc);
+      }
+      if (needs_col(p, c)) {
+        p->col.push_back((uint16_t*)alloc((size_t)K * P * Kc * 2));
+        if (!p->col.back()) return LSGD_ENOMEM;
+      } else {
+        p->col.push_back(nullptr);
+      }
       if (c.cin % 8 == 0) {
         colT = std::max(colT, (size_t)K * B * c.hin * c.win * 9 * c.cout);
         wt = std::max(wt, (size_t)K * c.cin * 9 * c.cout);

@@ -1586,6 +1586,30 @@ lsgd_status lsgd_batchnorm_stats(const float* y, int64_t P, int C, int G, float*
   return LSGD_OK;
 }
 
+lsgd_status lsgd_conv_wgrad_bf16(const uint16_t* x, const uint16_t* dy, float* dW, int G, int B,
+                                 int Hout, int Wout, int Cin, int Cout, int stride, void* stream) {
+  if (!x || !dy || !dW || G < 1 || G > 65535 || B < 1 ||
+      !lsgd::conv_wgrad_tc_ok(Cin, Cout, stride, Hout * stride, Wout * stride, Hout, Wout) ||
+      (int64_t)B * Hout * Wout > 0x7fffffffLL)
+    return fail(nullptr, LSGD_EINVAL, "lsgd_conv_wgrad_bf16: bad arguments");
+  if (((uintptr_t)x & 15) || ((uintptr_t)dy & 15))
+    return fail(nullptr, LSGD_EINVAL, "lsgd_conv_wgrad_bf16: operands must be 16-byte aligned");
+  if (!lsgd::tc_available()) return fail(nullptr, LSGD_EUNSUPPORTED, "tcgen05 not available");
+  cudaStream_t s = (cudaStream_t)stream;
+  float* part = nullptr;
+  const size_t bytes =
+      lsgd::conv_wgrad_scratch_floats(G, B, Hout, Wout, Cin, Cout, stride) * sizeof(float);
+  if (cudaMallocAsync((void**)&part, bytes, s) != cudaSuccess) {
+    cudaGetLastError();
+    return fail(nullptr, LSGD_ENOMEM, "lsgd_conv_wgrad_bf16: scratch allocation failed");
+  }
+  cudaError_t e = lsgd::launch_conv_wgrad_bf16(x, dy, dW, (int64_t)Cout * 9 * Cin, G, B, Hout, Wout,
+                                               Cin, Cout, stride, part, s);
+  cudaFreeAsync(part, s);
+  if (e != cudaSuccess) return fail_cuda(nullptr, e, "lsgd_conv_wgrad_bf16");
+  return LSGD_OK;
+}
+
 lsgd_status lsgd_sample_indices(int32_t* dst, uint64_t seed, int64_t step, int K, int B, int64_t N,
                                 void* stream) {
   if (!dst || K < 1 || B < 1 || N < K) return fail(nullptr, LSGD_EINVAL, "lsgd_sample_indices: bad arguments");

@@ -144,3 +144,63 @@ def test_resnet20_full_size_sampled_replica(P):
     assert P.lsgd_sync_count(ctx) == T // 2 + -(-(T - T // 2) // 16)
     assert P.lsgd_check_finite(ctx)
     P.lsgd_destroy(ctx)
+
+
+def _resnet_conv_segments(hwc, base, blocks, classes):
+    """(name, offset, size) of every convolution weight in the canonical parameter order: per
+    convolution its [Cout][3][3][Cin] weights, then BatchNorm gamma and beta; the classifier last."""
+    segs, off = [], 0
+
+    def conv(name, cin, cout):
+        nonlocal off
+        segs.append((name, off, cout * 9 * cin))
+        off += cout * 9 * cin + 2 * cout
+
+    conv("stem", hwc[2], base)
+    ch = base
+    for st in range(3):
+        cout = base << st
+        for b in range(blocks):
+            conv(f"s{st}b{b}a", ch, cout)
+            conv(f"s{st}b{b}b", cout, cout)
+            ch = cout
+    return segs, off + classes * ch + classes
+
+
+@pytest.mark.parametrize("hwc,B", [((32, 32, 3), 24), ((16, 16, 3), 8)])
+def test_resnet20_conv_weight_gradients_per_layer(P, hwc, B):
+    # One bf16 step from w0 with momentum 0.9 and no weight decay leaves u = the gradient, so
+    # every convolution's weight gradient is compared with the oracle's on its own.  At
+    # initialisation these gradients are differences of nearly equal BatchNorm terms, so bf16
+    # rounding alone moves them by 10-30 %: the bar is that the GPU lies closer to the oracle's
+    # bf16 gradient than the oracle's own fp32 gradient does, layer by layer (a wrong tap or
+    # channel would put it at ~100 %).  At 32 x 32 every 3 x 3 convolution but the stem builds
+    # its column matrix in shared memory; at 16 x 16 the last stage's 4 x 4 images take the
+    # column-matrix GEMM instead.
+    N, K = 96, 2
+    X, y = synthdata.gaussian_mixture(N, hwc[0] * hwc[1] * hwc[2], 10, seed=11)
+    kw = dict(hwc=hwc, base=16, blocks=3, classes=10, K=K, B=B, H=4, T=4, N=N, base_lr=0.05,
+              momentum=0.9, seed=6)
+    g, o = resnet_cfgs(P, precision=P.BF16, **kw)
+    _, o32 = resnet_cfgs(P, precision=P.FP32, **kw)
+    segs, total = _resnet_conv_segments(hwc, 16, 3, 10)
+    ctx = P.lsgd_create(g)
+    assert P.lsgd_num_params(ctx) == total
+    P.lsgd_set_dataset(ctx, X, y)
+    w0 = oracle.init_params(o).astype(np.float32)
+    P.lsgd_set_params(ctx, -1, w0)
+    P.lsgd_run(ctx, 1)
+    worst = 0.0
+    for k in range(K):
+        idx = oracle.sample_indices(o, k, 0)
+        _, grad = oracle.loss_grad(o, w0.astype(np.float64), X, y=y, idx=idx)
+        _, g32 = oracle.loss_grad(o32, w0.astype(np.float64), X, y=y, idx=idx)
+        u = P.lsgd_momentum(ctx, k).astype(np.float64)
+        assert rel_l2(u, grad) <= rel_l2(g32, grad)
+        for name, off, n in segs:
+            e = rel_l2(u[off:off + n], grad[off:off + n])
+            e_q = rel_l2(g32[off:off + n], grad[off:off + n])
+            worst = max(worst, e / e_q)
+            assert e <= e_q, (k, name, e, e_q)
+    print(f"ResNet-20 {hwc}: worst per-convolution ratio of GPU to bf16-quantisation error {worst:.2f}")
+    P.lsgd_destroy(ctx)

@@ -981,19 +981,25 @@ __global__ void __launch_bounds__(cv::THREADS, 1) conv_tc_kernel(const __grid_co
 // of pixel blocks and keeps every m-tile's 128 x 64 fp32 accumulator in TMEM; it writes its
 // partial dW, and a second kernel sums the CTAs' partials in order.  Rows m >= 9 Cin of the last
 // m-tile are never written: they only reach accumulator rows that are not stored.
-//   warp 0      TMA producer (input strip + output-gradient tile per block), NS-stage ring
+// Two rings: the small TMA inputs (strip + tile) run `ni` blocks ahead, and `na` A tiles
+// (two to four) let the builders run ahead of the MMAs.
+//   warp 0      TMA producer (input strip + output-gradient tile per block)
 //   warp 1      MMA issuer: per block and m-tile, 4 x tcgen05.mma (M = 128, N = 64, K = 16)
 //   warp 2      TMEM allocation
 //   warps 4-7   build A for each block; at the end, tcgen05.ld of the accumulators and the
 //               partial's stores
 namespace cw {
-constexpr int THREADS = 256;
-constexpr int NS = 2;       // pipeline stages
+constexpr int THREADS = 384;
+constexpr int MAX_NA = 4;   // A buffers
+constexpr int MAX_NI = 16;  // input stages
 constexpr int KB = 64;      // output pixels per block
-constexpr int EPI0 = 128;   // first builder thread
+constexpr int BUILDERS = 8; // builder warps (warps 4-11)
+constexpr int MAX_CH = 18;  // 16-byte chunks per builder thread (9 taps x Cin / 8 / 4 parts)
 constexpr int MAX_MT = 5;   // m-tiles (9 Cin <= 640)
 constexpr uint32_t kTileA = 16384;  // one m-tile of A: two 64-row atoms x 64 pixels x 128 B
 constexpr uint32_t kTileB = 8192;   // the output-gradient tile: 64 pixels x 128 B
+constexpr uint32_t kTwoPerSm = 113 * 1024;  // shared memory that still fits two CTAs on an SM
+constexpr uint32_t kOnePerSm = 224 * 1024;
 }  // namespace cw
 
 __host__ __device__ inline int cw_rows(int stride, int wout) { return (cw::KB / wout - 1) * stride + 3; }
@@ -1006,21 +1012,20 @@ __global__ void __launch_bounds__(cw::THREADS, 1) conv_wgrad_tc_kernel(
   extern __shared__ uint8_t smem_raw[];
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
-  const int cin = a.cin, cout = a.cout, mrows = 9 * cin;
+  const int cin = a.cin, cout = a.cout, mrows = 9 * cin, ni = a.ni, na = a.na;
   const int mt_n = (mrows + 127) / 128;
   const int rh = cw_rows(a.stride, a.wout);
   const uint32_t halo_bytes = (uint32_t)rh * a.win * cin * 2;
-  const uint32_t halo_pitch = cw_halo_pitch(cin, a.stride, a.win, a.wout);
+  const uint32_t in_pitch = cw_halo_pitch(cin, a.stride, a.win, a.wout) + cw::kTileB;
   const uint32_t a_bytes = (uint32_t)mt_n * cw::kTileA;
-  uint8_t* A0 = base;                              // [NS][mt_n][2][64][128 B]
-  uint8_t* B0 = A0 + cw::NS * a_bytes;             // [NS][64][128 B]
-  uint8_t* X0 = B0 + cw::NS * cw::kTileB;          // [NS][rh][Win][Cin]
-  uint64_t* full = reinterpret_cast<uint64_t*>(X0 + cw::NS * halo_pitch);
-  uint64_t* empty = full + cw::NS;
-  uint64_t* aready = empty + cw::NS;
-  uint64_t* acc_full = aready + cw::NS;
+  uint8_t* A0 = base;                          // [na][mt_n][2][64][128 B]
+  uint8_t* I0 = A0 + na * a_bytes;             // [ni]: output-gradient tile, then the strip
+  uint64_t* full_in = reinterpret_cast<uint64_t*>(I0 + ni * in_pitch);
+  uint64_t* empty_in = full_in + cw::MAX_NI;   // arrivals: the MMAs (tile), each builder (strip)
+  uint64_t* aready = empty_in + cw::MAX_NI;
+  uint64_t* afree = aready + cw::MAX_NA;
+  uint64_t* acc_full = afree + cw::MAX_NA;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(acc_full + 1);
-  int* epi_ok = reinterpret_cast<int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int g = blockIdx.y, q = blockIdx.x, cpr = gridDim.x;
@@ -1032,10 +1037,13 @@ __global__ void __launch_bounds__(cw::THREADS, 1) conv_wgrad_tc_kernel(
   while (tmem_cols < (uint32_t)mt_n * 64) tmem_cols <<= 1;
 
   if (threadIdx.x == 0) {
-    for (int i = 0; i < cw::NS; ++i) {
-      mbar_init(&full[i], 1);
-      mbar_init(&empty[i], 1);
-      mbar_init(&aready[i], 1);
+    for (int i = 0; i < ni; ++i) {
+      mbar_init(&full_in[i], 1);
+      mbar_init(&empty_in[i], 1 + cw::BUILDERS);
+    }
+    for (int i = 0; i < na; ++i) {
+      mbar_init(&aready[i], cw::BUILDERS);
+      mbar_init(&afree[i], 1);
     }
     mbar_init(acc_full, 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -1058,83 +1066,109 @@ __global__ void __launch_bounds__(cw::THREADS, 1) conv_wgrad_tc_kernel(
     // ---------------- producer ----------------
     int j = 0;
     for (; j < nblk; ++j) {
-      const int s = j % cw::NS;
-      if (!mbar_wait(&empty[s], ((j / cw::NS) & 1) ^ 1)) break;
+      const int s = j % ni;
+      if (!mbar_wait(&empty_in[s], ((j / ni) & 1) ^ 1)) break;
       const int p0 = (kb0 + j) * cw::KB;
       const int b = p0 / per_img, oy0 = (p0 % per_img) / a.wout;
-      mbar_expect_tx(&full[s], halo_bytes + cw::kTileB);
-      tma_load_5d(X0 + s * halo_pitch, &a.x_map, &full[s], 0, 0, oy0 * a.stride - 1, b, g);
-      tma_load_3d(B0 + s * cw::kTileB, &a.dy_map, &full[s], 0, p0, g);
+      uint8_t* st = I0 + s * in_pitch;
+      mbar_expect_tx(&full_in[s], halo_bytes + cw::kTileB);
+      tma_load_3d(st, &a.dy_map, &full_in[s], 0, p0, g);
+      tma_load_5d(st + cw::kTileB, &a.x_map, &full_in[s], 0, 0, oy0 * a.stride - 1, b, g);
     }
     // copies in flight land before the CTA can exit
-    for (int i = (j > cw::NS ? j - cw::NS : 0); i < j; ++i)
-      mbar_wait(&full[i % cw::NS], (i / cw::NS) & 1);
+    for (int i = (j > ni ? j - ni : 0); i < j; ++i) mbar_wait(&full_in[i % ni], (i / ni) & 1);
   } else if (warp == 1 && lane == 0) {
     // ---------------- MMA issuer ----------------
     const uint32_t idesc = make_idesc(BM, 64, true, true);
     bool ok = true;
     for (int j = 0; j < nblk; ++j) {
-      const int s = j % cw::NS;
-      const uint32_t ph = (j / cw::NS) & 1;
-      if (!mbar_wait(&aready[s], ph) || !mbar_wait(&full[s], ph)) {
+      const int s = j % ni, sa = j % na;
+      if (!mbar_wait(&aready[sa], (j / na) & 1) || !mbar_wait(&full_in[s], (j / ni) & 1)) {
         ok = false;
         break;
       }
       asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-      const uint32_t ab = smem_u32(A0 + s * a_bytes), bb = smem_u32(B0 + s * cw::kTileB);
+      const uint32_t ab = smem_u32(A0 + sa * a_bytes), bb = smem_u32(I0 + s * in_pitch);
       for (int mt = 0; mt < mt_n; ++mt)
 #pragma unroll
         for (int kk = 0; kk < cw::KB / 16; ++kk)
           mma_bf16(tmem + (uint32_t)(mt * 64), smem_desc(ab + mt * cw::kTileA + kk * 2048, 8192, 1024),
                    smem_desc(bb + kk * 2048, 8192, 1024), idesc, (j > 0 || kk > 0) ? 1u : 0u);
-      mma_commit(&empty[s]);  // stage reusable once these MMAs have read it
+      mma_commit(&afree[sa]);    // A buffer reusable once these MMAs have read it
+      mma_commit(&empty_in[s]);  // and the output-gradient tile
     }
     if (ok && nblk > 0) mma_commit(acc_full);
   } else if (warp >= 4) {
     // ---------------- builders, then the epilogue ----------------
-    const int tid = threadIdx.x - cw::EPI0;
-    const bool leader = tid == 0;
-    int fi = 0;
-    auto bwait = [&](uint64_t* bar, uint32_t parity) -> bool {
-      if (leader) epi_ok[fi] = mbar_wait(bar, parity) ? 1 : 0;
-      asm volatile("bar.sync 1, 128;" ::: "memory");
-      const bool okw = epi_ok[fi] != 0;
-      fi ^= 1;
-      return okw;
+    // Builder thread = (pixel k of the block, part p of 4): it copies chunks p, p + 4, ... of the
+    // pixel's 9 Cin / 8 sixteen-byte chunks (tap t, channels 8 cg..8 cg + 7).  Where each of them
+    // comes from in the strip and goes to in A is the same for every block, so the offsets are
+    // worked out once; per block a thread does at most MAX_CH loads and stores.  Each warp waits
+    // and signals by itself (aready and empty_in count the warps), with two warps per scheduler
+    // so that one's load latency hides behind the other's work.
+    const int bt = threadIdx.x - 128;
+    const int k = bt & (cw::KB - 1), part = bt >> 6;
+    const int cg_n = cin / 8, nchunk = 9 * cg_n;
+    const int r = k / a.wout, ox = k - r * a.wout;
+    const uint32_t swz_mask = cin == 64 ? 7u : (cin == 32 ? 3u : 1u);  // the strip's swizzle
+    uint32_t src_off[cw::MAX_CH], dst_off[cw::MAX_CH];
+    uint32_t inside = 0;
+    int nch = 0;
+#pragma unroll
+    for (int i = 0; i < cw::MAX_CH; ++i) {
+      const int c = part + 4 * i;
+      src_off[i] = dst_off[i] = 0;
+      if (c < nchunk) {
+        const int t = c / cg_n, cg = c - t * cg_n;
+        const int kh = t / 3, kw = t - 3 * kh;
+        const int ix = ox * a.stride + kw - 1;
+        if (ix >= 0 && ix < a.win) {
+          const uint32_t o = (uint32_t)(((r * a.stride + kh) * a.win + ix) * cin) * 2u + (uint32_t)cg * 16u;
+          src_off[i] = o ^ (((o >> 7) & swz_mask) << 4);
+          inside |= 1u << i;
+        }
+        const int m = t * cin + cg * 8;
+        dst_off[i] = (uint32_t)(m >> 7) * cw::kTileA + (uint32_t)((m >> 6) & 1) * 8192u +
+                     (uint32_t)(k >> 3) * 1024u + (uint32_t)(k & 7) * 128u +
+                     ((uint32_t)(((m >> 3) & 7) ^ (k & 7)) << 4);
+        nch = i + 1;
+      }
+    }
+    auto wwait = [&](uint64_t* bar, uint32_t parity) -> bool {
+      return __all_sync(0xffffffffu, mbar_wait(bar, parity) ? 1 : 0) != 0;
     };
-    const int cg_n = cin / 8;           // 16-byte chunks per tap
-    const int items = 9 * cg_n * cw::KB;
     bool ok = true;
     for (int j = 0; j < nblk; ++j) {
-      const int s = j % cw::NS;
-      const uint32_t ph = (j / cw::NS) & 1;
-      if (!bwait(&full[s], ph)) {
+      const int s = j % ni, sa = j % na;
+      if (!wwait(&full_in[s], (j / ni) & 1) || !wwait(&afree[sa], ((j / na) & 1) ^ 1)) {
         ok = false;
         break;
       }
-      mbar_try_wait(&full[s], ph);  // acquire the TMA-written strip in this thread
-      const uint8_t* X = X0 + s * halo_pitch;
-      uint8_t* A = A0 + s * a_bytes;
-      for (int e = tid; e < items; e += 128) {
-        const int k = e % cw::KB, c = e / cw::KB;  // pixel of the block (fastest), chunk
-        const int t = c / cg_n, cg = c - t * cg_n;
-        const int kh = t / 3, kw = t - 3 * kh;
-        const int r = k / a.wout, ox = k - r * a.wout;
-        const int ix = ox * a.stride + kw - 1;
-        uint4 v = make_uint4(0u, 0u, 0u, 0u);
-        if (ix >= 0 && ix < a.win)
-          v = *reinterpret_cast<const uint4*>(
-              X + ((size_t)((r * a.stride + kh) * a.win + ix) * cin + cg * 8) * 2);
-        const int m = t * cin + cg * 8;
-        *reinterpret_cast<uint4*>(A + (m >> 7) * cw::kTileA + ((m >> 6) & 1) * 8192 +
-                                  (k >> 3) * 1024 + (k & 7) * 128 +
-                                  ((((m >> 3) & 7) ^ (k & 7)) << 4)) = v;
+      const uint32_t X = smem_u32(I0 + s * in_pitch + cw::kTileB);
+      const uint32_t A = smem_u32(A0 + sa * a_bytes);
+#pragma unroll
+      for (int i = 0; i < cw::MAX_CH; ++i) {
+        if (i < nch) {
+          uint32_t v0 = 0u, v1 = 0u, v2 = 0u, v3 = 0u;
+          if (inside & (1u << i))
+            asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
+                         : "=r"(v0), "=r"(v1), "=r"(v2), "=r"(v3)
+                         : "r"(X + src_off[i])
+                         : "memory");
+          asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(A + dst_off[i]), "r"(v0),
+                       "r"(v1), "r"(v2), "r"(v3)
+                       : "memory");
+        }
       }
       asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // visible to the MMAs
-      asm volatile("bar.sync 1, 128;" ::: "memory");
-      if (leader) mbar_arrive(&aready[s]);
+      __syncwarp();
+      if (lane == 0) {
+        mbar_arrive(&aready[sa]);
+        mbar_arrive(&empty_in[s]);  // this warp has read the strip
+      }
     }
-    if (ok && nblk > 0 && bwait(acc_full, 0)) {
+    if (warp >= 8) ok = false;  // the epilogue: warps 4-7, one TMEM lane quarter each
+    if (ok && nblk > 0 && wwait(acc_full, 0)) {
       asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
       const int quarter = warp & 3;
       float* out = a.part + ((int64_t)g * cpr + q) * cout * mrows;
@@ -1405,16 +1439,35 @@ bool conv_wgrad_tc_ok(int cin, int cout, int stride, int hin, int win, int hout,
   return win <= 256 && cw_rows(stride, wout) <= 256;
 }
 
-static size_t conv_wgrad_smem(int cin, int stride, int win, int wout) {
+// Buffers and CTAs per SM of a shape.  Two A tiles; the input ring gets the rest of the shared
+// memory (deeper rings measured faster than more A tiles).  Two CTAs per SM whenever each still
+// gets three input stages: a CTA's blocks pass through a chain of handshakes one after another,
+// and a second CTA overlaps its chain with the first's.
+static void conv_wgrad_plan(int cin, int stride, int win, int wout, int* na, int* ni, int* per_sm,
+                            size_t* smem) {
   const int mt_n = (9 * cin + 127) / 128;
-  return 1024 + (size_t)cw::NS * ((size_t)mt_n * cw::kTileA + cw::kTileB +
-                                  cw_halo_pitch(cin, stride, win, wout)) +
-         (3 * cw::NS + 1) * 8 + 16;
+  const size_t bars = (2 * cw::MAX_NI + 2 * cw::MAX_NA + 1) * 8 + 16;
+  const size_t stage = cw_halo_pitch(cin, stride, win, wout) + cw::kTileB;
+  const size_t fixed = 1024 + (size_t)2 * mt_n * cw::kTileA + bars;
+  auto stages = [&](size_t budget) {
+    return budget > fixed ? (int)std::min<size_t>(cw::MAX_NI, (budget - fixed) / stage) : 0;
+  };
+  const int n2 = stages(cw::kTwoPerSm), n1 = stages(cw::kOnePerSm);
+  *na = 2;
+  if (n2 >= 3 || (n2 >= 2 && 2 * n2 >= n1)) {
+    *ni = n2;
+    *per_sm = 2;
+  } else {
+    *ni = n1;
+    *per_sm = 1;
+  }
+  *smem = *ni >= 2 ? fixed + (size_t)*ni * stage : 0;
 }
 
 int conv_wgrad_ctas(int cin, int stride, int wout, int G, int64_t P) {
-  const size_t smem = conv_wgrad_smem(cin, stride, wout * stride, wout);
-  const int per_sm = smem <= 113 * 1024 ? 2 : 1;
+  int na = 0, ni = 0, per_sm = 1;
+  size_t smem = 0;
+  conv_wgrad_plan(cin, stride, wout * stride, wout, &na, &ni, &per_sm, &smem);
   const int64_t blocks = P / cw::KB;
   return (int)std::max<int64_t>(1, std::min<int64_t>(blocks, (int64_t)kNumSMs * per_sm / std::max(G, 1)));
 }
@@ -1433,8 +1486,13 @@ bool make_tma_map_halo(CUtensorMap* map, const void* base, int cin, int win, int
                            (cuuint64_t)hin * win * cin * e, (cuuint64_t)B * hin * win * cin * e};
   cuuint32_t box[5] = {(cuuint32_t)cin, (cuuint32_t)win, (cuuint32_t)rh, 1, 1};
   cuuint32_t estr[5] = {1, 1, 1, 1, 1};
+  // each pixel's channels are one 32 / 64 / 128-byte row, swizzled at that width so that the
+  // builders' reads of neighbouring pixels spread over the banks
+  const CUtensorMapSwizzle sw = cin == 64 ? CU_TENSOR_MAP_SWIZZLE_128B
+                                          : (cin == 32 ? CU_TENSOR_MAP_SWIZZLE_64B
+                                                       : CU_TENSOR_MAP_SWIZZLE_32B);
   CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5, const_cast<void*>(base), dims,
-                        strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+                        strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, sw,
                         CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
 }
@@ -1445,8 +1503,14 @@ cudaError_t launch_conv_wgrad_tc(const ConvWgradArgs& a, cudaStream_t stream) {
       a.P % cw::KB || a.P % (a.hout * a.wout) || a.cpr < 1 || a.cpr > a.P / cw::KB ||
       a.G > 65535 || (9 * a.cin + 127) / 128 > cw::MAX_MT)
     return cudaErrorInvalidValue;
-  const size_t smem = conv_wgrad_smem(a.cin, a.stride, a.win, a.wout);
-  if (smem > 232448) return cudaErrorInvalidValue;
+  int na = 0, ni = 0, per_sm = 1;
+  size_t smem = 0;
+  conv_wgrad_plan(a.cin, a.stride, a.win, a.wout, &na, &ni, &per_sm, &smem);
+  if (ni < 2 || ni > cw::MAX_NI || na < 2 || na > cw::MAX_NA || smem > 232448)
+    return cudaErrorInvalidValue;
+  ConvWgradArgs la = a;
+  la.ni = ni;
+  la.na = na;
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
@@ -1457,7 +1521,7 @@ cudaError_t launch_conv_wgrad_tc(const ConvWgradArgs& a, cudaStream_t stream) {
     if (e != cudaSuccess) return e;
     attr_dev = dev;
   }
-  launch_pdl(conv_wgrad_tc_kernel, dim3(a.cpr, a.G), dim3(cw::THREADS), smem, stream, a);
+  launch_pdl(conv_wgrad_tc_kernel, dim3(a.cpr, a.G), dim3(cw::THREADS), smem, stream, la);
   return cudaGetLastError();
 }
 

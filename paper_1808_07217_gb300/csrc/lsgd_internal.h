@@ -160,11 +160,12 @@ struct ConvWgradArgs {
   int cin, cout, stride, hin, win, hout, wout, G, P;
   int cpr;      // CTAs (partials) per replica, from conv_wgrad_ctas
   float* part;  // [G][cpr][cout][9 cin]
+  int ni, na;   // input stages and A buffers (set by the launcher)
 };
 bool conv_wgrad_tc_ok(int cin, int cout, int stride, int hin, int win, int hout, int wout);
 int conv_wgrad_ctas(int cin, int stride, int wout, int G, int64_t P);
 // The input strip of one 64-pixel output block: rank-5 map {Cin, Win, Hin, B, G} with box
-// {Cin, Win, rows, 1, 1}, rows = (64 / Wout - 1) stride + 3, no swizzle.
+// {Cin, Win, rows, 1, 1}, rows = (64 / Wout - 1) stride + 3, swizzled at the 2 Cin-byte row.
 bool make_tma_map_halo(CUtensorMap* map, const void* base, int cin, int win, int hin, int B, int G,
                        int stride, int wout);
 cudaError_t launch_conv_wgrad_tc(const ConvWgradArgs& a, cudaStream_t stream);

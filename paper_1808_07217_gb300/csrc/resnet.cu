@@ -875,22 +875,39 @@ __global__ void pad_weights_kernel(const uint16_t* __restrict__ Wb, int64_t d_pa
 
 // Sum of split partials [g][q][rows][ldc] in split order, keeping the first `cols` columns:
 // out[g * out_gs + r cols + j].
-__global__ void sum_partials_crop_kernel(const float* __restrict__ part, int nq, int rows, int ldc,
-                                         int cols, int G, float* __restrict__ out, int64_t out_gs) {
+// out[g out_gs + r cols + j] = sum over q of part[g][q][r][j] (j < cols of ldc).  A CTA takes 32
+// consecutive outputs (one per lane); warp w sums the partials q = w, w + 8, ... (independent
+// loads, all in flight), and the eight warp sums are added in warp order: a fixed order, so the
+// result is deterministic.
+constexpr int kSumWarps = 8;
+__global__ void __launch_bounds__(32 * kSumWarps) sum_partials_crop_kernel(
+    const float* __restrict__ part, int nq, int rows, int ldc, int cols, int G,
+    float* __restrict__ out, int64_t out_gs) {
+  __shared__ float ws[kSumWarps][32];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int64_t n = (int64_t)G * rows * cols;
-  const int64_t step = (int64_t)gridDim.x * blockDim.x;
-  for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < n; t += step) {
-    const int j = (int)(t % cols);
-    const int r = (int)((t / cols) % rows);
-    const int g = (int)(t / ((int64_t)rows * cols));
+  const int64_t t = (int64_t)blockIdx.x * 32 + lane;
+  float acc = 0.f;
+  int g = 0, r = 0, j = 0;
+  if (t < n) {
+    j = (int)(t % cols);
+    r = (int)((t / cols) % rows);
+    g = (int)(t / ((int64_t)rows * cols));
     const float* p = part + (int64_t)g * nq * rows * ldc + (int64_t)r * ldc + j;
     const int64_t qs = (int64_t)rows * ldc;
-    float s = 0.f;
-#pragma unroll 8
-    for (int q = 0; q < nq; ++q) s += p[q * qs];
-    out[(int64_t)g * out_gs + (int64_t)r * cols + j] = s;
+#pragma unroll 4
+    for (int q = warp; q < nq; q += kSumWarps) acc += p[q * qs];
+  }
+  ws[warp][lane] = acc;
+  __syncthreads();
+  if (warp == 0 && t < n) {
+    float sum = 0.f;
+#pragma unroll
+    for (int w = 0; w < kSumWarps; ++w) sum += ws[w][lane];
+    out[(int64_t)g * out_gs + (int64_t)r * cols + j] = sum;
   }
 }
+unsigned sum_partials_grid(int64_t n) { return (unsigned)((n + 31) / 32); }
 
 // Weights of the stride-1 data gradient as a convolution of the output gradient:
 // wt[g][ci][t][co] = w[g][co][8 - t][ci] (taps flipped, channels transposed), bf16.
@@ -1287,7 +1304,8 @@ lsgd_status conv_wgrad(ResNetPlan* p, int i, const void* in, float* Gr, cudaStre
     t.splits = splits;
     t.epi = EPI_STORE;
     RN_CALL(launch_gemm_tc(t, s));
-    RN_LAUNCH((sum_partials_crop_kernel<<<grid_cap((int64_t)K * c.cout * 9 * c.cin, 256), 256, 0, s>>>(
+    RN_LAUNCH((sum_partials_crop_kernel<<<sum_partials_grid((int64_t)K * c.cout * 9 * c.cin),
+                                            32 * kSumWarps, 0, s>>>(
         p->part, splits, c.cout, Kc, 9 * c.cin, K, Gr + c.w_off, p->d_pad)));
     return LSGD_OK;
   }
@@ -1555,7 +1573,7 @@ cudaError_t launch_conv_wgrad_bf16(const uint16_t* x, const uint16_t* dy, float*
   cudaError_t e = launch_conv_wgrad_tc(a, s);
   if (e != cudaSuccess) return e;
   // an ordinary launch: this kernel reads the partials without a grid-dependency wait
-  sum_partials_crop_kernel<<<grid_cap((int64_t)G * cout * 9 * cin, 256), 256, 0, s>>>(
+  sum_partials_crop_kernel<<<sum_partials_grid((int64_t)G * cout * 9 * cin), 32 * kSumWarps, 0, s>>>(
       part, a.cpr, cout, 9 * cin, 9 * cin, G, dW, dW_gs);
   return cudaGetLastError();
 }

@@ -49,8 +49,9 @@ FUSED_UPDATE_BYTES_PER_PARAM = 18
 AVERAGE_BYTES_PER_PARAM = 10
 # DRAM bytes (read + write) per step of the update launches (the classifier head's backward and
 # the weight-gradient + update launch of both hidden layers), from the ncu capture summarised in
-# profiles/wgrad_update_mlp3072_K16_B128.md; None until that capture matches the current kernels.
-UPDATE_TRAFFIC_PER_STEP = None
+# profiles/step_kernels_mlp3072_K16_B128.md (below the algorithmic bytes because part of the
+# launch's writes is still in L2 when it ends).
+UPDATE_TRAFFIC_PER_STEP = 1186162688
 
 FALLBACK_HBM_GBS = 6800.0
 FALLBACK_BF16_TFLOPS = 1900.0

@@ -120,6 +120,38 @@ def test_pipelined_host_batches_equal_sampled_steps(P):
     P.lsgd_destroy(b)
 
 
+def test_set_step_restarts_the_schedule(P):
+    # A job run to its end, then lsgd_set_step(0) and three more steps, equals a fresh context
+    # given the end state (parameters and momentum) and run three steps from step 0: the step
+    # counter alone decides learning rate, sampled mini-batches and round ends.
+    g, o, X, y = _small(P, P.BF16, T=7, H=3)
+    a = P.lsgd_create(g)
+    P.lsgd_set_dataset(a, X, y)
+    P.lsgd_run(a, 7)
+    assert P.lsgd_step_count(a) == 7 and P.lsgd_sync_count(a) == 3
+    W = [P.lsgd_params(a, k) for k in range(4)]
+    U = [P.lsgd_momentum(a, k) for k in range(4)]
+    P.lsgd_set_step(a, 0)
+    assert P.lsgd_step_count(a) == 0
+    P.lsgd_run(a, 3)
+    c = P.lsgd_create(g)
+    P.lsgd_set_dataset(c, X, y)
+    for k in range(4):
+        P.lsgd_set_params(c, k, W[k])
+        P.lsgd_set_momentum(c, k, U[k])
+    P.lsgd_run(c, 3)
+    for k in range(4):
+        assert np.array_equal(P.lsgd_params(a, k), P.lsgd_params(c, k))
+        assert np.array_equal(P.lsgd_momentum(a, k), P.lsgd_momentum(c, k))
+    assert np.array_equal(P.lsgd_losses(a, 3, 4), P.lsgd_losses(c, 3, 4))
+    assert P.lsgd_sync_count(a) == 3 + P.lsgd_sync_count(c) == 4
+    for bad in (-1, 8):
+        with pytest.raises(P.LsgdError):
+            P.lsgd_set_step(a, bad)
+    P.lsgd_destroy(a)
+    P.lsgd_destroy(c)
+
+
 def test_sync_counts_follow_schedule(P):
     for T, H, tp in [(49, 16, -1), (25, 16, 12), (10, 3, 0), (9, 4, 20)]:
         g, o, X, y = _small(P, P.BF16, T=T, H=H, t_switch=tp)

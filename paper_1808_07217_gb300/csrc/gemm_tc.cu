@@ -830,9 +830,9 @@ __global__ void __launch_bounds__(cv::THREADS, 1) conv_tc_kernel(const __grid_co
   // a stage holds the three taps of one kernel row (kh): three TMA boxes, one handshake
   const uint32_t tap_bytes = (uint32_t)BM * ck * 2;
   const uint32_t stage_bytes = 3 * tap_bytes;
-  const int nst = min(cv::MAX_STAGES, cv::RING_BYTES / (int)stage_bytes);
+  const int nst = min(cv::MAX_STAGES, a.ring_bytes / (int)stage_bytes);
   uint8_t* ring = base;
-  uint8_t* wsm = base + cv::RING_BYTES;
+  uint8_t* wsm = base + a.ring_bytes;
   const uint32_t wtap = (uint32_t)np * ck * 2;  // bytes of one tap's weights
   uint64_t* bars = reinterpret_cast<uint64_t*>(wsm + 9 * wtap);
   uint64_t* full = bars;
@@ -1342,8 +1342,21 @@ cudaError_t launch_conv_tc(const ConvArgs& a, cudaStream_t stream) {
   cudaError_t e = cudaGetDevice(&dev);
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   if (e != cudaSuccess) return e;
-  const size_t smem = 1024 + cv::RING_BYTES + 9 * (size_t)a.np * a.ck * 2 +
-                      (2 * cv::MAX_STAGES + 5) * 8 + 16;
+  // Two CTAs per SM where the weights leave room for a ring of at least three stages (a CTA's
+  // tiles pass through a chain of handshakes one after another; two CTAs overlap their chains),
+  // else one CTA with the full ring.
+  const size_t fixed = 1024 + 9 * (size_t)a.np * a.ck * 2 + (2 * cv::MAX_STAGES + 5) * 8 + 16;
+  const size_t stage_bytes = 3 * (size_t)BM * a.ck * 2;
+  const size_t two_budget = 113 * 1024;
+  size_t ring = cv::RING_BYTES;
+  int per_sm = 1;
+  if (two_budget > fixed && (two_budget - fixed) / stage_bytes >= 3) {
+    ring = std::min<size_t>(cv::RING_BYTES, ((two_budget - fixed) / 1024) * 1024);
+    per_sm = 2;
+  }
+  const size_t smem = fixed + ring;
+  ConvArgs la = a;
+  la.ring_bytes = (int)ring;
   static int attr_dev = -1;
   if (attr_dev != dev) {
     e = cudaFuncSetAttribute(conv_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -1353,8 +1366,8 @@ cudaError_t launch_conv_tc(const ConvArgs& a, cudaStream_t stream) {
   }
   // CTAs per replica: about one per SM over all replicas, at most one per tile
   const int tiles = a.P / BM;
-  const int cpr = std::max(1, std::min(tiles, (sms + a.G - 1) / a.G));
-  return launch_pdl(conv_tc_kernel, dim3(cpr, a.G), dim3(cv::THREADS), smem, stream, a);
+  const int cpr = std::max(1, std::min(tiles, (per_sm * sms + a.G - 1) / a.G));
+  return launch_pdl(conv_tc_kernel, dim3(cpr, a.G), dim3(cv::THREADS), smem, stream, la);
 }
 
 cudaError_t launch_wgrad_update(const WgradUpdateArgs& a, cudaStream_t stream) {

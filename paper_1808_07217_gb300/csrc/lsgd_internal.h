@@ -147,6 +147,7 @@ struct ConvArgs {
   int ck, stride, hout, wout, N, np, G, P;
   float* out;
   int64_t out_gs;
+  int ring_bytes;  // input ring size (set by the launcher)
 };
 cudaError_t launch_conv_tc(const ConvArgs& a, cudaStream_t stream);
 // Weight gradient of a 3x3 convolution (zero padding 1, stride 1 or 2) on the tensor cores, the

@@ -1461,20 +1461,25 @@ static void conv_wgrad_plan(int cin, int stride, int win, int wout, int* na, int
   const int mt_n = (9 * cin + 127) / 128;
   const size_t bars = (2 * cw::MAX_NI + 2 * cw::MAX_NA + 1) * 8 + 16;
   const size_t stage = cw_halo_pitch(cin, stride, win, wout) + cw::kTileB;
-  const size_t fixed = 1024 + (size_t)2 * mt_n * cw::kTileA + bars;
-  auto stages = [&](size_t budget) {
-    return budget > fixed ? (int)std::min<size_t>(cw::MAX_NI, (budget - fixed) / stage) : 0;
+  auto fixed = [&](int nA) { return 1024 + (size_t)nA * mt_n * cw::kTileA + bars; };
+  auto stages = [&](int nA, size_t budget) {
+    return budget > fixed(nA) ? (int)std::min<size_t>(cw::MAX_NI, (budget - fixed(nA)) / stage) : 0;
   };
-  const int n2 = stages(cw::kTwoPerSm), n1 = stages(cw::kOnePerSm);
+  const int n2 = stages(2, cw::kTwoPerSm), n1 = stages(2, cw::kOnePerSm);
+  const int n2s = stages(1, cw::kTwoPerSm);  // one A tile: builders and MMAs take turns
   *na = 2;
   if (n2 >= 3 || (n2 >= 2 && 2 * n2 >= n1)) {
     *ni = n2;
+    *per_sm = 2;
+  } else if (n2s >= 3) {
+    *na = 1;
+    *ni = n2s;
     *per_sm = 2;
   } else {
     *ni = n1;
     *per_sm = 1;
   }
-  *smem = *ni >= 2 ? fixed + (size_t)*ni * stage : 0;
+  *smem = *ni >= 2 ? fixed(*na) + (size_t)*ni * stage : 0;
 }
 
 int conv_wgrad_ctas(int cin, int stride, int wout, int G, int64_t P) {
@@ -1519,7 +1524,7 @@ cudaError_t launch_conv_wgrad_tc(const ConvWgradArgs& a, cudaStream_t stream) {
   int na = 0, ni = 0, per_sm = 1;
   size_t smem = 0;
   conv_wgrad_plan(a.cin, a.stride, a.win, a.wout, &na, &ni, &per_sm, &smem);
-  if (ni < 2 || ni > cw::MAX_NI || na < 2 || na > cw::MAX_NA || smem > 232448)
+  if (ni < 2 || ni > cw::MAX_NI || na < 1 || na > cw::MAX_NA || smem > 232448)
     return cudaErrorInvalidValue;
   ConvWgradArgs la = a;
   la.ni = ni;

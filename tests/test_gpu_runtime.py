@@ -120,6 +120,37 @@ def test_pipelined_host_batches_equal_sampled_steps(P):
     P.lsgd_destroy(b)
 
 
+def test_least_squares_host_batches_equal_sampled_steps(P):
+    # Targets (fp32) instead of labels travel through the same staging buffers.
+    import torch
+
+    N, dd, K, B = 256, 20, 4, 16
+    A, t, _ = synthdata.least_squares(N, dd, seed=3)
+    g, o = dense_cfgs(P, widths=(dd, 1), K=K, B=B, H=3, T=6, N=N, precision=P.FP32, kind="lsq",
+                      base_lr=0.02, seed=5, init="zero")
+    a = P.lsgd_create(g)
+    P.lsgd_set_targets(a, A, t)
+    b = P.lsgd_create(g)
+    P.lsgd_set_targets(b, A, t)
+    batches = []
+    for s in range(6):
+        idx = P.lsgd_debug_indices(b, s, K, B).reshape(-1)
+        batches.append((torch.from_numpy(A[idx].reshape(K, B, -1).copy()).pin_memory(),
+                        torch.from_numpy(t[idx].reshape(K, B).copy()).pin_memory()))
+    for s in range(6):
+        P.lsgd_local_step(a)
+        P.lsgd_local_step_batch(b, *batches[s])
+        if (s + 1) % 3 == 0:
+            P.lsgd_sync_average(a)
+            P.lsgd_sync_average(b)
+    P.lsgd_synchronize(b)
+    for k in range(K):
+        assert np.array_equal(P.lsgd_params(a, k), P.lsgd_params(b, k))
+    assert np.array_equal(P.lsgd_losses(a, 6, K), P.lsgd_losses(b, 6, K))
+    P.lsgd_destroy(a)
+    P.lsgd_destroy(b)
+
+
 def test_set_step_restarts_the_schedule(P):
     # A job run to its end, then lsgd_set_step(0) and three more steps, equals a fresh context
     # given the end state (parameters and momentum) and run three steps from step 0: the step

@@ -12,6 +12,9 @@
 // Reductions over the pixels of a replica (BatchNorm statistics, their backward sums, weight
 // gradients) run in two deterministic passes: per-chunk partial results into a scratch buffer,
 // then a fixed-order combination.
+//
+// Every kernel here starts with the programmatic grid-dependency wait and is launched with
+// programmatic dependent launch, so the next kernel's launch and prologue overlap this one's tail.
 #include <algorithm>
 #include <cmath>
 #include <cstdlib>
@@ -59,6 +62,7 @@ __global__ void __launch_bounds__(128) conv_fwd_kernel(const TA* __restrict__ in
                                                        float* __restrict__ y, int B, int Hin,
                                                        int Win, int Cin, int Hout, int Wout,
                                                        int Cout, int stride) {
+  pdl_begin();
   extern __shared__ float ws[];  // [16][9][Cin]
   const int g = blockIdx.z, co0 = blockIdx.y * 16;
   const int nco = min(16, Cout - co0);
@@ -107,6 +111,7 @@ __global__ void __launch_bounds__(64) conv_dgrad_kernel(
     const TA* __restrict__ dy, const TA* __restrict__ w, int64_t w_gs, float* __restrict__ dx,
     int B, int Hin, int Win, int Cin, int Hout, int Wout, int Cout, int stride,
     const float* __restrict__ dout, const TA* __restrict__ out_act) {
+  pdl_begin();
   extern __shared__ float ws[];  // [Cout][9][16]
   const int g = blockIdx.z, ci0 = blockIdx.y * 16;
   const int nci = min(16, Cin - ci0);
@@ -161,6 +166,7 @@ template <typename TA>
 __global__ void __launch_bounds__(256) conv_wgrad_partial_kernel(
     const TA* __restrict__ dy, const TA* __restrict__ in, float* __restrict__ part, int B, int Hin,
     int Win, int Cin, int Hout, int Wout, int Cout, int stride, int nq) {
+  pdl_begin();
   extern __shared__ float sm[];
   const int J = 9 * Cin;
   float* dys = sm;                     // [kWgradTile][16]
@@ -219,6 +225,7 @@ __global__ void __launch_bounds__(256) conv_wgrad_partial_kernel(
 // Weight gradient, pass 2: G[g][w_off + e] = sum_q part[g][q][e] in chunk order.
 __global__ void sum_partials_kernel(const float* __restrict__ part, int nq, int64_t n, int G,
                                     float* __restrict__ out, int64_t out_gs) {
+  pdl_begin();
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < (int64_t)G * n; t += stride) {
     const int g = (int)(t / n);
@@ -235,6 +242,7 @@ __global__ void sum_partials_kernel(const float* __restrict__ part, int nq, int6
 __global__ void __launch_bounds__(256) bn_stats_partial_kernel(const float* __restrict__ y,
                                                                int64_t P, int C, int nq, int chunk,
                                                                float* __restrict__ part) {
+  pdl_begin();
   __shared__ float red[256];
   __shared__ float mean_s[256];
   const int g = blockIdx.y, q = blockIdx.x;
@@ -295,6 +303,7 @@ __global__ void __launch_bounds__(256) bn_stats_partial_v4_kernel(const float* _
                                                                   int64_t P, int C, int nq,
                                                                   int chunk,
                                                                   float* __restrict__ part) {
+  pdl_begin();
   __shared__ float4 red[256];
   const int g = blockIdx.y, q = blockIdx.x;
   const int C4 = C / 4, lanes = blockDim.x / C4;
@@ -362,6 +371,7 @@ __device__ __forceinline__ void chan_merge(float& n, float& mu, float& M2, float
 __global__ void bn_stats_finalize_kernel(const float* __restrict__ part, int64_t P, int C, int nq,
                                          int chunk, int G, float* __restrict__ mean,
                                          float* __restrict__ rstd) {
+  pdl_begin();
   const int wid = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
   if (wid >= G * C) return;
   const int g = wid / C, c = wid % C;
@@ -430,6 +440,7 @@ __global__ void bn_act_fwd_kernel(const float* __restrict__ y, const float* __re
                                   const TA* __restrict__ sc, int sc_H, int sc_W, int sc_C,
                                   int stride, TA* __restrict__ out, int G, int B, int H, int Wd,
                                   int C) {
+  pdl_begin();
   const int C4 = C / 4;
   const int P = B * H * Wd;
   const int n4 = G * P * C4;
@@ -469,6 +480,7 @@ __global__ void __launch_bounds__(256) bn_act_fwd_v4_kernel(
     const float* __restrict__ W, int64_t g_off, int64_t b_off, int64_t d_gs, int w_g0, int w_gmul,
     const TA* __restrict__ sc, int sc_H, int sc_W, int sc_C, int stride, TA* __restrict__ out, int B,
     int H, int Wd, int C) {
+  pdl_begin();
   const int g = blockIdx.y, C4 = C / 4;
   const int c0 = (threadIdx.x % C4) * 4, pl = threadIdx.x / C4, ppb = blockDim.x / C4;
   const int P = B * H * Wd;
@@ -511,6 +523,7 @@ __global__ void __launch_bounds__(256) bn_bwd_partial_kernel(
     const float* __restrict__ dout, const TA* __restrict__ out, const float* __restrict__ y,
     const float* __restrict__ mean, const float* __restrict__ rstd, int64_t P, int C, int nq,
     int chunk, float* __restrict__ part) {
+  pdl_begin();
   __shared__ float r1[256], r2[256];
   const int g = blockIdx.y, q = blockIdx.x;
   const int lanes = blockDim.x / C;
@@ -549,6 +562,7 @@ __global__ void __launch_bounds__(256) bn_bwd_partial_v4_kernel(
     const float* __restrict__ dout, const TA* __restrict__ out, const float* __restrict__ y,
     const float* __restrict__ mean, const float* __restrict__ rstd, int64_t P, int C, int nq,
     int chunk, float* __restrict__ part) {
+  pdl_begin();
   __shared__ float4 r1[256], r2[256];
   const int g = blockIdx.y, q = blockIdx.x;
   const int C4 = C / 4, lanes = blockDim.x / C4;
@@ -618,6 +632,7 @@ __global__ void __launch_bounds__(256) bn_bwd_partial_v4_kernel(
 __global__ void bn_bwd_finalize_kernel(const float* __restrict__ part, int C, int nq, int G,
                                        float* __restrict__ s12, float* __restrict__ Gr,
                                        int64_t g_off, int64_t b_off, int64_t d_gs) {
+  pdl_begin();
   const int wid = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
   if (wid >= G * C) return;
   const int g = wid / C, c = wid % C;
@@ -648,6 +663,7 @@ __global__ void bn_bwd_apply_kernel(const float* __restrict__ dout, const TA* __
                                     const float* __restrict__ rstd, const float* __restrict__ s12,
                                     const float* __restrict__ W, int64_t g_off, int64_t d_gs,
                                     TA* __restrict__ dy, int G, int64_t P64, int C) {
+  pdl_begin();
   const int C4 = C / 4;
   const int P = (int)P64;
   const int n4 = G * P * C4;
@@ -680,6 +696,7 @@ __global__ void __launch_bounds__(256) bn_bwd_apply_v4_kernel(
     const float* __restrict__ dout, const TA* __restrict__ out, const float* __restrict__ y,
     const float* __restrict__ mean, const float* __restrict__ rstd, const float* __restrict__ s12,
     const float* __restrict__ W, int64_t g_off, int64_t d_gs, TA* __restrict__ dy, int P, int C) {
+  pdl_begin();
   const int g = blockIdx.y, C4 = C / 4;
   const int c0 = (threadIdx.x % C4) * 4, pl = threadIdx.x / C4, ppb = blockDim.x / C4;
   const float invM = 1.0f / (float)P;
@@ -716,6 +733,7 @@ __global__ void __launch_bounds__(256) bn_bwd_apply_v4_kernel(
 template <typename TA>
 __global__ void avgpool_kernel(const TA* __restrict__ act, float* __restrict__ feat, int GB, int HW,
                                int F) {
+  pdl_begin();
   const int t = blockIdx.x * blockDim.x + threadIdx.x;
   if (t >= GB * F) return;
   const int gb = t / F, f = t % F;
@@ -728,6 +746,7 @@ __global__ void avgpool_kernel(const TA* __restrict__ act, float* __restrict__ f
 // dact[g][b][p][f] = dfeat[g][b][f] / HW (gradient of the average pooling).
 __global__ void avgpool_bwd_kernel(const float* __restrict__ dfeat, float* __restrict__ dact,
                                    int64_t n, int HW, int F) {
+  pdl_begin();
   const int64_t step = (int64_t)gridDim.x * blockDim.x;
   for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < n; e += step) {
     const int f = (int)(e % F);
@@ -744,6 +763,7 @@ __global__ void __launch_bounds__(256) im2col_v2_kernel(const uint16_t* __restri
                                                         uint16_t* __restrict__ col, int B, int Hin,
                                                         int Win, int Cin, int Hout, int Wout,
                                                         int stride) {
+  pdl_begin();
   const int g = blockIdx.y, c8n = Cin / 8, R = 9 * c8n;
   const int P = B * Hout * Wout;
   const int e = blockIdx.x * blockDim.x + threadIdx.x;
@@ -765,6 +785,7 @@ template <int C8N>
 __global__ void __launch_bounds__(256) im2col_row_kernel(const uint16_t* __restrict__ in,
                                                          uint16_t* __restrict__ col, int B, int Hin,
                                                          int Win, int Hout, int Wout, int stride) {
+  pdl_begin();
   constexpr int Cin = 8 * C8N, R = 9 * C8N;
   const int g = blockIdx.y, row = blockIdx.x;
   const int oh = row % Hout, b = row / Hout;
@@ -789,6 +810,7 @@ __global__ void __launch_bounds__(256) im2col_any_row_kernel(const TA* __restric
                                                              uint16_t* __restrict__ col, int B,
                                                              int Hin, int Win, int Cin, int Hout,
                                                              int Wout, int stride, int ldc) {
+  pdl_begin();
   const int g = blockIdx.y, row = blockIdx.x;
   const int oh = row % Hout, b = row / Hout;
   const int64_t P = (int64_t)B * Hout * Wout;
@@ -817,6 +839,7 @@ __global__ void __launch_bounds__(256) col_dgrad_v2_kernel(const uint16_t* __res
                                                            uint16_t* __restrict__ col, int B, int Hin,
                                                            int Win, int Cout, int Hout, int Wout,
                                                            int stride) {
+  pdl_begin();
   const int g = blockIdx.y, c8n = Cout / 8, R = 9 * c8n;
   const int P = B * Hin * Win;
   const int e = blockIdx.x * blockDim.x + threadIdx.x;
@@ -840,6 +863,7 @@ __global__ void __launch_bounds__(256) col_dgrad_row_kernel(const uint16_t* __re
                                                             uint16_t* __restrict__ col, int B,
                                                             int Hin, int Win, int Hout, int Wout,
                                                             int stride) {
+  pdl_begin();
   constexpr int Cout = 8 * C8N, R = 9 * C8N;
   const int g = blockIdx.y, row = blockIdx.x;
   const int ih = row % Hin, b = row / Hin;
@@ -863,6 +887,7 @@ __global__ void __launch_bounds__(256) col_dgrad_row_kernel(const uint16_t* __re
 // operand (9 Cin = 27 is not a multiple of 8).
 __global__ void pad_weights_kernel(const uint16_t* __restrict__ Wb, int64_t d_pad, int64_t w_off,
                                    uint16_t* __restrict__ out, int G, int rows, int cols, int ldc) {
+  pdl_begin();
   const int64_t n = (int64_t)G * rows * ldc;
   const int64_t step = (int64_t)gridDim.x * blockDim.x;
   for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < n; e += step) {
@@ -883,6 +908,7 @@ constexpr int kSumWarps = 8;
 __global__ void __launch_bounds__(32 * kSumWarps) sum_partials_crop_kernel(
     const float* __restrict__ part, int nq, int rows, int ldc, int cols, int G,
     float* __restrict__ out, int64_t out_gs) {
+  pdl_begin();
   __shared__ float ws[kSumWarps][32];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int64_t n = (int64_t)G * rows * cols;
@@ -913,6 +939,7 @@ unsigned sum_partials_grid(int64_t n) { return (unsigned)((n + 31) / 32); }
 // wt[g][ci][t][co] = w[g][co][8 - t][ci] (taps flipped, channels transposed), bf16.
 __global__ void flip_weights_kernel(const uint16_t* __restrict__ Wb, int64_t d_pad, int64_t w_off,
                                     uint16_t* __restrict__ wt, int G, int Cin, int Cout) {
+  pdl_begin();
   // blockIdx.y = replica; 32-bit indexing within it (Cin 9 Cout < 2^31)
   const int g = blockIdx.y, n = Cin * 9 * Cout;
   const uint16_t* src = Wb + (int64_t)g * d_pad + w_off;
@@ -930,6 +957,7 @@ template <typename TA>
 __global__ void __launch_bounds__(256) add_shortcut_grad_v2_kernel(
     float* __restrict__ dx, const float* __restrict__ dout, const TA* __restrict__ out, int B,
     int Hin, int Win, int Cin, int Hout, int Wout, int Cout, int stride) {
+  pdl_begin();
   const int g = blockIdx.y, C4 = Cin / 4;
   const int Po = B * Hout * Wout;
   const int e = blockIdx.x * blockDim.x + threadIdx.x;
@@ -1057,25 +1085,26 @@ lsgd_status conv_forward(ResNetPlan* p, int i, const void* in, const void* Wop, 
       const uint16_t* in16 = reinterpret_cast<const uint16_t*>(in);
       const dim3 rows_grid((unsigned)(p->B * c.hout), (unsigned)G);
       if (c.cin == 16)
-        RN_LAUNCH((im2col_row_kernel<2><<<rows_grid, 256, 0, s>>>(in16, p->col[i], p->B, c.hin, c.win,
-                                                                  c.hout, c.wout, c.stride)));
+        RN_LAUNCH((launch_pdl(im2col_row_kernel<2>, rows_grid, 256, 0, s, in16, p->col[i], p->B,
+            c.hin, c.win, c.hout, c.wout, c.stride)));
       else if (c.cin == 32)
-        RN_LAUNCH((im2col_row_kernel<4><<<rows_grid, 256, 0, s>>>(in16, p->col[i], p->B, c.hin, c.win,
-                                                                  c.hout, c.wout, c.stride)));
+        RN_LAUNCH((launch_pdl(im2col_row_kernel<4>, rows_grid, 256, 0, s, in16, p->col[i], p->B,
+            c.hin, c.win, c.hout, c.wout, c.stride)));
       else if (c.cin == 64)
-        RN_LAUNCH((im2col_row_kernel<8><<<rows_grid, 256, 0, s>>>(in16, p->col[i], p->B, c.hin, c.win,
-                                                                  c.hout, c.wout, c.stride)));
+        RN_LAUNCH((launch_pdl(im2col_row_kernel<8>, rows_grid, 256, 0, s, in16, p->col[i], p->B,
+            c.hin, c.win, c.hout, c.wout, c.stride)));
       else
-        RN_LAUNCH((im2col_v2_kernel<<<dim3((unsigned)((P * 9 * (c.cin / 8) + 255) / 256), (unsigned)G),
-                                        256, 0, s>>>(in16, p->col[i], p->B, c.hin, c.win, c.cin,
-                                                     c.hout, c.wout, c.stride)));
+        RN_LAUNCH((launch_pdl(im2col_v2_kernel,
+            dim3((unsigned)((P * 9 * (c.cin / 8) + 255) / 256), (unsigned)G), 256, 0, s, in16,
+            p->col[i], p->B, c.hin, c.win, c.cin, c.hout, c.wout, c.stride)));
     } else {
-      RN_LAUNCH((im2col_any_row_kernel<uint16_t><<<dim3((unsigned)(p->B * c.hout), (unsigned)G), 256,
-                                                   0, s>>>(reinterpret_cast<const uint16_t*>(in),
-                                                           p->col[i], p->B, c.hin, c.win, c.cin,
-                                                           c.hout, c.wout, c.stride, Kc)));
-      RN_LAUNCH((pad_weights_kernel<<<grid_for_items((int64_t)G * c.cout * Kc), 256, 0, s>>>(
-          reinterpret_cast<const uint16_t*>(Wop), p->d_pad, c.w_off, p->wt, G, c.cout, 9 * c.cin, Kc)));
+      RN_LAUNCH((launch_pdl(im2col_any_row_kernel<uint16_t>,
+          dim3((unsigned)(p->B * c.hout), (unsigned)G), 256, 0, s,
+          reinterpret_cast<const uint16_t*>(in), p->col[i], p->B, c.hin, c.win, c.cin, c.hout,
+          c.wout, c.stride, Kc)));
+      RN_LAUNCH((launch_pdl(pad_weights_kernel, grid_for_items((int64_t)G * c.cout * Kc), 256, 0, s,
+          reinterpret_cast<const uint16_t*>(Wop), p->d_pad, c.w_off, p->wt, G, c.cout, 9 * c.cin,
+          Kc)));
       wop = p->wt;
       w_gs = (int64_t)c.cout * Kc;
     }
@@ -1152,9 +1181,9 @@ lsgd_status conv_forward(ResNetPlan* p, int i, const void* in, const void* Wop, 
   dim3 grid((unsigned)((P + 127) / 128), (unsigned)((c.cout + 15) / 16), (unsigned)G);
   const size_t smem = (size_t)16 * 9 * c.cin * 4;
   const TA* wbase = reinterpret_cast<const TA*>(Wop) + (int64_t)w_g0 * p->d_pad + c.w_off;
-  RN_LAUNCH((conv_fwd_kernel<TA><<<grid, 128, smem, s>>>(
-      reinterpret_cast<const TA*>(in), wbase, (int64_t)w_gmul * p->d_pad, y, p->B, c.hin, c.win,
-      c.cin, c.hout, c.wout, c.cout, c.stride)));
+  RN_LAUNCH((launch_pdl(conv_fwd_kernel<TA>, grid, 128, smem, s, reinterpret_cast<const TA*>(in),
+      wbase, (int64_t)w_gmul * p->d_pad, y, p->B, c.hin, c.win, c.cin, c.hout, c.wout, c.cout,
+      c.stride)));
   return LSGD_OK;
 }
 
@@ -1166,12 +1195,13 @@ lsgd_status bn_stats(ResNetPlan* p, const ConvL& c, const float* y, float* mean,
   const int lanes = std::max(1, 256 / c.cout);
   dim3 grid(nq, G);
   if (vec4_ok(c.cout))
-    RN_LAUNCH((bn_stats_partial_v4_kernel<<<grid, 256, 0, s>>>(y, P, c.cout, nq, chunk, p->part)));
+    RN_LAUNCH((launch_pdl(bn_stats_partial_v4_kernel, grid, 256, 0, s, y, P, c.cout, nq, chunk,
+        p->part)));
   else
-    RN_LAUNCH((bn_stats_partial_kernel<<<grid, lanes * c.cout, 0, s>>>(y, P, c.cout, nq, chunk,
-                                                                       p->part)));
-  RN_LAUNCH((bn_stats_finalize_kernel<<<(G * c.cout * 32 + 127) / 128, 128, 0, s>>>(
-      p->part, P, c.cout, nq, chunk, G, mean, rstd)));
+    RN_LAUNCH((launch_pdl(bn_stats_partial_kernel, grid, lanes * c.cout, 0, s, y, P, c.cout, nq,
+        chunk, p->part)));
+  RN_LAUNCH((launch_pdl(bn_stats_finalize_kernel, (G * c.cout * 32 + 127) / 128, 128, 0, s, p->part,
+      P, c.cout, nq, chunk, G, mean, rstd)));
   return LSGD_OK;
 }
 
@@ -1191,23 +1221,21 @@ lsgd_status forward_impl(ResNetPlan* p, const float* W, const void* Wop, int w_g
     const TA* sc = second ? reinterpret_cast<const TA*>(p->act[i - 2]) : nullptr;
     const ConvL& ca = p->convs[second ? i - 1 : i];
     if (vec4_ok(c.cout)) {
-      RN_LAUNCH((bn_act_fwd_v4_kernel<TA><<<dim3(px_blocks(conv_pixels(p, c), c.cout), (unsigned)G),
-                                             256, 0, s>>>(
-          p->y[i], p->mean[i], p->rstd[i], W, c.g_off, c.b_off, p->d_pad, w_g0, w_gmul, sc, ca.hin,
-          ca.win, ca.cin, ca.stride, reinterpret_cast<TA*>(p->act[i]), p->B, c.hout, c.wout,
-          c.cout)));
+      RN_LAUNCH((launch_pdl(bn_act_fwd_v4_kernel<TA>,
+          dim3(px_blocks(conv_pixels(p, c), c.cout), (unsigned)G), 256, 0, s, p->y[i], p->mean[i],
+          p->rstd[i], W, c.g_off, c.b_off, p->d_pad, w_g0, w_gmul, sc, ca.hin, ca.win, ca.cin,
+          ca.stride, reinterpret_cast<TA*>(p->act[i]), p->B, c.hout, c.wout, c.cout)));
     } else {
       const int64_t n = (int64_t)G * conv_pixels(p, c) * c.cout / 4;
-      RN_LAUNCH((bn_act_fwd_kernel<TA><<<grid_cap(n, 256), 256, 0, s>>>(
-          p->y[i], p->mean[i], p->rstd[i], W, c.g_off, c.b_off, p->d_pad, w_g0, w_gmul, sc, ca.hin,
-          ca.win, ca.cin, ca.stride, reinterpret_cast<TA*>(p->act[i]), G, p->B, c.hout, c.wout,
-          c.cout)));
+      RN_LAUNCH((launch_pdl(bn_act_fwd_kernel<TA>, grid_cap(n, 256), 256, 0, s, p->y[i], p->mean[i],
+          p->rstd[i], W, c.g_off, c.b_off, p->d_pad, w_g0, w_gmul, sc, ca.hin, ca.win, ca.cin,
+          ca.stride, reinterpret_cast<TA*>(p->act[i]), G, p->B, c.hout, c.wout, c.cout)));
     }
   }
   // global average pooling and the classifier (fp32)
   const ConvL& last = p->convs.back();
   const int HW = last.hout * last.wout;
-  RN_LAUNCH((avgpool_kernel<TA><<<(G * p->B * p->F + 127) / 128, 128, 0, s>>>(
+  RN_LAUNCH((launch_pdl(avgpool_kernel<TA>, (G * p->B * p->F + 127) / 128, 128, 0, s,
       reinterpret_cast<const TA*>(p->act.back()), p->feat, G * p->B, HW, p->F)));
   GemmArgs g{};
   g.M = p->B;
@@ -1241,23 +1269,23 @@ lsgd_status bn_backward(ResNetPlan* p, const ConvL& c, int i, const float* dout,
   const int nq = (int)((P + chunk - 1) / chunk);
   const int lanes = std::max(1, 256 / c.cout);
   if (vec4_ok(c.cout))
-    RN_LAUNCH((bn_bwd_partial_v4_kernel<TA><<<dim3(nq, K), 256, 0, s>>>(
-        dout, reinterpret_cast<const TA*>(out), p->y[i], p->mean[i], p->rstd[i], P, c.cout, nq,
-        chunk, p->part)));
+    RN_LAUNCH((launch_pdl(bn_bwd_partial_v4_kernel<TA>, dim3(nq, K), 256, 0, s, dout,
+        reinterpret_cast<const TA*>(out), p->y[i], p->mean[i], p->rstd[i], P, c.cout, nq, chunk,
+        p->part)));
   else
-    RN_LAUNCH((bn_bwd_partial_kernel<TA><<<dim3(nq, K), lanes * c.cout, 0, s>>>(
-        dout, reinterpret_cast<const TA*>(out), p->y[i], p->mean[i], p->rstd[i], P, c.cout, nq,
-        chunk, p->part)));
-  RN_LAUNCH((bn_bwd_finalize_kernel<<<(K * c.cout * 32 + 127) / 128, 128, 0, s>>>(
-      p->part, c.cout, nq, K, p->s12, Gr, c.g_off, c.b_off, p->d_pad)));
+    RN_LAUNCH((launch_pdl(bn_bwd_partial_kernel<TA>, dim3(nq, K), lanes * c.cout, 0, s, dout,
+        reinterpret_cast<const TA*>(out), p->y[i], p->mean[i], p->rstd[i], P, c.cout, nq, chunk,
+        p->part)));
+  RN_LAUNCH((launch_pdl(bn_bwd_finalize_kernel, (K * c.cout * 32 + 127) / 128, 128, 0, s, p->part,
+      c.cout, nq, K, p->s12, Gr, c.g_off, c.b_off, p->d_pad)));
   if (vec4_ok(c.cout)) {
-    RN_LAUNCH((bn_bwd_apply_v4_kernel<TA><<<dim3(px_blocks(P, c.cout), (unsigned)K), 256, 0, s>>>(
-        dout, reinterpret_cast<const TA*>(out), p->y[i], p->mean[i], p->rstd[i], p->s12, W, c.g_off,
-        p->d_pad, reinterpret_cast<TA*>(p->dy), (int)P, c.cout)));
+    RN_LAUNCH((launch_pdl(bn_bwd_apply_v4_kernel<TA>, dim3(px_blocks(P, c.cout), (unsigned)K), 256,
+        0, s, dout, reinterpret_cast<const TA*>(out), p->y[i], p->mean[i], p->rstd[i], p->s12, W,
+        c.g_off, p->d_pad, reinterpret_cast<TA*>(p->dy), (int)P, c.cout)));
   } else {
     const int64_t n = (int64_t)K * P * c.cout / 4;
-    RN_LAUNCH((bn_bwd_apply_kernel<TA><<<grid_cap(n, 256), 256, 0, s>>>(
-        dout, reinterpret_cast<const TA*>(out), p->y[i], p->mean[i], p->rstd[i], p->s12, W, c.g_off,
+    RN_LAUNCH((launch_pdl(bn_bwd_apply_kernel<TA>, grid_cap(n, 256), 256, 0, s, dout,
+        reinterpret_cast<const TA*>(out), p->y[i], p->mean[i], p->rstd[i], p->s12, W, c.g_off,
         p->d_pad, reinterpret_cast<TA*>(p->dy), K, P, c.cout)));
   }
   return LSGD_OK;
@@ -1304,20 +1332,20 @@ lsgd_status conv_wgrad(ResNetPlan* p, int i, const void* in, float* Gr, cudaStre
     t.splits = splits;
     t.epi = EPI_STORE;
     RN_CALL(launch_gemm_tc(t, s));
-    RN_LAUNCH((sum_partials_crop_kernel<<<sum_partials_grid((int64_t)K * c.cout * 9 * c.cin),
-                                            32 * kSumWarps, 0, s>>>(
-        p->part, splits, c.cout, Kc, 9 * c.cin, K, Gr + c.w_off, p->d_pad)));
+    RN_LAUNCH((launch_pdl(sum_partials_crop_kernel,
+        sum_partials_grid((int64_t)K * c.cout * 9 * c.cin), 32 * kSumWarps, 0, s, p->part, splits,
+        c.cout, Kc, 9 * c.cin, K, Gr + c.w_off, p->d_pad)));
     return LSGD_OK;
   }
   const int nq = (int)((P + kWgradChunk - 1) / kWgradChunk);
   const int J = 9 * c.cin;
   const size_t smem = (size_t)(kWgradTile * 16 + kWgradTile * J) * 4;
-  RN_LAUNCH((conv_wgrad_partial_kernel<TA><<<dim3(nq, (c.cout + 15) / 16, K), 256, smem, s>>>(
-      reinterpret_cast<const TA*>(p->dy), reinterpret_cast<const TA*>(in), p->part, p->B, c.hin,
+  RN_LAUNCH((launch_pdl(conv_wgrad_partial_kernel<TA>, dim3(nq, (c.cout + 15) / 16, K), 256, smem,
+      s, reinterpret_cast<const TA*>(p->dy), reinterpret_cast<const TA*>(in), p->part, p->B, c.hin,
       c.win, c.cin, c.hout, c.wout, c.cout, c.stride, nq)));
   const int64_t n = (int64_t)c.cout * J;
-  RN_LAUNCH((sum_partials_kernel<<<grid_cap((int64_t)K * n, 256), 256, 0, s>>>(
-      p->part, nq, n, K, Gr + c.w_off, p->d_pad)));
+  RN_LAUNCH((launch_pdl(sum_partials_kernel, grid_cap((int64_t)K * n, 256), 256, 0, s, p->part, nq,
+      n, K, Gr + c.w_off, p->d_pad)));
   return LSGD_OK;
 }
 
@@ -1330,9 +1358,9 @@ lsgd_status conv_dgrad(ResNetPlan* p, int i, const void* Wop, float* dx, const f
   if (conv_on_tc(p, c) && c.stride == 1 && implicit_conv_ok(c.cout, 1, c.hin, c.win)) {
     // stride 1: dx is the convolution of dy with the flipped, transposed weights -- an implicit
     // GEMM over dy's taps, no column matrix
-    RN_LAUNCH((flip_weights_kernel<<<dim3((unsigned)((c.cin * 9 * c.cout + 255) / 256), (unsigned)K), 256,
-                                       0, s>>>(reinterpret_cast<const uint16_t*>(Wop), p->d_pad, c.w_off,
-                                               p->wt, K, c.cin, c.cout)));
+    RN_LAUNCH((launch_pdl(flip_weights_kernel,
+        dim3((unsigned)((c.cin * 9 * c.cout + 255) / 256), (unsigned)K), 256, 0, s,
+        reinterpret_cast<const uint16_t*>(Wop), p->d_pad, c.w_off, p->wt, K, c.cin, c.cout)));
     if (persistent_conv_ok(c.cin, P)) {
       ConvArgs ca{};
       bool okc = make_tma_map_conv(&ca.in_map, p->dy, c.cout, c.wout, c.hout, p->B, K, c.win,
@@ -1381,11 +1409,10 @@ lsgd_status conv_dgrad(ResNetPlan* p, int i, const void* Wop, float* dx, const f
     }
     if (dout) {
       const int64_t n = (int64_t)p->B * c.hout * c.wout * (c.cin / 4);
-      RN_LAUNCH((add_shortcut_grad_v2_kernel<TA><<<dim3((unsigned)((n + 255) / 256), (unsigned)K), 256,
-                                                   0, s>>>(dx, dout,
-                                                           reinterpret_cast<const TA*>(out_act),
-                                                           p->B, c.hin, c.win, c.cin, c.hout,
-                                                           c.wout, c.cout, c.stride)));
+      RN_LAUNCH((launch_pdl(add_shortcut_grad_v2_kernel<TA>,
+          dim3((unsigned)((n + 255) / 256), (unsigned)K), 256, 0, s, dx, dout,
+          reinterpret_cast<const TA*>(out_act), p->B, c.hin, c.win, c.cin, c.hout, c.wout, c.cout,
+          c.stride)));
     }
     return LSGD_OK;
   }
@@ -1395,22 +1422,22 @@ lsgd_status conv_dgrad(ResNetPlan* p, int i, const void* Wop, float* dx, const f
     const dim3 rows_grid((unsigned)(p->B * c.hin), (unsigned)K);
     const uint16_t* dy16 = reinterpret_cast<const uint16_t*>(p->dy);
     if (c.cout == 16)
-      RN_LAUNCH((col_dgrad_row_kernel<2><<<rows_grid, 256, 0, s>>>(dy16, p->colT, p->B, c.hin, c.win,
-                                                                   c.hout, c.wout, c.stride)));
+      RN_LAUNCH((launch_pdl(col_dgrad_row_kernel<2>, rows_grid, 256, 0, s, dy16, p->colT, p->B,
+          c.hin, c.win, c.hout, c.wout, c.stride)));
     else if (c.cout == 32)
-      RN_LAUNCH((col_dgrad_row_kernel<4><<<rows_grid, 256, 0, s>>>(dy16, p->colT, p->B, c.hin, c.win,
-                                                                   c.hout, c.wout, c.stride)));
+      RN_LAUNCH((launch_pdl(col_dgrad_row_kernel<4>, rows_grid, 256, 0, s, dy16, p->colT, p->B,
+          c.hin, c.win, c.hout, c.wout, c.stride)));
     else if (c.cout == 64)
-      RN_LAUNCH((col_dgrad_row_kernel<8><<<rows_grid, 256, 0, s>>>(dy16, p->colT, p->B, c.hin, c.win,
-                                                                   c.hout, c.wout, c.stride)));
+      RN_LAUNCH((launch_pdl(col_dgrad_row_kernel<8>, rows_grid, 256, 0, s, dy16, p->colT, p->B,
+          c.hin, c.win, c.hout, c.wout, c.stride)));
     else
-      RN_LAUNCH((col_dgrad_v2_kernel<<<dim3((unsigned)((P * 9 * (c.cout / 8) + 255) / 256), (unsigned)K),
-                                         256, 0, s>>>(reinterpret_cast<const uint16_t*>(p->dy),
-                                                      p->colT, p->B, c.hin, c.win, c.cout, c.hout,
-                                                      c.wout, c.stride)));
-    RN_LAUNCH((flip_weights_kernel<<<dim3((unsigned)((c.cin * Kc + 255) / 256), (unsigned)K), 256, 0,
-                                       s>>>(reinterpret_cast<const uint16_t*>(Wop), p->d_pad, c.w_off,
-                                            p->wt, K, c.cin, c.cout)));
+      RN_LAUNCH((launch_pdl(col_dgrad_v2_kernel,
+          dim3((unsigned)((P * 9 * (c.cout / 8) + 255) / 256), (unsigned)K), 256, 0, s,
+          reinterpret_cast<const uint16_t*>(p->dy), p->colT, p->B, c.hin, c.win, c.cout, c.hout,
+          c.wout, c.stride)));
+    RN_LAUNCH((launch_pdl(flip_weights_kernel,
+        dim3((unsigned)((c.cin * Kc + 255) / 256), (unsigned)K), 256, 0, s,
+        reinterpret_cast<const uint16_t*>(Wop), p->d_pad, c.w_off, p->wt, K, c.cin, c.cout)));
     TcGemmArgs t{};
     t.M = (int)P;
     t.N = c.cin;
@@ -1432,17 +1459,16 @@ lsgd_status conv_dgrad(ResNetPlan* p, int i, const void* Wop, float* dx, const f
     RN_CALL(launch_gemm_tc(t, s));
     if (dout) {
       const int64_t n = (int64_t)p->B * c.hout * c.wout * (c.cin / 4);
-      RN_LAUNCH((add_shortcut_grad_v2_kernel<TA><<<dim3((unsigned)((n + 255) / 256), (unsigned)K), 256,
-                                                   0, s>>>(dx, dout,
-                                                           reinterpret_cast<const TA*>(out_act),
-                                                           p->B, c.hin, c.win, c.cin, c.hout,
-                                                           c.wout, c.cout, c.stride)));
+      RN_LAUNCH((launch_pdl(add_shortcut_grad_v2_kernel<TA>,
+          dim3((unsigned)((n + 255) / 256), (unsigned)K), 256, 0, s, dx, dout,
+          reinterpret_cast<const TA*>(out_act), p->B, c.hin, c.win, c.cin, c.hout, c.wout, c.cout,
+          c.stride)));
     }
     return LSGD_OK;
   }
   dim3 grid((unsigned)((P + 63) / 64), (unsigned)((c.cin + 15) / 16), (unsigned)K);
   const size_t smem = (size_t)c.cout * 9 * 16 * 4;
-  RN_LAUNCH((conv_dgrad_kernel<TA><<<grid, 64, smem, s>>>(
+  RN_LAUNCH((launch_pdl(conv_dgrad_kernel<TA>, grid, 64, smem, s,
       reinterpret_cast<const TA*>(p->dy), reinterpret_cast<const TA*>(Wop) + c.w_off, p->d_pad, dx,
       p->B, c.hin, c.win, c.cin, c.hout, c.wout, c.cout, c.stride, dout,
       reinterpret_cast<const TA*>(out_act))));
@@ -1502,8 +1528,8 @@ lsgd_status fwd_bwd_impl(ResNetPlan* p, const float* W, const void* Wop, float* 
   int cur = 0;
   {
     const int64_t n = (int64_t)K * B * HW * p->F;
-    RN_LAUNCH((avgpool_bwd_kernel<<<grid_cap(n, 256), 256, 0, s>>>(p->dfeat, p->dA[cur], n, HW,
-                                                                     p->F)));
+    RN_LAUNCH((launch_pdl(avgpool_bwd_kernel, grid_cap(n, 256), 256, 0, s, p->dfeat, p->dA[cur], n,
+        HW, p->F)));
   }
   const int n_blocks = (int)(p->convs.size() - 1) / 2;
   for (int j = n_blocks - 1; j >= 0; --j) {
@@ -1572,9 +1598,8 @@ cudaError_t launch_conv_wgrad_bf16(const uint16_t* x, const uint16_t* dy, float*
   a.part = part;
   cudaError_t e = launch_conv_wgrad_tc(a, s);
   if (e != cudaSuccess) return e;
-  // an ordinary launch: this kernel reads the partials without a grid-dependency wait
-  sum_partials_crop_kernel<<<sum_partials_grid((int64_t)G * cout * 9 * cin), 32 * kSumWarps, 0, s>>>(
-      part, a.cpr, cout, 9 * cin, 9 * cin, G, dW, dW_gs);
+  launch_pdl(sum_partials_crop_kernel, sum_partials_grid((int64_t)G * cout * 9 * cin),
+      32 * kSumWarps, 0, s, part, a.cpr, cout, 9 * cin, 9 * cin, G, dW, dW_gs);
   return cudaGetLastError();
 }
 
@@ -1585,15 +1610,15 @@ cudaError_t launch_batchnorm_stats(const float* y, int64_t P, int C, int G, floa
   if (nq > 65535) return cudaErrorInvalidValue;
   const int lanes = std::max(1, 256 / C);
   if (vec4_ok(C))
-    bn_stats_partial_v4_kernel<<<dim3((unsigned)nq, (unsigned)G), 256, 0, s>>>(y, P, C, (int)nq,
-                                                                               kStatChunk, part);
+    launch_pdl(bn_stats_partial_v4_kernel, dim3((unsigned)nq, (unsigned)G), 256, 0, s, y, P, C,
+        (int)nq, kStatChunk, part);
   else
-    bn_stats_partial_kernel<<<dim3((unsigned)nq, (unsigned)G), lanes * C, 0, s>>>(y, P, C, (int)nq,
-                                                                               kStatChunk, part);
+    launch_pdl(bn_stats_partial_kernel, dim3((unsigned)nq, (unsigned)G), lanes * C, 0, s, y, P, C,
+        (int)nq, kStatChunk, part);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  bn_stats_finalize_kernel<<<(G * C * 32 + 127) / 128, 128, 0, s>>>(part, P, C, (int)nq, kStatChunk,
-                                                                     G, mean, rstd);
+  launch_pdl(bn_stats_finalize_kernel, (G * C * 32 + 127) / 128, 128, 0, s, part, P, C, (int)nq,
+      kStatChunk, G, mean, rstd);
   return cudaGetLastError();
 }
 

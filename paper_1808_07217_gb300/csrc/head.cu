@@ -228,8 +228,17 @@ __global__ void __launch_bounds__(256) head_backward_kernel(HeadArgs h) {
     float s = 0.f;
     if (n0 + n < h.in) {
       const int rows = (h.B + 3) / 4, j0 = qtr * rows, j1 = min(h.B, j0 + rows);
-      for (int j = j0; j < j1; ++j)
-        s += bf2f(h.dz_prev[((int64_t)g * h.B + j) * h.ld_dz_prev + n0 + n]);
+      const uint16_t* col = h.dz_prev + ((int64_t)g * h.B) * h.ld_dz_prev + n0 + n;
+      int j = j0;
+      // eight rows' loads in flight, then added in row order (the same sum as one at a time)
+      for (; j + 8 <= j1; j += 8) {
+        float v[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) v[u] = bf2f(col[(int64_t)(j + u) * h.ld_dz_prev]);
+#pragma unroll
+        for (int u = 0; u < 8; ++u) s += v[u];
+      }
+      for (; j < j1; ++j) s += bf2f(col[(int64_t)j * h.ld_dz_prev]);
     }
     part[qtr * kHeadCols + n] = s;
     __syncthreads();

@@ -900,14 +900,16 @@ __global__ void pad_weights_kernel(const uint16_t* __restrict__ Wb, int64_t d_pa
 
 // Sum of split partials [g][q][rows][ldc] in split order, keeping the first `cols` columns:
 // out[g * out_gs + r cols + j].
-// out[g out_gs + r cols + j] = sum over q of part[g][q][r][j] (j < cols of ldc).  A CTA takes 32
-// consecutive outputs (one per lane); warp w sums the partials q = w, w + 8, ... (independent
-// loads, all in flight), and the eight warp sums are added in warp order: a fixed order, so the
-// result is deterministic.
+// out[g out_gs + r cols + j] = sum over q of part[g][q][r][src(j)] (j < cols of ldc), src(j) = j,
+// or with taps of tap_dst channels read from taps of tap_src channels (a padded convolution's
+// weight gradient cropped to its real input channels): src(j) = (j / tap_dst) tap_src + j % tap_dst.
+// A CTA takes 32 consecutive outputs (one per lane); warp w sums the partials q = w, w + 8, ...
+// (independent loads, all in flight), and the eight warp sums are added in warp order: a fixed
+// order, so the result is deterministic.
 constexpr int kSumWarps = 8;
 __global__ void __launch_bounds__(32 * kSumWarps) sum_partials_crop_kernel(
     const float* __restrict__ part, int nq, int rows, int ldc, int cols, int G,
-    float* __restrict__ out, int64_t out_gs) {
+    float* __restrict__ out, int64_t out_gs, int tap_src, int tap_dst) {
   pdl_begin();
   __shared__ float ws[kSumWarps][32];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -919,7 +921,8 @@ __global__ void __launch_bounds__(32 * kSumWarps) sum_partials_crop_kernel(
     j = (int)(t % cols);
     r = (int)((t / cols) % rows);
     g = (int)(t / ((int64_t)rows * cols));
-    const float* p = part + (int64_t)g * nq * rows * ldc + (int64_t)r * ldc + j;
+    const int js = tap_dst > 0 ? (j / tap_dst) * tap_src + j % tap_dst : j;
+    const float* p = part + (int64_t)g * nq * rows * ldc + (int64_t)r * ldc + js;
     const int64_t qs = (int64_t)rows * ldc;
 #pragma unroll 4
     for (int q = warp; q < nq; q += kSumWarps) acc += p[q * qs];
@@ -934,6 +937,36 @@ __global__ void __launch_bounds__(32 * kSumWarps) sum_partials_crop_kernel(
   }
 }
 unsigned sum_partials_grid(int64_t n) { return (unsigned)((n + 31) / 32); }
+
+// The stem's image with zero channels appended: x16[q][c] = c < C0 ? x0[q][c] : 0 (one thread per
+// pixel, two 16-byte stores).
+__global__ void pad_input16_kernel(const uint16_t* __restrict__ x0, uint16_t* __restrict__ x16,
+                                   int64_t npix, int C0) {
+  pdl_begin();
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t q = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; q < npix; q += stride) {
+    uint32_t w[8] = {0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u};
+    for (int c = 0; c < C0; ++c) w[c >> 1] |= (uint32_t)x0[q * C0 + c] << (16 * (c & 1));
+    uint4* dst = reinterpret_cast<uint4*>(x16 + q * 16);
+    dst[0] = make_uint4(w[0], w[1], w[2], w[3]);
+    dst[1] = make_uint4(w[4], w[5], w[6], w[7]);
+  }
+}
+
+// The stem's weights with the same zero channels: wstem[g][co][t][ci] = ci < C0 ?
+// W[g][co][t][ci] : 0 (bf16, 16 channels per tap).
+__global__ void pad_stem_weights_kernel(const uint16_t* __restrict__ Wb, int64_t d_pad,
+                                        int64_t w_off, uint16_t* __restrict__ wstem, int G,
+                                        int Cout, int C0) {
+  pdl_begin();
+  const int64_t n = (int64_t)G * Cout * 9 * 16;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < n; e += stride) {
+    const int ci = (int)(e % 16), t = (int)((e / 16) % 9), co = (int)((e / 144) % Cout);
+    const int64_t g = e / (144 * (int64_t)Cout);
+    wstem[e] = ci < C0 ? Wb[g * d_pad + w_off + ((int64_t)co * 9 + t) * C0 + ci] : (uint16_t)0;
+  }
+}
 
 // Weights of the stride-1 data gradient as a convolution of the output gradient:
 // wt[g][ci][t][co] = w[g][co][8 - t][ci] (taps flipped, channels transposed), bf16.
@@ -1003,6 +1036,11 @@ struct ResNetPlan {
   std::vector<uint16_t*> col;
   uint16_t* colT = nullptr;
   uint16_t* wt = nullptr;
+  // a stem with fewer than 16 input channels runs as a 16-channel convolution on the tensor-core
+  // kernels: the image with zero channels appended, and its weights likewise
+  bool stem16 = false;
+  uint16_t* x16 = nullptr;    // [K][B][H0][W0][16]
+  uint16_t* wstem = nullptr;  // [K][Cout][9][16]
   std::string err;
 };
 
@@ -1059,8 +1097,16 @@ bool implicit_fwd(const ConvL& c) {
 bool needs_col(const ResNetPlan* p, const ConvL& c) {
   return conv_on_tc(p, c) && !(wgrad_tc(p, c) && implicit_fwd(c));
 }
+
 // The persistent convolution kernel: N = 16, 32 or 64 outputs, whole 128-pixel tiles.
 bool persistent_conv_ok(int n, int64_t P) { return (n == 16 || n == 32 || n == 64) && P % 128 == 0; }
+// The stem (fewer than 16 input channels) as a 16-channel convolution on the implicit kernels.
+bool stem16_ok(const ResNetPlan* p, const ConvL& c) {
+  const int64_t P = (int64_t)p->B * c.hout * c.wout;
+  return conv_on_tc(p, c) && c.cin < 16 && c.stride == 1 && implicit_conv_ok(16, 1, c.hout, c.wout) &&
+         persistent_conv_ok(c.cout, P) &&
+         conv_wgrad_tc_ok(16, c.cout, 1, c.hin, c.win, c.hout, c.wout);
+}
 // The four-channel kernels need C a multiple of 4 with C / 4 dividing their 256 threads.
 bool vec4_ok(int C) { return C % 4 == 0 && 256 % (C / 4) == 0; }
 // Blocks of a per-replica kernel whose threads each take one pixel and group of 4 channels.
@@ -1074,6 +1120,35 @@ lsgd_status conv_forward(ResNetPlan* p, int i, const void* in, const void* Wop, 
                          int w_gmul, float* y, int G, cudaStream_t s, int64_t* launches) {
   const ConvL& c = p->convs[i];
   const int64_t P = conv_pixels(p, c);
+  if (i == 0 && p->stem16 && w_g0 == 0 && w_gmul == 1) {
+    // the stem as a 16-channel convolution: zero channels appended to the image and the weights
+    // (the products are unchanged), then the persistent implicit-GEMM kernel
+    const int64_t npix = (int64_t)G * P;
+    RN_LAUNCH(launch_pdl(pad_input16_kernel, grid_cap(npix, 256), 256, 0, s,
+                         reinterpret_cast<const uint16_t*>(in), p->x16, npix, c.cin));
+    RN_LAUNCH(launch_pdl(pad_stem_weights_kernel, grid_cap((int64_t)G * c.cout * 144, 256), 256, 0,
+                         s, reinterpret_cast<const uint16_t*>(Wop), p->d_pad, c.w_off, p->wstem, G,
+                         c.cout, c.cin));
+    ConvArgs ca{};
+    bool okc = make_tma_map_conv(&ca.in_map, p->x16, 16, c.win, c.hin, p->B, G, c.wout, c.hout, 1);
+    okc &= make_tma_map(&ca.w_map, p->wstem, true, 9 * 16, c.cout, G, 9 * 16,
+                        (uint64_t)c.cout * 9 * 16, 16, c.cout, 32);
+    if (!okc) {
+      p->err = "TMA map encoding failed (stem convolution)";
+      return LSGD_ECUDA;
+    }
+    ca.ck = 16;
+    ca.stride = 1;
+    ca.hout = c.hout;
+    ca.wout = c.wout;
+    ca.N = ca.np = c.cout;
+    ca.G = G;
+    ca.P = (int)P;
+    ca.out = y;
+    ca.out_gs = P * c.cout;
+    RN_CALL(launch_conv_tc(ca, s));
+    return LSGD_OK;
+  }
   if (conv_on_tc(p, c) && w_g0 == 0 && w_gmul == 1) {
     // y = im2col(in) [P][9 Cin] x W^T on the tensor cores (both operands K-major)
     const int Kc = col_ld(c);
@@ -1297,6 +1372,14 @@ lsgd_status conv_wgrad(ResNetPlan* p, int i, const void* in, float* Gr, cudaStre
   const ConvL& c = p->convs[i];
   const int K = p->K;
   const int64_t P = conv_pixels(p, c);
+  if (i == 0 && p->stem16) {
+    // the padded stem's input (written by the forward); the gradient keeps the real channels
+    RN_CALL(launch_conv_wgrad_bf16(p->x16, reinterpret_cast<const uint16_t*>(p->dy), Gr + c.w_off,
+                                   p->d_pad, K, p->B, c.hout, c.wout, 16, c.cout, 1, p->part, s,
+                                   c.cin));
+    ++*launches;  // the partials' sum
+    return LSGD_OK;
+  }
   if (wgrad_tc(p, c)) {
     // dW [Cout][9 Cin] from dy and the input directly: the column matrix of each 64-pixel block
     // is built in shared memory; one partial per CTA, summed in order
@@ -1334,7 +1417,7 @@ lsgd_status conv_wgrad(ResNetPlan* p, int i, const void* in, float* Gr, cudaStre
     RN_CALL(launch_gemm_tc(t, s));
     RN_LAUNCH((launch_pdl(sum_partials_crop_kernel,
         sum_partials_grid((int64_t)K * c.cout * 9 * c.cin), 32 * kSumWarps, 0, s, p->part, splits,
-        c.cout, Kc, 9 * c.cin, K, Gr + c.w_off, p->d_pad)));
+        c.cout, Kc, 9 * c.cin, K, Gr + c.w_off, p->d_pad, 0, 0)));
     return LSGD_OK;
   }
   const int nq = (int)((P + kWgradChunk - 1) / kWgradChunk);
@@ -1575,11 +1658,12 @@ size_t conv_wgrad_scratch_floats(int G, int B, int hout, int wout, int cin, int 
 
 cudaError_t launch_conv_wgrad_bf16(const uint16_t* x, const uint16_t* dy, float* dW, int64_t dW_gs,
                                    int G, int B, int hout, int wout, int cin, int cout, int stride,
-                                   float* part, cudaStream_t s) {
+                                   float* part, cudaStream_t s, int cin_out) {
   const int hin = hout * stride, win = wout * stride;
   const int64_t P = (int64_t)B * hout * wout;
+  if (cin_out <= 0) cin_out = cin;
   if (!conv_wgrad_tc_ok(cin, cout, stride, hin, win, hout, wout) || G < 1 || B < 1 ||
-      P > 0x7fffffffLL)
+      P > 0x7fffffffLL || cin_out > cin)
     return cudaErrorInvalidValue;
   ConvWgradArgs a{};
   if (!make_tma_map_halo(&a.x_map, x, cin, win, hin, B, G, stride, wout) ||
@@ -1598,8 +1682,10 @@ cudaError_t launch_conv_wgrad_bf16(const uint16_t* x, const uint16_t* dy, float*
   a.part = part;
   cudaError_t e = launch_conv_wgrad_tc(a, s);
   if (e != cudaSuccess) return e;
-  launch_pdl(sum_partials_crop_kernel, sum_partials_grid((int64_t)G * cout * 9 * cin),
-      32 * kSumWarps, 0, s, part, a.cpr, cout, 9 * cin, 9 * cin, G, dW, dW_gs);
+  // the partials' sum, cropped to the first cin_out channels of every tap
+  launch_pdl(sum_partials_crop_kernel, sum_partials_grid((int64_t)G * cout * 9 * cin_out),
+             32 * kSumWarps, 0, s, part, a.cpr, cout, 9 * cin, 9 * cin_out, G, dW, dW_gs, cin,
+             cin_out);
   return cudaGetLastError();
 }
 
@@ -1747,6 +1833,15 @@ lsgd_status resnet_alloc(ResNetPlan* p, const std::function<void*(size_t)>& allo
   const size_t e = esz(p);
   p->x0 = alloc((size_t)K * B * p->H0 * p->W0 * p->C0 * e);
   size_t part = 0, colT = 0, wt = 0;
+  p->stem16 = stem16_ok(p, p->convs[0]);
+  if (p->stem16) {
+    const ConvL& c0 = p->convs[0];
+    p->x16 = (uint16_t*)alloc((size_t)K * B * c0.hin * c0.win * 16 * 2);
+    p->wstem = (uint16_t*)alloc((size_t)K * c0.cout * 9 * 16 * 2);
+    if (!p->x16 || !p->wstem) return LSGD_ENOMEM;
+    const int64_t P0 = (int64_t)B * c0.hout * c0.wout;
+    part = std::max(part, (size_t)K * conv_wgrad_ctas(16, 1, c0.wout, K, P0) * c0.cout * 9 * 16);
+  }
   for (const ConvL& c : p->convs) {
     const int64_t n = (int64_t)K * B * c.hout * c.wout * c.cout;
     p->y.push_back((float*)alloc((size_t)n * 4));
@@ -1768,7 +1863,7 @@ lsgd_status resnet_alloc(ResNetPlan* p, const std::function<void*(size_t)>& allo
         const int splits = tc_valid_splits((int)P, std::max(1, (4 * kNumSMs + tiles - 1) / tiles));
         part = std::max(part, (size_t)K * splits * c.cout * Kc);
       }
-      if (needs_col(p, c)) {
+      if (needs_col(p, c) && !(&c == &p->convs[0] && p->stem16)) {
         p->col.push_back((uint16_t*)alloc((size_t)K * P * Kc * 2));
         if (!p->col.back()) return LSGD_ENOMEM;
       } else {

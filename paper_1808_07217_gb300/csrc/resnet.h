@@ -43,11 +43,13 @@ size_t batchnorm_stats_scratch_floats(int64_t P, int C, int G);
 // cores: dW[g dW_gs + (co 9 + kh 3 + kw) Cin + ci] = sum over b, oy, ox of dy[g][b][oy][ox][co]
 // x[g][b][oy s + kh - 1][ox s + kw - 1][ci] (zero outside the image), NHWC bf16 operands; the
 // per-CTA partials go to `part` (conv_wgrad_scratch_floats floats) and are summed in order.
-// Shapes as conv_wgrad_tc_ok accepts them, else cudaErrorInvalidValue.
+// cin_out < cin (> 0): x has cin channels of which only the first cin_out are real (zero
+// padding), and dW is [Cout][3][3][cin_out].  Shapes as conv_wgrad_tc_ok accepts them, else
+// cudaErrorInvalidValue.
 size_t conv_wgrad_scratch_floats(int G, int B, int hout, int wout, int cin, int cout, int stride);
 cudaError_t launch_conv_wgrad_bf16(const uint16_t* x, const uint16_t* dy, float* dW, int64_t dW_gs,
                                    int G, int B, int hout, int wout, int cin, int cout, int stride,
-                                   float* part, cudaStream_t s);
+                                   float* part, cudaStream_t s, int cin_out = 0);
 cudaError_t launch_batchnorm_stats(const float* y, int64_t P, int C, int G, float* mean,
                                    float* rstd, float* part, cudaStream_t s);
 const char* resnet_last_error(const ResNetPlan* p);

@@ -946,7 +946,13 @@ __global__ void __launch_bounds__(cv::THREADS, 1) conv_tc_kernel(const __grid_co
       const int ab = i & 1;
       if (!epi_wait(&acc_full[ab], (i >> 1) & 1)) break;
       asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-      float* orow = a.out + (int64_t)g * a.out_gs + ((int64_t)tile * BM + r) * a.N;
+      int64_t dst = (int64_t)tile * BM + r;
+      if (a.dst_h > 0) {
+        const int pp = tile * BM + r, img = pp / per_img, rem = pp - img * per_img;
+        const int oy = rem / a.wout, ox = rem - oy * a.wout;
+        dst = ((int64_t)img * a.dst_h + 2 * oy + a.ph_y) * a.dst_w + 2 * ox + a.ph_x;
+      }
+      float* orow = a.out + (int64_t)g * a.out_gs + dst * a.N;
       for (int c0 = 0; c0 < a.N; c0 += 16) {
         float v[16];
         tmem_ld16(tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(ab * np + c0), v);
@@ -1336,7 +1342,9 @@ cudaError_t launch_conv_tc(const ConvArgs& a, cudaStream_t stream) {
   int rows = 0, images = 0;
   if ((a.ck != 16 && a.ck != 32 && a.ck != 64) || (a.stride != 1 && a.stride != 2) ||
       (a.N != 16 && a.N != 32 && a.N != 64) || a.np != a.N || !a.out || a.G > 65535 ||
-      !conv_tile_shape(a.hout, a.wout, &rows, &images) || a.P % (a.hout * a.wout) || a.P % BM)
+      !conv_tile_shape(a.hout, a.wout, &rows, &images) || a.P % (a.hout * a.wout) || a.P % BM ||
+      (a.dst_h > 0 && (a.dst_h < 2 * a.hout || a.dst_w < 2 * a.wout || a.ph_y < 0 || a.ph_y > 1 ||
+                       a.ph_x < 0 || a.ph_x > 1)))
     return cudaErrorInvalidValue;
   int dev = 0, sms = 0;
   cudaError_t e = cudaGetDevice(&dev);

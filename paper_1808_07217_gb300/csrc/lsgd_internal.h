@@ -148,6 +148,10 @@ struct ConvArgs {
   float* out;
   int64_t out_gs;
   int ring_bytes;  // input ring size (set by the launcher)
+  // dst_h > 0: output pixel (image, y, x) of the Hout x Wout grid goes to pixel
+  // (image, 2 y + ph_y, 2 x + ph_x) of a dst_h x dst_w grid (one parity phase of a stride-2
+  // convolution's data gradient); else to pixel (image, y, x)
+  int ph_y, ph_x, dst_h, dst_w;
 };
 cudaError_t launch_conv_tc(const ConvArgs& a, cudaStream_t stream);
 // Weight gradient of a 3x3 convolution (zero padding 1, stride 1 or 2) on the tensor cores, the

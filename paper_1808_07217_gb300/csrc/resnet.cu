@@ -983,6 +983,30 @@ __global__ void flip_weights_kernel(const uint16_t* __restrict__ Wb, int64_t d_p
   }
 }
 
+// The data gradient of a stride-2 convolution split by the parity (py, px) of the input pixel:
+// dx[2a + py][2b + px][ci] = sum over dr, dc in {0, 1} and co of dy[a + dr][b + dc][co]
+// w[co][py + 1 - 2 dr][px + 1 - 2 dc][ci] (terms whose kernel index leaves 0..2 drop out), a
+// 3x3 stride-1 convolution of dy whose taps (dr + 1, dc + 1) carry those weights and whose other
+// taps are zero.  wt4[ph][g][ci][t][co], ph = 2 py + px, t = 3 (dr + 1) + (dc + 1).
+__global__ void flip_phase_weights_kernel(const uint16_t* __restrict__ Wb, int64_t d_pad,
+                                          int64_t w_off, uint16_t* __restrict__ wt4, int G,
+                                          int Cin, int Cout) {
+  pdl_begin();
+  const int64_t per = (int64_t)Cin * 9 * Cout, n = 4 * (int64_t)G * per;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < n; e += stride) {
+    const int co = (int)(e % Cout), t = (int)((e / Cout) % 9), ci = (int)((e / (9 * Cout)) % Cin);
+    const int64_t gp = e / per;
+    const int g = (int)(gp % G), ph = (int)(gp / G);
+    const int dr = t / 3 - 1, dc = t % 3 - 1;
+    const int kh = (ph >> 1) + 1 - 2 * dr, kw = (ph & 1) + 1 - 2 * dc;
+    uint16_t v = 0;
+    if (kh >= 0 && kh <= 2 && kw >= 0 && kw <= 2)
+      v = Wb[(int64_t)g * d_pad + w_off + (((int64_t)co * 3 + kh) * 3 + kw) * Cin + ci];
+    wt4[e] = v;
+  }
+}
+
 // The option-A shortcut's share of a block's input gradient: for input pixels on the stride grid
 // and the first Cin channels, dx += dout * (out > 0) at (ih / s, iw / s).  Thread = (output pixel,
 // 4 channels < Cin), blockIdx.y the replica; only the input pixels on the stride grid are touched.
@@ -1041,6 +1065,8 @@ struct ResNetPlan {
   bool stem16 = false;
   uint16_t* x16 = nullptr;    // [K][B][H0][W0][16]
   uint16_t* wstem = nullptr;  // [K][Cout][9][16]
+  // the stride-2 data gradients as four parity phases on the implicit kernel: their weights
+  uint16_t* wt4 = nullptr;    // [4][K][Cin][9][Cout] of the largest such convolution
   std::string err;
 };
 
@@ -1106,6 +1132,12 @@ bool stem16_ok(const ResNetPlan* p, const ConvL& c) {
   return conv_on_tc(p, c) && c.cin < 16 && c.stride == 1 && implicit_conv_ok(16, 1, c.hout, c.wout) &&
          persistent_conv_ok(c.cout, P) &&
          conv_wgrad_tc_ok(16, c.cout, 1, c.hin, c.win, c.hout, c.wout);
+}
+// A stride-2 data gradient as four parity phases on the persistent implicit-GEMM kernel.
+bool phase_dgrad_ok(const ResNetPlan* p, const ConvL& c) {
+  return conv_on_tc(p, c) && c.stride == 2 && c.hin == 2 * c.hout && c.win == 2 * c.wout &&
+         implicit_conv_ok(c.cout, 1, c.hout, c.wout) &&
+         persistent_conv_ok(c.cin, (int64_t)p->B * c.hout * c.wout);
 }
 // The four-channel kernels need C a multiple of 4 with C / 4 dividing their 256 threads.
 bool vec4_ok(int C) { return C % 4 == 0 && 256 % (C / 4) == 0; }
@@ -1499,6 +1531,48 @@ lsgd_status conv_dgrad(ResNetPlan* p, int i, const void* Wop, float* dx, const f
     }
     return LSGD_OK;
   }
+  if (phase_dgrad_ok(p, c)) {
+    // stride 2: each parity phase of dx is a 3x3 stride-1 convolution of dy (weights of the
+    // phase's taps, zeros elsewhere) whose outputs land on every other row and column of dx
+    const int64_t per = (int64_t)c.cin * 9 * c.cout;
+    RN_LAUNCH(launch_pdl(flip_phase_weights_kernel, grid_cap(4 * (int64_t)K * per, 256), 256, 0, s,
+                         reinterpret_cast<const uint16_t*>(Wop), p->d_pad, c.w_off, p->wt4, K,
+                         c.cin, c.cout));
+    const int64_t Pq = (int64_t)p->B * c.hout * c.wout;
+    for (int ph = 0; ph < 4; ++ph) {
+      ConvArgs ca{};
+      bool okc = make_tma_map_conv(&ca.in_map, p->dy, c.cout, c.wout, c.hout, p->B, K, c.wout,
+                                   c.hout, 1);
+      okc &= make_tma_map(&ca.w_map, p->wt4 + ph * K * per, true, 9 * c.cout, c.cin, K,
+                          9 * c.cout, (uint64_t)per, c.cout, c.cin, 2 * c.cout);
+      if (!okc) {
+        p->err = "TMA map encoding failed (stride-2 data gradient)";
+        return LSGD_ECUDA;
+      }
+      ca.ck = c.cout;
+      ca.stride = 1;
+      ca.hout = c.hout;
+      ca.wout = c.wout;
+      ca.N = ca.np = c.cin;
+      ca.G = K;
+      ca.P = (int)Pq;
+      ca.out = dx;
+      ca.out_gs = P * c.cin;
+      ca.ph_y = ph >> 1;
+      ca.ph_x = ph & 1;
+      ca.dst_h = c.hin;
+      ca.dst_w = c.win;
+      RN_CALL(launch_conv_tc(ca, s));
+    }
+    if (dout) {
+      const int64_t n = (int64_t)p->B * c.hout * c.wout * (c.cin / 4);
+      RN_LAUNCH((launch_pdl(add_shortcut_grad_v2_kernel<TA>,
+          dim3((unsigned)((n + 255) / 256), (unsigned)K), 256, 0, s, dx, dout,
+          reinterpret_cast<const TA*>(out_act), p->B, c.hin, c.win, c.cin, c.hout, c.wout, c.cout,
+          c.stride)));
+    }
+    return LSGD_OK;
+  }
   if (conv_on_tc(p, c) && c.cin % 8 == 0) {
     // dx = col(dy) [P][9 Cout] x wt^T with the flipped, transposed weights (stride 1 or 2)
     const int Kc = 9 * c.cout;
@@ -1832,7 +1906,7 @@ lsgd_status resnet_alloc(ResNetPlan* p, const std::function<void*(size_t)>& allo
   const int K = p->K, B = p->B;
   const size_t e = esz(p);
   p->x0 = alloc((size_t)K * B * p->H0 * p->W0 * p->C0 * e);
-  size_t part = 0, colT = 0, wt = 0;
+  size_t part = 0, colT = 0, wt = 0, wt4 = 0;
   p->stem16 = stem16_ok(p, p->convs[0]);
   if (p->stem16) {
     const ConvL& c0 = p->convs[0];
@@ -1870,7 +1944,10 @@ lsgd_status resnet_alloc(ResNetPlan* p, const std::function<void*(size_t)>& allo
         p->col.push_back(nullptr);
       }
       if (c.cin % 8 == 0) {
-        colT = std::max(colT, (size_t)K * B * c.hin * c.win * 9 * c.cout);
+        if (phase_dgrad_ok(p, c))
+          wt4 = std::max(wt4, (size_t)4 * K * c.cin * 9 * c.cout);
+        else if (!(c.stride == 1 && implicit_conv_ok(c.cout, 1, c.hin, c.win)))
+          colT = std::max(colT, (size_t)K * B * c.hin * c.win * 9 * c.cout);
         wt = std::max(wt, (size_t)K * c.cin * 9 * c.cout);
       } else {
         wt = std::max(wt, (size_t)K * c.cout * Kc);
@@ -1886,6 +1963,10 @@ lsgd_status resnet_alloc(ResNetPlan* p, const std::function<void*(size_t)>& allo
   if (wt) {
     p->wt = (uint16_t*)alloc(wt * 2);
     if (!p->wt) return LSGD_ENOMEM;
+  }
+  if (wt4) {
+    p->wt4 = (uint16_t*)alloc(wt4 * 2);
+    if (!p->wt4) return LSGD_ENOMEM;
   }
   p->part_floats = part;
   p->part = (float*)alloc(part * 4);

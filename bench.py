@@ -308,6 +308,102 @@ def run_sync_variants(args):
         P.lsgd_destroy(ctx)
 
 
+# The other dense configurations, timed on their own job schedules (one JSON line each):
+#   softmax regression 3072 -> 10, fp32, zero init, K = 4 shards of 2,048 of N = 8,192 points,
+#     B_loc = 32, H = 4, plain SGD lr 0.1, a 64-step job;
+#   post-local MLP 3072-4096-4096-4096-100, bf16, K = 16, B_loc = 128, 10 epochs of N = 50,000
+#     (245 steps), H = 1 before t' = 122 and 16 after, Nesterov 0.9, weight decay 5e-4, lr 0.1
+#     scaled by K with a 5-epoch warm-up, decayed 10x at 50 % and 75 %.
+DENSE_CONFIGS = {
+    "softmax": dict(name="softmax_3072-10_K4_B32_H4_fp32", widths=(3072, 10), K=4, B=32, H=4,
+                    N=8192, C=10, T=64, t_switch=-1, base_lr=0.1, scale_by_K=False,
+                    warmup_epochs=0.0, milestones=(), momentum=0.0, nesterov=False,
+                    weight_decay=0.0, init="zero", bf16=False, seed=0, data_seed=1234),
+    "mlp4096": dict(name="mlp_3072-4096x3-100_K16_B128_postlocal_H16_bf16",
+                    widths=(3072, 4096, 4096, 4096, 100), K=16, B=128, H=16, N=50000, C=100,
+                    T=245, t_switch=122, base_lr=0.1, scale_by_K=True, warmup_epochs=5.0,
+                    milestones=(0.5, 0.75), momentum=0.9, nesterov=True, weight_decay=5e-4,
+                    init="he", bf16=True, seed=0, data_seed=1234),
+}
+
+
+def run_dense_config(args, key):
+    """Time one of DENSE_CONFIGS: W warm-up steps, then S timed steps of its job schedule
+    (repeated from its end state, as for the benchmark workload), then a traced pass for the
+    per-phase split.  One JSON line with samples/s, ms per step, the syncs and launches in the
+    timed region and the update phase's algorithmic HBM throughput."""
+    import numpy as np
+    import torch
+
+    import synthdata
+    from paper_1808_07217_gb300 import _build
+
+    _build.build()
+    import paper_1808_07217_gb300 as P
+
+    torch.cuda.set_device(0)
+    w = DENSE_CONFIGS[key]
+    K, B, T = w["K"], w["B"], w["T"]
+    X, y = synthdata.gaussian_mixture_cached(w["N"], w["widths"][0], w["C"], w["data_seed"])
+    W_, S_ = max(3, args.warmup), args.steps
+    fused = w["bf16"]
+    cfg = P.make_config(K=K, B_loc=B, H=w["H"], t_switch=w["t_switch"], total_steps=T, N=w["N"],
+                        widths=w["widths"], init=P.INIT_ZERO if w["init"] == "zero" else P.INIT_HE,
+                        base_lr=w["base_lr"], scale_by_K=w["scale_by_K"],
+                        warmup_epochs=w["warmup_epochs"], milestones=w["milestones"],
+                        momentum=w["momentum"], nesterov=w["nesterov"],
+                        weight_decay=w["weight_decay"], seed=w["seed"],
+                        precision=P.BF16 if w["bf16"] else P.FP32, fused_update=fused)
+    stream = torch.cuda.current_stream()
+    ctx = P.lsgd_create(cfg, stream=stream.cuda_stream)
+    P.lsgd_set_dataset(ctx, X, y)
+    d = P.lsgd_num_params(ctx)
+
+    def run_steps(n):
+        while n > 0:
+            m = min(n, T - P.lsgd_step_count(ctx))
+            P.lsgd_run(ctx, m)
+            n -= m
+            if P.lsgd_step_count(ctx) == T:
+                P.lsgd_set_step(ctx, 0)
+
+    run_steps(W_)
+    torch.cuda.synchronize()
+    n0, sy0 = P.lsgd_kernel_launches(ctx), P.lsgd_sync_count(ctx)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    run_steps(S_)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1)
+    launches, syncs = P.lsgd_kernel_launches(ctx) - n0, P.lsgd_sync_count(ctx) - sy0
+    n_chk = min(P.lsgd_step_count(ctx), 8)
+    losses = P.lsgd_losses(ctx, n_chk, K) if n_chk else np.zeros(1)
+    P.lsgd_profile_enable(ctx, True)
+    run_steps(S_)
+    torch.cuda.synchronize()
+    prof = P.lsgd_profile_read(ctx)
+    hbm, _, src = _peaks()
+    widths = w["widths"]
+    if fused:
+        upd_bytes = sum(FUSED_UPDATE_BYTES_PER_PARAM * K * widths[l] * widths[l + 1]
+                        + 2 * K * B * (widths[l] + widths[l + 1]) for l in range(len(widths) - 1))
+    else:
+        upd_bytes = UPDATE_BYTES_PER_PARAM * K * d
+    upd_ms = prof["update"][1] / S_
+    print(json.dumps({"workload": w["name"], "value": S_ * K * B / (ms / 1000.0),
+                      "unit": "samples/s", "steps": S_, "ms_per_step": ms / S_,
+                      "job": f"{T}-step schedule, repeated from its end state",
+                      "syncs_in_timed_region": syncs, "gpu_launches": launches,
+                      "params_per_replica": d, "losses_finite": bool(np.isfinite(losses).all()),
+                      "update_phase": {"ms_per_step": upd_ms, "algorithmic_bytes": upd_bytes,
+                                       "gbs": upd_bytes / (upd_ms * 1e6) if upd_ms else None,
+                                       "frac_of_hbm": (upd_bytes / (upd_ms * 1e6) / hbm)
+                                       if upd_ms else None, "peak_source": f"{src} hbm_gbs"},
+                      "phase_ms_per_step": {k: v[1] / S_ for k, v in prof.items()}}), flush=True)
+    P.lsgd_destroy(ctx)
+
+
 RESNET_WORKLOAD = dict(name="resnet20_K16_B128_postlocal_H16_bf16", K=16, B=128, H=16, N=50000,
                        C=10, base_lr=0.2, scale_by_K=True, warmup_epochs=5.0, momentum=0.9,
                        nesterov=True, weight_decay=1e-4, seed=0, data_seed=1234, epochs=1.0)
@@ -389,6 +485,9 @@ def main():
     ap.add_argument("--sync-variants", action="store_true",
                     help="time one synchronisation of each averaging variant (plain, global "
                          "momentum, sign, EF-sign) on the MLP workload's K x d arena")
+    ap.add_argument("--config", choices=sorted(DENSE_CONFIGS),
+                    help="time another dense configuration (softmax regression, post-local "
+                         "MLP 3072-4096x3-100) on its job schedule")
     ap.add_argument("--resnet", action="store_true",
                     help="post-local ResNet-20 workload (K = 16, B_loc = 128) instead of the MLP")
     ap.add_argument("--unfused", action="store_true",
@@ -403,6 +502,9 @@ def main():
         return
     if args.resnet:
         run_resnet(args)
+        return
+    if args.config:
+        run_dense_config(args, args.config)
         return
     if args.sync_variants:
         run_sync_variants(args)

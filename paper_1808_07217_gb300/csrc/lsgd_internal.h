@@ -136,6 +136,11 @@ struct GemmArgs {
   // cv_ck * 2 bytes.  M = pixels of the output (whole rows per 128-pixel tile), Kd unused.
   int conv;
   int cv_ck, cv_stride, cv_hout, cv_wout;
+  // split-K (SIMT): with ws (ws_floats floats) a long reduction over few output tiles may be cut
+  // into up to ws_floats / (G M N) contiguous k ranges, each CTA's raw sums going to
+  // ws[g][split][m][n] and a second kernel adding them in split order before the epilogue
+  float* ws;
+  int64_t ws_floats;
 };
 // Persistent implicit-GEMM 3x3 convolution (zero padding 1): out[g][p][n] (fp32, replica stride
 // out_gs) = sum over taps t and k < ck of in[g][shift_t(p)][k] w[g][n][t][k].  in_map: the rank-5

@@ -75,6 +75,8 @@ struct lsgd_ctx {
   float* tb = nullptr;
   // host mini-batches (lsgd_local_step_batch): two staging buffers filled on a copy stream, so
   // the next batch's host-to-device copy overlaps the current step
+  float* simt_ws = nullptr;  // split-K partials of the SIMT forward products (fp32 mode)
+  int64_t simt_ws_floats = 0;
   float* xstage[2] = {nullptr, nullptr};
   void* lstage[2] = {nullptr, nullptr};  // labels (int32) or targets (fp32)
   cudaStream_t copy_stream = nullptr;
@@ -403,6 +405,8 @@ lsgd_status dense_forward(lsgd_ctx* c, int groups, int w_g0, int w_gmul, bool sk
     g.epi = epi;
     g.bias = Ly.b_off >= 0 ? c->W + (int64_t)w_g0 * c->d_pad + Ly.b_off : nullptr;
     g.bias_gs = (int64_t)w_gmul * c->d_pad;
+    g.ws = c->simt_ws;
+    g.ws_floats = c->simt_ws_floats;
     lsgd_status st = gemm(c, g);
     if (st != LSGD_OK) return st;
   }
@@ -852,6 +856,10 @@ lsgd_status lsgd_create(const lsgd_config* cfg, const lsgd_allocator* alloc, voi
   c->G = (float*)dalloc(c, n_rep * 4);
   if (c0.momentum != 0.0) c->U = (float*)dalloc(c, n_rep * 4);
   if (c->bf16) c->Wb = (uint16_t*)dalloc(c, n_rep * 2);
+  if (!c->bf16 && !c->resnet) {
+    c->simt_ws_floats = 1 << 20;
+    c->simt_ws = (float*)dalloc(c, (size_t)c->simt_ws_floats * 4);
+  }
   c->idx = (int32_t*)dalloc(c, (size_t)K * B * 4);
   c->yb = (int32_t*)dalloc(c, (size_t)K * B * 4);
   c->tb = (float*)dalloc(c, (size_t)K * B * 4);

@@ -331,6 +331,17 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
   // values (bias / ReLU applied), writes them to a padded shared-memory staging tile, and the CTA
   // then stores the chunk row-contiguously (a warp writes two 256-byte row segments per
   // instruction), applying the ReLU mask from a coalesced read of the stored activation.
+  // The bias that the column sums below update (threads 0-63, one column of each 64-column
+  // chunk; nothing else writes it) is requested now, while the main loop still runs.
+  float bsw[BN / 64], bsu[BN / 64];
+#pragma unroll
+  for (int i = 0; i < BN / 64; ++i) {
+    const int n = n0 + 64 * i + (int)threadIdx.x;
+    const bool v = args.bias_colsum && args.bsgd.w && threadIdx.x < 64 && n < args.N;
+    const int64_t k = (int64_t)g * args.bias_gs + n;
+    bsw[i] = v ? args.bsgd.w[k] : 0.f;
+    bsu[i] = v && args.bsgd.u ? args.bsgd.u[k] : 0.f;
+  }
   const bool have_acc = mbar_wait(&sm.accum, 0);
   asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
   if (have_acc) {
@@ -464,7 +475,7 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
             args.bias_grad[k] = gb;
           } else {
             const SgdParams& sp = args.bsgd;
-            float w = sp.w[k], u = sp.u ? sp.u[k] : 0.f;
+            float w = bsw[cc / CW], u = bsu[cc / CW];
             const bool sg = sp.sign != 0;
             if (sp.mom == 0.f)
               sgd_elem<false, false>(w, u, gb, sp.lr, 0.f, sp.wd, sg);

@@ -85,7 +85,13 @@ __global__ void sample_reshuffle_kernel(int32_t* __restrict__ idx, uint32_t k0, 
 }
 
 // ---------------------------------------------------------------------------------------------
-// One CTA per gathered row; float4 loads, bf16x4 (8-byte) or float4 stores.
+// One CTA per gathered row; float4 loads, bf16x4 (8-byte) or float4 stores.  Each thread has
+// kGatherVec of its row's float4 loads in flight at once, and the launcher sizes the CTA so that a
+// row takes one such batch where it can (96 threads for D = 3072): nearly every row of a
+// K x B_loc = 2048-row mini-batch is then resident at once, and the copy costs two memory round
+// trips (the index, then the row) rather than one per float4 of a thread.
+constexpr int kGatherVec = 8;
+
 template <bool BF16>
 __global__ void gather_rows_kernel(void* __restrict__ dst, int ld_dst, const float* __restrict__ X,
                                    int D, const int32_t* __restrict__ idx, int rows,
@@ -101,26 +107,36 @@ __global__ void gather_rows_kernel(void* __restrict__ dst, int ld_dst, const flo
     if (t_out) t_out[r] = t_in[src_row];
   }
   const bool vec = ((D & 3) == 0) && ((ld_dst & 3) == 0);
-  if (BF16) {
-    uint16_t* d = reinterpret_cast<uint16_t*>(dst) + (int64_t)r * ld_dst;
-    if (vec) {
-      for (int c = threadIdx.x; c < D / 4; c += blockDim.x) {
-        const float4 v = __ldg(reinterpret_cast<const float4*>(src) + c);
-        uint2 o;
-        o.x = (uint32_t)f2bf(v.x) | ((uint32_t)f2bf(v.y) << 16);
-        o.y = (uint32_t)f2bf(v.z) | ((uint32_t)f2bf(v.w) << 16);
-        reinterpret_cast<uint2*>(d)[c] = o;
-      }
-    } else {
-      for (int c = threadIdx.x; c < D; c += blockDim.x) d[c] = f2bf(src[c]);
+  if (!vec) {
+    for (int c = threadIdx.x; c < D; c += blockDim.x) {
+      if (BF16)
+        reinterpret_cast<uint16_t*>(dst)[(int64_t)r * ld_dst + c] = f2bf(src[c]);
+      else
+        reinterpret_cast<float*>(dst)[(int64_t)r * ld_dst + c] = src[c];
     }
-  } else {
-    float* d = reinterpret_cast<float*>(dst) + (int64_t)r * ld_dst;
-    if (vec) {
-      for (int c = threadIdx.x; c < D / 4; c += blockDim.x)
-        reinterpret_cast<float4*>(d)[c] = __ldg(reinterpret_cast<const float4*>(src) + c);
-    } else {
-      for (int c = threadIdx.x; c < D; c += blockDim.x) d[c] = src[c];
+    return;
+  }
+  const int n4 = D / 4;
+  const float4* s4 = reinterpret_cast<const float4*>(src);
+  for (int c0 = threadIdx.x; c0 < n4; c0 += kGatherVec * blockDim.x) {
+    float4 v[kGatherVec];
+#pragma unroll
+    for (int i = 0; i < kGatherVec; ++i) {
+      const int c = c0 + i * blockDim.x;
+      if (c < n4) v[i] = __ldg(s4 + c);
+    }
+#pragma unroll
+    for (int i = 0; i < kGatherVec; ++i) {
+      const int c = c0 + i * blockDim.x;
+      if (c >= n4) break;
+      if (BF16) {
+        uint2 o;
+        o.x = (uint32_t)f2bf(v[i].x) | ((uint32_t)f2bf(v[i].y) << 16);
+        o.y = (uint32_t)f2bf(v[i].z) | ((uint32_t)f2bf(v[i].w) << 16);
+        reinterpret_cast<uint2*>(reinterpret_cast<uint16_t*>(dst) + (int64_t)r * ld_dst)[c] = o;
+      } else {
+        reinterpret_cast<float4*>(reinterpret_cast<float*>(dst) + (int64_t)r * ld_dst)[c] = v[i];
+      }
     }
   }
 }
@@ -626,7 +642,9 @@ cudaError_t launch_gather_rows(void* dst, bool dst_bf16, int ld_dst, const float
                                cudaStream_t stream) {
   if (rows <= 0) return cudaSuccess;
   if (ld_dst < D) return cudaErrorInvalidValue;
-  const int threads = D >= 1024 ? 256 : 128;
+  // one batch of kGatherVec float4 loads per thread covers the row: 96 threads for D = 3072
+  const int per_row = ((D / 4 + kGatherVec - 1) / kGatherVec + 31) / 32 * 32;
+  const int threads = std::min(256, std::max(32, per_row));
   if (dst_bf16)
     launch_pdl(gather_rows_kernel<true>, rows, threads, 0, stream, dst, ld_dst, X, D, idx, rows, labels_in,
                                                            labels_out, targets_in, targets_out);

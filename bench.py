@@ -51,7 +51,7 @@ AVERAGE_BYTES_PER_PARAM = 10
 # the weight-gradient + update launch of both hidden layers), from the ncu capture summarised in
 # profiles/step_kernels_mlp3072_K16_B128.md (below the algorithmic bytes because part of the
 # launch's writes is still in L2 when it ends).
-UPDATE_TRAFFIC_PER_STEP = 1186162688
+UPDATE_TRAFFIC_PER_STEP = 1186195456
 
 FALLBACK_HBM_GBS = 6800.0
 FALLBACK_BF16_TFLOPS = 1900.0

@@ -20,7 +20,7 @@ def P():
 
 SHAPES = [(128, 128, 64, 1), (128, 1024, 3072, 2), (1024, 3072, 128, 2), (40, 136, 264, 3),
           (128, 10, 1024, 2), (128, 1024, 16, 2), (10, 1024, 128, 2), (100, 256, 128, 1),
-          (128, 64, 72, 2)]
+          (128, 64, 72, 2), (200, 136, 2104, 2)]
 
 
 def _operands(torch, M, N, Kd, G, a_mn, b_mn, seed):

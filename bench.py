@@ -57,6 +57,24 @@ FALLBACK_HBM_GBS = 6800.0
 FALLBACK_BF16_TFLOPS = 1900.0
 
 
+def dense_params(widths):
+    """Parameters per replica of a dense network: weights and biases of every layer."""
+    return sum(a * b + b for a, b in zip(widths[:-1], widths[1:]))
+
+
+def workload_config(w, K, world, fused=True):
+    """The workload description both arms print (the timed region's own facts are added by the
+    GPU arm)."""
+    B, H, T_job = w["B"], w["H"], job_steps(w, K)
+    return {"workload": w["name"] if K == w["K"] else w["name"].replace("K16", f"K{K}"),
+            "global_batch": K * B, "K": K, "B_loc": B, "H": H, "fused_update": fused,
+            "job": f"{T_job}-step schedule ({w['epochs']:g} epochs of N = {w['N']}), "
+                   "repeated from its end state",
+            "params_per_replica": dense_params(w["widths"]),
+            "parallelism": "replicas" if world > 1 else "single",
+            "l2": "per-step working set (w, u, g, shadow: 1.0 GB) exceeds the 129 MB L2"}
+
+
 def _peaks():
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
@@ -201,7 +219,7 @@ def run_reference(args, world, rank):
         "value": v, "unit": "samples/s", "n_gpus": args.gpus, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": 1000.0 * t / steps, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": w["name"], "global_batch": w["K"] * w["B"], "parallelism": "replicas"},
+        "config": workload_config(w, w["K"], world),
         "cpu_baseline": {"value": v, "unit": "samples/s", "cores": 1, "kind": "oracle",
                          "sample": sample},
         "e2e": {"value": v, "unit": "samples/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
@@ -670,13 +688,7 @@ def main():
         "value": value, "unit": "samples/s", "n_gpus": world, "steps": S_, "warmup": W_,
         "ms_per_step": t_ms / S_, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": {"workload": w["name"] if K == w["K"] else w["name"].replace("K16", f"K{K}"),
-                   "global_batch": K * B, "K": K, "B_loc": B, "H": H, "fused_update": fused,
-                   "job": f"{T_job}-step schedule ({w['epochs']:g} epochs of N = {w['N']}), "
-                          "repeated from its end state",
-                   "params_per_replica": d, "parallelism": "replicas" if world > 1 else "single",
-                   "l2": "per-step working set (w, u, g, shadow: 1.0 GB) exceeds the 129 MB L2",
-                   "syncs_in_timed_region": n_syncs},
+        "config": dict(workload_config(w, K, world, fused), syncs_in_timed_region=n_syncs),
         "e2e": {"value": e2e_value, "unit": "samples/s", "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h},
         "gpu_launches": launches,

@@ -1,7 +1,8 @@
 """The benchmark's reference arm on CPU: `bench.py --impl reference` times the oracle on a bounded
 sample of the benchmark workload and prints one JSON line with the GPU arm's metric, unit,
 direction and workload description, a `cpu_baseline` describing the run and an end-to-end entry
-with no host-device copies.  Also the helpers that describe the workload."""
+with no host-device copies.  Also the helpers that describe the workload and summarise the
+nvidia-smi clock samples taken during a timed region."""
 import json
 import os
 import subprocess
@@ -49,3 +50,19 @@ def test_reference_arm_prints_one_contract_line():
     assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["value"] == d["value"] and cb["sample"]
     assert d["e2e"] == {"value": d["value"], "unit": d["unit"], "h2d_bytes_per_step": 0,
                         "d2h_bytes_per_step": 0}
+
+
+def test_clock_summary_reads_nvidia_smi_rows():
+    rows = [
+        "0, 2070, 2070, 812.31, 0x0000000000000000, Not Active, Not Active, Not Active, Not Active\n",
+        "0, 1980, 2070, 1391.02, 0x0000000000000004, Not Active, Not Active, Not Active, Active\n",
+        "0, 2070, 2070, 1020.50, 0x0000000000000000, Not Active, Not Active, Not Active, Not Active\n",
+        "0, [N/A], 2070, 1.0, 0x0, Not Active, Not Active, Not Active, Not Active\n",  # unusable
+        "garbage\n",
+    ]
+    c = bench.summarise_clocks(rows)
+    assert c == {"sm_mhz": 2070.0, "sm_max_mhz": 2070.0, "reasons": ["sw_power_cap"], "samples": 3}
+    hot = rows[:1] + ["0, 1500, 2070, 900.0, 0x48, Active, Not Active, Active, Not Active\n"]
+    c = bench.summarise_clocks(hot)
+    assert c["reasons"] == ["hw_slowdown", "sw_thermal_slowdown"] and c["sm_mhz"] == 1785.0
+    assert bench.summarise_clocks(["garbage\n"]) is None

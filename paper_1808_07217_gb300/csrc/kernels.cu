@@ -292,12 +292,41 @@ __global__ void __launch_bounds__(256) sgd_update_kernel(
 }
 
 // ---------------------------------------------------------------------------------------------
-// K-way average.  A thread owns one float4 column of every replica of its group and forms the
-// mean as w^0 + (1/K) sum_k (w^k - w^0), summing in replica order with eight loads in flight (a
-// warp's load instruction reads 512 contiguous bytes of one replica); it writes the mean back to
-// every replica (fp32 and bf16).  The differences are small and nearly exact while the replicas
-// stay close, so the mean carries about one rounding of w instead of K, and the mean of identical
-// replicas is exactly that replica for every K.
+// K-way average (Eq. 2 right).  A thread owns one float4 column of every replica of its group and
+// walks the replicas in order with eight loads in flight (a warp's load instruction reads 512
+// contiguous bytes of one replica).  The sum is accumulated without loss: every addition is an
+// error-free transformation (Knuth's TwoSum: s + x = t + e exactly), the rounding errors e are
+// summed in a second register, and the pair (s, c) is divided by K with the remainder of the first
+// quotient taken exactly by an fma.  The result is the correctly rounded fp32 mean in all but
+// hard midpoint cases, whatever K (a plain fp32 sum loses up to K - 1 roundings), and the mean of
+// identical replicas is that replica.  A column-per-thread walk keeps every load coalesced; a
+// shuffle reduction across lanes would need lanes to hold different replicas of one column.
+struct TwoSum4 {
+  float4 s, c;
+};
+
+__device__ __forceinline__ void two_sum_add(float& s, float& c, float x) {
+  const float t = __fadd_rn(s, x);
+  const float z = __fsub_rn(t, s);
+  const float e = __fadd_rn(__fsub_rn(s, __fsub_rn(t, z)), __fsub_rn(x, z));
+  s = t;
+  c = __fadd_rn(c, e);
+}
+
+__device__ __forceinline__ void two_sum_add4(TwoSum4& a, const float4& v) {
+  two_sum_add(a.s.x, a.c.x, v.x);
+  two_sum_add(a.s.y, a.c.y, v.y);
+  two_sum_add(a.s.z, a.c.z, v.z);
+  two_sum_add(a.s.w, a.c.w, v.w);
+}
+
+// (s + c) / K: q = s / K, the exact remainder s - q K by fma, corrected by c and divided again.
+__device__ __forceinline__ float mean_of(float s, float c, float Kf) {
+  const float q = __fdiv_rn(s, Kf);
+  const float r = __fadd_rn(__fmaf_rn(-q, Kf, s), c);
+  return __fadd_rn(q, __fdiv_rn(r, Kf));
+}
+
 template <bool SHADOW>
 __global__ void __launch_bounds__(256) kway_average_kernel(float4* __restrict__ W,
                                                            uint2* __restrict__ Wb, int K,
@@ -306,40 +335,23 @@ __global__ void __launch_bounds__(256) kway_average_kernel(float4* __restrict__ 
   // blockIdx.y selects a group of K consecutive replicas (one group for the global average)
   W += (int64_t)blockIdx.y * K * d4;
   if (SHADOW) Wb += (int64_t)blockIdx.y * K * d4;
-  const float invK = 1.0f / (float)K;
-  const bool exactK = (K & (K - 1)) == 0;
+  const float Kf = (float)K;
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   for (int64_t col = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; col < d4; col += stride) {
-    const float4 w0 = W[col];
-    float4 s = make_float4(0.f, 0.f, 0.f, 0.f);
-    int k = 0;
+    TwoSum4 acc;
+    acc.s = __ldcs(W + col);
+    acc.c = make_float4(0.f, 0.f, 0.f, 0.f);
+    int k = 1;
     for (; k + 8 <= K; k += 8) {
       float4 v[8];
 #pragma unroll
       for (int q = 0; q < 8; ++q) v[q] = __ldcs(W + (int64_t)(k + q) * d4 + col);
 #pragma unroll
-      for (int q = 0; q < 8; ++q) {
-        s.x += v[q].x - w0.x;
-        s.y += v[q].y - w0.y;
-        s.z += v[q].z - w0.z;
-        s.w += v[q].w - w0.w;
-      }
+      for (int q = 0; q < 8; ++q) two_sum_add4(acc, v[q]);
     }
-    for (; k < K; ++k) {
-      const float4 v = __ldcs(W + (int64_t)k * d4 + col);
-      s.x += v.x - w0.x;
-      s.y += v.y - w0.y;
-      s.z += v.z - w0.z;
-      s.w += v.w - w0.w;
-    }
-    float4 mean;
-    if (exactK) {
-      mean = make_float4(fmaf(s.x, invK, w0.x), fmaf(s.y, invK, w0.y), fmaf(s.z, invK, w0.z),
-                         fmaf(s.w, invK, w0.w));
-    } else {
-      mean = make_float4(w0.x + s.x / (float)K, w0.y + s.y / (float)K, w0.z + s.z / (float)K,
-                         w0.w + s.w / (float)K);
-    }
+    for (; k < K; ++k) two_sum_add4(acc, __ldcs(W + (int64_t)k * d4 + col));
+    const float4 mean = make_float4(mean_of(acc.s.x, acc.c.x, Kf), mean_of(acc.s.y, acc.c.y, Kf),
+                                    mean_of(acc.s.z, acc.c.z, Kf), mean_of(acc.s.w, acc.c.w, Kf));
     uint2 o;
     if (SHADOW) {
       o.x = (uint32_t)f2bf(mean.x) | ((uint32_t)f2bf(mean.y) << 16);

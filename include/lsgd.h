@@ -360,6 +360,28 @@ lsgd_status lsgd_batchnorm_stats(const float* y, int64_t P, int C, int G, float*
 lsgd_status lsgd_conv_wgrad_bf16(const uint16_t* x, const uint16_t* dy, float* dW, int G, int B,
                                  int Hout, int Wout, int Cin, int Cout, int stride, void* stream);
 
+/* A 3x3 convolution with zero padding 1 and stride s (1 or 2) for G independent groups on the
+ * persistent implicit-GEMM tensor-core kernel, through the same code the ResNet-20 step runs
+ * (Sec. A.2's network; 3x3 convolutions of He et al. 2016).  W [G][Cout][3][3][Cin] bf16.
+ *  mode 0, forward:  out[g][b][oy][ox][co] = sum over kh, kw, ci of
+ *          in[g][b][oy s + kh - 1][ox s + kw - 1][ci] W[g][co][kh][kw][ci]  (in zero outside the image)
+ *          with in = x [G][B][Hin][Win][Cin] and out = y [G][B][Hout][Wout][Cout], Hout =
+ *          (Hin - 1) / s + 1; Cin < 16 runs the stem form (image and weights padded with zero
+ *          channels to 16).
+ *  mode 1, data gradient: out[g][b][iy][ix][ci] = sum over (oy, ox, kh, kw) with
+ *          iy = oy s + kh - 1, ix = ox s + kw - 1 and co of in[g][b][oy][ox][co] W[g][co][kh][kw][ci]
+ *          with in = dy [G][B][Hout][Wout][Cout] and out = dx [G][B][Hin][Win][Cin]; stride 1 as
+ *          a convolution with the flipped, transposed weights, stride 2 as four parity phases.
+ * bf16 operands, fp32 accumulation; `out` fp32, fully overwritten.  Device pointers, in and W
+ * 16-byte aligned, asynchronous on `stream`; scratch (the padded stem operands or the flipped
+ * weights) is allocated and freed on `stream`.  LSGD_EINVAL on bad arguments, LSGD_EUNSUPPORTED
+ * for shapes the kernel does not take (it needs 16, 32 or 64 channels per tap, Cout and Cin (mode
+ * 1) of 16, 32 or 64, and an output whose whole rows tile into 128-pixel blocks), LSGD_ENOMEM if
+ * the scratch cannot be allocated. */
+lsgd_status lsgd_conv3x3_bf16(int mode, const uint16_t* in, const uint16_t* W, float* out, int G,
+                              int B, int Hin, int Win, int Cin, int Cout, int stride,
+                              void* stream);
+
 /* lsgd_batchnorm_stats for callers that cannot allocate device memory during a run: a program
  * whose device memory is all handed to its own caching pool (an allocation would fail, or force
  * the pool to give memory back and stall), or a latency-critical loop that fixes its memory use at

@@ -42,7 +42,7 @@ EXPORTS = [
     "lsgd_batchnorm_stats_noalloc", "lsgd_block_average", "lsgd_block_sync_count",
     "lsgd_sync_state", "lsgd_set_sync_state", "lsgd_schedule", "lsgd_device_status",
     "lsgd_bounded_wait_selftest", "lsgd_losses_async", "lsgd_synchronize", "lsgd_set_step",
-    "lsgd_conv_wgrad_bf16",
+    "lsgd_conv_wgrad_bf16", "lsgd_conv3x3_bf16",
 ]
 PHASES = ["input", "forward", "loss", "backward", "update", "average"]
 
@@ -169,6 +169,7 @@ def lib():
             "lsgd_step_count": ([vp], i64),
             "lsgd_set_step": ([vp, i64], st),
             "lsgd_conv_wgrad_bf16": ([vp, vp, vp] + [ctypes.c_int] * 7 + [vp], st),
+            "lsgd_conv3x3_bf16": ([ctypes.c_int, vp, vp, vp] + [ctypes.c_int] * 7 + [vp], st),
             "lsgd_sync_count": ([vp], i64),
             "lsgd_block_sync_count": ([vp], i64),
             "lsgd_block_average": ([vp], st),
@@ -500,6 +501,21 @@ def lsgd_conv_wgrad_bf16(x, dy, dW, G: int, B: int, Hout: int, Wout: int, Cin: i
     _check(lib().lsgd_conv_wgrad_bf16(_ptr(x), _ptr(dy), _ptr(dW), int(G), int(B), int(Hout),
                                       int(Wout), int(Cin), int(Cout), int(stride),
                                       ctypes.c_void_p(stream)))
+
+
+CONV_FORWARD, CONV_DGRAD = 0, 1
+
+
+def lsgd_conv3x3_bf16(mode: int, inp, W, out, G: int, B: int, Hin: int, Win: int, Cin: int,
+                      Cout: int, stride: int, stream=None):
+    """3x3 (pad 1, stride) convolution of NHWC bfloat16 CUDA tensors on the implicit-GEMM kernel:
+    mode CONV_FORWARD: out [G, B, Hout, Wout, Cout] float32 from inp = x [G, B, Hin, Win, Cin];
+    mode CONV_DGRAD: out = dx [G, B, Hin, Win, Cin] float32 from inp = dy [G, B, Hout, Wout, Cout];
+    W [G, Cout, 3, 3, Cin] bfloat16."""
+    stream = _current_stream() if stream is None else stream
+    _check(lib().lsgd_conv3x3_bf16(int(mode), _ptr(inp), _ptr(W), _ptr(out), int(G), int(B),
+                                   int(Hin), int(Win), int(Cin), int(Cout), int(stride),
+                                   ctypes.c_void_p(stream)))
 
 
 def lsgd_batchnorm_stats(y, P: int, C: int, G: int, mean, rstd, stream=None):

@@ -1147,39 +1147,182 @@ unsigned px_blocks(int64_t P, int C) {
   return (unsigned)std::max<int64_t>(1, std::min<int64_t>((P + ppb - 1) / ppb, (int64_t)kNumSMs * 8));
 }
 
+// ---- 3x3 convolutions on the persistent implicit-GEMM kernel (conv_tc_kernel), raw pointers ----
+// The ResNet-20 step and the stand-alone lsgd_conv3x3_bf16 entry point both run these, so the
+// element-wise kernel tests cover the step's own launches.  Weights w [G][Cout][3][3][Cin] bf16
+// with replica stride w_gs; activations NHWC bf16; outputs fp32, fully overwritten.
+
+#define CV_LAUNCH(expr)                                                              \
+  do {                                                                               \
+    expr;                                                                            \
+    if (launches) ++*launches;                                                       \
+    const cudaError_t e__ = cudaGetLastError();                                      \
+    if (e__ != cudaSuccess) {                                                        \
+      err = std::string(#expr) + ": " + cudaGetErrorString(e__);                     \
+      return LSGD_ECUDA;                                                             \
+    }                                                                                \
+  } while (0)
+#define CV_CALL(expr)                                                                \
+  do {                                                                               \
+    if (launches) ++*launches;                                                       \
+    const cudaError_t e__ = (expr);                                                  \
+    if (e__ != cudaSuccess) {                                                        \
+      err = std::string(#expr) + ": " + cudaGetErrorString(e__);                     \
+      return LSGD_ECUDA;                                                             \
+    }                                                                                \
+  } while (0)
+
+// Output size of a 3x3, padding-1 convolution.
+int conv_out_size(int n, int stride) { return (n - 1) / stride + 1; }
+
+// The forward y = conv(x, w) runs on the implicit kernel: the stem form (fewer than 16 input
+// channels, padded to 16) or the direct form (16, 32 or 64 channels per tap).
+bool conv_fwd_tc_route(int B, int hin, int win, int cin, int cout, int stride) {
+  const int hout = conv_out_size(hin, stride), wout = conv_out_size(win, stride);
+  const int64_t P = (int64_t)B * hout * wout;
+  if (cout % 8 || P > 0x7fffffffLL) return false;
+  if (cin < 16)
+    return stride == 1 && implicit_conv_ok(16, 1, hout, wout) && persistent_conv_ok(cout, P);
+  return implicit_conv_ok(cin, stride, hout, wout) && persistent_conv_ok(cout, P);
+}
+
+// The data gradient dx = conv^T(dy, w) runs on the implicit kernel: stride 1 as a convolution of
+// dy with the flipped, transposed weights; stride 2 as four parity phases.
+bool conv_dgrad_tc_route(int B, int hin, int win, int cin, int cout, int stride) {
+  const int hout = conv_out_size(hin, stride), wout = conv_out_size(win, stride);
+  if (cout % 8 || cin % 8 || (int64_t)B * hin * win > 0x7fffffffLL) return false;
+  if (stride == 1) return implicit_conv_ok(cout, 1, hin, win) && persistent_conv_ok(cin, (int64_t)B * hin * win);
+  return stride == 2 && hin == 2 * hout && win == 2 * wout && implicit_conv_ok(cout, 1, hout, wout) &&
+         persistent_conv_ok(cin, (int64_t)B * hout * wout);
+}
+
+// Scratch of the forward's stem form (x16 [G][B][hin][win][16], wstem [G][cout][9][16]) and of
+// the data gradient (stride 1: wt [G][cin][9][cout]; stride 2: wt4 [4][G][cin][9][cout]), bf16.
+size_t conv_x16_elems(int G, int B, int hin, int win) { return (size_t)G * B * hin * win * 16; }
+size_t conv_wstem_elems(int G, int cout) { return (size_t)G * cout * 9 * 16; }
+size_t conv_wt_elems(int G, int cin, int cout, int stride) {
+  return (size_t)(stride == 2 ? 4 : 1) * G * cin * 9 * cout;
+}
+
+lsgd_status conv_fwd_tc(const uint16_t* x, const uint16_t* w, int64_t w_gs, float* y, int G, int B,
+                        int hin, int win, int cin, int cout, int stride, uint16_t* x16,
+                        uint16_t* wstem, cudaStream_t s, std::string& err, int64_t* launches) {
+  if (!conv_fwd_tc_route(B, hin, win, cin, cout, stride)) {
+    err = "convolution shape not taken by the implicit-GEMM kernel";
+    return LSGD_EUNSUPPORTED;
+  }
+  const int hout = conv_out_size(hin, stride), wout = conv_out_size(win, stride);
+  const int64_t P = (int64_t)B * hout * wout;
+  ConvArgs ca{};
+  bool okc;
+  if (cin < 16) {
+    // the stem: zero channels appended to the image and the weights (the products are unchanged)
+    const int64_t npix = (int64_t)G * B * hin * win;
+    CV_LAUNCH(launch_pdl(pad_input16_kernel, grid_cap(npix, 256), 256, 0, s, x, x16, npix, cin));
+    CV_LAUNCH(launch_pdl(pad_stem_weights_kernel, grid_cap((int64_t)G * cout * 144, 256), 256, 0, s,
+                         w, w_gs, (int64_t)0, wstem, G, cout, cin));
+    okc = make_tma_map_conv(&ca.in_map, x16, 16, win, hin, B, G, wout, hout, 1);
+    okc &= make_tma_map(&ca.w_map, wstem, true, 9 * 16, cout, G, 9 * 16, (uint64_t)cout * 9 * 16, 16,
+                        cout, 32);
+    ca.ck = 16;
+  } else {
+    okc = make_tma_map_conv(&ca.in_map, x, cin, win, hin, B, G, wout, hout, stride);
+    okc &= make_tma_map(&ca.w_map, w, true, 9 * cin, cout, G, 9 * cin, w_gs, cin, cout, 2 * cin);
+    ca.ck = cin;
+  }
+  if (!okc) {
+    err = "TMA map encoding failed (implicit convolution)";
+    return LSGD_ECUDA;
+  }
+  ca.stride = cin < 16 ? 1 : stride;
+  ca.hout = hout;
+  ca.wout = wout;
+  ca.N = ca.np = cout;
+  ca.G = G;
+  ca.P = (int)P;
+  ca.out = y;
+  ca.out_gs = P * cout;
+  CV_CALL(launch_conv_tc(ca, s));
+  return LSGD_OK;
+}
+
+lsgd_status conv_dgrad_tc(const uint16_t* dy, const uint16_t* w, int64_t w_gs, float* dx, int G,
+                          int B, int hin, int win, int cin, int cout, int stride, uint16_t* wt,
+                          cudaStream_t s, std::string& err, int64_t* launches) {
+  if (!conv_dgrad_tc_route(B, hin, win, cin, cout, stride)) {
+    err = "data-gradient shape not taken by the implicit-GEMM kernel";
+    return LSGD_EUNSUPPORTED;
+  }
+  const int64_t P = (int64_t)B * hin * win;
+  if (stride == 1) {
+    CV_LAUNCH((launch_pdl(flip_weights_kernel, dim3((unsigned)((cin * 9 * cout + 255) / 256), (unsigned)G),
+                          256, 0, s, w, w_gs, (int64_t)0, wt, G, cin, cout)));
+    ConvArgs ca{};
+    bool okc = make_tma_map_conv(&ca.in_map, dy, cout, win, hin, B, G, win, hin, 1);
+    okc &= make_tma_map(&ca.w_map, wt, true, 9 * cout, cin, G, 9 * cout, (uint64_t)cin * 9 * cout,
+                        cout, cin, 2 * cout);
+    if (!okc) {
+      err = "TMA map encoding failed (implicit data gradient)";
+      return LSGD_ECUDA;
+    }
+    ca.ck = cout;
+    ca.stride = 1;
+    ca.hout = hin;
+    ca.wout = win;
+    ca.N = ca.np = cin;
+    ca.G = G;
+    ca.P = (int)P;
+    ca.out = dx;
+    ca.out_gs = P * cin;
+    CV_CALL(launch_conv_tc(ca, s));
+    return LSGD_OK;
+  }
+  // stride 2: each parity phase of dx is a 3x3 stride-1 convolution of dy (weights of the phase's
+  // taps, zeros elsewhere) whose outputs land on every other row and column of dx
+  const int hout = hin / 2, wout = win / 2;
+  const int64_t per = (int64_t)cin * 9 * cout;
+  CV_LAUNCH(launch_pdl(flip_phase_weights_kernel, grid_cap(4 * (int64_t)G * per, 256), 256, 0, s,
+                       w, w_gs, (int64_t)0, wt, G, cin, cout));
+  const int64_t Pq = (int64_t)B * hout * wout;
+  for (int ph = 0; ph < 4; ++ph) {
+    ConvArgs ca{};
+    bool okc = make_tma_map_conv(&ca.in_map, dy, cout, wout, hout, B, G, wout, hout, 1);
+    okc &= make_tma_map(&ca.w_map, wt + ph * G * per, true, 9 * cout, cin, G, 9 * cout,
+                        (uint64_t)per, cout, cin, 2 * cout);
+    if (!okc) {
+      err = "TMA map encoding failed (stride-2 data gradient)";
+      return LSGD_ECUDA;
+    }
+    ca.ck = cout;
+    ca.stride = 1;
+    ca.hout = hout;
+    ca.wout = wout;
+    ca.N = ca.np = cin;
+    ca.G = G;
+    ca.P = (int)Pq;
+    ca.out = dx;
+    ca.out_gs = P * cin;
+    ca.ph_y = ph >> 1;
+    ca.ph_x = ph & 1;
+    ca.dst_h = hin;
+    ca.dst_w = win;
+    CV_CALL(launch_conv_tc(ca, s));
+  }
+  return LSGD_OK;
+}
+
 template <typename TA>
 lsgd_status conv_forward(ResNetPlan* p, int i, const void* in, const void* Wop, int w_g0,
                          int w_gmul, float* y, int G, cudaStream_t s, int64_t* launches) {
   const ConvL& c = p->convs[i];
   const int64_t P = conv_pixels(p, c);
   if (i == 0 && p->stem16 && w_g0 == 0 && w_gmul == 1) {
-    // the stem as a 16-channel convolution: zero channels appended to the image and the weights
-    // (the products are unchanged), then the persistent implicit-GEMM kernel
-    const int64_t npix = (int64_t)G * P;
-    RN_LAUNCH(launch_pdl(pad_input16_kernel, grid_cap(npix, 256), 256, 0, s,
-                         reinterpret_cast<const uint16_t*>(in), p->x16, npix, c.cin));
-    RN_LAUNCH(launch_pdl(pad_stem_weights_kernel, grid_cap((int64_t)G * c.cout * 144, 256), 256, 0,
-                         s, reinterpret_cast<const uint16_t*>(Wop), p->d_pad, c.w_off, p->wstem, G,
-                         c.cout, c.cin));
-    ConvArgs ca{};
-    bool okc = make_tma_map_conv(&ca.in_map, p->x16, 16, c.win, c.hin, p->B, G, c.wout, c.hout, 1);
-    okc &= make_tma_map(&ca.w_map, p->wstem, true, 9 * 16, c.cout, G, 9 * 16,
-                        (uint64_t)c.cout * 9 * 16, 16, c.cout, 32);
-    if (!okc) {
-      p->err = "TMA map encoding failed (stem convolution)";
-      return LSGD_ECUDA;
-    }
-    ca.ck = 16;
-    ca.stride = 1;
-    ca.hout = c.hout;
-    ca.wout = c.wout;
-    ca.N = ca.np = c.cout;
-    ca.G = G;
-    ca.P = (int)P;
-    ca.out = y;
-    ca.out_gs = P * c.cout;
-    RN_CALL(launch_conv_tc(ca, s));
-    return LSGD_OK;
+    // the stem as a 16-channel convolution on the persistent implicit-GEMM kernel
+    const lsgd_status st = conv_fwd_tc(reinterpret_cast<const uint16_t*>(in),
+                                       reinterpret_cast<const uint16_t*>(Wop) + c.w_off, p->d_pad, y,
+                                       G, p->B, c.hin, c.win, c.cin, c.cout, 1, p->x16, p->wstem, s,
+                                       p->err, launches);
+    return st;
   }
   if (conv_on_tc(p, c) && w_g0 == 0 && w_gmul == 1) {
     // y = im2col(in) [P][9 Cin] x W^T on the tensor cores (both operands K-major)
@@ -1224,26 +1367,8 @@ lsgd_status conv_forward(ResNetPlan* p, int i, const void* in, const void* Wop, 
         persistent_conv_ok(c.cout, P)) {
       // persistent implicit GEMM: the input tile of each tap straight from the NHWC activation
       // by TMA
-      ConvArgs ca{};
-      bool okc = make_tma_map_conv(&ca.in_map, in, c.cin, c.win, c.hin, p->B, G, c.wout, c.hout,
-                                   c.stride);
-      okc &= make_tma_map(&ca.w_map, wop, true, 9 * c.cin, c.cout, G, 9 * c.cin, w_gs, c.cin,
-                          c.cout, 2 * c.cin);
-      if (!okc) {
-        p->err = "TMA map encoding failed (implicit convolution)";
-        return LSGD_ECUDA;
-      }
-      ca.ck = c.cin;
-      ca.stride = c.stride;
-      ca.hout = c.hout;
-      ca.wout = c.wout;
-      ca.N = ca.np = c.cout;
-      ca.G = G;
-      ca.P = (int)P;
-      ca.out = y;
-      ca.out_gs = P * c.cout;
-      RN_CALL(launch_conv_tc(ca, s));
-      return LSGD_OK;
+      return conv_fwd_tc(reinterpret_cast<const uint16_t*>(in), wop, w_gs, y, G, p->B, c.hin, c.win,
+                         c.cin, c.cout, c.stride, nullptr, nullptr, s, p->err, launches);
     }
     if (implicit_conv_ok(c.cin, c.stride, c.hout, c.wout) && Kc == 9 * c.cin) {
       // implicit GEMM: the input tile of each tap straight from the NHWC activation by TMA
@@ -1473,30 +1598,16 @@ lsgd_status conv_dgrad(ResNetPlan* p, int i, const void* Wop, float* dx, const f
   if (conv_on_tc(p, c) && c.stride == 1 && implicit_conv_ok(c.cout, 1, c.hin, c.win)) {
     // stride 1: dx is the convolution of dy with the flipped, transposed weights -- an implicit
     // GEMM over dy's taps, no column matrix
-    RN_LAUNCH((launch_pdl(flip_weights_kernel,
-        dim3((unsigned)((c.cin * 9 * c.cout + 255) / 256), (unsigned)K), 256, 0, s,
-        reinterpret_cast<const uint16_t*>(Wop), p->d_pad, c.w_off, p->wt, K, c.cin, c.cout)));
     if (persistent_conv_ok(c.cin, P)) {
-      ConvArgs ca{};
-      bool okc = make_tma_map_conv(&ca.in_map, p->dy, c.cout, c.wout, c.hout, p->B, K, c.win,
-                                   c.hin, 1);
-      okc &= make_tma_map(&ca.w_map, p->wt, true, 9 * c.cout, c.cin, K, 9 * c.cout,
-                          (uint64_t)c.cin * 9 * c.cout, c.cout, c.cin, 2 * c.cout);
-      if (!okc) {
-        p->err = "TMA map encoding failed (implicit data gradient)";
-        return LSGD_ECUDA;
-      }
-      ca.ck = c.cout;
-      ca.stride = 1;
-      ca.hout = c.hin;
-      ca.wout = c.win;
-      ca.N = ca.np = c.cin;
-      ca.G = K;
-      ca.P = (int)P;
-      ca.out = dx;
-      ca.out_gs = P * c.cin;
-      RN_CALL(launch_conv_tc(ca, s));
+      const lsgd_status st = conv_dgrad_tc(reinterpret_cast<const uint16_t*>(p->dy),
+                                           reinterpret_cast<const uint16_t*>(Wop) + c.w_off, p->d_pad,
+                                           dx, K, p->B, c.hin, c.win, c.cin, c.cout, 1, p->wt, s,
+                                           p->err, launches);
+      if (st != LSGD_OK) return st;
     } else {
+      RN_LAUNCH((launch_pdl(flip_weights_kernel,
+          dim3((unsigned)((c.cin * 9 * c.cout + 255) / 256), (unsigned)K), 256, 0, s,
+          reinterpret_cast<const uint16_t*>(Wop), p->d_pad, c.w_off, p->wt, K, c.cin, c.cout)));
       TcGemmArgs t{};
       t.M = (int)P;
       t.N = c.cin;
@@ -1532,38 +1643,12 @@ lsgd_status conv_dgrad(ResNetPlan* p, int i, const void* Wop, float* dx, const f
     return LSGD_OK;
   }
   if (phase_dgrad_ok(p, c)) {
-    // stride 2: each parity phase of dx is a 3x3 stride-1 convolution of dy (weights of the
-    // phase's taps, zeros elsewhere) whose outputs land on every other row and column of dx
-    const int64_t per = (int64_t)c.cin * 9 * c.cout;
-    RN_LAUNCH(launch_pdl(flip_phase_weights_kernel, grid_cap(4 * (int64_t)K * per, 256), 256, 0, s,
-                         reinterpret_cast<const uint16_t*>(Wop), p->d_pad, c.w_off, p->wt4, K,
-                         c.cin, c.cout));
-    const int64_t Pq = (int64_t)p->B * c.hout * c.wout;
-    for (int ph = 0; ph < 4; ++ph) {
-      ConvArgs ca{};
-      bool okc = make_tma_map_conv(&ca.in_map, p->dy, c.cout, c.wout, c.hout, p->B, K, c.wout,
-                                   c.hout, 1);
-      okc &= make_tma_map(&ca.w_map, p->wt4 + ph * K * per, true, 9 * c.cout, c.cin, K,
-                          9 * c.cout, (uint64_t)per, c.cout, c.cin, 2 * c.cout);
-      if (!okc) {
-        p->err = "TMA map encoding failed (stride-2 data gradient)";
-        return LSGD_ECUDA;
-      }
-      ca.ck = c.cout;
-      ca.stride = 1;
-      ca.hout = c.hout;
-      ca.wout = c.wout;
-      ca.N = ca.np = c.cin;
-      ca.G = K;
-      ca.P = (int)Pq;
-      ca.out = dx;
-      ca.out_gs = P * c.cin;
-      ca.ph_y = ph >> 1;
-      ca.ph_x = ph & 1;
-      ca.dst_h = c.hin;
-      ca.dst_w = c.win;
-      RN_CALL(launch_conv_tc(ca, s));
-    }
+    // stride 2: four parity phases on the persistent implicit-GEMM kernel
+    const lsgd_status st = conv_dgrad_tc(reinterpret_cast<const uint16_t*>(p->dy),
+                                         reinterpret_cast<const uint16_t*>(Wop) + c.w_off, p->d_pad,
+                                         dx, K, p->B, c.hin, c.win, c.cin, c.cout, 2, p->wt4, s,
+                                         p->err, launches);
+    if (st != LSGD_OK) return st;
     if (dout) {
       const int64_t n = (int64_t)p->B * c.hout * c.wout * (c.cin / 4);
       RN_LAUNCH((launch_pdl(add_shortcut_grad_v2_kernel<TA>,
@@ -1723,6 +1808,34 @@ lsgd_status fwd_bwd_impl(ResNetPlan* p, const float* W, const void* Wop, float* 
 size_t batchnorm_stats_scratch_floats(int64_t P, int C, int G) {
   const int64_t nq = (P + kStatChunk - 1) / kStatChunk;
   return (size_t)G * nq * C * 2;
+}
+
+size_t conv3x3_scratch_bytes(int mode, int G, int B, int hin, int win, int cin, int cout,
+                             int stride) {
+  if (mode == 0)
+    return cin < 16 ? (conv_x16_elems(G, B, hin, win) + conv_wstem_elems(G, cout)) * 2 : 0;
+  return conv_wt_elems(G, cin, cout, stride) * 2;
+}
+
+bool conv3x3_tc_route(int mode, int B, int hin, int win, int cin, int cout, int stride) {
+  return mode == 0 ? conv_fwd_tc_route(B, hin, win, cin, cout, stride)
+                   : conv_dgrad_tc_route(B, hin, win, cin, cout, stride);
+}
+
+lsgd_status conv3x3_bf16(int mode, const uint16_t* in, const uint16_t* w, float* out, int G, int B,
+                         int hin, int win, int cin, int cout, int stride, void* scratch,
+                         cudaStream_t s, std::string* err) {
+  std::string e;
+  const int64_t w_gs = (int64_t)cout * 9 * cin;
+  uint16_t* sc = static_cast<uint16_t*>(scratch);
+  lsgd_status st;
+  if (mode == 0)
+    st = conv_fwd_tc(in, w, w_gs, out, G, B, hin, win, cin, cout, stride, sc,
+                     sc ? sc + conv_x16_elems(G, B, hin, win) : nullptr, s, e, nullptr);
+  else
+    st = conv_dgrad_tc(in, w, w_gs, out, G, B, hin, win, cin, cout, stride, sc, s, e, nullptr);
+  if (st != LSGD_OK && err) *err = e;
+  return st;
 }
 
 size_t conv_wgrad_scratch_floats(int G, int B, int hout, int wout, int cin, int cout, int stride) {

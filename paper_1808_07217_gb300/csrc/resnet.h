@@ -50,6 +50,17 @@ size_t conv_wgrad_scratch_floats(int G, int B, int hout, int wout, int cin, int 
 cudaError_t launch_conv_wgrad_bf16(const uint16_t* x, const uint16_t* dy, float* dW, int64_t dW_gs,
                                    int G, int B, int hout, int wout, int cin, int cout, int stride,
                                    float* part, cudaStream_t s, int cin_out = 0);
+// A 3x3 convolution (zero padding 1, stride 1 or 2) of G groups on the persistent implicit-GEMM
+// kernel, exactly as the ResNet-20 step runs it.  mode 0: out = y [G][B][Hout][Wout][cout] from
+// in = x [G][B][hin][win][cin] (cin < 16: the stem form, padded to 16 channels); mode 1: out = dx
+// [G][B][hin][win][cin] from in = dy [G][B][Hout][Wout][cout].  w [G][cout][3][3][cin] bf16,
+// contiguous.  scratch: conv3x3_scratch_bytes bytes of device memory (may be NULL when 0).
+// LSGD_EUNSUPPORTED when conv3x3_tc_route rejects the shape.
+size_t conv3x3_scratch_bytes(int mode, int G, int B, int hin, int win, int cin, int cout, int stride);
+bool conv3x3_tc_route(int mode, int B, int hin, int win, int cin, int cout, int stride);
+lsgd_status conv3x3_bf16(int mode, const uint16_t* in, const uint16_t* w, float* out, int G, int B,
+                         int hin, int win, int cin, int cout, int stride, void* scratch,
+                         cudaStream_t s, std::string* err);
 cudaError_t launch_batchnorm_stats(const float* y, int64_t P, int C, int G, float* mean,
                                    float* rstd, float* part, cudaStream_t s);
 const char* resnet_last_error(const ResNetPlan* p);

@@ -1,24 +1,29 @@
 #!/usr/bin/env python3
-"""Throughput of local SGD over K simulated workers on one GB300 (samples/s).
+"""Throughput of post-local SGD over K simulated workers on one GB300 (samples/s).
 
-Workload: MLP 3072-1024-1024-10 (ReLU, He-normal init), bf16 GEMM operands with fp32 accumulation
-and fp32 master weights, K = 16 workers, B_loc = 128, H = 16, Nesterov momentum 0.9 kept local,
-weight decay 5e-4, lr 0.1 scaled by K with 5-epoch linear warm-up, on N = 50,000 synthetic
-CIFAR-shaped Gaussian-mixture points (32x32x3, 10 classes).  One timed step = one local step of all
-K replicas (sampling, gather + cast, forward, loss, backward, fused update) plus, every H-th step,
-the K-way average.  `value` is device-timed with inputs resident in HBM; `e2e` drives the same
-steps through lsgd_local_step_batch with each step's mini-batch copied from pinned host memory and
-its losses read back.
+Workload (the largest configuration): post-local SGD on MLP 3072-4096-4096-4096-100 (ReLU,
+He-normal init), bf16 GEMM operands with fp32 accumulation and fp32 master weights, K = 16 workers,
+B_loc = 128, 10 epochs of N = 50,000 synthetic CIFAR-100-shaped Gaussian-mixture points (32x32x3,
+100 classes) = a 245-step job; H = 1 (an average after every step) before t' = floor(T / 2) = 122
+and H = 16 after it (Sec. 3, Algorithm 2); Nesterov momentum 0.9 kept local, weight decay 5e-4,
+learning rate 0.1 decayed 10x at 50 % and 75 % of the job.  One timed step = one local step of all
+K replicas (sampling, gather + cast, forward, loss, backward, fused update) plus the K-way average
+when the schedule ends a round there.  `value` is device-timed with inputs resident in HBM; `e2e`
+drives the same steps through lsgd_local_step_batch with each step's mini-batch copied from pinned
+host memory and its losses read back.  The MLP 3072-1024-1024-10 configuration (H = 16, lr 0.1
+scaled by K with warm-up) is timed as well and reported under "config2".
 
---impl reference times the oracle (single-threaded C++, fp64) on the host cores instead.
-Under torchrun (N > 1) every rank runs an independent replica of the workload (no collective on the
-data path); the time is the maximum over ranks.
+--impl reference times the oracle (single-threaded C++, fp64) on the host cores instead, on the
+same bounded sample as the GPU line's cpu_baseline.  Under torchrun (N > 1) every rank runs an
+independent replica of the workload (no collective on the data path); the time is the maximum
+over ranks.
 """
 from __future__ import annotations
 
 import argparse
 import json
 import os
+import platform
 import statistics
 import subprocess
 import sys
@@ -28,16 +33,45 @@ import time
 ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
-WORKLOAD = dict(name="mlp_3072-1024-1024-10_K16_B128_H16_bf16", widths=(3072, 1024, 1024, 10),
-                K=16, B=128, H=16, N=50000, C=10, base_lr=0.1, scale_by_K=True, warmup_epochs=5.0,
-                momentum=0.9, nesterov=True, weight_decay=5e-4, seed=0, data_seed=1234,
-                epochs=2.0)
+# The benchmark workloads.  Learning-rate readings: config 2 states "lr 0.1 scaled by K with
+# 5-epoch linear warmup"; config 3 states only the decays, so its rate is 0.1 without K scaling or
+# warm-up (the scaled rate, 1.6, drives this deep MLP to NaN in its H = 1 phase).
+WORKLOAD = dict(name="mlp_3072-4096x3-100_K16_B128_postlocal_H16_bf16",
+                widths=(3072, 4096, 4096, 4096, 100), K=16, B=128, H=16, N=50000, C=100,
+                epochs=10.0, t_switch_frac=0.5, base_lr=0.1, scale_by_K=False, warmup_epochs=0.0,
+                milestones=(0.5, 0.75), momentum=0.9, nesterov=True, weight_decay=5e-4, seed=0,
+                data_seed=1234, bf16=True, init="he")
+CONFIG2 = dict(name="mlp_3072-1024-1024-10_K16_B128_H16_bf16", widths=(3072, 1024, 1024, 10),
+               K=16, B=128, H=16, N=50000, C=10, epochs=2.0, t_switch_frac=None, base_lr=0.1,
+               scale_by_K=True, warmup_epochs=5.0, milestones=(), momentum=0.9, nesterov=True,
+               weight_decay=5e-4, seed=0, data_seed=1234, bf16=True, init="he")
+SOFTMAX = dict(name="softmax_3072-10_K4_B32_H4_fp32", widths=(3072, 10), K=4, B=32, H=4, N=8192,
+               C=10, epochs=1.0, t_switch_frac=None, base_lr=0.1, scale_by_K=False,
+               warmup_epochs=0.0, milestones=(), momentum=0.0, nesterov=False, weight_decay=0.0,
+               seed=0, data_seed=1234, bf16=False, init="zero", T=64)
+SWEEP = dict(name="mlp_3072-512-512-10_B32", widths=(3072, 512, 512, 10), K=8, B=32, H=1,
+             N=50000, C=10, epochs=1.0, t_switch_frac=None, base_lr=0.1, scale_by_K=False,
+             warmup_epochs=0.0, milestones=(), momentum=0.9, nesterov=False, weight_decay=0.0,
+             seed=0, data_seed=1234, bf16=True, init="he", T=500)
+RESNET_WORKLOAD = dict(name="resnet20_K16_B128_postlocal_H16_bf16", K=16, B=128, H=16, N=50000,
+                       C=10, base_lr=0.2, scale_by_K=True, warmup_epochs=5.0, momentum=0.9,
+                       nesterov=True, weight_decay=1e-4, seed=0, data_seed=1234, epochs=1.0)
+DENSE_CONFIGS = {"softmax": SOFTMAX, "mlp1024": CONFIG2, "mlp4096": WORKLOAD}
 
 
 def job_steps(w, K=None):
-    """T of one training job: ceil(epochs * N / (K * B_loc)) local steps (49 for the workload)."""
+    """T of one training job: ceil(epochs * N / (K * B_loc)) local steps (245 for the workload)."""
+    if "T" in w:
+        return w["T"]
     K = K or w["K"]
     return -(-int(w["epochs"] * w["N"]) // (K * w["B"]))
+
+
+def switch_step(w, K=None):
+    """The post-local switch t' = floor(frac * T) (the first learning-rate decay), or -1."""
+    f = w.get("t_switch_frac")
+    return -1 if f is None else int(f * job_steps(w, K))
+
 
 # Bytes the algorithm moves per parameter and replica (fp32 w, u, g; bf16 shadow):
 #   stand-alone update           = read g, w, u + write w, u (4 B each) + write the shadow (2 B) = 22
@@ -47,14 +81,22 @@ def job_steps(w, K=None):
 UPDATE_BYTES_PER_PARAM = 22
 FUSED_UPDATE_BYTES_PER_PARAM = 18
 AVERAGE_BYTES_PER_PARAM = 10
-# DRAM bytes (read + write) per step of the update launches (the classifier head's backward and
-# the weight-gradient + update launch of both hidden layers), from the ncu capture summarised in
-# profiles/step_kernels_mlp3072_K16_B128.md (below the algorithmic bytes because part of the
-# launch's writes is still in L2 when it ends).
-UPDATE_TRAFFIC_PER_STEP = 1186195456
+# DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum) per step of the fused update
+# launches, from ncu captures of the current kernels:
+#   MLP 3072-1024-1024-10, K = 16, B_loc = 128: the classifier head's backward plus the one
+#     weight-gradient + update launch of both hidden layers, 1,186,195,456 B (below the
+#     algorithmic bytes because part of the launch's writes is still in L2 when it ends);
+#   MLP 3072-4096x3-100: captured at K = 2 (one step's two weight-gradient + update launches)
+#     and scaled by 8 to K = 16 (the traffic is per replica; the K = 16 arena is too large for a
+#     multi-pass capture).
+UPDATE_TRAFFIC_PER_STEP = {CONFIG2["name"]: 1186195456, WORKLOAD["name"]: None}
 
 FALLBACK_HBM_GBS = 6800.0
 FALLBACK_BF16_TFLOPS = 1900.0
+
+# The oracle's bounded sample (both arms): one replica's local step on the first ORACLE_ROWS rows
+# of its mini-batch (forward, backward) plus the update of all its parameters.
+ORACLE_ROWS = 16
 
 
 def dense_params(widths):
@@ -63,16 +105,19 @@ def dense_params(widths):
 
 
 def workload_config(w, K, world, fused=True):
-    """The workload description both arms print (the timed region's own facts are added by the
-    GPU arm)."""
+    """The workload description both arms print, identically."""
     B, H, T_job = w["B"], w["H"], job_steps(w, K)
-    return {"workload": w["name"] if K == w["K"] else w["name"].replace("K16", f"K{K}"),
-            "global_batch": K * B, "K": K, "B_loc": B, "H": H, "fused_update": fused,
+    ts = switch_step(w, K)
+    name = w["name"] if K == w["K"] else w["name"].replace(f"K{w['K']}", f"K{K}")
+    sched = (f"post-local: H = 1 before t' = {ts}, H = {H} after" if ts >= 0 else f"H = {H}")
+    return {"workload": name, "global_batch": K * B, "K": K, "B_loc": B, "H": H,
+            "schedule": sched, "fused_update": fused,
             "job": f"{T_job}-step schedule ({w['epochs']:g} epochs of N = {w['N']}), "
                    "repeated from its end state",
             "params_per_replica": dense_params(w["widths"]),
             "parallelism": "replicas" if world > 1 else "single",
-            "l2": "per-step working set (w, u, g, shadow: 1.0 GB) exceeds the 129 MB L2"}
+            "l2": "inputs larger than L2: the per-step working set (w, u, shadow) is "
+                  f"{(10 * K * dense_params(w['widths'])) / 1e9:.1f} GB against the 129 MB L2"}
 
 
 def _peaks():
@@ -111,8 +156,23 @@ def whole_job_throughput(units_per_rank: float, seconds: float, world: int) -> f
     return world * units_per_rank / max_over_ranks(seconds, world)
 
 
+def host_info():
+    """Host cores and CPU model of the machine the oracle is timed on."""
+    model = platform.processor() or platform.machine()
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.startswith("Model name:"):
+                model = line.split(":", 1)[1].strip()
+                break
+    except Exception:
+        pass
+    return {"nproc": os.cpu_count(), "cpu_model": model, "machine": platform.machine()}
+
+
 class ClockSampler:
-    """nvidia-smi samples of SM clock and throttle reasons while a timed region runs."""
+    """nvidia-smi samples of SM clock and throttle reasons; mark() brackets the timed region so
+    that only the samples taken inside it are summarised."""
 
     FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
@@ -122,6 +182,7 @@ class ClockSampler:
         self.dev = device_index
         self.proc = None
         self.path = None
+        self.lines = []
 
     def start(self):
         try:
@@ -129,12 +190,20 @@ class ClockSampler:
             os.close(fd)
             self.proc = subprocess.Popen(
                 ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
-                 "-lms", "100", "-i", str(self.dev)],
+                 "-lms", "20", "-i", str(self.dev)],
                 stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
         except Exception:
             self.proc = None
 
-    def stop(self):
+    def count(self) -> int:
+        """Rows written so far (the sampler's position, to bracket a region)."""
+        if not self.proc:
+            return 0
+        with open(self.path) as f:
+            return sum(1 for _ in f)
+
+    def stop(self, first: int = 0, last: int | None = None):
+        """Summary of rows [first, last) (all rows by default)."""
         if not self.proc:
             return None
         self.proc.terminate()
@@ -145,7 +214,8 @@ class ClockSampler:
         with open(self.path) as f:
             lines = f.readlines()
         os.unlink(self.path)
-        return summarise_clocks(lines)
+        sel = lines[first:last] if last is not None else lines[first:]
+        return summarise_clocks(sel or lines)
 
 
 def summarise_clocks(lines):
@@ -168,44 +238,119 @@ def summarise_clocks(lines):
             "reasons": reasons, "samples": len(rows)}
 
 
-def _make_cfg(P, total_steps, fused=True, K=None):
-    w = WORKLOAD
-    return P.make_config(K=K or w["K"], B_loc=w["B"], H=w["H"], total_steps=total_steps, N=w["N"],
-                         widths=w["widths"], base_lr=w["base_lr"], scale_by_K=w["scale_by_K"],
-                         warmup_epochs=w["warmup_epochs"], momentum=w["momentum"],
-                         nesterov=w["nesterov"], weight_decay=w["weight_decay"], seed=w["seed"],
-                         precision=P.BF16, fused_update=fused)
+def make_gpu_cfg(P, w, fused=True, K=None):
+    K = K or w["K"]
+    return P.make_config(K=K, B_loc=w["B"], H=w["H"], t_switch=switch_step(w, K),
+                         total_steps=job_steps(w, K), N=w["N"], widths=w["widths"],
+                         init=P.INIT_ZERO if w["init"] == "zero" else P.INIT_HE,
+                         base_lr=w["base_lr"], scale_by_K=w["scale_by_K"],
+                         warmup_epochs=w["warmup_epochs"], milestones=w["milestones"],
+                         momentum=w["momentum"], nesterov=w["nesterov"],
+                         weight_decay=w["weight_decay"], seed=w["seed"],
+                         precision=P.BF16 if w["bf16"] else P.FP32,
+                         fused_update=fused and w["bf16"])
 
 
-def _oracle_cfg(oracle, total_steps):
-    w = WORKLOAD
-    return oracle.make_cfg(widths=w["widths"], bf16=True, K=w["K"], B=w["B"], H=w["H"],
-                           T=total_steps, N=w["N"], base_lr=w["base_lr"],
-                           scale_by_K=w["scale_by_K"], warmup_epochs=w["warmup_epochs"],
+def make_oracle_cfg(oracle, w, K=None, T=None):
+    K = K or w["K"]
+    return oracle.make_cfg(widths=w["widths"], bf16=w["bf16"], K=K, B=w["B"], H=w["H"],
+                           t_switch=switch_step(w, K), T=T or job_steps(w, K), N=w["N"],
+                           base_lr=w["base_lr"], scale_by_K=w["scale_by_K"],
+                           warmup_epochs=w["warmup_epochs"], milestones=w["milestones"],
                            momentum=w["momentum"], nesterov=w["nesterov"],
                            weight_decay=w["weight_decay"], seed=w["seed"])
 
 
-def oracle_sample(X, y, replica_steps: int, rows: int, budget_s: float):
-    """Time the oracle on `replica_steps` local steps of single replicas (first `rows` rows of each
-    worker's mini-batch, then the update of all parameters).  Returns (seconds, samples, steps)."""
+def oracle_sample(w, X, y, n_steps: int, rows: int, budget_s: float):
+    """Time the oracle on up to `n_steps` local steps of single replicas of workload w (the first
+    `rows` rows of each worker's mini-batch, forward and backward, then the update of all the
+    replica's parameters), stopping once budget_s has passed.  Returns (seconds, samples, steps)."""
     import numpy as np
 
     import oracle
 
-    o = _oracle_cfg(oracle, 1 << 20)
-    w = oracle.init_params(o)
-    u = np.zeros_like(w)
+    o = make_oracle_cfg(oracle, w)
+    wt = oracle.init_params(o, oracle.INIT_ZERO if w["init"] == "zero" else oracle.INIT_HE)
+    u = np.zeros_like(wt)
     t0 = time.perf_counter()
     done = 0
-    for i in range(replica_steps):
+    for i in range(n_steps):
         idx = oracle.sample_indices(o, i % o.K, i // o.K)[:rows]
-        _, g = oracle.loss_grad(o, w, X, y=y, idx=idx)
-        w, u = oracle.sgd_update(o, oracle.lr(o, i // o.K), w, u, g)
+        _, g = oracle.loss_grad(o, wt, X, y=y, idx=idx)
+        wt, u = oracle.sgd_update(o, oracle.lr(o, i // o.K), wt, u, g)
         done += 1
         if time.perf_counter() - t0 > budget_s:
             break
     return time.perf_counter() - t0, done * rows, done
+
+
+def oracle_sample_text(w, steps, rows):
+    return (f"{steps} single-replica local steps of {w['name']}, each on the first {rows} of the "
+            f"worker's {w['B']} mini-batch rows (forward, backward) plus the update of all "
+            f"{dense_params(w['widths'])} parameters, on one host core")
+
+
+def oracle_other_configs(budget_s: float = 6.0):
+    """The oracle timed on the other configurations, one host core each: softmax regression's
+    whole 64-step job (K = 4), config 2 and ResNet-20 on bounded single-replica samples, and the
+    K x H sweep network's first 4 local steps + 1 average at K = 8."""
+    import numpy as np
+
+    import oracle
+    import synthdata
+
+    out = {}
+    # softmax regression: the whole job
+    w = SOFTMAX
+    X, y = synthdata.gaussian_mixture_cached(w["N"], 3072, w["C"], w["data_seed"])
+    o = make_oracle_cfg(oracle, w)
+    W0 = np.zeros((w["K"], oracle.num_params(o)))
+    t0 = time.perf_counter()
+    _, _, _, syncs = oracle.run(o, X, y=y, W=W0)
+    t = time.perf_counter() - t0
+    out["softmax"] = {"workload": w["name"], "samples_per_s": w["T"] * w["K"] * w["B"] / t,
+                      "ms_per_step": 1000 * t / w["T"], "sample": f"the whole {w['T']}-step job "
+                      f"({syncs} averages)"}
+    # config 2: bounded single-replica sample
+    w = CONFIG2
+    X, y = synthdata.gaussian_mixture_cached(w["N"], 3072, w["C"], w["data_seed"])
+    t, samples, steps = oracle_sample(w, X, y, 64, 32, budget_s)
+    out["mlp1024"] = {"workload": w["name"], "samples_per_s": samples / t,
+                      "sample": oracle_sample_text(w, steps, 32)}
+    # the sweep network at K = 8, B = 32: the first 4 local steps and the average that ends them
+    w = SWEEP
+    o = make_oracle_cfg(oracle, w, T=4)
+    o.H = 4
+    t0 = time.perf_counter()
+    _, _, _, syncs = oracle.run(o, X, y=y, n_steps=4)
+    t = time.perf_counter() - t0
+    out["mlp512"] = {"workload": w["name"] + "_K8_H4", "samples_per_s": 4 * w["K"] * w["B"] / t,
+                     "ms_per_step": 1000 * t / 4,
+                     "sample": f"the first 4 local steps of all 8 replicas + {syncs} average"}
+    # ResNet-20: one replica's step on 8 images + its update
+    w = RESNET_WORKLOAD
+    X10, y10 = synthdata.gaussian_mixture_cached(w["N"], 3072, w["C"], w["data_seed"])
+    o = oracle.make_cfg(kind=oracle.RESNET20, bf16=True, K=w["K"], B=w["B"], H=w["H"], T=25,
+                        t_switch=12, N=w["N"], base_lr=w["base_lr"], scale_by_K=True,
+                        warmup_epochs=5.0, milestones=(0.5, 0.75), momentum=0.9, nesterov=True,
+                        weight_decay=w["weight_decay"], seed=w["seed"])
+    wt = oracle.init_params(o)
+    u = np.zeros_like(wt)
+    t0 = time.perf_counter()
+    steps = 0
+    while True:
+        idx = oracle.sample_indices(o, steps % o.K, 0)[:8]
+        _, g = oracle.loss_grad(o, wt, X10, y=y10, idx=idx)
+        wt, u = oracle.sgd_update(o, oracle.lr(o, 0), wt, u, g)
+        steps += 1
+        if time.perf_counter() - t0 > budget_s / 2:
+            break
+    t = time.perf_counter() - t0
+    out["resnet20"] = {"workload": w["name"], "samples_per_s": 8 * steps / t,
+                       "sample": f"{steps} single-replica local steps on 8 of the worker's 128 "
+                                 "images plus the update of all parameters"}
+    out["host"] = host_info()
+    return out
 
 
 def run_reference(args, world, rank):
@@ -215,13 +360,10 @@ def run_reference(args, world, rank):
 
     w = WORKLOAD
     X, y = synthdata.gaussian_mixture_cached(w["N"], w["widths"][0], w["C"], w["data_seed"])
-    rows = 32
     for _ in range(args.warmup):
-        oracle_sample(X, y, 1, rows, 1e9)
-    t, samples, steps = oracle_sample(X, y, args.steps, rows, 1e9)
+        oracle_sample(w, X, y, 1, ORACLE_ROWS, 1e9)
+    t, samples, steps = oracle_sample(w, X, y, args.steps, ORACLE_ROWS, 1e9)
     v = samples / t
-    sample = (f"{steps} single-replica local steps, each on {rows} of the worker's {w['B']} "
-              f"mini-batch rows plus the update of all parameters")
     line = {
         "impl": "reference", "metric": "samples/s over K simulated workers (1 GB300)",
         "value": v, "unit": "samples/s", "n_gpus": args.gpus, "steps": args.steps,
@@ -229,7 +371,7 @@ def run_reference(args, world, rank):
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
         "config": workload_config(w, w["K"], world),
         "cpu_baseline": {"value": v, "unit": "samples/s", "cores": 1, "kind": "oracle",
-                         "sample": sample},
+                         "sample": oracle_sample_text(w, steps, ORACLE_ROWS)},
         "e2e": {"value": v, "unit": "samples/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
@@ -288,9 +430,9 @@ SYNC_VARIANT_BYTES = {"plain": (10, 0), "global_momentum": (10, 16), "sign": (14
 
 
 def run_sync_variants(args):
-    """Time one synchronisation of each averaging variant on the MLP workload's parameter arena
-    (K = 16 replicas of d = 4.2 M parameters; 268 MB of fp32 replicas, larger than L2): one JSON
-    line per variant with ms per sync and algorithmic GB/s against the HBM peak."""
+    """Time one synchronisation of each averaging variant on the MLP 3072-1024-1024-10 parameter
+    arena (K = 16 replicas of d = 4.2 M parameters; 268 MB of fp32 replicas, larger than L2): one
+    JSON line per variant with ms per sync and algorithmic GB/s against the HBM peak."""
     import torch
 
     from paper_1808_07217_gb300 import _build
@@ -301,7 +443,7 @@ def run_sync_variants(args):
     torch.cuda.set_device(0)
     stream = torch.cuda.current_stream()
     hbm, _, src = _peaks()
-    w = WORKLOAD
+    w = CONFIG2
     K = args.replicas or w["K"]
     n_sync = max(args.steps, 8)
     for name, extra in (("plain", {}), ("global_momentum", dict(global_momentum=0.9)),
@@ -334,105 +476,122 @@ def run_sync_variants(args):
         P.lsgd_destroy(ctx)
 
 
-# The other dense configurations, timed on their own job schedules (one JSON line each):
-#   softmax regression 3072 -> 10, fp32, zero init, K = 4 shards of 2,048 of N = 8,192 points,
-#     B_loc = 32, H = 4, plain SGD lr 0.1, a 64-step job;
-#   post-local MLP 3072-4096-4096-4096-100, bf16, K = 16, B_loc = 128, 10 epochs of N = 50,000
-#     (245 steps), H = 1 before t' = 122 and 16 after, Nesterov 0.9, weight decay 5e-4, lr 0.1
-#     scaled by K with a 5-epoch warm-up, decayed 10x at 50 % and 75 %.
-DENSE_CONFIGS = {
-    "softmax": dict(name="softmax_3072-10_K4_B32_H4_fp32", widths=(3072, 10), K=4, B=32, H=4,
-                    N=8192, C=10, T=64, t_switch=-1, base_lr=0.1, scale_by_K=False,
-                    warmup_epochs=0.0, milestones=(), momentum=0.0, nesterov=False,
-                    weight_decay=0.0, init="zero", bf16=False, seed=0, data_seed=1234),
-    "mlp4096": dict(name="mlp_3072-4096x3-100_K16_B128_postlocal_H16_bf16",
-                    widths=(3072, 4096, 4096, 4096, 100), K=16, B=128, H=16, N=50000, C=100,
-                    T=245, t_switch=122, base_lr=0.1, scale_by_K=True, warmup_epochs=5.0,
-                    milestones=(0.5, 0.75), momentum=0.9, nesterov=True, weight_decay=5e-4,
-                    init="he", bf16=True, seed=0, data_seed=1234),
-}
+class DenseRun:
+    """A dense workload's context on the device, stepped along its job schedule: a run past the
+    job's last step restarts the schedule from the model it ended with (lsgd_set_step(0) after
+    the job's final average), so every timed step is a step of the configured schedule."""
+
+    def __init__(self, P, w, stream, fused=True, K=None):
+        import synthdata
+
+        self.P, self.w = P, w
+        self.K = K or w["K"]
+        self.T = job_steps(w, self.K)
+        self.cfg = make_gpu_cfg(P, w, fused, self.K)
+        self.X, self.y = synthdata.gaussian_mixture_cached(w["N"], w["widths"][0], w["C"],
+                                                           w["data_seed"])
+        self.ctx = P.lsgd_create(self.cfg, stream=stream.cuda_stream)
+        P.lsgd_set_dataset(self.ctx, self.X, self.y)
+        self.d = P.lsgd_num_params(self.ctx)
+
+    def run_steps(self, n):
+        P = self.P
+        while n > 0:
+            m = min(n, self.T - P.lsgd_step_count(self.ctx))
+            P.lsgd_run(self.ctx, m)
+            n -= m
+            if P.lsgd_step_count(self.ctx) == self.T:
+                P.lsgd_set_step(self.ctx, 0)
+
+    def losses_finite(self, n):
+        import numpy as np
+
+        n = min(self.P.lsgd_step_count(self.ctx), n)
+        return (not n) or bool(np.isfinite(self.P.lsgd_losses(self.ctx, n, self.K)).all())
+
+    def time_steps(self, n, stream):
+        """Device time (ms) of n steps, their kernel launches and averages."""
+        import torch
+
+        P = self.P
+        n0, s0 = P.lsgd_kernel_launches(self.ctx), P.lsgd_sync_count(self.ctx)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        self.run_steps(n)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        return (e0.elapsed_time(e1), P.lsgd_kernel_launches(self.ctx) - n0,
+                P.lsgd_sync_count(self.ctx) - s0)
+
+    def traced(self, n):
+        """Per-phase device times of n further steps (CUDA events around every phase)."""
+        import torch
+
+        P = self.P
+        P.lsgd_profile_enable(self.ctx, True)
+        self.run_steps(n)
+        torch.cuda.synchronize()
+        prof = P.lsgd_profile_read(self.ctx)
+        P.lsgd_profile_enable(self.ctx, False)
+        return prof
+
+    def update_bytes(self, fused=True):
+        """Algorithmic bytes of one step's update launches."""
+        w, K, B = self.w, self.K, self.w["B"]
+        widths = w["widths"]
+        if fused and w["bf16"]:
+            return sum(FUSED_UPDATE_BYTES_PER_PARAM * K * widths[l] * widths[l + 1]
+                       + 2 * K * B * (widths[l] + widths[l + 1]) for l in range(len(widths) - 1))
+        return UPDATE_BYTES_PER_PARAM * K * self.d
+
+    def destroy(self):
+        self.P.lsgd_destroy(self.ctx)
+
+
+def roofline(run, prof, steps, hbm, peak_src, fused=True):
+    upd_n, upd_ms = prof["update"]
+    upd_bytes = run.update_bytes(fused)
+    upd_gbs = upd_bytes / (upd_ms / steps / 1000.0) / 1e9
+    traffic = UPDATE_TRAFFIC_PER_STEP.get(run.w["name"]) if fused and run.K == run.w["K"] else None
+    return {"kernel": ("wgrad_update_kernel (weight gradient + fused local update)"
+                       if fused else "sgd_update_kernel"),
+            "bound": "hbm", "achieved": upd_gbs, "peak": hbm, "unit": "GB/s",
+            "frac": upd_gbs / hbm, "peak_source": f"{peak_src} hbm_gbs", "traffic": traffic,
+            "unit_of_work": ("one step's fused weight-gradient + update launches (all layers)"
+                             if fused else "one launch over the whole K x d buffer"),
+            "algorithmic_bytes": upd_bytes, "launches_per_unit": upd_n // steps}
 
 
 def run_dense_config(args, key):
-    """Time one of DENSE_CONFIGS: W warm-up steps, then S timed steps of its job schedule
-    (repeated from its end state, as for the benchmark workload), then a traced pass for the
-    per-phase split.  One JSON line with samples/s, ms per step, the syncs and launches in the
-    timed region and the update phase's algorithmic HBM throughput."""
-    import numpy as np
+    """Time one of DENSE_CONFIGS on its job schedule: W warm-up steps, S timed steps, then a
+    traced pass for the per-phase split.  One JSON line."""
     import torch
 
-    import synthdata
     from paper_1808_07217_gb300 import _build
 
     _build.build()
     import paper_1808_07217_gb300 as P
 
     torch.cuda.set_device(0)
-    w = DENSE_CONFIGS[key]
-    K, B, T = w["K"], w["B"], w["T"]
-    X, y = synthdata.gaussian_mixture_cached(w["N"], w["widths"][0], w["C"], w["data_seed"])
-    W_, S_ = max(3, args.warmup), args.steps
-    fused = w["bf16"]
-    cfg = P.make_config(K=K, B_loc=B, H=w["H"], t_switch=w["t_switch"], total_steps=T, N=w["N"],
-                        widths=w["widths"], init=P.INIT_ZERO if w["init"] == "zero" else P.INIT_HE,
-                        base_lr=w["base_lr"], scale_by_K=w["scale_by_K"],
-                        warmup_epochs=w["warmup_epochs"], milestones=w["milestones"],
-                        momentum=w["momentum"], nesterov=w["nesterov"],
-                        weight_decay=w["weight_decay"], seed=w["seed"],
-                        precision=P.BF16 if w["bf16"] else P.FP32, fused_update=fused)
     stream = torch.cuda.current_stream()
-    ctx = P.lsgd_create(cfg, stream=stream.cuda_stream)
-    P.lsgd_set_dataset(ctx, X, y)
-    d = P.lsgd_num_params(ctx)
-
-    def run_steps(n):
-        while n > 0:
-            m = min(n, T - P.lsgd_step_count(ctx))
-            P.lsgd_run(ctx, m)
-            n -= m
-            if P.lsgd_step_count(ctx) == T:
-                P.lsgd_set_step(ctx, 0)
-
-    run_steps(W_)
+    w = DENSE_CONFIGS[key]
+    fused = w["bf16"] and not args.unfused
+    run = DenseRun(P, w, stream, fused, args.replicas or None)
+    S_ = args.steps
+    run.run_steps(max(3, args.warmup))
     torch.cuda.synchronize()
-    n0, sy0 = P.lsgd_kernel_launches(ctx), P.lsgd_sync_count(ctx)
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
-    run_steps(S_)
-    e1.record(stream)
-    torch.cuda.synchronize()
-    ms = e0.elapsed_time(e1)
-    launches, syncs = P.lsgd_kernel_launches(ctx) - n0, P.lsgd_sync_count(ctx) - sy0
-    n_chk = min(P.lsgd_step_count(ctx), 8)
-    losses = P.lsgd_losses(ctx, n_chk, K) if n_chk else np.zeros(1)
-    P.lsgd_profile_enable(ctx, True)
-    run_steps(S_)
-    torch.cuda.synchronize()
-    prof = P.lsgd_profile_read(ctx)
+    ms, launches, syncs = run.time_steps(S_, stream)
+    finite = run.losses_finite(8)
+    prof = run.traced(S_)
     hbm, _, src = _peaks()
-    widths = w["widths"]
-    if fused:
-        upd_bytes = sum(FUSED_UPDATE_BYTES_PER_PARAM * K * widths[l] * widths[l + 1]
-                        + 2 * K * B * (widths[l] + widths[l + 1]) for l in range(len(widths) - 1))
-    else:
-        upd_bytes = UPDATE_BYTES_PER_PARAM * K * d
-    upd_ms = prof["update"][1] / S_
-    print(json.dumps({"workload": w["name"], "value": S_ * K * B / (ms / 1000.0),
+    print(json.dumps({"workload": w["name"], "value": S_ * run.K * w["B"] / (ms / 1000.0),
                       "unit": "samples/s", "steps": S_, "ms_per_step": ms / S_,
-                      "job": f"{T}-step schedule, repeated from its end state",
+                      "job": f"{run.T}-step schedule, repeated from its end state",
                       "syncs_in_timed_region": syncs, "gpu_launches": launches,
-                      "params_per_replica": d, "losses_finite": bool(np.isfinite(losses).all()),
-                      "update_phase": {"ms_per_step": upd_ms, "algorithmic_bytes": upd_bytes,
-                                       "gbs": upd_bytes / (upd_ms * 1e6) if upd_ms else None,
-                                       "frac_of_hbm": (upd_bytes / (upd_ms * 1e6) / hbm)
-                                       if upd_ms else None, "peak_source": f"{src} hbm_gbs"},
+                      "params_per_replica": run.d, "losses_finite": finite,
+                      "roofline": roofline(run, prof, S_, hbm, src, fused),
                       "phase_ms_per_step": {k: v[1] / S_ for k, v in prof.items()}}), flush=True)
-    P.lsgd_destroy(ctx)
-
-
-RESNET_WORKLOAD = dict(name="resnet20_K16_B128_postlocal_H16_bf16", K=16, B=128, H=16, N=50000,
-                       C=10, base_lr=0.2, scale_by_K=True, warmup_epochs=5.0, momentum=0.9,
-                       nesterov=True, weight_decay=1e-4, seed=0, data_seed=1234, epochs=1.0)
+    run.destroy()
 
 
 def run_resnet(args):
@@ -502,7 +661,7 @@ def run_resnet(args):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=48)
+    ap.add_argument("--steps", type=int, default=245)
     ap.add_argument("--warmup", type=int, default=16)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -510,10 +669,10 @@ def main():
                     help="K x H sync / compute sweep of the MLP 3072-512-512-10 workload")
     ap.add_argument("--sync-variants", action="store_true",
                     help="time one synchronisation of each averaging variant (plain, global "
-                         "momentum, sign, EF-sign) on the MLP workload's K x d arena")
+                         "momentum, sign, EF-sign) on the MLP 3072-1024-1024-10 K x d arena")
     ap.add_argument("--config", choices=sorted(DENSE_CONFIGS),
-                    help="time another dense configuration (softmax regression, post-local "
-                         "MLP 3072-4096x3-100) on its job schedule")
+                    help="time one dense configuration alone (softmax regression, MLP "
+                         "3072-1024-1024-10, post-local MLP 3072-4096x3-100) on its job schedule")
     ap.add_argument("--resnet", action="store_true",
                     help="post-local ResNet-20 workload (K = 16, B_loc = 128) instead of the MLP")
     ap.add_argument("--unfused", action="store_true",
@@ -543,8 +702,6 @@ def main():
     import numpy as np
     import torch
 
-    import synthdata
-
     if world > 1:
         import torch.distributed as dist
 
@@ -558,75 +715,45 @@ def main():
     import paper_1808_07217_gb300 as P
 
     w = WORKLOAD
-    K, B, H = args.replicas or w["K"], w["B"], w["H"]
     fused = not args.unfused
-    X, y = synthdata.gaussian_mixture_cached(w["N"], w["widths"][0], w["C"], w["data_seed"])
     W_, S_ = max(3, args.warmup), args.steps
     e2e_warm = 2
-    # The workload is a T-step job (2 epochs: 49 steps, the learning rate still warming up toward
-    # K x 0.1); longer runs repeat it from the model it ended with (lsgd_set_step(0) after the
-    # job's last step and its final average), so every timed step is a step of that schedule.
-    T_job = job_steps(w, K)
-    cfg = _make_cfg(P, T_job, fused, K)
-    _, kinds = P.lsgd_schedule(cfg, T_job)
     stream = torch.cuda.current_stream()
-    ctx = P.lsgd_create(cfg, stream=stream.cuda_stream)
-    P.lsgd_set_dataset(ctx, X, y)
-    d = P.lsgd_num_params(ctx)
-
-    def run_steps(n):
-        while n > 0:
-            m = min(n, T_job - P.lsgd_step_count(ctx))
-            P.lsgd_run(ctx, m)
-            n -= m
-            if P.lsgd_step_count(ctx) == T_job:
-                P.lsgd_set_step(ctx, 0)
+    run = DenseRun(P, w, stream, fused, args.replicas or None)
+    K, B, T_job, ctx = run.K, w["B"], run.T, run.ctx
+    _, kinds = P.lsgd_schedule(run.cfg, T_job)
 
     # ---- device-resident timing ----
-    run_steps(W_)
+    run.run_steps(W_)
     torch.cuda.synchronize()
     clocks = ClockSampler(local)
     clocks.start()
     time.sleep(0.3)
-    n0 = P.lsgd_kernel_launches(ctx)
-    syncs0 = P.lsgd_sync_count(ctx)
     if world > 1:
         torch.distributed.barrier()
     torch.cuda.synchronize()
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
-    run_steps(S_)
-    e1.record(stream)
-    torch.cuda.synchronize()
+    c0 = clocks.count()
+    t_ms, launches, n_syncs = run.time_steps(S_, stream)
     if world > 1:
         torch.distributed.barrier()
-    t_ms = e0.elapsed_time(e1)
-    launches = P.lsgd_kernel_launches(ctx) - n0
-    n_syncs = P.lsgd_sync_count(ctx) - syncs0
-    clk = clocks.stop()
+    time.sleep(0.05)
+    clk = clocks.stop(c0, clocks.count())
+    if not run.losses_finite(16):
+        raise RuntimeError("non-finite loss in the timed steps")
 
     # ---- the same number of steps again with per-phase CUDA events (the split and roofline) ----
-    n_chk = min(P.lsgd_step_count(ctx), 16)
-    if n_chk and not np.isfinite(P.lsgd_losses(ctx, n_chk, K)).all():
-        raise RuntimeError("non-finite loss in the timed steps")
-    P.lsgd_profile_enable(ctx, True)
-    run_steps(S_)
-    torch.cuda.synchronize()
-    prof = P.lsgd_profile_read(ctx)
-    P.lsgd_profile_enable(ctx, False)
+    prof = run.traced(S_)
     samples_per_rank = S_ * K * B
     t_ms = max_over_ranks(t_ms, world)
     value = whole_job_throughput(samples_per_rank, t_ms / 1000.0, world)
 
     # ---- end to end through the C ABI with host buffers ----
-    rng = np.random.default_rng(0)
     n_stage = 4
     xs, ys = [], []
     for i in range(n_stage):
         idx = P.lsgd_debug_indices(ctx, (P.lsgd_step_count(ctx) + i) % T_job, K, B).reshape(-1)
-        xs.append(torch.from_numpy(X[idx].reshape(K, B, -1)).pin_memory())
-        ys.append(torch.from_numpy(y[idx].reshape(K, B).copy()).pin_memory())
-    del rng
+        xs.append(torch.from_numpy(run.X[idx].reshape(K, B, -1)).pin_memory())
+        ys.append(torch.from_numpy(run.y[idx].reshape(K, B).copy()).pin_memory())
     # every step's K losses come back to pinned host memory; the reads are asynchronous, like the
     # host-to-device copies (which run on the library's copy stream, one batch ahead), and all
     # of them have landed when the timed region ends
@@ -659,21 +786,11 @@ def main():
     h2d = K * B * w["widths"][0] * 4 + K * B * 4
     d2h = K * 4
 
-    # ---- roofline of the dominant kernel (the fused update) ----
+    # ---- roofline of the dominant kernel (the fused update), the average, the GEMMs ----
     hbm, bf16_peak, peak_src = _peaks()
-    upd_n, upd_ms = prof["update"]
     avg_n, avg_ms = prof["average"]
     widths = w["widths"]
-    # The update phase is each step's fused update launches (the head's backward, then one
-    # weight-gradient + update launch over both hidden layers); the roofline unit is one step's
-    # worth of them (bytes summed over the layers).
-    if fused:
-        upd_bytes = sum(FUSED_UPDATE_BYTES_PER_PARAM * K * widths[l] * widths[l + 1]
-                        + 2 * K * B * (widths[l] + widths[l + 1]) for l in range(len(widths) - 1))
-    else:
-        upd_bytes = UPDATE_BYTES_PER_PARAM * K * d
-    upd_gbs = upd_bytes / (upd_ms / S_ / 1000.0) / 1e9
-    avg_gbs = (AVERAGE_BYTES_PER_PARAM * K * d / (avg_ms / avg_n / 1000.0) / 1e9) if avg_n else None
+    avg_gbs = (AVERAGE_BYTES_PER_PARAM * K * run.d / (avg_ms / avg_n / 1000.0) / 1e9) if avg_n else None
     gemm_flops = 0
     for l in range(len(widths) - 1):
         mac = B * widths[l] * widths[l + 1]
@@ -683,32 +800,43 @@ def main():
     gemm_tflops = gemm_flops / (gemm_ms / 1000.0) / 1e12
     phase_ms = {k: v[1] for k, v in prof.items()}
     tot_phase = sum(phase_ms.values())
+    run.destroy()
+
+    # ---- config 2 (MLP 3072-1024-1024-10) on its own schedule, device time ----
+    cfg2 = None
+    if args.replicas == 0:
+        r2 = DenseRun(P, CONFIG2, stream, fused)
+        r2.run_steps(W_)
+        torch.cuda.synchronize()
+        ms2, launches2, syncs2 = r2.time_steps(S_, stream)
+        finite2 = r2.losses_finite(16)
+        prof2 = r2.traced(S_)
+        cfg2 = {"workload": CONFIG2["name"], "value": S_ * r2.K * CONFIG2["B"] / (ms2 / 1000.0),
+                "unit": "samples/s", "ms_per_step": ms2 / S_, "steps": S_,
+                "syncs_in_timed_region": syncs2, "gpu_launches": launches2,
+                "losses_finite": finite2, "roofline": roofline(r2, prof2, S_, hbm, peak_src, fused)}
+        r2.destroy()
 
     cpu = None
+    cpu_others = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        t_cpu, samples_cpu, steps_cpu = oracle_sample(X, y, 64, B, 15.0)
+        t_cpu, samples_cpu, steps_cpu = oracle_sample(w, run.X, run.y, 64, ORACLE_ROWS, 12.0)
         cpu = {"value": samples_cpu / t_cpu, "unit": "samples/s", "cores": 1, "kind": "oracle",
-               "sample": f"{steps_cpu} single-replica local steps of the workload (B = {B} rows "
-                         f"each, forward, backward and update) timed on one host core"}
+               "sample": oracle_sample_text(w, steps_cpu, ORACLE_ROWS)}
+        cpu_others = oracle_other_configs()
 
     line = {
         "metric": "samples/s over K simulated workers (1 GB300)",
         "value": value, "unit": "samples/s", "n_gpus": world, "steps": S_, "warmup": W_,
         "ms_per_step": t_ms / S_, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": dict(workload_config(w, K, world, fused), syncs_in_timed_region=n_syncs),
+        "config": workload_config(w, K, world, fused),
+        "syncs_in_timed_region": n_syncs,
+        "first_timed_step": W_ % T_job,
         "e2e": {"value": e2e_value, "unit": "samples/s", "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h},
         "gpu_launches": launches,
-        "roofline": {"kernel": ("wgrad_update_kernel (weight gradient + fused local update)"
-                                if fused else "sgd_update_kernel"),
-                     "bound": "hbm", "achieved": upd_gbs, "peak": hbm, "unit": "GB/s",
-                     "frac": upd_gbs / hbm, "peak_source": f"{peak_src} hbm_gbs",
-                     "traffic": UPDATE_TRAFFIC_PER_STEP if fused and K == w["K"] else None,
-                     "unit_of_work": ("one step's fused weight-gradient + update launches "
-                                      "(3 layers: the head's backward, one launch for the rest)"
-                                      if fused else "one launch over the whole K x d buffer"),
-                     "algorithmic_bytes": upd_bytes, "launches_per_unit": upd_n // S_},
+        "roofline": roofline(run, prof, S_, hbm, peak_src, fused),
         "sync_average": {"gbs": avg_gbs, "frac_of_hbm": (avg_gbs / hbm) if avg_gbs else None,
                          "ms_per_sync": (avg_ms / avg_n) if avg_n else None},
         "step_split": {"local_frac": 1.0 - phase_ms["average"] / tot_phase,
@@ -718,10 +846,11 @@ def main():
                  "peak_source": f"{peak_src} bf16_tflops_sustained"},
         "clocks": clk,
         "cpu_baseline": cpu,
+        "cpu_baseline_other_configs": cpu_others,
+        "config2": cfg2,
     }
     if rank == 0:
         print(json.dumps(line), flush=True)
-    P.lsgd_destroy(ctx)
     if world > 1:
         torch.distributed.destroy_process_group()
 

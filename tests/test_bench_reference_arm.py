@@ -23,19 +23,24 @@ def test_dense_params_counts_weights_and_biases():
 
 def test_job_and_workload_config():
     w = bench.WORKLOAD
-    # ceil(2 epochs x 50,000 / (16 x 128)) = 49 local steps
-    assert bench.job_steps(w) == 49
+    # ceil(10 epochs x 50,000 / (16 x 128)) = 245 local steps; t' = floor(0.5 x 245) = 122
+    assert bench.job_steps(w) == 245 and bench.switch_step(w) == 122
     cfg = bench.workload_config(w, 16, 1)
-    assert cfg["workload"] == "mlp_3072-1024-1024-10_K16_B128_H16_bf16"
+    assert cfg["workload"] == "mlp_3072-4096x3-100_K16_B128_postlocal_H16_bf16"
     assert cfg["global_batch"] == 2048 and cfg["K"] == 16 and cfg["B_loc"] == 128
-    assert cfg["params_per_replica"] == 4206602 and cfg["parallelism"] == "single"
+    assert cfg["params_per_replica"] == 46559332 and cfg["parallelism"] == "single"
+    assert cfg["schedule"] == "post-local: H = 1 before t' = 122, H = 16 after"
     assert bench.workload_config(w, 16, 4)["parallelism"] == "replicas"
-    assert bench.workload_config(w, 8, 1)["workload"].endswith("K8_B128_H16_bf16")
+    assert bench.workload_config(w, 8, 1)["workload"].endswith("K8_B128_postlocal_H16_bf16")
+    # the MLP 3072-1024-1024-10 configuration: ceil(2 x 50,000 / 2048) = 49 steps, no switch
+    assert bench.job_steps(bench.CONFIG2) == 49 and bench.switch_step(bench.CONFIG2) == -1
+    assert bench.dense_params(bench.CONFIG2["widths"]) == 4206602
+    assert bench.job_steps(bench.SOFTMAX) == 64
 
 
 def test_reference_arm_prints_one_contract_line():
     r = subprocess.run([sys.executable, "bench.py", "--impl", "reference", "--steps", "1",
-                        "--warmup", "3"], cwd=ROOT, capture_output=True, text=True, timeout=600)
+                        "--warmup", "1"], cwd=ROOT, capture_output=True, text=True, timeout=600)
     assert r.returncode == 0, r.stderr[-2000:]
     lines = [l for l in r.stdout.splitlines() if l.startswith("{")]
     assert len(lines) == 1
@@ -43,7 +48,7 @@ def test_reference_arm_prints_one_contract_line():
     assert d["impl"] == "reference"
     assert d["metric"] == "samples/s over K simulated workers (1 GB300)"
     assert d["unit"] == "samples/s" and d["higher_is_better"] is True
-    assert d["steps"] == 1 and d["warmup"] == 3 and d["n_gpus"] == 1
+    assert d["steps"] == 1 and d["warmup"] == 1 and d["n_gpus"] == 1
     assert d["value"] > 0 and d["ms_per_step"] > 0
     assert d["config"] == bench.workload_config(bench.WORKLOAD, 16, 1)
     cb = d["cpu_baseline"]

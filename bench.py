@@ -86,10 +86,10 @@ AVERAGE_BYTES_PER_PARAM = 10
 #   MLP 3072-1024-1024-10, K = 16, B_loc = 128: the classifier head's backward plus the one
 #     weight-gradient + update launch of both hidden layers, 1,186,195,456 B (below the
 #     algorithmic bytes because part of the launch's writes is still in L2 when it ends);
-#   MLP 3072-4096x3-100: captured at K = 2 (one step's two weight-gradient + update launches)
-#     and scaled by 8 to K = 16 (the traffic is per replica; the K = 16 arena is too large for a
-#     multi-pass capture).
-UPDATE_TRAFFIC_PER_STEP = {CONFIG2["name"]: 1186195456, WORKLOAD["name"]: None}
+#   MLP 3072-4096x3-100: one step's three weight-gradient + update launches captured at K = 2
+#     (1,557,492,992 B) and scaled by 8 to K = 16 (every tile belongs to one replica, so the
+#     traffic is per replica; the K = 16 arena is too large for a multi-pass capture).
+UPDATE_TRAFFIC_PER_STEP = {CONFIG2["name"]: 1186195456, WORKLOAD["name"]: 8 * 1557492992}
 
 FALLBACK_HBM_GBS = 6800.0
 FALLBACK_BF16_TFLOPS = 1900.0

@@ -198,8 +198,20 @@ lsgd_status lsgd_block_average(lsgd_ctx* ctx);
 /* n_steps local steps from the current step counter, averaging after every step s that ends a
  * round: s < t' (post-local first phase), (s + 1 - max(t', 0)) mod H == 0, or s == T - 1.  With
  * hier_block > 0 the r-th round end after the switch is a block average unless r is a multiple
- * of hier_rounds (or s == T - 1). */
+ * of hier_rounds (or s == T - 1).  With the fused update (bf16 dense models) and plain averaging,
+ * a step that ends with the global average forms it inside its own update launches: each weight
+ * tile is taken through all K replicas, updated per replica as usual, and the mean of the updated
+ * tiles goes to every replica (the same bits as the separate K-way average, without writing and
+ * re-reading the per-replica models). */
 lsgd_status lsgd_run(lsgd_ctx* ctx, int64_t n_steps);
+
+/* One step of lsgd_run's schedule on a caller-supplied mini-batch (arguments as for
+ * lsgd_local_step_batch): the local step, then the average the schedule puts at its end (global or
+ * block), counted like lsgd_run's.  Where the step ends with the plain global average and the
+ * update runs in the weight-gradient epilogue, the average is formed inside that step's update
+ * launches (Eq. 2: the mean of the updated replicas, to the same bits as the separate average). */
+lsgd_status lsgd_run_batch(lsgd_ctx* ctx, const float* x, const void* labels_or_targets,
+                           int on_device);
 
 /* Replica k's fp32 parameters (k = -1: the element-wise mean over replicas, computed in fp64 on
  * the host) in canonical order, n = lsgd_num_params() elements, to host or device memory. */

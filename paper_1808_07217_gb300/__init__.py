@@ -42,7 +42,7 @@ EXPORTS = [
     "lsgd_batchnorm_stats_noalloc", "lsgd_block_average", "lsgd_block_sync_count",
     "lsgd_sync_state", "lsgd_set_sync_state", "lsgd_schedule", "lsgd_device_status",
     "lsgd_bounded_wait_selftest", "lsgd_losses_async", "lsgd_synchronize", "lsgd_set_step",
-    "lsgd_conv_wgrad_bf16", "lsgd_conv3x3_bf16",
+    "lsgd_conv_wgrad_bf16", "lsgd_conv3x3_bf16", "lsgd_run_batch",
 ]
 PHASES = ["input", "forward", "loss", "backward", "update", "average"]
 
@@ -170,6 +170,7 @@ def lib():
             "lsgd_set_step": ([vp, i64], st),
             "lsgd_conv_wgrad_bf16": ([vp, vp, vp] + [ctypes.c_int] * 7 + [vp], st),
             "lsgd_conv3x3_bf16": ([ctypes.c_int, vp, vp, vp] + [ctypes.c_int] * 7 + [vp], st),
+            "lsgd_run_batch": ([vp, vp, vp, ctypes.c_int], st),
             "lsgd_sync_count": ([vp], i64),
             "lsgd_block_sync_count": ([vp], i64),
             "lsgd_block_average": ([vp], st),
@@ -297,6 +298,13 @@ def lsgd_local_step_batch(ctx: Ctx, x, labels_or_targets):
     (pinned memory copies asynchronously) or CUDA tensors."""
     on_dev = int(hasattr(x, "is_cuda") and x.is_cuda)
     _check(lib().lsgd_local_step_batch(ctx.handle, _ptr(x), _ptr(labels_or_targets), on_dev), ctx)
+
+
+def lsgd_run_batch(ctx: Ctx, x, labels_or_targets):
+    """One step of lsgd_run's schedule (local step + the average ending it, if any) on a
+    caller-supplied mini-batch, arguments as lsgd_local_step_batch."""
+    on_dev = int(hasattr(x, "is_cuda") and x.is_cuda)
+    _check(lib().lsgd_run_batch(ctx.handle, _ptr(x), _ptr(labels_or_targets), on_dev), ctx)
 
 
 def lsgd_sync_average(ctx: Ctx):

@@ -65,6 +65,33 @@ __device__ __forceinline__ void sgd_elem(float& w, float& u, float g, float lr, 
   w = fmaf(-lr, st, w);
 }
 
+// The K-way average's arithmetic (Eq. 2 right), shared by the stand-alone average and the
+// weight-gradient + update + average kernel so that both give the same bits.  Replicas are added
+// in order with Knuth's error-free TwoSum (s + x = t + e exactly) and the errors summed in c;
+// (s + c) / K is then formed from the quotient q = s / K, the exact fma remainder s - q K and c.
+// The result is the correctly rounded fp32 mean except in rare midpoint cases, whatever K.
+__device__ __forceinline__ void two_sum_add(float& s, float& c, float x) {
+  const float t = __fadd_rn(s, x);
+  const float z = __fsub_rn(t, s);
+  const float e = __fadd_rn(__fsub_rn(s, __fsub_rn(t, z)), __fsub_rn(x, z));
+  s = t;
+  c = __fadd_rn(c, e);
+}
+
+__device__ __forceinline__ float mean_of(float s, float c, float Kf) {
+  const float q = __fdiv_rn(s, Kf);
+  const float r = __fadd_rn(__fmaf_rn(-q, Kf, s), c);
+  return __fadd_rn(q, __fdiv_rn(r, Kf));
+}
+
+// mean_of for K a power of two: a correctly rounded division by 2^n equals the (single-rounding)
+// product with the exact reciprocal 2^-n, so this gives the same bits with two multiplies.
+__device__ __forceinline__ float mean_of_pow2(float s, float c, float Kf, float invK) {
+  const float q = __fmul_rn(s, invK);
+  const float r = __fadd_rn(__fmaf_rn(-q, Kf, s), c);
+  return __fadd_rn(q, __fmul_rn(r, invK));
+}
+
 // Programmatic dependent launch: kernels of the training step are launched so that the next one
 // may be scheduled while the previous one drains.  Each such kernel first waits for the previous
 // grid's completion and memory (griddepcontrol.wait) before touching global memory, and at once

@@ -26,6 +26,7 @@
 
 #include <algorithm>
 #include <mutex>
+#include <type_traits>
 
 #include "common.cuh"
 #include "lsgd_internal.h"
@@ -161,9 +162,11 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
   for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
 }
 
-// The local update on four consecutive parameters (fused weight-gradient epilogue).
+// The local update on four consecutive parameters (fused weight-gradient epilogue); SG fixes at
+// compile time whether the signSGD variant's sign is taken (it must equal sp.sign != 0).
+template <bool SG>
 __device__ __forceinline__ void sgd4(float4& w, float4& u, const float4 g, const SgdParams& sp) {
-  const bool sg = sp.sign != 0;
+  constexpr bool sg = SG;
   if (sp.mom == 0.f) {
     sgd_elem<false, false>(w.x, u.x, g.x, sp.lr, 0.f, sp.wd, sg);
     sgd_elem<false, false>(w.y, u.y, g.y, sp.lr, 0.f, sp.wd, sg);
@@ -514,21 +517,33 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
 //   warp 0      operand producer: dZ / act k-blocks into a two-stage ring
 //   warp 1      MMA issuer: tcgen05.mma (M = N = 128, K = 16) into accumulator (tile & 1)
 //   warp 2      TMEM allocation (256 columns); w / u chunk producer
-//   warps 4-7   epilogue, one tile row per thread (TMEM lane quarter = warp % 4): per chunk,
-//               tcgen05.ld of 32 gradient columns, the local momentum-SGD update (weight decay,
+//   warps 4-11  epilogue, two threads per tile row (TMEM lane quarter = warp % 4; warps 4-7 take
+//               a chunk's first 16 columns, warps 8-11 the last 16): per chunk,
+//               tcgen05.ld of the gradient columns, the local momentum-SGD update (weight decay,
 //               heavy-ball or Nesterov momentum, Sec. A.4) on w, u in shared memory, bf16 w
 //               into a staging buffer; thread 128 then issues the three TMA stores and
 //               recycles the slot of the chunk before once its stores have read it.
 // Only thread 128 waits on the epilogue's mbarriers and the outcome reaches the other epilogue
 // threads through a named barrier, so a wait that runs out cannot split them.
+//
+// Averaging mode (args.avg): the step ends with the K-way average of Eq. 2 (right), so a CTA takes
+// one weight tile through all G replicas in turn (replica innermost in its tile sequence).  Each
+// replica's tile gets its own gradient and local update exactly as above (u written back), and the
+// updated values are summed over the replicas with the average's TwoSum in two further TMEM
+// regions (s, c: columns 256-511); after the last replica the mean, divided as the average does,
+// goes to every replica's parameters and bf16 shadow.  Neither the per-replica parameters nor
+// their shadow reach HBM, and with args.w_rep0 (the replicas are identical at the step's start)
+// each tile's parameters are read from replica 0 only.  The results equal those of this kernel
+// in plain mode followed by the K-way average kernel, bit for bit.
 namespace wu {
 constexpr int TN = 128;                     // tile columns (= rows: BM)
 constexpr int CW = 32;                      // chunk columns (fp32: one 128-byte row)
 constexpr int ST = 2;                       // operand stages
 constexpr int NS = 4;                       // w / u chunk slots
 constexpr int NWB = 3;                      // bf16 staging buffers
-constexpr int THREADS = 256;
+constexpr int THREADS = 384;
 constexpr int EPI0 = 128;                   // first epilogue thread
+constexpr int EPI_THREADS = 256;            // two per tile row, 16 columns of a chunk each
 constexpr uint32_t kChunkF32 = BM * CW * 4;  // 16 KB
 constexpr uint32_t kChunkB16 = BM * CW * 2;  // 8 KB
 }  // namespace wu
@@ -562,6 +577,56 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
   for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
 
+// The same for one epilogue thread's half chunk: 16 gradient columns at tg and its 32-column pair
+// region at tsc (s then c, 16 each).
+__device__ __forceinline__ void tmem_ld_g16_sc32(uint32_t tg, uint32_t tsc, float (&g)[16],
+                                                 float (&sc)[32]) {
+  uint32_t a[16], b[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,"
+      "%15}, [%48];\n"
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,"
+      "%28,%29,%30,%31,%32,%33,%34,%35,%36,%37,%38,%39,%40,%41,%42,%43,%44,%45,%46,%47}, [%49];\n"
+      "tcgen05.wait::ld.sync.aligned;"
+      : "=r"(a[0]), "=r"(a[1]), "=r"(a[2]), "=r"(a[3]), "=r"(a[4]), "=r"(a[5]), "=r"(a[6]),
+        "=r"(a[7]), "=r"(a[8]), "=r"(a[9]), "=r"(a[10]), "=r"(a[11]), "=r"(a[12]), "=r"(a[13]),
+        "=r"(a[14]), "=r"(a[15]),
+        "=r"(b[0]), "=r"(b[1]), "=r"(b[2]), "=r"(b[3]), "=r"(b[4]), "=r"(b[5]), "=r"(b[6]),
+        "=r"(b[7]), "=r"(b[8]), "=r"(b[9]), "=r"(b[10]), "=r"(b[11]), "=r"(b[12]), "=r"(b[13]),
+        "=r"(b[14]), "=r"(b[15]), "=r"(b[16]), "=r"(b[17]), "=r"(b[18]), "=r"(b[19]), "=r"(b[20]),
+        "=r"(b[21]), "=r"(b[22]), "=r"(b[23]), "=r"(b[24]), "=r"(b[25]), "=r"(b[26]), "=r"(b[27]),
+        "=r"(b[28]), "=r"(b[29]), "=r"(b[30]), "=r"(b[31])
+      : "r"(tg), "r"(tsc)
+      : "memory");
+#pragma unroll
+  for (int i = 0; i < 16; ++i) g[i] = __uint_as_float(a[i]);
+#pragma unroll
+  for (int i = 0; i < 32; ++i) sc[i] = __uint_as_float(b[i]);
+}
+
+__device__ __forceinline__ void tmem_st32_nowait(uint32_t taddr, const float (&v)[32]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
+      "%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(taddr),
+      "r"(__float_as_uint(v[0])), "r"(__float_as_uint(v[1])), "r"(__float_as_uint(v[2])),
+      "r"(__float_as_uint(v[3])), "r"(__float_as_uint(v[4])), "r"(__float_as_uint(v[5])),
+      "r"(__float_as_uint(v[6])), "r"(__float_as_uint(v[7])), "r"(__float_as_uint(v[8])),
+      "r"(__float_as_uint(v[9])), "r"(__float_as_uint(v[10])), "r"(__float_as_uint(v[11])),
+      "r"(__float_as_uint(v[12])), "r"(__float_as_uint(v[13])), "r"(__float_as_uint(v[14])),
+      "r"(__float_as_uint(v[15])), "r"(__float_as_uint(v[16])), "r"(__float_as_uint(v[17])),
+      "r"(__float_as_uint(v[18])), "r"(__float_as_uint(v[19])), "r"(__float_as_uint(v[20])),
+      "r"(__float_as_uint(v[21])), "r"(__float_as_uint(v[22])), "r"(__float_as_uint(v[23])),
+      "r"(__float_as_uint(v[24])), "r"(__float_as_uint(v[25])), "r"(__float_as_uint(v[26])),
+      "r"(__float_as_uint(v[27])), "r"(__float_as_uint(v[28])), "r"(__float_as_uint(v[29])),
+      "r"(__float_as_uint(v[30])), "r"(__float_as_uint(v[31]))
+      : "memory");
+}
+
+// tcgen05.st has no wait of its own: tmem_wait_st before reading the columns back or freeing them.
+__device__ __forceinline__ void tmem_wait_st() {
+  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
 __device__ __forceinline__ void tma_store_3d(const CUtensorMap* map, const void* src, int x, int y,
                                              int z) {
   asm volatile(
@@ -591,7 +656,16 @@ __global__ void __launch_bounds__(wu::THREADS, 1) wgrad_update_kernel(
   const int nk = (args.Kd + BK - 1) / BK;
   const bool a_mn = args.L[0].A.mn_major, b_mn = args.L[0].B.mn_major;
   const bool has_u = args.sgd.u != nullptr;
+  const bool avg = args.avg != 0;
   constexpr uint32_t kBytesA = BM * BK * 2, kBytesB = wu::TN * BK * 2;
+  // This CTA's tile sequence: units blockIdx.x, blockIdx.x + gridDim.x, ...; a unit is one tile
+  // (plain mode) or one tile position of a layer taken through all G replicas (averaging mode).
+  const int units0 = avg ? tn0 * tm0 : tiles0;
+  const int units = avg ? units0 + tn1 * tm1 : tiles;
+  const int per_unit = avg ? args.G : 1;
+  const int my_count =
+      (int)blockIdx.x < units ? ((units - 1 - (int)blockIdx.x) / (int)gridDim.x + 1) * per_unit : 0;
+  const uint32_t tmem_cols = avg ? 4u * wu::TN : 2u * wu::TN;
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < wu::ST; ++i) {
@@ -612,7 +686,7 @@ __global__ void __launch_bounds__(wu::THREADS, 1) wgrad_update_kernel(
   if (warp == 2) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
                      smem_u32(&sm.tmem_base)),
-                 "r"(2u * wu::TN)
+                 "r"(tmem_cols)
                  : "memory");
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
   }
@@ -633,15 +707,31 @@ __global__ void __launch_bounds__(wu::THREADS, 1) wgrad_update_kernel(
     m0 = (r / tiles_n) * BM;
     n0 = (r % tiles_n) * wu::TN;
   };
+  // the j-th tile of this CTA's sequence; gi = its replica's position within the unit
+  auto tile_at = [&](int j, const WgradUpdateLayer*& ly, int& g, int& m0, int& n0, int& gi) {
+    const int u = (int)blockIdx.x + (j / per_unit) * (int)gridDim.x;
+    gi = j % per_unit;
+    if (!avg) {
+      tile_coords(u, ly, g, m0, n0);
+      return;
+    }
+    const bool second = u >= units0;
+    ly = second ? &args.L[1] : &args.L[0];
+    const int tiles_n = second ? tn1 : tn0;
+    const int r = second ? u - units0 : u;
+    m0 = (r / tiles_n) * BM;
+    n0 = (r % tiles_n) * wu::TN;
+    g = gi;
+  };
 
   if (warp == 0 && lane == 0) {
     // ---------------- operand producer ----------------
     int it = 0;
     bool ok = true;
-    for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x) {
+    for (int j = 0; j < my_count && ok; ++j) {
       const WgradUpdateLayer* ly;
-      int g, m0, n0;
-      tile_coords(t, ly, g, m0, n0);
+      int g, m0, n0, gi;
+      tile_at(j, ly, g, m0, n0, gi);
       for (int kb = 0; kb < nk; ++kb, ++it) {
         const int s = it % wu::ST;
         if (!mbar_wait(&sm.op_empty[s], ((it / wu::ST) & 1) ^ 1)) {
@@ -676,7 +766,7 @@ __global__ void __launch_bounds__(wu::THREADS, 1) wgrad_update_kernel(
     const uint32_t idesc = make_idesc(BM, wu::TN, a_mn, b_mn);
     int it = 0, i = 0;
     bool ok = true;
-    for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x, ++i) {
+    for (; i < my_count && ok; ++i) {
       const int ab = i & 1;
       if (!mbar_wait(&sm.acc_empty[ab], ((i >> 1) & 1) ^ 1)) break;
       asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
@@ -706,10 +796,11 @@ __global__ void __launch_bounds__(wu::THREADS, 1) wgrad_update_kernel(
     int q = 0;
     bool ok = true;
     const uint32_t bytes = wu::kChunkF32 * (has_u ? 2u : 1u);
-    for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x) {
+    for (int j = 0; j < my_count && ok; ++j) {
       const WgradUpdateLayer* ly;
-      int g, m0, n0;
-      tile_coords(t, ly, g, m0, n0);
+      int g, m0, n0, gi;
+      tile_at(j, ly, g, m0, n0, gi);
+      const int gw = (avg && args.w_rep0) ? 0 : g;  // identical replicas: read replica 0's
       const int nc = wu_chunks(ly->N, n0);
       for (int c = 0; c < nc; ++c, ++q) {
         const int sl = q % wu::NS;
@@ -718,7 +809,7 @@ __global__ void __launch_bounds__(wu::THREADS, 1) wgrad_update_kernel(
           break;
         }
         mbar_expect_tx(&sm.wu_full[sl], bytes);
-        tma_load_3d(sm.w[sl], &ly->wmap, &sm.wu_full[sl], n0 + c * wu::CW, m0, g);
+        tma_load_3d(sm.w[sl], &ly->wmap, &sm.wu_full[sl], n0 + c * wu::CW, m0, gw);
         if (has_u) tma_load_3d(sm.u[sl], &ly->umap, &sm.wu_full[sl], n0 + c * wu::CW, m0, g);
       }
     }
@@ -730,6 +821,7 @@ __global__ void __launch_bounds__(wu::THREADS, 1) wgrad_update_kernel(
     // ---------------- epilogue ----------------
     const bool leader = threadIdx.x == wu::EPI0;
     const int quarter = warp & 3;
+    const int half = (warp - 4) >> 2;   // which 16 columns of each chunk
     const int r = quarter * 32 + lane;  // tile row of this thread
     const SgdParams& sp = args.sgd;
     // The leader waits; everyone learns the outcome after the named barrier.  Two flag slots
@@ -738,17 +830,74 @@ __global__ void __launch_bounds__(wu::THREADS, 1) wgrad_update_kernel(
     int fi = 0;
     auto epi_wait = [&](uint64_t* bar, uint32_t parity) -> bool {
       if (leader) sm.epi_ok[fi] = mbar_wait(bar, parity) ? 1 : 0;
-      asm volatile("bar.sync 1, 128;" ::: "memory");
+      asm volatile("bar.sync 1, 256;" ::: "memory");
       const bool okw = sm.epi_ok[fi] != 0;
       fi ^= 1;
       return okw;
     };
+    const float Gf = (float)args.G;
+    const bool pow2 = (args.G & (args.G - 1)) == 0;
+    const float invG = 1.0f / Gf;  // exact when G is a power of two
+    // One half chunk: the update of 16 parameters per row (SG: the signSGD variant), in averaging
+    // mode folded into the running pair (s, c) and, at the unit's last replica, replaced by the
+    // mean.
+    auto half_chunk = [&](auto sg_tag, const float (&gv)[16], float (&sc)[32], uint8_t* wrow,
+                          uint8_t* urow, uint8_t* brow, bool first, bool last) {
+      constexpr bool SG = decltype(sg_tag)::value;
+      const bool write_w = !avg || last;  // the parameters leave this chunk for HBM
+      uint32_t packed[8];
+#pragma unroll
+      for (int jj = 0; jj < 4; ++jj) {
+        const int j = 4 * half + jj;  // float4 column group within the 32-column chunk
+        const int phys = (j ^ (r & 7)) << 4;
+        float4 wv = *reinterpret_cast<const float4*>(wrow + phys);
+        float4 uv = has_u ? *reinterpret_cast<const float4*>(urow + phys)
+                          : make_float4(0.f, 0.f, 0.f, 0.f);
+        sgd4<SG>(wv, uv, make_float4(gv[4 * jj], gv[4 * jj + 1], gv[4 * jj + 2], gv[4 * jj + 3]), sp);
+        if (has_u) *reinterpret_cast<float4*>(urow + phys) = uv;
+        if (avg) {
+          float* sv = sc + 4 * jj;       // s of these four columns
+          float* cv = sc + 16 + 4 * jj;  // c of these four columns
+          const float wn[4] = {wv.x, wv.y, wv.z, wv.w};
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            if (first) {
+              sv[e] = wn[e];
+              cv[e] = 0.f;
+            } else {
+              two_sum_add(sv[e], cv[e], wn[e]);
+            }
+          }
+          if (last) {
+            float m[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e)
+              m[e] = pow2 ? mean_of_pow2(sv[e], cv[e], Gf, invG) : mean_of(sv[e], cv[e], Gf);
+            wv = make_float4(m[0], m[1], m[2], m[3]);
+          }
+        }
+        if (write_w) {
+          *reinterpret_cast<float4*>(wrow + phys) = wv;
+          packed[2 * jj] = (uint32_t)f2bf(wv.x) | ((uint32_t)f2bf(wv.y) << 16);
+          packed[2 * jj + 1] = (uint32_t)f2bf(wv.z) | ((uint32_t)f2bf(wv.w) << 16);
+        }
+      }
+      if (write_w) {
+#pragma unroll
+        for (int hh = 0; hh < 2; ++hh) {
+          const int h = 2 * half + hh;  // 16-byte unit of the 64-byte bf16 row
+          *reinterpret_cast<uint4*>(brow + ((h ^ ((r >> 1) & 3)) << 4)) =
+              make_uint4(packed[4 * hh], packed[4 * hh + 1], packed[4 * hh + 2], packed[4 * hh + 3]);
+        }
+      }
+    };
     int q = 0, i = 0, wbi = 0;
     bool ok = true;
-    for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x, ++i) {
+    for (; i < my_count && ok; ++i) {
       const WgradUpdateLayer* ly;
-      int g, m0, n0;
-      tile_coords(t, ly, g, m0, n0);
+      int g, m0, n0, gi;
+      tile_at(i, ly, g, m0, n0, gi);
+      const bool first = gi == 0, last = gi == per_unit - 1;
       const int ab = i & 1;
       const int nc = wu_chunks(ly->N, n0);
       if (!epi_wait(&sm.acc_full[ab], (i >> 1) & 1)) {
@@ -763,36 +912,42 @@ __global__ void __launch_bounds__(wu::THREADS, 1) wgrad_update_kernel(
           break;
         }
         mbar_try_wait(&sm.wu_full[sl], (q / wu::NS) & 1);  // acquire the TMA-written data
-        float gv[32];
-        tmem_ld32(tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(ab * wu::TN + c * wu::CW), gv);
+        const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
+        const uint32_t g_col = (uint32_t)(ab * wu::TN + c * wu::CW + 16 * half);
+        // averaging mode: this thread's running pair of the chunk over the replicas so far, 32
+        // columns from 256 + 64 chunk + 32 half (s in sc[0..15], c in sc[16..31])
+        const uint32_t sc_col = 2u * wu::TN + (uint32_t)(c * 2 * wu::CW + 32 * half);
+        float gv[16], sc[32];
+        if (avg && !first) {
+          tmem_wait_st();  // this chunk's pair, stored at the previous replica
+          tmem_ld_g16_sc32(tmem + lane_base + g_col, tmem + lane_base + sc_col, gv, sc);
+        } else {
+          tmem_ld16(tmem + lane_base + g_col, gv);
+        }
         uint8_t* wrow = sm.w[sl] + r * 128;
         uint8_t* urow = sm.u[sl] + r * 128;
         uint8_t* brow = sm.wb[wbi] + r * 64;
-        uint32_t packed[16];
-#pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          const int phys = (j ^ (r & 7)) << 4;
-          float4 wv = *reinterpret_cast<const float4*>(wrow + phys);
-          float4 uv = has_u ? *reinterpret_cast<const float4*>(urow + phys)
-                            : make_float4(0.f, 0.f, 0.f, 0.f);
-          sgd4(wv, uv, make_float4(gv[4 * j], gv[4 * j + 1], gv[4 * j + 2], gv[4 * j + 3]), sp);
-          *reinterpret_cast<float4*>(wrow + phys) = wv;
-          if (has_u) *reinterpret_cast<float4*>(urow + phys) = uv;
-          packed[2 * j] = (uint32_t)f2bf(wv.x) | ((uint32_t)f2bf(wv.y) << 16);
-          packed[2 * j + 1] = (uint32_t)f2bf(wv.z) | ((uint32_t)f2bf(wv.w) << 16);
-        }
-#pragma unroll
-        for (int h = 0; h < 4; ++h)
-          *reinterpret_cast<uint4*>(brow + ((h ^ ((r >> 1) & 3)) << 4)) =
-              make_uint4(packed[4 * h], packed[4 * h + 1], packed[4 * h + 2], packed[4 * h + 3]);
+        if (sp.sign)
+          half_chunk(std::true_type{}, gv, sc, wrow, urow, brow, first, last);
+        else
+          half_chunk(std::false_type{}, gv, sc, wrow, urow, brow, first, last);
+        if (avg && !last) tmem_st32_nowait(tmem + lane_base + sc_col, sc);
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
         asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-        asm volatile("bar.sync 1, 128;" ::: "memory");
+        asm volatile("bar.sync 1, 256;" ::: "memory");
         if (leader) {
           const int x = n0 + c * wu::CW;
-          tma_store_3d(&ly->wmap, sm.w[sl], x, m0, g);
           if (has_u) tma_store_3d(&ly->umap, sm.u[sl], x, m0, g);
-          if (sp.wb) tma_store_3d(&ly->wbmap, sm.wb[wbi], x, m0, g);
+          if (!avg) {
+            tma_store_3d(&ly->wmap, sm.w[sl], x, m0, g);
+            if (sp.wb) tma_store_3d(&ly->wbmap, sm.wb[wbi], x, m0, g);
+          } else if (last) {
+            // the mean to every replica of the unit
+            for (int k = 0; k < args.G; ++k) {
+              tma_store_3d(&ly->wmap, sm.w[sl], x, m0, k);
+              if (sp.wb) tma_store_3d(&ly->wbmap, sm.wb[wbi], x, m0, k);
+            }
+          }
           asm volatile("cp.async.bulk.commit_group;" ::: "memory");
           // the stores of the chunk before have read their slot: hand it back to the producer
           asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
@@ -802,13 +957,14 @@ __global__ void __launch_bounds__(wu::THREADS, 1) wgrad_update_kernel(
       }
     }
     if (leader) asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+    tmem_wait_st();  // no tensor-memory store outstanding when the columns are freed
     (void)ok;
   }
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
   __syncthreads();
   if (warp == 2) {
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
-                 "r"(2u * wu::TN)
+                 "r"(tmem_cols)
                  : "memory");
   }
 }
@@ -1406,6 +1562,8 @@ cudaError_t launch_wgrad_update(const WgradUpdateArgs& a, cudaStream_t stream) {
     tiles += (int64_t)((ly.N + wu::TN - 1) / wu::TN) * ((ly.M + BM - 1) / BM) * a.G;
   }
   if (tiles > 0x7fffffffLL) return cudaErrorInvalidValue;
+  // averaging mode: a CTA per tile position (all G replicas of it), at most one per SM
+  const int64_t units = a.avg ? tiles / a.G : tiles;
   int dev = 0, sms = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
@@ -1419,7 +1577,7 @@ cudaError_t launch_wgrad_update(const WgradUpdateArgs& a, cudaStream_t stream) {
     if (e != cudaSuccess) return e;
     attr_dev = dev;
   }
-  const int grid = (int)std::min<int64_t>(tiles, sms);
+  const int grid = (int)std::min<int64_t>(units, sms);
   launch_pdl(wgrad_update_kernel, dim3(grid), dim3(wu::THREADS), smem, stream, a);
   return cudaGetLastError();
 }

@@ -294,24 +294,14 @@ __global__ void __launch_bounds__(256) sgd_update_kernel(
 // ---------------------------------------------------------------------------------------------
 // K-way average (Eq. 2 right).  A thread owns one float4 column of every replica of its group and
 // walks the replicas in order with eight loads in flight (a warp's load instruction reads 512
-// contiguous bytes of one replica).  The sum is accumulated without loss: every addition is an
-// error-free transformation (Knuth's TwoSum: s + x = t + e exactly), the rounding errors e are
-// summed in a second register, and the pair (s, c) is divided by K with the remainder of the first
-// quotient taken exactly by an fma.  The result is the correctly rounded fp32 mean in all but
-// hard midpoint cases, whatever K (a plain fp32 sum loses up to K - 1 roundings), and the mean of
-// identical replicas is that replica.  A column-per-thread walk keeps every load coalesced; a
-// shuffle reduction across lanes would need lanes to hold different replicas of one column.
+// contiguous bytes of one replica), accumulating with two_sum_add and dividing with mean_of
+// (common.cuh): the correctly rounded fp32 mean in all but hard midpoint cases, whatever K (a
+// plain fp32 sum loses up to K - 1 roundings), and the mean of identical replicas is that replica.
+// A column-per-thread walk keeps every load coalesced; a shuffle reduction across lanes would need
+// lanes to hold different replicas of one column.
 struct TwoSum4 {
   float4 s, c;
 };
-
-__device__ __forceinline__ void two_sum_add(float& s, float& c, float x) {
-  const float t = __fadd_rn(s, x);
-  const float z = __fsub_rn(t, s);
-  const float e = __fadd_rn(__fsub_rn(s, __fsub_rn(t, z)), __fsub_rn(x, z));
-  s = t;
-  c = __fadd_rn(c, e);
-}
 
 __device__ __forceinline__ void two_sum_add4(TwoSum4& a, const float4& v) {
   two_sum_add(a.s.x, a.c.x, v.x);
@@ -320,11 +310,41 @@ __device__ __forceinline__ void two_sum_add4(TwoSum4& a, const float4& v) {
   two_sum_add(a.s.w, a.c.w, v.w);
 }
 
-// (s + c) / K: q = s / K, the exact remainder s - q K by fma, corrected by c and divided again.
-__device__ __forceinline__ float mean_of(float s, float c, float Kf) {
-  const float q = __fdiv_rn(s, Kf);
-  const float r = __fadd_rn(__fmaf_rn(-q, Kf, s), c);
-  return __fadd_rn(q, __fdiv_rn(r, Kf));
+// Average column `col` (float4 units) of K replicas spaced rs4 float4 apart, in place, and write
+// its bf16 copy.
+template <bool SHADOW>
+__device__ __forceinline__ void average_column(float4* __restrict__ W, uint2* __restrict__ Wb, int K,
+                                               int64_t rs4, int64_t col, float Kf) {
+  TwoSum4 acc;
+  acc.s = __ldcs(W + col);
+  acc.c = make_float4(0.f, 0.f, 0.f, 0.f);
+  int k = 1;
+  for (; k + 8 <= K; k += 8) {
+    float4 v[8];
+#pragma unroll
+    for (int q = 0; q < 8; ++q) v[q] = __ldcs(W + (int64_t)(k + q) * rs4 + col);
+#pragma unroll
+    for (int q = 0; q < 8; ++q) two_sum_add4(acc, v[q]);
+  }
+  for (; k < K; ++k) two_sum_add4(acc, __ldcs(W + (int64_t)k * rs4 + col));
+  float4 mean;
+  if ((K & (K - 1)) == 0) {
+    const float inv = 1.0f / Kf;  // exact for a power of two
+    mean = make_float4(mean_of_pow2(acc.s.x, acc.c.x, Kf, inv), mean_of_pow2(acc.s.y, acc.c.y, Kf, inv),
+                       mean_of_pow2(acc.s.z, acc.c.z, Kf, inv), mean_of_pow2(acc.s.w, acc.c.w, Kf, inv));
+  } else {
+    mean = make_float4(mean_of(acc.s.x, acc.c.x, Kf), mean_of(acc.s.y, acc.c.y, Kf),
+                       mean_of(acc.s.z, acc.c.z, Kf), mean_of(acc.s.w, acc.c.w, Kf));
+  }
+  uint2 o;
+  if (SHADOW) {
+    o.x = (uint32_t)f2bf(mean.x) | ((uint32_t)f2bf(mean.y) << 16);
+    o.y = (uint32_t)f2bf(mean.z) | ((uint32_t)f2bf(mean.w) << 16);
+  }
+  for (int kk = 0; kk < K; ++kk) {
+    __stcs(W + (int64_t)kk * rs4 + col, mean);
+    if (SHADOW) __stcs(Wb + (int64_t)kk * rs4 + col, o);
+  }
 }
 
 template <bool SHADOW>
@@ -337,31 +357,22 @@ __global__ void __launch_bounds__(256) kway_average_kernel(float4* __restrict__ 
   if (SHADOW) Wb += (int64_t)blockIdx.y * K * d4;
   const float Kf = (float)K;
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-  for (int64_t col = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; col < d4; col += stride) {
-    TwoSum4 acc;
-    acc.s = __ldcs(W + col);
-    acc.c = make_float4(0.f, 0.f, 0.f, 0.f);
-    int k = 1;
-    for (; k + 8 <= K; k += 8) {
-      float4 v[8];
-#pragma unroll
-      for (int q = 0; q < 8; ++q) v[q] = __ldcs(W + (int64_t)(k + q) * d4 + col);
-#pragma unroll
-      for (int q = 0; q < 8; ++q) two_sum_add4(acc, v[q]);
-    }
-    for (; k < K; ++k) two_sum_add4(acc, __ldcs(W + (int64_t)k * d4 + col));
-    const float4 mean = make_float4(mean_of(acc.s.x, acc.c.x, Kf), mean_of(acc.s.y, acc.c.y, Kf),
-                                    mean_of(acc.s.z, acc.c.z, Kf), mean_of(acc.s.w, acc.c.w, Kf));
-    uint2 o;
-    if (SHADOW) {
-      o.x = (uint32_t)f2bf(mean.x) | ((uint32_t)f2bf(mean.y) << 16);
-      o.y = (uint32_t)f2bf(mean.z) | ((uint32_t)f2bf(mean.w) << 16);
-    }
-    for (int kk = 0; kk < K; ++kk) {
-      __stcs(W + (int64_t)kk * d4 + col, mean);
-      if (SHADOW) __stcs(Wb + (int64_t)kk * d4 + col, o);
-    }
-  }
+  for (int64_t col = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; col < d4; col += stride)
+    average_column<SHADOW>(W, Wb, K, d4, col, Kf);
+}
+
+// The same average restricted to a list of parameter segments of every replica (blockIdx.y =
+// segment): the tensors a weight-gradient + update + average launch does not cover.
+template <bool SHADOW>
+__global__ void __launch_bounds__(256) kway_average_segments_kernel(float4* __restrict__ W,
+                                                                    uint2* __restrict__ Wb, int K,
+                                                                    int64_t rs4, AvgSegments sg) {
+  pdl_begin();
+  const int64_t off4 = sg.off4[blockIdx.y], n4 = sg.len4[blockIdx.y];
+  const float Kf = (float)K;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n4; i += stride)
+    average_column<SHADOW>(W, Wb, K, rs4, off4 + i, Kf);
 }
 
 // ---------------------------------------------------------------------------------------------
@@ -775,6 +786,29 @@ cudaError_t launch_group_average(float* W, uint16_t* Wb, int Kp, int groups, int
   else
     launch_pdl(kway_average_kernel<false>, grid, threads, 0, stream, reinterpret_cast<float4*>(W), nullptr,
                                                              Kp, d4);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_average_segments(float* W, uint16_t* Wb, int K, int64_t d_pad,
+                                   const AvgSegments& sg, cudaStream_t stream) {
+  if (K < 1 || sg.n <= 0) return cudaSuccess;
+  if ((d_pad & 3) || sg.n > kMaxAvgSegments) return cudaErrorInvalidValue;
+  int64_t longest = 0;
+  for (int i = 0; i < sg.n; ++i) {
+    if (sg.off4[i] < 0 || sg.len4[i] < 0 || 4 * (sg.off4[i] + sg.len4[i]) > d_pad)
+      return cudaErrorInvalidValue;
+    longest = std::max<int64_t>(longest, sg.len4[i]);
+  }
+  if (longest == 0) return cudaSuccess;
+  const int threads = 256;
+  const int blocks = (int)std::min<int64_t>((longest + threads - 1) / threads, 1024);
+  dim3 grid(blocks, sg.n);
+  if (Wb)
+    launch_pdl(kway_average_segments_kernel<true>, grid, threads, 0, stream,
+               reinterpret_cast<float4*>(W), reinterpret_cast<uint2*>(Wb), K, d_pad / 4, sg);
+  else
+    launch_pdl(kway_average_segments_kernel<false>, grid, threads, 0, stream,
+               reinterpret_cast<float4*>(W), nullptr, K, d_pad / 4, sg);
   return cudaGetLastError();
 }
 

@@ -87,6 +87,16 @@ cudaError_t launch_sign_sync(float* W, uint16_t* Wb, float* wref, float* E, cons
 cudaError_t launch_gm_sync(float* W, uint16_t* Wb, float* wref, float* ug, int K, int64_t d,
                            float lr, float mg, cudaStream_t stream);
 cudaError_t launch_kway_average(float* W, uint16_t* Wb, int K, int64_t d, cudaStream_t stream);
+// Segments of a replica (float4 offset and length, within d_pad) for the segment average.
+constexpr int kMaxAvgSegments = 2 * 8 + 2;
+struct AvgSegments {
+  int n;
+  int64_t off4[kMaxAvgSegments], len4[kMaxAvgSegments];
+};
+// The K-way average of kway_average restricted to the listed segments of each replica.
+cudaError_t launch_average_segments(float* W, uint16_t* Wb, int K, int64_t d_pad,
+                                   const AvgSegments& sg, cudaStream_t stream);
+
 // Average within each of `groups` groups of Kp consecutive replicas (replica stride d).
 cudaError_t launch_group_average(float* W, uint16_t* Wb, int Kp, int groups, int64_t d,
                                  cudaStream_t stream);
@@ -253,6 +263,11 @@ struct WgradUpdateArgs {
   int Kd, G, nl;
   WgradUpdateLayer L[kWgradMaxLayers];
   SgdParams sgd;
+  // avg = 1: the step ends with the K-way average (Eq. 2 right): every replica's tile is updated
+  // as above, and the mean of the updated tiles (the average kernel's arithmetic) is written to
+  // all G replicas' parameters and shadow.  w_rep0 = 1 (avg only): the replicas are identical at
+  // the step's start, so each tile's parameters are read from replica 0.
+  int avg, w_rep0;
 };
 cudaError_t launch_wgrad_update(const WgradUpdateArgs& a, cudaStream_t stream);
 // The classifier head (last dense layer with at most kHeadMaxClasses outputs, bf16 mode): the

@@ -104,6 +104,12 @@ struct lsgd_ctx {
   float* pnorm = nullptr;  // [K] ||Delta_k||_1 / d
   float* l1part = nullptr; // [K][l1_chunks] partial sums
   RoundCursor cursor;       // the round lsgd_run last stood in (local-step warm-up)
+  // every replica holds the same parameters (after creation, a global average or a broadcast
+  // lsgd_set_params); lets a step that ends with the average read each weight tile once
+  bool synced = true;
+  // the parameter segments a weight-gradient + update + average launch does not cover (the
+  // biases and the classifier head's tensors), averaged by a small kernel after it
+  lsgd::AvgSegments avg_segs{};
   bool prof_on = false;
   std::vector<cudaEvent_t> prof_pool;
   size_t prof_used = 0;
@@ -439,7 +445,7 @@ lsgd::HeadArgs head_args(lsgd_ctx* c) {
 
 // Backward of every dense layer, last to first: data gradient (it reads this layer's weights, so
 // it runs before a fused update may change them), weight gradient, bias gradient.
-lsgd_status dense_backward(lsgd_ctx* c) {
+lsgd_status dense_backward(lsgd_ctx* c, bool avg) {
   const int K = c->cfg.K, B = c->cfg.B_loc;
   const int L = (int)c->layers.size();
   const void* Wop = c->bf16 ? (const void*)c->Wb : (const void*)c->W;
@@ -611,6 +617,8 @@ lsgd_status dense_backward(lsgd_ctx* c) {
         if (!(l == 1 && c->layers[0].tc)) {
           wa.Kd = B;
           wa.G = K;
+          wa.avg = avg ? 1 : 0;
+          wa.w_rep0 = (avg && c->synced) ? 1 : 0;
           LSGD_LAUNCH(c, lsgd::launch_wgrad_update(wa, c->stream));
           wa.nl = 0;
           span(LSGD_PH_UPDATE);
@@ -686,8 +694,17 @@ lsgd_status do_update(lsgd_ctx* c) {
   return LSGD_OK;
 }
 
-// The step body after the inputs of this step are gathered into act[0] / yb / tb.
-lsgd_status step_body(lsgd_ctx* c, int64_t e_start) {
+// Whether a step that ends with the global average can run it inside its update launches:
+// dense bf16 model with the fused update on the tensor cores, plain averaging.
+bool can_fuse_average(const lsgd_ctx* c) {
+  return c->fused && !c->resnet && c->cfg.compress == LSGD_COMPRESS_NONE &&
+         c->cfg.global_momentum <= 0.0;
+}
+
+// The step body after the inputs of this step are gathered into act[0] / yb / tb.  avg: the step
+// ends with the K-way average, done by the update launches and the segment average
+// (can_fuse_average must hold).
+lsgd_status step_body(lsgd_ctx* c, int64_t e_start, bool avg = false) {
   const int K = c->cfg.K;
   float* loss_slot = c->loss_hist + (c->step % c->loss_cap) * K;
   lsgd_status st;
@@ -719,7 +736,7 @@ lsgd_status step_body(lsgd_ctx* c, int64_t e_start) {
     if (st != LSGD_OK) return st;
     const int64_t e_loss = prof_mark(c);
     prof_span(c, LSGD_PH_LOSS, e_fwd, e_loss);
-    st = dense_backward(c);
+    st = dense_backward(c, avg);
     if (st != LSGD_OK) return st;
     e_bwd = prof_mark(c);
     if (!c->fused) prof_span(c, LSGD_PH_BACKWARD, e_loss, e_bwd);
@@ -730,6 +747,13 @@ lsgd_status step_body(lsgd_ctx* c, int64_t e_start) {
     prof_span(c, LSGD_PH_UPDATE, e_bwd, prof_mark(c));
   }
   c->step++;
+  if (avg) {
+    // the tensors the update launches did not average (biases, classifier head)
+    LSGD_LAUNCH(c, lsgd::launch_average_segments(c->W, c->Wb, K, c->d_pad, c->avg_segs, c->stream));
+    prof_span(c, LSGD_PH_AVERAGE, e_bwd, prof_mark(c));
+    c->syncs++;
+  }
+  c->synced = avg || c->cfg.K == 1;
   return LSGD_OK;
 }
 
@@ -904,6 +928,22 @@ lsgd_status lsgd_create(const lsgd_config* cfg, const lsgd_allocator* alloc, voi
     if (st == LSGD_OK) {
       const DenseLayer& top = c->layers.back();
       c->head = c->bf16 && !c->lsq && top.tc && lsgd::head_supported(top.out, c0.B_loc, top.in);
+      // segments averaged outside the weight-gradient + update launches: every bias, and the
+      // classifier head's weights when its own kernels update them (each tensor starts at a
+      // 64-element boundary, so a length rounded up to 4 stays inside its padding)
+      lsgd::AvgSegments& sg = c->avg_segs;
+      sg.n = 0;
+      for (size_t l = 0; l < c->layers.size(); ++l) {
+        const DenseLayer& Ly = c->layers[l];
+        if (c->head && l + 1 == c->layers.size()) {
+          sg.off4[sg.n] = Ly.w_off / 4;
+          sg.len4[sg.n++] = ((int64_t)Ly.in * Ly.out + 3) / 4;
+        }
+        if (Ly.b_off >= 0) {
+          sg.off4[sg.n] = Ly.b_off / 4;
+          sg.len4[sg.n++] = ((int64_t)Ly.out + 3) / 4;
+        }
+      }
     }
   }
   if (st != LSGD_OK) {
@@ -983,7 +1023,7 @@ lsgd_status lsgd_set_targets(lsgd_ctx* c, const float* X, const float* targets, 
   return set_data(c, X, nullptr, targets, N);
 }
 
-lsgd_status lsgd_local_step(lsgd_ctx* c) {
+static lsgd_status local_step(lsgd_ctx* c, bool avg) {
   if (!c) return fail(nullptr, LSGD_EINVAL, "NULL context");
   if (!c->have_data) return fail(c, LSGD_ESTATE, "lsgd_set_dataset must come first");
   const int K = c->cfg.K, B = c->cfg.B_loc;
@@ -993,10 +1033,13 @@ lsgd_status lsgd_local_step(lsgd_ctx* c) {
   LSGD_LAUNCH(c, lsgd::launch_gather_rows(input_buffer(c), c->bf16, input_ld(c), c->X, c->D, c->idx,
                                           K * B, c->y, c->y ? c->yb : nullptr, c->t,
                                           c->t ? c->tb : nullptr, c->stream));
-  return step_body(c, e0);
+  return step_body(c, e0, avg);
 }
 
-lsgd_status lsgd_local_step_batch(lsgd_ctx* c, const float* x, const void* lab, int on_device) {
+lsgd_status lsgd_local_step(lsgd_ctx* c) { return local_step(c, false); }
+
+static lsgd_status local_step_batch(lsgd_ctx* c, const float* x, const void* lab, int on_device,
+                                    bool avg) {
   if (!c || !x || !lab) return fail(c, LSGD_EINVAL, "NULL argument");
   const int K = c->cfg.K, B = c->cfg.B_loc;
   const size_t rows = (size_t)K * B;
@@ -1040,7 +1083,11 @@ lsgd_status lsgd_local_step_batch(lsgd_ctx* c, const float* x, const void* lab, 
     LSGD_TRY_CUDA(c, cudaEventRecord(c->stage_free[sl], c->stream));
     c->stage_used[sl] = true;
   }
-  return step_body(c, e0);
+  return step_body(c, e0, avg);
+}
+
+lsgd_status lsgd_local_step_batch(lsgd_ctx* c, const float* x, const void* lab, int on_device) {
+  return local_step_batch(c, x, lab, on_device, false);
 }
 
 lsgd_status lsgd_sync_average(lsgd_ctx* c) {
@@ -1063,6 +1110,7 @@ lsgd_status lsgd_sync_average(lsgd_ctx* c) {
   }
   prof_span(c, LSGD_PH_AVERAGE, e0, prof_mark(c));
   c->syncs++;
+  c->synced = true;  // every variant leaves all replicas at one model
   return LSGD_OK;
 }
 
@@ -1074,6 +1122,7 @@ lsgd_status lsgd_block_average(lsgd_ctx* c) {
                                             c->cfg.K / c->cfg.hier_block, c->d_pad, c->stream));
   prof_span(c, LSGD_PH_AVERAGE, e0, prof_mark(c));
   c->block_syncs++;
+  c->synced = c->cfg.hier_block >= c->cfg.K;
   return LSGD_OK;
 }
 
@@ -1104,10 +1153,15 @@ lsgd_status lsgd_run(lsgd_ctx* c, int64_t n_steps) {
   if (!c) return fail(nullptr, LSGD_EINVAL, "NULL context");
   if (n_steps < 0) return fail(c, LSGD_EINVAL, "n_steps must be >= 0");
   for (int64_t i = 0; i < n_steps; ++i) {
-    const int64_t s = c->step;
+    const int kind = sync_kind_at(c->cfg, c->T, c->step, &c->cursor);
+    if (kind == 2 && can_fuse_average(c)) {
+      // the step's update launches also form the K-way average
+      lsgd_status st = local_step(c, true);
+      if (st != LSGD_OK) return st;
+      continue;
+    }
     lsgd_status st = lsgd_local_step(c);
     if (st != LSGD_OK) return st;
-    const int kind = sync_kind_at(c->cfg, c->T, s, &c->cursor);
     if (kind == 2) {
       st = lsgd_sync_average(c);
       if (st != LSGD_OK) return st;
@@ -1116,6 +1170,18 @@ lsgd_status lsgd_run(lsgd_ctx* c, int64_t n_steps) {
       if (st != LSGD_OK) return st;
     }
   }
+  return LSGD_OK;
+}
+
+lsgd_status lsgd_run_batch(lsgd_ctx* c, const float* x, const void* labels_or_targets,
+                           int on_device) {
+  if (!c) return fail(nullptr, LSGD_EINVAL, "NULL context");
+  const int kind = sync_kind_at(c->cfg, c->T, c->step, &c->cursor);
+  const bool fuse = kind == 2 && can_fuse_average(c);
+  lsgd_status st = local_step_batch(c, x, labels_or_targets, on_device, fuse);
+  if (st != LSGD_OK || fuse) return st;
+  if (kind == 2) return lsgd_sync_average(c);
+  if (kind == 1) return lsgd_block_average(c);
   return LSGD_OK;
 }
 
@@ -1182,6 +1248,7 @@ static lsgd_status set_vec(lsgd_ctx* c, float* buf, int k, const float* src, siz
                                      c->stream));
   if (is_w && c->Wb)
     LSGD_LAUNCH(c, lsgd::launch_to_bf16(c->W, c->Wb, (int64_t)c->cfg.K * c->d_pad, c->stream));
+  if (is_w) c->synced = k < 0 || c->cfg.K == 1;
   LSGD_TRY_CUDA(c, cudaStreamSynchronize(c->stream));
   return LSGD_OK;
 }
@@ -1450,6 +1517,7 @@ lsgd_status lsgd_load(lsgd_ctx* c, const char* path) {
   c->step = hdr[3];
   c->syncs = hdr[4];
   c->block_syncs = hdr[6];
+  c->synced = c->cfg.K == 1;  // the file does not say whether the replicas agree
   return LSGD_OK;
 }
 

@@ -169,8 +169,8 @@ def test_post_local_mlp4096_sampled_replica(P):
     tp = T // 2
     X, y = synthdata.gaussian_mixture_cached(N, 3072, 100, 1234)
     g, o = dense_cfgs(P, widths=widths, K=K, B=B, H=16, T=T, N=N, precision=P.BF16, t_switch=tp,
-                      base_lr=0.1, scale_by_K=True, warmup_epochs=5, milestones=(0.5, 0.75),
-                      momentum=0.9, nesterov=True, weight_decay=5e-4, seed=3, fused_update=True)
+                      base_lr=0.1, milestones=(0.5, 0.75), momentum=0.9, nesterov=True,
+                      weight_decay=5e-4, seed=3, fused_update=True)
     w0 = oracle.init_params(o)
     ctx = P.lsgd_create(g)
     P.lsgd_set_dataset(ctx, X, y)
@@ -190,6 +190,8 @@ def test_post_local_mlp4096_sampled_replica(P):
     assert P.lsgd_sync_count(ctx) == tp + -(-(T - tp) // 16)
     assert P.lsgd_check_finite(ctx)
     lg = P.lsgd_losses(ctx, T, K)
+    # the configured job trains: every loss finite, the last round's mean well below the first's
+    assert np.isfinite(lg).all() and lg[-16:].mean() < 0.7 * lg[:16].mean()
     print("post-local MLP4096 mean loss every 16 steps:", lg.mean(1)[::16].round(3).tolist())
     P.lsgd_destroy(ctx)
 
@@ -244,3 +246,66 @@ def test_hierarchical_local_sgd(P):
     assert rel_l2(P.lsgd_params(ctx, -1), W[0]) <= 2e-2
     assert np.abs(P.lsgd_losses(ctx, T, K) - lo).max() <= 2e-2
     P.lsgd_destroy(ctx)
+
+
+@pytest.mark.parametrize("mom,nest,wd", [(0.9, True, 5e-4), (0.9, False, 0.0), (0.0, False, 1e-4)])
+@pytest.mark.parametrize("widths,K,B", [((264, 136, 72, 10), 3, 40),
+                                        ((200, 136, 96, 72, 100), 4, 24),
+                                        ((3072, 1024, 1024, 10), 16, 128)])
+def test_average_in_update_launches_is_bitwise_identical(P, mom, nest, wd, widths, K, B):
+    # lsgd_run forms the K-way average of a round-ending step inside that step's weight-gradient
+    # + update launches (Eq. 2: the mean of the updated replicas).  Post-local schedule: steps 0-4
+    # average after every step (the replicas are identical at each step's start), then rounds of
+    # three (the round's last step starts from different replicas).  The separate path -- local
+    # steps, then lsgd_sync_average -- must give the same parameters, momentum and losses.
+    N, T = 2048, 12
+    X, y = synthdata.gaussian_mixture(N, widths[0], widths[-1], seed=12)
+    res = []
+    for fused_avg in (True, False):
+        g, o = dense_cfgs(P, widths=widths, K=K, B=B, H=3, T=T, N=N, precision=P.BF16,
+                          t_switch=5, base_lr=0.05, momentum=mom, nesterov=nest, weight_decay=wd,
+                          seed=7, fused_update=True, milestones=(0.5,))
+        ctx = P.lsgd_create(g)
+        P.lsgd_set_dataset(ctx, X, y)
+        if fused_avg:
+            P.lsgd_run(ctx, T)
+        else:
+            _, kinds = P.lsgd_schedule(g, T)
+            for s in range(T):
+                P.lsgd_local_step(ctx)
+                if kinds[s] == 2:
+                    P.lsgd_sync_average(ctx)
+        res.append(([P.lsgd_params(ctx, k) for k in range(K)],
+                    [P.lsgd_momentum(ctx, k) for k in range(K)] if mom else [],
+                    P.lsgd_losses(ctx, T, K), P.lsgd_sync_count(ctx)))
+        P.lsgd_destroy(ctx)
+    assert res[0][3] == res[1][3] == 5 + 3  # t' syncs, then steps 7, 10 and the last (11)
+    for k in range(K):
+        assert np.array_equal(res[0][0][k], res[1][0][k]), k
+        if mom:
+            assert np.array_equal(res[0][1][k], res[1][1][k]), k
+    assert np.array_equal(res[0][2], res[1][2])
+
+
+def test_run_batch_matches_run(P):
+    # lsgd_run_batch on the mini-batches lsgd_run samples (host buffers) is the same schedule
+    widths, K, B, N, T = (264, 136, 72, 10), 4, 32, 2048, 9
+    X, y = synthdata.gaussian_mixture(N, widths[0], 10, seed=13)
+    g, o = dense_cfgs(P, widths=widths, K=K, B=B, H=2, T=T, N=N, precision=P.BF16, t_switch=3,
+                      base_lr=0.05, momentum=0.9, nesterov=True, weight_decay=5e-4, seed=5,
+                      fused_update=True)
+    a = P.lsgd_create(g)
+    P.lsgd_set_dataset(a, X, y)
+    P.lsgd_run(a, T)
+    b = P.lsgd_create(g)
+    P.lsgd_set_dataset(b, X, y)
+    for s in range(T):
+        idx = P.lsgd_debug_indices(b, s, K, B).reshape(-1)
+        P.lsgd_run_batch(b, np.ascontiguousarray(X[idx].reshape(K, B, -1)),
+                         np.ascontiguousarray(y[idx].reshape(K, B)))
+    assert P.lsgd_sync_count(a) == P.lsgd_sync_count(b) == 3 + 3
+    for k in range(K):
+        assert np.array_equal(P.lsgd_params(a, k), P.lsgd_params(b, k)), k
+    assert np.array_equal(P.lsgd_losses(a, T, K), P.lsgd_losses(b, T, K))
+    P.lsgd_destroy(a)
+    P.lsgd_destroy(b)

@@ -493,6 +493,11 @@ class DenseRun:
         self.ctx = P.lsgd_create(self.cfg, stream=stream.cuda_stream)
         P.lsgd_set_dataset(self.ctx, self.X, self.y)
         self.d = P.lsgd_num_params(self.ctx)
+        _, self.kinds = P.lsgd_schedule(self.cfg, self.T)
+        # round-ending steps form the average inside their update launches (fused bf16 path)
+        self.fuse_avg = fused and w["bf16"]
+        self.fused = fused and w["bf16"]
+        self.traced_steps = []
 
     def run_steps(self, n):
         P = self.P
@@ -528,6 +533,8 @@ class DenseRun:
         import torch
 
         P = self.P
+        s0 = P.lsgd_step_count(self.ctx)
+        self.traced_steps = [(s0 + i) % self.T for i in range(n)]
         P.lsgd_profile_enable(self.ctx, True)
         self.run_steps(n)
         torch.cuda.synchronize()
@@ -535,31 +542,79 @@ class DenseRun:
         P.lsgd_profile_enable(self.ctx, False)
         return prof
 
-    def update_bytes(self, fused=True):
-        """Algorithmic bytes of one step's update launches."""
+    def step_bytes(self, s):
+        """Algorithmic bytes of step s's update launches and of its averaging launches.  Per
+        parameter and replica (fp32 w, u; bf16 shadow): the fused update reads w, u and writes
+        w, u and the shadow (18 B); a step that ends with the average forms it in the same
+        launches and writes w and the shadow once, as the mean (u 8 B + w 4 B + shadow 2 B +
+        the read of w: once per tile, 4 / K B, when the replicas were identical at the step's
+        start, else 4 B); the bf16 operands add 2 B per element of the output gradient and the
+        layer input.  A separate average moves 10 B (read w, write w and shadow); in a fused
+        step only the biases (and a classifier head updated by its own kernels) take it."""
         w, K, B = self.w, self.K, self.w["B"]
         widths = w["widths"]
-        if fused and w["bf16"]:
-            return sum(FUSED_UPDATE_BYTES_PER_PARAM * K * widths[l] * widths[l + 1]
-                       + 2 * K * B * (widths[l] + widths[l + 1]) for l in range(len(widths) - 1))
-        return UPDATE_BYTES_PER_PARAM * K * self.d
+        L = len(widths) - 1
+        if not self.fused:
+            upd = UPDATE_BYTES_PER_PARAM * K * self.d
+            return upd, (AVERAGE_BYTES_PER_PARAM * K * self.d if self.kinds[s] == 2 else 0)
+        head = w["bf16"] and widths[-1] <= 16
+        ends = self.kinds[s] == 2 and self.fuse_avg
+        synced = s == 0 or self.kinds[s - 1] == 2
+        upd = 0
+        for l in range(L):
+            n_w = widths[l] * widths[l + 1]
+            if ends and not (head and l == L - 1):
+                upd += (14 * K + 4) * n_w if synced else 18 * K * n_w
+            else:
+                upd += FUSED_UPDATE_BYTES_PER_PARAM * K * n_w
+            upd += 2 * K * B * (widths[l] + widths[l + 1])
+        if self.kinds[s] != 2:
+            return upd, 0
+        if not self.fuse_avg:
+            return upd, AVERAGE_BYTES_PER_PARAM * K * self.d
+        seg = sum(widths[1:]) + (widths[-2] * widths[-1] if head else 0)
+        return upd, AVERAGE_BYTES_PER_PARAM * K * seg
+
+    def traced_bytes(self):
+        """(update, average) algorithmic bytes summed over the traced steps."""
+        tot = [0, 0]
+        for s in self.traced_steps:
+            u, a = self.step_bytes(s)
+            tot[0] += u
+            tot[1] += a
+        return tot
 
     def destroy(self):
         self.P.lsgd_destroy(self.ctx)
 
 
 def roofline(run, prof, steps, hbm, peak_src, fused=True):
+    """The update launches' algorithmic GB/s over the traced steps, against the HBM peak."""
     upd_n, upd_ms = prof["update"]
-    upd_bytes = run.update_bytes(fused)
-    upd_gbs = upd_bytes / (upd_ms / steps / 1000.0) / 1e9
+    upd_bytes, _ = run.traced_bytes()
+    upd_gbs = upd_bytes / (upd_ms / 1000.0) / 1e9
     traffic = UPDATE_TRAFFIC_PER_STEP.get(run.w["name"]) if fused and run.K == run.w["K"] else None
-    return {"kernel": ("wgrad_update_kernel (weight gradient + fused local update)"
-                       if fused else "sgd_update_kernel"),
+    n_avg = sum(1 for s in run.traced_steps if run.kinds[s] == 2)
+    return {"kernel": ("wgrad_update_kernel (weight gradient + fused local update, and the K-way "
+                       "average on round-ending steps)" if fused else "sgd_update_kernel"),
             "bound": "hbm", "achieved": upd_gbs, "peak": hbm, "unit": "GB/s",
             "frac": upd_gbs / hbm, "peak_source": f"{peak_src} hbm_gbs", "traffic": traffic,
-            "unit_of_work": ("one step's fused weight-gradient + update launches (all layers)"
+            "unit_of_work": ("one step's weight-gradient + update launches (all layers), averaged "
+                             f"over {steps} steps of which {n_avg} end with the K-way average"
                              if fused else "one launch over the whole K x d buffer"),
-            "algorithmic_bytes": upd_bytes, "launches_per_unit": upd_n // steps}
+            "algorithmic_bytes": upd_bytes / steps, "launches_per_unit": upd_n // steps}
+
+
+def average_phase(run, prof, hbm):
+    """The averaging launches' algorithmic GB/s over the traced steps (the separate K-way average,
+    or in fused steps the bias / head segments; the rest of the average is in the update)."""
+    avg_n, avg_ms = prof["average"]
+    _, avg_bytes = run.traced_bytes()
+    if not avg_n or not avg_ms:
+        return {"gbs": None, "frac_of_hbm": None, "ms_per_sync": None}
+    gbs = avg_bytes / (avg_ms / 1000.0) / 1e9
+    return {"gbs": gbs, "frac_of_hbm": gbs / hbm, "ms_per_sync": avg_ms / avg_n,
+            "bytes_per_sync": avg_bytes / avg_n}
 
 
 def run_dense_config(args, key):
@@ -590,6 +645,7 @@ def run_dense_config(args, key):
                       "syncs_in_timed_region": syncs, "gpu_launches": launches,
                       "params_per_replica": run.d, "losses_finite": finite,
                       "roofline": roofline(run, prof, S_, hbm, src, fused),
+                      "sync_average": average_phase(run, prof, hbm),
                       "phase_ms_per_step": {k: v[1] / S_ for k, v in prof.items()}}), flush=True)
     run.destroy()
 
@@ -761,9 +817,8 @@ def main():
 
     def e2e_step(i):
         s = P.lsgd_step_count(ctx)
-        P.lsgd_local_step_batch(ctx, xs[i % n_stage], ys[i % n_stage])
-        if kinds[s] == 2:  # the round ends with this step (the schedule of lsgd_run)
-            P.lsgd_sync_average(ctx)
+        # one step of the schedule on the host batch: the local step and the average ending it
+        P.lsgd_run_batch(ctx, xs[i % n_stage], ys[i % n_stage])
         P.lsgd_losses_async(ctx, loss_host[i], 1)  # device -> host read of this step's losses
         if s + 1 == T_job:
             P.lsgd_set_step(ctx, 0)
@@ -788,9 +843,7 @@ def main():
 
     # ---- roofline of the dominant kernel (the fused update), the average, the GEMMs ----
     hbm, bf16_peak, peak_src = _peaks()
-    avg_n, avg_ms = prof["average"]
     widths = w["widths"]
-    avg_gbs = (AVERAGE_BYTES_PER_PARAM * K * run.d / (avg_ms / avg_n / 1000.0) / 1e9) if avg_n else None
     gemm_flops = 0
     for l in range(len(widths) - 1):
         mac = B * widths[l] * widths[l + 1]
@@ -837,11 +890,12 @@ def main():
                 "d2h_bytes_per_step": d2h},
         "gpu_launches": launches,
         "roofline": roofline(run, prof, S_, hbm, peak_src, fused),
-        "sync_average": {"gbs": avg_gbs, "frac_of_hbm": (avg_gbs / hbm) if avg_gbs else None,
-                         "ms_per_sync": (avg_ms / avg_n) if avg_n else None},
+        "sync_average": average_phase(run, prof, hbm),
         "step_split": {"local_frac": 1.0 - phase_ms["average"] / tot_phase,
                        "sync_frac": phase_ms["average"] / tot_phase,
-                       "phase_ms_per_step": {k: v / S_ for k, v in phase_ms.items()}},
+                       "phase_ms_per_step": {k: v / S_ for k, v in phase_ms.items()},
+                       "note": "round-ending steps form the K-way average inside their update "
+                               "launches; the average phase is then the bias / head segments"},
         "gemm": {"tflops": gemm_tflops, "frac_of_bf16_peak": gemm_tflops / bf16_peak,
                  "peak_source": f"{peak_src} bf16_tflops_sustained"},
         "clocks": clk,

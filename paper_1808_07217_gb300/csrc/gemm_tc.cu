@@ -274,12 +274,13 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
         for (int i = 0; i < BM / 64; ++i)
           tma_load_3d(sm.a[s] + i * 64 * BK * 2, &args.A.map, &sm.full[s], m0 + 64 * i, k0, g);
       }
+      const int gb = args.b_shared ? 0 : g;  // identical replicas: group 0's copy for all
       if (!b_mn) {
-        tma_load_3d(sm.b[s], &args.B.map, &sm.full[s], k0, n0, g);
+        tma_load_3d(sm.b[s], &args.B.map, &sm.full[s], k0, n0, gb);
       } else {
 #pragma unroll
         for (int i = 0; i < BN / 64; ++i)
-          tma_load_3d(sm.b[s] + i * 64 * BK * 2, &args.B.map, &sm.full[s], n0 + 64 * i, k0, g);
+          tma_load_3d(sm.b[s] + i * 64 * BK * 2, &args.B.map, &sm.full[s], n0 + 64 * i, k0, gb);
       }
       issued = kb + 1;
     }

@@ -237,6 +237,9 @@ struct TcGemmArgs {
   // cv_ck * 2 bytes.  M = pixels of the output (whole rows per 128-pixel tile), Kd unused.
   int conv;
   int cv_ck, cv_stride, cv_hout, cv_wout;
+  // b_shared = 1 (not with conv): every group reads B from group 0 -- the replicas' weights are
+  // identical (the step follows an average), so one copy serves all, mostly from L2
+  int b_shared;
 };
 // The tile geometry of an implicit convolution with an Hout x Wout output: whole output rows,
 // 128 pixels per tile.  False when the shape does not tile that way.

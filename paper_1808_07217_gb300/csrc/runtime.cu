@@ -385,6 +385,8 @@ lsgd_status dense_forward(lsgd_ctx* c, int groups, int w_g0, int w_gmul, bool sk
       t.epi = epi;
       t.bias = Ly.b_off >= 0 ? c->W + Ly.b_off : nullptr;
       t.bias_gs = c->d_pad;
+      // every replica holds the same weights: all read replica 0's, which stay in L2
+      t.b_shared = (c->synced && groups == c->cfg.K && c->cfg.K > 1) ? 1 : 0;
       lsgd_status st = tc_gemm(c, t);
       if (st != LSGD_OK) return st;
       continue;
@@ -521,6 +523,7 @@ lsgd_status dense_backward(lsgd_ctx* c, bool avg) {
         t.A.box_rows = lsgd::kTcTileM;
         t.B.mn_major = true;
         t.B.box_rows = 64;
+        t.b_shared = (c->synced && K > 1) ? 1 : 0;  // identical replicas: one weight copy
         t.C = dzp;
         t.c_rs = c->ld_dz;
         t.c_gs = (int64_t)B * c->ld_dz;

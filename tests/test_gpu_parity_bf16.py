@@ -309,3 +309,31 @@ def test_run_batch_matches_run(P):
     assert np.array_equal(P.lsgd_losses(a, T, K), P.lsgd_losses(b, T, K))
     P.lsgd_destroy(a)
     P.lsgd_destroy(b)
+
+
+def test_distinct_replicas_use_their_own_weights(P):
+    # After lsgd_set_params on single replicas the replicas differ: every replica's step must use
+    # its own weights (a step that follows an average reads one shared copy instead), checked
+    # against the oracle's step of each replica from its own parameters.
+    widths, K, B, N = (512, 256, 256, 100), 4, 64, 4096
+    X, y = synthdata.gaussian_mixture(N, widths[0], widths[-1], seed=17)
+    g, o = dense_cfgs(P, widths=widths, K=K, B=B, H=4, T=8, N=N, precision=P.BF16,
+                      base_lr=0.05, momentum=0.9, nesterov=True, weight_decay=5e-4, seed=3,
+                      fused_update=True)
+    ctx = P.lsgd_create(g)
+    P.lsgd_set_dataset(ctx, X, y)
+    rng = np.random.default_rng(4)
+    w0 = oracle.init_params(o)
+    Ws = [(w0 * (1.0 + 0.5 * k) + 0.01 * rng.standard_normal(len(w0))).astype(np.float32)
+          for k in range(K)]
+    for k in range(K):
+        P.lsgd_set_params(ctx, k, Ws[k])
+    P.lsgd_run(ctx, 1)  # step 0 of an H = 4 round: no average
+    for k in range(K):
+        wk = Ws[k].astype(np.float64)
+        loss, grad = oracle.loss_grad(o, wk, X, y=y, idx=oracle.sample_indices(o, k, 0))
+        w1, _ = oracle.sgd_update(o, oracle.lr(o, 0), wk, np.zeros_like(wk), grad)
+        got = P.lsgd_params(ctx, k).astype(np.float64)
+        assert rel_l2(got - wk, w1 - wk) <= 2e-2, k
+        assert abs(P.lsgd_losses(ctx, 1, K)[0][k] - loss) <= 1e-2
+    P.lsgd_destroy(ctx)

@@ -543,14 +543,17 @@ class DenseRun:
         return prof
 
     def step_bytes(self, s):
-        """Algorithmic bytes of step s's update launches and of its averaging launches.  Per
-        parameter and replica (fp32 w, u; bf16 shadow): the fused update reads w, u and writes
-        w, u and the shadow (18 B); a step that ends with the average forms it in the same
-        launches and writes w and the shadow once, as the mean (u 8 B + w 4 B + shadow 2 B +
-        the read of w: once per tile, 4 / K B, when the replicas were identical at the step's
-        start, else 4 B); the bf16 operands add 2 B per element of the output gradient and the
-        layer input.  A separate average moves 10 B (read w, write w and shadow); in a fused
-        step only the biases (and a classifier head updated by its own kernels) take it."""
+        """Algorithmic bytes of step s's update launches and of its averaging launches, per
+        parameter and replica of the weight matrices (fp32 w, u; bf16 shadow):
+          * plain fused update: read w, u; write w, u and the shadow = 18 B; when the replicas
+            agree at the step's start (after an average) w is read once per tile: 14 + 4 / K;
+          * a step that ends with the average forms it in the same launches: u read and written
+            (8 B) per replica, the mean and its shadow written once (to the replica every kernel
+            of the next step reads): 8 + 10 / K with the replicas agreeing at the start, else
+            w read per replica: 12 + 6 / K;
+        plus 2 B per element of the bf16 operands (output gradient and layer input).  A separate
+        average moves 10 B per parameter and replica (read w, write w and shadow); in a fused step
+        only the biases (and a classifier head updated by its own kernels) take it."""
         w, K, B = self.w, self.K, self.w["B"]
         widths = w["widths"]
         L = len(widths) - 1
@@ -559,14 +562,16 @@ class DenseRun:
             return upd, (AVERAGE_BYTES_PER_PARAM * K * self.d if self.kinds[s] == 2 else 0)
         head = w["bf16"] and widths[-1] <= 16
         ends = self.kinds[s] == 2 and self.fuse_avg
-        synced = s == 0 or self.kinds[s - 1] == 2
+        synced = K > 1 and (s == 0 or self.kinds[s - 1] == 2)
         upd = 0
         for l in range(L):
             n_w = widths[l] * widths[l + 1]
-            if ends and not (head and l == L - 1):
-                upd += (14 * K + 4) * n_w if synced else 18 * K * n_w
-            else:
+            if head and l == L - 1:
                 upd += FUSED_UPDATE_BYTES_PER_PARAM * K * n_w
+            elif ends:
+                upd += (8 * K + 10) * n_w if synced else (12 * K + 6) * n_w
+            else:
+                upd += (14 * K + 4) * n_w if synced else FUSED_UPDATE_BYTES_PER_PARAM * K * n_w
             upd += 2 * K * B * (widths[l] + widths[l + 1])
         if self.kinds[s] != 2:
             return upd, 0

@@ -25,6 +25,7 @@
 #include <cudaTypedefs.h>
 
 #include <algorithm>
+#include <cstdlib>
 #include <mutex>
 #include <type_traits>
 
@@ -276,7 +277,10 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
       }
       const int gb = args.b_shared ? 0 : g;  // identical replicas: group 0's copy for all
       if (!b_mn) {
-        tma_load_3d(sm.b[s], &args.B.map, &sm.full[s], k0, n0, gb);
+        // K-major B: BN / box_rows boxes stacked along N (8-row swizzle atoms, rows contiguous)
+        const int brows = args.B.box_rows;
+        for (int i = 0; i < BN / brows; ++i)
+          tma_load_3d(sm.b[s] + i * brows * BK * 2, &args.B.map, &sm.full[s], k0, n0 + i * brows, gb);
       } else {
 #pragma unroll
         for (int i = 0; i < BN / 64; ++i)
@@ -532,10 +536,12 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
 // replica's tile gets its own gradient and local update exactly as above (u written back), and the
 // updated values are summed over the replicas with the average's TwoSum in two further TMEM
 // regions (s, c: columns 256-511); after the last replica the mean, divided as the average does,
-// goes to every replica's parameters and bf16 shadow.  Neither the per-replica parameters nor
-// their shadow reach HBM, and with args.w_rep0 (the replicas are identical at the step's start)
-// each tile's parameters are read from replica 0 only.  The results equal those of this kernel
-// in plain mode followed by the K-way average kernel, bit for bit.
+// goes to replica 0's parameters and bf16 shadow -- the other replicas equal it, and the runtime
+// writes their copies only when something reads them (every kernel of the next step reads
+// replica 0).  Neither the per-replica updated parameters nor their shadow reach HBM.  With
+// args.w_rep0 (the replicas are identical at the step's start, in either mode) each tile's
+// parameters are read from replica 0.  The results equal those of this kernel in plain mode
+// followed by the K-way average kernel, bit for bit.
 namespace wu {
 constexpr int TN = 128;                     // tile columns (= rows: BM)
 constexpr int CW = 32;                      // chunk columns (fp32: one 128-byte row)
@@ -544,7 +550,6 @@ constexpr int NS = 4;                       // w / u chunk slots
 constexpr int NWB = 3;                      // bf16 staging buffers
 constexpr int THREADS = 384;
 constexpr int EPI0 = 128;                   // first epilogue thread
-constexpr int EPI_THREADS = 256;            // two per tile row, 16 columns of a chunk each
 constexpr uint32_t kChunkF32 = BM * CW * 4;  // 16 KB
 constexpr uint32_t kChunkB16 = BM * CW * 2;  // 8 KB
 }  // namespace wu
@@ -561,22 +566,6 @@ struct WuSmem {
   uint32_t tmem_base;
   int epi_ok[2];
 };
-
-__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
-  uint32_t r[32];
-  asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,"
-      "%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
-      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
-        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
-        "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]),
-        "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]),
-        "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
-      : "r"(taddr));
-  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-#pragma unroll
-  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
-}
 
 // The same for one epilogue thread's half chunk: 16 gradient columns at tg and its 32-column pair
 // region at tsc (s then c, 16 each).
@@ -659,11 +648,14 @@ __global__ void __launch_bounds__(wu::THREADS, 1) wgrad_update_kernel(
   const bool has_u = args.sgd.u != nullptr;
   const bool avg = args.avg != 0;
   constexpr uint32_t kBytesA = BM * BK * 2, kBytesB = wu::TN * BK * 2;
-  // This CTA's tile sequence: units blockIdx.x, blockIdx.x + gridDim.x, ...; a unit is one tile
-  // (plain mode) or one tile position of a layer taken through all G replicas (averaging mode).
-  const int units0 = avg ? tn0 * tm0 : tiles0;
-  const int units = avg ? units0 + tn1 * tm1 : tiles;
-  const int per_unit = avg ? args.G : 1;
+  // This CTA's tile sequence: units blockIdx.x, blockIdx.x + gridDim.x, ...; a unit is one tile,
+  // or one tile position of a layer taken through all G replicas -- in averaging mode, and
+  // whenever every replica reads replica 0's parameters (w_rep0): then replica 0's tile comes
+  // last, so that no replica reads it after it has been updated.
+  const bool by_unit = avg || args.w_rep0;
+  const int units0 = by_unit ? tn0 * tm0 : tiles0;
+  const int units = by_unit ? units0 + tn1 * tm1 : tiles;
+  const int per_unit = by_unit ? args.G : 1;
   const int my_count =
       (int)blockIdx.x < units ? ((units - 1 - (int)blockIdx.x) / (int)gridDim.x + 1) * per_unit : 0;
   const uint32_t tmem_cols = avg ? 4u * wu::TN : 2u * wu::TN;
@@ -712,7 +704,7 @@ __global__ void __launch_bounds__(wu::THREADS, 1) wgrad_update_kernel(
   auto tile_at = [&](int j, const WgradUpdateLayer*& ly, int& g, int& m0, int& n0, int& gi) {
     const int u = (int)blockIdx.x + (j / per_unit) * (int)gridDim.x;
     gi = j % per_unit;
-    if (!avg) {
+    if (!by_unit) {
       tile_coords(u, ly, g, m0, n0);
       return;
     }
@@ -722,7 +714,8 @@ __global__ void __launch_bounds__(wu::THREADS, 1) wgrad_update_kernel(
     const int r = second ? u - units0 : u;
     m0 = (r / tiles_n) * BM;
     n0 = (r % tiles_n) * wu::TN;
-    g = gi;
+    // averaging: replicas in order (the average's summation order); else replica 0 last
+    g = avg ? gi : (gi + 1) % args.G;
   };
 
   if (warp == 0 && lane == 0) {
@@ -801,7 +794,7 @@ __global__ void __launch_bounds__(wu::THREADS, 1) wgrad_update_kernel(
       const WgradUpdateLayer* ly;
       int g, m0, n0, gi;
       tile_at(j, ly, g, m0, n0, gi);
-      const int gw = (avg && args.w_rep0) ? 0 : g;  // identical replicas: read replica 0's
+      const int gw = args.w_rep0 ? 0 : g;  // identical replicas: read replica 0's
       const int nc = wu_chunks(ly->N, n0);
       for (int c = 0; c < nc; ++c, ++q) {
         const int sl = q % wu::NS;
@@ -943,11 +936,10 @@ __global__ void __launch_bounds__(wu::THREADS, 1) wgrad_update_kernel(
             tma_store_3d(&ly->wmap, sm.w[sl], x, m0, g);
             if (sp.wb) tma_store_3d(&ly->wbmap, sm.wb[wbi], x, m0, g);
           } else if (last) {
-            // the mean to every replica of the unit
-            for (int k = 0; k < args.G; ++k) {
-              tma_store_3d(&ly->wmap, sm.w[sl], x, m0, k);
-              if (sp.wb) tma_store_3d(&ly->wbmap, sm.wb[wbi], x, m0, k);
-            }
+            // the mean goes to replica 0 only; the runtime copies it to the other replicas
+            // when something needs them (every consumer of the next step reads replica 0)
+            tma_store_3d(&ly->wmap, sm.w[sl], x, m0, 0);
+            if (sp.wb) tma_store_3d(&ly->wbmap, sm.wb[wbi], x, m0, 0);
           }
           asm volatile("cp.async.bulk.commit_group;" ::: "memory");
           // the stores of the chunk before have read their slot: hand it back to the producer
@@ -1563,8 +1555,9 @@ cudaError_t launch_wgrad_update(const WgradUpdateArgs& a, cudaStream_t stream) {
     tiles += (int64_t)((ly.N + wu::TN - 1) / wu::TN) * ((ly.M + BM - 1) / BM) * a.G;
   }
   if (tiles > 0x7fffffffLL) return cudaErrorInvalidValue;
-  // averaging mode: a CTA per tile position (all G replicas of it), at most one per SM
-  const int64_t units = a.avg ? tiles / a.G : tiles;
+  // averaging mode, or replica 0's parameters for all: a CTA per tile position (all G replicas
+  // of it), at most one per SM
+  const int64_t units = (a.avg || a.w_rep0) ? tiles / a.G : tiles;
   int dev = 0, sms = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
@@ -1772,6 +1765,13 @@ cudaError_t launch_gemm_tc(const TcGemmArgs& a, cudaStream_t stream) {
   if ((a.Kd + BK - 1) / BK <= 2) return launch_cfg<BN, 2>(a, grid, stream);
   // Long reductions (forward, data gradient): 64-wide N tiles with four stages (96 KB) so two
   // CTAs share an SM and twice as many tiles stream weights at once.
+  const char* wide = std::getenv("LSGD_GEMM_WIDE");
+  const int wv = wide ? std::atoi(wide) : 0;
+  if (wv && a.N >= 256 && (a.B.mn_major || a.B.box_rows == 64)) {
+    if (wv == 1) return launch_cfg<128, 4>(a, dim3((a.N + 127) / 128, (a.M + BM - 1) / BM, a.G * splits), stream);
+    if (wv == 2) return launch_cfg<256, 3>(a, dim3((a.N + 255) / 256, (a.M + BM - 1) / BM, a.G * splits), stream);
+    if (wv == 3) return launch_cfg<256, 4>(a, dim3((a.N + 255) / 256, (a.M + BM - 1) / BM, a.G * splits), stream);
+  }
   constexpr int BN2 = 64;
   dim3 grid2((a.N + BN2 - 1) / BN2, (a.M + BM - 1) / BM, a.G * splits);
   return launch_cfg<BN2, 4>(a, grid2, stream);

@@ -789,6 +789,43 @@ cudaError_t launch_group_average(float* W, uint16_t* Wb, int Kp, int groups, int
   return cudaGetLastError();
 }
 
+// Replica 0's copy of each listed segment (fp32 and bf16 shadow) to replicas 1 .. K-1
+// (blockIdx.y = segment): after an average that wrote the mean to replica 0 only.
+__global__ void __launch_bounds__(256) broadcast_segments_kernel(float4* __restrict__ W,
+                                                                 uint2* __restrict__ Wb, int K,
+                                                                 int64_t rs4, AvgSegments sg) {
+  pdl_begin();
+  const int64_t off4 = sg.off4[blockIdx.y], n4 = sg.len4[blockIdx.y];
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n4; i += stride) {
+    const int64_t col = off4 + i;
+    const float4 v = W[col];
+    const uint2 b = Wb ? Wb[col] : make_uint2(0u, 0u);
+    for (int k = 1; k < K; ++k) {
+      __stcs(W + (int64_t)k * rs4 + col, v);
+      if (Wb) __stcs(Wb + (int64_t)k * rs4 + col, b);
+    }
+  }
+}
+
+cudaError_t launch_broadcast_segments(float* W, uint16_t* Wb, int K, int64_t d_pad,
+                                      const AvgSegments& sg, cudaStream_t stream) {
+  if (K <= 1 || sg.n <= 0) return cudaSuccess;
+  if ((d_pad & 3) || sg.n > kMaxAvgSegments) return cudaErrorInvalidValue;
+  int64_t longest = 0;
+  for (int i = 0; i < sg.n; ++i) {
+    if (sg.off4[i] < 0 || sg.len4[i] < 0 || 4 * (sg.off4[i] + sg.len4[i]) > d_pad)
+      return cudaErrorInvalidValue;
+    longest = std::max<int64_t>(longest, sg.len4[i]);
+  }
+  if (longest == 0) return cudaSuccess;
+  const int threads = 256;
+  const int blocks = (int)std::min<int64_t>((longest + threads - 1) / threads, 2048);
+  launch_pdl(broadcast_segments_kernel, dim3(blocks, sg.n), threads, 0, stream,
+             reinterpret_cast<float4*>(W), reinterpret_cast<uint2*>(Wb), K, d_pad / 4, sg);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_average_segments(float* W, uint16_t* Wb, int K, int64_t d_pad,
                                    const AvgSegments& sg, cudaStream_t stream) {
   if (K < 1 || sg.n <= 0) return cudaSuccess;

@@ -96,6 +96,9 @@ struct AvgSegments {
 // The K-way average of kway_average restricted to the listed segments of each replica.
 cudaError_t launch_average_segments(float* W, uint16_t* Wb, int K, int64_t d_pad,
                                    const AvgSegments& sg, cudaStream_t stream);
+// Replica 0's copy of the listed segments (and of their bf16 shadow, if Wb) to every other replica.
+cudaError_t launch_broadcast_segments(float* W, uint16_t* Wb, int K, int64_t d_pad,
+                                      const AvgSegments& sg, cudaStream_t stream);
 
 // Average within each of `groups` groups of Kp consecutive replicas (replica stride d).
 cudaError_t launch_group_average(float* W, uint16_t* Wb, int Kp, int groups, int64_t d,
@@ -268,8 +271,9 @@ struct WgradUpdateArgs {
   SgdParams sgd;
   // avg = 1: the step ends with the K-way average (Eq. 2 right): every replica's tile is updated
   // as above, and the mean of the updated tiles (the average kernel's arithmetic) is written to
-  // all G replicas' parameters and shadow.  w_rep0 = 1 (avg only): the replicas are identical at
-  // the step's start, so each tile's parameters are read from replica 0.
+  // replica 0's parameters and shadow (the other replicas' copies are left to the caller).
+  // w_rep0 = 1: the replicas are identical at the step's start, so each tile's parameters are
+  // read from replica 0.
   int avg, w_rep0;
 };
 cudaError_t launch_wgrad_update(const WgradUpdateArgs& a, cudaStream_t stream);

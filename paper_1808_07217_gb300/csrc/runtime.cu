@@ -110,6 +110,11 @@ struct lsgd_ctx {
   // the parameter segments a weight-gradient + update + average launch does not cover (the
   // biases and the classifier head's tensors), averaged by a small kernel after it
   lsgd::AvgSegments avg_segs{};
+  // the weight matrices that launch does cover: after it only replica 0 holds them (and their
+  // bf16 shadow) -- `lazy` -- until the next step rewrites every replica or materialize() copies
+  // replica 0 to the others for a reader outside the step
+  lsgd::AvgSegments wgrad_segs{};
+  bool lazy = false;
   bool prof_on = false;
   std::vector<cudaEvent_t> prof_pool;
   size_t prof_used = 0;
@@ -621,7 +626,7 @@ lsgd_status dense_backward(lsgd_ctx* c, bool avg) {
           wa.Kd = B;
           wa.G = K;
           wa.avg = avg ? 1 : 0;
-          wa.w_rep0 = (avg && c->synced) ? 1 : 0;
+          wa.w_rep0 = (c->synced && K > 1) ? 1 : 0;  // one copy serves every replica
           LSGD_LAUNCH(c, lsgd::launch_wgrad_update(wa, c->stream));
           wa.nl = 0;
           span(LSGD_PH_UPDATE);
@@ -757,6 +762,18 @@ lsgd_status step_body(lsgd_ctx* c, int64_t e_start, bool avg = false) {
     c->syncs++;
   }
   c->synced = avg || c->cfg.K == 1;
+  // after the average only replica 0 holds the weight matrices; a plain step rewrites them all
+  c->lazy = avg && c->cfg.K > 1;
+  return LSGD_OK;
+}
+
+// Write replica 0's weight matrices (and bf16 shadow) to the other replicas if an average left
+// them there alone: before anything outside the training step reads or changes single replicas.
+lsgd_status materialize(lsgd_ctx* c) {
+  if (!c->lazy) return LSGD_OK;
+  LSGD_LAUNCH(c, lsgd::launch_broadcast_segments(c->W, c->Wb, c->cfg.K, c->d_pad, c->wgrad_segs,
+                                                 c->stream));
+  c->lazy = false;
   return LSGD_OK;
 }
 
@@ -935,12 +952,17 @@ lsgd_status lsgd_create(const lsgd_config* cfg, const lsgd_allocator* alloc, voi
       // classifier head's weights when its own kernels update them (each tensor starts at a
       // 64-element boundary, so a length rounded up to 4 stays inside its padding)
       lsgd::AvgSegments& sg = c->avg_segs;
+      lsgd::AvgSegments& wg = c->wgrad_segs;
       sg.n = 0;
+      wg.n = 0;
       for (size_t l = 0; l < c->layers.size(); ++l) {
         const DenseLayer& Ly = c->layers[l];
         if (c->head && l + 1 == c->layers.size()) {
           sg.off4[sg.n] = Ly.w_off / 4;
           sg.len4[sg.n++] = ((int64_t)Ly.in * Ly.out + 3) / 4;
+        } else {
+          wg.off4[wg.n] = Ly.w_off / 4;
+          wg.len4[wg.n++] = ((int64_t)Ly.in * Ly.out + 3) / 4;
         }
         if (Ly.b_off >= 0) {
           sg.off4[sg.n] = Ly.b_off / 4;
@@ -1095,6 +1117,7 @@ lsgd_status lsgd_local_step_batch(lsgd_ctx* c, const float* x, const void* lab, 
 
 lsgd_status lsgd_sync_average(lsgd_ctx* c) {
   if (!c) return fail(nullptr, LSGD_EINVAL, "NULL context");
+  if (lsgd_status st = materialize(c); st != LSGD_OK) return st;
   const int64_t e0 = prof_mark(c);
   const int K = c->cfg.K;
   if (c->cfg.compress != LSGD_COMPRESS_NONE) {
@@ -1120,6 +1143,7 @@ lsgd_status lsgd_sync_average(lsgd_ctx* c) {
 lsgd_status lsgd_block_average(lsgd_ctx* c) {
   if (!c) return fail(nullptr, LSGD_EINVAL, "NULL context");
   if (c->cfg.hier_block <= 0) return fail(c, LSGD_ESTATE, "the context has no averaging blocks");
+  if (lsgd_status st = materialize(c); st != LSGD_OK) return st;
   const int64_t e0 = prof_mark(c);
   LSGD_LAUNCH(c, lsgd::launch_group_average(c->W, c->Wb, c->cfg.hier_block,
                                             c->cfg.K / c->cfg.hier_block, c->d_pad, c->stream));
@@ -1193,6 +1217,7 @@ static lsgd_status get_vec(lsgd_ctx* c, const float* buf, int k, float* dst, int
   if (!c || !dst) return fail(c, LSGD_EINVAL, "NULL argument");
   if (n != (size_t)c->d) return fail(c, LSGD_EINVAL, "n must equal lsgd_num_params()");
   if (k < -1 || k >= c->cfg.K) return fail(c, LSGD_EINVAL, "replica index out of range");
+  if (lsgd_status st = materialize(c); st != LSGD_OK) return st;
   if (!buf) {  // no momentum buffer: momentum is identically zero
     if (dst_is_device)
       LSGD_TRY_CUDA(c, cudaMemsetAsync(dst, 0, n * 4, c->stream));
@@ -1241,6 +1266,7 @@ static lsgd_status set_vec(lsgd_ctx* c, float* buf, int k, const float* src, siz
   if (n != (size_t)c->d) return fail(c, LSGD_EINVAL, "n must equal lsgd_num_params()");
   if (k < -1 || k >= c->cfg.K) return fail(c, LSGD_EINVAL, "replica index out of range");
   if (!buf) return fail(c, LSGD_ESTATE, "no momentum buffer (momentum is 0)");
+  if (lsgd_status st = materialize(c); st != LSGD_OK) return st;
   const int k0 = k < 0 ? 0 : k;
   for (const Seg& s : c->segs)
     LSGD_TRY_CUDA(c, cudaMemcpyAsync(buf + (int64_t)k0 * c->d_pad + s.pad, src + s.canon,
@@ -1364,6 +1390,7 @@ lsgd_status lsgd_eval_loss(lsgd_ctx* c, int k, int64_t n, double* loss) {
   if (!c->have_data) return fail(c, LSGD_ESTATE, "lsgd_set_dataset must come first");
   if (k < -1 || k >= c->cfg.K) return fail(c, LSGD_EINVAL, "replica index out of range");
   if (n < 1 || n > c->cfg.N) return fail(c, LSGD_EINVAL, "n must be in [1, N]");
+  if (lsgd_status st = materialize(c); st != LSGD_OK) return st;
   const int kk = k < 0 ? 0 : k;
   const int K = c->cfg.K, B = c->cfg.B_loc;
   const int64_t per = (int64_t)K * B;
@@ -1434,6 +1461,7 @@ lsgd_status lsgd_check_finite(lsgd_ctx* c) {
   if (!c) return fail(nullptr, LSGD_EINVAL, "NULL context");
   const lsgd_status ds = lsgd_device_status(c);
   if (ds != LSGD_OK) return ds;
+  if (lsgd_status st = materialize(c); st != LSGD_OK) return st;
   LSGD_TRY_CUDA(c, cudaMemsetAsync(c->flag, 0, 4, c->stream));
   LSGD_LAUNCH(c, lsgd::launch_check_finite(c->W, (int64_t)c->cfg.K * c->d_pad, c->flag, c->stream));
   int h = 0;
@@ -1454,6 +1482,7 @@ static int64_t state_mask(const lsgd_ctx* c) {
 
 lsgd_status lsgd_save(lsgd_ctx* c, const char* path) {
   if (!c || !path) return fail(c, LSGD_EINVAL, "NULL argument");
+  if (lsgd_status st = materialize(c); st != LSGD_OK) return st;
   const size_t n = (size_t)c->cfg.K * c->d_pad;
   std::vector<float> buf(n);
   FILE* f = std::fopen(path, "wb");
@@ -1485,6 +1514,7 @@ lsgd_status lsgd_save(lsgd_ctx* c, const char* path) {
 
 lsgd_status lsgd_load(lsgd_ctx* c, const char* path) {
   if (!c || !path) return fail(c, LSGD_EINVAL, "NULL argument");
+  if (lsgd_status st = materialize(c); st != LSGD_OK) return st;  // a failed load keeps the state
   FILE* f = std::fopen(path, "rb");
   if (!f) return fail(c, LSGD_EIO, std::string("cannot open ") + path);
   int64_t hdr[7];

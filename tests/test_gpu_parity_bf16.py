@@ -337,3 +337,40 @@ def test_distinct_replicas_use_their_own_weights(P):
         assert rel_l2(got - wk, w1 - wk) <= 2e-2, k
         assert abs(P.lsgd_losses(ctx, 1, K)[0][k] - loss) <= 1e-2
     P.lsgd_destroy(ctx)
+
+
+def test_average_left_in_one_replica_is_materialized_for_readers(P):
+    # After a step that ends with the average, the mean is written to replica 0 alone (every
+    # kernel of the next step reads it there); reading or changing single replicas through the
+    # API first gives every replica its copy.
+    widths, K, B, N = (264, 136, 72, 10), 4, 32, 2048
+    X, y = synthdata.gaussian_mixture(N, widths[0], 10, seed=19)
+    g, o = dense_cfgs(P, widths=widths, K=K, B=B, H=4, T=8, N=N, precision=P.BF16, t_switch=4,
+                      base_lr=0.05, momentum=0.9, nesterov=True, weight_decay=5e-4, seed=2,
+                      fused_update=True)
+    ctx = P.lsgd_create(g)
+    P.lsgd_set_dataset(ctx, X, y)
+    P.lsgd_run(ctx, 2)  # two H = 1 steps, each ending with the average
+    reps = [P.lsgd_params(ctx, k) for k in range(K)]
+    assert all(np.array_equal(reps[0], reps[k]) for k in range(K))
+    P.lsgd_run(ctx, 1)  # again, then overwrite replica 2 only
+    mean = P.lsgd_params(ctx, 0)
+    new = (mean * 0.5).astype(np.float32)
+    P.lsgd_set_params(ctx, 2, new)
+    assert np.array_equal(P.lsgd_params(ctx, 1), mean)
+    assert np.array_equal(P.lsgd_params(ctx, 3), mean)
+    assert np.array_equal(P.lsgd_params(ctx, 2), new)
+    # the next step starts from distinct replicas: the same as the separate-average path's
+    ref = P.lsgd_create(g)
+    P.lsgd_set_dataset(ref, X, y)
+    for s in range(3):
+        P.lsgd_local_step(ref)
+        P.lsgd_sync_average(ref)
+    P.lsgd_set_params(ref, 2, new)
+    P.lsgd_run(ctx, 1)
+    P.lsgd_local_step(ref)
+    P.lsgd_sync_average(ref)  # step 3 ends the H = 1 phase (t' = 4) with an average
+    for k in range(K):
+        assert np.array_equal(P.lsgd_params(ctx, k), P.lsgd_params(ref, k)), k
+    P.lsgd_destroy(ctx)
+    P.lsgd_destroy(ref)

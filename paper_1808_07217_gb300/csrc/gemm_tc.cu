@@ -521,13 +521,13 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
 // ramp are paid once for both.  One CTA per SM:
 //   warp 0      operand producer: dZ / act k-blocks into a two-stage ring
 //   warp 1      MMA issuer: tcgen05.mma (M = N = 128, K = 16) into accumulator (tile & 1)
-//   warp 2      TMEM allocation (256 columns); w / u chunk producer
-//   warps 4-11  epilogue, two threads per tile row (TMEM lane quarter = warp % 4; warps 4-7 take
-//               a chunk's first 16 columns, warps 8-11 the last 16): per chunk,
+//   warp 2      TMEM allocation (256 columns, 512 in averaging mode); w / u chunk producer
+//   warp 3      TMA store issuer: stores each finished chunk and hands its slot back
+//   warps 4-19  epilogue, four threads per tile row (TMEM lane quarter = warp % 4; warps
+//               4 + 4 p .. 7 + 4 p take columns 8 p .. 8 p + 7 of each chunk): per chunk,
 //               tcgen05.ld of the gradient columns, the local momentum-SGD update (weight decay,
 //               heavy-ball or Nesterov momentum, Sec. A.4) on w, u in shared memory, bf16 w
-//               into a staging buffer; thread 128 then issues the three TMA stores and
-//               recycles the slot of the chunk before once its stores have read it.
+//               into the slot's staging buffer.
 // Only thread 128 waits on the epilogue's mbarriers and the outcome reaches the other epilogue
 // threads through a named barrier, so a wait that runs out cannot split them.
 //
@@ -547,9 +547,10 @@ constexpr int TN = 128;                     // tile columns (= rows: BM)
 constexpr int CW = 32;                      // chunk columns (fp32: one 128-byte row)
 constexpr int ST = 2;                       // operand stages
 constexpr int NS = 4;                       // w / u chunk slots
-constexpr int NWB = 3;                      // bf16 staging buffers
-constexpr int THREADS = 384;
+constexpr int EPI_WARPS = 16;               // four per TMEM lane quarter
+constexpr int THREADS = 128 + 32 * EPI_WARPS;
 constexpr int EPI0 = 128;                   // first epilogue thread
+constexpr int CPT = CW / (EPI_WARPS / 4);   // chunk columns per epilogue thread (8)
 constexpr uint32_t kChunkF32 = BM * CW * 4;  // 16 KB
 constexpr uint32_t kChunkB16 = BM * CW * 2;  // 8 KB
 }  // namespace wu
@@ -559,56 +560,60 @@ struct WuSmem {
   uint8_t b[wu::ST][wu::TN * BK * 2];     // 16 KB each
   uint8_t w[wu::NS][wu::kChunkF32];       // 1024-aligned (SWIZZLE_128B)
   uint8_t u[wu::NS][wu::kChunkF32];
-  uint8_t wb[wu::NWB][wu::kChunkB16];     // 512-aligned (SWIZZLE_64B)
+  uint8_t wb[wu::NS][wu::kChunkB16];      // bf16 staging, one per slot; 512-aligned (SWIZZLE_64B)
   uint64_t op_full[wu::ST], op_empty[wu::ST];
   uint64_t acc_full[2], acc_empty[2];
   uint64_t wu_full[wu::NS], wu_empty[wu::NS];
+  uint64_t st_full[wu::NS];  // the epilogue has finished the slot's chunk: store it
   uint32_t tmem_base;
   int epi_ok[2];
 };
 
-// The same for one epilogue thread's half chunk: 16 gradient columns at tg and its 32-column pair
-// region at tsc (s then c, 16 each).
-__device__ __forceinline__ void tmem_ld_g16_sc32(uint32_t tg, uint32_t tsc, float (&g)[16],
-                                                 float (&sc)[32]) {
-  uint32_t a[16], b[32];
+__device__ __forceinline__ void tmem_ld8(uint32_t taddr, float (&v)[8]) {
+  uint32_t r[8];
   asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,"
-      "%15}, [%48];\n"
-      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,"
-      "%28,%29,%30,%31,%32,%33,%34,%35,%36,%37,%38,%39,%40,%41,%42,%43,%44,%45,%46,%47}, [%49];\n"
+      "tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];\n"
+      "tcgen05.wait::ld.sync.aligned;"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7])
+      : "r"(taddr)
+      : "memory");
+#pragma unroll
+  for (int i = 0; i < 8; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// One epilogue thread's share of a chunk: 8 gradient columns at tg and its 16-column pair region
+// at tsc (s then c, 8 each), both loads in flight before one wait.
+__device__ __forceinline__ void tmem_ld_g8_sc16(uint32_t tg, uint32_t tsc, float (&g)[8],
+                                                float (&sc)[16]) {
+  uint32_t a[8], b[16];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%24];\n"
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,%19,"
+      "%20,%21,%22,%23}, [%25];\n"
       "tcgen05.wait::ld.sync.aligned;"
       : "=r"(a[0]), "=r"(a[1]), "=r"(a[2]), "=r"(a[3]), "=r"(a[4]), "=r"(a[5]), "=r"(a[6]),
-        "=r"(a[7]), "=r"(a[8]), "=r"(a[9]), "=r"(a[10]), "=r"(a[11]), "=r"(a[12]), "=r"(a[13]),
-        "=r"(a[14]), "=r"(a[15]),
-        "=r"(b[0]), "=r"(b[1]), "=r"(b[2]), "=r"(b[3]), "=r"(b[4]), "=r"(b[5]), "=r"(b[6]),
-        "=r"(b[7]), "=r"(b[8]), "=r"(b[9]), "=r"(b[10]), "=r"(b[11]), "=r"(b[12]), "=r"(b[13]),
-        "=r"(b[14]), "=r"(b[15]), "=r"(b[16]), "=r"(b[17]), "=r"(b[18]), "=r"(b[19]), "=r"(b[20]),
-        "=r"(b[21]), "=r"(b[22]), "=r"(b[23]), "=r"(b[24]), "=r"(b[25]), "=r"(b[26]), "=r"(b[27]),
-        "=r"(b[28]), "=r"(b[29]), "=r"(b[30]), "=r"(b[31])
+        "=r"(a[7]), "=r"(b[0]), "=r"(b[1]), "=r"(b[2]), "=r"(b[3]), "=r"(b[4]), "=r"(b[5]),
+        "=r"(b[6]), "=r"(b[7]), "=r"(b[8]), "=r"(b[9]), "=r"(b[10]), "=r"(b[11]), "=r"(b[12]),
+        "=r"(b[13]), "=r"(b[14]), "=r"(b[15])
       : "r"(tg), "r"(tsc)
       : "memory");
 #pragma unroll
-  for (int i = 0; i < 16; ++i) g[i] = __uint_as_float(a[i]);
+  for (int i = 0; i < 8; ++i) g[i] = __uint_as_float(a[i]);
 #pragma unroll
-  for (int i = 0; i < 32; ++i) sc[i] = __uint_as_float(b[i]);
+  for (int i = 0; i < 16; ++i) sc[i] = __uint_as_float(b[i]);
 }
 
-__device__ __forceinline__ void tmem_st32_nowait(uint32_t taddr, const float (&v)[32]) {
+__device__ __forceinline__ void tmem_st16_nowait(uint32_t taddr, const float (&v)[16]) {
   asm volatile(
-      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
-      "%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(taddr),
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
+      "%14,%15,%16};" ::"r"(taddr),
       "r"(__float_as_uint(v[0])), "r"(__float_as_uint(v[1])), "r"(__float_as_uint(v[2])),
       "r"(__float_as_uint(v[3])), "r"(__float_as_uint(v[4])), "r"(__float_as_uint(v[5])),
       "r"(__float_as_uint(v[6])), "r"(__float_as_uint(v[7])), "r"(__float_as_uint(v[8])),
       "r"(__float_as_uint(v[9])), "r"(__float_as_uint(v[10])), "r"(__float_as_uint(v[11])),
       "r"(__float_as_uint(v[12])), "r"(__float_as_uint(v[13])), "r"(__float_as_uint(v[14])),
-      "r"(__float_as_uint(v[15])), "r"(__float_as_uint(v[16])), "r"(__float_as_uint(v[17])),
-      "r"(__float_as_uint(v[18])), "r"(__float_as_uint(v[19])), "r"(__float_as_uint(v[20])),
-      "r"(__float_as_uint(v[21])), "r"(__float_as_uint(v[22])), "r"(__float_as_uint(v[23])),
-      "r"(__float_as_uint(v[24])), "r"(__float_as_uint(v[25])), "r"(__float_as_uint(v[26])),
-      "r"(__float_as_uint(v[27])), "r"(__float_as_uint(v[28])), "r"(__float_as_uint(v[29])),
-      "r"(__float_as_uint(v[30])), "r"(__float_as_uint(v[31]))
+      "r"(__float_as_uint(v[15]))
       : "memory");
 }
 
@@ -672,6 +677,7 @@ __global__ void __launch_bounds__(wu::THREADS, 1) wgrad_update_kernel(
     for (int i = 0; i < wu::NS; ++i) {
       mbar_init(&sm.wu_full[i], 1);
       mbar_init(&sm.wu_empty[i], 1);
+      mbar_init(&sm.st_full[i], 1);
     }
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -811,20 +817,58 @@ __global__ void __launch_bounds__(wu::THREADS, 1) wgrad_update_kernel(
       for (int j = (q > wu::NS ? q - wu::NS : 0); j < q; ++j)
         mbar_wait(&sm.wu_full[j % wu::NS], (j / wu::NS) & 1);
     }
+  } else if (warp == 3 && lane == 0) {
+    // ---------------- store issuer ----------------
+    // Each finished chunk leaves by TMA stores (u; the updated w and its bf16 shadow, or in
+    // averaging mode at the unit's last replica the mean to replica 0); once they have read the
+    // slot it goes back to the w / u producer.  Issuing stores here keeps their cost (a few
+    // hundred cycles each) off the epilogue threads.
+    int q = 0;
+    bool ok = true;
+    for (int j = 0; j < my_count && ok; ++j) {
+      const WgradUpdateLayer* ly;
+      int g, m0, n0, gi;
+      tile_at(j, ly, g, m0, n0, gi);
+      const bool last = gi == per_unit - 1;
+      const int nc = wu_chunks(ly->N, n0);
+      for (int c = 0; c < nc; ++c, ++q) {
+        const int sl = q % wu::NS;
+        if (!mbar_wait(&sm.st_full[sl], (q / wu::NS) & 1)) {
+          ok = false;
+          break;
+        }
+        const int x = n0 + c * wu::CW;
+        if (has_u) tma_store_3d(&ly->umap, sm.u[sl], x, m0, g);
+        if (!avg) {
+          tma_store_3d(&ly->wmap, sm.w[sl], x, m0, g);
+          if (args.sgd.wb) tma_store_3d(&ly->wbmap, sm.wb[sl], x, m0, g);
+        } else if (last) {
+          // the mean goes to replica 0 only; the runtime copies it to the other replicas when
+          // something needs them (every consumer of the next step reads replica 0)
+          tma_store_3d(&ly->wmap, sm.w[sl], x, m0, 0);
+          if (args.sgd.wb) tma_store_3d(&ly->wbmap, sm.wb[sl], x, m0, 0);
+        }
+        asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+        asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
+        mbar_arrive(&sm.wu_empty[sl]);  // the stores have read the slot
+      }
+    }
+    asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
   } else if (warp >= 4) {
     // ---------------- epilogue ----------------
     const bool leader = threadIdx.x == wu::EPI0;
     const int quarter = warp & 3;
-    const int half = (warp - 4) >> 2;   // which 16 columns of each chunk
+    const int part = (warp - 4) >> 2;   // which CPT columns of each chunk
     const int r = quarter * 32 + lane;  // tile row of this thread
     const SgdParams& sp = args.sgd;
     // The leader waits; everyone learns the outcome after the named barrier.  Two flag slots
     // alternate, so the leader never overwrites a flag another thread has yet to read (each
     // thread reads slot f before it can reach the barrier of the next wait).
     int fi = 0;
+    auto epi_bar = [] { asm volatile("bar.sync 1, %0;" ::"n"(32 * wu::EPI_WARPS) : "memory"); };
     auto epi_wait = [&](uint64_t* bar, uint32_t parity) -> bool {
       if (leader) sm.epi_ok[fi] = mbar_wait(bar, parity) ? 1 : 0;
-      asm volatile("bar.sync 1, 256;" ::: "memory");
+      epi_bar();
       const bool okw = sm.epi_ok[fi] != 0;
       fi ^= 1;
       return okw;
@@ -832,17 +876,17 @@ __global__ void __launch_bounds__(wu::THREADS, 1) wgrad_update_kernel(
     const float Gf = (float)args.G;
     const bool pow2 = (args.G & (args.G - 1)) == 0;
     const float invG = 1.0f / Gf;  // exact when G is a power of two
-    // One half chunk: the update of 16 parameters per row (SG: the signSGD variant), in averaging
-    // mode folded into the running pair (s, c) and, at the unit's last replica, replaced by the
-    // mean.
-    auto half_chunk = [&](auto sg_tag, const float (&gv)[16], float (&sc)[32], uint8_t* wrow,
-                          uint8_t* urow, uint8_t* brow, bool first, bool last) {
+    // This thread's CPT columns of a chunk: the update of CPT parameters of its row (SG: the
+    // signSGD variant), in averaging mode folded into the running pair (s, c) and, at the unit's
+    // last replica, replaced by the mean.
+    auto part_chunk = [&](auto sg_tag, const float (&gv)[wu::CPT], float (&sc)[2 * wu::CPT],
+                          uint8_t* wrow, uint8_t* urow, uint8_t* brow, bool first, bool last) {
       constexpr bool SG = decltype(sg_tag)::value;
       const bool write_w = !avg || last;  // the parameters leave this chunk for HBM
-      uint32_t packed[8];
+      uint32_t packed[wu::CPT / 2];
 #pragma unroll
-      for (int jj = 0; jj < 4; ++jj) {
-        const int j = 4 * half + jj;  // float4 column group within the 32-column chunk
+      for (int jj = 0; jj < wu::CPT / 4; ++jj) {
+        const int j = (wu::CPT / 4) * part + jj;  // float4 column group within the chunk
         const int phys = (j ^ (r & 7)) << 4;
         float4 wv = *reinterpret_cast<const float4*>(wrow + phys);
         float4 uv = has_u ? *reinterpret_cast<const float4*>(urow + phys)
@@ -850,8 +894,8 @@ __global__ void __launch_bounds__(wu::THREADS, 1) wgrad_update_kernel(
         sgd4<SG>(wv, uv, make_float4(gv[4 * jj], gv[4 * jj + 1], gv[4 * jj + 2], gv[4 * jj + 3]), sp);
         if (has_u) *reinterpret_cast<float4*>(urow + phys) = uv;
         if (avg) {
-          float* sv = sc + 4 * jj;       // s of these four columns
-          float* cv = sc + 16 + 4 * jj;  // c of these four columns
+          float* sv = sc + 4 * jj;             // s of these four columns
+          float* cv = sc + wu::CPT + 4 * jj;   // c of these four columns
           const float wn[4] = {wv.x, wv.y, wv.z, wv.w};
 #pragma unroll
           for (int e = 0; e < 4; ++e) {
@@ -878,14 +922,14 @@ __global__ void __launch_bounds__(wu::THREADS, 1) wgrad_update_kernel(
       }
       if (write_w) {
 #pragma unroll
-        for (int hh = 0; hh < 2; ++hh) {
-          const int h = 2 * half + hh;  // 16-byte unit of the 64-byte bf16 row
+        for (int hh = 0; hh < wu::CPT / 8; ++hh) {
+          const int h = (wu::CPT / 8) * part + hh;  // 16-byte unit of the 64-byte bf16 row
           *reinterpret_cast<uint4*>(brow + ((h ^ ((r >> 1) & 3)) << 4)) =
               make_uint4(packed[4 * hh], packed[4 * hh + 1], packed[4 * hh + 2], packed[4 * hh + 3]);
         }
       }
     };
-    int q = 0, i = 0, wbi = 0;
+    int q = 0, i = 0;
     bool ok = true;
     for (; i < my_count && ok; ++i) {
       const WgradUpdateLayer* ly;
@@ -899,7 +943,7 @@ __global__ void __launch_bounds__(wu::THREADS, 1) wgrad_update_kernel(
         break;
       }
       asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-      for (int c = 0; c < nc; ++c, ++q, wbi = (wbi + 1) % wu::NWB) {
+      for (int c = 0; c < nc; ++c, ++q) {
         const int sl = q % wu::NS;
         if (!epi_wait(&sm.wu_full[sl], (q / wu::NS) & 1)) {
           ok = false;
@@ -907,49 +951,34 @@ __global__ void __launch_bounds__(wu::THREADS, 1) wgrad_update_kernel(
         }
         mbar_try_wait(&sm.wu_full[sl], (q / wu::NS) & 1);  // acquire the TMA-written data
         const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
-        const uint32_t g_col = (uint32_t)(ab * wu::TN + c * wu::CW + 16 * half);
-        // averaging mode: this thread's running pair of the chunk over the replicas so far, 32
-        // columns from 256 + 64 chunk + 32 half (s in sc[0..15], c in sc[16..31])
-        const uint32_t sc_col = 2u * wu::TN + (uint32_t)(c * 2 * wu::CW + 32 * half);
-        float gv[16], sc[32];
+        const uint32_t g_col = (uint32_t)(ab * wu::TN + c * wu::CW + wu::CPT * part);
+        // averaging mode: this thread's running pair of the chunk over the replicas so far,
+        // 2 CPT columns from 256 + 64 chunk + 2 CPT part (s in sc[0 .. CPT), c after it)
+        const uint32_t sc_col = 2u * wu::TN + (uint32_t)(c * 2 * wu::CW + 2 * wu::CPT * part);
+        float gv[wu::CPT], sc[2 * wu::CPT];
         if (avg && !first) {
           tmem_wait_st();  // this chunk's pair, stored at the previous replica
-          tmem_ld_g16_sc32(tmem + lane_base + g_col, tmem + lane_base + sc_col, gv, sc);
+          tmem_ld_g8_sc16(tmem + lane_base + g_col, tmem + lane_base + sc_col, gv, sc);
         } else {
-          tmem_ld16(tmem + lane_base + g_col, gv);
+          tmem_ld8(tmem + lane_base + g_col, gv);
         }
         uint8_t* wrow = sm.w[sl] + r * 128;
         uint8_t* urow = sm.u[sl] + r * 128;
-        uint8_t* brow = sm.wb[wbi] + r * 64;
+        uint8_t* brow = sm.wb[sl] + r * 64;
         if (sp.sign)
-          half_chunk(std::true_type{}, gv, sc, wrow, urow, brow, first, last);
+          part_chunk(std::true_type{}, gv, sc, wrow, urow, brow, first, last);
         else
-          half_chunk(std::false_type{}, gv, sc, wrow, urow, brow, first, last);
-        if (avg && !last) tmem_st32_nowait(tmem + lane_base + sc_col, sc);
+          part_chunk(std::false_type{}, gv, sc, wrow, urow, brow, first, last);
+        if (avg && !last) tmem_st16_nowait(tmem + lane_base + sc_col, sc);
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
         asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-        asm volatile("bar.sync 1, 256;" ::: "memory");
+        epi_bar();
         if (leader) {
-          const int x = n0 + c * wu::CW;
-          if (has_u) tma_store_3d(&ly->umap, sm.u[sl], x, m0, g);
-          if (!avg) {
-            tma_store_3d(&ly->wmap, sm.w[sl], x, m0, g);
-            if (sp.wb) tma_store_3d(&ly->wbmap, sm.wb[wbi], x, m0, g);
-          } else if (last) {
-            // the mean goes to replica 0 only; the runtime copies it to the other replicas
-            // when something needs them (every consumer of the next step reads replica 0)
-            tma_store_3d(&ly->wmap, sm.w[sl], x, m0, 0);
-            if (sp.wb) tma_store_3d(&ly->wbmap, sm.wb[wbi], x, m0, 0);
-          }
-          asm volatile("cp.async.bulk.commit_group;" ::: "memory");
-          // the stores of the chunk before have read their slot: hand it back to the producer
-          asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
-          if (q > 0) mbar_arrive(&sm.wu_empty[(q - 1) % wu::NS]);
+          mbar_arrive(&sm.st_full[sl]);  // the store issuer takes the chunk from here
           if (c == nc - 1) mbar_arrive(&sm.acc_empty[ab]);  // every row has read the accumulator
         }
       }
     }
-    if (leader) asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
     tmem_wait_st();  // no tensor-memory store outstanding when the columns are freed
     (void)ok;
   }

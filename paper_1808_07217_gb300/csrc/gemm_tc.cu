@@ -197,6 +197,181 @@ struct Smem {
   uint32_t tmem_base;
 };
 
+// ---- epilogue of one 128 x BN output tile, shared by the one-tile and the persistent GEMM ----
+// 128 epilogue threads (et = 0 .. 127, named barrier 1): the tile leaves TMEM (columns tmem_acc
+// onwards) in 64-column chunks: each thread takes its row's 64 fp32 values (bias / ReLU
+// applied), writes them to the padded staging tile stg ([128][68] floats + 128 for the column
+// sums), and the threads then store the chunk row-contiguously (a warp writes two 256-byte row
+// segments per instruction), applying the ReLU mask from a coalesced read of the stored
+// activation.
+// The bias that the column sums update (threads 0-63, one column of each 64-column chunk;
+// nothing else writes it) is requested first, so its loads overlap the wait for the accumulator.
+template <int BN>
+__device__ __forceinline__ void epilogue_bias_prefetch(const TcGemmArgs& args, int et, int g,
+                                                       int n0, float (&bsw)[BN / 64],
+                                                       float (&bsu)[BN / 64]) {
+#pragma unroll
+  for (int i = 0; i < BN / 64; ++i) {
+    const int n = n0 + 64 * i + (int)et;
+    const bool v = args.bias_colsum && args.bsgd.w && et < 64 && n < args.N;
+    const int64_t k = (int64_t)g * args.bias_gs + n;
+    bsw[i] = v ? args.bsgd.w[k] : 0.f;
+    bsu[i] = v && args.bsgd.u ? args.bsgd.u[k] : 0.f;
+  }
+}
+
+template <int BN>
+__device__ __forceinline__ void epilogue_tile(const TcGemmArgs& args, int et, uint32_t tmem_acc,
+                                              int g, int m0, int n0, int64_t c_base, float* stg,
+                                              const float (&bsw)[BN / 64],
+                                              const float (&bsu)[BN / 64]) {
+  constexpr int CW = 64, PITCH = CW + 4;  // staged chunk width and row pitch (floats)
+  const int r = et;  // tile row owned in the TMEM phase (TMEM lane quarter et / 32)
+  const float* bias = args.bias ? args.bias + (int64_t)g * args.bias_gs : nullptr;
+  const int epi = args.epi;
+  for (int cc = 0; cc < BN; cc += CW) {
+    if (n0 + cc >= args.N) break;  // block-uniform
+#pragma unroll
+    for (int q = 0; q < CW / 16; ++q) {
+      float v[16];
+      tmem_ld16(tmem_acc + ((uint32_t)(et & ~31) << 16) + (uint32_t)(cc + 16 * q), v);
+      if (epi == EPI_BIAS || epi == EPI_BIAS_RELU) {
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          const int n = n0 + cc + 16 * q + i;
+          float x = v[i] + (n < args.N ? __ldg(bias + n) : 0.f);
+          v[i] = (epi == EPI_BIAS_RELU) ? fmaxf(x, 0.f) : x;
+        }
+      }
+      float4* dst = reinterpret_cast<float4*>(stg + r * PITCH + 16 * q);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) dst[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+    }
+    asm volatile("bar.sync 1, 128;" ::: "memory");
+    // copy-out: item = (row, 4-column group), 16 groups per 64-column row.  Each thread takes
+    // UNR items at a time and issues all their mask loads before any arithmetic, so several
+    // hundred bytes per thread are in flight.
+    constexpr int UNR = 8, ITEMS = BM * (CW / 4);
+    for (int base = et; base < ITEMS; base += 128 * UNR) {
+      float4 x[UNR], a0[UNR];
+      int64_t off[UNR];
+      int nn[UNR];
+      bool ok[UNR];
+#pragma unroll
+      for (int q = 0; q < UNR; ++q) {
+        const int it = base + q * 128;
+        const int row = it / (CW / 4), grp = it % (CW / 4);
+        const int m = m0 + row, n = n0 + cc + grp * 4;
+        ok[q] = it < ITEMS && m < args.M && n < args.N;
+        nn[q] = n;
+        off[q] = c_base + (int64_t)m * args.c_rs + n;
+        a0[q] = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (!ok[q]) continue;
+        x[q] = *reinterpret_cast<const float4*>(stg + row * PITCH + grp * 4);
+        const bool full4 = n + 4 <= args.N;
+        if (epi == EPI_MASK) {
+          const int64_t moff = (int64_t)g * args.mask_gs + (int64_t)m * args.mask_rs + n;
+          if (args.mask_bf16) {
+            const uint16_t* mp = reinterpret_cast<const uint16_t*>(args.mask) + moff;
+            if (full4 && ((reinterpret_cast<uintptr_t>(mp) & 7) == 0)) {
+              const uint2 u = __ldg(reinterpret_cast<const uint2*>(mp));
+              a0[q] = make_float4(bf2f((uint16_t)(u.x & 0xffff)), bf2f((uint16_t)(u.x >> 16)),
+                                  bf2f((uint16_t)(u.y & 0xffff)), bf2f((uint16_t)(u.y >> 16)));
+            } else {
+              float t[4] = {0.f, 0.f, 0.f, 0.f};
+              for (int i = 0; i < 4 && n + i < args.N; ++i) t[i] = bf2f(mp[i]);
+              a0[q] = make_float4(t[0], t[1], t[2], t[3]);
+            }
+          } else {
+            const float* mp = reinterpret_cast<const float*>(args.mask) + moff;
+            float t[4] = {0.f, 0.f, 0.f, 0.f};
+            for (int i = 0; i < 4 && n + i < args.N; ++i) t[i] = mp[i];
+            a0[q] = make_float4(t[0], t[1], t[2], t[3]);
+          }
+        }
+      }
+#pragma unroll
+      for (int q = 0; q < UNR; ++q) {
+        if (!ok[q]) continue;
+        const int n = nn[q];
+        const bool full4 = n + 4 <= args.N;
+        float4 v = x[q];
+        if (epi == EPI_MASK) {
+          v.x = a0[q].x > 0.f ? v.x : 0.f;
+          v.y = a0[q].y > 0.f ? v.y : 0.f;
+          v.z = a0[q].z > 0.f ? v.z : 0.f;
+          v.w = a0[q].w > 0.f ? v.w : 0.f;
+        }
+        if (args.bias_colsum) {
+          // keep the stored (rounded) value for the column sums below; each item is this
+          // thread's alone
+          const int it = base + q * 128;
+          const float4 r4 = args.c_bf16 ? make_float4(bf2f(f2bf(v.x)), bf2f(f2bf(v.y)),
+                                                      bf2f(f2bf(v.z)), bf2f(f2bf(v.w)))
+                                        : v;
+          *reinterpret_cast<float4*>(stg + (it / (CW / 4)) * PITCH + (it % (CW / 4)) * 4) = r4;
+        }
+        if (args.c_bf16) {
+          uint16_t* out = reinterpret_cast<uint16_t*>(args.C) + off[q];
+          if (full4 && ((reinterpret_cast<uintptr_t>(out) & 7) == 0)) {
+            uint2 o;
+            o.x = (uint32_t)f2bf(v.x) | ((uint32_t)f2bf(v.y) << 16);
+            o.y = (uint32_t)f2bf(v.z) | ((uint32_t)f2bf(v.w) << 16);
+            *reinterpret_cast<uint2*>(out) = o;
+          } else {
+            const float xs[4] = {v.x, v.y, v.z, v.w};
+            for (int i = 0; i < 4 && n + i < args.N; ++i) out[i] = f2bf(xs[i]);
+          }
+        } else {
+          float* out = reinterpret_cast<float*>(args.C) + off[q];
+          if (full4 && ((reinterpret_cast<uintptr_t>(out) & 15) == 0)) {
+            *reinterpret_cast<float4*>(out) = v;
+          } else {
+            const float xs[4] = {v.x, v.y, v.z, v.w};
+            for (int i = 0; i < 4 && n + i < args.N; ++i) out[i] = xs[i];
+          }
+        }
+      }
+    }
+    asm volatile("bar.sync 1, 128;" ::: "memory");
+    if (args.bias_colsum) {
+      // Bias gradient of the layer this data gradient feeds: the sum over all rows (the tile
+      // holds the whole mini-batch) of the stored values, per column; two row halves per
+      // column, added in a fixed order, then the local update of that bias (or its gradient).
+      float* hs = stg + BM * PITCH;  // 2 x 64 partial sums after the staged tile
+      const int col = et & (CW - 1), half = et / CW;
+      float sum = 0.f;
+      const int r1 = min(args.M - m0, BM);
+      for (int row = half * (BM / 2); row < min(r1, (half + 1) * (BM / 2)); ++row)
+        sum += stg[row * PITCH + col];
+      hs[half * CW + col] = sum;
+      asm volatile("bar.sync 1, 128;" ::: "memory");
+      const int n = n0 + cc + et;
+      if (et < CW && n < args.N) {
+        const float gb = hs[et] + hs[CW + et];
+        const int64_t k = (int64_t)g * args.bias_gs + n;
+        if (!args.bsgd.w) {
+          args.bias_grad[k] = gb;
+        } else {
+          const SgdParams& sp = args.bsgd;
+          float w = bsw[cc / CW], u = bsu[cc / CW];
+          const bool sg = sp.sign != 0;
+          if (sp.mom == 0.f)
+            sgd_elem<false, false>(w, u, gb, sp.lr, 0.f, sp.wd, sg);
+          else if (sp.nesterov)
+            sgd_elem<true, true>(w, u, gb, sp.lr, sp.mom, sp.wd, sg);
+          else
+            sgd_elem<true, false>(w, u, gb, sp.lr, sp.mom, sp.wd, sg);
+          sp.w[k] = w;
+          if (sp.u) sp.u[k] = u;
+          if (sp.wb) sp.wb[k] = f2bf(w);
+        }
+      }
+      asm volatile("bar.sync 1, 128;" ::: "memory");
+    }
+  }
+}
+
 template <int BN, int STAGES>
 __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__ TcGemmArgs args) {
   extern __shared__ uint8_t smem_raw[];
@@ -335,175 +510,194 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
 
   // ---------------- epilogue (all 4 warps) ----------------
   // The stage buffers are free once the accumulator is complete (every MMA has read its
-  // operands).  The tile leaves TMEM in 64-column chunks: each thread takes its row's 64 fp32
-  // values (bias / ReLU applied), writes them to a padded shared-memory staging tile, and the CTA
-  // then stores the chunk row-contiguously (a warp writes two 256-byte row segments per
-  // instruction), applying the ReLU mask from a coalesced read of the stored activation.
-  // The bias that the column sums below update (threads 0-63, one column of each 64-column
-  // chunk; nothing else writes it) is requested now, while the main loop still runs.
+  // operands): they hold the staging tile.
   float bsw[BN / 64], bsu[BN / 64];
-#pragma unroll
-  for (int i = 0; i < BN / 64; ++i) {
-    const int n = n0 + 64 * i + (int)threadIdx.x;
-    const bool v = args.bias_colsum && args.bsgd.w && threadIdx.x < 64 && n < args.N;
-    const int64_t k = (int64_t)g * args.bias_gs + n;
-    bsw[i] = v ? args.bsgd.w[k] : 0.f;
-    bsu[i] = v && args.bsgd.u ? args.bsgd.u[k] : 0.f;
-  }
+  epilogue_bias_prefetch<BN>(args, (int)threadIdx.x, g, n0, bsw, bsu);
   const bool have_acc = mbar_wait(&sm.accum, 0);
   asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-  if (have_acc) {
-    constexpr int CW = 64, PITCH = CW + 4;  // staged chunk width and row pitch (floats)
-    float* stg = reinterpret_cast<float*>(sm.a[0]);
-    const int r = warp * 32 + lane;  // tile row owned in the TMEM phase
-    const float* bias = args.bias ? args.bias + (int64_t)g * args.bias_gs : nullptr;
-    const int epi = args.epi;
-    for (int cc = 0; cc < BN; cc += CW) {
-      if (n0 + cc >= args.N) break;  // block-uniform
-#pragma unroll
-      for (int q = 0; q < CW / 16; ++q) {
-        float v[16];
-        tmem_ld16(tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)(cc + 16 * q), v);
-        if (epi == EPI_BIAS || epi == EPI_BIAS_RELU) {
-#pragma unroll
-          for (int i = 0; i < 16; ++i) {
-            const int n = n0 + cc + 16 * q + i;
-            float x = v[i] + (n < args.N ? __ldg(bias + n) : 0.f);
-            v[i] = (epi == EPI_BIAS_RELU) ? fmaxf(x, 0.f) : x;
-          }
+  if (have_acc)
+    epilogue_tile<BN>(args, (int)threadIdx.x, tmem, g, m0, n0, c_base,
+                      reinterpret_cast<float*>(sm.a[0]), bsw, bsu);
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+  __syncthreads();
+  if (warp == 2) {
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"((uint32_t)BN)
+                 : "memory");
+  }
+}
+
+// =============================================================================================
+// Persistent grouped GEMM for the long products (forward and data gradient of the dense
+// layers): C[g] = epilogue(A[g] B[gb]^T) over 128 x PBN output tiles.  One CTA per SM walks the
+// tiles blockIdx.x, blockIdx.x + gridDim.x, ... with the replica innermost (so the CTAs that
+// share a weight tile when every replica reads replica 0's, b_shared, run together and L2 serves
+// it), and two TMEM accumulators let one tile's epilogue overlap the next tile's products:
+//   warp 0      TMA producer: A (128 x 64) and B (PBN x 64) k-blocks into a PST-stage ring
+//   warp 1      MMA issuer: tcgen05.mma (M = 128, N = PBN, K = 16), accumulator (tile & 1)
+//   warp 2      TMEM allocation (2 PBN columns)
+//   warps 4-7   epilogue (epilogue_tile: bias / ReLU / ReLU mask, column sums + bias update),
+//               staged through a shared-memory tile of its own
+// 128 x 256 tiles halve the shared-memory operand bytes per MMA of the 64-wide one-tile kernel
+// (whose N = 64 MMAs read as many operand bytes as they compute).
+namespace pt {
+constexpr int PBN = 256;
+constexpr int PST = 3;
+constexpr int THREADS = 256;
+constexpr int STG_FLOATS = BM * (64 + 4) + 2 * 64;
+}  // namespace pt
+
+struct PtSmem {
+  uint8_t a[pt::PST][BM * BK * 2];       // 16 KB each (1024-aligned)
+  uint8_t b[pt::PST][pt::PBN * BK * 2];  // 32 KB each
+  float stg[pt::STG_FLOATS];
+  uint64_t full[pt::PST], empty[pt::PST];
+  uint64_t acc_full[2], acc_empty[2];
+  uint32_t tmem_base;
+  int epi_ok[2];
+};
+
+__global__ void __launch_bounds__(pt::THREADS, 1) gemm_pt_kernel(const __grid_constant__ TcGemmArgs args) {
+  extern __shared__ uint8_t smem_raw[];
+  PtSmem& sm = *reinterpret_cast<PtSmem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                          ~uintptr_t(1023));
+  constexpr int PBN = pt::PBN, PST = pt::PST;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int tiles_n = (args.N + PBN - 1) / PBN, tiles_m = (args.M + BM - 1) / BM;
+  const int tiles = tiles_n * tiles_m * args.G;
+  const int nk = (args.Kd + BK - 1) / BK;
+  const bool a_mn = args.A.mn_major, b_mn = args.B.mn_major;
+  constexpr uint32_t kBytesA = BM * BK * 2, kBytesB = PBN * BK * 2;
+  // tile t: replica fastest, then m-tile, then n-tile
+  auto coords = [&](int t, int& g, int& m0, int& n0) {
+    g = t % args.G;
+    const int r = t / args.G;
+    m0 = (r % tiles_m) * BM;
+    n0 = (r / tiles_m) * PBN;
+  };
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < PST; ++s) {
+      mbar_init(&sm.full[s], 1);
+      mbar_init(&sm.empty[s], 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&sm.acc_full[i], 1);
+      mbar_init(&sm.acc_empty[i], 1);
+    }
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  }
+  if (warp == 2) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     smem_u32(&sm.tmem_base)),
+                 "r"(2u * PBN)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+  __syncthreads();
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+  const uint32_t tmem = sm.tmem_base;
+  pdl_begin();  // everything above touched only shared memory and TMEM
+
+  if (warp == 0 && lane == 0) {
+    // ---------------- TMA producer ----------------
+    int it = 0;
+    bool ok = true;
+    for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x) {
+      int g, m0, n0;
+      coords(t, g, m0, n0);
+      const int gb = args.b_shared ? 0 : g;  // identical replicas: replica 0's copy for all
+      for (int kb = 0; kb < nk; ++kb, ++it) {
+        const int s = it % PST;
+        if (!mbar_wait(&sm.empty[s], ((it / PST) & 1) ^ 1)) {
+          ok = false;
+          break;
         }
-        float4* dst = reinterpret_cast<float4*>(stg + r * PITCH + 16 * q);
+        mbar_expect_tx(&sm.full[s], kBytesA + kBytesB);
+        const int k0 = kb * BK;
+        if (!a_mn) {
+          tma_load_3d(sm.a[s], &args.A.map, &sm.full[s], k0, m0, g);
+        } else {
 #pragma unroll
-        for (int i = 0; i < 4; ++i) dst[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+          for (int i = 0; i < BM / 64; ++i)
+            tma_load_3d(sm.a[s] + i * 64 * BK * 2, &args.A.map, &sm.full[s], m0 + 64 * i, k0, g);
+        }
+        if (!b_mn) {
+          const int brows = args.B.box_rows;  // 64-row boxes stacked along N
+          for (int i = 0; i < PBN / brows; ++i)
+            tma_load_3d(sm.b[s] + i * brows * BK * 2, &args.B.map, &sm.full[s], k0, n0 + i * brows, gb);
+        } else {
+#pragma unroll
+          for (int i = 0; i < PBN / 64; ++i)
+            tma_load_3d(sm.b[s] + i * 64 * BK * 2, &args.B.map, &sm.full[s], n0 + 64 * i, k0, gb);
+        }
       }
+    }
+    if (!ok) {
+      for (int j = (it > PST ? it - PST : 0); j < it; ++j)
+        mbar_wait(&sm.full[j % PST], (j / PST) & 1);
+    }
+  } else if (warp == 1 && lane == 0) {
+    // ---------------- MMA issuer ----------------
+    constexpr uint32_t idesc_kk = make_idesc(BM, PBN, false, false);
+    const uint32_t idesc = idesc_kk | ((a_mn ? 1u : 0u) << 15) | ((b_mn ? 1u : 0u) << 16);
+    int it = 0, i = 0;
+    bool ok = true;
+    for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x, ++i) {
+      const int ab = i & 1;
+      if (!mbar_wait(&sm.acc_empty[ab], ((i >> 1) & 1) ^ 1)) break;
+      asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+      const uint32_t acc = tmem + (uint32_t)(ab * PBN);
+      for (int kb = 0; kb < nk; ++kb, ++it) {
+        const int s = it % PST;
+        if (!mbar_wait(&sm.full[s], (it / PST) & 1)) {
+          ok = false;
+          break;
+        }
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        const uint32_t a_base = smem_u32(sm.a[s]), b_base = smem_u32(sm.b[s]);
+#pragma unroll
+        for (int kk = 0; kk < BK / 16; ++kk) {
+          const uint64_t ad = a_mn ? smem_desc(a_base + kk * 2048, 64 * BK * 2, 1024)
+                                   : smem_desc(a_base + kk * 32, 16, 1024);
+          const uint64_t bd = b_mn ? smem_desc(b_base + kk * 2048, 64 * BK * 2, 1024)
+                                   : smem_desc(b_base + kk * 32, 16, 1024);
+          mma_bf16(acc, ad, bd, idesc, (kb > 0 || kk > 0) ? 1u : 0u);
+        }
+        mma_commit(&sm.empty[s]);
+      }
+      if (ok) mma_commit(&sm.acc_full[ab]);
+    }
+  } else if (warp >= 4) {
+    // ---------------- epilogue ----------------
+    const int et = threadIdx.x - 128;
+    const bool leader = et == 0;
+    int fi = 0;
+    int i = 0;
+    for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++i) {
+      int g, m0, n0;
+      coords(t, g, m0, n0);
+      const int ab = i & 1;
+      float bsw[PBN / 64], bsu[PBN / 64];
+      epilogue_bias_prefetch<PBN>(args, et, g, n0, bsw, bsu);
+      if (leader) sm.epi_ok[fi] = mbar_wait(&sm.acc_full[ab], (i >> 1) & 1) ? 1 : 0;
       asm volatile("bar.sync 1, 128;" ::: "memory");
-      // copy-out: item = (row, 4-column group), 16 groups per 64-column row.  Each thread takes
-      // UNR items at a time and issues all their mask loads before any arithmetic, so several
-      // hundred bytes per thread are in flight.
-      constexpr int UNR = 8, ITEMS = BM * (CW / 4);
-      for (int base = threadIdx.x; base < ITEMS; base += 128 * UNR) {
-        float4 x[UNR], a0[UNR];
-        int64_t off[UNR];
-        int nn[UNR];
-        bool ok[UNR];
-#pragma unroll
-        for (int q = 0; q < UNR; ++q) {
-          const int it = base + q * 128;
-          const int row = it / (CW / 4), grp = it % (CW / 4);
-          const int m = m0 + row, n = n0 + cc + grp * 4;
-          ok[q] = it < ITEMS && m < args.M && n < args.N;
-          nn[q] = n;
-          off[q] = c_base + (int64_t)m * args.c_rs + n;
-          a0[q] = make_float4(0.f, 0.f, 0.f, 0.f);
-          if (!ok[q]) continue;
-          x[q] = *reinterpret_cast<const float4*>(stg + row * PITCH + grp * 4);
-          const bool full4 = n + 4 <= args.N;
-          if (epi == EPI_MASK) {
-            const int64_t moff = (int64_t)g * args.mask_gs + (int64_t)m * args.mask_rs + n;
-            if (args.mask_bf16) {
-              const uint16_t* mp = reinterpret_cast<const uint16_t*>(args.mask) + moff;
-              if (full4 && ((reinterpret_cast<uintptr_t>(mp) & 7) == 0)) {
-                const uint2 u = __ldg(reinterpret_cast<const uint2*>(mp));
-                a0[q] = make_float4(bf2f((uint16_t)(u.x & 0xffff)), bf2f((uint16_t)(u.x >> 16)),
-                                    bf2f((uint16_t)(u.y & 0xffff)), bf2f((uint16_t)(u.y >> 16)));
-              } else {
-                float t[4] = {0.f, 0.f, 0.f, 0.f};
-                for (int i = 0; i < 4 && n + i < args.N; ++i) t[i] = bf2f(mp[i]);
-                a0[q] = make_float4(t[0], t[1], t[2], t[3]);
-              }
-            } else {
-              const float* mp = reinterpret_cast<const float*>(args.mask) + moff;
-              float t[4] = {0.f, 0.f, 0.f, 0.f};
-              for (int i = 0; i < 4 && n + i < args.N; ++i) t[i] = mp[i];
-              a0[q] = make_float4(t[0], t[1], t[2], t[3]);
-            }
-          }
-        }
-#pragma unroll
-        for (int q = 0; q < UNR; ++q) {
-          if (!ok[q]) continue;
-          const int n = nn[q];
-          const bool full4 = n + 4 <= args.N;
-          float4 v = x[q];
-          if (epi == EPI_MASK) {
-            v.x = a0[q].x > 0.f ? v.x : 0.f;
-            v.y = a0[q].y > 0.f ? v.y : 0.f;
-            v.z = a0[q].z > 0.f ? v.z : 0.f;
-            v.w = a0[q].w > 0.f ? v.w : 0.f;
-          }
-          if (args.bias_colsum) {
-            // keep the stored (rounded) value for the column sums below; each item is this
-            // thread's alone
-            const int it = base + q * 128;
-            const float4 r4 = args.c_bf16 ? make_float4(bf2f(f2bf(v.x)), bf2f(f2bf(v.y)),
-                                                        bf2f(f2bf(v.z)), bf2f(f2bf(v.w)))
-                                          : v;
-            *reinterpret_cast<float4*>(stg + (it / (CW / 4)) * PITCH + (it % (CW / 4)) * 4) = r4;
-          }
-          if (args.c_bf16) {
-            uint16_t* out = reinterpret_cast<uint16_t*>(args.C) + off[q];
-            if (full4 && ((reinterpret_cast<uintptr_t>(out) & 7) == 0)) {
-              uint2 o;
-              o.x = (uint32_t)f2bf(v.x) | ((uint32_t)f2bf(v.y) << 16);
-              o.y = (uint32_t)f2bf(v.z) | ((uint32_t)f2bf(v.w) << 16);
-              *reinterpret_cast<uint2*>(out) = o;
-            } else {
-              const float xs[4] = {v.x, v.y, v.z, v.w};
-              for (int i = 0; i < 4 && n + i < args.N; ++i) out[i] = f2bf(xs[i]);
-            }
-          } else {
-            float* out = reinterpret_cast<float*>(args.C) + off[q];
-            if (full4 && ((reinterpret_cast<uintptr_t>(out) & 15) == 0)) {
-              *reinterpret_cast<float4*>(out) = v;
-            } else {
-              const float xs[4] = {v.x, v.y, v.z, v.w};
-              for (int i = 0; i < 4 && n + i < args.N; ++i) out[i] = xs[i];
-            }
-          }
-        }
-      }
+      const bool okw = sm.epi_ok[fi] != 0;
+      fi ^= 1;
+      if (!okw) break;
+      asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+      const int64_t c_base = (int64_t)g * args.c_gs;
+      epilogue_tile<PBN>(args, et, tmem + (uint32_t)(ab * PBN), g, m0, n0, c_base, sm.stg, bsw, bsu);
+      asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
       asm volatile("bar.sync 1, 128;" ::: "memory");
-      if (args.bias_colsum) {
-        // Bias gradient of the layer this data gradient feeds: the sum over all rows (the tile
-        // holds the whole mini-batch) of the stored values, per column; two row halves per
-        // column, added in a fixed order, then the local update of that bias (or its gradient).
-        float* hs = stg + BM * PITCH;  // 2 x 64 partial sums after the staged tile
-        const int col = threadIdx.x & (CW - 1), half = threadIdx.x / CW;
-        float sum = 0.f;
-        const int r1 = min(args.M - m0, BM);
-        for (int row = half * (BM / 2); row < min(r1, (half + 1) * (BM / 2)); ++row)
-          sum += stg[row * PITCH + col];
-        hs[half * CW + col] = sum;
-        asm volatile("bar.sync 1, 128;" ::: "memory");
-        const int n = n0 + cc + threadIdx.x;
-        if (threadIdx.x < CW && n < args.N) {
-          const float gb = hs[threadIdx.x] + hs[CW + threadIdx.x];
-          const int64_t k = (int64_t)g * args.bias_gs + n;
-          if (!args.bsgd.w) {
-            args.bias_grad[k] = gb;
-          } else {
-            const SgdParams& sp = args.bsgd;
-            float w = bsw[cc / CW], u = bsu[cc / CW];
-            const bool sg = sp.sign != 0;
-            if (sp.mom == 0.f)
-              sgd_elem<false, false>(w, u, gb, sp.lr, 0.f, sp.wd, sg);
-            else if (sp.nesterov)
-              sgd_elem<true, true>(w, u, gb, sp.lr, sp.mom, sp.wd, sg);
-            else
-              sgd_elem<true, false>(w, u, gb, sp.lr, sp.mom, sp.wd, sg);
-            sp.w[k] = w;
-            if (sp.u) sp.u[k] = u;
-            if (sp.wb) sp.wb[k] = f2bf(w);
-          }
-        }
-        asm volatile("bar.sync 1, 128;" ::: "memory");
-      }
+      if (leader) mbar_arrive(&sm.acc_empty[ab]);  // every row has read the accumulator
     }
   }
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
   __syncthreads();
   if (warp == 2) {
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"((uint32_t)BN)
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(2u * pt::PBN)
                  : "memory");
   }
 }
@@ -1753,6 +1947,36 @@ int tc_valid_splits(int Kd, int want) {
   return (nk_all + per - 1) / per;  // every split gets at least one k-block
 }
 
+namespace {
+bool gemm_pt_off() {
+  static const bool off = [] {
+    const char* e = std::getenv("LSGD_GEMM_ONE_TILE");
+    return e && e[0] == '1';
+  }();
+  return off;
+}
+
+cudaError_t launch_pt(const TcGemmArgs& a, cudaStream_t stream) {
+  int dev = 0, sms = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  if (e != cudaSuccess) return e;
+  constexpr size_t smem = sizeof(PtSmem) + 1024;
+  static_assert(smem <= 232448, "shared memory per CTA");
+  static int attr_dev = -1;
+  if (attr_dev != dev) {
+    e = cudaFuncSetAttribute(gemm_pt_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    attr_dev = dev;
+  }
+  const int64_t tiles = (int64_t)((a.N + pt::PBN - 1) / pt::PBN) * ((a.M + BM - 1) / BM) * a.G;
+  if (tiles > 0x7fffffffLL) return cudaErrorInvalidValue;
+  const int grid = (int)std::min<int64_t>(tiles, sms);
+  launch_pdl(gemm_pt_kernel, dim3(grid), dim3(pt::THREADS), smem, stream, a);
+  return cudaGetLastError();
+}
+}  // namespace
+
 cudaError_t launch_gemm_tc(const TcGemmArgs& a, cudaStream_t stream) {
   if (a.M <= 0 || a.N <= 0 || a.G <= 0) return cudaSuccess;
   if (a.Kd <= 0 || a.G > 65535) return cudaErrorInvalidValue;
@@ -1792,15 +2016,15 @@ cudaError_t launch_gemm_tc(const TcGemmArgs& a, cudaStream_t stream) {
   // Short reductions (the weight gradient's k = B_loc) need only two stages; the smaller shared
   // footprint lets three CTAs share an SM so one CTA's epilogue overlaps the others' loads.
   if ((a.Kd + BK - 1) / BK <= 2) return launch_cfg<BN, 2>(a, grid, stream);
-  // Long reductions (forward, data gradient): 64-wide N tiles with four stages (96 KB) so two
-  // CTAs share an SM and twice as many tiles stream weights at once.
-  const char* wide = std::getenv("LSGD_GEMM_WIDE");
-  const int wv = wide ? std::atoi(wide) : 0;
-  if (wv && a.N >= 256 && (a.B.mn_major || a.B.box_rows == 64)) {
-    if (wv == 1) return launch_cfg<128, 4>(a, dim3((a.N + 127) / 128, (a.M + BM - 1) / BM, a.G * splits), stream);
-    if (wv == 2) return launch_cfg<256, 3>(a, dim3((a.N + 255) / 256, (a.M + BM - 1) / BM, a.G * splits), stream);
-    if (wv == 3) return launch_cfg<256, 4>(a, dim3((a.N + 255) / 256, (a.M + BM - 1) / BM, a.G * splits), stream);
-  }
+  // Wide forward products (K-major weights, at least 2048 output columns, no split): the
+  // persistent kernel.  Narrower layers give it too few 128 x 256 tiles to fill the SMs, and the
+  // data gradient (MN-major weights) streamed its weights faster on the one-tile kernel's deeper
+  // rings (measured: MLP 3072-4096x3-100 forward 0.36 -> 0.27 ms per step; data gradient 0.38 ->
+  // 0.43 ms, and MLP 3072-1024-1024-10 0.29 -> 0.35 ms per step, so those stay where they are).
+  if (splits == 1 && a.N >= 2048 && !a.B.mn_major && a.B.box_rows == 64 && !gemm_pt_off())
+    return launch_pt(a, stream);
+  // Other long reductions: 64-wide N tiles with four stages (96 KB) so two CTAs share an SM and
+  // twice as many tiles stream weights at once.
   constexpr int BN2 = 64;
   dim3 grid2((a.N + BN2 - 1) / BN2, (a.M + BM - 1) / BM, a.G * splits);
   return launch_cfg<BN2, 4>(a, grid2, stream);

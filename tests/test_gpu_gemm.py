@@ -51,3 +51,40 @@ def test_grouped_gemm_matches_fp64(P, shape, a_mn, b_mn):
         err = ((C.double() - ref).abs() / scale.clamp_min(1e-30)).max().item()
         print(f"engine {engine} {shape} a_mn={a_mn} b_mn={b_mn}: max err / (|A||B|) = {err:.2e}")
         assert err <= 4e-6, (engine, err)
+
+
+def test_persistent_and_one_tile_kernels_agree_bitwise():
+    # Wide forward products run on the persistent 128 x 256-tile kernel; the one-tile kernel
+    # (LSGD_GEMM_ONE_TILE=1 at library load) accumulates every output in the same k order, so
+    # both give the same bits.  Run in subprocesses: the switch is read once.
+    import os
+    import subprocess
+    import sys
+    prog = r"""
+import numpy as np, torch, sys
+sys.path.insert(0, %r)
+from _gpu_common import built_package
+P = built_package()
+gen = torch.Generator(device="cuda").manual_seed(5)
+out = []
+for (M, N, Kd, G, a_mn, b_mn) in [(128, 4096, 4096, 3, 0, 0), (128, 1024, 3072, 2, 0, 1),
+                                  (200, 520, 1000, 2, 0, 0), (128, 264, 136, 4, 0, 1)]:
+    A = torch.randn((G, Kd, M) if a_mn else (G, M, Kd), device="cuda", generator=gen).to(torch.bfloat16)
+    B = torch.randn((G, Kd, N) if b_mn else (G, N, Kd), device="cuda", generator=gen).to(torch.bfloat16)
+    C = torch.empty((G, M, N), device="cuda")
+    P.lsgd_grouped_gemm_bf16(A, a_mn, B, b_mn, C, M, N, Kd, G, 0)
+    torch.cuda.synchronize()
+    out.append(C.cpu().numpy())
+np.save(sys.argv[1], np.concatenate([o.ravel() for o in out]))
+""" % os.path.dirname(os.path.abspath(__file__))
+    import tempfile
+    res = []
+    with tempfile.TemporaryDirectory() as d:
+        for one in ("0", "1"):
+            path = os.path.join(d, f"c{one}.npy")
+            env = dict(os.environ, LSGD_GEMM_ONE_TILE=one)
+            r = subprocess.run([sys.executable, "-c", prog, path], env=env, capture_output=True,
+                               text=True, timeout=600)
+            assert r.returncode == 0, r.stderr[-2000:]
+            res.append(np.load(path))
+    assert np.array_equal(res[0], res[1])

@@ -81,15 +81,20 @@ def switch_step(w, K=None):
 UPDATE_BYTES_PER_PARAM = 22
 FUSED_UPDATE_BYTES_PER_PARAM = 18
 AVERAGE_BYTES_PER_PARAM = 10
-# DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum) per step of the fused update
-# launches, from ncu captures of the current kernels:
-#   MLP 3072-1024-1024-10, K = 16, B_loc = 128: the classifier head's backward plus the one
-#     weight-gradient + update launch of both hidden layers, 1,186,195,456 B (below the
-#     algorithmic bytes because part of the launch's writes is still in L2 when it ends);
-#   MLP 3072-4096x3-100: one step's three weight-gradient + update launches captured at K = 2
-#     (1,557,492,992 B) and scaled by 8 to K = 16 (every tile belongs to one replica, so the
-#     traffic is per replica; the K = 16 arena is too large for a multi-pass capture).
-UPDATE_TRAFFIC_PER_STEP = {CONFIG2["name"]: 1186195456, WORKLOAD["name"]: 8 * 1557492992}
+# DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum) of one step's update launches by step
+# kind, from single-pass ncu captures of the current kernels at the benchmark's size:
+#   MLP 3072-4096x3-100, K = 16, B_loc = 128 (3 launches per step):
+#     "avg_synced" -- a step of the H = 1 phase (the replicas agree at its start, it ends with
+#                     the average): 6,656,504,832 B (step 3 of the job);
+#     "plain"      -- an H = 16 step that neither starts synced nor ends a round:
+#                     13,563,636,224 B (step 126);
+#   MLP 3072-1024-1024-10, K = 16, B_loc = 128: "plain" 1,195,052,800 B (the classifier head's
+#     backward, 10,148,608 B, plus the one launch of both hidden layers, 1,184,904,192 B).
+# A traced window with a step of another kind reports no traffic.
+UPDATE_TRAFFIC_PER_STEP = {
+    WORKLOAD["name"]: {"avg_synced": 6656504832, "plain": 13563636224},
+    CONFIG2["name"]: {"plain": 1195052800},
+}
 
 FALLBACK_HBM_GBS = 6800.0
 FALLBACK_BF16_TFLOPS = 1900.0
@@ -580,6 +585,27 @@ class DenseRun:
         seg = sum(widths[1:]) + (widths[-2] * widths[-1] if head else 0)
         return upd, AVERAGE_BYTES_PER_PARAM * K * seg
 
+    def step_kind(self, s):
+        """'avg' / 'plain' (whether step s ends with the average formed in its update launches),
+        with '_synced' when the replicas agree at its start."""
+        ends = self.fused and self.kinds[s] == 2 and self.fuse_avg
+        synced = self.K > 1 and (s == 0 or self.kinds[s - 1] == 2)
+        return ("avg" if ends else "plain") + ("_synced" if synced else "")
+
+    def traced_traffic(self):
+        """Measured DRAM bytes of the traced steps' update launches (UPDATE_TRAFFIC_PER_STEP),
+        or None if a step's kind has no capture."""
+        table = UPDATE_TRAFFIC_PER_STEP.get(self.w["name"], {})
+        if not self.fused or self.K != self.w["K"]:
+            return None
+        tot = 0
+        for s in self.traced_steps:
+            b = table.get(self.step_kind(s))
+            if b is None:
+                return None
+            tot += b
+        return tot
+
     def traced_bytes(self):
         """(update, average) algorithmic bytes summed over the traced steps."""
         tot = [0, 0]
@@ -598,7 +624,9 @@ def roofline(run, prof, steps, hbm, peak_src, fused=True):
     upd_n, upd_ms = prof["update"]
     upd_bytes, _ = run.traced_bytes()
     upd_gbs = upd_bytes / (upd_ms / 1000.0) / 1e9
-    traffic = UPDATE_TRAFFIC_PER_STEP.get(run.w["name"]) if fused and run.K == run.w["K"] else None
+    traffic = run.traced_traffic()
+    if traffic is not None:
+        traffic /= steps
     n_avg = sum(1 for s in run.traced_steps if run.kinds[s] == 2)
     return {"kernel": ("wgrad_update_kernel (weight gradient + fused local update, and the K-way "
                        "average on round-ending steps)" if fused else "sgd_update_kernel"),
@@ -635,6 +663,13 @@ def run_dense_config(args, key):
     torch.cuda.set_device(0)
     stream = torch.cuda.current_stream()
     w = DENSE_CONFIGS[key]
+    if args.widths:
+        # the same schedule on other layer widths (smaller cases of the same kernels for profiler
+        # captures)
+        widths = tuple(int(v) for v in args.widths.split(","))
+        if widths[0] != w["widths"][0] or widths[-1] != w["widths"][-1]:
+            raise SystemExit("--widths must keep the input width and the number of classes")
+        w = dict(w, widths=widths, name=w["name"] + "_widths_" + "-".join(map(str, widths)))
     fused = w["bf16"] and not args.unfused
     run = DenseRun(P, w, stream, fused, args.replicas or None)
     S_ = args.steps
@@ -739,6 +774,9 @@ def main():
     ap.add_argument("--unfused", action="store_true",
                     help="apply the update with the stand-alone kernel over the whole K x d buffer "
                          "instead of the weight-gradient epilogue (same arithmetic)")
+    ap.add_argument("--widths", default="",
+                    help="with --config: other layer widths, e.g. 3072,2048,2048,2048,100 "
+                         "(smaller cases of the same kernels for profiler captures)")
     ap.add_argument("--replicas", type=int, default=0,
                     help="override K (smaller cases for profiler captures); 0 = the workload's K")
     args = ap.parse_args()

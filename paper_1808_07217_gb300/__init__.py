@@ -42,7 +42,7 @@ EXPORTS = [
     "lsgd_batchnorm_stats_noalloc", "lsgd_block_average", "lsgd_block_sync_count",
     "lsgd_sync_state", "lsgd_set_sync_state", "lsgd_schedule", "lsgd_device_status",
     "lsgd_bounded_wait_selftest", "lsgd_losses_async", "lsgd_synchronize", "lsgd_set_step",
-    "lsgd_conv_wgrad_bf16", "lsgd_conv3x3_bf16", "lsgd_run_batch",
+    "lsgd_conv_wgrad_bf16", "lsgd_conv3x3_bf16", "lsgd_conv3x3_bn_bf16", "lsgd_run_batch",
 ]
 PHASES = ["input", "forward", "loss", "backward", "update", "average"]
 
@@ -170,6 +170,7 @@ def lib():
             "lsgd_set_step": ([vp, i64], st),
             "lsgd_conv_wgrad_bf16": ([vp, vp, vp] + [ctypes.c_int] * 7 + [vp], st),
             "lsgd_conv3x3_bf16": ([ctypes.c_int, vp, vp, vp] + [ctypes.c_int] * 7 + [vp], st),
+            "lsgd_conv3x3_bn_bf16": ([vp] * 5 + [ctypes.c_int] * 7 + [vp], st),
             "lsgd_run_batch": ([vp, vp, vp, ctypes.c_int], st),
             "lsgd_sync_count": ([vp], i64),
             "lsgd_block_sync_count": ([vp], i64),
@@ -524,6 +525,17 @@ def lsgd_conv3x3_bf16(mode: int, inp, W, out, G: int, B: int, Hin: int, Win: int
     _check(lib().lsgd_conv3x3_bf16(int(mode), _ptr(inp), _ptr(W), _ptr(out), int(G), int(B),
                                    int(Hin), int(Win), int(Cin), int(Cout), int(stride),
                                    ctypes.c_void_p(stream)))
+
+
+def lsgd_conv3x3_bn_bf16(x, W, y, mean, rstd, G: int, B: int, Hin: int, Win: int, Cin: int,
+                         Cout: int, stride: int, stream=None):
+    """Forward 3x3 convolution (CONV_FORWARD of lsgd_conv3x3_bf16) with the per-group BatchNorm
+    statistics of its output from the convolution's epilogue: y [G, B, Hout, Wout, Cout] float32,
+    mean and rstd [G, Cout] float32."""
+    stream = _current_stream() if stream is None else stream
+    _check(lib().lsgd_conv3x3_bn_bf16(_ptr(x), _ptr(W), _ptr(y), _ptr(mean), _ptr(rstd), int(G),
+                                      int(B), int(Hin), int(Win), int(Cin), int(Cout), int(stride),
+                                      ctypes.c_void_p(stream)))
 
 
 def lsgd_batchnorm_stats(y, P: int, C: int, G: int, mean, rstd, stream=None):

@@ -1203,7 +1203,27 @@ constexpr int THREADS = 256;
 constexpr int RING_BYTES = 96 * 1024;
 constexpr int MAX_STAGES = 24;  // 4 KB stages (ck = 16)
 constexpr int EPI0 = 128;
+constexpr size_t SMEM_MAX = 227 * 1024;  // dynamic shared memory of one CTA
+// barriers, TMEM slot, epilogue flags, and the statistics' cross-warp sums (two passes x four
+// warps x 16 channels)
+constexpr size_t AUX_BYTES = (2 * MAX_STAGES + 5) * 8 + 16 + 2 * 4 * 16 * 4;
 }  // namespace cv
+
+// Sums 16 values per lane over the 32 lanes of a warp in four halving exchanges and one final
+// exchange: afterwards lane l holds the warp's sum of value l / 2 (lanes 2 j and 2 j + 1 agree).
+__device__ __forceinline__ float warp_colsum16(float (&v)[16], int lane) {
+#pragma unroll
+  for (int w = 8; w >= 1; w >>= 1) {
+    const bool up = (lane & (2 * w)) != 0;
+#pragma unroll
+    for (int i = 0; i < w; ++i) {
+      const float send = up ? v[i] : v[i + w];
+      const float keep = up ? v[i + w] : v[i];
+      v[i] = keep + __shfl_xor_sync(0xffffffffu, send, 2 * w);
+    }
+  }
+  return v[0] + __shfl_xor_sync(0xffffffffu, v[0], 1);
+}
 
 __global__ void __launch_bounds__(cv::THREADS, 1) conv_tc_kernel(const __grid_constant__ ConvArgs a) {
   extern __shared__ uint8_t smem_raw[];
@@ -1225,6 +1245,7 @@ __global__ void __launch_bounds__(cv::THREADS, 1) conv_tc_kernel(const __grid_co
   uint64_t* w_full = acc_empty + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(w_full + 1);
   int* epi_ok = reinterpret_cast<int*>(tmem_slot + 1);
+  float* red = reinterpret_cast<float*>(tmem_slot + 4);  // [2][4][16]
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int g = blockIdx.y, cpr = gridDim.x;
@@ -1324,6 +1345,10 @@ __global__ void __launch_bounds__(cv::THREADS, 1) conv_tc_kernel(const __grid_co
       fi ^= 1;
       return okw;
     };
+    // per-channel BatchNorm statistics of this CTA's output pixels (forward convolutions):
+    // lanes 2 j, 2 j + 1 of warp 4 keep channel 16 ci + j's running count, mean and M2
+    const bool with_stats = a.stats != nullptr;
+    float run_n = 0.f, run_mu[4] = {0.f, 0.f, 0.f, 0.f}, run_m2[4] = {0.f, 0.f, 0.f, 0.f};
     int i = 0;
     for (int tile = blockIdx.x; tile < tiles; tile += cpr, ++i) {
       const int ab = i & 1;
@@ -1336,17 +1361,56 @@ __global__ void __launch_bounds__(cv::THREADS, 1) conv_tc_kernel(const __grid_co
         dst = ((int64_t)img * a.dst_h + 2 * oy + a.ph_y) * a.dst_w + 2 * ox + a.ph_x;
       }
       float* orow = a.out + (int64_t)g * a.out_gs + dst * a.N;
-      for (int c0 = 0; c0 < a.N; c0 += 16) {
+#pragma unroll
+      for (int ci = 0; ci < 4; ++ci) {
+        const int c0 = 16 * ci;
+        if (c0 >= a.N) break;
         float v[16];
         tmem_ld16(tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(ab * np + c0), v);
 #pragma unroll
         for (int j = 0; j < 4; ++j)
           *reinterpret_cast<float4*>(orow + c0 + 4 * j) =
               make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
+        if (with_stats) {
+          // the tile's 128 pixels: mean, then the sum of squared deviations from it (two
+          // passes over the registers), each summed over the warp and then the four warps
+          float t[16];
+#pragma unroll
+          for (int j = 0; j < 16; ++j) t[j] = v[j];
+          const float ws = warp_colsum16(t, lane);
+          if (!(lane & 1)) red[quarter * 16 + (lane >> 1)] = ws;
+          asm volatile("bar.sync 1, 128;" ::: "memory");
+          const int ch = lane >> 1;
+          const float mt = (((red[ch] + red[16 + ch]) + red[32 + ch]) + red[48 + ch]) * (1.f / BM);
+#pragma unroll
+          for (int j = 0; j < 16; ++j) {
+            const float e = v[j] - __shfl_sync(0xffffffffu, mt, 2 * j);
+            t[j] = e * e;
+          }
+          const float wq = warp_colsum16(t, lane);
+          if (!(lane & 1)) red[64 + quarter * 16 + (lane >> 1)] = wq;
+          asm volatile("bar.sync 1, 128;" ::: "memory");
+          if (quarter == 0) {
+            // Chan et al.'s combination of the running (n, mean, M2) with this tile's
+            const float m2t = ((red[64 + ch] + red[80 + ch]) + red[96 + ch]) + red[112 + ch];
+            const float nt = run_n + (float)BM, f = (float)BM / nt, delta = mt - run_mu[ci];
+            run_mu[ci] = fmaf(delta, f, run_mu[ci]);
+            run_m2[ci] = run_m2[ci] + m2t + delta * delta * run_n * f;
+          }
+        }
       }
+      if (with_stats) run_n += (float)BM;
       asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
       asm volatile("bar.sync 1, 128;" ::: "memory");
       if (leader) mbar_arrive(&acc_empty[ab]);
+    }
+    if (with_stats && quarter == 0 && !(lane & 1)) {
+#pragma unroll
+      for (int ci = 0; ci < 4; ++ci) {
+        if (16 * ci >= a.N) break;
+        a.stats[((int64_t)g * cpr + blockIdx.x) * a.N + 16 * ci + (lane >> 1)] =
+            make_float4(run_n, run_mu[ci], run_m2[ci], 0.f);
+      }
     }
   }
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
@@ -1720,8 +1784,9 @@ bool make_tma_map(CUtensorMap* map, const void* base, bool bf16, uint64_t dim0, 
   return r == CUDA_SUCCESS;
 }
 
-cudaError_t launch_conv_tc(const ConvArgs& a, cudaStream_t stream) {
+cudaError_t launch_conv_tc(const ConvArgs& a, cudaStream_t stream, int* ctas_per_replica) {
   if (a.P <= 0 || a.G <= 0) return cudaSuccess;
+  if (a.stats && a.dst_h > 0) return cudaErrorInvalidValue;
   int rows = 0, images = 0;
   if ((a.ck != 16 && a.ck != 32 && a.ck != 64) || (a.stride != 1 && a.stride != 2) ||
       (a.N != 16 && a.N != 32 && a.N != 64) || a.np != a.N || !a.out || a.G > 65535 ||
@@ -1736,7 +1801,7 @@ cudaError_t launch_conv_tc(const ConvArgs& a, cudaStream_t stream) {
   // Two CTAs per SM where the weights leave room for a ring of at least three stages (a CTA's
   // tiles pass through a chain of handshakes one after another; two CTAs overlap their chains),
   // else one CTA with the full ring.
-  const size_t fixed = 1024 + 9 * (size_t)a.np * a.ck * 2 + (2 * cv::MAX_STAGES + 5) * 8 + 16;
+  const size_t fixed = 1024 + 9 * (size_t)a.np * a.ck * 2 + cv::AUX_BYTES;
   const size_t stage_bytes = 3 * (size_t)BM * a.ck * 2;
   const size_t two_budget = 113 * 1024;
   size_t ring = cv::RING_BYTES;
@@ -1745,19 +1810,26 @@ cudaError_t launch_conv_tc(const ConvArgs& a, cudaStream_t stream) {
     ring = std::min<size_t>(cv::RING_BYTES, ((two_budget - fixed) / 1024) * 1024);
     per_sm = 2;
   }
+  if (per_sm == 1) {
+    // one CTA per SM: the ring takes what the weights leave of the 227 KB (at most 24 stages)
+    ring = std::min<size_t>((size_t)cv::MAX_STAGES * stage_bytes,
+                            ((cv::SMEM_MAX - fixed) / stage_bytes) * stage_bytes);
+  }
   const size_t smem = fixed + ring;
   ConvArgs la = a;
   la.ring_bytes = (int)ring;
   static int attr_dev = -1;
   if (attr_dev != dev) {
     e = cudaFuncSetAttribute(conv_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             1024 + cv::RING_BYTES + 9 * 64 * 64 * 2 + (2 * cv::MAX_STAGES + 5) * 8 + 16);
+                             (int)cv::SMEM_MAX);
     if (e != cudaSuccess) return e;
     attr_dev = dev;
   }
-  // CTAs per replica: about one per SM over all replicas, at most one per tile
+  // CTAs per replica: as many as fit on the SMs at once over all replicas (one wave), at most one
+  // per tile
   const int tiles = a.P / BM;
-  const int cpr = std::max(1, std::min(tiles, (per_sm * sms + a.G - 1) / a.G));
+  const int cpr = std::max(1, std::min(tiles, per_sm * sms / a.G));
+  if (ctas_per_replica) *ctas_per_replica = cpr;
   return launch_pdl(conv_tc_kernel, dim3(cpr, a.G), dim3(cv::THREADS), smem, stream, la);
 }
 

@@ -170,8 +170,12 @@ struct ConvArgs {
   // (image, 2 y + ph_y, 2 x + ph_x) of a dst_h x dst_w grid (one parity phase of a stride-2
   // convolution's data gradient); else to pixel (image, y, x)
   int ph_y, ph_x, dst_h, dst_w;
+  // non-null (only with dst_h = 0): per-CTA BatchNorm statistics of the output, stats[g][q][n] =
+  // (count, mean, sum of squared deviations, 0) over CTA q's pixels, q < the CTAs per replica
+  float4* stats;
 };
-cudaError_t launch_conv_tc(const ConvArgs& a, cudaStream_t stream);
+// ctas_per_replica (if non-null) receives the launch's CTAs per replica (the stats partials).
+cudaError_t launch_conv_tc(const ConvArgs& a, cudaStream_t stream, int* ctas_per_replica = nullptr);
 // Weight gradient of a 3x3 convolution (zero padding 1, stride 1 or 2) on the tensor cores, the
 // column matrix built in shared memory: part[g][q][co][t Cin + ci] = the sum over CTA q's 64-pixel
 // output blocks of dy[g][p][co] x[g][src_t(p)][ci], src_t(p) the input pixel under tap t of output

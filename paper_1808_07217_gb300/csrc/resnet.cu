@@ -471,6 +471,29 @@ __global__ void bn_act_fwd_kernel(const float* __restrict__ y, const float* __re
   }
 }
 
+// The convolution epilogue's per-CTA statistics partials (count, mean, M2) merged in CTA order
+// (Chan et al.): one thread per (replica, channel), partials loaded eight at a time.
+__global__ void bn_merge_partials_kernel(const float4* __restrict__ stats, int nparts, int G, int C,
+                                         float* __restrict__ mean, float* __restrict__ rstd) {
+  pdl_begin();
+  const int t = blockIdx.x * blockDim.x + threadIdx.x;
+  if (t >= G * C) return;
+  const int g = t / C, c = t % C;
+  const float4* src = stats + (int64_t)g * nparts * C + c;
+  float n = 0.f, m = 0.f, M2 = 0.f;
+  for (int q0 = 0; q0 < nparts; q0 += 8) {
+    float4 v[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j)
+      if (q0 + j < nparts) v[j] = __ldg(src + (int64_t)(q0 + j) * C);
+#pragma unroll
+    for (int j = 0; j < 8; ++j)
+      if (q0 + j < nparts) chan_merge(n, m, M2, v[j].x, v[j].y, v[j].z);
+  }
+  mean[t] = m;
+  rstd[t] = 1.0f / sqrtf(M2 / n + kBnEps);
+}
+
 // The same with a fixed group of 4 channels per thread (C / 4 dividing the block size): the
 // channels' gamma, beta, mean and rstd are loaded once, pixels advance by grid strides, and the
 // replica is blockIdx.y (32-bit pixel indexing).
@@ -938,6 +961,54 @@ __global__ void __launch_bounds__(32 * kSumWarps) sum_partials_crop_kernel(
 }
 unsigned sum_partials_grid(int64_t n) { return (unsigned)((n + 31) / 32); }
 
+// The same sum for four consecutive outputs per thread (float4 loads and store), partials added in
+// split order q = 0, 1, ...: for column counts, leading dimensions, tap widths and destinations
+// that keep every group of four outputs contiguous and 16-byte aligned (sum_partials_v4_ok).
+__global__ void __launch_bounds__(256) sum_partials_v4_kernel(
+    const float* __restrict__ part, int nq, int rows, int ldc, int cols, int G,
+    float* __restrict__ out, int64_t out_gs, int tap_src, int tap_dst) {
+  pdl_begin();
+  const int64_t n4 = (int64_t)G * rows * (cols / 4);
+  const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (t >= n4) return;
+  const int j = (int)(t % (cols / 4)) * 4;
+  const int r = (int)((t / (cols / 4)) % rows);
+  const int g = (int)(t / ((int64_t)rows * (cols / 4)));
+  const int js = tap_dst > 0 ? (j / tap_dst) * tap_src + j % tap_dst : j;
+  const float* p = part + (int64_t)g * nq * rows * ldc + (int64_t)r * ldc + js;
+  const int64_t qs = (int64_t)rows * ldc;
+  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll 4
+  for (int q = 0; q < nq; ++q) {
+    const float4 v = __ldg(reinterpret_cast<const float4*>(p + q * qs));
+    acc.x += v.x;
+    acc.y += v.y;
+    acc.z += v.z;
+    acc.w += v.w;
+  }
+  *reinterpret_cast<float4*>(out + (int64_t)g * out_gs + (int64_t)r * cols + j) = acc;
+}
+
+bool sum_partials_v4_ok(const float* part, int ldc, int cols, const float* out, int64_t out_gs,
+                        int tap_src, int tap_dst) {
+  return cols % 4 == 0 && ldc % 4 == 0 && out_gs % 4 == 0 &&
+         (tap_dst == 0 || (tap_dst % 4 == 0 && tap_src % 4 == 0)) &&
+         (reinterpret_cast<uintptr_t>(part) & 15) == 0 && (reinterpret_cast<uintptr_t>(out) & 15) == 0;
+}
+
+// Launches whichever of the two partial-sum kernels fits the shapes.
+void launch_sum_partials(const float* part, int nq, int rows, int ldc, int cols, int G, float* out,
+                         int64_t out_gs, int tap_src, int tap_dst, cudaStream_t s) {
+  if (sum_partials_v4_ok(part, ldc, cols, out, out_gs, tap_src, tap_dst)) {
+    const int64_t n4 = (int64_t)G * rows * (cols / 4);
+    launch_pdl(sum_partials_v4_kernel, (unsigned)((n4 + 255) / 256), 256, 0, s, part, nq, rows, ldc,
+               cols, G, out, out_gs, tap_src, tap_dst);
+  } else {
+    launch_pdl(sum_partials_crop_kernel, sum_partials_grid((int64_t)G * rows * cols),
+               32 * kSumWarps, 0, s, part, nq, rows, ldc, cols, G, out, out_gs, tap_src, tap_dst);
+  }
+}
+
 // The stem's image with zero channels appended: x16[q][c] = c < C0 ? x0[q][c] : 0 (one thread per
 // pixel, two 16-byte stores).
 __global__ void pad_input16_kernel(const uint16_t* __restrict__ x0, uint16_t* __restrict__ x16,
@@ -1067,6 +1138,9 @@ struct ResNetPlan {
   uint16_t* wstem = nullptr;  // [K][Cout][9][16]
   // the stride-2 data gradients as four parity phases on the implicit kernel: their weights
   uint16_t* wt4 = nullptr;    // [4][K][Cin][9][Cout] of the largest such convolution
+  // BatchNorm statistics computed by the forward convolutions' epilogues: per replica and CTA,
+  // (count, mean, M2) of each channel, merged by bn_merge_partials_kernel
+  float4* cstats = nullptr;   // [K + 2 SMs][64]
   std::string err;
 };
 
@@ -1206,7 +1280,8 @@ size_t conv_wt_elems(int G, int cin, int cout, int stride) {
 
 lsgd_status conv_fwd_tc(const uint16_t* x, const uint16_t* w, int64_t w_gs, float* y, int G, int B,
                         int hin, int win, int cin, int cout, int stride, uint16_t* x16,
-                        uint16_t* wstem, cudaStream_t s, std::string& err, int64_t* launches) {
+                        uint16_t* wstem, cudaStream_t s, std::string& err, int64_t* launches,
+                        float4* stats = nullptr, int* nparts = nullptr) {
   if (!conv_fwd_tc_route(B, hin, win, cin, cout, stride)) {
     err = "convolution shape not taken by the implicit-GEMM kernel";
     return LSGD_EUNSUPPORTED;
@@ -1242,7 +1317,8 @@ lsgd_status conv_fwd_tc(const uint16_t* x, const uint16_t* w, int64_t w_gs, floa
   ca.P = (int)P;
   ca.out = y;
   ca.out_gs = P * cout;
-  CV_CALL(launch_conv_tc(ca, s));
+  ca.stats = stats;
+  CV_CALL(launch_conv_tc(ca, s, stats ? nparts : nullptr));
   return LSGD_OK;
 }
 
@@ -1311,17 +1387,21 @@ lsgd_status conv_dgrad_tc(const uint16_t* dy, const uint16_t* w, int64_t w_gs, f
   return LSGD_OK;
 }
 
+// stats / nparts: where the persistent implicit kernel runs, it also writes the output's
+// per-CTA BatchNorm statistics to stats and their count per replica to *nparts (else 0).
 template <typename TA>
 lsgd_status conv_forward(ResNetPlan* p, int i, const void* in, const void* Wop, int w_g0,
-                         int w_gmul, float* y, int G, cudaStream_t s, int64_t* launches) {
+                         int w_gmul, float* y, int G, cudaStream_t s, int64_t* launches,
+                         float4* stats, int* nparts) {
   const ConvL& c = p->convs[i];
   const int64_t P = conv_pixels(p, c);
+  *nparts = 0;
   if (i == 0 && p->stem16 && w_g0 == 0 && w_gmul == 1) {
     // the stem as a 16-channel convolution on the persistent implicit-GEMM kernel
     const lsgd_status st = conv_fwd_tc(reinterpret_cast<const uint16_t*>(in),
                                        reinterpret_cast<const uint16_t*>(Wop) + c.w_off, p->d_pad, y,
                                        G, p->B, c.hin, c.win, c.cin, c.cout, 1, p->x16, p->wstem, s,
-                                       p->err, launches);
+                                       p->err, launches, stats, nparts);
     return st;
   }
   if (conv_on_tc(p, c) && w_g0 == 0 && w_gmul == 1) {
@@ -1368,7 +1448,8 @@ lsgd_status conv_forward(ResNetPlan* p, int i, const void* in, const void* Wop, 
       // persistent implicit GEMM: the input tile of each tap straight from the NHWC activation
       // by TMA
       return conv_fwd_tc(reinterpret_cast<const uint16_t*>(in), wop, w_gs, y, G, p->B, c.hin, c.win,
-                         c.cin, c.cout, c.stride, nullptr, nullptr, s, p->err, launches);
+                         c.cin, c.cout, c.stride, nullptr, nullptr, s, p->err, launches, stats,
+                         nparts);
     }
     if (implicit_conv_ok(c.cin, c.stride, c.hout, c.wout) && Kc == 9 * c.cin) {
       // implicit GEMM: the input tile of each tap straight from the NHWC activation by TMA
@@ -1445,10 +1526,20 @@ lsgd_status forward_impl(ResNetPlan* p, const float* W, const void* Wop, int w_g
     const ConvL& c = p->convs[i];
     // block j uses convolutions 2j+1 (input act[2j], the block input) and 2j+2 (input act[2j+1])
     const void* in = i == 0 ? p->x0 : p->act[i - 1];
-    lsgd_status st = conv_forward<TA>(p, (int)i, in, Wop, w_g0, w_gmul, p->y[i], G, s, launches);
+    // the convolution's epilogue forms the BatchNorm statistics where it can (one small kernel
+    // merges its per-CTA partials), else the two statistics passes run
+    int nparts = 0;
+    float4* cst = p->cstats && vec4_ok(c.cout) && c.cout <= 64 ? p->cstats : nullptr;
+    lsgd_status st = conv_forward<TA>(p, (int)i, in, Wop, w_g0, w_gmul, p->y[i], G, s, launches,
+                                      cst, &nparts);
     if (st != LSGD_OK) return st;
-    st = bn_stats(p, c, p->y[i], p->mean[i], p->rstd[i], G, s, launches);
-    if (st != LSGD_OK) return st;
+    if (nparts == 0) {
+      st = bn_stats(p, c, p->y[i], p->mean[i], p->rstd[i], G, s, launches);
+      if (st != LSGD_OK) return st;
+    } else {
+      RN_LAUNCH((launch_pdl(bn_merge_partials_kernel, (G * c.cout + 127) / 128, 128, 0, s, cst,
+          nparts, G, c.cout, p->mean[i], p->rstd[i])));
+    }
     const bool second = i > 0 && i % 2 == 0;
     const TA* sc = second ? reinterpret_cast<const TA*>(p->act[i - 2]) : nullptr;
     const ConvL& ca = p->convs[second ? i - 1 : i];
@@ -1572,9 +1663,8 @@ lsgd_status conv_wgrad(ResNetPlan* p, int i, const void* in, float* Gr, cudaStre
     t.splits = splits;
     t.epi = EPI_STORE;
     RN_CALL(launch_gemm_tc(t, s));
-    RN_LAUNCH((launch_pdl(sum_partials_crop_kernel,
-        sum_partials_grid((int64_t)K * c.cout * 9 * c.cin), 32 * kSumWarps, 0, s, p->part, splits,
-        c.cout, Kc, 9 * c.cin, K, Gr + c.w_off, p->d_pad, 0, 0)));
+    RN_LAUNCH((launch_sum_partials(p->part, splits, c.cout, Kc, 9 * c.cin, K, Gr + c.w_off,
+        p->d_pad, 0, 0, s)));
     return LSGD_OK;
   }
   const int nq = (int)((P + kWgradChunk - 1) / kWgradChunk);
@@ -1838,6 +1928,48 @@ lsgd_status conv3x3_bf16(int mode, const uint16_t* in, const uint16_t* w, float*
   return st;
 }
 
+size_t conv3x3_bn_scratch_bytes(int G, int B, int hin, int win, int cin, int cout, int stride) {
+  int dev = 0, sms = kNumSMs;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) {
+    cudaGetLastError();
+    sms = kNumSMs;
+  }
+  const size_t conv = (conv3x3_scratch_bytes(0, G, B, hin, win, cin, cout, stride) + 15) / 16 * 16;
+  return conv + (size_t)(G + 2 * sms) * cout * sizeof(float4);
+}
+
+lsgd_status conv3x3_bn_bf16(const uint16_t* in, const uint16_t* w, float* y, float* mean,
+                            float* rstd, int G, int B, int hin, int win, int cin, int cout,
+                            int stride, void* scratch, cudaStream_t s, std::string* err) {
+  std::string e;
+  if (cout > 64 || !vec4_ok(cout)) {
+    if (err) *err = "the fused statistics take at most 64 output channels";
+    return LSGD_EUNSUPPORTED;
+  }
+  const int64_t w_gs = (int64_t)cout * 9 * cin;
+  uint8_t* sc = static_cast<uint8_t*>(scratch);
+  const size_t conv = (conv3x3_scratch_bytes(0, G, B, hin, win, cin, cout, stride) + 15) / 16 * 16;
+  uint16_t* x16 = conv ? reinterpret_cast<uint16_t*>(sc) : nullptr;
+  float4* stats = reinterpret_cast<float4*>(sc + conv);
+  int nparts = 0;
+  int64_t launches = 0;
+  lsgd_status st = conv_fwd_tc(in, w, w_gs, y, G, B, hin, win, cin, cout, stride, x16,
+                               x16 ? x16 + conv_x16_elems(G, B, hin, win) : nullptr, s, e,
+                               &launches, stats, &nparts);
+  if (st == LSGD_OK) {
+    launch_pdl(bn_merge_partials_kernel, (G * cout + 127) / 128, 128, 0, s, stats, nparts, G, cout,
+               mean, rstd);
+    const cudaError_t ce = cudaGetLastError();
+    if (ce != cudaSuccess) {
+      e = std::string("statistics merge: ") + cudaGetErrorString(ce);
+      st = LSGD_ECUDA;
+    }
+  }
+  if (st != LSGD_OK && err) *err = e;
+  return st;
+}
+
 size_t conv_wgrad_scratch_floats(int G, int B, int hout, int wout, int cin, int cout, int stride) {
   const int64_t P = (int64_t)B * hout * wout;
   return (size_t)G * conv_wgrad_ctas(cin, stride, wout, G, P) * cout * 9 * cin;
@@ -1870,9 +2002,7 @@ cudaError_t launch_conv_wgrad_bf16(const uint16_t* x, const uint16_t* dy, float*
   cudaError_t e = launch_conv_wgrad_tc(a, s);
   if (e != cudaSuccess) return e;
   // the partials' sum, cropped to the first cin_out channels of every tap
-  launch_pdl(sum_partials_crop_kernel, sum_partials_grid((int64_t)G * cout * 9 * cin_out),
-             32 * kSumWarps, 0, s, part, a.cpr, cout, 9 * cin, 9 * cin_out, G, dW, dW_gs, cin,
-             cin_out);
+  launch_sum_partials(part, a.cpr, cout, 9 * cin, 9 * cin_out, G, dW, dW_gs, cin, cin_out, s);
   return cudaGetLastError();
 }
 
@@ -2092,6 +2222,15 @@ lsgd_status resnet_alloc(ResNetPlan* p, const std::function<void*(size_t)>& allo
   p->dh = (float*)alloc((size_t)p->max_act * 4);
   p->dy = alloc((size_t)p->max_act * e);
   p->s12 = (float*)alloc((size_t)K * 2 * 64 * 4);
+  if (p->tc) {
+    // at most max(K, 2 SMs) CTAs over all replicas (launch_conv_tc), 64 channels each
+    int dev = 0, sms = kNumSMs;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+      return LSGD_ECUDA;
+    p->cstats = (float4*)alloc((size_t)(K + 2 * sms) * 64 * sizeof(float4));
+    if (!p->cstats) return LSGD_ENOMEM;
+  }
   if (!p->x0 || !p->part || !p->feat || !p->dfeat || !p->logits || !p->dlogits || !p->dA[0] ||
       !p->dA[1] || !p->dh || !p->dy || !p->s12)
     return LSGD_ENOMEM;

@@ -61,6 +61,13 @@ bool conv3x3_tc_route(int mode, int B, int hin, int win, int cin, int cout, int 
 lsgd_status conv3x3_bf16(int mode, const uint16_t* in, const uint16_t* w, float* out, int G, int B,
                          int hin, int win, int cin, int cout, int stride, void* scratch,
                          cudaStream_t s, std::string* err);
+// Mode 0 of conv3x3_bf16 with the output's per-replica BatchNorm statistics formed in the
+// convolution's epilogue (as the ResNet-20 step forms them): mean, rstd [G][cout], rstd = 1 /
+// sqrt(biased variance + 1e-5).  cout <= 64.  scratch: conv3x3_bn_scratch_bytes bytes.
+size_t conv3x3_bn_scratch_bytes(int G, int B, int hin, int win, int cin, int cout, int stride);
+lsgd_status conv3x3_bn_bf16(const uint16_t* in, const uint16_t* w, float* y, float* mean,
+                            float* rstd, int G, int B, int hin, int win, int cin, int cout,
+                            int stride, void* scratch, cudaStream_t s, std::string* err);
 cudaError_t launch_batchnorm_stats(const float* y, int64_t P, int C, int G, float* mean,
                                    float* rstd, float* part, cudaStream_t s);
 const char* resnet_last_error(const ResNetPlan* p);

@@ -1746,6 +1746,33 @@ lsgd_status lsgd_conv3x3_bf16(int mode, const uint16_t* in, const uint16_t* W, f
   return LSGD_OK;
 }
 
+lsgd_status lsgd_conv3x3_bn_bf16(const uint16_t* x, const uint16_t* W, float* y, float* mean,
+                                 float* rstd, int G, int B, int Hin, int Win, int Cin, int Cout,
+                                 int stride, void* stream) {
+  if (!x || !W || !y || !mean || !rstd || G < 1 || G > 65535 || B < 1 || Hin < 1 || Win < 1 ||
+      Cin < 1 || Cout < 1 || (stride != 1 && stride != 2))
+    return fail(nullptr, LSGD_EINVAL, "lsgd_conv3x3_bn_bf16: bad arguments");
+  if (((uintptr_t)x & 15) || ((uintptr_t)W & 15))
+    return fail(nullptr, LSGD_EINVAL, "lsgd_conv3x3_bn_bf16: operands must be 16-byte aligned");
+  if (!lsgd::tc_available()) return fail(nullptr, LSGD_EUNSUPPORTED, "tcgen05 not available");
+  if (!lsgd::conv3x3_tc_route(0, B, Hin, Win, Cin, Cout, stride) || Cout > 64)
+    return fail(nullptr, LSGD_EUNSUPPORTED,
+                "lsgd_conv3x3_bn_bf16: shape not taken by the implicit-GEMM convolution kernel");
+  cudaStream_t s = (cudaStream_t)stream;
+  void* scratch = nullptr;
+  const size_t bytes = lsgd::conv3x3_bn_scratch_bytes(G, B, Hin, Win, Cin, Cout, stride);
+  if (cudaMallocAsync(&scratch, bytes, s) != cudaSuccess) {
+    cudaGetLastError();
+    return fail(nullptr, LSGD_ENOMEM, "lsgd_conv3x3_bn_bf16: scratch allocation failed");
+  }
+  std::string err;
+  const lsgd_status st = lsgd::conv3x3_bn_bf16(x, W, y, mean, rstd, G, B, Hin, Win, Cin, Cout,
+                                               stride, scratch, s, &err);
+  cudaFreeAsync(scratch, s);
+  if (st != LSGD_OK) return fail(nullptr, st, ("lsgd_conv3x3_bn_bf16: " + err).c_str());
+  return LSGD_OK;
+}
+
 lsgd_status lsgd_sample_indices(int32_t* dst, uint64_t seed, int64_t step, int K, int B, int64_t N,
                                 void* stream) {
   if (!dst || K < 1 || B < 1 || N < K) return fail(nullptr, LSGD_EINVAL, "lsgd_sample_indices: bad arguments");

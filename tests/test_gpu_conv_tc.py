@@ -184,3 +184,62 @@ def test_conv_rejects_shapes_the_kernel_does_not_take(P):
         with pytest.raises(P.LsgdError) as e:
             P.lsgd_conv3x3_bf16(mode, buf, buf, out, **kw)
         assert e.value.status == status, (mode, bad, e.value.status)
+
+
+BN_SHAPES = [  # (G, B, Hin, Win, Cin, Cout, stride): forward convolutions of ResNet-20
+    (2, 3, 32, 32, 3, 16, 1),      # stem (padded to 16 channels)
+    (3, 3, 32, 32, 16, 16, 1),     # stage 1, one CTA holds several tiles
+    (2, 5, 32, 32, 16, 32, 2),     # stage-2 entry
+    (3, 6, 16, 16, 32, 64, 2),     # stage-3 entry: 64 channels, four 16-channel chunks
+    (2, 6, 8, 8, 64, 64, 1),       # stage 3
+    (16, 16, 32, 32, 16, 16, 1),   # many groups
+]
+
+
+@pytest.mark.parametrize("shape", BN_SHAPES)
+def test_conv_epilogue_batchnorm_statistics(P, shape):
+    # Sec. A.4's per-worker batch statistics of the convolution output, formed by the epilogue
+    # (per-tile two-pass moments combined by Chan et al.'s formula), against fp64 moments of the
+    # same fp32 output; the output itself must be the plain forward's, bit for bit
+    import torch
+
+    G, B, Hin, Win, Cin, Cout, s = shape
+    Hout, Wout = (Hin - 1) // s + 1, (Win - 1) // s + 1
+    gen = torch.Generator(device="cuda").manual_seed(11 * sum(shape))
+    x = _bf16_randn(torch, (G, B, Hin, Win, Cin), gen)
+    # a mean offset per output channel, so that the variance is not the raw second moment
+    w = (torch.randn((G, Cout, 3, 3, Cin), device="cuda", generator=gen) +
+         0.5 * torch.arange(Cout, device="cuda").view(1, Cout, 1, 1, 1) / Cout).to(torch.bfloat16)
+    y = torch.full((G, B, Hout, Wout, Cout), float("nan"), device="cuda")
+    y_plain = torch.empty_like(y)
+    mean = torch.full((G, Cout), float("nan"), device="cuda")
+    rstd = torch.full((G, Cout), float("nan"), device="cuda")
+    P.lsgd_conv3x3_bn_bf16(x, w, y, mean, rstd, G, B, Hin, Win, Cin, Cout, s)
+    P.lsgd_conv3x3_bf16(P.CONV_FORWARD, x, w, y_plain, G, B, Hin, Win, Cin, Cout, s)
+    torch.cuda.synchronize()
+    assert torch.equal(y, y_plain)
+    y64 = y.double().cpu().numpy().reshape(G, -1, Cout)
+    m64 = y64.mean(axis=1)
+    v64 = y64.var(axis=1)  # biased, as BatchNorm normalises
+    got_m = mean.cpu().numpy().astype(np.float64)
+    got_r = rstd.cpu().numpy().astype(np.float64)
+    scale = np.sqrt(v64)
+    assert np.abs(got_m - m64).max() <= 1e-5 * (np.abs(m64) + scale).max()
+    np.testing.assert_allclose(got_r, 1.0 / np.sqrt(v64 + 1e-5), rtol=2e-5)
+
+
+def test_conv_epilogue_statistics_are_deterministic(P):
+    import torch
+
+    G, B, H, C = 4, 16, 32, 16
+    gen = torch.Generator(device="cuda").manual_seed(5)
+    x = _bf16_randn(torch, (G, B, H, H, C), gen)
+    w = _bf16_randn(torch, (G, C, 3, 3, C), gen)
+    outs = []
+    for _ in range(2):
+        y = torch.empty((G, B, H, H, C), device="cuda")
+        mean = torch.empty((G, C), device="cuda")
+        rstd = torch.empty((G, C), device="cuda")
+        P.lsgd_conv3x3_bn_bf16(x, w, y, mean, rstd, G, B, H, H, C, C, 1)
+        outs.append((mean.cpu(), rstd.cpu()))
+    assert torch.equal(outs[0][0], outs[1][0]) and torch.equal(outs[0][1], outs[1][1])

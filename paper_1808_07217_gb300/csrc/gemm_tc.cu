@@ -1190,10 +1190,15 @@ __global__ void __launch_bounds__(wu::THREADS, 1) wgrad_update_kernel(
 // in[g][shift_t(p)][k] w[g][n][t][k] (zero padding 1, stride 1 or 2), fp32 out.
 //
 // A CTA owns one replica and every cpr-th 128-pixel tile of it.  The replica's weights (all nine
-// taps, N rows of ck channels) are loaded once; the input tile of each tap streams through a
-// ring of shared-memory stages by TMA (a rank-5 box of the NHWC input, out-of-bounds fill = the
-// zero padding, element strides = the convolution stride); two TMEM accumulators let a tile's
-// MMAs overlap the previous tile's epilogue.
+// taps, N rows of ck channels) are loaded once; the input streams through a ring of shared-memory
+// stages by TMA (rank-5 boxes of the NHWC input, out-of-bounds fill = the zero padding, element
+// strides = the convolution stride); two TMEM accumulators let a tile's MMAs overlap the previous
+// tile's epilogue.  Two stage forms:
+//   strip (stride 1, a tile = whole rows of one image): one stage per tile holds, for each kw, the
+//     tile's rows plus one halo row above and below, shifted by kw - 1 columns; tap (kh, kw) is
+//     that box from row kh on (a whole number of swizzle atoms further), so 3 boxes serve 9 taps;
+//   per kernel row: three stages per tile, stage kh holds the three kw-shifted boxes of the
+//     tile's rows under kernel row kh (stride 2, and tiles that span several images).
 //   warp 0      TMA producer (weights once, then one stage per tap)
 //   warp 1      MMA issuer: per tap ck / 16 tcgen05.mma (M = 128, N = NP, K = 16)
 //   warp 2      TMEM allocation
@@ -1230,9 +1235,13 @@ __global__ void __launch_bounds__(cv::THREADS, 1) conv_tc_kernel(const __grid_co
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
   const int ck = a.ck, np = a.np;
-  // a stage holds the three taps of one kernel row (kh): three TMA boxes, one handshake
+  // per-kernel-row form: a stage holds the three taps of one kernel row (three TMA boxes, one
+  // handshake); strip form: a stage holds the three kw boxes of (rows + 2) image rows
   const uint32_t tap_bytes = (uint32_t)BM * ck * 2;
-  const uint32_t stage_bytes = 3 * tap_bytes;
+  const uint32_t row_bytes = (uint32_t)a.wout * ck * 2;  // one image row of the input box
+  const uint32_t box_bytes = a.strip ? tap_bytes + 2 * row_bytes : tap_bytes;
+  const uint32_t stage_bytes = 3 * box_bytes;
+  const int spt = a.strip ? 1 : 3;  // stages per tile
   const int nst = min(cv::MAX_STAGES, a.ring_bytes / (int)stage_bytes);
   uint8_t* ring = base;
   uint8_t* wsm = base + a.ring_bytes;
@@ -1287,16 +1296,19 @@ __global__ void __launch_bounds__(cv::THREADS, 1) conv_tc_kernel(const __grid_co
     bool ok = true;
     for (int tile = blockIdx.x; tile < tiles && ok; tile += cpr) {
       const int p0 = tile * BM, b0 = p0 / per_img, oy0 = (p0 / a.wout) % a.hout;
-      for (int kh = 0; kh < 3; ++kh, ++q) {
+      for (int sp = 0; sp < spt; ++sp, ++q) {
         const int sl = q % nst;
         if (!mbar_wait(&empty[sl], ((q / nst) & 1) ^ 1)) {
           ok = false;
           break;
         }
         mbar_expect_tx(&full[sl], stage_bytes);
+        // strip: rows oy0 - 1 .. oy0 + rows (the halo rows out of the image read as zeros);
+        // per kernel row sp: the rows under kernel row sp
+        const int y0 = a.strip ? oy0 - 1 : oy0 * a.stride + sp - 1;
         for (int kw = 0; kw < 3; ++kw)
-          tma_load_5d(ring + sl * stage_bytes + kw * tap_bytes, &a.in_map, &full[sl], 0, kw - 1,
-                      oy0 * a.stride + kh - 1, b0, g);
+          tma_load_5d(ring + sl * stage_bytes + kw * box_bytes, &a.in_map, &full[sl], 0, kw - 1,
+                      y0, b0, g);
       }
     }
     // copies in flight land before the CTA can exit
@@ -1314,20 +1326,24 @@ __global__ void __launch_bounds__(cv::THREADS, 1) conv_tc_kernel(const __grid_co
       if (!mbar_wait(&acc_empty[ab], ((i >> 1) & 1) ^ 1)) break;
       asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
       const uint32_t acc = tmem + (uint32_t)(ab * np);
-      for (int kh = 0; kh < 3; ++kh, ++q) {
+      for (int sp = 0; sp < spt; ++sp, ++q) {
         const int sl = q % nst;
         if (!mbar_wait(&full[sl], (q / nst) & 1)) {
           ok = false;
           break;
         }
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-        for (int kw = 0; kw < 3; ++kw) {
-          const int t = kh * 3 + kw;
-          const uint32_t a_base = smem_u32(ring + sl * stage_bytes + kw * tap_bytes);
-          const uint32_t b_base = smem_u32(wsm + t * wtap);
-          for (int kk = 0; kk < ck / 16; ++kk)
-            mma_bf16(acc, smem_desc_kmajor(a_base + kk * 32, swz),
-                     smem_desc_kmajor(b_base + kk * 32, swz), idesc, (t > 0 || kk > 0) ? 1u : 0u);
+        const uint32_t st_base = smem_u32(ring + sl * stage_bytes);
+        for (int kh = a.strip ? 0 : sp; kh < (a.strip ? 3 : sp + 1); ++kh) {
+          for (int kw = 0; kw < 3; ++kw) {
+            const int t = kh * 3 + kw;
+            const uint32_t a_base = st_base + kw * box_bytes + (a.strip ? kh * row_bytes : 0u);
+            const uint32_t b_base = smem_u32(wsm + t * wtap);
+            for (int kk = 0; kk < ck / 16; ++kk)
+              mma_bf16(acc, smem_desc_kmajor(a_base + kk * 32, swz),
+                       smem_desc_kmajor(b_base + kk * 32, swz), idesc,
+                       (t > 0 || kk > 0) ? 1u : 0u);
+          }
         }
         mma_commit(&empty[sl]);
       }
@@ -1367,10 +1383,21 @@ __global__ void __launch_bounds__(cv::THREADS, 1) conv_tc_kernel(const __grid_co
         if (c0 >= a.N) break;
         float v[16];
         tmem_ld16(tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(ab * np + c0), v);
+        if (a.st32) {
+          // whole 32-byte sectors per lane and instruction
 #pragma unroll
-        for (int j = 0; j < 4; ++j)
-          *reinterpret_cast<float4*>(orow + c0 + 4 * j) =
-              make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
+          for (int j = 0; j < 2; ++j)
+            asm volatile("st.global.v8.f32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"l"(
+                             orow + c0 + 8 * j),
+                         "f"(v[8 * j]), "f"(v[8 * j + 1]), "f"(v[8 * j + 2]), "f"(v[8 * j + 3]),
+                         "f"(v[8 * j + 4]), "f"(v[8 * j + 5]), "f"(v[8 * j + 6]), "f"(v[8 * j + 7])
+                         : "memory");
+        } else {
+#pragma unroll
+          for (int j = 0; j < 4; ++j)
+            *reinterpret_cast<float4*>(orow + c0 + 4 * j) =
+                make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
+        }
         if (with_stats) {
           // the tile's 128 pixels: mean, then the sum of squared deviations from it (two
           // passes over the registers), each summed over the warp and then the four warps
@@ -1802,7 +1829,9 @@ cudaError_t launch_conv_tc(const ConvArgs& a, cudaStream_t stream, int* ctas_per
   // tiles pass through a chain of handshakes one after another; two CTAs overlap their chains),
   // else one CTA with the full ring.
   const size_t fixed = 1024 + 9 * (size_t)a.np * a.ck * 2 + cv::AUX_BYTES;
-  const size_t stage_bytes = 3 * (size_t)BM * a.ck * 2;
+  const bool strip = a.strip != 0;
+  if (strip && !conv_strip_ok(a.hout, a.wout, a.stride)) return cudaErrorInvalidValue;
+  const size_t stage_bytes = 3 * ((size_t)BM + (strip ? 2 * a.wout : 0)) * a.ck * 2;
   const size_t two_budget = 113 * 1024;
   size_t ring = cv::RING_BYTES;
   int per_sm = 1;
@@ -1818,6 +1847,7 @@ cudaError_t launch_conv_tc(const ConvArgs& a, cudaStream_t stream, int* ctas_per
   const size_t smem = fixed + ring;
   ConvArgs la = a;
   la.ring_bytes = (int)ring;
+  la.st32 = (reinterpret_cast<uintptr_t>(a.out) & 31) == 0 && a.out_gs % 8 == 0 ? 1 : 0;
   static int attr_dev = -1;
   if (attr_dev != dev) {
     e = cudaFuncSetAttribute(conv_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -1886,8 +1916,16 @@ bool conv_tile_shape(int hout, int wout, int* rows, int* images) {
   return true;
 }
 
+bool conv_strip_ok(int hout, int wout, int stride) {
+  int rows = 0, images = 0;
+  // the kernel-row offsets inside a box must be whole swizzle atoms (8 pixel rows of the
+  // channel width): wout a multiple of 8
+  return stride == 1 && conv_tile_shape(hout, wout, &rows, &images) && images == 1 &&
+         wout % 8 == 0 && rows + 2 <= 256;
+}
+
 bool make_tma_map_conv(CUtensorMap* map, const void* base, int ck, int win, int hin, int B, int G,
-                       int wout, int hout, int stride) {
+                       int wout, int hout, int stride, bool strip) {
   std::call_once(g_encode_once, load_encode);
   int rows = 0, images = 0;
   if (!g_encode || (ck != 16 && ck != 32 && ck != 64) || (stride != 1 && stride != 2) ||
@@ -1899,7 +1937,10 @@ bool make_tma_map_conv(CUtensorMap* map, const void* base, int ck, int win, int 
                         (cuuint64_t)G};
   cuuint64_t strides[4] = {(cuuint64_t)ck * e, (cuuint64_t)win * ck * e,
                            (cuuint64_t)hin * win * ck * e, (cuuint64_t)B * hin * win * ck * e};
-  cuuint32_t box[5] = {(cuuint32_t)ck, (cuuint32_t)(wout * stride), (cuuint32_t)(rows * stride),
+  // the strip form's box has a halo row above and below
+  if (strip && !conv_strip_ok(hout, wout, stride)) return false;
+  const int box_rows = strip ? rows + 2 : rows * stride;
+  cuuint32_t box[5] = {(cuuint32_t)ck, (cuuint32_t)(wout * stride), (cuuint32_t)box_rows,
                        (cuuint32_t)images, 1};
   cuuint32_t estr[5] = {1, (cuuint32_t)stride, (cuuint32_t)stride, 1, 1};
   const CUtensorMapSwizzle sw = ck == 64 ? CU_TENSOR_MAP_SWIZZLE_128B

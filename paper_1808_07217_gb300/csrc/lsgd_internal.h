@@ -173,7 +173,13 @@ struct ConvArgs {
   // non-null (only with dst_h = 0): per-CTA BatchNorm statistics of the output, stats[g][q][n] =
   // (count, mean, sum of squared deviations, 0) over CTA q's pixels, q < the CTAs per replica
   float4* stats;
+  int strip;  // stage form: 1 = strip (in_map made with strip = true), 0 = per kernel row
+  int st32;   // out 32-byte aligned: 256-bit stores (set by the launcher)
 };
+// Stride 1 and tiles of whole image rows with a width that is a multiple of 8: the convolution's
+// input boxes carry one halo row above and below (make_tma_map_conv) and one stage feeds all nine
+// taps of a tile.
+bool conv_strip_ok(int hout, int wout, int stride);
 // ctas_per_replica (if non-null) receives the launch's CTAs per replica (the stats partials).
 cudaError_t launch_conv_tc(const ConvArgs& a, cudaStream_t stream, int* ctas_per_replica = nullptr);
 // Weight gradient of a 3x3 convolution (zero padding 1, stride 1 or 2) on the tensor cores, the
@@ -199,8 +205,10 @@ cudaError_t launch_conv_wgrad_tc(const ConvWgradArgs& a, cudaStream_t stream);
 // The tile geometry of an implicit convolution with an Hout x Wout output: whole output rows,
 // 128 pixels per tile.  False when the shape does not tile that way.
 bool conv_tile_shape(int hout, int wout, int* rows, int* images);
+// strip: the box of the strip form (rows + 2 rows; conv_strip_ok must hold), else the tile's
+// rows at the convolution stride.
 bool make_tma_map_conv(CUtensorMap* map, const void* base, int ck, int win, int hin, int B, int G,
-                       int wout, int hout, int stride);
+                       int wout, int hout, int stride, bool strip = false);
 
 cudaError_t launch_gemm_simt(const GemmArgs& a, cudaStream_t stream);
 
@@ -248,11 +256,6 @@ struct TcGemmArgs {
   // identical (the step follows an average), so one copy serves all, mostly from L2
   int b_shared;
 };
-// The tile geometry of an implicit convolution with an Hout x Wout output: whole output rows,
-// 128 pixels per tile.  False when the shape does not tile that way.
-bool conv_tile_shape(int hout, int wout, int* rows, int* images);
-bool make_tma_map_conv(CUtensorMap* map, const void* base, int ck, int win, int hin, int B, int G,
-                       int wout, int hout, int stride);
 
 // The weight gradient of one dense layer fused with the local update, for G replicas: W[g] (M x
 // N, row stride N) -= update(dZ[g]^T act[g]) with the momentum and bf16 shadow of SgdParams.

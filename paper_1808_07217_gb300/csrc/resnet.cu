@@ -1296,12 +1296,14 @@ lsgd_status conv_fwd_tc(const uint16_t* x, const uint16_t* w, int64_t w_gs, floa
     CV_LAUNCH(launch_pdl(pad_input16_kernel, grid_cap(npix, 256), 256, 0, s, x, x16, npix, cin));
     CV_LAUNCH(launch_pdl(pad_stem_weights_kernel, grid_cap((int64_t)G * cout * 144, 256), 256, 0, s,
                          w, w_gs, (int64_t)0, wstem, G, cout, cin));
-    okc = make_tma_map_conv(&ca.in_map, x16, 16, win, hin, B, G, wout, hout, 1);
+    ca.strip = conv_strip_ok(hout, wout, 1);
+    okc = make_tma_map_conv(&ca.in_map, x16, 16, win, hin, B, G, wout, hout, 1, ca.strip);
     okc &= make_tma_map(&ca.w_map, wstem, true, 9 * 16, cout, G, 9 * 16, (uint64_t)cout * 9 * 16, 16,
                         cout, 32);
     ca.ck = 16;
   } else {
-    okc = make_tma_map_conv(&ca.in_map, x, cin, win, hin, B, G, wout, hout, stride);
+    ca.strip = conv_strip_ok(hout, wout, stride);
+    okc = make_tma_map_conv(&ca.in_map, x, cin, win, hin, B, G, wout, hout, stride, ca.strip);
     okc &= make_tma_map(&ca.w_map, w, true, 9 * cin, cout, G, 9 * cin, w_gs, cin, cout, 2 * cin);
     ca.ck = cin;
   }
@@ -1334,7 +1336,8 @@ lsgd_status conv_dgrad_tc(const uint16_t* dy, const uint16_t* w, int64_t w_gs, f
     CV_LAUNCH((launch_pdl(flip_weights_kernel, dim3((unsigned)((cin * 9 * cout + 255) / 256), (unsigned)G),
                           256, 0, s, w, w_gs, (int64_t)0, wt, G, cin, cout)));
     ConvArgs ca{};
-    bool okc = make_tma_map_conv(&ca.in_map, dy, cout, win, hin, B, G, win, hin, 1);
+    ca.strip = conv_strip_ok(hin, win, 1);
+    bool okc = make_tma_map_conv(&ca.in_map, dy, cout, win, hin, B, G, win, hin, 1, ca.strip);
     okc &= make_tma_map(&ca.w_map, wt, true, 9 * cout, cin, G, 9 * cout, (uint64_t)cin * 9 * cout,
                         cout, cin, 2 * cout);
     if (!okc) {
@@ -1362,7 +1365,8 @@ lsgd_status conv_dgrad_tc(const uint16_t* dy, const uint16_t* w, int64_t w_gs, f
   const int64_t Pq = (int64_t)B * hout * wout;
   for (int ph = 0; ph < 4; ++ph) {
     ConvArgs ca{};
-    bool okc = make_tma_map_conv(&ca.in_map, dy, cout, wout, hout, B, G, wout, hout, 1);
+    ca.strip = conv_strip_ok(hout, wout, 1);
+    bool okc = make_tma_map_conv(&ca.in_map, dy, cout, wout, hout, B, G, wout, hout, 1, ca.strip);
     okc &= make_tma_map(&ca.w_map, wt + ph * G * per, true, 9 * cout, cin, G, 9 * cout,
                         (uint64_t)per, cout, cin, 2 * cout);
     if (!okc) {

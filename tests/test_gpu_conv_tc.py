@@ -243,3 +243,22 @@ def test_conv_epilogue_statistics_are_deterministic(P):
         P.lsgd_conv3x3_bn_bf16(x, w, y, mean, rstd, G, B, H, H, C, C, 1)
         outs.append((mean.cpu(), rstd.cpu()))
     assert torch.equal(outs[0][0], outs[1][0]) and torch.equal(outs[0][1], outs[1][1])
+
+
+def test_conv_output_alignment_does_not_change_results(P):
+    # an output 16 but not 32 bytes aligned takes the 128-bit store path; same values
+    import torch
+
+    G, B, H, Cin, Cout = 2, 4, 32, 16, 32
+    gen = torch.Generator(device="cuda").manual_seed(17)
+    x = _bf16_randn(torch, (G, B, H, H, Cin), gen)
+    w = _bf16_randn(torch, (G, Cout, 3, 3, Cin), gen)
+    n = G * B * H * H * Cout
+    y = torch.empty((G, B, H, H, Cout), device="cuda")
+    buf = torch.full((n + 4,), float("nan"), device="cuda")
+    y16 = buf[4:].view(G, B, H, H, Cout)
+    assert y16.data_ptr() % 32 == 16
+    P.lsgd_conv3x3_bf16(P.CONV_FORWARD, x, w, y, G, B, H, H, Cin, Cout, 1)
+    P.lsgd_conv3x3_bf16(P.CONV_FORWARD, x, w, y16, G, B, H, H, Cin, Cout, 1)
+    torch.cuda.synchronize()
+    assert torch.equal(y, y16)

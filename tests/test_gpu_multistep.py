@@ -102,7 +102,11 @@ def test_multistep_parity_against_oracle(P, name):
         assert sens < 2e-2, sens
         assert rel <= 2e-2, rel
         assert d_ev <= 1e-2, d_ev
-        assert np.abs(lg - g["losses"]).max() <= 2e-2, float(np.abs(lg - g["losses"]).max())
+        # every step's mini-batch losses, against the oracle's own spread between roundings
+        # (100-class losses reach ~12 early on, where the two oracle runs differ by up to 0.14)
+        loss_sens = float(np.abs(g["losses"] - g32["losses"]).max())
+        d_loss = float(np.abs(lg - g["losses"]).max())
+        assert d_loss <= max(2e-2, 2 * loss_sens), (d_loss, loss_sens)
     else:
         # one pair of trajectories (oracle bf16 vs fp32) samples how far a change of rounding
         # carries the run; another pair (GPU vs oracle bf16) may land up to about twice as far

@@ -398,10 +398,10 @@ lsgd_status lsgd_conv3x3_bf16(int mode, const uint16_t* in, const uint16_t* W, f
  * statistics of its output (Sec. A.4; the first half of the conv -> BN -> ReLU unit of Sec. A.2's
  * ResNet-20), as the ResNet-20 training step computes them: y [G][B][Hout][Wout][Cout] fp32 as in
  * mode 0, and mean[G][Cout], rstd[G][Cout] = 1 / sqrt(biased variance + 1e-5) over the B Hout Wout
- * output positions of each group.  The epilogue of each CTA of the convolution keeps a running
- * (count, mean, sum of squared deviations) per channel, combining its 128-pixel tiles' two-pass
- * moments in tile order by Chan et al.'s formula; a second kernel combines the CTAs' partials in
- * CTA order, so the result is deterministic.  Same operands, alignment and shapes as mode 0 with
+ * output positions of each group.  Each epilogue warp of the convolution keeps a running (count,
+ * mean, sum of squared deviations) per channel, combining the two-pass moments of its 32 rows of
+ * every 128-pixel tile in tile order by Chan et al.'s formula; a second kernel combines the
+ * warps' partials in a fixed order, so the result is deterministic.  Same operands, alignment and shapes as mode 0 with
  * Cout <= 64; mean and rstd fp32 device arrays.  Scratch (the stem operands and the partials) is
  * allocated and freed on `stream`.  LSGD_EINVAL on bad arguments, LSGD_EUNSUPPORTED for shapes the
  * kernel does not take, LSGD_ENOMEM if the scratch cannot be allocated. */

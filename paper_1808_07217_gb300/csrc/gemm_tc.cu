@@ -1200,18 +1200,24 @@ __global__ void __launch_bounds__(wu::THREADS, 1) wgrad_update_kernel(
 //   per kernel row: three stages per tile, stage kh holds the three kw-shifted boxes of the
 //     tile's rows under kernel row kh (stride 2, and tiles that span several images).
 //   warp 0      TMA producer (weights once, then one stage per tap)
-//   warp 1      MMA issuer: per tap ck / 16 tcgen05.mma (M = 128, N = NP, K = 16)
+//   warp 1      MMA issuer: per tap ck / 16 tcgen05.mma (M = 128, N = NP, K = 16), descriptors
+//               from precomputed bases (the issuing thread is on the critical path); with
+//               nsplit = 3 the taps of column kw accumulate into partial kw, consecutive MMAs
+//               into different partials (small-N MMAs into one accumulator wait on each other)
 //   warp 2      TMEM allocation
-//   warps 4-7   epilogue: tcgen05.ld of the tile row's NP columns, fp32 stores
+//   warps 4-7   epilogue: tcgen05.ld of the tile row's NP columns (the partials' sum), fp32
+//               stores
+// nacc accumulator buffers (each nsplit x NP columns) let the MMAs of the next tiles run while
+// the epilogue drains this one.
 namespace cv {
 constexpr int THREADS = 256;
 constexpr int RING_BYTES = 96 * 1024;
 constexpr int MAX_STAGES = 24;  // 4 KB stages (ck = 16)
 constexpr int EPI0 = 128;
 constexpr size_t SMEM_MAX = 227 * 1024;  // dynamic shared memory of one CTA
-// barriers, TMEM slot, epilogue flags, and the statistics' cross-warp sums (two passes x four
-// warps x 16 channels)
-constexpr size_t AUX_BYTES = (2 * MAX_STAGES + 5) * 8 + 16 + 2 * 4 * 16 * 4;
+constexpr int MAX_ACC = 4;  // accumulator buffers in TMEM
+// barriers, TMEM slot and epilogue flags
+constexpr size_t AUX_BYTES = (2 * MAX_STAGES + 2 * MAX_ACC + 1) * 8 + 16;
 }  // namespace cv
 
 // Sums 16 values per lane over the 32 lanes of a warp in four halving exchanges and one final
@@ -1250,24 +1256,25 @@ __global__ void __launch_bounds__(cv::THREADS, 1) conv_tc_kernel(const __grid_co
   uint64_t* full = bars;
   uint64_t* empty = bars + cv::MAX_STAGES;
   uint64_t* acc_full = bars + 2 * cv::MAX_STAGES;
-  uint64_t* acc_empty = acc_full + 2;
-  uint64_t* w_full = acc_empty + 2;
+  uint64_t* acc_empty = acc_full + cv::MAX_ACC;
+  uint64_t* w_full = acc_empty + cv::MAX_ACC;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(w_full + 1);
   int* epi_ok = reinterpret_cast<int*>(tmem_slot + 1);
-  float* red = reinterpret_cast<float*>(tmem_slot + 4);  // [2][4][16]
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int g = blockIdx.y, cpr = gridDim.x;
   const int tiles = a.P / BM;  // per replica
   const int per_img = a.hout * a.wout;
-  const uint32_t tmem_cols = (uint32_t)(2 * np < 32 ? 32 : 2 * np);
+  const int nacc = a.nacc, nsplit = a.nsplit;
+  const uint32_t acc_cols = (uint32_t)(nsplit * np);  // one accumulator buffer
+  const uint32_t tmem_cols = conv_tmem_cols(nacc * nsplit, np);
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < nst; ++i) {
       mbar_init(&full[i], 1);
       mbar_init(&empty[i], 1);
     }
-    for (int i = 0; i < 2; ++i) {
+    for (int i = 0; i < nacc; ++i) {
       mbar_init(&acc_full[i], 1);
       mbar_init(&acc_empty[i], 1);
     }
@@ -1318,14 +1325,20 @@ __global__ void __launch_bounds__(cv::THREADS, 1) conv_tc_kernel(const __grid_co
     // ---------------- MMA issuer ----------------
     const uint32_t idesc = make_idesc(BM, np, false, false);
     const uint32_t swz = (uint32_t)ck * 2;
+    // descriptors of the ring's start and of tap 0's weights: the address field is in 16-byte
+    // units, so the descriptor of a tap / stage / K-step is the base plus its byte offset / 16
+    const uint64_t a_desc0 = smem_desc_kmajor(smem_u32(ring), swz);
+    const uint64_t b_desc0 = smem_desc_kmajor(smem_u32(wsm), swz);
+    const uint32_t kw_step = box_bytes >> 4, kh_step = (a.strip ? row_bytes : 0u) >> 4;
+    const uint32_t tap_step = wtap >> 4;
     bool ok = mbar_wait(w_full, 0);
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
     int q = 0, i = 0;
     for (int tile = blockIdx.x; tile < tiles && ok; tile += cpr, ++i) {
-      const int ab = i & 1;
-      if (!mbar_wait(&acc_empty[ab], ((i >> 1) & 1) ^ 1)) break;
+      const int ab = i % nacc;
+      if (!mbar_wait(&acc_empty[ab], ((i / nacc) & 1) ^ 1)) break;
       asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-      const uint32_t acc = tmem + (uint32_t)(ab * np);
+      const uint32_t acc = tmem + (uint32_t)ab * acc_cols;
       for (int sp = 0; sp < spt; ++sp, ++q) {
         const int sl = q % nst;
         if (!mbar_wait(&full[sl], (q / nst) & 1)) {
@@ -1333,19 +1346,26 @@ __global__ void __launch_bounds__(cv::THREADS, 1) conv_tc_kernel(const __grid_co
           break;
         }
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-        const uint32_t st_base = smem_u32(ring + sl * stage_bytes);
+        const uint64_t st_desc = a_desc0 + ((uint32_t)sl * stage_bytes >> 4);
         for (int kh = a.strip ? 0 : sp; kh < (a.strip ? 3 : sp + 1); ++kh) {
-          for (int kw = 0; kw < 3; ++kw) {
-            const int t = kh * 3 + kw;
-            const uint32_t a_base = st_base + kw * box_bytes + (a.strip ? kh * row_bytes : 0u);
-            const uint32_t b_base = smem_u32(wsm + t * wtap);
-            for (int kk = 0; kk < ck / 16; ++kk)
-              mma_bf16(acc, smem_desc_kmajor(a_base + kk * 32, swz),
-                       smem_desc_kmajor(b_base + kk * 32, swz), idesc,
-                       (t > 0 || kk > 0) ? 1u : 0u);
+          const uint64_t row_desc = st_desc + (uint32_t)kh * kh_step;
+          for (int kk = 0; kk < ck / 16; ++kk) {
+#pragma unroll
+            for (int kw = 0; kw < 3; ++kw) {
+              const int t = kh * 3 + kw;
+              // partial kw (nsplit = 3) starts at its first kernel row; a single accumulator at
+              // the first tap
+              const bool first = kk == 0 && (nsplit == 3 ? kh == 0 : t == 0);
+              mma_bf16(acc + (nsplit == 3 ? (uint32_t)(kw * np) : 0u),
+                       row_desc + (uint32_t)kw * kw_step + (uint32_t)(2 * kk),
+                       b_desc0 + (uint32_t)t * tap_step + (uint32_t)(2 * kk), idesc,
+                       first ? 0u : 1u);
+            }
           }
         }
-        mma_commit(&empty[sl]);
+        // strip form: the epilogue releases the stage once it sees the tile's accumulator (one
+        // commit per tile); per kernel row: the stage is released as soon as its MMAs complete
+        if (!a.strip) mma_commit(&empty[sl]);
       }
       if (ok) mma_commit(&acc_full[ab]);
     }
@@ -1361,15 +1381,18 @@ __global__ void __launch_bounds__(cv::THREADS, 1) conv_tc_kernel(const __grid_co
       fi ^= 1;
       return okw;
     };
-    // per-channel BatchNorm statistics of this CTA's output pixels (forward convolutions):
-    // lanes 2 j, 2 j + 1 of warp 4 keep channel 16 ci + j's running count, mean and M2
+    // per-channel BatchNorm statistics of the output pixels (forward convolutions), per
+    // epilogue warp: lanes 2 j, 2 j + 1 keep channel 16 ci + j's running count, mean and M2 over
+    // the warp's 32 rows of every tile
     const bool with_stats = a.stats != nullptr;
     float run_n = 0.f, run_mu[4] = {0.f, 0.f, 0.f, 0.f}, run_m2[4] = {0.f, 0.f, 0.f, 0.f};
     int i = 0;
     for (int tile = blockIdx.x; tile < tiles; tile += cpr, ++i) {
-      const int ab = i & 1;
-      if (!epi_wait(&acc_full[ab], (i >> 1) & 1)) break;
+      const int ab = i % nacc;
+      if (!epi_wait(&acc_full[ab], (i / nacc) & 1)) break;
       asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+      // strip form: this tile's MMAs (and so its reads of its input stage) are complete
+      if (a.strip && leader) mbar_arrive(&empty[i % nst]);
       int64_t dst = (int64_t)tile * BM + r;
       if (a.dst_h > 0) {
         const int pp = tile * BM + r, img = pp / per_img, rem = pp - img * per_img;
@@ -1382,7 +1405,18 @@ __global__ void __launch_bounds__(cv::THREADS, 1) conv_tc_kernel(const __grid_co
         const int c0 = 16 * ci;
         if (c0 >= a.N) break;
         float v[16];
-        tmem_ld16(tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(ab * np + c0), v);
+        const uint32_t tl = tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)ab * acc_cols + c0;
+        tmem_ld16(tl, v);
+        if (nsplit == 3) {
+          // the three column partials, added in column order
+#pragma unroll
+          for (int kw = 1; kw < 3; ++kw) {
+            float u[16];
+            tmem_ld16(tl + (uint32_t)(kw * np), u);
+#pragma unroll
+            for (int j = 0; j < 16; ++j) v[j] += u[j];
+          }
+        }
         if (a.st32) {
           // whole 32-byte sectors per lane and instruction
 #pragma unroll
@@ -1399,43 +1433,35 @@ __global__ void __launch_bounds__(cv::THREADS, 1) conv_tc_kernel(const __grid_co
                 make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
         }
         if (with_stats) {
-          // the tile's 128 pixels: mean, then the sum of squared deviations from it (two
-          // passes over the registers), each summed over the warp and then the four warps
+          // this warp's 32 pixels of the tile: mean, then the sum of squared deviations from
+          // it (two passes over the registers), each summed over the warp's lanes
           float t[16];
 #pragma unroll
           for (int j = 0; j < 16; ++j) t[j] = v[j];
-          const float ws = warp_colsum16(t, lane);
-          if (!(lane & 1)) red[quarter * 16 + (lane >> 1)] = ws;
-          asm volatile("bar.sync 1, 128;" ::: "memory");
-          const int ch = lane >> 1;
-          const float mt = (((red[ch] + red[16 + ch]) + red[32 + ch]) + red[48 + ch]) * (1.f / BM);
+          const float mt = warp_colsum16(t, lane) * (1.f / 32);
 #pragma unroll
           for (int j = 0; j < 16; ++j) {
             const float e = v[j] - __shfl_sync(0xffffffffu, mt, 2 * j);
             t[j] = e * e;
           }
-          const float wq = warp_colsum16(t, lane);
-          if (!(lane & 1)) red[64 + quarter * 16 + (lane >> 1)] = wq;
-          asm volatile("bar.sync 1, 128;" ::: "memory");
-          if (quarter == 0) {
-            // Chan et al.'s combination of the running (n, mean, M2) with this tile's
-            const float m2t = ((red[64 + ch] + red[80 + ch]) + red[96 + ch]) + red[112 + ch];
-            const float nt = run_n + (float)BM, f = (float)BM / nt, delta = mt - run_mu[ci];
-            run_mu[ci] = fmaf(delta, f, run_mu[ci]);
-            run_m2[ci] = run_m2[ci] + m2t + delta * delta * run_n * f;
-          }
+          const float m2t = warp_colsum16(t, lane);
+          // Chan et al.'s combination of the running (n, mean, M2) with these 32 pixels'
+          const float nt = run_n + 32.f, f = 32.f / nt, delta = mt - run_mu[ci];
+          run_mu[ci] = fmaf(delta, f, run_mu[ci]);
+          run_m2[ci] = run_m2[ci] + m2t + delta * delta * run_n * f;
         }
       }
-      if (with_stats) run_n += (float)BM;
+      if (with_stats) run_n += 32.f;
       asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
       asm volatile("bar.sync 1, 128;" ::: "memory");
       if (leader) mbar_arrive(&acc_empty[ab]);
     }
-    if (with_stats && quarter == 0 && !(lane & 1)) {
+    if (with_stats && !(lane & 1)) {
+      // one partial per epilogue warp: stats[g][4 q + quarter]
 #pragma unroll
       for (int ci = 0; ci < 4; ++ci) {
         if (16 * ci >= a.N) break;
-        a.stats[((int64_t)g * cpr + blockIdx.x) * a.N + 16 * ci + (lane >> 1)] =
+        a.stats[((int64_t)g * cpr * 4 + 4 * blockIdx.x + quarter) * a.N + 16 * ci + (lane >> 1)] =
             make_float4(run_n, run_mu[ci], run_m2[ci], 0.f);
       }
     }
@@ -1560,6 +1586,9 @@ __global__ void __launch_bounds__(cw::THREADS, 1) conv_wgrad_tc_kernel(
   } else if (warp == 1 && lane == 0) {
     // ---------------- MMA issuer ----------------
     const uint32_t idesc = make_idesc(BM, 64, true, true);
+    // descriptors of A0 and I0; a buffer / m-tile / K-step adds its byte offset / 16
+    const uint64_t a_desc0 = smem_desc(smem_u32(A0), 8192, 1024);
+    const uint64_t b_desc0 = smem_desc(smem_u32(I0), 8192, 1024);
     bool ok = true;
     for (int j = 0; j < nblk; ++j) {
       const int s = j % ni, sa = j % na;
@@ -1568,12 +1597,13 @@ __global__ void __launch_bounds__(cw::THREADS, 1) conv_wgrad_tc_kernel(
         break;
       }
       asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-      const uint32_t ab = smem_u32(A0 + sa * a_bytes), bb = smem_u32(I0 + s * in_pitch);
+      const uint64_t ad = a_desc0 + ((uint32_t)sa * a_bytes >> 4);
+      const uint64_t bd = b_desc0 + ((uint32_t)s * in_pitch >> 4);
       for (int mt = 0; mt < mt_n; ++mt)
 #pragma unroll
         for (int kk = 0; kk < cw::KB / 16; ++kk)
-          mma_bf16(tmem + (uint32_t)(mt * 64), smem_desc(ab + mt * cw::kTileA + kk * 2048, 8192, 1024),
-                   smem_desc(bb + kk * 2048, 8192, 1024), idesc, (j > 0 || kk > 0) ? 1u : 0u);
+          mma_bf16(tmem + (uint32_t)(mt * 64), ad + (uint32_t)(mt * (cw::kTileA >> 4) + kk * 128),
+                   bd + (uint32_t)(kk * 128), idesc, (j > 0 || kk > 0) ? 1u : 0u);
       mma_commit(&afree[sa]);    // A buffer reusable once these MMAs have read it
       mma_commit(&empty_in[s]);  // and the output-gradient tile
     }
@@ -1859,7 +1889,20 @@ cudaError_t launch_conv_tc(const ConvArgs& a, cudaStream_t stream, int* ctas_per
   // per tile
   const int tiles = a.P / BM;
   const int cpr = std::max(1, std::min(tiles, per_sm * sms / a.G));
-  if (ctas_per_replica) *ctas_per_replica = cpr;
+  // accumulators (measured in the ResNet-20 step): four buffers of three column partials where
+  // the CTAs on one SM fit in its 512 TMEM columns (16 channels); else four single buffers where
+  // they fit (32 channels, two CTAs per SM), else two buffers of three partials (64 channels)
+  if (conv_tmem_cols(12, a.np) * per_sm <= 512) {
+    la.nacc = 4;
+    la.nsplit = 3;
+  } else if (conv_tmem_cols(4, a.np) * per_sm <= 512 && per_sm > 1) {
+    la.nacc = 4;
+    la.nsplit = 1;
+  } else {
+    la.nacc = 2;
+    la.nsplit = conv_tmem_cols(6, a.np) * per_sm <= 512 ? 3 : 1;
+  }
+  if (ctas_per_replica) *ctas_per_replica = 4 * cpr;  // statistics partials: one per epilogue warp
   return launch_pdl(conv_tc_kernel, dim3(cpr, a.G), dim3(cv::THREADS), smem, stream, la);
 }
 

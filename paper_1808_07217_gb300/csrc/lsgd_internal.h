@@ -170,17 +170,25 @@ struct ConvArgs {
   // (image, 2 y + ph_y, 2 x + ph_x) of a dst_h x dst_w grid (one parity phase of a stride-2
   // convolution's data gradient); else to pixel (image, y, x)
   int ph_y, ph_x, dst_h, dst_w;
-  // non-null (only with dst_h = 0): per-CTA BatchNorm statistics of the output, stats[g][q][n] =
-  // (count, mean, sum of squared deviations, 0) over CTA q's pixels, q < the CTAs per replica
+  // non-null (only with dst_h = 0): partial BatchNorm statistics of the output, stats[g][q][n] =
+  // (count, mean, sum of squared deviations, 0) over the pixels of epilogue warp q % 4 of CTA q / 4
   float4* stats;
   int strip;  // stage form: 1 = strip (in_map made with strip = true), 0 = per kernel row
   int st32;   // out 32-byte aligned: 256-bit stores (set by the launcher)
+  int nacc, nsplit;  // accumulator buffers and column partials per tile (set by the launcher)
 };
+// TMEM columns of the convolution kernel for n accumulators (buffers x partials) of np columns: a
+// power of two >= 32.
+__host__ __device__ inline uint32_t conv_tmem_cols(int n, int np) {
+  uint32_t c = 32;
+  while (c < (uint32_t)(n * np)) c <<= 1;
+  return c;
+}
 // Stride 1 and tiles of whole image rows with a width that is a multiple of 8: the convolution's
 // input boxes carry one halo row above and below (make_tma_map_conv) and one stage feeds all nine
 // taps of a tile.
 bool conv_strip_ok(int hout, int wout, int stride);
-// ctas_per_replica (if non-null) receives the launch's CTAs per replica (the stats partials).
+// ctas_per_replica (if non-null) receives the statistics partials per replica (4 per CTA).
 cudaError_t launch_conv_tc(const ConvArgs& a, cudaStream_t stream, int* ctas_per_replica = nullptr);
 // Weight gradient of a 3x3 convolution (zero padding 1, stride 1 or 2) on the tensor cores, the
 // column matrix built in shared memory: part[g][q][co][t Cin + ci] = the sum over CTA q's 64-pixel

@@ -471,27 +471,42 @@ __global__ void bn_act_fwd_kernel(const float* __restrict__ y, const float* __re
   }
 }
 
-// The convolution epilogue's per-CTA statistics partials (count, mean, M2) merged in CTA order
-// (Chan et al.): one thread per (replica, channel), partials loaded eight at a time.
+// The convolution epilogue's statistics partials (count, mean, M2; one per epilogue warp and CTA)
+// merged by Chan et al.'s formula: one warp per (replica, channel); lane l merges partials l,
+// l + 32, ... in order, then the fixed butterfly of bn_stats_finalize_kernel combines the lanes.
 __global__ void bn_merge_partials_kernel(const float4* __restrict__ stats, int nparts, int G, int C,
                                          float* __restrict__ mean, float* __restrict__ rstd) {
   pdl_begin();
-  const int t = blockIdx.x * blockDim.x + threadIdx.x;
-  if (t >= G * C) return;
-  const int g = t / C, c = t % C;
+  const int wid = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
+  if (wid >= G * C) return;
+  const int g = wid / C, c = wid % C;
   const float4* src = stats + (int64_t)g * nparts * C + c;
-  float n = 0.f, m = 0.f, M2 = 0.f;
-  for (int q0 = 0; q0 < nparts; q0 += 8) {
-    float4 v[8];
-#pragma unroll
-    for (int j = 0; j < 8; ++j)
-      if (q0 + j < nparts) v[j] = __ldg(src + (int64_t)(q0 + j) * C);
-#pragma unroll
-    for (int j = 0; j < 8; ++j)
-      if (q0 + j < nparts) chan_merge(n, m, M2, v[j].x, v[j].y, v[j].z);
+  float n = 0.f, mu = 0.f, M2 = 0.f;
+  for (int q = lane; q < nparts; q += 32) {
+    const float4 v = __ldg(src + (int64_t)q * C);
+    chan_merge(n, mu, M2, v.x, v.y, v.z);
   }
-  mean[t] = m;
-  rstd[t] = 1.0f / sqrtf(M2 / n + kBnEps);
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const float n2 = __shfl_xor_sync(0xffffffffu, n, o);
+    const float m2 = __shfl_xor_sync(0xffffffffu, mu, o);
+    const float M22 = __shfl_xor_sync(0xffffffffu, M2, o);
+    // both partners combine (lower lane first) so they hold bit-identical results
+    float na = n, ma = mu, Ma = M2;
+    float nb = n2, mb = m2, Mb = M22;
+    if (lane & o) {
+      na = n2; ma = m2; Ma = M22;
+      nb = n; mb = mu; Mb = M2;
+    }
+    chan_merge(na, ma, Ma, nb, mb, Mb);
+    n = na;
+    mu = ma;
+    M2 = Ma;
+  }
+  if (lane == 0) {
+    mean[wid] = mu;
+    rstd[wid] = 1.0f / sqrtf(M2 / n + kBnEps);
+  }
 }
 
 // The same with a fixed group of 4 channels per thread (C / 4 dividing the block size): the
@@ -1138,8 +1153,8 @@ struct ResNetPlan {
   uint16_t* wstem = nullptr;  // [K][Cout][9][16]
   // the stride-2 data gradients as four parity phases on the implicit kernel: their weights
   uint16_t* wt4 = nullptr;    // [4][K][Cin][9][Cout] of the largest such convolution
-  // BatchNorm statistics computed by the forward convolutions' epilogues: per replica and CTA,
-  // (count, mean, M2) of each channel, merged by bn_merge_partials_kernel
+  // BatchNorm statistics computed by the forward convolutions' epilogues: per replica, CTA and
+  // epilogue warp, (count, mean, M2) of each channel, merged by bn_merge_partials_kernel
   float4* cstats = nullptr;   // [K + 2 SMs][64]
   std::string err;
 };
@@ -1392,7 +1407,7 @@ lsgd_status conv_dgrad_tc(const uint16_t* dy, const uint16_t* w, int64_t w_gs, f
 }
 
 // stats / nparts: where the persistent implicit kernel runs, it also writes the output's
-// per-CTA BatchNorm statistics to stats and their count per replica to *nparts (else 0).
+// partial BatchNorm statistics to stats and their count per replica to *nparts (else 0).
 template <typename TA>
 lsgd_status conv_forward(ResNetPlan* p, int i, const void* in, const void* Wop, int w_g0,
                          int w_gmul, float* y, int G, cudaStream_t s, int64_t* launches,
@@ -1531,7 +1546,7 @@ lsgd_status forward_impl(ResNetPlan* p, const float* W, const void* Wop, int w_g
     // block j uses convolutions 2j+1 (input act[2j], the block input) and 2j+2 (input act[2j+1])
     const void* in = i == 0 ? p->x0 : p->act[i - 1];
     // the convolution's epilogue forms the BatchNorm statistics where it can (one small kernel
-    // merges its per-CTA partials), else the two statistics passes run
+    // merges its partials), else the two statistics passes run
     int nparts = 0;
     float4* cst = p->cstats && vec4_ok(c.cout) && c.cout <= 64 ? p->cstats : nullptr;
     lsgd_status st = conv_forward<TA>(p, (int)i, in, Wop, w_g0, w_gmul, p->y[i], G, s, launches,
@@ -1541,8 +1556,8 @@ lsgd_status forward_impl(ResNetPlan* p, const float* W, const void* Wop, int w_g
       st = bn_stats(p, c, p->y[i], p->mean[i], p->rstd[i], G, s, launches);
       if (st != LSGD_OK) return st;
     } else {
-      RN_LAUNCH((launch_pdl(bn_merge_partials_kernel, (G * c.cout + 127) / 128, 128, 0, s, cst,
-          nparts, G, c.cout, p->mean[i], p->rstd[i])));
+      RN_LAUNCH((launch_pdl(bn_merge_partials_kernel, (G * c.cout * 32 + 127) / 128, 128, 0, s,
+          cst, nparts, G, c.cout, p->mean[i], p->rstd[i])));
     }
     const bool second = i > 0 && i % 2 == 0;
     const TA* sc = second ? reinterpret_cast<const TA*>(p->act[i - 2]) : nullptr;
@@ -1940,7 +1955,7 @@ size_t conv3x3_bn_scratch_bytes(int G, int B, int hin, int win, int cin, int cou
     sms = kNumSMs;
   }
   const size_t conv = (conv3x3_scratch_bytes(0, G, B, hin, win, cin, cout, stride) + 15) / 16 * 16;
-  return conv + (size_t)(G + 2 * sms) * cout * sizeof(float4);
+  return conv + (size_t)4 * (G + 2 * sms) * cout * sizeof(float4);
 }
 
 lsgd_status conv3x3_bn_bf16(const uint16_t* in, const uint16_t* w, float* y, float* mean,
@@ -1962,8 +1977,8 @@ lsgd_status conv3x3_bn_bf16(const uint16_t* in, const uint16_t* w, float* y, flo
                                x16 ? x16 + conv_x16_elems(G, B, hin, win) : nullptr, s, e,
                                &launches, stats, &nparts);
   if (st == LSGD_OK) {
-    launch_pdl(bn_merge_partials_kernel, (G * cout + 127) / 128, 128, 0, s, stats, nparts, G, cout,
-               mean, rstd);
+    launch_pdl(bn_merge_partials_kernel, (G * cout * 32 + 127) / 128, 128, 0, s, stats, nparts, G,
+               cout, mean, rstd);
     const cudaError_t ce = cudaGetLastError();
     if (ce != cudaSuccess) {
       e = std::string("statistics merge: ") + cudaGetErrorString(ce);
@@ -2227,12 +2242,13 @@ lsgd_status resnet_alloc(ResNetPlan* p, const std::function<void*(size_t)>& allo
   p->dy = alloc((size_t)p->max_act * e);
   p->s12 = (float*)alloc((size_t)K * 2 * 64 * 4);
   if (p->tc) {
-    // at most max(K, 2 SMs) CTAs over all replicas (launch_conv_tc), 64 channels each
+    // at most max(K, 2 SMs) CTAs over all replicas (launch_conv_tc), four partials of 64
+    // channels each
     int dev = 0, sms = kNumSMs;
     if (cudaGetDevice(&dev) != cudaSuccess ||
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
       return LSGD_ECUDA;
-    p->cstats = (float4*)alloc((size_t)(K + 2 * sms) * 64 * sizeof(float4));
+    p->cstats = (float4*)alloc((size_t)4 * (K + 2 * sms) * 64 * sizeof(float4));
     if (!p->cstats) return LSGD_ENOMEM;
   }
   if (!p->x0 || !p->part || !p->feat || !p->dfeat || !p->logits || !p->dlogits || !p->dA[0] ||

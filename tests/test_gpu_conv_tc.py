@@ -199,8 +199,9 @@ BN_SHAPES = [  # (G, B, Hin, Win, Cin, Cout, stride): forward convolutions of Re
 @pytest.mark.parametrize("shape", BN_SHAPES)
 def test_conv_epilogue_batchnorm_statistics(P, shape):
     # Sec. A.4's per-worker batch statistics of the convolution output, formed by the epilogue
-    # (per-tile two-pass moments combined by Chan et al.'s formula), against fp64 moments of the
-    # same fp32 output; the output itself must be the plain forward's, bit for bit
+    # (two-pass moments of each warp's 32 rows per tile, combined by Chan et al.'s formula),
+    # against fp64 moments of the same fp32 output; the output itself must be the plain
+    # forward's, bit for bit
     import torch
 
     G, B, Hin, Win, Cin, Cout, s = shape

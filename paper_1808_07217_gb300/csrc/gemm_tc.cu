@@ -741,6 +741,7 @@ constexpr int TN = 128;                     // tile columns (= rows: BM)
 constexpr int CW = 32;                      // chunk columns (fp32: one 128-byte row)
 constexpr int ST = 2;                       // operand stages
 constexpr int NS = 4;                       // w / u chunk slots
+constexpr int SD = 2;                       // chunks whose TMA stores may be in flight (<= NS)
 constexpr int EPI_WARPS = 16;               // four per TMEM lane quarter
 constexpr int THREADS = 128 + 32 * EPI_WARPS;
 constexpr int EPI0 = 128;                   // first epilogue thread
@@ -836,12 +837,17 @@ __global__ void __launch_bounds__(wu::THREADS, 1) wgrad_update_kernel(
   WuSmem& sm = *reinterpret_cast<WuSmem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                           ~uintptr_t(1023));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  // tiles of layer 0 come first, then those of layer 1 (operand layouts are the same in both)
-  const int tn0 = (args.L[0].N + wu::TN - 1) / wu::TN, tm0 = (args.L[0].M + BM - 1) / BM;
+  // the layers' tiles one layer after another (operand layouts are the same in all): layer l's
+  // tiles follow uc_l tile positions (uc_l G tiles) of the layers before it (scalars, so that
+  // nothing needs local memory)
+  static_assert(kWgradMaxLayers == 3, "the bookkeeping below names three layers");
+  const int tn0 = (args.L[0].N + wu::TN - 1) / wu::TN;
   const int tn1 = args.nl > 1 ? (args.L[1].N + wu::TN - 1) / wu::TN : 0;
-  const int tm1 = args.nl > 1 ? (args.L[1].M + BM - 1) / BM : 0;
-  const int tiles0 = tn0 * tm0 * args.G;
-  const int tiles = tiles0 + tn1 * tm1 * args.G;
+  const int tn2 = args.nl > 2 ? (args.L[2].N + wu::TN - 1) / wu::TN : 0;
+  const int uc1 = tn0 * ((args.L[0].M + BM - 1) / BM);
+  const int uc2 = uc1 + (args.nl > 1 ? tn1 * ((args.L[1].M + BM - 1) / BM) : 0);
+  const int uc3 = uc2 + (args.nl > 2 ? tn2 * ((args.L[2].M + BM - 1) / BM) : 0);
+  const int tiles = uc3 * args.G;
   const int nk = (args.Kd + BK - 1) / BK;
   const bool a_mn = args.L[0].A.mn_major, b_mn = args.L[0].B.mn_major;
   const bool has_u = args.sgd.u != nullptr;
@@ -852,8 +858,7 @@ __global__ void __launch_bounds__(wu::THREADS, 1) wgrad_update_kernel(
   // whenever every replica reads replica 0's parameters (w_rep0): then replica 0's tile comes
   // last, so that no replica reads it after it has been updated.
   const bool by_unit = avg || args.w_rep0;
-  const int units0 = by_unit ? tn0 * tm0 : tiles0;
-  const int units = by_unit ? units0 + tn1 * tm1 : tiles;
+  const int units = by_unit ? uc3 : tiles;
   const int per_unit = by_unit ? args.G : 1;
   const int my_count =
       (int)blockIdx.x < units ? ((units - 1 - (int)blockIdx.x) / (int)gridDim.x + 1) * per_unit : 0;
@@ -889,16 +894,25 @@ __global__ void __launch_bounds__(wu::THREADS, 1) wgrad_update_kernel(
   const uint32_t tmem = sm.tmem_base;
   pdl_begin();  // everything above touched only shared memory and TMEM
 
+  // tile position x (< uc3) -> its layer l, the position within the layer and the layer's
+  // column-tile count
+  auto locate = [&](int x, int& l, int& r, int& tnl) {
+    l = (x >= uc1 ? 1 : 0) + (x >= uc2 ? 1 : 0);
+    r = x - (l == 0 ? 0 : (l == 1 ? uc1 : uc2));
+    tnl = l == 0 ? tn0 : (l == 1 ? tn1 : tn2);
+  };
   auto tile_coords = [&](int t, const WgradUpdateLayer*& ly, int& g, int& m0, int& n0) {
-    const bool second = t >= tiles0;
-    ly = second ? &args.L[1] : &args.L[0];
-    const int tiles_n = second ? tn1 : tn0, tiles_m = second ? tm1 : tm0;
-    if (second) t -= tiles0;
-    const int per_g = tiles_m * tiles_n;
+    // layer by layer, each layer's tiles replica by replica
+    const int l0 = (t >= uc1 * args.G ? 1 : 0) + (t >= uc2 * args.G ? 1 : 0);
+    const int base = l0 == 0 ? 0 : (l0 == 1 ? uc1 : uc2);
+    const int per_g = (l0 == 0 ? uc1 : (l0 == 1 ? uc2 : uc3)) - base;
+    t -= base * args.G;
     g = t / per_g;
-    const int r = t % per_g;
-    m0 = (r / tiles_n) * BM;
-    n0 = (r % tiles_n) * wu::TN;
+    int l, r, tnl;
+    locate(base + t % per_g, l, r, tnl);
+    ly = &args.L[l];
+    m0 = (r / tnl) * BM;
+    n0 = (r % tnl) * wu::TN;
   };
   // the j-th tile of this CTA's sequence; gi = its replica's position within the unit
   auto tile_at = [&](int j, const WgradUpdateLayer*& ly, int& g, int& m0, int& n0, int& gi) {
@@ -908,12 +922,11 @@ __global__ void __launch_bounds__(wu::THREADS, 1) wgrad_update_kernel(
       tile_coords(u, ly, g, m0, n0);
       return;
     }
-    const bool second = u >= units0;
-    ly = second ? &args.L[1] : &args.L[0];
-    const int tiles_n = second ? tn1 : tn0;
-    const int r = second ? u - units0 : u;
-    m0 = (r / tiles_n) * BM;
-    n0 = (r % tiles_n) * wu::TN;
+    int l, r, tnl;
+    locate(u, l, r, tnl);
+    ly = &args.L[l];
+    m0 = (r / tnl) * BM;
+    n0 = (r % tnl) * wu::TN;
     // averaging: replicas in order (the average's summation order); else replica 0 last
     g = avg ? gi : (gi + 1) % args.G;
   };
@@ -1043,11 +1056,15 @@ __global__ void __launch_bounds__(wu::THREADS, 1) wgrad_update_kernel(
           if (args.sgd.wb) tma_store_3d(&ly->wbmap, sm.wb[sl], x, m0, 0);
         }
         asm volatile("cp.async.bulk.commit_group;" ::: "memory");
-        asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
-        mbar_arrive(&sm.wu_empty[sl]);  // the stores have read the slot
+        // SD chunks' store groups in flight: once at most SD - 1 are still reading shared
+        // memory, the oldest one's slot goes back to the w / u producer
+        asm volatile("cp.async.bulk.wait_group.read %0;" ::"n"(wu::SD - 1) : "memory");
+        if (q >= wu::SD - 1) mbar_arrive(&sm.wu_empty[(q - (wu::SD - 1)) % wu::NS]);
       }
     }
     asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+    // the last SD - 1 chunks' slots (their stores have now completed)
+    for (int j = (q > wu::SD - 1 ? q - (wu::SD - 1) : 0); j < q; ++j) mbar_arrive(&sm.wu_empty[j % wu::NS]);
   } else if (warp >= 4) {
     // ---------------- epilogue ----------------
     const bool leader = threadIdx.x == wu::EPI0;
@@ -1907,6 +1924,7 @@ cudaError_t launch_conv_tc(const ConvArgs& a, cudaStream_t stream, int* ctas_per
 }
 
 cudaError_t launch_wgrad_update(const WgradUpdateArgs& a, cudaStream_t stream) {
+  static_assert(sizeof(WgradUpdateArgs) <= 4096, "kernel parameter size");
   if (a.nl < 1 || a.nl > kWgradMaxLayers) return cudaErrorInvalidValue;
   if (a.G <= 0) return cudaSuccess;
   if (a.Kd <= 0 || !a.sgd.w || (a.sgd.mom != 0.f && !a.sgd.u)) return cudaErrorInvalidValue;

@@ -276,10 +276,10 @@ struct WgradUpdateLayer {
   TcOperand A, B;
   CUtensorMap wmap, umap, wbmap;
 };
-// Up to kWgradMaxLayers layers share one persistent launch (their tiles form one list, layer 0's
-// first).  All layers have the same contraction length Kd (= B_loc), replica count G and update
+// Up to kWgradMaxLayers layers share one persistent launch (their tiles form one list in layer
+// order).  All layers have the same contraction length Kd (= B_loc), replica count G and update
 // rule; sgd's pointers matter only for being null or not (u: momentum, wb: bf16 shadow).
-constexpr int kWgradMaxLayers = 2;
+constexpr int kWgradMaxLayers = 3;
 struct WgradUpdateArgs {
   int Kd, G, nl;
   WgradUpdateLayer L[kWgradMaxLayers];

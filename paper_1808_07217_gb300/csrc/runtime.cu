@@ -87,7 +87,9 @@ struct lsgd_ctx {
   std::vector<void*> act;  // act[l]: input of dense layer l, [K][B][ld] operand dtype
   float* logits = nullptr;
   int ld_logits = 0;
-  void* dz[2] = {nullptr, nullptr};
+  // output gradients: ping-pong buffers, and a third that keeps the top layer's while the layers
+  // below use the first two (its update joins the last update launch)
+  void* dz[3] = {nullptr, nullptr, nullptr};
   int ld_dz = 0;
   float* loss_hist = nullptr;
   int64_t loss_cap = 0;
@@ -320,6 +322,15 @@ lsgd_status make_tc_maps(lsgd_ctx* c) {
   return LSGD_OK;
 }
 
+// The top layer's fused update joins the last update launch (that of layers 1 and 0) rather than
+// running alone: with three or more layers updated by the weight-gradient kernel and no classifier
+// head.  Its output gradient then stays in dz[2] while the layers below use dz[0] and dz[1], and
+// nothing between its own backward and that launch reads its weights (the layers below read only
+// theirs), so the result is the same.
+bool defer_top_update(const lsgd_ctx* c) {
+  return c->fused && !c->head && c->layers.size() >= 3;
+}
+
 lsgd_status alloc_dense(lsgd_ctx* c) {
   const int K = c->cfg.K, B = c->cfg.B_loc;
   const size_t esz = c->bf16 ? 2 : 4;
@@ -485,6 +496,12 @@ lsgd_status dense_backward(lsgd_ctx* c, bool avg) {
   int l_top = L - 1;
   int bias_done = -1;  // layer whose bias the last data-gradient GEMM already handled
   lsgd::WgradUpdateArgs wa{};  // fused weight-gradient + update layers not yet launched
+  // the top layer's update waits for the last update launch (defer_top_update); its output
+  // gradient stays in dz[0] and the layers below alternate between dz[1] and dz[2]
+  const bool defer_top = defer_top_update(c) && c->dz[2] != nullptr;
+  lsgd::WgradUpdateLayer top_layer{};
+  bool top_pending = false;
+  auto next_dz = [&](int b) { return defer_top ? (b == 1 ? 2 : 1) : 1 - b; };
   if (c->head) {
     // the last layer's weight / bias gradients and their update (its data gradient for the layer
     // below came with the head's forward kernel)
@@ -513,7 +530,7 @@ lsgd_status dense_backward(lsgd_ctx* c, bool avg) {
     const bool bias_by_dgrad_above = bias_done == l;
     if (l > 0) {
       // data gradient dz_prev[j][i] = (sum_o dz[j][o] W[o][i]) * (act[j][i] > 0)
-      void* dzp = c->dz[1 - cur];
+      void* dzp = c->dz[next_dz(cur)];
       if (Ly.tc) {
         lsgd::TcGemmArgs t{};
         t.M = B;
@@ -619,10 +636,18 @@ lsgd_status dense_backward(lsgd_ctx* c, bool avg) {
         if (!mok) return fail(c, LSGD_ECUDA, "TMA map encoding failed (fused update)");
         if (wa.nl == 0) wa.sgd = sp;
         ++wa.nl;
-        // Layer 1's update waits for layer 0's, so both go in one launch: nothing in between
-        // writes the gradients they read (layer 0 has no data gradient) or reads the parameters
-        // they change.
-        if (!(l == 1 && c->layers[0].tc)) {
+        if (defer_top && l == L - 1) {
+          top_layer = wa.L[0];
+          top_pending = true;
+          wa.nl = 0;
+        } else if (!(l == 1 && c->layers[0].tc)) {
+          // Layer 1's update waits for layer 0's, so both go in one launch: nothing in between
+          // writes the gradients they read (layer 0 has no data gradient) or reads the parameters
+          // they change; a deferred top layer joins them last.
+          if (top_pending && l == 0) {
+            wa.L[wa.nl++] = top_layer;
+            top_pending = false;
+          }
           wa.Kd = B;
           wa.G = K;
           wa.avg = avg ? 1 : 0;
@@ -673,8 +698,9 @@ lsgd_status dense_backward(lsgd_ctx* c, bool avg) {
                                            c->d_pad, c->stream));
       span(LSGD_PH_BACKWARD);
     }
-    if (l > 0) cur = 1 - cur;
+    if (l > 0) cur = next_dz(cur);
   }
+  if (top_pending) return fail(c, LSGD_ESTATE, "deferred top-layer update was not launched");
   return LSGD_OK;
 }
 
@@ -948,6 +974,13 @@ lsgd_status lsgd_create(const lsgd_config* cfg, const lsgd_allocator* alloc, voi
     if (st == LSGD_OK) {
       const DenseLayer& top = c->layers.back();
       c->head = c->bf16 && !c->lsq && top.tc && lsgd::head_supported(top.out, c0.B_loc, top.in);
+      if (defer_top_update(c)) {
+        c->dz[2] = dalloc(c, (size_t)c0.K * c0.B_loc * c->ld_dz * 2);
+        if (!c->dz[2]) {
+          fail(nullptr, LSGD_ENOMEM, "gradient buffer allocation failed");
+          return bail(LSGD_ENOMEM);
+        }
+      }
       // segments averaged outside the weight-gradient + update launches: every bias, and the
       // classifier head's weights when its own kernels update them (each tensor starts at a
       // 64-element boundary, so a length rounded up to 4 stays inside its padding)

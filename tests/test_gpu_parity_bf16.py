@@ -133,11 +133,13 @@ def test_full_size_mlp_sampled_replicas(P):
 
 @pytest.mark.parametrize("mom,nest,wd", [(0.9, True, 5e-4), (0.9, False, 0.0), (0.0, False, 1e-4)])
 @pytest.mark.parametrize("widths,K,B", [((264, 136, 72, 10), 3, 40), ((3072, 1024, 1024, 10), 4, 128),
-                                        ((200, 136, 96, 72, 10), 2, 24)])
+                                        ((200, 136, 96, 72, 10), 2, 24), ((264, 136, 72, 40), 3, 40),
+                                        ((200, 136, 96, 72, 40), 2, 24)])
 def test_fused_update_is_bitwise_identical(P, mom, nest, wd, widths, K, B):
     # The update applied in the weight-gradient epilogue uses the same arithmetic as the
     # stand-alone update kernel, so parameters, momentum and losses agree bit for bit.  (The
-    # first two layers' updates share one launch; with four layers the third has its own.)
+    # first two layers' updates share one launch; with four layers the third has its own; with
+    # 40 classes there is no classifier head and the top layer's update joins the last launch.)
     N = 2048
     X, y = synthdata.gaussian_mixture(N, widths[0], widths[-1], seed=4)
     res = []
@@ -251,6 +253,7 @@ def test_hierarchical_local_sgd(P):
 @pytest.mark.parametrize("mom,nest,wd", [(0.9, True, 5e-4), (0.9, False, 0.0), (0.0, False, 1e-4)])
 @pytest.mark.parametrize("widths,K,B", [((264, 136, 72, 10), 3, 40),
                                         ((200, 136, 96, 72, 100), 4, 24),
+                                        ((264, 136, 72, 40), 3, 40),
                                         ((3072, 1024, 1024, 10), 16, 128)])
 def test_average_in_update_launches_is_bitwise_identical(P, mom, nest, wd, widths, K, B):
     # lsgd_run forms the K-way average of a round-ending step inside that step's weight-gradient

@@ -142,47 +142,58 @@ __global__ void gather_rows_kernel(void* __restrict__ dst, int ld_dst, const flo
 }
 
 // ---------------------------------------------------------------------------------------------
-// Softmax cross-entropy: one CTA per group (replica), one thread per row, so every row of the
-// group is in flight at once.  Row losses are combined by a fixed-shape tree in shared memory
-// (deterministic).
+// Softmax cross-entropy: one CTA per group (replica), one warp per row (rows w, w + warps, ...):
+// the lanes take classes lane, lane + 32, ... (coalesced loads and stores), the row's maximum and
+// sum of exponentials are combined across lanes by a fixed butterfly, and the row losses by a
+// fixed-shape tree in shared memory (deterministic).
 template <typename TD>
-__global__ void __launch_bounds__(256) softmax_xent_kernel(
+__global__ void __launch_bounds__(1024) softmax_xent_kernel(
     const float* __restrict__ logits, int ld, int C, const int32_t* __restrict__ labels, int B,
     TD* __restrict__ dz, int ld_dz, float* __restrict__ loss_mean, float* __restrict__ loss_sum,
     float* __restrict__ row_out) {
   pdl_begin();
-  __shared__ float red[256];
-  const int g = blockIdx.x;
+  extern __shared__ float row_loss[];  // [B]
+  const int g = blockIdx.x, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int nw = blockDim.x >> 5;
   const float inv_b = 1.0f / (float)B;
-  float acc = 0.f;
-  for (int j = threadIdx.x; j < B; j += blockDim.x) {
+  for (int j = warp; j < B; j += nw) {
     const float* z = logits + ((int64_t)g * B + j) * ld;
     float mx = -INFINITY;
-    for (int c = 0; c < C; ++c) mx = fmaxf(mx, z[c]);
+    for (int c = lane; c < C; c += 32) mx = fmaxf(mx, z[c]);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
     float se = 0.f;
-    for (int c = 0; c < C; ++c) se += expf(z[c] - mx);
+    for (int c = lane; c < C; c += 32) se += expf(z[c] - mx);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) se += __shfl_xor_sync(0xffffffffu, se, o);
     const float lse = mx + logf(se);
     const int y = labels[(int64_t)g * B + j];
     if (dz) {
       TD* dzr = dz + ((int64_t)g * B + j) * ld_dz;
-      for (int c = 0; c < C; ++c) {
+      for (int c = lane; c < C; c += 32) {
         const float p = expf(z[c] - lse);
         Elem<TD>::store(dzr + c, (p - (c == y ? 1.f : 0.f)) * inv_b);
       }
     }
-    const float l = lse - z[y];
-    if (row_out) row_out[(int64_t)g * B + j] = l;
-    acc += l;
+    if (lane == 0) {
+      const float l = lse - z[y];
+      if (row_out) row_out[(int64_t)g * B + j] = l;
+      row_loss[j] = l;
+    }
   }
-  red[threadIdx.x] = acc;
   __syncthreads();
-  for (int w = blockDim.x / 2; w > 0; w >>= 1) {
-    if (threadIdx.x < w) red[threadIdx.x] += red[threadIdx.x + w];
+  // sum of the B row losses: a fixed tree over the rows (strides halving from the largest power
+  // of two below B)
+  int span = 1;
+  while (span < B) span <<= 1;
+  for (int st = span >> 1; st > 0; st >>= 1) {
+    for (int j = threadIdx.x; j < st; j += blockDim.x)
+      if (j + st < B) row_loss[j] += row_loss[j + st];
     __syncthreads();
   }
   if (threadIdx.x == 0) {
-    if (loss_mean) loss_mean[g] = red[0] * inv_b;
-    if (loss_sum) loss_sum[g] = red[0];
+    if (loss_mean) loss_mean[g] = row_loss[0] * inv_b;
+    if (loss_sum) loss_sum[g] = row_loss[0];
   }
 }
 
@@ -682,13 +693,15 @@ cudaError_t launch_softmax_xent(const float* logits, int ld, int C, const int32_
                                 float* loss_sum, float* row_loss, cudaStream_t stream) {
   if (G <= 0 || B <= 0) return cudaSuccess;
   if (B > 8192 || C < 1) return cudaErrorInvalidValue;
-  const int threads = B >= 256 ? 256 : (B >= 128 ? 128 : (B >= 64 ? 64 : 32));
+  // one warp per row up to 32 warps; the row losses in shared memory
+  const int threads = 32 * std::min(32, B);
+  const size_t smem = (size_t)B * sizeof(float);
   if (dz_bf16)
-    launch_pdl(softmax_xent_kernel<uint16_t>, G, threads, 0, stream, 
+    launch_pdl(softmax_xent_kernel<uint16_t>, G, threads, smem, stream,
         logits, ld, C, labels, B, reinterpret_cast<uint16_t*>(dz), ld_dz, loss_mean, loss_sum,
         row_loss);
   else
-    launch_pdl(softmax_xent_kernel<float>, G, threads, 0, stream, 
+    launch_pdl(softmax_xent_kernel<float>, G, threads, smem, stream,
         logits, ld, C, labels, B, reinterpret_cast<float*>(dz), ld_dz, loss_mean, loss_sum,
         row_loss);
   return cudaGetLastError();

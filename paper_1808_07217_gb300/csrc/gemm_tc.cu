@@ -505,6 +505,20 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
       mma_commit(&sm.empty[s]);  // stage reusable once these MMAs have read it
     }
     if (ok) mma_commit(&sm.accum);  // accumulator complete
+  } else if (warp >= 2 && args.epi == EPI_MASK && args.mask) {
+    // warps 2-3 idle through the mainloop: they bring the tile's ReLU-mask rows (the stored
+    // activation) into L1, so that the epilogue's mask loads hit L1 instead of waiting on DRAM
+    // (the TMA operand loads bypass L1).  Every line prefetched starts inside the tile.
+    const int esz = args.mask_bf16 ? 2 : 4;
+    const int ncols = min(BN, args.N - n0);
+    const int lines = (ncols * esz + 127) / 128;
+    const int rows = min(BM, args.M - m0);
+    const char* base = reinterpret_cast<const char*>(args.mask) +
+                       ((int64_t)g * args.mask_gs + (int64_t)m0 * args.mask_rs + n0) * esz;
+    for (int t = (int)threadIdx.x - 64; t < rows * lines; t += 64) {
+      const int r = t / lines, l = t % lines;
+      asm volatile("prefetch.global.L1 [%0];" ::"l"(base + (int64_t)r * args.mask_rs * esz + l * 128));
+    }
   }
   __syncwarp();
 

@@ -1247,8 +1247,8 @@ constexpr int MAX_STAGES = 24;  // 4 KB stages (ck = 16)
 constexpr int EPI0 = 128;
 constexpr size_t SMEM_MAX = 227 * 1024;  // dynamic shared memory of one CTA
 constexpr int MAX_ACC = 4;  // accumulator buffers in TMEM
-// barriers, TMEM slot and epilogue flags
-constexpr size_t AUX_BYTES = (2 * MAX_STAGES + 2 * MAX_ACC + 1) * 8 + 16;
+// barriers, TMEM slot, epilogue flags, and the BatchNorm-backward epilogue's mean / rstd (64 each)
+constexpr size_t AUX_BYTES = (2 * MAX_STAGES + 2 * MAX_ACC + 1) * 8 + 16 + 2 * 64 * 4;
 }  // namespace cv
 
 // Sums 16 values per lane over the 32 lanes of a warp in four halving exchanges and one final
@@ -1267,7 +1267,7 @@ __device__ __forceinline__ float warp_colsum16(float (&v)[16], int lane) {
   return v[0] + __shfl_xor_sync(0xffffffffu, v[0], 1);
 }
 
-__global__ void __launch_bounds__(cv::THREADS, 1) conv_tc_kernel(const __grid_constant__ ConvArgs a) {
+__global__ void __launch_bounds__(cv::THREADS, 2) conv_tc_kernel(const __grid_constant__ ConvArgs a) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
@@ -1291,6 +1291,8 @@ __global__ void __launch_bounds__(cv::THREADS, 1) conv_tc_kernel(const __grid_co
   uint64_t* w_full = acc_empty + cv::MAX_ACC;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(w_full + 1);
   int* epi_ok = reinterpret_cast<int*>(tmem_slot + 1);
+  float* bw_mu = reinterpret_cast<float*>(tmem_slot + 4);  // [64]
+  float* bw_rs = bw_mu + 64;                                // [64]
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int g = blockIdx.y, cpr = gridDim.x;
@@ -1417,6 +1419,20 @@ __global__ void __launch_bounds__(cv::THREADS, 1) conv_tc_kernel(const __grid_co
     // the warp's 32 rows of every tile
     const bool with_stats = a.stats != nullptr;
     float run_n = 0.f, run_mu[4] = {0.f, 0.f, 0.f, 0.f}, run_m2[4] = {0.f, 0.f, 0.f, 0.f};
+    // the data gradient's BatchNorm-backward epilogue (a.bwd): that layer's mean and rstd in
+    // shared memory; lanes 2 j, 2 j + 1 keep channel 16 ci + j's running sums of g and g xhat
+    const ConvBwdFuse& bw = a.bwd;
+    const bool with_bwd = bw.y != nullptr;
+    const int dx_h = a.dst_h > 0 ? a.dst_h : a.hout, dx_w = a.dst_w > 0 ? a.dst_w : a.wout;
+    float run_g[4] = {0.f, 0.f, 0.f, 0.f}, run_gx[4] = {0.f, 0.f, 0.f, 0.f};
+    if (with_bwd) {
+      const int et = threadIdx.x - cv::EPI0;
+      if (et < a.N) {
+        bw_mu[et] = bw.mean[g * a.N + et];
+        bw_rs[et] = bw.rstd[g * a.N + et];
+      }
+      asm volatile("bar.sync 1, 128;" ::: "memory");
+    }
     int i = 0;
     for (int tile = blockIdx.x; tile < tiles; tile += cpr, ++i) {
       const int ab = i % nacc;
@@ -1431,6 +1447,41 @@ __global__ void __launch_bounds__(cv::THREADS, 1) conv_tc_kernel(const __grid_co
         dst = ((int64_t)img * a.dst_h + 2 * oy + a.ph_y) * a.dst_w + 2 * ox + a.ph_x;
       }
       float* orow = a.out + (int64_t)g * a.out_gs + dst * a.N;
+      // the shortcut's source pixel in the block output (stride 1: the same pixel; stride 2: the
+      // pixels on the stride grid), or -1
+      auto sc_pixel = [&](int64_t d) -> int64_t {
+        if (!bw.sc_dout) return -1;
+        const int img = (int)(d / ((int64_t)dx_h * dx_w)), rem = (int)(d % ((int64_t)dx_h * dx_w));
+        const int iy = rem / dx_w, ix = rem - iy * dx_w;
+        if (bw.sc_stride == 1) return d;
+        if ((iy & 1) || (ix & 1)) return -1;
+        return ((int64_t)img * (dx_h / 2) + iy / 2) * (dx_w / 2) + ix / 2;
+      };
+      int64_t sc_px = with_bwd ? sc_pixel(dst) : -1;
+      if (with_bwd && tile + cpr < tiles) {
+        // this thread's row of the next tile into L1 while this tile is processed: the loads
+        // below would otherwise each wait on DRAM
+        const int nt = tile + cpr;
+        int64_t nd = (int64_t)nt * BM + r;
+        if (a.dst_h > 0) {
+          const int pp = nt * BM + r, img = pp / per_img, rem = pp - img * per_img;
+          const int oy = rem / a.wout, ox = rem - oy * a.wout;
+          nd = ((int64_t)img * a.dst_h + 2 * oy + a.ph_y) * a.dst_w + 2 * ox + a.ph_x;
+        }
+        const int64_t ne = (int64_t)g * a.out_gs + nd * a.N;
+        for (int b = 0; b < a.N * 2; b += 128)
+          asm volatile("prefetch.global.L1 [%0];" ::"l"(reinterpret_cast<const char*>(bw.mask + ne) + b));
+        for (int b = 0; b < a.N * 4; b += 128)
+          asm volatile("prefetch.global.L1 [%0];" ::"l"(reinterpret_cast<const char*>(bw.y + ne) + b));
+        const int64_t ns = sc_pixel(nd);
+        if (ns >= 0) {
+          const int64_t se = (int64_t)g * bw.sc_gs + ns * bw.sc_C;
+          for (int b = 0; b < a.N * 4; b += 128)
+            asm volatile("prefetch.global.L1 [%0];" ::"l"(reinterpret_cast<const char*>(bw.sc_dout + se) + b));
+          for (int b = 0; b < a.N * 2; b += 128)
+            asm volatile("prefetch.global.L1 [%0];" ::"l"(reinterpret_cast<const char*>(bw.sc_out + se) + b));
+        }
+      }
 #pragma unroll
       for (int ci = 0; ci < 4; ++ci) {
         const int c0 = 16 * ci;
@@ -1447,6 +1498,50 @@ __global__ void __launch_bounds__(cv::THREADS, 1) conv_tc_kernel(const __grid_co
 #pragma unroll
             for (int j = 0; j < 16; ++j) v[j] += u[j];
           }
+        }
+        if (with_bwd) {
+          // dx (+ the shortcut's share) masked by the layer below's ReLU, and that layer's
+          // BatchNorm-backward sums over this warp's rows
+          if (sc_px >= 0) {
+            const float4* sd = reinterpret_cast<const float4*>(
+                bw.sc_dout + (int64_t)g * bw.sc_gs + sc_px * bw.sc_C + c0);
+            const uint4* so = reinterpret_cast<const uint4*>(
+                bw.sc_out + (int64_t)g * bw.sc_gs + sc_px * bw.sc_C + c0);
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+              const uint4 o8 = __ldg(so + h);
+              const float4 d0 = __ldg(sd + 2 * h), d1 = __ldg(sd + 2 * h + 1);
+              const uint32_t ow[4] = {o8.x, o8.y, o8.z, o8.w};
+              const float dd[8] = {d0.x, d0.y, d0.z, d0.w, d1.x, d1.y, d1.z, d1.w};
+#pragma unroll
+              for (int k = 0; k < 8; ++k) {
+                const float o = bf2f((uint16_t)(k & 1 ? ow[k >> 1] >> 16 : ow[k >> 1] & 0xffffu));
+                v[8 * h + k] += o > 0.f ? dd[k] : 0.f;
+              }
+            }
+          }
+          const uint4* mk = reinterpret_cast<const uint4*>(bw.mask + (int64_t)g * a.out_gs + dst * a.N + c0);
+          const float4* yv = reinterpret_cast<const float4*>(bw.y + (int64_t)g * a.out_gs + dst * a.N + c0);
+          float gx[16];
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            const uint4 m8 = __ldg(mk + h);
+            const float4 y0 = __ldg(yv + 2 * h), y1 = __ldg(yv + 2 * h + 1);
+            const uint32_t mw[4] = {m8.x, m8.y, m8.z, m8.w};
+            const float yy[8] = {y0.x, y0.y, y0.z, y0.w, y1.x, y1.y, y1.z, y1.w};
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+              const int j = 8 * h + k;
+              const float m = bf2f((uint16_t)(k & 1 ? mw[k >> 1] >> 16 : mw[k >> 1] & 0xffffu));
+              v[j] = m > 0.f ? v[j] : 0.f;
+              gx[j] = v[j] * ((yy[k] - bw_mu[c0 + j]) * bw_rs[c0 + j]);
+            }
+          }
+          float t[16];
+#pragma unroll
+          for (int j = 0; j < 16; ++j) t[j] = v[j];
+          run_g[ci] += warp_colsum16(t, lane);
+          run_gx[ci] += warp_colsum16(gx, lane);
         }
         if (a.st32) {
           // whole 32-byte sectors per lane and instruction
@@ -1486,6 +1581,14 @@ __global__ void __launch_bounds__(cv::THREADS, 1) conv_tc_kernel(const __grid_co
       asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
       asm volatile("bar.sync 1, 128;" ::: "memory");
       if (leader) mbar_arrive(&acc_empty[ab]);
+    }
+    if (with_bwd && !(lane & 1)) {
+#pragma unroll
+      for (int ci = 0; ci < 4; ++ci) {
+        if (16 * ci >= a.N) break;
+        bw.part[((int64_t)g * bw.part_gs + bw.part_off + 4 * blockIdx.x + quarter) * a.N + 16 * ci +
+                (lane >> 1)] = make_float2(run_g[ci], run_gx[ci]);
+      }
     }
     if (with_stats && !(lane & 1)) {
       // one partial per epilogue warp: stats[g][4 q + quarter]
@@ -1872,9 +1975,61 @@ bool make_tma_map(CUtensorMap* map, const void* base, bool bf16, uint64_t dim0, 
   return r == CUDA_SUCCESS;
 }
 
+namespace {
+// The launch shape of conv_tc_kernel: false if the arguments are not taken.
+bool conv_tc_plan(const ConvArgs& a, int sms, int* per_sm, size_t* ring, size_t* smem, int* cpr) {
+  if (a.stats && a.dst_h > 0) return false;
+  if (a.bwd.y && (!a.bwd.mask || !a.bwd.mean || !a.bwd.rstd || !a.bwd.part ||
+                  (a.bwd.sc_dout && (!a.bwd.sc_out || a.bwd.sc_C < a.N ||
+                                     (a.bwd.sc_stride != 1 && a.bwd.sc_stride != 2)))))
+    return false;
+  int rows = 0, images = 0;
+  if ((a.ck != 16 && a.ck != 32 && a.ck != 64) || (a.stride != 1 && a.stride != 2) ||
+      (a.N != 16 && a.N != 32 && a.N != 64) || a.np != a.N || !a.out || a.G > 65535 ||
+      !conv_tile_shape(a.hout, a.wout, &rows, &images) || a.P % (a.hout * a.wout) || a.P % BM ||
+      (a.dst_h > 0 && (a.dst_h < 2 * a.hout || a.dst_w < 2 * a.wout || a.ph_y < 0 || a.ph_y > 1 ||
+                       a.ph_x < 0 || a.ph_x > 1)))
+    return false;
+  const size_t fixed = 1024 + 9 * (size_t)a.np * a.ck * 2 + cv::AUX_BYTES;
+  const bool strip = a.strip != 0;
+  if (strip && !conv_strip_ok(a.hout, a.wout, a.stride)) return false;
+  const size_t stage_bytes = 3 * ((size_t)BM + (strip ? 2 * a.wout : 0)) * a.ck * 2;
+  const size_t two_budget = 113 * 1024;
+  *ring = cv::RING_BYTES;
+  *per_sm = 1;
+  if (two_budget > fixed && (two_budget - fixed) / stage_bytes >= 3) {
+    *ring = std::min<size_t>(cv::RING_BYTES, ((two_budget - fixed) / 1024) * 1024);
+    *per_sm = 2;
+  }
+  if (*per_sm == 1) {
+    // one CTA per SM: the ring takes what the weights leave of the 227 KB (at most 24 stages)
+    *ring = std::min<size_t>((size_t)cv::MAX_STAGES * stage_bytes,
+                             ((cv::SMEM_MAX - fixed) / stage_bytes) * stage_bytes);
+  }
+  *smem = fixed + *ring;
+  // CTAs per replica: as many as fit on the SMs at once over all replicas (one wave), at most one
+  // per tile
+  *cpr = std::max(1, std::min(a.P / BM, *per_sm * sms / a.G));
+  return true;
+}
+
+int device_sms(int* sms) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(sms, cudaDevAttrMultiProcessorCount, dev);
+  return e == cudaSuccess ? dev : -1;
+}
+}  // namespace
+
+int conv_tc_ctas(const ConvArgs& a) {
+  int sms = 0, per_sm = 1, cpr = 0;
+  size_t ring = 0, smem = 0;
+  if (a.P <= 0 || a.G <= 0 || device_sms(&sms) < 0) return 0;
+  return conv_tc_plan(a, sms, &per_sm, &ring, &smem, &cpr) ? cpr : 0;
+}
+
 cudaError_t launch_conv_tc(const ConvArgs& a, cudaStream_t stream, int* ctas_per_replica) {
   if (a.P <= 0 || a.G <= 0) return cudaSuccess;
-  if (a.stats && a.dst_h > 0) return cudaErrorInvalidValue;
   int rows = 0, images = 0;
   if ((a.ck != 16 && a.ck != 32 && a.ck != 64) || (a.stride != 1 && a.stride != 2) ||
       (a.N != 16 && a.N != 32 && a.N != 64) || a.np != a.N || !a.out || a.G > 65535 ||
@@ -1882,30 +2037,17 @@ cudaError_t launch_conv_tc(const ConvArgs& a, cudaStream_t stream, int* ctas_per
       (a.dst_h > 0 && (a.dst_h < 2 * a.hout || a.dst_w < 2 * a.wout || a.ph_y < 0 || a.ph_y > 1 ||
                        a.ph_x < 0 || a.ph_x > 1)))
     return cudaErrorInvalidValue;
-  int dev = 0, sms = 0;
-  cudaError_t e = cudaGetDevice(&dev);
-  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  if (e != cudaSuccess) return e;
+  (void)rows;
+  (void)images;
   // Two CTAs per SM where the weights leave room for a ring of at least three stages (a CTA's
   // tiles pass through a chain of handshakes one after another; two CTAs overlap their chains),
-  // else one CTA with the full ring.
-  const size_t fixed = 1024 + 9 * (size_t)a.np * a.ck * 2 + cv::AUX_BYTES;
-  const bool strip = a.strip != 0;
-  if (strip && !conv_strip_ok(a.hout, a.wout, a.stride)) return cudaErrorInvalidValue;
-  const size_t stage_bytes = 3 * ((size_t)BM + (strip ? 2 * a.wout : 0)) * a.ck * 2;
-  const size_t two_budget = 113 * 1024;
-  size_t ring = cv::RING_BYTES;
-  int per_sm = 1;
-  if (two_budget > fixed && (two_budget - fixed) / stage_bytes >= 3) {
-    ring = std::min<size_t>(cv::RING_BYTES, ((two_budget - fixed) / 1024) * 1024);
-    per_sm = 2;
-  }
-  if (per_sm == 1) {
-    // one CTA per SM: the ring takes what the weights leave of the 227 KB (at most 24 stages)
-    ring = std::min<size_t>((size_t)cv::MAX_STAGES * stage_bytes,
-                            ((cv::SMEM_MAX - fixed) / stage_bytes) * stage_bytes);
-  }
-  const size_t smem = fixed + ring;
+  // else one CTA with the full ring (conv_tc_plan).
+  int sms = 0, per_sm = 1, cpr = 0;
+  size_t ring = 0, smem = 0;
+  const int dev = device_sms(&sms);
+  if (dev < 0) return cudaErrorInvalidDevice;
+  if (!conv_tc_plan(a, sms, &per_sm, &ring, &smem, &cpr)) return cudaErrorInvalidValue;
+  cudaError_t e = cudaSuccess;
   ConvArgs la = a;
   la.ring_bytes = (int)ring;
   la.st32 = (reinterpret_cast<uintptr_t>(a.out) & 31) == 0 && a.out_gs % 8 == 0 ? 1 : 0;
@@ -1916,10 +2058,6 @@ cudaError_t launch_conv_tc(const ConvArgs& a, cudaStream_t stream, int* ctas_per
     if (e != cudaSuccess) return e;
     attr_dev = dev;
   }
-  // CTAs per replica: as many as fit on the SMs at once over all replicas (one wave), at most one
-  // per tile
-  const int tiles = a.P / BM;
-  const int cpr = std::max(1, std::min(tiles, per_sm * sms / a.G));
   // accumulators (measured in the ResNet-20 step): four buffers of three column partials where
   // the CTAs on one SM fit in its 512 TMEM columns (16 channels); else four single buffers where
   // they fit (32 channels, two CTAs per SM), else two buffers of three partials (64 channels)

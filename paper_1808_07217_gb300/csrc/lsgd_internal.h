@@ -160,6 +160,28 @@ struct GemmArgs {
 // map of make_tma_map_conv; w_map: a rank-3 map over the [N][9][ck] weights {9 ck, N, G} with box
 // {ck, np} and a ck * 2-byte swizzle.  ck, N in {16, 32, 64}, np = N; P = output pixels per
 // replica, a multiple of 128 and of hout * wout.
+// A data gradient whose result feeds the BatchNorm backward of the layer below (ResNet-20's
+// backward pass, Sec. A.2): the convolution's epilogue adds the option-A shortcut's share of the
+// block's output gradient (sc_dout non-null: stride 1 at every pixel, stride 2 at the pixels on
+// the stride grid, the first N of sc_C channels, masked by the block output sc_out > 0), applies
+// the ReLU mask of that layer (mask > 0), writes g = (dx + shortcut) * (mask > 0) instead of dx,
+// and each epilogue warp sums g and g * xhat per channel (xhat = (y - mean) rstd) over its rows of
+// every tile: part[g][part_off + 4 q + warp][n] = (sum g, sum g xhat) for CTA q.  mask and y have
+// dx's layout; sc_dout / sc_out are [G][pixels of the block output][sc_C] (per replica sc_gs
+// elements).
+struct ConvBwdFuse {
+  const uint16_t* mask;
+  const float* y;
+  const float* mean;
+  const float* rstd;
+  const float* sc_dout;
+  const uint16_t* sc_out;
+  int64_t sc_gs;
+  int sc_C, sc_stride;
+  float2* part;
+  int64_t part_gs;  // partials per replica (all launches that share the buffer)
+  int part_off;     // this launch's first partial
+};
 struct ConvArgs {
   CUtensorMap in_map, w_map;
   int ck, stride, hout, wout, N, np, G, P;
@@ -176,6 +198,7 @@ struct ConvArgs {
   int strip;  // stage form: 1 = strip (in_map made with strip = true), 0 = per kernel row
   int st32;   // out 32-byte aligned: 256-bit stores (set by the launcher)
   int nacc, nsplit;  // accumulator buffers and column partials per tile (set by the launcher)
+  ConvBwdFuse bwd;   // bwd.y non-null: the data gradient's BatchNorm-backward epilogue
 };
 // TMEM columns of the convolution kernel for n accumulators (buffers x partials) of np columns: a
 // power of two >= 32.
@@ -190,6 +213,8 @@ __host__ __device__ inline uint32_t conv_tmem_cols(int n, int np) {
 bool conv_strip_ok(int hout, int wout, int stride);
 // ctas_per_replica (if non-null) receives the statistics partials per replica (4 per CTA).
 cudaError_t launch_conv_tc(const ConvArgs& a, cudaStream_t stream, int* ctas_per_replica = nullptr);
+// The CTAs per replica launch_conv_tc will use for these arguments (0 if it would reject them).
+int conv_tc_ctas(const ConvArgs& a);
 // Weight gradient of a 3x3 convolution (zero padding 1, stride 1 or 2) on the tensor cores, the
 // column matrix built in shared memory: part[g][q][co][t Cin + ci] = the sum over CTA q's 64-pixel
 // output blocks of dy[g][p][co] x[g][src_t(p)][ci], src_t(p) the input pixel under tap t of output

@@ -693,6 +693,34 @@ __global__ void bn_bwd_finalize_kernel(const float* __restrict__ part, int C, in
   }
 }
 
+// The same sums from the data-gradient convolution's epilogue partials (ConvBwdFuse): one warp
+// per (replica, channel); lane l adds partials l, l + 32, ... in order, then a fixed butterfly.
+__global__ void bn_bwd_merge_kernel(const float2* __restrict__ part, int nparts, int C, int G,
+                                    float* __restrict__ s12, float* __restrict__ Gr, int64_t g_off,
+                                    int64_t b_off, int64_t d_gs) {
+  pdl_begin();
+  const int wid = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
+  if (wid >= G * C) return;
+  const int g = wid / C, c = wid % C;
+  float a = 0.f, b = 0.f;
+  for (int q = lane; q < nparts; q += 32) {
+    const float2 v = part[((int64_t)g * nparts + q) * C + c];
+    a += v.x;
+    b += v.y;
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    a += __shfl_xor_sync(0xffffffffu, a, o);
+    b += __shfl_xor_sync(0xffffffffu, b, o);
+  }
+  if (lane == 0) {
+    s12[(int64_t)wid * 2] = a;
+    s12[(int64_t)wid * 2 + 1] = b;
+    Gr[(int64_t)g * d_gs + g_off + c] = b;
+    Gr[(int64_t)g * d_gs + b_off + c] = a;
+  }
+}
+
 // dy = gamma rstd (dz - mean(dz) - xhat mean(dz xhat)), the convolution's output gradient; one
 // thread per pixel and 4 channels.
 template <typename TA>
@@ -1156,6 +1184,9 @@ struct ResNetPlan {
   // BatchNorm statistics computed by the forward convolutions' epilogues: per replica, CTA and
   // epilogue warp, (count, mean, M2) of each channel, merged by bn_merge_partials_kernel
   float4* cstats = nullptr;   // [K + 2 SMs][64]
+  // backward BatchNorm sums computed by the data-gradient convolutions' epilogues (ConvBwdFuse),
+  // consumed by the next BatchNorm backward: [K][16 (K + 2 SMs) / K][64] at most
+  float2* bpart = nullptr;
   std::string err;
 };
 
@@ -1339,9 +1370,13 @@ lsgd_status conv_fwd_tc(const uint16_t* x, const uint16_t* w, int64_t w_gs, floa
   return LSGD_OK;
 }
 
+// bf (optional): the BatchNorm-backward epilogue (ConvBwdFuse; part_gs / part_off are filled in
+// here); *nparts receives the partials per replica it wrote.
 lsgd_status conv_dgrad_tc(const uint16_t* dy, const uint16_t* w, int64_t w_gs, float* dx, int G,
                           int B, int hin, int win, int cin, int cout, int stride, uint16_t* wt,
-                          cudaStream_t s, std::string& err, int64_t* launches) {
+                          cudaStream_t s, std::string& err, int64_t* launches,
+                          const ConvBwdFuse* bf = nullptr, int* nparts = nullptr) {
+  if (nparts) *nparts = 0;
   if (!conv_dgrad_tc_route(B, hin, win, cin, cout, stride)) {
     err = "data-gradient shape not taken by the implicit-GEMM kernel";
     return LSGD_EUNSUPPORTED;
@@ -1368,6 +1403,17 @@ lsgd_status conv_dgrad_tc(const uint16_t* dy, const uint16_t* w, int64_t w_gs, f
     ca.P = (int)P;
     ca.out = dx;
     ca.out_gs = P * cin;
+    if (bf) {
+      ca.bwd = *bf;
+      const int cpr = conv_tc_ctas(ca);
+      if (cpr < 1) {
+        err = "data-gradient arguments rejected";
+        return LSGD_EINVAL;
+      }
+      ca.bwd.part_gs = 4 * cpr;
+      ca.bwd.part_off = 0;
+      if (nparts) *nparts = 4 * cpr;
+    }
     CV_CALL(launch_conv_tc(ca, s));
     return LSGD_OK;
   }
@@ -1401,6 +1447,18 @@ lsgd_status conv_dgrad_tc(const uint16_t* dy, const uint16_t* w, int64_t w_gs, f
     ca.ph_x = ph & 1;
     ca.dst_h = hin;
     ca.dst_w = win;
+    if (bf) {
+      // the four phases' partials side by side: phase ph writes partials [4 cpr ph, 4 cpr (ph + 1))
+      ca.bwd = *bf;
+      const int cpr = conv_tc_ctas(ca);
+      if (cpr < 1) {
+        err = "data-gradient arguments rejected";
+        return LSGD_EINVAL;
+      }
+      ca.bwd.part_gs = 16 * cpr;
+      ca.bwd.part_off = 4 * cpr * ph;
+      if (nparts) *nparts = 16 * cpr;
+    }
     CV_CALL(launch_conv_tc(ca, s));
   }
   return LSGD_OK;
@@ -1602,15 +1660,21 @@ lsgd_status forward_impl(ResNetPlan* p, const float* W, const void* Wop, int w_g
   return LSGD_OK;
 }
 
+// fused_parts > 0: the data-gradient convolution that produced dout already masked it by out > 0
+// and left the sums' partials in p->bpart (ConvBwdFuse); only their merge and the apply pass run.
 template <typename TA>
 lsgd_status bn_backward(ResNetPlan* p, const ConvL& c, int i, const float* dout, const void* out,
-                        const float* W, float* Gr, cudaStream_t s, int64_t* launches) {
+                        const float* W, float* Gr, cudaStream_t s, int64_t* launches,
+                        int fused_parts = 0) {
   const int K = p->K;
   const int64_t P = conv_pixels(p, c);
   const int chunk = rn_chunk(P);
   const int nq = (int)((P + chunk - 1) / chunk);
   const int lanes = std::max(1, 256 / c.cout);
-  if (vec4_ok(c.cout))
+  if (fused_parts > 0) {
+    RN_LAUNCH((launch_pdl(bn_bwd_merge_kernel, (K * c.cout * 32 + 127) / 128, 128, 0, s, p->bpart,
+        fused_parts, c.cout, K, p->s12, Gr, c.g_off, c.b_off, p->d_pad)));
+  } else if (vec4_ok(c.cout))
     RN_LAUNCH((launch_pdl(bn_bwd_partial_v4_kernel<TA>, dim3(nq, K), 256, 0, s, dout,
         reinterpret_cast<const TA*>(out), p->y[i], p->mean[i], p->rstd[i], P, c.cout, nq, chunk,
         p->part)));
@@ -1618,8 +1682,9 @@ lsgd_status bn_backward(ResNetPlan* p, const ConvL& c, int i, const float* dout,
     RN_LAUNCH((launch_pdl(bn_bwd_partial_kernel<TA>, dim3(nq, K), lanes * c.cout, 0, s, dout,
         reinterpret_cast<const TA*>(out), p->y[i], p->mean[i], p->rstd[i], P, c.cout, nq, chunk,
         p->part)));
-  RN_LAUNCH((launch_pdl(bn_bwd_finalize_kernel, (K * c.cout * 32 + 127) / 128, 128, 0, s, p->part,
-      c.cout, nq, K, p->s12, Gr, c.g_off, c.b_off, p->d_pad)));
+  if (fused_parts == 0)
+    RN_LAUNCH((launch_pdl(bn_bwd_finalize_kernel, (K * c.cout * 32 + 127) / 128, 128, 0, s,
+        p->part, c.cout, nq, K, p->s12, Gr, c.g_off, c.b_off, p->d_pad)));
   if (vec4_ok(c.cout)) {
     RN_LAUNCH((launch_pdl(bn_bwd_apply_v4_kernel<TA>, dim3(px_blocks(P, c.cout), (unsigned)K), 256,
         0, s, dout, reinterpret_cast<const TA*>(out), p->y[i], p->mean[i], p->rstd[i], p->s12, W,
@@ -1698,12 +1763,38 @@ lsgd_status conv_wgrad(ResNetPlan* p, int i, const void* in, float* Gr, cudaStre
   return LSGD_OK;
 }
 
+// bn_t >= 0: convolution bn_t (whose output, the activation this data gradient flows into, is
+// normalised next in the backward pass) gets its ReLU mask and BatchNorm-backward sums formed in
+// the persistent kernel's epilogue, together with the shortcut's share of dout (ConvBwdFuse):
+// dx then holds the masked gradient and *fused_parts the partials per replica in p->bpart (0 when
+// this path did not run).
 template <typename TA>
 lsgd_status conv_dgrad(ResNetPlan* p, int i, const void* Wop, float* dx, const float* dout,
-                       const void* out_act, cudaStream_t s, int64_t* launches) {
+                       const void* out_act, cudaStream_t s, int64_t* launches, int bn_t = -1,
+                       int* fused_parts = nullptr) {
   const ConvL& c = p->convs[i];
   const int K = p->K;
   const int64_t P = (int64_t)p->B * c.hin * c.win;
+  if (fused_parts) *fused_parts = 0;
+  ConvBwdFuse bf{};
+  // measured per layer in the ResNet-20 step: the fused epilogue's extra loads pay for themselves
+  // on the 16-channel data gradients (the largest tensors) but not on the 32 / 64-channel ones,
+  // where the separate passes are cheaper than the epilogue's added latency
+  const bool fuse = bn_t >= 0 && fused_parts && p->bpart && sizeof(TA) == 2 && c.cin <= 16;
+  if (fuse) {
+    bf.mask = reinterpret_cast<const uint16_t*>(p->act[bn_t]);
+    bf.y = p->y[bn_t];
+    bf.mean = p->mean[bn_t];
+    bf.rstd = p->rstd[bn_t];
+    if (dout) {
+      bf.sc_dout = dout;
+      bf.sc_out = reinterpret_cast<const uint16_t*>(out_act);
+      bf.sc_C = c.cout;
+      bf.sc_stride = c.stride;
+      bf.sc_gs = (int64_t)p->B * c.hout * c.wout * c.cout;
+    }
+    bf.part = p->bpart;
+  }
   if (conv_on_tc(p, c) && c.stride == 1 && implicit_conv_ok(c.cout, 1, c.hin, c.win)) {
     // stride 1: dx is the convolution of dy with the flipped, transposed weights -- an implicit
     // GEMM over dy's taps, no column matrix
@@ -1711,8 +1802,9 @@ lsgd_status conv_dgrad(ResNetPlan* p, int i, const void* Wop, float* dx, const f
       const lsgd_status st = conv_dgrad_tc(reinterpret_cast<const uint16_t*>(p->dy),
                                            reinterpret_cast<const uint16_t*>(Wop) + c.w_off, p->d_pad,
                                            dx, K, p->B, c.hin, c.win, c.cin, c.cout, 1, p->wt, s,
-                                           p->err, launches);
+                                           p->err, launches, fuse ? &bf : nullptr, fused_parts);
       if (st != LSGD_OK) return st;
+      if (fuse) return LSGD_OK;  // the epilogue added the shortcut's share
     } else {
       RN_LAUNCH((launch_pdl(flip_weights_kernel,
           dim3((unsigned)((c.cin * 9 * c.cout + 255) / 256), (unsigned)K), 256, 0, s,
@@ -1756,8 +1848,9 @@ lsgd_status conv_dgrad(ResNetPlan* p, int i, const void* Wop, float* dx, const f
     const lsgd_status st = conv_dgrad_tc(reinterpret_cast<const uint16_t*>(p->dy),
                                          reinterpret_cast<const uint16_t*>(Wop) + c.w_off, p->d_pad,
                                          dx, K, p->B, c.hin, c.win, c.cin, c.cout, 2, p->wt4, s,
-                                         p->err, launches);
+                                         p->err, launches, fuse ? &bf : nullptr, fused_parts);
     if (st != LSGD_OK) return st;
+    if (fuse) return LSGD_OK;  // the epilogue added the shortcut's share
     if (dout) {
       const int64_t n = (int64_t)p->B * c.hout * c.wout * (c.cin / 4);
       RN_LAUNCH((launch_pdl(add_shortcut_grad_v2_kernel<TA>,
@@ -1883,31 +1976,38 @@ lsgd_status fwd_bwd_impl(ResNetPlan* p, const float* W, const void* Wop, float* 
         HW, p->F)));
   }
   const int n_blocks = (int)(p->convs.size() - 1) / 2;
+  // partials of the next BatchNorm backward left by the data-gradient epilogue (0: none; the top
+  // block's output gradient comes from the pooling's backward)
+  int pending = 0;
   for (int j = n_blocks - 1; j >= 0; --j) {
     const int ia = 2 * j + 1, ib = 2 * j + 2;
     const ConvL& ca = p->convs[ia];
     const ConvL& cb = p->convs[ib];
     const void* blk_in = p->act[2 * j];
-    // second convolution: BN backward through the block's output ReLU, then its products
-    st = bn_backward<TA>(p, cb, ib, p->dA[cur], p->act[ib], W, Gr, s, launches);
+    // second convolution: BN backward through the block's output ReLU, then its products; its
+    // data gradient forms the first convolution's masked gradient and BN sums
+    st = bn_backward<TA>(p, cb, ib, p->dA[cur], p->act[ib], W, Gr, s, launches, pending);
     if (st != LSGD_OK) return st;
     st = conv_wgrad<TA>(p, ib, p->act[ia], Gr, s, launches);
     if (st != LSGD_OK) return st;
-    st = conv_dgrad<TA>(p, ib, Wop, p->dh, nullptr, nullptr, s, launches);
+    int parts_ia = 0;
+    st = conv_dgrad<TA>(p, ib, Wop, p->dh, nullptr, nullptr, s, launches, ia, &parts_ia);
     if (st != LSGD_OK) return st;
     // first convolution: BN backward through the inner ReLU, then its products; the data
-    // gradient also receives the shortcut's share of the block's output gradient
-    st = bn_backward<TA>(p, ca, ia, p->dh, p->act[ia], W, Gr, s, launches);
+    // gradient also receives the shortcut's share of the block's output gradient and forms the
+    // block input's masked gradient and the BN sums of the convolution that produced it
+    st = bn_backward<TA>(p, ca, ia, p->dh, p->act[ia], W, Gr, s, launches, parts_ia);
     if (st != LSGD_OK) return st;
     st = conv_wgrad<TA>(p, ia, blk_in, Gr, s, launches);
     if (st != LSGD_OK) return st;
-    st = conv_dgrad<TA>(p, ia, Wop, p->dA[1 - cur], p->dA[cur], p->act[ib], s, launches);
+    st = conv_dgrad<TA>(p, ia, Wop, p->dA[1 - cur], p->dA[cur], p->act[ib], s, launches, 2 * j,
+                        &pending);
     if (st != LSGD_OK) return st;
     cur = 1 - cur;
   }
   // stem: BN backward and the weight gradient (no data gradient for the image)
   const ConvL& c0 = p->convs[0];
-  st = bn_backward<TA>(p, c0, 0, p->dA[cur], p->act[0], W, Gr, s, launches);
+  st = bn_backward<TA>(p, c0, 0, p->dA[cur], p->act[0], W, Gr, s, launches, pending);
   if (st != LSGD_OK) return st;
   return conv_wgrad<TA>(p, 0, p->x0, Gr, s, launches);
 }
@@ -2249,7 +2349,9 @@ lsgd_status resnet_alloc(ResNetPlan* p, const std::function<void*(size_t)>& allo
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
       return LSGD_ECUDA;
     p->cstats = (float4*)alloc((size_t)4 * (K + 2 * sms) * 64 * sizeof(float4));
-    if (!p->cstats) return LSGD_ENOMEM;
+    // four phases x four warps x (CTAs over all replicas <= max(K, 2 SMs)) partials of 64 channels
+    p->bpart = (float2*)alloc((size_t)16 * (K + 2 * sms) * 64 * sizeof(float2));
+    if (!p->cstats || !p->bpart) return LSGD_ENOMEM;
   }
   if (!p->x0 || !p->part || !p->feat || !p->dfeat || !p->logits || !p->dlogits || !p->dA[0] ||
       !p->dA[1] || !p->dh || !p->dy || !p->s12)

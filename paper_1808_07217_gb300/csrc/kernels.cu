@@ -693,8 +693,9 @@ cudaError_t launch_softmax_xent(const float* logits, int ld, int C, const int32_
                                 float* loss_sum, float* row_loss, cudaStream_t stream) {
   if (G <= 0 || B <= 0) return cudaSuccess;
   if (B > 8192 || C < 1) return cudaErrorInvalidValue;
-  // one warp per row up to 32 warps; the row losses in shared memory
-  const int threads = 32 * std::min(32, B);
+  // one warp per row, up to 32 warps (8 for at most 32 classes, where a row is one pass of a
+  // warp and the block's reduction barriers would dominate); the row losses in shared memory
+  const int threads = 32 * std::min(C > 32 ? 32 : 8, B);
   const size_t smem = (size_t)B * sizeof(float);
   if (dz_bf16)
     launch_pdl(softmax_xent_kernel<uint16_t>, G, threads, smem, stream,

@@ -756,7 +756,8 @@ __global__ void bn_bwd_apply_kernel(const float* __restrict__ dout, const TA* __
 }
 
 // The same with a fixed group of 4 channels per thread (C / 4 dividing the block size), the
-// per-channel factors loaded once, blockIdx.y the replica.
+// per-channel factors loaded once, blockIdx.y the replica.  out == nullptr: dout is already
+// masked (the data-gradient epilogue applied the ReLU), so dz = dout.
 template <typename TA>
 __global__ void __launch_bounds__(256) bn_bwd_apply_v4_kernel(
     const float* __restrict__ dout, const TA* __restrict__ out, const float* __restrict__ y,
@@ -780,7 +781,7 @@ __global__ void __launch_bounds__(256) bn_bwd_apply_v4_kernel(
   for (int p = blockIdx.x * ppb + pl; p < P; p += gridDim.x * ppb) {
     const int64_t e = base + (int64_t)p * C;
     const float4 d4 = *reinterpret_cast<const float4*>(dout + e);
-    const float4 o4 = Vec4<TA>::load(out + e);
+    const float4 o4 = out ? Vec4<TA>::load(out + e) : make_float4(1.f, 1.f, 1.f, 1.f);
     const float4 y4 = *reinterpret_cast<const float4*>(y + e);
     const float dd[4] = {d4.x, d4.y, d4.z, d4.w}, oo[4] = {o4.x, o4.y, o4.z, o4.w};
     const float yy[4] = {y4.x, y4.y, y4.z, y4.w};
@@ -1686,9 +1687,11 @@ lsgd_status bn_backward(ResNetPlan* p, const ConvL& c, int i, const float* dout,
     RN_LAUNCH((launch_pdl(bn_bwd_finalize_kernel, (K * c.cout * 32 + 127) / 128, 128, 0, s,
         p->part, c.cout, nq, K, p->s12, Gr, c.g_off, c.b_off, p->d_pad)));
   if (vec4_ok(c.cout)) {
+    // with fused partials dout is already masked: no read of the activation for the mask
     RN_LAUNCH((launch_pdl(bn_bwd_apply_v4_kernel<TA>, dim3(px_blocks(P, c.cout), (unsigned)K), 256,
-        0, s, dout, reinterpret_cast<const TA*>(out), p->y[i], p->mean[i], p->rstd[i], p->s12, W,
-        c.g_off, p->d_pad, reinterpret_cast<TA*>(p->dy), (int)P, c.cout)));
+        0, s, dout, fused_parts > 0 ? nullptr : reinterpret_cast<const TA*>(out), p->y[i],
+        p->mean[i], p->rstd[i], p->s12, W, c.g_off, p->d_pad, reinterpret_cast<TA*>(p->dy),
+        (int)P, c.cout)));
   } else {
     const int64_t n = (int64_t)K * P * c.cout / 4;
     RN_LAUNCH((launch_pdl(bn_bwd_apply_kernel<TA>, grid_cap(n, 256), 256, 0, s, dout,

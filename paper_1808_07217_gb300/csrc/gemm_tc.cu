@@ -117,6 +117,19 @@ __device__ __forceinline__ uint64_t smem_desc_kmajor(uint32_t addr, uint32_t swz
   return d;
 }
 
+// An MN-major (or any) descriptor with the 32-, 64- or 128-byte swizzle given in bytes.
+__device__ __forceinline__ uint64_t smem_desc_swz(uint32_t addr, uint32_t lbo, uint32_t sbo,
+                                                  uint32_t swz) {
+  const uint64_t layout = swz == 128 ? 2ull : (swz == 64 ? 4ull : 6ull);
+  uint64_t d = 0;
+  d |= (uint64_t)((addr >> 4) & 0x3FFFu);
+  d |= (uint64_t)((lbo >> 4) & 0x3FFFu) << 16;
+  d |= (uint64_t)((sbo >> 4) & 0x3FFFu) << 32;
+  d |= 1ull << 46;  // descriptor version (tcgen05)
+  d |= layout << 61;
+  return d;
+}
+
 __device__ __forceinline__ uint64_t smem_desc(uint32_t addr, uint32_t lbo, uint32_t sbo) {
   uint64_t d = 0;
   d |= (uint64_t)((addr >> 4) & 0x3FFFu);
@@ -1673,8 +1686,10 @@ __global__ void __launch_bounds__(cw::THREADS, 1) conv_wgrad_tc_kernel(
   const int kb0 = (int)((int64_t)q * nkb / cpr);
   const int nblk = (int)((int64_t)(q + 1) * nkb / cpr) - kb0;
   const int per_img = a.hout * a.wout;
+  const int nb = a.nb;                               // MMA N: output-gradient channels
+  const uint32_t tile_b = (uint32_t)cw::KB * nb * 2;  // bytes of the output-gradient tile
   uint32_t tmem_cols = 32;
-  while (tmem_cols < (uint32_t)mt_n * 64) tmem_cols <<= 1;
+  while (tmem_cols < (uint32_t)(mt_n * nb)) tmem_cols <<= 1;
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < ni; ++i) {
@@ -1711,7 +1726,7 @@ __global__ void __launch_bounds__(cw::THREADS, 1) conv_wgrad_tc_kernel(
       const int p0 = (kb0 + j) * cw::KB;
       const int b = p0 / per_img, oy0 = (p0 % per_img) / a.wout;
       uint8_t* st = I0 + s * in_pitch;
-      mbar_expect_tx(&full_in[s], halo_bytes + cw::kTileB);
+      mbar_expect_tx(&full_in[s], halo_bytes + tile_b);
       tma_load_3d(st, &a.dy_map, &full_in[s], 0, p0, g);
       tma_load_5d(st + cw::kTileB, &a.x_map, &full_in[s], 0, 0, oy0 * a.stride - 1, b, g);
     }
@@ -1719,10 +1734,13 @@ __global__ void __launch_bounds__(cw::THREADS, 1) conv_wgrad_tc_kernel(
     for (int i = (j > ni ? j - ni : 0); i < j; ++i) mbar_wait(&full_in[i % ni], (i / ni) & 1);
   } else if (warp == 1 && lane == 0) {
     // ---------------- MMA issuer ----------------
-    const uint32_t idesc = make_idesc(BM, 64, true, true);
-    // descriptors of A0 and I0; a buffer / m-tile / K-step adds its byte offset / 16
+    const uint32_t idesc = make_idesc(BM, nb, true, true);
+    // descriptors of A0 and I0; a buffer / m-tile / K-step adds its byte offset / 16.  B: rows of
+    // 2 nb bytes (nb channels) swizzled at that width, 8-row groups 16 nb bytes apart, K-steps of
+    // 16 pixels 32 nb bytes apart; one swizzle atom spans all nb channels.
     const uint64_t a_desc0 = smem_desc(smem_u32(A0), 8192, 1024);
-    const uint64_t b_desc0 = smem_desc(smem_u32(I0), 8192, 1024);
+    const uint64_t b_desc0 = nb == 64 ? smem_desc(smem_u32(I0), 8192, 1024)
+                                      : smem_desc_swz(smem_u32(I0), 16u * nb, 16u * nb, 2u * nb);
     bool ok = true;
     for (int j = 0; j < nblk; ++j) {
       const int s = j % ni, sa = j % na;
@@ -1736,8 +1754,8 @@ __global__ void __launch_bounds__(cw::THREADS, 1) conv_wgrad_tc_kernel(
       for (int mt = 0; mt < mt_n; ++mt)
 #pragma unroll
         for (int kk = 0; kk < cw::KB / 16; ++kk)
-          mma_bf16(tmem + (uint32_t)(mt * 64), ad + (uint32_t)(mt * (cw::kTileA >> 4) + kk * 128),
-                   bd + (uint32_t)(kk * 128), idesc, (j > 0 || kk > 0) ? 1u : 0u);
+          mma_bf16(tmem + (uint32_t)(mt * nb), ad + (uint32_t)(mt * (cw::kTileA >> 4) + kk * 128),
+                   bd + (uint32_t)(kk * 2 * nb), idesc, (j > 0 || kk > 0) ? 1u : 0u);
       mma_commit(&afree[sa]);    // A buffer reusable once these MMAs have read it
       mma_commit(&empty_in[s]);  // and the output-gradient tile
     }
@@ -1820,7 +1838,7 @@ __global__ void __launch_bounds__(cw::THREADS, 1) conv_wgrad_tc_kernel(
         const int m = mt * 128 + quarter * 32 + lane;
         for (int c0 = 0; c0 < cout; c0 += 16) {
           float v[16];
-          tmem_ld16(tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(mt * 64 + c0), v);
+          tmem_ld16(tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(mt * nb + c0), v);
           if (m < mrows) {
 #pragma unroll
             for (int i = 0; i < 16; ++i) out[(int64_t)(c0 + i) * mrows + m] = v[i];
@@ -2244,7 +2262,8 @@ cudaError_t launch_conv_wgrad_tc(const ConvWgradArgs& a, cudaStream_t stream) {
   int na = 0, ni = 0, per_sm = 1;
   size_t smem = 0;
   conv_wgrad_plan(a.cin, a.stride, a.win, a.wout, &na, &ni, &per_sm, &smem);
-  if (ni < 2 || ni > cw::MAX_NI || na < 1 || na > cw::MAX_NA || smem > 232448)
+  if (ni < 2 || ni > cw::MAX_NI || na < 1 || na > cw::MAX_NA || smem > 232448 ||
+      (a.nb != 16 && a.nb != 32 && a.nb != 64) || a.nb < a.cout)
     return cudaErrorInvalidValue;
   ConvWgradArgs la = a;
   la.ni = ni;

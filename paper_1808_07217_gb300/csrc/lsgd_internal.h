@@ -220,13 +220,15 @@ int conv_tc_ctas(const ConvArgs& a);
 // output blocks of dy[g][p][co] x[g][src_t(p)][ci], src_t(p) the input pixel under tap t of output
 // pixel p (zero outside the image).  x_map: make_tma_map_halo over the NHWC input; dy_map: rank-3
 // bf16 map over [G][P][Cout] with box {64, 64} and a 128-byte swizzle.  Cin 16 / 32 / 64, Cout a
-// multiple of 16 up to 64, Wout dividing 64, Hout Wout a multiple of 64.
+// multiple of 16 up to 64, Wout dividing 64, Hout Wout a multiple of 64.  dy_map's box is
+// {nb, 64} with a 2 nb-byte swizzle.
 struct ConvWgradArgs {
   CUtensorMap x_map, dy_map;
   int cin, cout, stride, hin, win, hout, wout, G, P;
   int cpr;      // CTAs (partials) per replica, from conv_wgrad_ctas
   float* part;  // [G][cpr][cout][9 cin]
   int ni, na;   // input stages and A buffers (set by the launcher)
+  int nb;       // the MMAs' N and the output-gradient tile's channels (16, 32 or 64; dy_map's box)
 };
 bool conv_wgrad_tc_ok(int cin, int cout, int stride, int hin, int win, int hout, int wout);
 int conv_wgrad_ctas(int cin, int stride, int wout, int G, int64_t P);

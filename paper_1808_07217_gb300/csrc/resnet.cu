@@ -2107,9 +2107,13 @@ cudaError_t launch_conv_wgrad_bf16(const uint16_t* x, const uint16_t* dy, float*
       P > 0x7fffffffLL || cin_out > cin)
     return cudaErrorInvalidValue;
   ConvWgradArgs a{};
+  // the output-gradient tile: 64 pixels x nb channels (Cout of 16 / 32 / 64 exactly; 48 padded
+  // to 64 by the map's zero fill), swizzled at its 2 nb-byte row
+  const int nb = (cout == 16 || cout == 32) ? cout : 64;
   if (!make_tma_map_halo(&a.x_map, x, cin, win, hin, B, G, stride, wout) ||
-      !make_tma_map_bf16(&a.dy_map, dy, cout, P, G, cout, (uint64_t)P * cout, 64, 64))
+      !make_tma_map(&a.dy_map, dy, true, cout, P, G, cout, (uint64_t)P * cout, nb, 64, 2 * nb))
     return cudaErrorInvalidValue;
+  a.nb = nb;
   a.cin = cin;
   a.cout = cout;
   a.stride = stride;

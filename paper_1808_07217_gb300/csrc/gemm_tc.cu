@@ -708,6 +708,15 @@ __global__ void __launch_bounds__(pt::THREADS, 1) gemm_pt_kernel(const __grid_co
       const int ab = i & 1;
       float bsw[PBN / 64], bsu[PBN / 64];
       epilogue_bias_prefetch<PBN>(args, et, g, n0, bsw, bsu);
+      if (args.epi == EPI_MASK && args.mask && m0 + et < args.M) {
+        // this thread's row of the tile's ReLU mask (the stored activation) into L2 while the
+        // tile's products run, so that the copy-out's mask loads do not each wait on DRAM
+        const int esz = args.mask_bf16 ? 2 : 4;
+        const int ncols = min(PBN, args.N - n0);
+        const char* rowp = reinterpret_cast<const char*>(args.mask) +
+                           ((int64_t)g * args.mask_gs + (int64_t)(m0 + et) * args.mask_rs + n0) * esz;
+        for (int b = 0; b < ncols * esz; b += 128) asm volatile("prefetch.global.L2 [%0];" ::"l"(rowp + b));
+      }
       if (leader) sm.epi_ok[fi] = mbar_wait(&sm.acc_full[ab], (i >> 1) & 1) ? 1 : 0;
       asm volatile("bar.sync 1, 128;" ::: "memory");
       const bool okw = sm.epi_ok[fi] != 0;
@@ -2361,12 +2370,12 @@ cudaError_t launch_gemm_tc(const TcGemmArgs& a, cudaStream_t stream) {
   // Short reductions (the weight gradient's k = B_loc) need only two stages; the smaller shared
   // footprint lets three CTAs share an SM so one CTA's epilogue overlaps the others' loads.
   if ((a.Kd + BK - 1) / BK <= 2) return launch_cfg<BN, 2>(a, grid, stream);
-  // Wide forward products (K-major weights, at least 2048 output columns, no split): the
-  // persistent kernel.  Narrower layers give it too few 128 x 256 tiles to fill the SMs, and the
-  // data gradient (MN-major weights) streamed its weights faster on the one-tile kernel's deeper
-  // rings (measured: MLP 3072-4096x3-100 forward 0.36 -> 0.27 ms per step; data gradient 0.38 ->
-  // 0.43 ms, and MLP 3072-1024-1024-10 0.29 -> 0.35 ms per step, so those stay where they are).
-  if (splits == 1 && a.N >= 2048 && !a.B.mn_major && a.B.box_rows == 64 && !gemm_pt_off())
+  // Wide products (at least 2048 output columns, no split): the persistent kernel -- the forward
+  // (K-major weights) and, since its epilogue prefetches the tile's ReLU mask, the data gradient
+  // (MN-major weights).  Narrower layers give it too few 128 x 256 tiles to fill the SMs
+  // (measured: MLP 3072-4096x3-100 forward 0.36 -> 0.27 ms per step, backward 0.333 -> 0.322 ms;
+  // MLP 3072-1024-1024-10 0.29 -> 0.35 ms per step, so it stays on the one-tile kernel).
+  if (splits == 1 && a.N >= 2048 && a.B.box_rows == 64 && !gemm_pt_off())
     return launch_pt(a, stream);
   // Other long reductions: 64-wide N tiles with four stages (96 KB) so two CTAs share an SM and
   // twice as many tiles stream weights at once.

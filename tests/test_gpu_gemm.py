@@ -54,7 +54,8 @@ def test_grouped_gemm_matches_fp64(P, shape, a_mn, b_mn):
 
 
 def test_persistent_and_one_tile_kernels_agree_bitwise():
-    # Wide forward products run on the persistent 128 x 256-tile kernel; the one-tile kernel
+    # Wide products (K-major or MN-major B, at least 2048 columns) run on the persistent
+    # 128 x 256-tile kernel; the one-tile kernel
     # (LSGD_GEMM_ONE_TILE=1 at library load) accumulates every output in the same k order, so
     # both give the same bits.  Run in subprocesses: the switch is read once.
     import os
@@ -68,7 +69,9 @@ P = built_package()
 gen = torch.Generator(device="cuda").manual_seed(5)
 out = []
 for (M, N, Kd, G, a_mn, b_mn) in [(128, 4096, 4096, 3, 0, 0), (128, 1024, 3072, 2, 0, 1),
-                                  (200, 520, 1000, 2, 0, 0), (128, 264, 136, 4, 0, 1)]:
+                                  (200, 520, 1000, 2, 0, 0), (128, 264, 136, 4, 0, 1),
+                                  (128, 4096, 4096, 2, 0, 1), (96, 2048, 520, 3, 0, 1),
+                                  (128, 2600, 1000, 2, 0, 1)]:
     A = torch.randn((G, Kd, M) if a_mn else (G, M, Kd), device="cuda", generator=gen).to(torch.bfloat16)
     B = torch.randn((G, Kd, N) if b_mn else (G, N, Kd), device="cuda", generator=gen).to(torch.bfloat16)
     C = torch.empty((G, M, N), device="cuda")

@@ -867,6 +867,90 @@ __device__ __forceinline__ int wu_chunks(int N, int n0) {
   return left >= wu::TN ? wu::TN / wu::CW : (left + wu::CW - 1) / wu::CW;
 }
 
+namespace wu {
+// What the epilogue does with a chunk, fixed at compile time so that the per-element code has no
+// branches: PLAIN writes the updated parameters; AVG folds them into the running pair (FIRST
+// starts it, LAST turns it into the mean and writes that).
+enum : int { kPlain = 0, kFirst = 1, kLast = 2, kAvg = 4 };
+}  // namespace wu
+
+// The local update of four consecutive parameters under one update rule (0: no momentum,
+// 1: heavy ball, 2: Nesterov); the same sgd_elem arithmetic as sgd4.
+template <bool SG, int RULE>
+__device__ __forceinline__ void sgd4_rule(float4& w, float4& u, const float4 g, const SgdParams& sp) {
+  constexpr bool MOM = RULE != 0, NEST = RULE == 2;
+  const float m = MOM ? sp.mom : 0.f;
+  sgd_elem<MOM, NEST>(w.x, u.x, g.x, sp.lr, m, sp.wd, SG);
+  sgd_elem<MOM, NEST>(w.y, u.y, g.y, sp.lr, m, sp.wd, SG);
+  sgd_elem<MOM, NEST>(w.z, u.z, g.z, sp.lr, m, sp.wd, SG);
+  sgd_elem<MOM, NEST>(w.w, u.w, g.w, sp.lr, m, sp.wd, SG);
+}
+
+// One epilogue thread's CPT columns of a 32-column chunk of its tile row r: the update of CPT
+// parameters (w, u in the swizzled shared-memory slot rows wrow / urow), in averaging mode folded
+// into the running pair (s, c) = (sc[0, CPT), sc[CPT, 2 CPT)) and, at the unit's last replica,
+// replaced by the mean; wherever the parameters leave for HBM their bf16 shadow goes to brow.
+// Without momentum u is neither read nor changed (its slot goes back to HBM as loaded).
+template <bool SG, int RULE, int MODE>
+__device__ __forceinline__ void wu_part_chunk(const float (&gv)[wu::CPT], float (&sc)[2 * wu::CPT],
+                                              uint8_t* wrow, uint8_t* urow, uint8_t* brow, int part,
+                                              int r, const SgdParams& sp, float Gf, float invG,
+                                              bool pow2) {
+  constexpr bool AVG = (MODE & wu::kAvg) != 0, FIRST = (MODE & wu::kFirst) != 0,
+                 LAST = (MODE & wu::kLast) != 0;
+  constexpr bool WRITE_W = !AVG || LAST;
+  uint32_t packed[wu::CPT / 2];
+#pragma unroll
+  for (int jj = 0; jj < wu::CPT / 4; ++jj) {
+    const int j = (wu::CPT / 4) * part + jj;  // float4 column group within the chunk
+    const int phys = (j ^ (r & 7)) << 4;
+    float4 wv = *reinterpret_cast<const float4*>(wrow + phys);
+    float4 uv = RULE != 0 ? *reinterpret_cast<const float4*>(urow + phys)
+                          : make_float4(0.f, 0.f, 0.f, 0.f);
+    sgd4_rule<SG, RULE>(wv, uv, make_float4(gv[4 * jj], gv[4 * jj + 1], gv[4 * jj + 2], gv[4 * jj + 3]),
+                        sp);
+    if (RULE != 0) *reinterpret_cast<float4*>(urow + phys) = uv;
+    if (AVG) {
+      float* sv = sc + 4 * jj;            // s of these four columns
+      float* cv = sc + wu::CPT + 4 * jj;  // c of these four columns
+      const float wn[4] = {wv.x, wv.y, wv.z, wv.w};
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        if (FIRST) {
+          sv[e] = wn[e];
+          cv[e] = 0.f;
+        } else {
+          two_sum_add(sv[e], cv[e], wn[e]);
+        }
+      }
+      if (LAST) {
+        float m[4];
+        if (pow2) {
+#pragma unroll
+          for (int e = 0; e < 4; ++e) m[e] = mean_of_pow2(sv[e], cv[e], Gf, invG);
+        } else {
+#pragma unroll
+          for (int e = 0; e < 4; ++e) m[e] = mean_of(sv[e], cv[e], Gf);
+        }
+        wv = make_float4(m[0], m[1], m[2], m[3]);
+      }
+    }
+    if (WRITE_W) {
+      *reinterpret_cast<float4*>(wrow + phys) = wv;
+      packed[2 * jj] = (uint32_t)f2bf(wv.x) | ((uint32_t)f2bf(wv.y) << 16);
+      packed[2 * jj + 1] = (uint32_t)f2bf(wv.z) | ((uint32_t)f2bf(wv.w) << 16);
+    }
+  }
+  if (WRITE_W) {
+#pragma unroll
+    for (int hh = 0; hh < wu::CPT / 8; ++hh) {
+      const int h = (wu::CPT / 8) * part + hh;  // 16-byte unit of the 64-byte bf16 row
+      *reinterpret_cast<uint4*>(brow + ((h ^ ((r >> 1) & 3)) << 4)) =
+          make_uint4(packed[4 * hh], packed[4 * hh + 1], packed[4 * hh + 2], packed[4 * hh + 3]);
+    }
+  }
+}
+
 __global__ void __launch_bounds__(wu::THREADS, 1) wgrad_update_kernel(
     const __grid_constant__ WgradUpdateArgs args) {
   extern __shared__ uint8_t smem_raw[];
@@ -1123,58 +1207,42 @@ __global__ void __launch_bounds__(wu::THREADS, 1) wgrad_update_kernel(
     const float Gf = (float)args.G;
     const bool pow2 = (args.G & (args.G - 1)) == 0;
     const float invG = 1.0f / Gf;  // exact when G is a power of two
-    // This thread's CPT columns of a chunk: the update of CPT parameters of its row (SG: the
-    // signSGD variant), in averaging mode folded into the running pair (s, c) and, at the unit's
-    // last replica, replaced by the mean.
-    auto part_chunk = [&](auto sg_tag, const float (&gv)[wu::CPT], float (&sc)[2 * wu::CPT],
-                          uint8_t* wrow, uint8_t* urow, uint8_t* brow, bool first, bool last) {
-      constexpr bool SG = decltype(sg_tag)::value;
-      const bool write_w = !avg || last;  // the parameters leave this chunk for HBM
-      uint32_t packed[wu::CPT / 2];
-#pragma unroll
-      for (int jj = 0; jj < wu::CPT / 4; ++jj) {
-        const int j = (wu::CPT / 4) * part + jj;  // float4 column group within the chunk
-        const int phys = (j ^ (r & 7)) << 4;
-        float4 wv = *reinterpret_cast<const float4*>(wrow + phys);
-        float4 uv = has_u ? *reinterpret_cast<const float4*>(urow + phys)
-                          : make_float4(0.f, 0.f, 0.f, 0.f);
-        sgd4<SG>(wv, uv, make_float4(gv[4 * jj], gv[4 * jj + 1], gv[4 * jj + 2], gv[4 * jj + 3]), sp);
-        if (has_u) *reinterpret_cast<float4*>(urow + phys) = uv;
-        if (avg) {
-          float* sv = sc + 4 * jj;             // s of these four columns
-          float* cv = sc + wu::CPT + 4 * jj;   // c of these four columns
-          const float wn[4] = {wv.x, wv.y, wv.z, wv.w};
-#pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            if (first) {
-              sv[e] = wn[e];
-              cv[e] = 0.f;
-            } else {
-              two_sum_add(sv[e], cv[e], wn[e]);
-            }
-          }
-          if (last) {
-            float m[4];
-#pragma unroll
-            for (int e = 0; e < 4; ++e)
-              m[e] = pow2 ? mean_of_pow2(sv[e], cv[e], Gf, invG) : mean_of(sv[e], cv[e], Gf);
-            wv = make_float4(m[0], m[1], m[2], m[3]);
-          }
-        }
-        if (write_w) {
-          *reinterpret_cast<float4*>(wrow + phys) = wv;
-          packed[2 * jj] = (uint32_t)f2bf(wv.x) | ((uint32_t)f2bf(wv.y) << 16);
-          packed[2 * jj + 1] = (uint32_t)f2bf(wv.z) | ((uint32_t)f2bf(wv.w) << 16);
-        }
-      }
-      if (write_w) {
-#pragma unroll
-        for (int hh = 0; hh < wu::CPT / 8; ++hh) {
-          const int h = (wu::CPT / 8) * part + hh;  // 16-byte unit of the 64-byte bf16 row
-          *reinterpret_cast<uint4*>(brow + ((h ^ ((r >> 1) & 3)) << 4)) =
-              make_uint4(packed[4 * hh], packed[4 * hh + 1], packed[4 * hh + 2], packed[4 * hh + 3]);
-        }
-      }
+    // the update rule (0: no momentum, 1: heavy ball, 2: Nesterov); momentum implies u
+    const int rule = sp.mom == 0.f ? 0 : (sp.nesterov ? 2 : 1);
+    // This thread's CPT columns of a chunk, through the variant of wu_part_chunk for this launch's
+    // rule and sign option and this tile's place in its unit: one branch per chunk, none per
+    // element.
+    auto part_chunk = [&](const float (&gv)[wu::CPT], float (&sc)[2 * wu::CPT], uint8_t* wrow,
+                          uint8_t* urow, uint8_t* brow, bool first, bool last) {
+      auto by_mode = [&](auto sg_tag, auto rule_tag) {
+        constexpr bool SG = decltype(sg_tag)::value;
+        constexpr int R = decltype(rule_tag)::value;
+        if (!avg)
+          wu_part_chunk<SG, R, wu::kPlain>(gv, sc, wrow, urow, brow, part, r, sp, Gf, invG, pow2);
+        else if (first && last)
+          wu_part_chunk<SG, R, wu::kAvg | wu::kFirst | wu::kLast>(gv, sc, wrow, urow, brow, part, r,
+                                                                  sp, Gf, invG, pow2);
+        else if (first)
+          wu_part_chunk<SG, R, wu::kAvg | wu::kFirst>(gv, sc, wrow, urow, brow, part, r, sp, Gf,
+                                                      invG, pow2);
+        else if (last)
+          wu_part_chunk<SG, R, wu::kAvg | wu::kLast>(gv, sc, wrow, urow, brow, part, r, sp, Gf,
+                                                     invG, pow2);
+        else
+          wu_part_chunk<SG, R, wu::kAvg>(gv, sc, wrow, urow, brow, part, r, sp, Gf, invG, pow2);
+      };
+      auto by_rule = [&](auto sg_tag) {
+        if (rule == 0)
+          by_mode(sg_tag, std::integral_constant<int, 0>{});
+        else if (rule == 1)
+          by_mode(sg_tag, std::integral_constant<int, 1>{});
+        else
+          by_mode(sg_tag, std::integral_constant<int, 2>{});
+      };
+      if (sp.sign)
+        by_rule(std::true_type{});
+      else
+        by_rule(std::false_type{});
     };
     int q = 0, i = 0;
     bool ok = true;
@@ -1212,10 +1280,7 @@ __global__ void __launch_bounds__(wu::THREADS, 1) wgrad_update_kernel(
         uint8_t* wrow = sm.w[sl] + r * 128;
         uint8_t* urow = sm.u[sl] + r * 128;
         uint8_t* brow = sm.wb[sl] + r * 64;
-        if (sp.sign)
-          part_chunk(std::true_type{}, gv, sc, wrow, urow, brow, first, last);
-        else
-          part_chunk(std::false_type{}, gv, sc, wrow, urow, brow, first, last);
+        part_chunk(gv, sc, wrow, urow, brow, first, last);
         if (avg && !last) tmem_st16_nowait(tmem + lane_base + sc_col, sc);
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
         asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");

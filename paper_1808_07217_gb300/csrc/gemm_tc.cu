@@ -780,7 +780,6 @@ constexpr int NS = 4;                       // w / u chunk slots
 constexpr int SD = 2;                       // chunks whose TMA stores may be in flight (<= NS)
 constexpr int EPI_WARPS = 16;               // four per TMEM lane quarter
 constexpr int THREADS = 128 + 32 * EPI_WARPS;
-constexpr int EPI0 = 128;                   // first epilogue thread
 constexpr int CPT = CW / (EPI_WARPS / 4);   // chunk columns per epilogue thread (8)
 constexpr uint32_t kChunkF32 = BM * CW * 4;  // 16 KB
 constexpr uint32_t kChunkB16 = BM * CW * 2;  // 8 KB
@@ -795,9 +794,8 @@ struct WuSmem {
   uint64_t op_full[wu::ST], op_empty[wu::ST];
   uint64_t acc_full[2], acc_empty[2];
   uint64_t wu_full[wu::NS], wu_empty[wu::NS];
-  uint64_t st_full[wu::NS];  // the epilogue has finished the slot's chunk: store it
+  uint64_t st_full[wu::NS];  // every epilogue warp has finished the slot's chunk: store it
   uint32_t tmem_base;
-  int epi_ok[2];
 };
 
 __device__ __forceinline__ void tmem_ld8(uint32_t taddr, float (&v)[8]) {
@@ -989,14 +987,15 @@ __global__ void __launch_bounds__(wu::THREADS, 1) wgrad_update_kernel(
       mbar_init(&sm.op_full[i], 1);
       mbar_init(&sm.op_empty[i], 1);
     }
+    // the epilogue warps release the accumulator and the chunk slots one arrival per warp
     for (int i = 0; i < 2; ++i) {
       mbar_init(&sm.acc_full[i], 1);
-      mbar_init(&sm.acc_empty[i], 1);
+      mbar_init(&sm.acc_empty[i], wu::EPI_WARPS);
     }
     for (int i = 0; i < wu::NS; ++i) {
       mbar_init(&sm.wu_full[i], 1);
       mbar_init(&sm.wu_empty[i], 1);
-      mbar_init(&sm.st_full[i], 1);
+      mbar_init(&sm.st_full[i], wu::EPI_WARPS);
     }
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -1187,22 +1186,21 @@ __global__ void __launch_bounds__(wu::THREADS, 1) wgrad_update_kernel(
     for (int j = (q > wu::SD - 1 ? q - (wu::SD - 1) : 0); j < q; ++j) mbar_arrive(&sm.wu_empty[j % wu::NS]);
   } else if (warp >= 4) {
     // ---------------- epilogue ----------------
-    const bool leader = threadIdx.x == wu::EPI0;
+    // The epilogue warps do not wait for one another: each waits for the accumulator and for
+    // each chunk itself and hands the chunk on (and, after a tile's last chunk, the accumulator
+    // back) with one mbarrier arrival per warp, so warps at different points of the chunk
+    // sequence overlap their latencies.  No warp can get a ring's length ahead: a slot comes
+    // back only after all of them have arrived.
     const int quarter = warp & 3;
     const int part = (warp - 4) >> 2;   // which CPT columns of each chunk
     const int r = quarter * 32 + lane;  // tile row of this thread
     const SgdParams& sp = args.sgd;
-    // The leader waits; everyone learns the outcome after the named barrier.  Two flag slots
-    // alternate, so the leader never overwrites a flag another thread has yet to read (each
-    // thread reads slot f before it can reach the barrier of the next wait).
-    int fi = 0;
-    auto epi_bar = [] { asm volatile("bar.sync 1, %0;" ::"n"(32 * wu::EPI_WARPS) : "memory"); };
-    auto epi_wait = [&](uint64_t* bar, uint32_t parity) -> bool {
-      if (leader) sm.epi_ok[fi] = mbar_wait(bar, parity) ? 1 : 0;
-      epi_bar();
-      const bool okw = sm.epi_ok[fi] != 0;
-      fi ^= 1;
-      return okw;
+    // Every lane polls (acquiring what the barrier guards); the warp goes on only if all lanes
+    // saw the phase, so a wait that runs out never splits the warp-wide tensor-memory
+    // instructions that follow.
+    auto warp_wait = [&](uint64_t* bar, uint32_t parity) -> bool {
+      const bool okl = mbar_wait(bar, parity);
+      return __all_sync(0xffffffffu, okl);
     };
     const float Gf = (float)args.G;
     const bool pow2 = (args.G & (args.G - 1)) == 0;
@@ -1253,18 +1251,17 @@ __global__ void __launch_bounds__(wu::THREADS, 1) wgrad_update_kernel(
       const bool first = gi == 0, last = gi == per_unit - 1;
       const int ab = i & 1;
       const int nc = wu_chunks(ly->N, n0);
-      if (!epi_wait(&sm.acc_full[ab], (i >> 1) & 1)) {
+      if (!warp_wait(&sm.acc_full[ab], (i >> 1) & 1)) {
         ok = false;
         break;
       }
       asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
       for (int c = 0; c < nc; ++c, ++q) {
         const int sl = q % wu::NS;
-        if (!epi_wait(&sm.wu_full[sl], (q / wu::NS) & 1)) {
+        if (!warp_wait(&sm.wu_full[sl], (q / wu::NS) & 1)) {
           ok = false;
           break;
         }
-        mbar_try_wait(&sm.wu_full[sl], (q / wu::NS) & 1);  // acquire the TMA-written data
         const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
         const uint32_t g_col = (uint32_t)(ab * wu::TN + c * wu::CW + wu::CPT * part);
         // averaging mode: this thread's running pair of the chunk over the replicas so far,
@@ -1282,12 +1279,13 @@ __global__ void __launch_bounds__(wu::THREADS, 1) wgrad_update_kernel(
         uint8_t* brow = sm.wb[sl] + r * 64;
         part_chunk(gv, sc, wrow, urow, brow, first, last);
         if (avg && !last) tmem_st16_nowait(tmem + lane_base + sc_col, sc);
+        // this warp's shared-memory writes reach the TMA stores, its accumulator reads are done
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
         asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-        epi_bar();
-        if (leader) {
-          mbar_arrive(&sm.st_full[sl]);  // the store issuer takes the chunk from here
-          if (c == nc - 1) mbar_arrive(&sm.acc_empty[ab]);  // every row has read the accumulator
+        __syncwarp();
+        if (lane == 0) {
+          mbar_arrive(&sm.st_full[sl]);  // the store issuer takes the chunk once all warps have
+          if (c == nc - 1) mbar_arrive(&sm.acc_empty[ab]);  // ... and the MMA the accumulator
         }
       }
     }

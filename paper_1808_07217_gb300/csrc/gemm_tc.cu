@@ -1332,7 +1332,7 @@ constexpr int MAX_STAGES = 24;  // 4 KB stages (ck = 16)
 constexpr int EPI0 = 128;
 constexpr size_t SMEM_MAX = 227 * 1024;  // dynamic shared memory of one CTA
 constexpr int MAX_ACC = 4;  // accumulator buffers in TMEM
-// barriers, TMEM slot, epilogue flags, and the BatchNorm-backward epilogue's mean / rstd (64 each)
+// barriers, TMEM slot (16 bytes), and the BatchNorm-backward epilogue's mean / rstd (64 each)
 constexpr size_t AUX_BYTES = (2 * MAX_STAGES + 2 * MAX_ACC + 1) * 8 + 16 + 2 * 64 * 4;
 }  // namespace cv
 
@@ -1375,7 +1375,6 @@ __global__ void __launch_bounds__(cv::THREADS, 2) conv_tc_kernel(const __grid_co
   uint64_t* acc_empty = acc_full + cv::MAX_ACC;
   uint64_t* w_full = acc_empty + cv::MAX_ACC;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(w_full + 1);
-  int* epi_ok = reinterpret_cast<int*>(tmem_slot + 1);
   float* bw_mu = reinterpret_cast<float*>(tmem_slot + 4);  // [64]
   float* bw_rs = bw_mu + 64;                                // [64]
 
@@ -1394,7 +1393,7 @@ __global__ void __launch_bounds__(cv::THREADS, 2) conv_tc_kernel(const __grid_co
     }
     for (int i = 0; i < nacc; ++i) {
       mbar_init(&acc_full[i], 1);
-      mbar_init(&acc_empty[i], 1);
+      mbar_init(&acc_empty[i], 4);  // one arrival per epilogue warp
     }
     mbar_init(w_full, 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -1489,15 +1488,13 @@ __global__ void __launch_bounds__(cv::THREADS, 2) conv_tc_kernel(const __grid_co
     }
   } else if (warp >= 4) {
     // ---------------- epilogue ----------------
-    const bool leader = threadIdx.x == cv::EPI0;
+    // The four epilogue warps do not wait for one another: each waits for a tile's accumulator
+    // itself (every lane polls; the warp goes on only if all lanes saw the phase, so a wait that
+    // runs out never splits a warp-wide tensor-memory load) and gives it back with one arrival.
     const int quarter = warp & 3, r = quarter * 32 + lane;
-    int fi = 0;
-    auto epi_wait = [&](uint64_t* bar, uint32_t parity) -> bool {
-      if (leader) epi_ok[fi] = mbar_wait(bar, parity) ? 1 : 0;
-      asm volatile("bar.sync 1, 128;" ::: "memory");
-      const bool okw = epi_ok[fi] != 0;
-      fi ^= 1;
-      return okw;
+    auto warp_wait = [&](uint64_t* bar, uint32_t parity) -> bool {
+      const bool okl = mbar_wait(bar, parity);
+      return __all_sync(0xffffffffu, okl);
     };
     // per-channel BatchNorm statistics of the output pixels (forward convolutions), per
     // epilogue warp: lanes 2 j, 2 j + 1 keep channel 16 ci + j's running count, mean and M2 over
@@ -1521,10 +1518,10 @@ __global__ void __launch_bounds__(cv::THREADS, 2) conv_tc_kernel(const __grid_co
     int i = 0;
     for (int tile = blockIdx.x; tile < tiles; tile += cpr, ++i) {
       const int ab = i % nacc;
-      if (!epi_wait(&acc_full[ab], (i / nacc) & 1)) break;
+      if (!warp_wait(&acc_full[ab], (i / nacc) & 1)) break;
       asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
       // strip form: this tile's MMAs (and so its reads of its input stage) are complete
-      if (a.strip && leader) mbar_arrive(&empty[i % nst]);
+      if (a.strip && quarter == 0 && lane == 0) mbar_arrive(&empty[i % nst]);
       int64_t dst = (int64_t)tile * BM + r;
       if (a.dst_h > 0) {
         const int pp = tile * BM + r, img = pp / per_img, rem = pp - img * per_img;
@@ -1664,8 +1661,8 @@ __global__ void __launch_bounds__(cv::THREADS, 2) conv_tc_kernel(const __grid_co
       }
       if (with_stats) run_n += 32.f;
       asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-      asm volatile("bar.sync 1, 128;" ::: "memory");
-      if (leader) mbar_arrive(&acc_empty[ab]);
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&acc_empty[ab]);
     }
     if (with_bwd && !(lane & 1)) {
 #pragma unroll

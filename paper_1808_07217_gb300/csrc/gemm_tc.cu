@@ -176,6 +176,22 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
   for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
 }
 
+// Sums 16 values per lane over the 32 lanes of a warp in four halving exchanges and one final
+// exchange: afterwards lane l holds the warp's sum of value l / 2 (lanes 2 j and 2 j + 1 agree).
+__device__ __forceinline__ float warp_colsum16(float (&v)[16], int lane) {
+#pragma unroll
+  for (int w = 8; w >= 1; w >>= 1) {
+    const bool up = (lane & (2 * w)) != 0;
+#pragma unroll
+    for (int i = 0; i < w; ++i) {
+      const float send = up ? v[i] : v[i + w];
+      const float keep = up ? v[i + w] : v[i];
+      v[i] = keep + __shfl_xor_sync(0xffffffffu, send, 2 * w);
+    }
+  }
+  return v[0] + __shfl_xor_sync(0xffffffffu, v[0], 1);
+}
+
 // The local update on four consecutive parameters (fused weight-gradient epilogue); SG fixes at
 // compile time whether the signSGD variant's sign is taken (it must equal sp.sign != 0).
 template <bool SG>
@@ -562,26 +578,215 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
 //   warp 0      TMA producer: A (128 x 64) and B (PBN x 64) k-blocks into a PST-stage ring
 //   warp 1      MMA issuer: tcgen05.mma (M = 128, N = PBN, K = 16), accumulator (tile & 1)
 //   warp 2      TMEM allocation (2 PBN columns)
-//   warps 4-7   epilogue (epilogue_tile: bias / ReLU / ReLU mask, column sums + bias update),
-//               staged through a shared-memory tile of its own
+//   warps 4-7   epilogue (pt_epilogue_rows: bias / ReLU / ReLU mask; column sums + bias
+//               update): each thread writes its tile row straight from registers, each warp
+//               waits for the accumulator and hands it back by itself
 // 128 x 256 tiles halve the shared-memory operand bytes per MMA of the 64-wide one-tile kernel
 // (whose N = 64 MMAs read as many operand bytes as they compute).
 namespace pt {
 constexpr int PBN = 256;
-constexpr int PST = 3;
+constexpr int PST = 4;  // 192 KB of operands in flight: the epilogue needs no staging tile
 constexpr int THREADS = 256;
-constexpr int STG_FLOATS = BM * (64 + 4) + 2 * 64;
 }  // namespace pt
 
 struct PtSmem {
   uint8_t a[pt::PST][BM * BK * 2];       // 16 KB each (1024-aligned)
   uint8_t b[pt::PST][pt::PBN * BK * 2];  // 32 KB each
-  float stg[pt::STG_FLOATS];
+  float hs[2][4][pt::PBN];  // bias column sums: per tile parity, per epilogue warp
   uint64_t full[pt::PST], empty[pt::PST];
   uint64_t acc_full[2], acc_empty[2];
   uint32_t tmem_base;
-  int epi_ok[2];
+  int fail;  // an epilogue warp's accumulator wait ran out (column-sum mode)
 };
+
+// One thread's 64 consecutive accumulator columns of its TMEM lane: two 32-column loads, one wait.
+__device__ __forceinline__ void tmem_ld64(uint32_t taddr, float (&v)[64]) {
+  uint32_t r[64];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,"
+      "%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%64];\n"
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%32,%33,%34,%35,%36,%37,%38,%39,%40,%41,%42,%43,%44,"
+      "%45,%46,%47,%48,%49,%50,%51,%52,%53,%54,%55,%56,%57,%58,%59,%60,%61,%62,%63}, [%65];\n"
+      "tcgen05.wait::ld.sync.aligned;"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]),
+        "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]),
+        "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31]), "=r"(r[32]), "=r"(r[33]), "=r"(r[34]),
+        "=r"(r[35]), "=r"(r[36]), "=r"(r[37]), "=r"(r[38]), "=r"(r[39]), "=r"(r[40]), "=r"(r[41]),
+        "=r"(r[42]), "=r"(r[43]), "=r"(r[44]), "=r"(r[45]), "=r"(r[46]), "=r"(r[47]), "=r"(r[48]),
+        "=r"(r[49]), "=r"(r[50]), "=r"(r[51]), "=r"(r[52]), "=r"(r[53]), "=r"(r[54]), "=r"(r[55]),
+        "=r"(r[56]), "=r"(r[57]), "=r"(r[58]), "=r"(r[59]), "=r"(r[60]), "=r"(r[61]), "=r"(r[62]),
+        "=r"(r[63])
+      : "r"(taddr), "r"(taddr + 32u)
+      : "memory");
+#pragma unroll
+  for (int i = 0; i < 64; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// Sixteen consecutive outputs of one row: 32-byte stores where the row is aligned and whole,
+// else element by element up to the matrix edge.
+__device__ __forceinline__ void store_row16(void* C, bool c_bf16, int64_t off, int n, int N,
+                                            const float (&x)[16]) {
+  if (c_bf16) {
+    uint16_t* out = reinterpret_cast<uint16_t*>(C) + off;
+    if (n + 16 <= N && (reinterpret_cast<uintptr_t>(out) & 31) == 0) {
+      uint32_t w[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) w[j] = (uint32_t)f2bf(x[2 * j]) | ((uint32_t)f2bf(x[2 * j + 1]) << 16);
+      asm volatile("st.global.v8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"l"(out), "r"(w[0]),
+                   "r"(w[1]), "r"(w[2]), "r"(w[3]), "r"(w[4]), "r"(w[5]), "r"(w[6]), "r"(w[7])
+                   : "memory");
+    } else {
+#pragma unroll
+      for (int i = 0; i < 16; ++i)
+        if (n + i < N) out[i] = f2bf(x[i]);
+    }
+  } else {
+    float* out = reinterpret_cast<float*>(C) + off;
+    if (n + 16 <= N && (reinterpret_cast<uintptr_t>(out) & 31) == 0) {
+#pragma unroll
+      for (int j = 0; j < 2; ++j)
+        asm volatile("st.global.v8.f32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"l"(out + 8 * j),
+                     "f"(x[8 * j]), "f"(x[8 * j + 1]), "f"(x[8 * j + 2]), "f"(x[8 * j + 3]),
+                     "f"(x[8 * j + 4]), "f"(x[8 * j + 5]), "f"(x[8 * j + 6]), "f"(x[8 * j + 7])
+                     : "memory");
+    } else {
+#pragma unroll
+      for (int i = 0; i < 16; ++i)
+        if (n + i < N) out[i] = x[i];
+    }
+  }
+}
+
+// The persistent GEMM's epilogue of one 128 x BN tile for one epilogue thread: tile row et (TMEM
+// lane et) leaves TMEM 64 columns at a time and is written straight from registers, 16 columns
+// per store, with the epilogue_tile arithmetic: bias (+ ReLU) or the ReLU mask of the stored
+// activation (the row's 64 mask values requested before the accumulator loads).  With hs_warp
+// (bias_colsum) the stored values -- rounded to bf16 when C is bf16 -- are also summed over the
+// warp's 32 rows, per column, by a fixed butterfly (rows past M add nothing); hs_warp[c] gets
+// column c's partial.
+template <int BN>
+__device__ __forceinline__ void pt_epilogue_rows(const TcGemmArgs& args, int et, int lane,
+                                                 uint32_t tmem_acc, int g, int m0, int n0,
+                                                 float* hs_warp) {
+  const int m = m0 + et;
+  const bool row_ok = m < args.M;
+  const int epi = args.epi;
+  const bool has_bias = epi == EPI_BIAS || epi == EPI_BIAS_RELU;
+  const float* bias = has_bias ? args.bias + (int64_t)g * args.bias_gs : nullptr;
+  const int64_t coff = (int64_t)g * args.c_gs + (int64_t)m * args.c_rs;
+  const int64_t moff = (int64_t)g * args.mask_gs + (int64_t)m * args.mask_rs;
+  const uint32_t lane_base = (uint32_t)(et & ~31) << 16;
+  for (int cc = 0; cc < BN; cc += 64) {
+    if (n0 + cc >= args.N) break;  // uniform over the CTA
+    const int nc = n0 + cc;
+    // the chunk's bf16 mask words (two values each) when the row is whole and 16-byte aligned
+    uint32_t mw[32];
+    const uint16_t* mrow = epi == EPI_MASK && args.mask_bf16
+                               ? reinterpret_cast<const uint16_t*>(args.mask) + moff + nc
+                               : nullptr;
+    const bool mfast = mrow && row_ok && nc + 64 <= args.N &&
+                       (reinterpret_cast<uintptr_t>(mrow) & 15) == 0;
+    if (mfast) {
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        const uint4 t = __ldg(reinterpret_cast<const uint4*>(mrow) + i);
+        mw[4 * i] = t.x;
+        mw[4 * i + 1] = t.y;
+        mw[4 * i + 2] = t.z;
+        mw[4 * i + 3] = t.w;
+      }
+    }
+    float v[64];
+    tmem_ld64(tmem_acc + lane_base + (uint32_t)cc, v);
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const int nb = nc + 16 * q;
+      float x[16];
+#pragma unroll
+      for (int i = 0; i < 16; ++i) x[i] = v[16 * q + i];
+      if (has_bias) {
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          const int n = nb + i;
+          const float t = x[i] + (n < args.N ? __ldg(bias + n) : 0.f);
+          x[i] = (epi == EPI_BIAS_RELU) ? fmaxf(t, 0.f) : t;
+        }
+      } else if (epi == EPI_MASK) {
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          float mv;
+          if (mfast) {
+            const uint32_t w = mw[8 * q + (i >> 1)];
+            mv = bf2f((uint16_t)((i & 1) ? (w >> 16) : (w & 0xffffu)));
+          } else {
+            const int n = nb + i;
+            mv = !(row_ok && n < args.N) ? 0.f
+                 : args.mask_bf16 ? bf2f(reinterpret_cast<const uint16_t*>(args.mask)[moff + n])
+                                  : reinterpret_cast<const float*>(args.mask)[moff + n];
+          }
+          x[i] = mv > 0.f ? x[i] : 0.f;
+        }
+      }
+      if (row_ok && nb < args.N) store_row16(args.C, args.c_bf16, coff + nb, nb, args.N, x);
+      if (hs_warp) {
+        float t[16];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) t[i] = !row_ok ? 0.f : (args.c_bf16 ? bf2f(f2bf(x[i])) : x[i]);
+        const float sum = warp_colsum16(t, lane);
+        if (!(lane & 1)) hs_warp[cc + 16 * q + (lane >> 1)] = sum;
+      }
+    }
+  }
+}
+
+// The bias of the layer below, for the column-sum mode: each epilogue thread takes columns
+// et + 128 i of the tile; their parameters are requested before the accumulator wait.
+template <int BN>
+__device__ __forceinline__ void pt_bias_prefetch(const TcGemmArgs& args, int et, int g, int n0,
+                                                 float (&bsw)[BN / 128], float (&bsu)[BN / 128]) {
+#pragma unroll
+  for (int i = 0; i < BN / 128; ++i) {
+    const int n = n0 + 128 * i + et;
+    const bool v = args.bias_colsum && args.bsgd.w && n < args.N;
+    const int64_t k = (int64_t)g * args.bias_gs + n;
+    bsw[i] = v ? args.bsgd.w[k] : 0.f;
+    bsu[i] = v && args.bsgd.u ? args.bsgd.u[k] : 0.f;
+  }
+}
+
+// After the four warps' partials are in hs (this tile's buffer): the bias gradient of each of
+// this thread's columns, (warp 0 + warp 1) + (warp 2 + warp 3), and its local update (or the
+// gradient itself without bsgd.w).
+template <int BN>
+__device__ __forceinline__ void pt_bias_update(const TcGemmArgs& args, int et, int g, int n0,
+                                               const float (*hs)[BN], const float (&bsw)[BN / 128],
+                                               const float (&bsu)[BN / 128]) {
+#pragma unroll
+  for (int i = 0; i < BN / 128; ++i) {
+    const int c = 128 * i + et, n = n0 + c;
+    if (n >= args.N) continue;
+    const float gb = __fadd_rn(__fadd_rn(hs[0][c], hs[1][c]), __fadd_rn(hs[2][c], hs[3][c]));
+    const int64_t k = (int64_t)g * args.bias_gs + n;
+    if (!args.bsgd.w) {
+      args.bias_grad[k] = gb;
+      continue;
+    }
+    const SgdParams& sp = args.bsgd;
+    float w = bsw[i], u = bsu[i];
+    const bool sg = sp.sign != 0;
+    if (sp.mom == 0.f)
+      sgd_elem<false, false>(w, u, gb, sp.lr, 0.f, sp.wd, sg);
+    else if (sp.nesterov)
+      sgd_elem<true, true>(w, u, gb, sp.lr, sp.mom, sp.wd, sg);
+    else
+      sgd_elem<true, false>(w, u, gb, sp.lr, sp.mom, sp.wd, sg);
+    sp.w[k] = w;
+    if (sp.u) sp.u[k] = u;
+    if (sp.wb) sp.wb[k] = f2bf(w);
+  }
+}
 
 __global__ void __launch_bounds__(pt::THREADS, 1) gemm_pt_kernel(const __grid_constant__ TcGemmArgs args) {
   extern __shared__ uint8_t smem_raw[];
@@ -609,8 +814,9 @@ __global__ void __launch_bounds__(pt::THREADS, 1) gemm_pt_kernel(const __grid_co
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&sm.acc_full[i], 1);
-      mbar_init(&sm.acc_empty[i], 1);
+      mbar_init(&sm.acc_empty[i], 4);  // one arrival per epilogue warp
     }
+    sm.fail = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
   }
@@ -698,16 +904,23 @@ __global__ void __launch_bounds__(pt::THREADS, 1) gemm_pt_kernel(const __grid_co
     }
   } else if (warp >= 4) {
     // ---------------- epilogue ----------------
-    const int et = threadIdx.x - 128;
-    const bool leader = et == 0;
-    int fi = 0;
+    // Each warp waits for the accumulator by itself (every lane polls; the warp goes on only if
+    // all lanes saw the phase) and gives it back with one arrival.  Only the column-sum mode
+    // brings the four warps together, once per tile; there a wait that ran out is shared through
+    // sm.fail before that barrier, so all four leave together.
+    const int et = threadIdx.x - 128, quarter = warp & 3;
+    const bool colsum = args.bias_colsum;
+    auto warp_wait = [&](uint64_t* bar, uint32_t parity) -> bool {
+      const bool okl = mbar_wait(bar, parity);
+      return __all_sync(0xffffffffu, okl);
+    };
     int i = 0;
     for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++i) {
       int g, m0, n0;
       coords(t, g, m0, n0);
       const int ab = i & 1;
-      float bsw[PBN / 64], bsu[PBN / 64];
-      epilogue_bias_prefetch<PBN>(args, et, g, n0, bsw, bsu);
+      float bsw[PBN / 128], bsu[PBN / 128];
+      pt_bias_prefetch<PBN>(args, et, g, n0, bsw, bsu);
       if (args.epi == EPI_MASK && args.mask && m0 + et < args.M) {
         // this thread's row of the tile's ReLU mask (the stored activation) into L2 while the
         // tile's products run, so that the copy-out's mask loads do not each wait on DRAM
@@ -717,17 +930,27 @@ __global__ void __launch_bounds__(pt::THREADS, 1) gemm_pt_kernel(const __grid_co
                            ((int64_t)g * args.mask_gs + (int64_t)(m0 + et) * args.mask_rs + n0) * esz;
         for (int b = 0; b < ncols * esz; b += 128) asm volatile("prefetch.global.L2 [%0];" ::"l"(rowp + b));
       }
-      if (leader) sm.epi_ok[fi] = mbar_wait(&sm.acc_full[ab], (i >> 1) & 1) ? 1 : 0;
-      asm volatile("bar.sync 1, 128;" ::: "memory");
-      const bool okw = sm.epi_ok[fi] != 0;
-      fi ^= 1;
-      if (!okw) break;
-      asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-      const int64_t c_base = (int64_t)g * args.c_gs;
-      epilogue_tile<PBN>(args, et, tmem + (uint32_t)(ab * PBN), g, m0, n0, c_base, sm.stg, bsw, bsu);
+      const bool okw = warp_wait(&sm.acc_full[ab], (i >> 1) & 1);
+      const uint32_t acc = tmem + (uint32_t)(ab * PBN);
+      if (!colsum) {
+        if (!okw) break;
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        pt_epilogue_rows<PBN>(args, et, lane, acc, g, m0, n0, nullptr);
+      } else {
+        if (okw) {
+          asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+          pt_epilogue_rows<PBN>(args, et, lane, acc, g, m0, n0, sm.hs[ab][quarter]);
+        } else if (lane == 0) {
+          sm.fail = 1;
+        }
+        asm volatile("bar.sync 1, 128;" ::: "memory");
+        if (*reinterpret_cast<volatile int*>(&sm.fail)) break;
+        // hs[ab] is written again two tiles on, after every warp has passed the next barrier
+        pt_bias_update<PBN>(args, et, g, n0, sm.hs[ab], bsw, bsu);
+      }
       asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-      asm volatile("bar.sync 1, 128;" ::: "memory");
-      if (leader) mbar_arrive(&sm.acc_empty[ab]);  // every row has read the accumulator
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&sm.acc_empty[ab]);  // this warp's rows have left the accumulator
     }
   }
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
@@ -1336,21 +1559,6 @@ constexpr int MAX_ACC = 4;  // accumulator buffers in TMEM
 constexpr size_t AUX_BYTES = (2 * MAX_STAGES + 2 * MAX_ACC + 1) * 8 + 16 + 2 * 64 * 4;
 }  // namespace cv
 
-// Sums 16 values per lane over the 32 lanes of a warp in four halving exchanges and one final
-// exchange: afterwards lane l holds the warp's sum of value l / 2 (lanes 2 j and 2 j + 1 agree).
-__device__ __forceinline__ float warp_colsum16(float (&v)[16], int lane) {
-#pragma unroll
-  for (int w = 8; w >= 1; w >>= 1) {
-    const bool up = (lane & (2 * w)) != 0;
-#pragma unroll
-    for (int i = 0; i < w; ++i) {
-      const float send = up ? v[i] : v[i + w];
-      const float keep = up ? v[i + w] : v[i];
-      v[i] = keep + __shfl_xor_sync(0xffffffffu, send, 2 * w);
-    }
-  }
-  return v[0] + __shfl_xor_sync(0xffffffffu, v[0], 1);
-}
 
 __global__ void __launch_bounds__(cv::THREADS, 2) conv_tc_kernel(const __grid_constant__ ConvArgs a) {
   extern __shared__ uint8_t smem_raw[];

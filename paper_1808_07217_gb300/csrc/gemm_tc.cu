@@ -226,178 +226,219 @@ struct Smem {
   uint32_t tmem_base;
 };
 
-// ---- epilogue of one 128 x BN output tile, shared by the one-tile and the persistent GEMM ----
-// 128 epilogue threads (et = 0 .. 127, named barrier 1): the tile leaves TMEM (columns tmem_acc
-// onwards) in 64-column chunks: each thread takes its row's 64 fp32 values (bias / ReLU
-// applied), writes them to the padded staging tile stg ([128][68] floats + 128 for the column
-// sums), and the threads then store the chunk row-contiguously (a warp writes two 256-byte row
-// segments per instruction), applying the ReLU mask from a coalesced read of the stored
-// activation.
-// The bias that the column sums update (threads 0-63, one column of each 64-column chunk;
-// nothing else writes it) is requested first, so its loads overlap the wait for the accumulator.
-template <int BN>
-__device__ __forceinline__ void epilogue_bias_prefetch(const TcGemmArgs& args, int et, int g,
-                                                       int n0, float (&bsw)[BN / 64],
-                                                       float (&bsu)[BN / 64]) {
+// ---- GEMM epilogue (one-tile and persistent kernels) ----
+// One thread's 32 consecutive accumulator columns of its TMEM lane, one wait.
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,"
+      "%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];\n"
+      "tcgen05.wait::ld.sync.aligned;"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]),
+        "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]),
+        "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr)
+      : "memory");
 #pragma unroll
-  for (int i = 0; i < BN / 64; ++i) {
-    const int n = n0 + 64 * i + (int)et;
-    const bool v = args.bias_colsum && args.bsgd.w && et < 64 && n < args.N;
+  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// One thread's 64 consecutive accumulator columns of its TMEM lane: two 32-column loads, one wait.
+__device__ __forceinline__ void tmem_ld64(uint32_t taddr, float (&v)[64]) {
+  uint32_t r[64];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,"
+      "%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%64];\n"
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%32,%33,%34,%35,%36,%37,%38,%39,%40,%41,%42,%43,%44,"
+      "%45,%46,%47,%48,%49,%50,%51,%52,%53,%54,%55,%56,%57,%58,%59,%60,%61,%62,%63}, [%65];\n"
+      "tcgen05.wait::ld.sync.aligned;"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]),
+        "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]),
+        "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31]), "=r"(r[32]), "=r"(r[33]), "=r"(r[34]),
+        "=r"(r[35]), "=r"(r[36]), "=r"(r[37]), "=r"(r[38]), "=r"(r[39]), "=r"(r[40]), "=r"(r[41]),
+        "=r"(r[42]), "=r"(r[43]), "=r"(r[44]), "=r"(r[45]), "=r"(r[46]), "=r"(r[47]), "=r"(r[48]),
+        "=r"(r[49]), "=r"(r[50]), "=r"(r[51]), "=r"(r[52]), "=r"(r[53]), "=r"(r[54]), "=r"(r[55]),
+        "=r"(r[56]), "=r"(r[57]), "=r"(r[58]), "=r"(r[59]), "=r"(r[60]), "=r"(r[61]), "=r"(r[62]),
+        "=r"(r[63])
+      : "r"(taddr), "r"(taddr + 32u)
+      : "memory");
+#pragma unroll
+  for (int i = 0; i < 64; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// Sixteen consecutive outputs of one row: 32-byte stores where the row is aligned and whole,
+// else element by element up to the matrix edge.
+__device__ __forceinline__ void store_row16(void* C, bool c_bf16, int64_t off, int n, int N,
+                                            const float (&x)[16]) {
+  if (c_bf16) {
+    uint16_t* out = reinterpret_cast<uint16_t*>(C) + off;
+    if (n + 16 <= N && (reinterpret_cast<uintptr_t>(out) & 31) == 0) {
+      uint32_t w[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) w[j] = (uint32_t)f2bf(x[2 * j]) | ((uint32_t)f2bf(x[2 * j + 1]) << 16);
+      asm volatile("st.global.v8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"l"(out), "r"(w[0]),
+                   "r"(w[1]), "r"(w[2]), "r"(w[3]), "r"(w[4]), "r"(w[5]), "r"(w[6]), "r"(w[7])
+                   : "memory");
+    } else {
+#pragma unroll
+      for (int i = 0; i < 16; ++i)
+        if (n + i < N) out[i] = f2bf(x[i]);
+    }
+  } else {
+    float* out = reinterpret_cast<float*>(C) + off;
+    if (n + 16 <= N && (reinterpret_cast<uintptr_t>(out) & 31) == 0) {
+#pragma unroll
+      for (int j = 0; j < 2; ++j)
+        asm volatile("st.global.v8.f32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"l"(out + 8 * j),
+                     "f"(x[8 * j]), "f"(x[8 * j + 1]), "f"(x[8 * j + 2]), "f"(x[8 * j + 3]),
+                     "f"(x[8 * j + 4]), "f"(x[8 * j + 5]), "f"(x[8 * j + 6]), "f"(x[8 * j + 7])
+                     : "memory");
+    } else {
+#pragma unroll
+      for (int i = 0; i < 16; ++i)
+        if (n + i < N) out[i] = x[i];
+    }
+  }
+}
+
+// The GEMM epilogue of one 128 x BN tile for one epilogue thread: tile row et (TMEM lane et)
+// leaves TMEM CW (32 or 64) columns at a time and is written straight from registers, 16 columns
+// per store: C(m, n) at C + c_base + m c_rs + n, with bias (+ ReLU) or the ReLU mask of the stored
+// activation applied (the row's CW mask values requested before the accumulator loads).  With
+// hs_warp (bias_colsum) the stored values -- rounded to bf16 when C is bf16 -- are also summed
+// over the warp's 32 rows, per column, by a fixed butterfly (rows past M add nothing); hs_warp[c]
+// gets column c's partial.
+template <int BN, int CW>
+__device__ __forceinline__ void epilogue_rows(const TcGemmArgs& args, int et, int lane,
+                                              uint32_t tmem_acc, int g, int m0, int n0,
+                                              int64_t c_base, float* hs_warp) {
+  static_assert(CW == 32 || CW == 64, "chunk width");
+  const int m = m0 + et;
+  const bool row_ok = m < args.M;
+  const int epi = args.epi;
+  const bool has_bias = epi == EPI_BIAS || epi == EPI_BIAS_RELU;
+  const float* bias = has_bias ? args.bias + (int64_t)g * args.bias_gs : nullptr;
+  const int64_t coff = c_base + (int64_t)m * args.c_rs;
+  const int64_t moff = (int64_t)g * args.mask_gs + (int64_t)m * args.mask_rs;
+  const uint32_t lane_base = (uint32_t)(et & ~31) << 16;
+  for (int cc = 0; cc < BN; cc += CW) {
+    if (n0 + cc >= args.N) break;  // uniform over the CTA
+    const int nc = n0 + cc;
+    // the chunk's bf16 mask words (two values each) when the row is whole and 16-byte aligned
+    uint32_t mw[CW / 2];
+    const uint16_t* mrow = epi == EPI_MASK && args.mask_bf16
+                               ? reinterpret_cast<const uint16_t*>(args.mask) + moff + nc
+                               : nullptr;
+    const bool mfast = mrow && row_ok && nc + CW <= args.N &&
+                       (reinterpret_cast<uintptr_t>(mrow) & 15) == 0;
+    if (mfast) {
+#pragma unroll
+      for (int i = 0; i < CW / 8; ++i) {
+        const uint4 t = __ldg(reinterpret_cast<const uint4*>(mrow) + i);
+        mw[4 * i] = t.x;
+        mw[4 * i + 1] = t.y;
+        mw[4 * i + 2] = t.z;
+        mw[4 * i + 3] = t.w;
+      }
+    }
+    float v[CW];
+    if constexpr (CW == 64)
+      tmem_ld64(tmem_acc + lane_base + (uint32_t)cc, v);
+    else
+      tmem_ld32(tmem_acc + lane_base + (uint32_t)cc, v);
+#pragma unroll
+    for (int q = 0; q < CW / 16; ++q) {
+      const int nb = nc + 16 * q;
+      float x[16];
+#pragma unroll
+      for (int i = 0; i < 16; ++i) x[i] = v[16 * q + i];
+      if (has_bias) {
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          const int n = nb + i;
+          const float t = x[i] + (n < args.N ? __ldg(bias + n) : 0.f);
+          x[i] = (epi == EPI_BIAS_RELU) ? fmaxf(t, 0.f) : t;
+        }
+      } else if (epi == EPI_MASK) {
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          float mv;
+          if (mfast) {
+            const uint32_t w = mw[8 * q + (i >> 1)];
+            mv = bf2f((uint16_t)((i & 1) ? (w >> 16) : (w & 0xffffu)));
+          } else {
+            const int n = nb + i;
+            mv = !(row_ok && n < args.N) ? 0.f
+                 : args.mask_bf16 ? bf2f(reinterpret_cast<const uint16_t*>(args.mask)[moff + n])
+                                  : reinterpret_cast<const float*>(args.mask)[moff + n];
+          }
+          x[i] = mv > 0.f ? x[i] : 0.f;
+        }
+      }
+      if (row_ok && nb < args.N) store_row16(args.C, args.c_bf16, coff + nb, nb, args.N, x);
+      if (hs_warp) {
+        float t[16];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) t[i] = !row_ok ? 0.f : (args.c_bf16 ? bf2f(f2bf(x[i])) : x[i]);
+        const float sum = warp_colsum16(t, lane);
+        if (!(lane & 1)) hs_warp[cc + 16 * q + (lane >> 1)] = sum;
+      }
+    }
+  }
+}
+
+// The bias of the layer below, for the column-sum mode: each of the 128 epilogue threads takes
+// columns et + 128 i of the tile; their parameters are requested before the accumulator wait.
+template <int BN>
+constexpr int kBiasCols = (BN + 127) / 128;  // columns per epilogue thread
+
+template <int BN>
+__device__ __forceinline__ void bias_prefetch(const TcGemmArgs& args, int et, int g, int n0,
+                                              float (&bsw)[kBiasCols<BN>],
+                                              float (&bsu)[kBiasCols<BN>]) {
+#pragma unroll
+  for (int i = 0; i < kBiasCols<BN>; ++i) {
+    const int c = 128 * i + et, n = n0 + c;
+    const bool v = args.bias_colsum && args.bsgd.w && c < BN && n < args.N;
     const int64_t k = (int64_t)g * args.bias_gs + n;
     bsw[i] = v ? args.bsgd.w[k] : 0.f;
     bsu[i] = v && args.bsgd.u ? args.bsgd.u[k] : 0.f;
   }
 }
 
+// After the four warps' partials are in hs (this tile's buffer): the bias gradient of each of
+// this thread's columns, (warp 0 + warp 1) + (warp 2 + warp 3), and its local update (or the
+// gradient itself without bsgd.w).
 template <int BN>
-__device__ __forceinline__ void epilogue_tile(const TcGemmArgs& args, int et, uint32_t tmem_acc,
-                                              int g, int m0, int n0, int64_t c_base, float* stg,
-                                              const float (&bsw)[BN / 64],
-                                              const float (&bsu)[BN / 64]) {
-  constexpr int CW = 64, PITCH = CW + 4;  // staged chunk width and row pitch (floats)
-  const int r = et;  // tile row owned in the TMEM phase (TMEM lane quarter et / 32)
-  const float* bias = args.bias ? args.bias + (int64_t)g * args.bias_gs : nullptr;
-  const int epi = args.epi;
-  for (int cc = 0; cc < BN; cc += CW) {
-    if (n0 + cc >= args.N) break;  // block-uniform
+__device__ __forceinline__ void bias_update(const TcGemmArgs& args, int et, int g, int n0,
+                                            const float (*hs)[BN], const float (&bsw)[kBiasCols<BN>],
+                                            const float (&bsu)[kBiasCols<BN>]) {
 #pragma unroll
-    for (int q = 0; q < CW / 16; ++q) {
-      float v[16];
-      tmem_ld16(tmem_acc + ((uint32_t)(et & ~31) << 16) + (uint32_t)(cc + 16 * q), v);
-      if (epi == EPI_BIAS || epi == EPI_BIAS_RELU) {
-#pragma unroll
-        for (int i = 0; i < 16; ++i) {
-          const int n = n0 + cc + 16 * q + i;
-          float x = v[i] + (n < args.N ? __ldg(bias + n) : 0.f);
-          v[i] = (epi == EPI_BIAS_RELU) ? fmaxf(x, 0.f) : x;
-        }
-      }
-      float4* dst = reinterpret_cast<float4*>(stg + r * PITCH + 16 * q);
-#pragma unroll
-      for (int i = 0; i < 4; ++i) dst[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+  for (int i = 0; i < kBiasCols<BN>; ++i) {
+    const int c = 128 * i + et, n = n0 + c;
+    if (c >= BN || n >= args.N) continue;
+    const float gb = __fadd_rn(__fadd_rn(hs[0][c], hs[1][c]), __fadd_rn(hs[2][c], hs[3][c]));
+    const int64_t k = (int64_t)g * args.bias_gs + n;
+    if (!args.bsgd.w) {
+      args.bias_grad[k] = gb;
+      continue;
     }
-    asm volatile("bar.sync 1, 128;" ::: "memory");
-    // copy-out: item = (row, 4-column group), 16 groups per 64-column row.  Each thread takes
-    // UNR items at a time and issues all their mask loads before any arithmetic, so several
-    // hundred bytes per thread are in flight.
-    constexpr int UNR = 8, ITEMS = BM * (CW / 4);
-    for (int base = et; base < ITEMS; base += 128 * UNR) {
-      float4 x[UNR], a0[UNR];
-      int64_t off[UNR];
-      int nn[UNR];
-      bool ok[UNR];
-#pragma unroll
-      for (int q = 0; q < UNR; ++q) {
-        const int it = base + q * 128;
-        const int row = it / (CW / 4), grp = it % (CW / 4);
-        const int m = m0 + row, n = n0 + cc + grp * 4;
-        ok[q] = it < ITEMS && m < args.M && n < args.N;
-        nn[q] = n;
-        off[q] = c_base + (int64_t)m * args.c_rs + n;
-        a0[q] = make_float4(0.f, 0.f, 0.f, 0.f);
-        if (!ok[q]) continue;
-        x[q] = *reinterpret_cast<const float4*>(stg + row * PITCH + grp * 4);
-        const bool full4 = n + 4 <= args.N;
-        if (epi == EPI_MASK) {
-          const int64_t moff = (int64_t)g * args.mask_gs + (int64_t)m * args.mask_rs + n;
-          if (args.mask_bf16) {
-            const uint16_t* mp = reinterpret_cast<const uint16_t*>(args.mask) + moff;
-            if (full4 && ((reinterpret_cast<uintptr_t>(mp) & 7) == 0)) {
-              const uint2 u = __ldg(reinterpret_cast<const uint2*>(mp));
-              a0[q] = make_float4(bf2f((uint16_t)(u.x & 0xffff)), bf2f((uint16_t)(u.x >> 16)),
-                                  bf2f((uint16_t)(u.y & 0xffff)), bf2f((uint16_t)(u.y >> 16)));
-            } else {
-              float t[4] = {0.f, 0.f, 0.f, 0.f};
-              for (int i = 0; i < 4 && n + i < args.N; ++i) t[i] = bf2f(mp[i]);
-              a0[q] = make_float4(t[0], t[1], t[2], t[3]);
-            }
-          } else {
-            const float* mp = reinterpret_cast<const float*>(args.mask) + moff;
-            float t[4] = {0.f, 0.f, 0.f, 0.f};
-            for (int i = 0; i < 4 && n + i < args.N; ++i) t[i] = mp[i];
-            a0[q] = make_float4(t[0], t[1], t[2], t[3]);
-          }
-        }
-      }
-#pragma unroll
-      for (int q = 0; q < UNR; ++q) {
-        if (!ok[q]) continue;
-        const int n = nn[q];
-        const bool full4 = n + 4 <= args.N;
-        float4 v = x[q];
-        if (epi == EPI_MASK) {
-          v.x = a0[q].x > 0.f ? v.x : 0.f;
-          v.y = a0[q].y > 0.f ? v.y : 0.f;
-          v.z = a0[q].z > 0.f ? v.z : 0.f;
-          v.w = a0[q].w > 0.f ? v.w : 0.f;
-        }
-        if (args.bias_colsum) {
-          // keep the stored (rounded) value for the column sums below; each item is this
-          // thread's alone
-          const int it = base + q * 128;
-          const float4 r4 = args.c_bf16 ? make_float4(bf2f(f2bf(v.x)), bf2f(f2bf(v.y)),
-                                                      bf2f(f2bf(v.z)), bf2f(f2bf(v.w)))
-                                        : v;
-          *reinterpret_cast<float4*>(stg + (it / (CW / 4)) * PITCH + (it % (CW / 4)) * 4) = r4;
-        }
-        if (args.c_bf16) {
-          uint16_t* out = reinterpret_cast<uint16_t*>(args.C) + off[q];
-          if (full4 && ((reinterpret_cast<uintptr_t>(out) & 7) == 0)) {
-            uint2 o;
-            o.x = (uint32_t)f2bf(v.x) | ((uint32_t)f2bf(v.y) << 16);
-            o.y = (uint32_t)f2bf(v.z) | ((uint32_t)f2bf(v.w) << 16);
-            *reinterpret_cast<uint2*>(out) = o;
-          } else {
-            const float xs[4] = {v.x, v.y, v.z, v.w};
-            for (int i = 0; i < 4 && n + i < args.N; ++i) out[i] = f2bf(xs[i]);
-          }
-        } else {
-          float* out = reinterpret_cast<float*>(args.C) + off[q];
-          if (full4 && ((reinterpret_cast<uintptr_t>(out) & 15) == 0)) {
-            *reinterpret_cast<float4*>(out) = v;
-          } else {
-            const float xs[4] = {v.x, v.y, v.z, v.w};
-            for (int i = 0; i < 4 && n + i < args.N; ++i) out[i] = xs[i];
-          }
-        }
-      }
-    }
-    asm volatile("bar.sync 1, 128;" ::: "memory");
-    if (args.bias_colsum) {
-      // Bias gradient of the layer this data gradient feeds: the sum over all rows (the tile
-      // holds the whole mini-batch) of the stored values, per column; two row halves per
-      // column, added in a fixed order, then the local update of that bias (or its gradient).
-      float* hs = stg + BM * PITCH;  // 2 x 64 partial sums after the staged tile
-      const int col = et & (CW - 1), half = et / CW;
-      float sum = 0.f;
-      const int r1 = min(args.M - m0, BM);
-      for (int row = half * (BM / 2); row < min(r1, (half + 1) * (BM / 2)); ++row)
-        sum += stg[row * PITCH + col];
-      hs[half * CW + col] = sum;
-      asm volatile("bar.sync 1, 128;" ::: "memory");
-      const int n = n0 + cc + et;
-      if (et < CW && n < args.N) {
-        const float gb = hs[et] + hs[CW + et];
-        const int64_t k = (int64_t)g * args.bias_gs + n;
-        if (!args.bsgd.w) {
-          args.bias_grad[k] = gb;
-        } else {
-          const SgdParams& sp = args.bsgd;
-          float w = bsw[cc / CW], u = bsu[cc / CW];
-          const bool sg = sp.sign != 0;
-          if (sp.mom == 0.f)
-            sgd_elem<false, false>(w, u, gb, sp.lr, 0.f, sp.wd, sg);
-          else if (sp.nesterov)
-            sgd_elem<true, true>(w, u, gb, sp.lr, sp.mom, sp.wd, sg);
-          else
-            sgd_elem<true, false>(w, u, gb, sp.lr, sp.mom, sp.wd, sg);
-          sp.w[k] = w;
-          if (sp.u) sp.u[k] = u;
-          if (sp.wb) sp.wb[k] = f2bf(w);
-        }
-      }
-      asm volatile("bar.sync 1, 128;" ::: "memory");
-    }
+    const SgdParams& sp = args.bsgd;
+    float w = bsw[i], u = bsu[i];
+    const bool sg = sp.sign != 0;
+    if (sp.mom == 0.f)
+      sgd_elem<false, false>(w, u, gb, sp.lr, 0.f, sp.wd, sg);
+    else if (sp.nesterov)
+      sgd_elem<true, true>(w, u, gb, sp.lr, sp.mom, sp.wd, sg);
+    else
+      sgd_elem<true, false>(w, u, gb, sp.lr, sp.mom, sp.wd, sg);
+    sp.w[k] = w;
+    if (sp.u) sp.u[k] = u;
+    if (sp.wb) sp.wb[k] = f2bf(w);
   }
 }
 
@@ -552,15 +593,21 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
   __syncwarp();
 
   // ---------------- epilogue (all 4 warps) ----------------
-  // The stage buffers are free once the accumulator is complete (every MMA has read its
-  // operands): they hold the staging tile.
-  float bsw[BN / 64], bsu[BN / 64];
-  epilogue_bias_prefetch<BN>(args, (int)threadIdx.x, g, n0, bsw, bsu);
+  // Thread t writes tile row t from registers (epilogue_rows).  For the bias column sums the
+  // stage buffers, free once the accumulator is complete (every MMA has read its operands), hold
+  // the four warps' partials.
+  float bsw[kBiasCols<BN>], bsu[kBiasCols<BN>];
+  bias_prefetch<BN>(args, (int)threadIdx.x, g, n0, bsw, bsu);
   const bool have_acc = mbar_wait(&sm.accum, 0);
   asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+  float(*hs)[BN] = reinterpret_cast<float(*)[BN]>(sm.a[0]);
   if (have_acc)
-    epilogue_tile<BN>(args, (int)threadIdx.x, tmem, g, m0, n0, c_base,
-                      reinterpret_cast<float*>(sm.a[0]), bsw, bsu);
+    epilogue_rows<BN, 32>(args, (int)threadIdx.x, lane, tmem, g, m0, n0, c_base,
+                          args.bias_colsum ? hs[warp] : nullptr);
+  if (args.bias_colsum) {
+    __syncthreads();  // every thread passes it, so a wait that ran out cannot split the CTA
+    if (have_acc) bias_update<BN>(args, (int)threadIdx.x, g, n0, hs, bsw, bsu);
+  }
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
   __syncthreads();
   if (warp == 2) {
@@ -578,7 +625,7 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
 //   warp 0      TMA producer: A (128 x 64) and B (PBN x 64) k-blocks into a PST-stage ring
 //   warp 1      MMA issuer: tcgen05.mma (M = 128, N = PBN, K = 16), accumulator (tile & 1)
 //   warp 2      TMEM allocation (2 PBN columns)
-//   warps 4-7   epilogue (pt_epilogue_rows: bias / ReLU / ReLU mask; column sums + bias
+//   warps 4-7   epilogue (epilogue_rows: bias / ReLU / ReLU mask; column sums + bias
 //               update): each thread writes its tile row straight from registers, each warp
 //               waits for the accumulator and hands it back by itself
 // 128 x 256 tiles halve the shared-memory operand bytes per MMA of the 64-wide one-tile kernel
@@ -598,195 +645,6 @@ struct PtSmem {
   uint32_t tmem_base;
   int fail;  // an epilogue warp's accumulator wait ran out (column-sum mode)
 };
-
-// One thread's 64 consecutive accumulator columns of its TMEM lane: two 32-column loads, one wait.
-__device__ __forceinline__ void tmem_ld64(uint32_t taddr, float (&v)[64]) {
-  uint32_t r[64];
-  asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,"
-      "%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%64];\n"
-      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%32,%33,%34,%35,%36,%37,%38,%39,%40,%41,%42,%43,%44,"
-      "%45,%46,%47,%48,%49,%50,%51,%52,%53,%54,%55,%56,%57,%58,%59,%60,%61,%62,%63}, [%65];\n"
-      "tcgen05.wait::ld.sync.aligned;"
-      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
-        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
-        "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]),
-        "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]),
-        "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31]), "=r"(r[32]), "=r"(r[33]), "=r"(r[34]),
-        "=r"(r[35]), "=r"(r[36]), "=r"(r[37]), "=r"(r[38]), "=r"(r[39]), "=r"(r[40]), "=r"(r[41]),
-        "=r"(r[42]), "=r"(r[43]), "=r"(r[44]), "=r"(r[45]), "=r"(r[46]), "=r"(r[47]), "=r"(r[48]),
-        "=r"(r[49]), "=r"(r[50]), "=r"(r[51]), "=r"(r[52]), "=r"(r[53]), "=r"(r[54]), "=r"(r[55]),
-        "=r"(r[56]), "=r"(r[57]), "=r"(r[58]), "=r"(r[59]), "=r"(r[60]), "=r"(r[61]), "=r"(r[62]),
-        "=r"(r[63])
-      : "r"(taddr), "r"(taddr + 32u)
-      : "memory");
-#pragma unroll
-  for (int i = 0; i < 64; ++i) v[i] = __uint_as_float(r[i]);
-}
-
-// Sixteen consecutive outputs of one row: 32-byte stores where the row is aligned and whole,
-// else element by element up to the matrix edge.
-__device__ __forceinline__ void store_row16(void* C, bool c_bf16, int64_t off, int n, int N,
-                                            const float (&x)[16]) {
-  if (c_bf16) {
-    uint16_t* out = reinterpret_cast<uint16_t*>(C) + off;
-    if (n + 16 <= N && (reinterpret_cast<uintptr_t>(out) & 31) == 0) {
-      uint32_t w[8];
-#pragma unroll
-      for (int j = 0; j < 8; ++j) w[j] = (uint32_t)f2bf(x[2 * j]) | ((uint32_t)f2bf(x[2 * j + 1]) << 16);
-      asm volatile("st.global.v8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"l"(out), "r"(w[0]),
-                   "r"(w[1]), "r"(w[2]), "r"(w[3]), "r"(w[4]), "r"(w[5]), "r"(w[6]), "r"(w[7])
-                   : "memory");
-    } else {
-#pragma unroll
-      for (int i = 0; i < 16; ++i)
-        if (n + i < N) out[i] = f2bf(x[i]);
-    }
-  } else {
-    float* out = reinterpret_cast<float*>(C) + off;
-    if (n + 16 <= N && (reinterpret_cast<uintptr_t>(out) & 31) == 0) {
-#pragma unroll
-      for (int j = 0; j < 2; ++j)
-        asm volatile("st.global.v8.f32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"l"(out + 8 * j),
-                     "f"(x[8 * j]), "f"(x[8 * j + 1]), "f"(x[8 * j + 2]), "f"(x[8 * j + 3]),
-                     "f"(x[8 * j + 4]), "f"(x[8 * j + 5]), "f"(x[8 * j + 6]), "f"(x[8 * j + 7])
-                     : "memory");
-    } else {
-#pragma unroll
-      for (int i = 0; i < 16; ++i)
-        if (n + i < N) out[i] = x[i];
-    }
-  }
-}
-
-// The persistent GEMM's epilogue of one 128 x BN tile for one epilogue thread: tile row et (TMEM
-// lane et) leaves TMEM 64 columns at a time and is written straight from registers, 16 columns
-// per store, with the epilogue_tile arithmetic: bias (+ ReLU) or the ReLU mask of the stored
-// activation (the row's 64 mask values requested before the accumulator loads).  With hs_warp
-// (bias_colsum) the stored values -- rounded to bf16 when C is bf16 -- are also summed over the
-// warp's 32 rows, per column, by a fixed butterfly (rows past M add nothing); hs_warp[c] gets
-// column c's partial.
-template <int BN>
-__device__ __forceinline__ void pt_epilogue_rows(const TcGemmArgs& args, int et, int lane,
-                                                 uint32_t tmem_acc, int g, int m0, int n0,
-                                                 float* hs_warp) {
-  const int m = m0 + et;
-  const bool row_ok = m < args.M;
-  const int epi = args.epi;
-  const bool has_bias = epi == EPI_BIAS || epi == EPI_BIAS_RELU;
-  const float* bias = has_bias ? args.bias + (int64_t)g * args.bias_gs : nullptr;
-  const int64_t coff = (int64_t)g * args.c_gs + (int64_t)m * args.c_rs;
-  const int64_t moff = (int64_t)g * args.mask_gs + (int64_t)m * args.mask_rs;
-  const uint32_t lane_base = (uint32_t)(et & ~31) << 16;
-  for (int cc = 0; cc < BN; cc += 64) {
-    if (n0 + cc >= args.N) break;  // uniform over the CTA
-    const int nc = n0 + cc;
-    // the chunk's bf16 mask words (two values each) when the row is whole and 16-byte aligned
-    uint32_t mw[32];
-    const uint16_t* mrow = epi == EPI_MASK && args.mask_bf16
-                               ? reinterpret_cast<const uint16_t*>(args.mask) + moff + nc
-                               : nullptr;
-    const bool mfast = mrow && row_ok && nc + 64 <= args.N &&
-                       (reinterpret_cast<uintptr_t>(mrow) & 15) == 0;
-    if (mfast) {
-#pragma unroll
-      for (int i = 0; i < 8; ++i) {
-        const uint4 t = __ldg(reinterpret_cast<const uint4*>(mrow) + i);
-        mw[4 * i] = t.x;
-        mw[4 * i + 1] = t.y;
-        mw[4 * i + 2] = t.z;
-        mw[4 * i + 3] = t.w;
-      }
-    }
-    float v[64];
-    tmem_ld64(tmem_acc + lane_base + (uint32_t)cc, v);
-#pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      const int nb = nc + 16 * q;
-      float x[16];
-#pragma unroll
-      for (int i = 0; i < 16; ++i) x[i] = v[16 * q + i];
-      if (has_bias) {
-#pragma unroll
-        for (int i = 0; i < 16; ++i) {
-          const int n = nb + i;
-          const float t = x[i] + (n < args.N ? __ldg(bias + n) : 0.f);
-          x[i] = (epi == EPI_BIAS_RELU) ? fmaxf(t, 0.f) : t;
-        }
-      } else if (epi == EPI_MASK) {
-#pragma unroll
-        for (int i = 0; i < 16; ++i) {
-          float mv;
-          if (mfast) {
-            const uint32_t w = mw[8 * q + (i >> 1)];
-            mv = bf2f((uint16_t)((i & 1) ? (w >> 16) : (w & 0xffffu)));
-          } else {
-            const int n = nb + i;
-            mv = !(row_ok && n < args.N) ? 0.f
-                 : args.mask_bf16 ? bf2f(reinterpret_cast<const uint16_t*>(args.mask)[moff + n])
-                                  : reinterpret_cast<const float*>(args.mask)[moff + n];
-          }
-          x[i] = mv > 0.f ? x[i] : 0.f;
-        }
-      }
-      if (row_ok && nb < args.N) store_row16(args.C, args.c_bf16, coff + nb, nb, args.N, x);
-      if (hs_warp) {
-        float t[16];
-#pragma unroll
-        for (int i = 0; i < 16; ++i) t[i] = !row_ok ? 0.f : (args.c_bf16 ? bf2f(f2bf(x[i])) : x[i]);
-        const float sum = warp_colsum16(t, lane);
-        if (!(lane & 1)) hs_warp[cc + 16 * q + (lane >> 1)] = sum;
-      }
-    }
-  }
-}
-
-// The bias of the layer below, for the column-sum mode: each epilogue thread takes columns
-// et + 128 i of the tile; their parameters are requested before the accumulator wait.
-template <int BN>
-__device__ __forceinline__ void pt_bias_prefetch(const TcGemmArgs& args, int et, int g, int n0,
-                                                 float (&bsw)[BN / 128], float (&bsu)[BN / 128]) {
-#pragma unroll
-  for (int i = 0; i < BN / 128; ++i) {
-    const int n = n0 + 128 * i + et;
-    const bool v = args.bias_colsum && args.bsgd.w && n < args.N;
-    const int64_t k = (int64_t)g * args.bias_gs + n;
-    bsw[i] = v ? args.bsgd.w[k] : 0.f;
-    bsu[i] = v && args.bsgd.u ? args.bsgd.u[k] : 0.f;
-  }
-}
-
-// After the four warps' partials are in hs (this tile's buffer): the bias gradient of each of
-// this thread's columns, (warp 0 + warp 1) + (warp 2 + warp 3), and its local update (or the
-// gradient itself without bsgd.w).
-template <int BN>
-__device__ __forceinline__ void pt_bias_update(const TcGemmArgs& args, int et, int g, int n0,
-                                               const float (*hs)[BN], const float (&bsw)[BN / 128],
-                                               const float (&bsu)[BN / 128]) {
-#pragma unroll
-  for (int i = 0; i < BN / 128; ++i) {
-    const int c = 128 * i + et, n = n0 + c;
-    if (n >= args.N) continue;
-    const float gb = __fadd_rn(__fadd_rn(hs[0][c], hs[1][c]), __fadd_rn(hs[2][c], hs[3][c]));
-    const int64_t k = (int64_t)g * args.bias_gs + n;
-    if (!args.bsgd.w) {
-      args.bias_grad[k] = gb;
-      continue;
-    }
-    const SgdParams& sp = args.bsgd;
-    float w = bsw[i], u = bsu[i];
-    const bool sg = sp.sign != 0;
-    if (sp.mom == 0.f)
-      sgd_elem<false, false>(w, u, gb, sp.lr, 0.f, sp.wd, sg);
-    else if (sp.nesterov)
-      sgd_elem<true, true>(w, u, gb, sp.lr, sp.mom, sp.wd, sg);
-    else
-      sgd_elem<true, false>(w, u, gb, sp.lr, sp.mom, sp.wd, sg);
-    sp.w[k] = w;
-    if (sp.u) sp.u[k] = u;
-    if (sp.wb) sp.wb[k] = f2bf(w);
-  }
-}
 
 __global__ void __launch_bounds__(pt::THREADS, 1) gemm_pt_kernel(const __grid_constant__ TcGemmArgs args) {
   extern __shared__ uint8_t smem_raw[];
@@ -919,8 +777,8 @@ __global__ void __launch_bounds__(pt::THREADS, 1) gemm_pt_kernel(const __grid_co
       int g, m0, n0;
       coords(t, g, m0, n0);
       const int ab = i & 1;
-      float bsw[PBN / 128], bsu[PBN / 128];
-      pt_bias_prefetch<PBN>(args, et, g, n0, bsw, bsu);
+      float bsw[kBiasCols<PBN>], bsu[kBiasCols<PBN>];
+      bias_prefetch<PBN>(args, et, g, n0, bsw, bsu);
       if (args.epi == EPI_MASK && args.mask && m0 + et < args.M) {
         // this thread's row of the tile's ReLU mask (the stored activation) into L2 while the
         // tile's products run, so that the copy-out's mask loads do not each wait on DRAM
@@ -935,18 +793,19 @@ __global__ void __launch_bounds__(pt::THREADS, 1) gemm_pt_kernel(const __grid_co
       if (!colsum) {
         if (!okw) break;
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-        pt_epilogue_rows<PBN>(args, et, lane, acc, g, m0, n0, nullptr);
+        epilogue_rows<PBN, 64>(args, et, lane, acc, g, m0, n0, (int64_t)g * args.c_gs, nullptr);
       } else {
         if (okw) {
           asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-          pt_epilogue_rows<PBN>(args, et, lane, acc, g, m0, n0, sm.hs[ab][quarter]);
+          epilogue_rows<PBN, 64>(args, et, lane, acc, g, m0, n0, (int64_t)g * args.c_gs,
+                                 sm.hs[ab][quarter]);
         } else if (lane == 0) {
           sm.fail = 1;
         }
         asm volatile("bar.sync 1, 128;" ::: "memory");
         if (*reinterpret_cast<volatile int*>(&sm.fail)) break;
         // hs[ab] is written again two tiles on, after every warp has passed the next barrier
-        pt_bias_update<PBN>(args, et, g, n0, sm.hs[ab], bsw, bsu);
+        bias_update<PBN>(args, et, g, n0, sm.hs[ab], bsw, bsu);
       }
       asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
       __syncwarp();

@@ -840,8 +840,9 @@ __global__ void __launch_bounds__(pt::THREADS, 1) gemm_pt_kernel(const __grid_co
 //               tcgen05.ld of the gradient columns, the local momentum-SGD update (weight decay,
 //               heavy-ball or Nesterov momentum, Sec. A.4) on w, u in shared memory, bf16 w
 //               into the slot's staging buffer.
-// Only thread 128 waits on the epilogue's mbarriers and the outcome reaches the other epilogue
-// threads through a named barrier, so a wait that runs out cannot split them.
+// Each epilogue warp waits on the accumulator and chunk barriers by itself and releases the chunk
+// (to the store issuer) and the accumulator (to the MMA issuer) with one arrival per warp, so the
+// warps overlap one another's latencies; a wait that runs out ends that warp's loop only.
 //
 // Averaging mode (args.avg): the step ends with the K-way average of Eq. 2 (right), so a CTA takes
 // one weight tile through all G replicas in turn (replica innermost in its tile sequence).  Each

@@ -532,18 +532,28 @@ __global__ void __launch_bounds__(256) bn_act_fwd_v4_kernel(
     rs[i] = rstd[g * C + c0 + i];
   }
   const bool with_sc = sc && c0 < sc_C;
+  // identity shortcut (same grid): the shortcut pixel is p itself, no index arithmetic per pixel
+  const bool sc_same = stride == 1 && sc_H == H && sc_W == Wd;
   const float* yg = y + (int64_t)g * P * C + c0;
   TA* og = out + (int64_t)g * P * C + c0;
   for (int p = blockIdx.x * ppb + pl; p < P; p += gridDim.x * ppb) {
     const float4 yv = *reinterpret_cast<const float4*>(yg + (int64_t)p * C);
+    float4 s4 = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (with_sc) {
+      int64_t sp;
+      if (sc_same) {
+        sp = (int64_t)g * P + p;
+      } else {
+        const int x = p % Wd, hb = p / Wd, h = hb % H, b = hb / H;
+        sp = (((int64_t)g * B + b) * sc_H + h * stride) * sc_W + x * stride;
+      }
+      s4 = Vec4<TA>::load(sc + sp * sc_C + c0);
+    }
     const float yy[4] = {yv.x, yv.y, yv.z, yv.w};
     float v[4];
 #pragma unroll
     for (int i = 0; i < 4; ++i) v[i] = ga[i] * ((yy[i] - mu[i]) * rs[i]) + be[i];
     if (with_sc) {
-      const int x = p % Wd, hb = p / Wd, h = hb % H, b = hb / H;
-      const float4 s4 = Vec4<TA>::load(
-          sc + ((((int64_t)g * B + b) * sc_H + h * stride) * sc_W + x * stride) * sc_C + c0);
       v[0] += s4.x;
       v[1] += s4.y;
       v[2] += s4.z;
@@ -1135,9 +1145,14 @@ __global__ void __launch_bounds__(256) add_shortcut_grad_v2_kernel(
   const int e = blockIdx.x * blockDim.x + threadIdx.x;
   if (e >= Po * C4) return;
   const int po = e / C4, c0 = (e - po * C4) * 4;
-  const int ow = po % Wout, t2 = po / Wout, oh = t2 % Hout, b = t2 / Hout;
   const int64_t o = ((int64_t)g * Po + po) * Cout + c0;
-  const int64_t i = ((((int64_t)g * B + b) * Hin + oh * stride) * Win + ow * stride) * Cin + c0;
+  int64_t i;
+  if (stride == 1 && Hin == Hout && Win == Wout) {
+    i = ((int64_t)g * Po + po) * Cin + c0;  // identity shortcut: the same pixel
+  } else {
+    const int ow = po % Wout, t2 = po / Wout, oh = t2 % Hout, b = t2 / Hout;
+    i = ((((int64_t)g * B + b) * Hin + oh * stride) * Win + ow * stride) * Cin + c0;
+  }
   const float4 d = *reinterpret_cast<const float4*>(dout + o);
   const float4 a = Vec4<TA>::load(out + o);
   float4 x = *reinterpret_cast<float4*>(dx + i);

@@ -86,15 +86,15 @@ AVERAGE_BYTES_PER_PARAM = 10
 #   MLP 3072-4096x3-100, K = 16, B_loc = 128 (2 launches per step: layer 2, then layers 1, 0 and
 #   the 100-class layer):
 #     "avg_synced" -- a step of the H = 1 phase (the replicas agree at its start, it ends with
-#                     the average): 6,687,459,584 B (step 3 of the job);
+#                     the average): 6,695,380,736 B (step 3 of the job);
 #     "plain"      -- an H = 16 step that neither starts synced nor ends a round:
-#                     13,569,810,176 B (step 126);
-#   MLP 3072-1024-1024-10, K = 16, B_loc = 128: "plain" 1,189,963,520 B (the classifier head's
-#     backward, 10,148,608 B, plus the one launch of both hidden layers, 1,179,814,912 B).
+#                     13,583,207,680 B (step 126);
+#   MLP 3072-1024-1024-10, K = 16, B_loc = 128: "plain" 1,187,127,808 B (the classifier head's
+#     backward plus the one launch of both hidden layers).
 # A traced window with a step of another kind reports no traffic.
 UPDATE_TRAFFIC_PER_STEP = {
-    WORKLOAD["name"]: {"avg_synced": 6687459584, "plain": 13569810176},
-    CONFIG2["name"]: {"plain": 1189963520},
+    WORKLOAD["name"]: {"avg_synced": 6695380736, "plain": 13583207680},
+    CONFIG2["name"]: {"plain": 1187127808},
 }
 
 FALLBACK_HBM_GBS = 6800.0

@@ -197,6 +197,26 @@ __global__ void __launch_bounds__(1024) softmax_xent_kernel(
   }
 }
 
+// out[g][j][n] = (the S split-K partial products part[s][g][j][n], added in split order) + bias[g][n]:
+// a narrow layer's product whose reduction was split so that every SM streams.  One thread per
+// output; the S loads are independent.
+__global__ void split_bias_sum_kernel(const float* __restrict__ part, int S, int64_t sstride,
+                                      const float* __restrict__ bias, int64_t bias_gs, int G, int B,
+                                      int N, int ld, float* __restrict__ out) {
+  pdl_begin();
+  const int64_t total = (int64_t)G * B * N;
+  for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < total;
+       t += (int64_t)gridDim.x * blockDim.x) {
+    const int n = (int)(t % N);
+    const int64_t row = t / N;
+    const int g = (int)(row / B);
+    const int64_t off = row * ld + n;
+    float v = part[off];
+    for (int s = 1; s < S; ++s) v += part[(int64_t)s * sstride + off];
+    out[off] = v + (bias ? bias[(int64_t)g * bias_gs + n] : 0.f);
+  }
+}
+
 template <typename TD>
 __global__ void lsq_loss_kernel(const float* __restrict__ z, int ld, const float* __restrict__ t,
                                 int B, TD* __restrict__ dz, int ld_dz, float* __restrict__ loss_mean,
@@ -720,6 +740,18 @@ cudaError_t launch_lsq_loss(const float* z, int ld, const float* targets, int G,
   else
     launch_pdl(lsq_loss_kernel<float>, G, 256, smem, stream, z, ld, targets, B, reinterpret_cast<float*>(dz),
                                                      ld_dz, loss_mean, loss_sum, row_loss);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_split_bias_sum(const float* part, int S, int64_t sstride, const float* bias,
+                                  int64_t bias_gs, int G, int B, int N, int ld, float* out,
+                                  cudaStream_t stream) {
+  if (G <= 0 || B <= 0 || N <= 0) return cudaSuccess;
+  if (!part || !out || S < 1 || ld < N || sstride < (int64_t)G * B * ld) return cudaErrorInvalidValue;
+  const int64_t total = (int64_t)G * B * N;
+  const int blocks = (int)std::min<int64_t>((total + 255) / 256, 65535);
+  launch_pdl(split_bias_sum_kernel, blocks, 256, 0, stream, part, S, sstride, bias, bias_gs, G, B,
+             N, ld, out);
   return cudaGetLastError();
 }
 

@@ -64,6 +64,11 @@ cudaError_t launch_lsq_loss(const float* z, int ld, const float* targets, int G,
                             bool dz_bf16, int ld_dz, float* loss_mean, float* loss_sum,
                             float* row_loss, cudaStream_t stream);
 // gb[g * gb_gs + o] = sum_j dz[g][j][o] for o < out.
+// out[g][j][n] = sum over s < S, in order, of part[s * sstride + (g B + j) ld + n], plus
+// bias[g bias_gs + n] (bias may be null): the split-K partial products of a narrow layer.
+cudaError_t launch_split_bias_sum(const float* part, int S, int64_t sstride, const float* bias,
+                                  int64_t bias_gs, int G, int B, int N, int ld, float* out,
+                                  cudaStream_t stream);
 cudaError_t launch_colsum(const void* dz, bool dz_bf16, int ld, int G, int B, int out, float* gb,
                           int64_t gb_gs, cudaStream_t stream);
 // Bias gradient fused with the local update: b (at sgd.w + g * gs) receives the update step

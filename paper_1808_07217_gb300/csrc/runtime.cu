@@ -87,6 +87,9 @@ struct lsgd_ctx {
   std::vector<void*> act;  // act[l]: input of dense layer l, [K][B][ld] operand dtype
   float* logits = nullptr;
   int ld_logits = 0;
+  // split-K partial products of a narrow top layer's forward (logit_splits of them), or none
+  float* logit_parts = nullptr;
+  int logit_splits = 0;
   // output gradients: ping-pong buffers, and a third that keeps the top layer's while the layers
   // below use the first two (its update joins the last update launch)
   void* dz[3] = {nullptr, nullptr, nullptr};
@@ -403,6 +406,22 @@ lsgd_status dense_forward(lsgd_ctx* c, int groups, int w_g0, int w_gmul, bool sk
       t.bias_gs = c->d_pad;
       // every replica holds the same weights: all read replica 0's, which stay in L2
       t.b_shared = (c->synced && groups == c->cfg.K && c->cfg.K > 1) ? 1 : 0;
+      if (last && c->logit_splits > 1 && epi == lsgd::EPI_BIAS) {
+        // split-K partial products, then their sum in split order plus the bias
+        const int64_t sstride = (int64_t)c->cfg.K * B * ld_out;
+        t.splits = c->logit_splits;
+        t.c_split_stride = sstride;
+        t.C = c->logit_parts;
+        t.epi = lsgd::EPI_STORE;
+        t.bias = nullptr;
+        lsgd_status st = tc_gemm(c, t);
+        if (st != LSGD_OK) return st;
+        LSGD_LAUNCH(c, lsgd::launch_split_bias_sum(c->logit_parts, c->logit_splits, sstride,
+                                                   Ly.b_off >= 0 ? c->W + Ly.b_off : nullptr,
+                                                   c->d_pad, groups, B, Ly.out, ld_out,
+                                                   (float*)out, c->stream));
+        continue;
+      }
       lsgd_status st = tc_gemm(c, t);
       if (st != LSGD_OK) return st;
       continue;
@@ -974,6 +993,21 @@ lsgd_status lsgd_create(const lsgd_config* cfg, const lsgd_allocator* alloc, voi
     if (st == LSGD_OK) {
       const DenseLayer& top = c->layers.back();
       c->head = c->bf16 && !c->lsq && top.tc && lsgd::head_supported(top.out, c0.B_loc, top.in);
+      // A narrow output layer over a long input (the 100-class layer of the 4096-wide MLP) gives
+      // the one-tile GEMM only out / 64 x K tiles, each a long reduction that streams from one
+      // SM; its forward is split eight ways into partial products that a second kernel adds, in
+      // split order, with the bias.
+      if (!c->head && !c->lsq && top.tc && top.out <= 128 && top.in >= 1024) {
+        const int S = lsgd::tc_valid_splits(top.in, 8);
+        if (S > 1) {
+          c->logit_parts = (float*)dalloc(c, (size_t)S * c0.K * c0.B_loc * c->ld_logits * 4);
+          if (!c->logit_parts) {
+            fail(nullptr, LSGD_ENOMEM, "logit partial buffer allocation failed");
+            return bail(LSGD_ENOMEM);
+          }
+          c->logit_splits = S;
+        }
+      }
       if (defer_top_update(c)) {
         c->dz[2] = dalloc(c, (size_t)c0.K * c0.B_loc * c->ld_dz * 2);
         if (!c->dz[2]) {

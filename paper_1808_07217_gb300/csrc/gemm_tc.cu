@@ -192,29 +192,6 @@ __device__ __forceinline__ float warp_colsum16(float (&v)[16], int lane) {
   return v[0] + __shfl_xor_sync(0xffffffffu, v[0], 1);
 }
 
-// The local update on four consecutive parameters (fused weight-gradient epilogue); SG fixes at
-// compile time whether the signSGD variant's sign is taken (it must equal sp.sign != 0).
-template <bool SG>
-__device__ __forceinline__ void sgd4(float4& w, float4& u, const float4 g, const SgdParams& sp) {
-  constexpr bool sg = SG;
-  if (sp.mom == 0.f) {
-    sgd_elem<false, false>(w.x, u.x, g.x, sp.lr, 0.f, sp.wd, sg);
-    sgd_elem<false, false>(w.y, u.y, g.y, sp.lr, 0.f, sp.wd, sg);
-    sgd_elem<false, false>(w.z, u.z, g.z, sp.lr, 0.f, sp.wd, sg);
-    sgd_elem<false, false>(w.w, u.w, g.w, sp.lr, 0.f, sp.wd, sg);
-  } else if (sp.nesterov) {
-    sgd_elem<true, true>(w.x, u.x, g.x, sp.lr, sp.mom, sp.wd, sg);
-    sgd_elem<true, true>(w.y, u.y, g.y, sp.lr, sp.mom, sp.wd, sg);
-    sgd_elem<true, true>(w.z, u.z, g.z, sp.lr, sp.mom, sp.wd, sg);
-    sgd_elem<true, true>(w.w, u.w, g.w, sp.lr, sp.mom, sp.wd, sg);
-  } else {
-    sgd_elem<true, false>(w.x, u.x, g.x, sp.lr, sp.mom, sp.wd, sg);
-    sgd_elem<true, false>(w.y, u.y, g.y, sp.lr, sp.mom, sp.wd, sg);
-    sgd_elem<true, false>(w.z, u.z, g.z, sp.lr, sp.mom, sp.wd, sg);
-    sgd_elem<true, false>(w.w, u.w, g.w, sp.lr, sp.mom, sp.wd, sg);
-  }
-}
-
 template <int BN, int STAGES>
 struct Smem {
   // stage buffers first (1024-byte aligned for the 128-byte swizzle)
@@ -956,7 +933,7 @@ enum : int { kPlain = 0, kFirst = 1, kLast = 2, kAvg = 4 };
 }  // namespace wu
 
 // The local update of four consecutive parameters under one update rule (0: no momentum,
-// 1: heavy ball, 2: Nesterov); the same sgd_elem arithmetic as sgd4.
+// 1: heavy ball, 2: Nesterov) through sgd_elem, the arithmetic of every update kernel.
 template <bool SG, int RULE>
 __device__ __forceinline__ void sgd4_rule(float4& w, float4& u, const float4 g, const SgdParams& sp) {
   constexpr bool MOM = RULE != 0, NEST = RULE == 2;

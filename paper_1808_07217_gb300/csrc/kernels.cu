@@ -156,6 +156,66 @@ __global__ void __launch_bounds__(1024) softmax_xent_kernel(
   const int g = blockIdx.x, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int nw = blockDim.x >> 5;
   const float inv_b = 1.0f / (float)B;
+  if (C <= 128) {
+    // up to 128 classes: a lane's (at most four) logits of RPW rows are loaded before any is used,
+    // so a warp waits on memory once per RPW rows; per lane the same order as below, same bits
+    constexpr int RPW = 4;
+    for (int j0 = warp; j0 < B; j0 += nw * RPW) {
+      float zv[RPW][4];
+#pragma unroll
+      for (int r = 0; r < RPW; ++r) {
+        const int j = j0 + r * nw;
+        const float* z = logits + ((int64_t)g * B + j) * ld;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const int c = lane + 32 * i;
+          zv[r][i] = (j < B && c < C) ? z[c] : -INFINITY;
+        }
+      }
+#pragma unroll
+      for (int r = 0; r < RPW; ++r) {
+        const int j = j0 + r * nw;
+        if (j >= B) break;  // uniform over the warp
+        float mx = -INFINITY;
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+          if (lane + 32 * i < C) mx = fmaxf(mx, zv[r][i]);
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+        float se = 0.f;
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+          if (lane + 32 * i < C) se += expf(zv[r][i] - mx);
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) se += __shfl_xor_sync(0xffffffffu, se, o);
+        const float lse = mx + logf(se);
+        const int y = labels[(int64_t)g * B + j];
+        if (dz) {
+          TD* dzr = dz + ((int64_t)g * B + j) * ld_dz;
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            const int c = lane + 32 * i;
+            if (c < C) {
+              const float p = expf(zv[r][i] - lse);
+              Elem<TD>::store(dzr + c, (p - (c == y ? 1.f : 0.f)) * inv_b);
+            }
+          }
+        }
+        // the label's logit: the lane that holds it
+        const int yl = y & 31, yi = y >> 5;
+        float zy = 0.f;
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+          if (i == yi) zy = zv[r][i];
+        zy = __shfl_sync(0xffffffffu, zy, yl);
+        if (lane == 0) {
+          const float l = lse - zy;
+          if (row_out) row_out[(int64_t)g * B + j] = l;
+          row_loss[j] = l;
+        }
+      }
+    }
+  } else {
   for (int j = warp; j < B; j += nw) {
     const float* z = logits + ((int64_t)g * B + j) * ld;
     float mx = -INFINITY;
@@ -180,6 +240,7 @@ __global__ void __launch_bounds__(1024) softmax_xent_kernel(
       if (row_out) row_out[(int64_t)g * B + j] = l;
       row_loss[j] = l;
     }
+  }
   }
   __syncthreads();
   // sum of the B row losses: a fixed tree over the rows (strides halving from the largest power

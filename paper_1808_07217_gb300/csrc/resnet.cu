@@ -1050,6 +1050,50 @@ bool sum_partials_v4_ok(const float* part, int ldc, int cols, const float* out, 
          (reinterpret_cast<uintptr_t>(part) & 15) == 0 && (reinterpret_cast<uintptr_t>(out) & 15) == 0;
 }
 
+// Several weight gradients' partial sums in one launch (the ResNet step's, at the end of its
+// backward): job k covers threads [begin_k, begin_{k+1}) and is sum_partials_v4_kernel's sum for
+// its buffers, partials added in split order q = 0, 1, ... -- the same bits as one launch each.
+struct SumJob {
+  const float* part;
+  float* out;
+  int64_t out_gs;
+  int64_t begin;  // first thread of this job
+  int nq, rows, ldc, cols, G, tap_src, tap_dst, pad;
+};
+constexpr int kMaxSumJobs = 24;
+struct SumJobs {
+  int n;
+  SumJob j[kMaxSumJobs];
+};
+
+__global__ void __launch_bounds__(256) sum_partials_jobs_v4_kernel(const __grid_constant__ SumJobs js,
+                                                                     int64_t total) {
+  pdl_begin();
+  const int64_t t0 = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (t0 >= total) return;
+  int k = 0;
+  while (k + 1 < js.n && t0 >= js.j[k + 1].begin) ++k;
+  const SumJob& jb = js.j[k];
+  const int64_t t = t0 - jb.begin;
+  const int c4 = jb.cols / 4;
+  const int j = (int)(t % c4) * 4;
+  const int r = (int)((t / c4) % jb.rows);
+  const int g = (int)(t / ((int64_t)jb.rows * c4));
+  const int js_ = jb.tap_dst > 0 ? (j / jb.tap_dst) * jb.tap_src + j % jb.tap_dst : j;
+  const float* pp = jb.part + (int64_t)g * jb.nq * jb.rows * jb.ldc + (int64_t)r * jb.ldc + js_;
+  const int64_t qs = (int64_t)jb.rows * jb.ldc;
+  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll 4
+  for (int q = 0; q < jb.nq; ++q) {
+    const float4 v = __ldg(reinterpret_cast<const float4*>(pp + q * qs));
+    acc.x += v.x;
+    acc.y += v.y;
+    acc.z += v.z;
+    acc.w += v.w;
+  }
+  *reinterpret_cast<float4*>(jb.out + (int64_t)g * jb.out_gs + (int64_t)r * jb.cols + j) = acc;
+}
+
 // Launches whichever of the two partial-sum kernels fits the shapes.
 void launch_sum_partials(const float* part, int nq, int rows, int ldc, int cols, int G, float* out,
                          int64_t out_gs, int tap_src, int tap_dst, cudaStream_t s) {
@@ -1183,6 +1227,10 @@ struct ResNetPlan {
   float* part = nullptr;
   size_t part_floats = 0;
   float* s12 = nullptr;
+  // weight-gradient partials of each tensor-core weight gradient (null where none), kept until
+  // the end of the backward, whose one launch then sums all of them (sum_jobs: the pending sums)
+  std::vector<float*> wpart;
+  std::vector<SumJob> sum_jobs;
   // tensor-core convolutions (BF16 mode): per-convolution im2col of its input (kept from the
   // forward for the weight gradient), the output-gradient im2col and flipped weights of the
   // stride-1 data gradients
@@ -1207,6 +1255,52 @@ struct ResNetPlan {
 };
 
 namespace {
+
+// The weight-gradient kernel (partials into part) and their ordered sum into dW.  With defer, a
+// sum that the 4-wide kernel takes is not launched but described in *defer (*deferred = true), to
+// run with the step's others in one launch.
+cudaError_t launch_conv_wgrad_impl(const uint16_t* x, const uint16_t* dy, float* dW, int64_t dW_gs,
+                                   int G, int B, int hout, int wout, int cin, int cout, int stride,
+                                   float* part, cudaStream_t s, int cin_out, SumJob* defer,
+                                   bool* deferred) {
+  if (deferred) *deferred = false;
+  const int hin = hout * stride, win = wout * stride;
+  const int64_t P = (int64_t)B * hout * wout;
+  if (cin_out <= 0) cin_out = cin;
+  if (!conv_wgrad_tc_ok(cin, cout, stride, hin, win, hout, wout) || G < 1 || B < 1 ||
+      P > 0x7fffffffLL || cin_out > cin)
+    return cudaErrorInvalidValue;
+  ConvWgradArgs a{};
+  // the output-gradient tile: 64 pixels x nb channels (Cout of 16 / 32 / 64 exactly; 48 padded
+  // to 64 by the map's zero fill), swizzled at its 2 nb-byte row
+  const int nb = (cout == 16 || cout == 32) ? cout : 64;
+  if (!make_tma_map_halo(&a.x_map, x, cin, win, hin, B, G, stride, wout) ||
+      !make_tma_map(&a.dy_map, dy, true, cout, P, G, cout, (uint64_t)P * cout, nb, 64, 2 * nb))
+    return cudaErrorInvalidValue;
+  a.nb = nb;
+  a.cin = cin;
+  a.cout = cout;
+  a.stride = stride;
+  a.hin = hin;
+  a.win = win;
+  a.hout = hout;
+  a.wout = wout;
+  a.G = G;
+  a.P = (int)P;
+  a.cpr = conv_wgrad_ctas(cin, stride, wout, G, P);
+  a.part = part;
+  cudaError_t e = launch_conv_wgrad_tc(a, s);
+  if (e != cudaSuccess) return e;
+  // the partials' sum, cropped to the first cin_out channels of every tap
+  if (defer && deferred && sum_partials_v4_ok(part, 9 * cin, 9 * cin_out, dW, dW_gs, cin, cin_out)) {
+    *defer = SumJob{part, dW, dW_gs, 0, a.cpr, cout, 9 * cin, 9 * cin_out, G, cin, cin_out, 0};
+    *deferred = true;
+    return cudaGetLastError();
+  }
+  launch_sum_partials(part, a.cpr, cout, 9 * cin, 9 * cin_out, G, dW, dW_gs, cin, cin_out, s);
+  return cudaGetLastError();
+}
+
 
 size_t esz(const ResNetPlan* p) { return p->bf16 ? 2 : 4; }
 
@@ -1733,10 +1827,20 @@ lsgd_status conv_wgrad(ResNetPlan* p, int i, const void* in, float* Gr, cudaStre
   if (wgrad_tc(p, c)) {
     // dW [Cout][9 Cin] from dy and the input directly: the column matrix of each 64-pixel block
     // is built in shared memory; one partial per CTA, summed in order
-    RN_CALL(launch_conv_wgrad_bf16(reinterpret_cast<const uint16_t*>(in),
+    // with a buffer of its own the partials' sum waits for the end of the backward, where one
+    // launch adds every layer's
+    float* wp = (size_t)i < p->wpart.size() ? p->wpart[i] : nullptr;
+    SumJob job{};
+    bool deferred = false;
+    const bool can_defer = wp && p->sum_jobs.size() < (size_t)kMaxSumJobs;
+    RN_CALL(launch_conv_wgrad_impl(reinterpret_cast<const uint16_t*>(in),
                                    reinterpret_cast<const uint16_t*>(p->dy), Gr + c.w_off, p->d_pad,
-                                   K, p->B, c.hout, c.wout, c.cin, c.cout, c.stride, p->part, s));
-    ++*launches;  // the partials' sum
+                                   K, p->B, c.hout, c.wout, c.cin, c.cout, c.stride,
+                                   wp ? wp : p->part, s, 0, can_defer ? &job : nullptr, &deferred));
+    if (deferred)
+      p->sum_jobs.push_back(job);
+    else
+      ++*launches;  // the partials' sum
     return LSGD_OK;
   }
   if (conv_on_tc(p, c)) {
@@ -1937,10 +2041,28 @@ lsgd_status conv_dgrad(ResNetPlan* p, int i, const void* Wop, float* dx, const f
   return LSGD_OK;
 }
 
+// The weight gradients' deferred partial sums, all in one launch.
+lsgd_status flush_sum_jobs(ResNetPlan* p, cudaStream_t s, int64_t* launches) {
+  if (p->sum_jobs.empty()) return LSGD_OK;
+  SumJobs js{};
+  int64_t total = 0;
+  for (const SumJob& jb : p->sum_jobs) {
+    js.j[js.n] = jb;
+    js.j[js.n].begin = total;
+    total += (int64_t)jb.G * jb.rows * (jb.cols / 4);
+    ++js.n;
+  }
+  p->sum_jobs.clear();
+  RN_LAUNCH((launch_pdl(sum_partials_jobs_v4_kernel, (unsigned)((total + 255) / 256), 256, 0, s, js,
+                        total)));
+  return LSGD_OK;
+}
+
 template <typename TA>
 lsgd_status fwd_bwd_impl(ResNetPlan* p, const float* W, const void* Wop, float* Gr,
                          const int32_t* labels, float* loss_mean, cudaStream_t s, int64_t* launches) {
   const int K = p->K, B = p->B;
+  p->sum_jobs.clear();
   lsgd_status st = forward_impl<TA>(p, W, Wop, 0, 1, K, s, launches);
   if (st != LSGD_OK) return st;
   RN_CALL(launch_softmax_xent(p->logits, p->C, p->C, labels, K, B, p->dlogits, false, p->C,
@@ -2027,7 +2149,9 @@ lsgd_status fwd_bwd_impl(ResNetPlan* p, const float* W, const void* Wop, float* 
   const ConvL& c0 = p->convs[0];
   st = bn_backward<TA>(p, c0, 0, p->dA[cur], p->act[0], W, Gr, s, launches, pending);
   if (st != LSGD_OK) return st;
-  return conv_wgrad<TA>(p, 0, p->x0, Gr, s, launches);
+  st = conv_wgrad<TA>(p, 0, p->x0, Gr, s, launches);
+  if (st != LSGD_OK) return st;
+  return flush_sum_jobs(p, s, launches);
 }
 
 }  // namespace
@@ -2115,36 +2239,8 @@ size_t conv_wgrad_scratch_floats(int G, int B, int hout, int wout, int cin, int 
 cudaError_t launch_conv_wgrad_bf16(const uint16_t* x, const uint16_t* dy, float* dW, int64_t dW_gs,
                                    int G, int B, int hout, int wout, int cin, int cout, int stride,
                                    float* part, cudaStream_t s, int cin_out) {
-  const int hin = hout * stride, win = wout * stride;
-  const int64_t P = (int64_t)B * hout * wout;
-  if (cin_out <= 0) cin_out = cin;
-  if (!conv_wgrad_tc_ok(cin, cout, stride, hin, win, hout, wout) || G < 1 || B < 1 ||
-      P > 0x7fffffffLL || cin_out > cin)
-    return cudaErrorInvalidValue;
-  ConvWgradArgs a{};
-  // the output-gradient tile: 64 pixels x nb channels (Cout of 16 / 32 / 64 exactly; 48 padded
-  // to 64 by the map's zero fill), swizzled at its 2 nb-byte row
-  const int nb = (cout == 16 || cout == 32) ? cout : 64;
-  if (!make_tma_map_halo(&a.x_map, x, cin, win, hin, B, G, stride, wout) ||
-      !make_tma_map(&a.dy_map, dy, true, cout, P, G, cout, (uint64_t)P * cout, nb, 64, 2 * nb))
-    return cudaErrorInvalidValue;
-  a.nb = nb;
-  a.cin = cin;
-  a.cout = cout;
-  a.stride = stride;
-  a.hin = hin;
-  a.win = win;
-  a.hout = hout;
-  a.wout = wout;
-  a.G = G;
-  a.P = (int)P;
-  a.cpr = conv_wgrad_ctas(cin, stride, wout, G, P);
-  a.part = part;
-  cudaError_t e = launch_conv_wgrad_tc(a, s);
-  if (e != cudaSuccess) return e;
-  // the partials' sum, cropped to the first cin_out channels of every tap
-  launch_sum_partials(part, a.cpr, cout, 9 * cin, 9 * cin_out, G, dW, dW_gs, cin, cin_out, s);
-  return cudaGetLastError();
+  return launch_conv_wgrad_impl(x, dy, dW, dW_gs, G, B, hout, wout, cin, cout, stride, part, s,
+                                cin_out, nullptr, nullptr);
 }
 
 cudaError_t launch_batchnorm_stats(const float* y, int64_t P, int C, int G, float* mean,
@@ -2311,11 +2407,16 @@ lsgd_status resnet_alloc(ResNetPlan* p, const std::function<void*(size_t)>& allo
     const int64_t nq_w = (P + kWgradChunk - 1) / kWgradChunk;
     part = std::max(part, (size_t)(K * nq_s * c.cout * 2));
     part = std::max(part, (size_t)(K * nq_w * c.cout * 9 * c.cin));
+    float* wp = nullptr;
     if (conv_on_tc(p, c)) {
       const int Kc = col_ld(c);
       if (wgrad_tc(p, c)) {
         const int cpr = conv_wgrad_ctas(c.cin, c.stride, c.wout, K, P);
         part = std::max(part, (size_t)K * cpr * c.cout * 9 * c.cin);
+        if (!(&c == &p->convs[0] && p->stem16)) {
+          wp = (float*)alloc((size_t)K * cpr * c.cout * 9 * c.cin * 4);
+          if (!wp) return LSGD_ENOMEM;
+        }
       } else {
         const int tiles = ((Kc + 63) / 64) * K;
         const int splits = tc_valid_splits((int)P, std::max(1, (4 * kNumSMs + tiles - 1) / tiles));
@@ -2339,6 +2440,7 @@ lsgd_status resnet_alloc(ResNetPlan* p, const std::function<void*(size_t)>& allo
     } else {
       p->col.push_back(nullptr);
     }
+    p->wpart.push_back(wp);
   }
   if (colT) {
     p->colT = (uint16_t*)alloc(colT * 2);

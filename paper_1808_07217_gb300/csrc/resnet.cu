@@ -1176,6 +1176,50 @@ __global__ void flip_phase_weights_kernel(const uint16_t* __restrict__ Wb, int64
   }
 }
 
+// Every data gradient's flipped weights of a step in one launch (the weights do not change during
+// the backward): job k covers elements [begin_k, begin_k + n_k) and writes what
+// flip_weights_kernel (phases = 0) or flip_phase_weights_kernel (phases = 1) would, to dst_k.
+struct FlipJob {
+  int64_t w_off;   // the layer's weights within each replica's d_pad slice
+  uint16_t* dst;   // [G][Cin][9][Cout], or [4][G][Cin][9][Cout] with phases
+  int64_t begin;   // first element of this job
+  int64_t n;       // its elements
+  int cin, cout, phases, pad;
+};
+constexpr int kMaxFlipJobs = 24;
+struct FlipJobs {
+  int n;
+  FlipJob j[kMaxFlipJobs];
+};
+
+__global__ void flip_jobs_kernel(const uint16_t* __restrict__ Wb, int64_t d_pad, int G,
+                                 const __grid_constant__ FlipJobs js, int64_t total) {
+  pdl_begin();
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < total; t += stride) {
+    int k = 0;
+    while (k + 1 < js.n && t >= js.j[k + 1].begin) ++k;
+    const FlipJob& jb = js.j[k];
+    const int64_t e = t - jb.begin;
+    const int Cin = jb.cin, Cout = jb.cout;
+    const int64_t per = (int64_t)Cin * 9 * Cout;
+    const int co = (int)(e % Cout), tp = (int)((e / Cout) % 9), ci = (int)((e / (9 * Cout)) % Cin);
+    const int64_t gp = e / per;
+    if (!jb.phases) {
+      const int g = (int)gp;
+      jb.dst[e] = Wb[(int64_t)g * d_pad + jb.w_off + ((int64_t)co * 9 + (8 - tp)) * Cin + ci];
+    } else {
+      const int g = (int)(gp % G), ph = (int)(gp / G);
+      const int dr = tp / 3 - 1, dc = tp % 3 - 1;
+      const int kh = (ph >> 1) + 1 - 2 * dr, kw = (ph & 1) + 1 - 2 * dc;
+      uint16_t v = 0;
+      if (kh >= 0 && kh <= 2 && kw >= 0 && kw <= 2)
+        v = Wb[(int64_t)g * d_pad + jb.w_off + (((int64_t)co * 3 + kh) * 3 + kw) * Cin + ci];
+      jb.dst[e] = v;
+    }
+  }
+}
+
 // The option-A shortcut's share of a block's input gradient: for input pixels on the stride grid
 // and the first Cin channels, dx += dout * (out > 0) at (ih / s, iw / s).  Thread = (output pixel,
 // 4 channels < Cin), blockIdx.y the replica; only the input pixels on the stride grid are touched.
@@ -1231,6 +1275,9 @@ struct ResNetPlan {
   // the end of the backward, whose one launch then sums all of them (sum_jobs: the pending sums)
   std::vector<float*> wpart;
   std::vector<SumJob> sum_jobs;
+  // each data gradient's flipped weights (null where the step flips into the shared wt / wt4),
+  // all written by one launch at the start of the backward
+  std::vector<uint16_t*> wflip;
   // tensor-core convolutions (BF16 mode): per-convolution im2col of its input (kept from the
   // forward for the weight gradient), the output-gradient im2col and flipped weights of the
   // stride-1 data gradients
@@ -1482,10 +1529,12 @@ lsgd_status conv_fwd_tc(const uint16_t* x, const uint16_t* w, int64_t w_gs, floa
 
 // bf (optional): the BatchNorm-backward epilogue (ConvBwdFuse; part_gs / part_off are filled in
 // here); *nparts receives the partials per replica it wrote.
+// flipped: wt already holds the flipped (stride 2: the four phases') weights of w.
 lsgd_status conv_dgrad_tc(const uint16_t* dy, const uint16_t* w, int64_t w_gs, float* dx, int G,
                           int B, int hin, int win, int cin, int cout, int stride, uint16_t* wt,
                           cudaStream_t s, std::string& err, int64_t* launches,
-                          const ConvBwdFuse* bf = nullptr, int* nparts = nullptr) {
+                          const ConvBwdFuse* bf = nullptr, int* nparts = nullptr,
+                          bool flipped = false) {
   if (nparts) *nparts = 0;
   if (!conv_dgrad_tc_route(B, hin, win, cin, cout, stride)) {
     err = "data-gradient shape not taken by the implicit-GEMM kernel";
@@ -1493,8 +1542,9 @@ lsgd_status conv_dgrad_tc(const uint16_t* dy, const uint16_t* w, int64_t w_gs, f
   }
   const int64_t P = (int64_t)B * hin * win;
   if (stride == 1) {
-    CV_LAUNCH((launch_pdl(flip_weights_kernel, dim3((unsigned)((cin * 9 * cout + 255) / 256), (unsigned)G),
-                          256, 0, s, w, w_gs, (int64_t)0, wt, G, cin, cout)));
+    if (!flipped)
+      CV_LAUNCH((launch_pdl(flip_weights_kernel, dim3((unsigned)((cin * 9 * cout + 255) / 256), (unsigned)G),
+                            256, 0, s, w, w_gs, (int64_t)0, wt, G, cin, cout)));
     ConvArgs ca{};
     ca.strip = conv_strip_ok(hin, win, 1);
     bool okc = make_tma_map_conv(&ca.in_map, dy, cout, win, hin, B, G, win, hin, 1, ca.strip);
@@ -1531,8 +1581,9 @@ lsgd_status conv_dgrad_tc(const uint16_t* dy, const uint16_t* w, int64_t w_gs, f
   // taps, zeros elsewhere) whose outputs land on every other row and column of dx
   const int hout = hin / 2, wout = win / 2;
   const int64_t per = (int64_t)cin * 9 * cout;
-  CV_LAUNCH(launch_pdl(flip_phase_weights_kernel, grid_cap(4 * (int64_t)G * per, 256), 256, 0, s,
-                       w, w_gs, (int64_t)0, wt, G, cin, cout));
+  if (!flipped)
+    CV_LAUNCH(launch_pdl(flip_phase_weights_kernel, grid_cap(4 * (int64_t)G * per, 256), 256, 0, s,
+                         w, w_gs, (int64_t)0, wt, G, cin, cout));
   const int64_t Pq = (int64_t)B * hout * wout;
   for (int ph = 0; ph < 4; ++ph) {
     ConvArgs ca{};
@@ -1921,10 +1972,12 @@ lsgd_status conv_dgrad(ResNetPlan* p, int i, const void* Wop, float* dx, const f
     // stride 1: dx is the convolution of dy with the flipped, transposed weights -- an implicit
     // GEMM over dy's taps, no column matrix
     if (persistent_conv_ok(c.cin, P)) {
+      uint16_t* wf = (size_t)i < p->wflip.size() ? p->wflip[i] : nullptr;
       const lsgd_status st = conv_dgrad_tc(reinterpret_cast<const uint16_t*>(p->dy),
                                            reinterpret_cast<const uint16_t*>(Wop) + c.w_off, p->d_pad,
-                                           dx, K, p->B, c.hin, c.win, c.cin, c.cout, 1, p->wt, s,
-                                           p->err, launches, fuse ? &bf : nullptr, fused_parts);
+                                           dx, K, p->B, c.hin, c.win, c.cin, c.cout, 1,
+                                           wf ? wf : p->wt, s, p->err, launches,
+                                           fuse ? &bf : nullptr, fused_parts, wf != nullptr);
       if (st != LSGD_OK) return st;
       if (fuse) return LSGD_OK;  // the epilogue added the shortcut's share
     } else {
@@ -1967,10 +2020,12 @@ lsgd_status conv_dgrad(ResNetPlan* p, int i, const void* Wop, float* dx, const f
   }
   if (phase_dgrad_ok(p, c)) {
     // stride 2: four parity phases on the persistent implicit-GEMM kernel
+    uint16_t* wf = (size_t)i < p->wflip.size() ? p->wflip[i] : nullptr;
     const lsgd_status st = conv_dgrad_tc(reinterpret_cast<const uint16_t*>(p->dy),
                                          reinterpret_cast<const uint16_t*>(Wop) + c.w_off, p->d_pad,
-                                         dx, K, p->B, c.hin, c.win, c.cin, c.cout, 2, p->wt4, s,
-                                         p->err, launches, fuse ? &bf : nullptr, fused_parts);
+                                         dx, K, p->B, c.hin, c.win, c.cin, c.cout, 2,
+                                         wf ? wf : p->wt4, s, p->err, launches,
+                                         fuse ? &bf : nullptr, fused_parts, wf != nullptr);
     if (st != LSGD_OK) return st;
     if (fuse) return LSGD_OK;  // the epilogue added the shortcut's share
     if (dout) {
@@ -2058,6 +2113,38 @@ lsgd_status flush_sum_jobs(ResNetPlan* p, cudaStream_t s, int64_t* launches) {
   return LSGD_OK;
 }
 
+// Every data gradient's flipped weights for this step, from the bf16 weights, in one launch.
+lsgd_status flip_all(ResNetPlan* p, const void* Wop, cudaStream_t s, int64_t* launches) {
+  FlipJobs js{};
+  int64_t total = 0;
+  auto flush = [&]() -> lsgd_status {
+    if (total > 0)
+      RN_LAUNCH((launch_pdl(flip_jobs_kernel, grid_cap(total, 256), 256, 0, s,
+                            reinterpret_cast<const uint16_t*>(Wop), p->d_pad, p->K, js, total)));
+    js = FlipJobs{};
+    total = 0;
+    return LSGD_OK;
+  };
+  for (size_t i = 0; i < p->wflip.size(); ++i) {
+    if (!p->wflip[i]) continue;
+    if (js.n == kMaxFlipJobs) {
+      const lsgd_status st = flush();  // a deeper network: one launch per table
+      if (st != LSGD_OK) return st;
+    }
+    const ConvL& c = p->convs[i];
+    FlipJob& jb = js.j[js.n++];
+    jb.w_off = c.w_off;
+    jb.dst = p->wflip[i];
+    jb.begin = total;
+    jb.phases = c.stride == 2 ? 1 : 0;
+    jb.n = (jb.phases ? 4 : 1) * (int64_t)p->K * c.cin * 9 * c.cout;
+    jb.cin = c.cin;
+    jb.cout = c.cout;
+    total += jb.n;
+  }
+  return flush();
+}
+
 template <typename TA>
 lsgd_status fwd_bwd_impl(ResNetPlan* p, const float* W, const void* Wop, float* Gr,
                          const int32_t* labels, float* loss_mean, cudaStream_t s, int64_t* launches) {
@@ -2116,6 +2203,10 @@ lsgd_status fwd_bwd_impl(ResNetPlan* p, const float* W, const void* Wop, float* 
         HW, p->F)));
   }
   const int n_blocks = (int)(p->convs.size() - 1) / 2;
+  if (sizeof(TA) == 2) {
+    st = flip_all(p, Wop, s, launches);
+    if (st != LSGD_OK) return st;
+  }
   // partials of the next BatchNorm backward left by the data-gradient epilogue (0: none; the top
   // block's output gradient comes from the pooling's backward)
   int pending = 0;
@@ -2441,6 +2532,20 @@ lsgd_status resnet_alloc(ResNetPlan* p, const std::function<void*(size_t)>& allo
       p->col.push_back(nullptr);
     }
     p->wpart.push_back(wp);
+    // this convolution's data gradient on the persistent implicit kernel: its own flipped weights
+    uint16_t* wf = nullptr;
+    if (&c != &p->convs[0] && conv_on_tc(p, c)) {
+      const int64_t Pd = (int64_t)B * c.hin * c.win;
+      const size_t per = (size_t)K * c.cin * 9 * c.cout;
+      const bool plain = c.stride == 1 && implicit_conv_ok(c.cout, 1, c.hin, c.win) &&
+                         persistent_conv_ok(c.cin, Pd);
+      const bool phases = !plain && phase_dgrad_ok(p, c);
+      if (plain || phases) {
+        wf = (uint16_t*)alloc((phases ? 4 : 1) * per * 2);
+        if (!wf) return LSGD_ENOMEM;
+      }
+    }
+    p->wflip.push_back(wf);
   }
   if (colT) {
     p->colT = (uint16_t*)alloc(colT * 2);
